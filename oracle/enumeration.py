@@ -1,0 +1,158 @@
+"""Exact output distributions of the autoregressive and speculative frame procedures.
+TEST INFRASTRUCTURE ONLY.
+
+The paper's correctness claim (Abstract; Sec. 3.2) is that the speculative decoder is
+distributionally lossless under the deployed top-k sampling: the law of the emitted
+codes c1..c_P equals the autoregressive law prod_s p_s(c_s | c_<s).  On a small model
+both laws can be written out exactly in fp64:
+
+  * AR: product of the top-k/temperature probabilities along every sequence.
+  * speculative: the procedure of oracle.frame, with every random choice replaced by
+    its probability -- drafts d_j ~ q_j (independent, all from h_a + b_j), a draft kept
+    with probability min(1, p(d)/q(d)), otherwise a residual code with probability
+    r(x)/R, and a bonus code ~ p when every draft is kept.
+
+Hidden states and distributions are memoised by code prefix: the row at sequence
+position s depends only on c0 and c1..c_{s-1}.
+"""
+from __future__ import annotations
+
+import itertools
+from collections import defaultdict
+from typing import Dict, Tuple
+
+import numpy as np
+
+from paper_2609_37007_gb300.synth import DRAFT_GREEDY, FrameInput
+
+from .model import Model
+from .sampler import Dist, greedy_dist, residual_weights, topk_dist
+
+
+def to_f32(x) -> np.ndarray:
+    return np.asarray(x, dtype=np.float64).astype(np.float32)
+
+
+class PrefixModel:
+    """h_s, p_s and the drafts of one frame input, memoised by code prefix."""
+
+    def __init__(self, model: Model, frame: FrameInput, draft_mode: int = 0):
+        self.m, self.frame, self.mode = model, frame, draft_mode
+        self.k, self.T = model.cfg.top_k, model.cfg.temperature
+        self._h: Dict[Tuple[int, ...], Tuple[np.ndarray, np.ndarray]] = {}
+        self._p: Dict[Tuple[int, ...], Dist] = {}
+        self._q: Dict[Tuple[Tuple[int, ...], int], Dist] = {}
+
+    def state(self, prefix: Tuple[int, ...]):
+        """(KV cache, h_s) after the rows up to position s = len(prefix) + 1."""
+        if prefix not in self._h:
+            if not prefix:
+                kv = self.m.new_kv()
+                self.m.row(kv, np.asarray(self.frame.cond, dtype=np.float64), 0)
+                h = self.m.row(kv, self.m.c0_row(self.frame.c0, self.frame.c0_emb), 1)
+            else:
+                kv0, _ = self.state(prefix[:-1])
+                kv = kv0.copy()
+                s = len(prefix) + 1
+                h = self.m.row(kv, self.m.code_row(s - 1, prefix[-1]), s)
+            self._h[prefix] = (kv, h)
+        return self._h[prefix]
+
+    def target(self, prefix: Tuple[int, ...]) -> Dist:
+        """p for c_{len(prefix)+1} given c1..c_len."""
+        if prefix not in self._p:
+            s = len(prefix) + 1
+            self._p[prefix] = topk_dist(to_f32(self.m.verify_logits(s, self.state(prefix)[1])),
+                                        self.k, self.T)
+        return self._p[prefix]
+
+    def draft(self, prefix: Tuple[int, ...], j: int) -> Dist:
+        """q for c_{a+j} drafted from h_a, a = len(prefix) (prefix = c1..c_a)."""
+        key = (prefix, j)
+        if key not in self._q:
+            a = len(prefix)
+            h = self.state(prefix[:-1])[1]
+            z = to_f32(self.m.draft_logits(a, j, h))
+            self._q[key] = greedy_dist(z) if self.mode == DRAFT_GREEDY else \
+                topk_dist(z, self.k, self.T)
+        return self._q[key]
+
+
+def ar_distribution(pm: PrefixModel, n_pos: int) -> Dict[Tuple[int, ...], float]:
+    out: Dict[Tuple[int, ...], float] = {}
+
+    def rec(prefix, pr):
+        if len(prefix) == n_pos:
+            out[prefix] = pr
+            return
+        p = pm.target(prefix)
+        for x in p.ids:
+            rec(prefix + (x,), pr * p.prob(x))
+
+    rec((), 1.0)
+    return out
+
+
+def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
+    """(law of c1..c_P, expected model calls per frame) of the speculative procedure."""
+    memo: Dict[Tuple[int, ...], Tuple[Dict[Tuple[int, ...], float], float]] = {}
+
+    def add(res, calls, head, sub, w):
+        sub_law, sub_calls = sub
+        for tail, pv in sub_law.items():
+            res[head + tail] += w * pv
+        return calls + w * sub_calls
+
+    def from_state(prefix):
+        """Law of the remaining codes and expected remaining calls, drafts pending."""
+        if prefix in memo:
+            return memo[prefix]
+        a = len(prefix)
+        res: Dict[Tuple[int, ...], float] = defaultdict(float)
+        calls = 1.0
+        if a == n_pos:
+            memo[prefix] = ({(): 1.0}, 0.0)
+            return memo[prefix]
+        n_d = min(draft_len, n_pos - a)
+        qs = [pm.draft(prefix, j) for j in range(1, n_d + 1)]
+        for dt in itertools.product(*[q.ids for q in qs]):
+            pr = 1.0
+            for q, d in zip(qs, dt):
+                pr *= q.prob(d)
+            cur = prefix
+            for i in range(n_d):
+                p, q, d = pm.target(cur), qs[i], dt[i]
+                alpha = min(1.0, p.prob(d) / q.prob(d))
+                if alpha < 1.0:
+                    xs, r, R = residual_weights(p, q)
+                    for x, rx in zip(xs, r):
+                        if rx > 0.0:
+                            calls = add(res, calls, cur[a:] + (x,), from_state(cur + (x,)),
+                                        pr * (1.0 - alpha) * rx / R)
+                pr *= alpha
+                if pr == 0.0:
+                    break
+                cur = cur + (d,)
+            else:
+                if len(cur) < n_pos:
+                    p = pm.target(cur)
+                    for x in p.ids:
+                        calls = add(res, calls, cur[a:] + (x,), from_state(cur + (x,)),
+                                    pr * p.prob(x))
+                else:
+                    res[cur[a:]] += pr
+        memo[prefix] = (dict(res), calls)
+        return memo[prefix]
+
+    # first call: rows (cond, c0), emits c1 from LM head 1 -- plain AR
+    p1 = pm.target(())
+    law: Dict[Tuple[int, ...], float] = defaultdict(float)
+    calls = 1.0
+    for x in p1.ids:
+        calls = add(law, calls, (x,), from_state((x,)), p1.prob(x))
+    return dict(law), calls
+
+
+def alpha(p: Dist, q: Dist) -> float:
+    """Acceptance probability of one draft: sum_x min(p(x), q(x))."""
+    return sum(min(p.prob(x), q.prob(x)) for x in set(p.ids) | set(q.ids))
