@@ -1,0 +1,361 @@
+#!/usr/bin/env python3
+"""Benchmark: accepted RVQ tokens/s of single-stream speculative decoding on one GB300.
+
+Workload: the MultiCodeDecoder-shaped bf16 model (5 layers, hidden 1024, 16q/8kv heads x
+128, SwiGLU 3072, 15 positions with 2048-entry codebooks and LM heads, random-init
+weights N(0, 0.02) from seed 0), single stream, draft length K = 3, top-k 50,
+temperature 0.9.  One step = one frame (c1..c15) decoded by one cooperative launch of the
+persistent frame kernel; frame inputs (conditioning vector ~ N(0,1), c0 ~ U[0,2048)) are
+synthetic and resident in HBM before the timed region.
+
+Printed JSON line: value = accepted tokens/s (15 codes per frame), plus microseconds per
+verify call, tokens per call, the autoregressive baseline built from the same kernels
+(K = 0), the roofline of the frame kernel against the measured HBM copy bandwidth, the
+end-to-end number through the C ABI with host buffers, and the CPU oracle as a baseline.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+For N > 1 (torchrun) every rank decodes its own replica stream (no collective on the
+data path); value = all ranks' tokens / max over ranks of the timed region.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "accepted RVQ tokens/s single-stream"
+UNIT = "tokens/s"
+WORKLOAD = ("MultiCodeDecoder bf16, 5 layers, hidden 1024, 16q/8kv x 128, SwiGLU 3072, "
+            "15 RVQ positions x 2048 codes, K=3 drafts, top-k 50, T 0.9, single stream, "
+            "one frame (c1..c15) per step")
+
+
+def read_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        self.f.close()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------------------
+def cpu_oracle_baseline(cfg, weights, budget_s: float, first_frame: int):
+    """The oracle as it stands on the host cores, whole frames until budget_s is spent."""
+    from paper_2609_37007_gb300.synth import make_frame, weights_as_f32
+    from oracle.model import Model
+    from oracle.frame import decode_frame
+    model = Model(cfg, weights_as_f32(cfg, weights))
+    t0 = time.perf_counter()
+    frames = codes = calls = 0
+    while frames < 2 or time.perf_counter() - t0 < budget_s:
+        r = decode_frame(model, make_frame(cfg, first_frame + frames), frame_idx=first_frame + frames)
+        frames += 1
+        codes += len(r.codes)
+        calls += r.calls
+    dt = time.perf_counter() - t0
+    return {"value": codes / dt, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": f"{frames} whole frames of the same workload ({calls} model calls) decoded by the "
+                      f"fp64 numpy oracle in {dt:.1f} s"}
+
+
+def blas_threads() -> int:
+    v = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS")
+    return int(v) if v else (os.cpu_count() or 1)
+
+
+def run_reference(args, cfg, weights):
+    """Reference arm: the CPU oracle, one oracle model call per step."""
+    from paper_2609_37007_gb300.synth import make_frame, weights_as_f32
+    from oracle.model import Model
+    from oracle.frame import decode_frame
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    model = Model(cfg, weights_as_f32(cfg, weights))
+    # The oracle decodes whole frames; a step is one of its model calls, timed as an
+    # equal share of the frame that contains it.
+    t_calls = []
+    f = 0
+    need = args.warmup + args.steps
+    codes = 0
+    calls = 0
+    while calls < need:
+        t0 = time.perf_counter()
+        r = decode_frame(model, make_frame(cfg, f), frame_idx=f)
+        dt = time.perf_counter() - t0
+        for rec in r.rounds:
+            if args.warmup <= calls < need:
+                codes += len(rec.emitted)
+                t_calls.append(dt / len(r.rounds))
+            calls += 1
+        f += 1
+    elapsed = sum(t_calls)
+    value = codes / elapsed
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "step": "one model call of the CPU oracle"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                             "sample": f"{args.steps} oracle model calls ({codes} codes) after "
+                                       f"{args.warmup} warm-up calls"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------------------
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--ar-frames", type=int, default=200)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    from paper_2609_37007_gb300.synth import MCD, make_frames, make_weights
+    cfg = MCD
+    weights = make_weights(cfg)
+    if args.impl == "reference":
+        return run_reference(args, cfg, weights)
+
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    if rank == 0 or world > 1:
+        _build.build()
+    if dist:
+        dist.barrier()
+    dev = torch.device("cuda", local if world > 1 else 0)
+    stream = torch.cuda.current_stream(dev)
+
+    # CPU baseline first, before any GPU state exists (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = cpu_oracle_baseline(cfg, weights, args.cpu_budget, first_frame=100_000)
+
+    dec = mcd.Decoder(cfg, weights, stream)
+    ctx = dec.ctx
+    n_frames = args.warmup + args.steps
+    cond_h, c0_h, _ = make_frames(cfg, n_frames, first=rank * 1_000_000)
+    cond = torch.from_numpy(cond_h).to(dev)
+    c0 = torch.from_numpy(c0_h).to(dev)
+    codes = torch.zeros((n_frames, cfg.n_pos), dtype=torch.int32, device=dev)
+    stats = torch.zeros((n_frames, 8), dtype=torch.int32, device=dev)
+
+    def decode(i, c_ctx=ctx, cds=codes, sts=stats):
+        mcd.mcd_decode_frame(c_ctx, rank, i, cond[i], c0[i:i + 1], None, cds[i], sts[i])
+
+    for i in range(args.warmup):
+        decode(i)
+    mcd.mcd_sync(ctx)
+
+    # ---- timed region: K frames, per-launch events on the launching stream ------------
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    clocks = Clocks(local if world > 1 else 0)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    ev[0].record(stream)
+    for s in range(args.steps):
+        decode(args.warmup + s)
+        ev[s + 1].record(stream)
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    mcd.mcd_sync(ctx)
+    per = [ev[s].elapsed_time(ev[s + 1]) for s in range(args.steps)]        # ms
+    elapsed = ev[0].elapsed_time(ev[-1]) / 1e3
+    st = stats.cpu().numpy()[args.warmup:]
+    assert (st[:, 4] == 0).all() and (st[:, 1] == cfg.n_pos).all(), "device-side failure"
+    tokens = int(st[:, 1].sum())
+    calls = int(st[:, 0].sum())
+    if dist:
+        t = torch.tensor([elapsed, tokens, calls], dtype=torch.float64, device=dev)
+        mx = t.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        elapsed_all, tokens_all, calls_all = float(mx[0]), int(t[1]), int(t[2])
+    else:
+        elapsed_all, tokens_all, calls_all = elapsed, tokens, calls
+
+    # ---- roofline of the frame kernel ---------------------------------------------------
+    H, L, NKV, D = cfg.hidden, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim
+    backbone = mcd.mcd_call_weight_bytes(ctx, 0)
+    head = mcd.mcd_call_weight_bytes(ctx, 1) - backbone
+    heads = int(st[:, 5].sum())
+    kv_rows = int(st[:, 6].sum())
+    rows = int(st[:, 7].sum())
+    kv_bytes = kv_rows * L * 2 * NKV * D * 4               # fp32 K/V read (and new rows written)
+    emb_bytes = rows * H * 2
+    alg_bytes = calls * backbone + heads * head + kv_bytes + emb_bytes
+    launch_s = statistics.mean(per) / 1e3
+    bytes_per_launch = alg_bytes / args.steps
+    peak, peak_kind = read_peaks()
+    achieved = bytes_per_launch / launch_s / 1e9
+    traffic = None
+    tf = os.path.join(ROOT, "profiles", "frame_kernel_traffic.json")
+    if os.path.exists(tf):
+        try:
+            traffic = json.load(open(tf)).get("dram_bytes_per_launch")
+        except Exception:
+            traffic = None
+
+    # ---- AR baseline (same kernels, K = 0) --------------------------------------------
+    ar = None
+    if rank == 0 and args.ar_frames > 0:
+        cfg_ar = cfg.replace(draft_len=0)
+        dec_ar = mcd.Decoder(cfg_ar, weights, stream)
+        n_ar = args.ar_frames
+        cds = torch.zeros((n_ar, cfg.n_pos), dtype=torch.int32, device=dev)
+        sts = torch.zeros((n_ar, 8), dtype=torch.int32, device=dev)
+        for i in range(5):
+            mcd.mcd_decode_frame(dec_ar.ctx, rank, i, cond[i], c0[i:i + 1], None, cds[i], sts[i])
+        mcd.mcd_sync(dec_ar.ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(n_ar):
+            j = i % n_frames
+            mcd.mcd_decode_frame(dec_ar.ctx, rank, j, cond[j], c0[j:j + 1], None, cds[i], sts[i])
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mcd.mcd_sync(dec_ar.ctx)
+        s_ar = sts.cpu().numpy()
+        t_ar = e0.elapsed_time(e1) / 1e3
+        ar = {"tokens_per_s": float(s_ar[:, 1].sum() / t_ar), "us_per_call": 1e6 * t_ar / float(s_ar[:, 0].sum()),
+              "frames": n_ar, "tokens_per_call": float(s_ar[:, 1].sum() / s_ar[:, 0].sum())}
+        dec_ar.close()
+
+    # ---- end to end through the C ABI with host buffers --------------------------------
+    e2e = None
+    if rank == 0 or world > 1:
+        n_e = min(args.steps, 300)
+        cond_p = torch.from_numpy(cond_h[:n_e]).pin_memory()
+        c0_p = torch.from_numpy(c0_h[:n_e]).pin_memory()
+        out_p = torch.zeros((n_e, cfg.n_pos), dtype=torch.int32).pin_memory()
+        cond_d = torch.empty((cfg.hidden,), dtype=torch.float32, device=dev)
+        c0_d = torch.empty((1,), dtype=torch.int32, device=dev)
+        out_d = torch.empty((cfg.n_pos,), dtype=torch.int32, device=dev)
+        st_d = torch.zeros((n_e, 8), dtype=torch.int32, device=dev)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(n_e):
+            cond_d.copy_(cond_p[i], non_blocking=True)
+            c0_d.copy_(c0_p[i:i + 1], non_blocking=True)
+            mcd.mcd_decode_frame(ctx, rank, 5_000_000 + i, cond_d, c0_d, None, out_d, st_d[i])
+            out_p[i].copy_(out_d, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mcd.mcd_sync(ctx)
+        t_e = e0.elapsed_time(e1) / 1e3
+        e2e = {"value": float(n_e * cfg.n_pos / t_e), "unit": UNIT,
+               "h2d_bytes_per_step": cfg.hidden * 4 + 4, "d2h_bytes_per_step": cfg.n_pos * 4,
+               "frames": n_e}
+
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": tokens_all / elapsed_all, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed_all / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "frames_per_rank": args.steps,
+                   "arithmetic": "bf16 weights x fp32 activations (bf16 hi+lo split), fp32 accumulate, "
+                                 "fp64 sampler",
+                   "l2": "inputs larger than L2: 287 MB of weights per context, ~175-187 MB streamed per call",
+                   "parallelism": f"replicas x{world}"},
+        "us_per_call": 1e6 * elapsed / calls,
+        "tokens_per_call": tokens_all / calls_all,
+        "calls_per_frame": calls_all / (args.steps * world),
+        "ar_baseline": ar,
+        "speedup_vs_ar": (tokens_all / elapsed_all) / ar["tokens_per_s"] if ar else None,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "kernel": "frame_kernel<bf16>",
+                     "bytes_per_launch": bytes_per_launch,
+                     "launch_us": launch_s * 1e6},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 2 * args.steps * world,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    dec.close()
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,206 @@
+/*
+ * mcd.h -- C ABI of the GB300 MultiCodeDecoder speculative-decoding library (libmcd.so).
+ *
+ * Operation (arXiv 2609.37007): per 80 ms audio frame the MultiCodeDecoder (MCD) emits
+ * the 15 residual RVQ codes c1..c15 after the outer model's c0 (Sec. 1, Fig. 1).  This
+ * library runs that inner loop with RVQ-position-aware speculative decoding
+ * (Sec. 2.2, Fig. 3): each model call feeds the last emitted code plus K drafted codes,
+ * verifies the drafts with the lossless acceptance rule min(1, p/q) with residual
+ * resampling under the deployed top-k / temperature sampling (Abstract, Sec. 3.2), and
+ * drafts the next K codes from LM head k+j applied to h_k + b_j, where h_k is the
+ * hidden state that emitted the last code and b_1..b_K are the per-lookahead offsets.
+ *
+ * Conventions
+ *   - Every call returns an mcd_status; nothing aborts or throws across the ABI.
+ *   - "dev" pointers are CUDA device pointers owned by the caller, valid until the work
+ *     queued on the context's stream has finished.  "host" pointers are read before the
+ *     call returns.  The context owns its weights, KV cache, scratch and counters.
+ *   - Calls that launch work are asynchronous on the stream given to mcd_create unless
+ *     stated otherwise.  Device-side failures (a bounded wait that ran out) are recorded
+ *     in the context and reported by mcd_sync() and by the `status` field of
+ *     mcd_frame_stats.
+ *   - There is no CPU fallback: without a usable CUDA device mcd_create fails.
+ *   - A context is not thread-safe; use one context per host thread.
+ *
+ * Random numbers: Philox4x32-10 (Salmon et al., SC'11) with key = (seed lo, seed hi) and
+ * counter = (stream id, frame index, (call index << 8) | position, purpose); purpose
+ * 0 = target / residual / bonus sample, 1 = accept test, 2 = draft sample,
+ * 3 + v/2 = Gaussian pair for vocabulary entries (v, v+1) of a noisy draft row.
+ * A uniform is ((w0 >> 5) * 2^26 + (w1 >> 6)) * 2^-53 from words 0 and 1.
+ */
+#ifndef MCD_H
+#define MCD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct mcd_ctx mcd_ctx;
+
+typedef enum {
+  MCD_OK = 0,
+  MCD_ERR_INVALID_ARG = 1,   /* bad pointer, size or configuration value               */
+  MCD_ERR_STATE = 2,         /* call out of order (e.g. decode before weights)         */
+  MCD_ERR_CUDA = 3,          /* a CUDA runtime call failed; context must be destroyed  */
+  MCD_ERR_OOM = 4,           /* device allocation failed                               */
+  MCD_ERR_TIMEOUT = 5,       /* a bounded device-side wait ran out                     */
+  MCD_ERR_WEIGHTS = 6,       /* missing, duplicate or wrongly sized weight tensor      */
+  MCD_ERR_UNSUPPORTED = 7    /* shape outside the kernels' limits                      */
+} mcd_status;
+
+enum { MCD_WEIGHT_F32 = 0, MCD_WEIGHT_BF16 = 1 };
+enum { MCD_DRAFT_SAMPLE = 0, MCD_DRAFT_GREEDY = 1, MCD_DRAFT_NOISY_TARGET = 2 };
+
+/* Model and sampling configuration.  Limits: hidden, ffn multiples of 128; head_dim 64
+ * or 128; n_q_heads multiple of n_kv_heads; vocab multiple of 16 and <= 4096;
+ * n_pos <= 15; draft_len (K) <= 7; top_k in 1..256 and <= vocab; c0_vocab <= 4096. */
+typedef struct {
+  int32_t n_layers, hidden, n_q_heads, n_kv_heads, head_dim, ffn;
+  int32_t n_pos;        /* residual positions c1..c_{n_pos} (15 in the paper)           */
+  int32_t vocab;        /* codebook size of c1..c_{n_pos}                               */
+  int32_t c0_vocab;     /* rows of table 0; 0 = frames pass a c0 embedding vector       */
+  float rms_eps, rope_base;
+  int32_t qk_norm;      /* per-head RMSNorm of q and k before RoPE                      */
+  int32_t weight_dtype; /* MCD_WEIGHT_F32 or MCD_WEIGHT_BF16                            */
+  int32_t draft_len;    /* K; 0 = plain autoregressive decoding                         */
+  int32_t top_k;
+  float temperature;
+  int32_t draft_mode;   /* MCD_DRAFT_*                                                   */
+  float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only                                  */
+  uint64_t seed;        /* Philox key                                                    */
+} mcd_config;
+
+/* Per-frame counters written by the device (device memory, caller-owned). */
+typedef struct {
+  int32_t calls;     /* model calls (rounds) spent on the frame                */
+  int32_t codes;     /* codes emitted (n_pos on success)                        */
+  int32_t drafted;   /* drafts tested                                           */
+  int32_t accepted;  /* drafts kept                                             */
+  int32_t status;    /* 0, or an mcd_status value set by a failed device wait   */
+  int32_t heads_read;/* LM heads streamed, summed over the calls (byte accounting) */
+  int32_t kv_rows;   /* sum over calls of (first row position + rows): KV touched   */
+  int32_t rows_fed;  /* sum over calls of rows fed                                  */
+} mcd_frame_stats;
+
+/* Per-call record written when tracing is on (mcd_set_trace).  One record per call, in
+ * call order; logits of record r live in the trace buffer after all records (see
+ * mcd_trace_bytes for the layout). */
+typedef struct {
+  int32_t a;              /* codes emitted before this call                           */
+  int32_t n_rows;         /* rows fed                                                 */
+  int32_t pos0;           /* sequence position of the first row                       */
+  int32_t n_drafts;       /* drafts tested                                            */
+  int32_t input_ids[8];   /* code fed at each row (-1: conditioning / c0 vector)      */
+  int32_t drafts[8];      /* drafts tested (positions a+1..)                          */
+  int32_t n_acc;          /* drafts kept                                              */
+  int32_t n_emit;         /* codes emitted                                            */
+  int32_t emitted[8];
+  int32_t n_next;         /* drafts made for the next call                            */
+  int32_t next_drafts[8];
+  int32_t draft_row;      /* row whose hidden state drafted them (= n_acc)            */
+  int32_t reserved[24];
+} mcd_call_trace;
+
+/* Create a context on the current CUDA device.  `cfg` (host) is copied.  `cuda_stream`
+ * is a cudaStream_t (NULL = legacy default stream) used by every later call.
+ * Allocates device buffers and sets kernel attributes.  On failure *out is NULL. */
+mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out);
+
+/* Load all weights.  `names`, `host_ptrs`, `nbytes`: n host arrays describing named
+ * tensors in the dtype of cfg.weight_dtype (bf16 as raw 16-bit patterns), row-major,
+ * matrices [out, in].  Required names (l = layer, i = table, P = position, j = offset):
+ *   layers.l.{attn_norm[H], wq[Hq*D,H], wk[Hkv*D,H], wv[Hkv*D,H], q_norm[D], k_norm[D]
+ *            (qk_norm only), wo[H,Hq*D], ffn_norm[H], wg[F,H], wu[F,H], wd[H,F]},
+ *   final_norm[H], embed.0[c0_vocab,H] (c0_vocab > 0), embed.i[V,H] (i = 1..n_pos-1),
+ *   head.P[V,H] (P = 1..n_pos), offset.j[H] (j = 1..max(K,1)).
+ * The library copies and re-tiles them (the caller keeps ownership) and synchronises
+ * the stream before returning.  Extra names are ignored. */
+mcd_status mcd_load_weights(mcd_ctx* ctx, int32_t n, const char* const* names,
+                            const void* const* host_ptrs, const int64_t* nbytes);
+
+/* Decode one frame: emit c1..c_{n_pos} into codes_out (dev int32 [n_pos]).
+ *   cond   dev float [hidden], 16-byte aligned: the outer model's hidden state
+ *          (sequence position 0).
+ *   c0     dev int32 [1]: the frame's c0 id (c0_vocab > 0), else NULL; an id outside
+ *          [0, c0_vocab) fails the frame with MCD_ERR_INVALID_ARG (reported by mcd_sync).
+ *   c0_emb dev float [hidden], 16-byte aligned: c0 embedding (c0_vocab == 0), else NULL.
+ *   stats  dev mcd_frame_stats, optional (NULL).
+ * One cooperative persistent-kernel launch runs every call of the frame on device. */
+mcd_status mcd_decode_frame(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx,
+                            const float* cond, const int32_t* c0, const float* c0_emb,
+                            int32_t* codes_out, mcd_frame_stats* stats);
+
+/* Stepwise use of the same kernels.  mcd_begin_frame resets the per-frame state and
+ * selects the (stream id, frame index) of the Philox counters; it needs no weights, so
+ * the sampler hooks below can run on a context without them;
+ * mcd_verify_accept runs exactly one model call (the first call feeds cond and c0),
+ * writing the codes it emitted to emitted (dev int32 [K+1]) and their count to
+ * n_emitted (dev int32 [1]); a call after the frame is complete emits 0 codes.
+ * logits_out (dev float [K+1, vocab], optional) receives the verify logits of the
+ * call's rows that read an LM head. */
+mcd_status mcd_begin_frame(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx,
+                           const float* cond, const int32_t* c0, const float* c0_emb);
+mcd_status mcd_verify_accept(mcd_ctx* ctx, int32_t* emitted, int32_t* n_emitted,
+                             float* logits_out);
+
+/* Position-aware drafting on its own (Sec. 2.2, Fig. 3): for j = 1..min(K, n_pos-k)
+ * z_j = LMH_{k+j}(h_k + b_j); q_j = top-k/temperature softmax of z_j; d_j ~ q_j with the
+ * draft-purpose uniform of (call_idx, k+j) under the frame set by mcd_begin_frame.
+ *   h_k      dev float [hidden], the post-norm hidden state read by LM head k (1 <= k < n_pos)
+ *   draft_ids dev int32 [K]; q_ids dev int32 [K, top_k]; q_probs dev double [K, top_k]
+ *   z_out    dev float [K, vocab], optional.  Unused rows are left untouched. */
+mcd_status mcd_draft(mcd_ctx* ctx, int32_t pos_k, int32_t call_idx, const float* h_k,
+                     int32_t* draft_ids, int32_t* q_ids, double* q_probs, float* z_out);
+
+/* Sampler on given fp32 logits (parity hook for the acceptance rule).  p_logits dev
+ * float [n_drafts+1, vocab] are the verify rows of positions a+1..a+1+n_drafts (the last
+ * row is only read when a bonus position exists), q_logits dev float [n_drafts, vocab]
+ * the draft rows, draft_ids dev int32 [n_drafts].  Uniforms use (call_idx, position)
+ * under the frame set by mcd_begin_frame.  Writes emitted (dev int32 [n_drafts+1]) and
+ * out2 (dev int32 [2]) = {n_acc, n_emit}.  Uses cfg.top_k, temperature, draft_mode
+ * (SAMPLE or GREEDY). */
+mcd_status mcd_accept_from_logits(mcd_ctx* ctx, int32_t a, int32_t n_drafts, int32_t call_idx,
+                                  const float* p_logits, const float* q_logits,
+                                  const int32_t* draft_ids, int32_t* emitted, int32_t* out2);
+
+/* Top-k / temperature softmax of n_rows fp32 logits rows (dev float [n_rows, vocab]):
+ * ids (dev int32 [n_rows, top_k]) in sampling order (logit desc, id asc), probs
+ * (dev double [n_rows, top_k]) = exp(z_i - z_max) / S with z = logit / temperature. */
+mcd_status mcd_topk_softmax(mcd_ctx* ctx, int32_t n_rows, const float* logits,
+                            int32_t* ids, double* probs);
+
+/* Tracing for parity tests: while `trace` (dev, mcd_trace_bytes() bytes) is set, frame
+ * decoding writes one mcd_call_trace per call followed, after 16 records, by float
+ * logits [16 calls][8 rows][vocab] (verify rows) and [16 calls][8 drafts][vocab] (the
+ * draft rows used).  NULL turns tracing off. */
+int64_t mcd_trace_bytes(const mcd_ctx* ctx);
+mcd_status mcd_set_trace(mcd_ctx* ctx, void* trace);
+
+/* Profiling hook: while `timeline` (dev, uint64 [16 calls][128], zeroed by the caller)
+ * is set, frame decoding writes %globaltimer stamps (ns) per call: slot 0 call start;
+ * 1 top-k inputs ready; 2 / 3 top-k done by CTA 0 / by the last CTA; 4..7 acceptance
+ * start, records staged, decided, end.  Stage s (s = 4l + k for step k of layer l:
+ * 0 QKV, 1 attention + Wo, 2 gate/up, 3 down; s = 4L heads) uses slots 8+4s..: +0 inputs
+ * ready and +1 first weight unit in shared memory (CTA 0), +2 last epilogue done and +3
+ * completion signalled (maximum over CTAs).  NULL turns it off. */
+mcd_status mcd_set_timeline(mcd_ctx* ctx, uint64_t* timeline);
+
+/* Wait for the context's stream; returns the first device-side failure, if any. */
+mcd_status mcd_sync(mcd_ctx* ctx);
+
+/* Bytes of weights one verify call streams for a call that reads `n_heads` LM heads
+ * (backbone + heads), the algorithmic traffic used for roofline accounting. */
+int64_t mcd_call_weight_bytes(const mcd_ctx* ctx, int32_t n_heads);
+
+/* Number of persistent CTAs (one per SM) the frame kernel launches. */
+int32_t mcd_num_ctas(const mcd_ctx* ctx);
+
+void mcd_destroy(mcd_ctx* ctx);
+const char* mcd_status_str(mcd_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MCD_H */

@@ -1,0 +1,715 @@
+// C ABI of libmcd (declared in include/mcd.h): context management, weight loading and
+// re-tiling, frame decoding through the persistent frame kernel, the stepwise API and
+// the sampler parity hooks.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "mcd_internal.cuh"
+#include "mcd_sampler.cuh"
+
+namespace mcd {
+cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream);
+cudaError_t prepare_frame_kernel(int* max_ctas_per_sm);
+int frame_smem_bytes();
+
+// ------------------------------------------------------------------------------------
+// Auxiliary kernels
+// ------------------------------------------------------------------------------------
+struct RowSrc {
+  const uint8_t* seg[3];
+  int seg_rows[3];
+  int nseg;
+  int interleave_gu;  // 1: logical tile t = [gate rows 8t..8t+7 ; up rows 8t..8t+7]
+  int src_cols;       // elements per source row
+};
+
+// Logical element (r, c) -> offset (in elements) inside the tiled matrix.
+__host__ __device__ inline long long tiled_offset(const MatGeom& g, int r, int c, int wdtype) {
+  const int kc = c / (g.Ku * 16), kt = (c % (g.Ku * 16)) / 16;
+  const int mb = r / (g.Mu * 16), mi = (r % (g.Mu * 16)) / 16;
+  const long long u = (long long)kc * g.n_mb + mb;
+  const long long tile = (u * g.Mu + mi) * g.Ku + kt;
+  const int rr = r & 15, cc = c & 15;
+  int pos;
+  if (wdtype == MCD_WEIGHT_BF16) {
+    const int lane = (rr & 7) * 4 + ((cc & 7) >> 1);
+    const int reg = (rr >> 3) + 2 * (cc >> 3);
+    pos = lane * 8 + reg * 2 + (cc & 1);
+  } else {
+    pos = (rr + 16 * (cc >> 3)) * 8 + (cc & 7);
+  }
+  return tile * 256 + pos;
+}
+
+__global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst) {
+  const long long total = (long long)g.M * g.K;
+  const int es = wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int r = (int)(e / g.K), c = (int)(e % g.K);
+    const uint8_t* src;
+    int sr;
+    if (rs.interleave_gu) {
+      const int t = r >> 4, rr = r & 15;
+      src = rs.seg[rr < 8 ? 0 : 1];
+      sr = 8 * t + (rr & 7);
+    } else {
+      int rem = r, s = 0;
+      while (s < rs.nseg - 1 && rem >= rs.seg_rows[s]) rem -= rs.seg_rows[s++];
+      src = rs.seg[s];
+      sr = rem;
+    }
+    const long long so = ((long long)sr * rs.src_cols + c) * es;
+    const long long d = tiled_offset(g, r, c, wdtype) * es;
+    if (es == 2)
+      *reinterpret_cast<uint16_t*>(dst + d) = *reinterpret_cast<const uint16_t*>(src + so);
+    else
+      *reinterpret_cast<uint32_t*>(dst + d) = *reinterpret_cast<const uint32_t*>(src + so);
+  }
+}
+
+__global__ void to_f32_kernel(const uint8_t* src, int wdtype, long long n, float* dst) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+    dst[i] = wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(src)[i])
+                                       : reinterpret_cast<const float*>(src)[i];
+}
+
+__global__ void rope_kernel(float2* rope, int D, double base) {
+  const int half = D / 2;
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < kMaxPos * half; idx += gridDim.x * blockDim.x) {
+    const int pos = idx / half, i = idx % half;
+    const double ang = (double)pos * pow(base, -2.0 * (double)i / (double)D);
+    rope[idx] = make_float2((float)cos(ang), (float)sin(ang));
+  }
+}
+
+__global__ void begin_frame_kernel(DevState* st, unsigned* ctr, int n_ctr, const int* c0, int C0V) {
+  for (int i = threadIdx.x; i < n_ctr; i += blockDim.x) ctr[i] = 0u;
+  if (threadIdx.x == 0) {
+    st->call = 0;
+    st->a = 0;
+    st->done = 0;
+    st->n_d = 0;
+    st->pos0 = 0;
+    st->n_rows = 2;
+    st->first_head_row = 1;
+    st->n_acc_last = 0;
+    st->q_row = 0;
+    for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
+    st->codes[0] = C0V > 0 ? c0[0] : -1;
+    for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
+    st->n_emit_last = 0;
+    st->calls = st->drafted = st->accepted = 0;
+    st->heads_read = st->kv_rows = st->rows_fed = 0;
+  }
+}
+
+// Reset counters of a single stepwise call (the call index of the state).
+__global__ void reset_call_counters_kernel(const DevState* st, unsigned* ctr, int stride) {
+  const int call = st->call;
+  if (call < kMaxCalls)
+    for (int i = threadIdx.x; i < stride; i += blockDim.x) ctr[call * stride + i] = 0u;
+  if (call + 1 < kMaxCalls)
+    for (int i = threadIdx.x; i < stride; i += blockDim.x) ctr[(call + 1) * stride + i] = 0u;
+}
+
+__global__ void zero_emitted_kernel(const DevState* st, int* n_emitted) {
+  if (threadIdx.x == 0 && st->done && n_emitted) *n_emitted = 0;
+}
+
+// Top-k of n rows (one CTA of 256 threads per row).
+__global__ void __launch_bounds__(kConsumerThreads) topk_rows_kernel(const float* logits, int V, int k, float T,
+                                                                     TopkRec* recs, int32_t* ids, double* probs) {
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
+  const int row = blockIdx.x;
+  TopkRec* r = recs + row;
+  block_topk(logits + (size_t)row * V, V, k, T, 0, ts, r);
+  consumer_sync();
+  __threadfence_block();
+  for (int i = threadIdx.x; i < k; i += kConsumerThreads) {
+    if (ids) ids[(size_t)row * k + i] = r->ids[i];
+    if (probs) probs[(size_t)row * k + i] = r->e[i] / r->S;
+  }
+}
+
+// Acceptance on given logits: rows 0..n_d of p, rows 0..n_d-1 of q, one CTA.
+__global__ void __launch_bounds__(kConsumerThreads) accept_logits_kernel(FrameParams p, int a, int n_d, int call,
+                                                                         const float* pl, const float* ql,
+                                                                         const int* draft_ids, TopkRec* recs,
+                                                                         int* emitted, int* out2) {
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
+  const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
+  for (int i = 0; i < n_p; ++i) {
+    block_topk(pl + (size_t)i * p.V, p.V, p.top_k, p.T, 0, ts, recs + i);
+    consumer_sync();
+  }
+  for (int i = 0; i < n_d; ++i) {
+    block_topk(ql + (size_t)i * p.V, p.V, p.top_k, p.T, p.draft_mode == MCD_DRAFT_GREEDY, ts,
+               recs + kMaxRows + i);
+    consumer_sync();
+  }
+  __threadfence();
+  consumer_sync();
+  ResidualScratch& rs = *reinterpret_cast<ResidualScratch*>(smem_raw);
+  if (threadIdx.x < 32) {
+    int drafts[kMaxDraft + 1];
+    for (int i = 0; i < n_d; ++i) drafts[i] = draft_ids[i];
+    AcceptResult r = warp_accept(
+        a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(recs + i); },
+        [&](int i) { return (const TopkRec*)(recs + kMaxRows + i); }, p.seed, p.stream_id, p.frame_idx, call, rs);
+    if (threadIdx.x == 0) {
+      for (int t = 0; t < r.n_emit; ++t) emitted[t] = r.emitted[t];
+      out2[0] = r.n_acc;
+      out2[1] = r.n_emit;
+    }
+  }
+}
+
+// Draft logits z_j = LMH_{k+j}(h + b_j), one warp per (j, output id), from tiled heads.
+__global__ void draft_logits_kernel(FrameParams p, int pos_k, int n_j, const float* h, float* z) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= n_j * p.V) return;
+  const int j = warp / p.V + 1, id = warp % p.V;
+  const MatGeom& g = p.g[MAT_HEAD];
+  const uint8_t* W = p.w_head + (long long)(pos_k + j - 1) * g.stride;
+  float acc = 0.f;
+  for (int k = lane; k < p.H; k += 32) {
+    const long long off = tiled_offset(g, id, k, p.wdtype);
+    const float w = p.wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(W)[off])
+                                                : reinterpret_cast<const float*>(W)[off];
+    acc += w * (h[k] + p.offsets[(size_t)(j - 1) * p.H + k]);
+  }
+  for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+  if (lane == 0) z[(size_t)(j - 1) * p.V + id] = acc;
+}
+
+__global__ void __launch_bounds__(kConsumerThreads) draft_sample_kernel(FrameParams p, int pos_k, int call,
+                                                                        const float* z, TopkRec* recs, int* draft_ids,
+                                                                        int* q_ids, double* q_probs) {
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
+  const int j = blockIdx.x + 1;
+  TopkRec* r = recs + blockIdx.x;
+  block_topk(z + (size_t)(j - 1) * p.V, p.V, p.top_k, p.T, p.draft_mode == MCD_DRAFT_GREEDY, ts, r);
+  consumer_sync();
+  __threadfence_block();
+  if (threadIdx.x == 0) {
+    const double u = uniform_u(p.seed, p.stream_id, p.frame_idx, call, pos_k + j, PURPOSE_DRAFT);
+    draft_ids[j - 1] = seq_draw(r, u);
+  }
+  for (int i = threadIdx.x; i < p.top_k; i += kConsumerThreads) {
+    if (q_ids) q_ids[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->ids[i] : -1;
+    if (q_probs) q_probs[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->e[i] / r->S : 0.0;
+  }
+}
+
+}  // namespace mcd
+
+using namespace mcd;
+
+// ------------------------------------------------------------------------------------
+// Context
+// ------------------------------------------------------------------------------------
+struct mcd_ctx {
+  mcd_config cfg;
+  cudaStream_t stream;
+  int device;
+  FrameParams fp;
+  std::vector<void*> allocs;
+  uint8_t* w_arena = nullptr;
+  size_t w_bytes = 0;
+  size_t off_qkv = 0, off_wo = 0, off_gu = 0, off_wd = 0, off_head = 0, off_embed = 0;
+  float* f32_arena = nullptr;   // norms + offsets
+  bool weights_loaded = false;
+  bool frame_begun = false;
+  int h_err = 0;                 // host-side sticky CUDA error
+};
+
+static mcd_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return MCD_OK;
+  if (e == cudaErrorMemoryAllocation) return MCD_ERR_OOM;
+  return MCD_ERR_CUDA;
+}
+
+#define MCD_CHECK(call)                                 \
+  do {                                                  \
+    cudaError_t e__ = (call);                           \
+    if (e__ != cudaSuccess) {                           \
+      if (getenv("MCD_DEBUG"))                          \
+        fprintf(stderr, "mcd: %s failed: %s (%s:%d)\n", #call, cudaGetErrorString(e__), __FILE__, __LINE__); \
+      return cuda_status(e__);                          \
+    }                                                   \
+  } while (0)
+
+template <class T>
+static cudaError_t ctx_alloc(mcd_ctx* c, T** p, size_t bytes) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, bytes < 256 ? 256 : bytes);
+  if (e != cudaSuccess) return e;
+  c->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return cudaSuccess;
+}
+
+static bool make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeom& g) {
+  const int Gk = kConsumerWarps / Mu;
+  if (M % (Mu * 16) || K % 16) return false;
+  const int kt = K / 16;
+  int Ku = 0;
+  for (int cand = kt; cand >= Gk; --cand) {
+    if (kt % cand == 0 && cand % Gk == 0 && Mu * cand * tile_bytes <= kSlotBytes && cand * 16 <= max_cols) {
+      Ku = cand;
+      break;
+    }
+  }
+  if (!Ku) return false;
+  g.M = M;
+  g.K = K;
+  g.Mu = Mu;
+  g.Ku = Ku;
+  g.n_mb = M / (Mu * 16);
+  g.n_kc = kt / Ku;
+  g.n_units = g.n_mb * g.n_kc;
+  g.unit_bytes = Mu * Ku * tile_bytes;
+  g.stride = (long long)g.n_units * g.unit_bytes;
+  return true;
+}
+
+static mcd_status validate_config(const mcd_config& c) {
+  if (c.n_layers < 1 || c.hidden < 128 || c.hidden % 128 || c.hidden > 1024) return MCD_ERR_UNSUPPORTED;
+  if (!(c.head_dim == 64 || c.head_dim == 128)) return MCD_ERR_UNSUPPORTED;
+  if (c.n_q_heads < 1 || c.n_kv_heads < 1 || c.n_q_heads % c.n_kv_heads) return MCD_ERR_INVALID_ARG;
+  if (c.ffn < 128 || c.ffn % 128) return MCD_ERR_UNSUPPORTED;
+  if (c.n_pos < 1 || c.n_pos > 15) return MCD_ERR_UNSUPPORTED;
+  if (c.vocab < 16 || c.vocab % 16 || c.vocab > kMaxVocab) return MCD_ERR_UNSUPPORTED;
+  if (c.c0_vocab < 0 || c.c0_vocab > kMaxVocab) return MCD_ERR_UNSUPPORTED;
+  if (c.draft_len < 0 || c.draft_len > kMaxDraft) return MCD_ERR_UNSUPPORTED;
+  if (c.top_k < 1 || c.top_k > kMaxTopK || c.top_k > c.vocab) return MCD_ERR_UNSUPPORTED;
+  if (!(c.temperature > 0.f) || !(c.rms_eps > 0.f) || !(c.rope_base > 1.f)) return MCD_ERR_INVALID_ARG;
+  if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
+  if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
+  if (c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;  // see mcd.h
+  if ((long long)c.n_q_heads * c.head_dim + 2LL * c.n_kv_heads * c.head_dim > 8192) return MCD_ERR_UNSUPPORTED;
+  return MCD_OK;
+}
+
+extern "C" {
+
+const char* mcd_status_str(mcd_status s) {
+  switch (s) {
+    case MCD_OK: return "ok";
+    case MCD_ERR_INVALID_ARG: return "invalid argument";
+    case MCD_ERR_STATE: return "call out of order";
+    case MCD_ERR_CUDA: return "CUDA error";
+    case MCD_ERR_OOM: return "out of device memory";
+    case MCD_ERR_TIMEOUT: return "device-side wait timed out";
+    case MCD_ERR_WEIGHTS: return "missing or malformed weight tensor";
+    case MCD_ERR_UNSUPPORTED: return "shape outside the kernels' limits";
+  }
+  return "unknown status";
+}
+
+mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
+  if (!out) return MCD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg) return MCD_ERR_INVALID_ARG;
+  mcd_status vs = validate_config(*cfg);
+  if (vs != MCD_OK) return vs;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) return MCD_ERR_CUDA;
+  mcd_ctx* c = new mcd_ctx();
+  c->cfg = *cfg;
+  c->stream = static_cast<cudaStream_t>(cuda_stream);
+  auto fail = [&](mcd_status s) {
+    mcd_destroy(c);
+    return s;
+  };
+  if (cudaGetDevice(&c->device) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  int n_sm = 0, coop = 0, max_blocks = 0;
+  if (cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, c->device) != cudaSuccess || !coop)
+    return fail(MCD_ERR_UNSUPPORTED);
+  if (prepare_frame_kernel(&max_blocks) != cudaSuccess || max_blocks < 1) return fail(MCD_ERR_UNSUPPORTED);
+
+  const mcd_config& k = *cfg;
+  FrameParams& p = c->fp;
+  memset(&p, 0, sizeof(p));
+  p.L = k.n_layers;
+  p.H = k.hidden;
+  p.NH = k.n_q_heads;
+  p.NKV = k.n_kv_heads;
+  p.D = k.head_dim;
+  p.F = k.ffn;
+  p.P = k.n_pos;
+  p.V = k.vocab;
+  p.C0V = k.c0_vocab;
+  p.K = k.draft_len;
+  p.top_k = k.top_k;
+  p.qk_norm = k.qk_norm;
+  p.wdtype = k.weight_dtype;
+  p.draft_mode = k.draft_mode;
+  p.eps = k.rms_eps;
+  p.T = k.temperature;
+  p.sigma = k.noise_sigma;
+  p.seed = k.seed;
+  p.qkv_dim = p.NH * p.D + 2 * p.NKV * p.D;
+  p.n_cta = n_sm;
+  p.wait_ns = 2000000000ull;  // 2 s
+  const char* wn = getenv("MCD_WAIT_NS");
+  if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
+
+  const int tb = k.weight_dtype == MCD_WEIGHT_BF16 ? 512 : 1024;
+  const int es = k.weight_dtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  bool ok = make_geom(p.qkv_dim, p.H, 1, tb, 1024, p.g[MAT_QKV]) && p.g[MAT_QKV].n_kc == 1;
+  int mu_o = 8;
+  while (mu_o > 1 && (mu_o * (p.D / 16) * tb > kSlotBytes || p.H % (mu_o * 16))) mu_o >>= 1;
+  ok = ok && make_geom(p.H, p.NH * p.D, mu_o, tb, p.D, p.g[MAT_WO]) && p.g[MAT_WO].Ku * 16 == p.D;
+  ok = ok && make_geom(2 * p.F, p.H, 1, tb, 1024, p.g[MAT_GU]) && p.g[MAT_GU].n_kc == 1;
+  ok = ok && make_geom(p.H, p.F, 1, tb, 1024, p.g[MAT_WD]);
+  ok = ok && make_geom(p.V, p.H, 1, tb, 1024, p.g[MAT_HEAD]) && p.g[MAT_HEAD].n_kc == 1;
+  if (!ok) return fail(MCD_ERR_UNSUPPORTED);
+  p.ctr_stride = ctr_ready(p.L) + 2;
+
+  // weight arena
+  const size_t sq = p.g[MAT_QKV].stride, so = p.g[MAT_WO].stride, sg = p.g[MAT_GU].stride, sd = p.g[MAT_WD].stride;
+  c->off_qkv = 0;
+  c->off_wo = c->off_qkv + sq * p.L;
+  c->off_gu = c->off_wo + so * p.L;
+  c->off_wd = c->off_gu + sg * p.L;
+  c->off_head = c->off_wd + sd * p.L;
+  c->off_embed = c->off_head + (size_t)p.g[MAT_HEAD].stride * p.P;
+  p.embed_stride = (long long)std::max(p.C0V, p.V) * p.H * es;
+  c->w_bytes = c->off_embed + (size_t)p.embed_stride * p.P;
+  cudaError_t e;
+  if ((e = ctx_alloc(c, &c->w_arena, c->w_bytes)) != cudaSuccess) return fail(cuda_status(e));
+  p.w_qkv = c->w_arena + c->off_qkv;
+  p.w_wo = c->w_arena + c->off_wo;
+  p.w_gu = c->w_arena + c->off_gu;
+  p.w_wd = c->w_arena + c->off_wd;
+  p.w_head = c->w_arena + c->off_head;
+  p.embed = c->w_arena + c->off_embed;
+
+  const int Kd = std::max(p.K, 1);
+  const size_t nf = (size_t)p.L * p.H * 2 + (size_t)p.L * p.D * 2 + p.H + (size_t)Kd * p.H;
+  if ((e = ctx_alloc(c, &c->f32_arena, nf * 4)) != cudaSuccess) return fail(cuda_status(e));
+  p.attn_norm = c->f32_arena;
+  p.ffn_norm = p.attn_norm + (size_t)p.L * p.H;
+  p.q_norm = p.ffn_norm + (size_t)p.L * p.H;
+  p.k_norm = p.q_norm + (size_t)p.L * p.D;
+  p.final_norm = p.k_norm + (size_t)p.L * p.D;
+  p.offsets = p.final_norm + p.H;
+
+  float2* rope = nullptr;
+  if ((e = ctx_alloc(c, &rope, sizeof(float2) * kMaxPos * (p.D / 2))) != cudaSuccess) return fail(cuda_status(e));
+  p.rope = rope;
+  if ((e = ctx_alloc(c, &p.x, sizeof(float) * kMaxRows * p.H)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.qkv, sizeof(float) * kMaxRows * p.qkv_dim)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxRows * p.F)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxRows * (kMaxDraft + 1) * p.V)) != cudaSuccess)
+    return fail(cuda_status(e));
+  const size_t kvsz = sizeof(float) * (size_t)p.L * p.NKV * kMaxPos * p.D;
+  if ((e = ctx_alloc(c, &p.kcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.vcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * 2 * kMaxRows * (kMaxDraft + 1))) != cudaSuccess)
+    return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.draftq, sizeof(TopkRec) * (kMaxDraft + 1))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.st, sizeof(DevState))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxCalls * p.ctr_stride)) != cudaSuccess)
+    return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
+  if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaMemsetAsync(p.vcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaMemsetAsync(p.st, 0, sizeof(DevState), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base);
+  if (cudaGetLastError() != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  *out = c;
+  return MCD_OK;
+}
+
+void mcd_destroy(mcd_ctx* c) {
+  if (!c) return;
+  cudaStreamSynchronize(c->stream);
+  for (void* q : c->allocs) cudaFree(q);
+  delete c;
+}
+
+int32_t mcd_num_ctas(const mcd_ctx* c) { return c ? c->fp.n_cta : 0; }
+
+int64_t mcd_call_weight_bytes(const mcd_ctx* c, int32_t n_heads) {
+  if (!c) return 0;
+  const FrameParams& p = c->fp;
+  return (int64_t)p.L * (p.g[MAT_QKV].stride + p.g[MAT_WO].stride + p.g[MAT_GU].stride + p.g[MAT_WD].stride) +
+         (int64_t)n_heads * p.g[MAT_HEAD].stride;
+}
+
+mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, const void* const* host_ptrs,
+                            const int64_t* nbytes) {
+  if (!c || n <= 0 || !names || !host_ptrs || !nbytes) return MCD_ERR_INVALID_ARG;
+  FrameParams& p = c->fp;
+  const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  const int Kd = std::max(p.K, 1);
+  std::map<std::string, std::pair<const void*, int64_t>> given;
+  for (int i = 0; i < n; ++i) {
+    if (!names[i] || !host_ptrs[i]) return MCD_ERR_INVALID_ARG;
+    if (given.count(names[i])) return MCD_ERR_WEIGHTS;
+    given[names[i]] = {host_ptrs[i], nbytes[i]};
+  }
+  // required tensors and their element counts
+  std::vector<std::pair<std::string, int64_t>> req;
+  const int64_t H = p.H, D = p.D, qd = (int64_t)p.NH * D, kd = (int64_t)p.NKV * D, F = p.F;
+  for (int l = 0; l < p.L; ++l) {
+    const std::string pre = "layers." + std::to_string(l) + ".";
+    req.push_back({pre + "attn_norm", H});
+    req.push_back({pre + "wq", qd * H});
+    req.push_back({pre + "wk", kd * H});
+    req.push_back({pre + "wv", kd * H});
+    if (p.qk_norm) {
+      req.push_back({pre + "q_norm", D});
+      req.push_back({pre + "k_norm", D});
+    }
+    req.push_back({pre + "wo", H * qd});
+    req.push_back({pre + "ffn_norm", H});
+    req.push_back({pre + "wg", F * H});
+    req.push_back({pre + "wu", F * H});
+    req.push_back({pre + "wd", H * F});
+  }
+  req.push_back({"final_norm", H});
+  if (p.C0V > 0) req.push_back({"embed.0", (int64_t)p.C0V * H});
+  for (int i = 1; i < p.P; ++i) req.push_back({"embed." + std::to_string(i), (int64_t)p.V * H});
+  for (int P = 1; P <= p.P; ++P) req.push_back({"head." + std::to_string(P), (int64_t)p.V * H});
+  for (int j = 1; j <= Kd; ++j) req.push_back({"offset." + std::to_string(j), H});
+  size_t stage_bytes = 0;
+  std::map<std::string, size_t> soff;
+  for (auto& r : req) {
+    auto it = given.find(r.first);
+    if (it == given.end() || it->second.second != r.second * es) {
+      if (getenv("MCD_DEBUG")) fprintf(stderr, "mcd: weight %s missing or wrong size\n", r.first.c_str());
+      return MCD_ERR_WEIGHTS;
+    }
+    soff[r.first] = stage_bytes;
+    stage_bytes += (size_t)((it->second.second + 255) / 256 * 256);
+  }
+  uint8_t* stage = nullptr;
+  MCD_CHECK(cudaMalloc(&stage, stage_bytes));
+  auto cleanup = [&](mcd_status s) {
+    cudaStreamSynchronize(c->stream);
+    cudaFree(stage);
+    return s;
+  };
+  for (auto& r : req) {
+    auto& gv = given[r.first];
+    if (cudaMemcpyAsync(stage + soff[r.first], gv.first, (size_t)gv.second, cudaMemcpyHostToDevice, c->stream) !=
+        cudaSuccess)
+      return cleanup(MCD_ERR_CUDA);
+  }
+  auto S = [&](const std::string& name) { return (const uint8_t*)(stage + soff[name]); };
+  auto tile = [&](RowSrc rs, const MatGeom& g, uint8_t* dst) {
+    tile_kernel<<<1024, 256, 0, c->stream>>>(rs, g, p.wdtype, dst);
+  };
+  auto conv = [&](const std::string& name, int64_t count, const float* dst) {
+    to_f32_kernel<<<64, 256, 0, c->stream>>>(S(name), p.wdtype, count, const_cast<float*>(dst));
+  };
+  for (int l = 0; l < p.L; ++l) {
+    const std::string pre = "layers." + std::to_string(l) + ".";
+    RowSrc rs{};
+    rs.seg[0] = S(pre + "wq");
+    rs.seg[1] = S(pre + "wk");
+    rs.seg[2] = S(pre + "wv");
+    rs.seg_rows[0] = (int)qd;
+    rs.seg_rows[1] = (int)kd;
+    rs.seg_rows[2] = (int)kd;
+    rs.nseg = 3;
+    rs.src_cols = (int)H;
+    tile(rs, p.g[MAT_QKV], c->w_arena + c->off_qkv + (size_t)l * p.g[MAT_QKV].stride);
+    RowSrc ro{};
+    ro.seg[0] = S(pre + "wo");
+    ro.seg_rows[0] = (int)H;
+    ro.nseg = 1;
+    ro.src_cols = (int)qd;
+    tile(ro, p.g[MAT_WO], c->w_arena + c->off_wo + (size_t)l * p.g[MAT_WO].stride);
+    RowSrc rg{};
+    rg.seg[0] = S(pre + "wg");
+    rg.seg[1] = S(pre + "wu");
+    rg.nseg = 2;
+    rg.interleave_gu = 1;
+    rg.src_cols = (int)H;
+    tile(rg, p.g[MAT_GU], c->w_arena + c->off_gu + (size_t)l * p.g[MAT_GU].stride);
+    RowSrc rd{};
+    rd.seg[0] = S(pre + "wd");
+    rd.seg_rows[0] = (int)H;
+    rd.nseg = 1;
+    rd.src_cols = (int)F;
+    tile(rd, p.g[MAT_WD], c->w_arena + c->off_wd + (size_t)l * p.g[MAT_WD].stride);
+    conv(pre + "attn_norm", H, p.attn_norm + (size_t)l * H);
+    conv(pre + "ffn_norm", H, p.ffn_norm + (size_t)l * H);
+    if (p.qk_norm) {
+      conv(pre + "q_norm", D, p.q_norm + (size_t)l * D);
+      conv(pre + "k_norm", D, p.k_norm + (size_t)l * D);
+    }
+  }
+  conv("final_norm", H, p.final_norm);
+  for (int j = 1; j <= Kd; ++j) conv("offset." + std::to_string(j), H, p.offsets + (size_t)(j - 1) * H);
+  for (int P = 1; P <= p.P; ++P) {
+    RowSrc rh{};
+    rh.seg[0] = S("head." + std::to_string(P));
+    rh.seg_rows[0] = p.V;
+    rh.nseg = 1;
+    rh.src_cols = (int)H;
+    tile(rh, p.g[MAT_HEAD], c->w_arena + c->off_head + (size_t)(P - 1) * p.g[MAT_HEAD].stride);
+  }
+  if (p.C0V > 0)
+    if (cudaMemcpyAsync(c->w_arena + c->off_embed, S("embed.0"), (size_t)p.C0V * H * es, cudaMemcpyDeviceToDevice,
+                        c->stream) != cudaSuccess)
+      return cleanup(MCD_ERR_CUDA);
+  for (int i = 1; i < p.P; ++i)
+    if (cudaMemcpyAsync(c->w_arena + c->off_embed + (size_t)i * p.embed_stride, S("embed." + std::to_string(i)),
+                        (size_t)p.V * H * es, cudaMemcpyDeviceToDevice, c->stream) != cudaSuccess)
+      return cleanup(MCD_ERR_CUDA);
+  if (cudaGetLastError() != cudaSuccess) return cleanup(MCD_ERR_CUDA);
+  mcd_status s = cleanup(MCD_OK);
+  if (cudaGetLastError() != cudaSuccess) return MCD_ERR_CUDA;
+  c->weights_loaded = true;
+  return s;
+}
+
+static mcd_status launch_begin(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
+                               const int32_t* c0, const float* c0_emb) {
+  FrameParams& p = c->fp;
+  if (!cond) return MCD_ERR_INVALID_ARG;
+  // the kernel reads these rows with 16-byte loads
+  if ((reinterpret_cast<uintptr_t>(cond) & 15u) || (reinterpret_cast<uintptr_t>(c0_emb) & 15u))
+    return MCD_ERR_INVALID_ARG;
+  if (p.C0V > 0 && !c0) return MCD_ERR_INVALID_ARG;
+  if (p.C0V == 0 && !c0_emb) return MCD_ERR_INVALID_ARG;
+  p.cond = cond;
+  p.c0 = c0;
+  p.c0emb = c0_emb;
+  p.stream_id = stream_id;
+  p.frame_idx = frame_idx;
+  begin_frame_kernel<<<1, 256, 0, c->stream>>>(p.st, p.ctr, kMaxCalls * p.ctr_stride, c0, p.C0V);
+  MCD_CHECK(cudaGetLastError());
+  c->frame_begun = true;
+  return MCD_OK;
+}
+
+mcd_status mcd_decode_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
+                            const int32_t* c0, const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats) {
+  if (!c || !codes_out) return MCD_ERR_INVALID_ARG;
+  if (!c->weights_loaded) return MCD_ERR_STATE;
+  mcd_status s = launch_begin(c, stream_id, frame_idx, cond, c0, c0_emb);
+  if (s != MCD_OK) return s;
+  FrameParams p = c->fp;
+  p.codes_out = codes_out;
+  p.stats = stats;
+  p.single_call = 0;
+  p.logits_out = nullptr;
+  p.emitted_out = nullptr;
+  p.n_emitted_out = nullptr;
+  MCD_CHECK(launch_frame_kernel(p, c->stream));
+  return MCD_OK;
+}
+
+mcd_status mcd_begin_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond, const int32_t* c0,
+                           const float* c0_emb) {
+  if (!c) return MCD_ERR_INVALID_ARG;
+  return launch_begin(c, stream_id, frame_idx, cond, c0, c0_emb);
+}
+
+mcd_status mcd_verify_accept(mcd_ctx* c, int32_t* emitted, int32_t* n_emitted, float* logits_out) {
+  if (!c || !emitted || !n_emitted) return MCD_ERR_INVALID_ARG;
+  if (!c->weights_loaded || !c->frame_begun) return MCD_ERR_STATE;
+  FrameParams p = c->fp;
+  p.codes_out = nullptr;
+  p.stats = nullptr;
+  p.single_call = 1;
+  p.emitted_out = emitted;
+  p.n_emitted_out = n_emitted;
+  p.logits_out = logits_out;
+  reset_call_counters_kernel<<<1, 64, 0, c->stream>>>(p.st, p.ctr, p.ctr_stride);
+  zero_emitted_kernel<<<1, 32, 0, c->stream>>>(p.st, n_emitted);
+  MCD_CHECK(cudaGetLastError());
+  MCD_CHECK(launch_frame_kernel(p, c->stream));
+  return MCD_OK;
+}
+
+mcd_status mcd_draft(mcd_ctx* c, int32_t pos_k, int32_t call_idx, const float* h_k, int32_t* draft_ids,
+                     int32_t* q_ids, double* q_probs, float* z_out) {
+  if (!c || !h_k || !draft_ids) return MCD_ERR_INVALID_ARG;
+  if (!c->weights_loaded || !c->frame_begun) return MCD_ERR_STATE;
+  FrameParams& p = c->fp;
+  if (pos_k < 1 || pos_k >= p.P || call_idx < 0 || call_idx >= kMaxCalls) return MCD_ERR_INVALID_ARG;
+  const int n_j = std::min(p.K, p.P - pos_k);
+  if (n_j <= 0) return MCD_OK;
+  float* z = z_out ? z_out : p.logits;  // scratch: the context's logits buffer
+  const int warps = n_j * p.V;
+  draft_logits_kernel<<<(warps * 32 + 255) / 256, 256, 0, c->stream>>>(p, pos_k, n_j, h_k, z);
+  draft_sample_kernel<<<n_j, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(p, pos_k, call_idx, z, p.topk,
+                                                                                  draft_ids, q_ids, q_probs);
+  MCD_CHECK(cudaGetLastError());
+  return MCD_OK;
+}
+
+mcd_status mcd_accept_from_logits(mcd_ctx* c, int32_t a, int32_t n_drafts, int32_t call_idx, const float* p_logits,
+                                  const float* q_logits, const int32_t* draft_ids, int32_t* emitted, int32_t* out2) {
+  if (!c || !p_logits || !emitted || !out2) return MCD_ERR_INVALID_ARG;
+  FrameParams& p = c->fp;
+  if (!c->frame_begun) return MCD_ERR_STATE;
+  if (n_drafts < 0 || n_drafts > p.K || a < 0 || a + n_drafts > p.P || a >= p.P) return MCD_ERR_INVALID_ARG;
+  if (n_drafts > 0 && (!q_logits || !draft_ids)) return MCD_ERR_INVALID_ARG;
+  if (call_idx < 0 || call_idx >= kMaxCalls) return MCD_ERR_INVALID_ARG;
+  accept_logits_kernel<<<1, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(
+      p, a, n_drafts, call_idx, p_logits, q_logits, draft_ids, p.topk, emitted, out2);
+  MCD_CHECK(cudaGetLastError());
+  return MCD_OK;
+}
+
+mcd_status mcd_topk_softmax(mcd_ctx* c, int32_t n_rows, const float* logits, int32_t* ids, double* probs) {
+  if (!c || !logits || n_rows < 0) return MCD_ERR_INVALID_ARG;
+  if (n_rows == 0) return MCD_OK;
+  FrameParams& p = c->fp;
+  if (n_rows > 2 * kMaxRows * (kMaxDraft + 1)) return MCD_ERR_UNSUPPORTED;
+  topk_rows_kernel<<<n_rows, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(logits, p.V, p.top_k, p.T, p.topk,
+                                                                                  ids, probs);
+  MCD_CHECK(cudaGetLastError());
+  return MCD_OK;
+}
+
+int64_t mcd_trace_bytes(const mcd_ctx* c) {
+  if (!c) return 0;
+  return (int64_t)sizeof(mcd_call_trace) * kMaxCalls + (int64_t)2 * kMaxCalls * kMaxRows * c->fp.V * 4;
+}
+
+mcd_status mcd_set_trace(mcd_ctx* c, void* trace) {
+  if (!c) return MCD_ERR_INVALID_ARG;
+  c->fp.trace = static_cast<uint8_t*>(trace);
+  return MCD_OK;
+}
+
+mcd_status mcd_set_timeline(mcd_ctx* c, uint64_t* timeline) {
+  if (!c) return MCD_ERR_INVALID_ARG;
+  c->fp.timeline = reinterpret_cast<unsigned long long*>(timeline);
+  return MCD_OK;
+}
+
+mcd_status mcd_sync(mcd_ctx* c) {
+  if (!c) return MCD_ERR_INVALID_ARG;
+  MCD_CHECK(cudaStreamSynchronize(c->stream));
+  int err = 0;
+  MCD_CHECK(cudaMemcpy(&err, c->fp.err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (err != 0) {
+    MCD_CHECK(cudaMemset(c->fp.err, 0, sizeof(int)));
+    return (mcd_status)err;
+  }
+  return MCD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,1065 @@
+// Persistent frame kernel: every model call of one frame of RVQ-position-aware
+// speculative decoding (arXiv 2609.37007, Sec. 2.2 and Fig. 3) in a single cooperative
+// launch with one CTA per SM.
+//
+// Per call (a "round"): the rows [c_a, d_{a+1}, ..., d_{a+n}] (first call: [cond, c0]) go
+// through the MultiCodeDecoder (5 pre-norm layers: RMSNorm -> QKV -> QK-norm -> RoPE ->
+// causal GQA attention over the per-frame KV cache -> Wo + residual -> RMSNorm ->
+// gate/up -> SwiGLU -> down + residual), the final RMSNorm gives h, LM head a+1+i reads
+// row i (verify) and LM head s+j reads h_s + b_j (draft of position s+j from row s).  Then
+// top-k/temperature softmax of every row, the acceptance step and the next drafts.
+//
+// Work split.  Weight matrices are cut into units of <= 32 KB (see mcd_internal.cuh).
+// Unit u of the call's k-th stage goes to CTA (u + rot) mod n_cta, rot being the number of
+// units of all earlier stages, so every CTA streams about the same bytes.  In each CTA a
+// producer warp issues 1-D bulk copies (cp.async.bulk, evict-first) of its units into a
+// 4-slot shared-memory ring as fast as slots free up -- across stage and call boundaries --
+// while 8 consumer warps wait for the stage's inputs (a global counter reaching n_cta),
+// turn the fp32 activations into bf16 hi/lo mma operands and multiply each unit with
+// mma.m16n8k16 (weights as the 16-row A side, up to 8 activation columns as B).
+// Dependencies between stages are per-call counters; every wait is bounded by wait_ns.
+#include <cooperative_groups.h>
+
+#include "mcd_internal.cuh"
+#include "mcd_sampler.cuh"
+
+namespace mcd {
+
+struct Smem {
+  uint8_t* ring;
+  float* act;
+  uint8_t* bfrag;
+  float* red;
+  float* vec;     // norm gains / final norm + offsets of the current stage
+  uint64_t* full;
+  uint64_t* empty;
+  int* flags;     // [0] stop, [1] abort, [2] last-arriver, [3] cur head/chunk
+  float* inv_rms; // [kMaxRows]
+  int* call_info; // snapshot of the call's state
+};
+
+constexpr int kRingOff = 0;
+constexpr int kActOff = kRingOff + kNumSlots * kSlotBytes;
+constexpr int kBfragOff = kActOff + kActBytes;
+constexpr int kRedOff = kBfragOff + kBfragBytes;
+constexpr int kVecOff = kRedOff + 2 * kRedBytes;
+constexpr int kVecFloats = 6 * 1024;   // final norm + up to 5 offset vectors of hidden <= 1024
+constexpr int kBarOff = kVecOff + kVecFloats * 4;
+constexpr int kFlagOff = kBarOff + 2 * kNumSlots * 8;
+constexpr int kRmsOff = kFlagOff + 64;
+constexpr int kInfoOff = kRmsOff + 64;
+constexpr int kInfoInts = 48;
+constexpr int kSmemBytes = kInfoOff + kInfoInts * 4;
+
+// call_info slots
+enum { CI_CALL = 0, CI_A, CI_ND, CI_POS0, CI_NROWS, CI_FR, CI_DONE, CI_QROW, CI_PLO, CI_PHI, CI_IDS = 16,
+       CI_CALLS = 24, CI_HEADS, CI_KVROWS, CI_ROWSFED, CI_DRAFTED, CI_ACCEPTED };
+
+__device__ __forceinline__ Smem smem_layout(uint8_t* base) {
+  Smem s;
+  s.ring = base + kRingOff;
+  s.act = reinterpret_cast<float*>(base + kActOff);
+  s.bfrag = base + kBfragOff;
+  s.red = reinterpret_cast<float*>(base + kRedOff);
+  s.vec = reinterpret_cast<float*>(base + kVecOff);
+  s.full = reinterpret_cast<uint64_t*>(base + kBarOff);
+  s.empty = s.full + kNumSlots;
+  s.flags = reinterpret_cast<int*>(base + kFlagOff);
+  s.inv_rms = reinterpret_cast<float*>(base + kRmsOff);
+  s.call_info = reinterpret_cast<int*>(base + kInfoOff);
+  return s;
+}
+
+// ------------------------------------------------------------------------------------
+// Schedule shared by producer and consumers
+// ------------------------------------------------------------------------------------
+__device__ __forceinline__ int n_stages(const FrameParams& p) { return 4 * p.L + 1; }
+__device__ __forceinline__ int stage_kind(int si, int L) { return si < 4 * L ? (si & 3) : MAT_HEAD; }
+
+__device__ __forceinline__ int stage_units(const FrameParams& p, int si, int n_heads) {
+  const int kind = stage_kind(si, p.L);
+  return kind == MAT_HEAD ? n_heads * p.g[MAT_HEAD].n_units : p.g[kind].n_units;
+}
+
+__device__ __forceinline__ const uint8_t* unit_src(const FrameParams& p, int si, int u, int p_lo) {
+  const int kind = stage_kind(si, p.L);
+  const MatGeom& g = p.g[kind];
+  if (kind == MAT_HEAD) {
+    const int hi = u / g.n_units, uu = u % g.n_units;
+    return p.w_head + (long long)(p_lo + hi - 1) * g.stride + (long long)uu * g.unit_bytes;
+  }
+  const int layer = si >> 2;
+  const uint8_t* base = kind == MAT_QKV ? p.w_qkv : kind == MAT_WO ? p.w_wo : kind == MAT_GU ? p.w_gu : p.w_wd;
+  return base + (long long)layer * g.stride + (long long)u * g.unit_bytes;
+}
+
+__device__ __forceinline__ int first_unit(int cta, int rot, int n_cta) {
+  int f = cta - rot;
+  f %= n_cta;
+  return f < 0 ? f + n_cta : f;
+}
+
+// heads touched by a call: P_lo = a+1, P_hi = min(n_pos, last row position + K)
+__device__ __forceinline__ void head_range(const FrameParams& p, int a, int pos0, int n_rows, int& p_lo,
+                                           int& p_hi) {
+  p_lo = a + 1;
+  p_hi = min(p.P, pos0 + n_rows - 1 + p.K);
+}
+
+// ------------------------------------------------------------------------------------
+// Producer: one thread streams this CTA's units into the ring.
+// ------------------------------------------------------------------------------------
+__device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
+  const int cta = blockIdx.x, n_cta = p.n_cta;
+  const uint64_t pol = policy_evict_first();
+  uint32_t issued = 0;
+  int rot = 0;
+  volatile int* stop = sm.flags;
+  bool halt = false;
+  for (int call = call0; call < kMaxCalls && !halt; ++call) {
+    int p_lo = 0, p_hi = -1;
+    for (int si = 0; si < n_stages(p) && !halt; ++si) {
+      int n_heads = 0;
+      if (stage_kind(si, p.L) == MAT_HEAD) {
+        if (call != call0) {
+          if (!wait_counter(p.ctr + call * p.ctr_stride + ctr_ready(p.L), 1u, p.err, p.wait_ns)) {
+            halt = true;
+            break;
+          }
+        }
+        const int4 s0 = __ldcg(reinterpret_cast<const int4*>(p.st));        // call, a, done, n_d
+        const int2 s1 = __ldcg(reinterpret_cast<const int2*>(p.st) + 2);    // pos0, n_rows
+        if (s0.z) {
+          halt = true;
+          break;
+        }
+        head_range(p, s0.y, s1.x, s1.y, p_lo, p_hi);
+        n_heads = p_hi - p_lo + 1;
+      }
+      const int n = stage_units(p, si, n_heads);
+      const uint32_t bytes = (uint32_t)p.g[stage_kind(si, p.L)].unit_bytes;
+      for (int u = first_unit(cta, rot, n_cta); u < n; u += n_cta) {
+        const uint32_t slot = issued % kNumSlots;
+        if (issued >= (uint32_t)kNumSlots) {
+          if (!wait_mbar(&sm.empty[slot], ((issued / kNumSlots) - 1u) & 1u, p.err, p.wait_ns, stop)) {
+            halt = true;
+            break;
+          }
+        }
+        mbar_arrive_expect_tx(&sm.full[slot], bytes);
+        bulk_g2s(sm.ring + (size_t)slot * kSlotBytes, unit_src(p, si, u, p_lo), bytes, &sm.full[slot], pol);
+        ++issued;
+      }
+      rot = (rot + n) % n_cta;
+    }
+    if (p.single_call) break;
+  }
+  // Drain: every issued copy must land before the CTA may exit.
+  const uint32_t first = issued > (uint32_t)kNumSlots ? issued - kNumSlots : 0u;
+  for (uint32_t i = first; i < issued; ++i) {
+    const uint32_t slot = i % kNumSlots;
+    uint64_t t0 = globaltimer();
+    while (!mbar_try_wait(&sm.full[slot], (i / kNumSlots) & 1u)) {
+      if (globaltimer() - t0 > p.wait_ns) {
+        atomicCAS(p.err, 0, (int)MCD_ERR_TIMEOUT);
+        break;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// Consumer helpers
+// ------------------------------------------------------------------------------------
+struct Cons {
+  const FrameParams& p;
+  Smem& sm;
+  uint32_t seq;   // units consumed (ring sequence)
+  int buf;        // reduction buffer parity
+  int rot;
+  bool abort_;
+  __device__ Cons(const FrameParams& pp, Smem& s) : p(pp), sm(s), seq(0), buf(0), rot(0), abort_(false) {}
+};
+
+__device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned target) {
+  if (threadIdx.x == 0) {
+    bool ok = wait_counter(ctr, target, c.p.err, c.p.wait_ns);
+    if (!ok) c.sm.flags[1] = 1;
+  }
+  consumer_sync();
+  if (*(volatile int*)&c.sm.flags[1]) c.abort_ = true;
+  return !c.abort_;
+}
+
+__device__ __forceinline__ void timeline_max(const Cons& c, int call, int idx);
+__device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call = 0, int slot = -1) {
+  consumer_sync();
+  if (slot >= 0) timeline_max(c, call, slot);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(ctr, 1u);
+  }
+  if (slot >= 0) timeline_max(c, call, slot + 1);
+}
+
+// Optional profiling stamps (%globaltimer, ns), 128 per call.  Slots: 0 call start;
+// 1 top-k inputs ready; 2 top-k done (CTA 0); 3 top-k done (last CTA); 4..7 acceptance
+// start / records staged / decided / end.  Stage s (0..4L, 4l+k = layer l step k, 4L =
+// heads) at 8+4s: +0 inputs ready (CTA 0), +1 first unit's weights in smem (CTA 0),
+// +2 last epilogue done and +3 signalled (latest CTA).
+constexpr int kTimelineSlots = 128;
+__device__ __forceinline__ void timeline(const Cons& c, int call, int idx, bool any_cta = false) {
+  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots)
+    c.p.timeline[call * kTimelineSlots + idx] = globaltimer();
+}
+__device__ __forceinline__ void timeline_max(const Cons& c, int call, int idx) {
+  if (c.p.timeline && threadIdx.x == 0 && idx < kTimelineSlots)
+    atomicMax(c.p.timeline + call * kTimelineSlots + idx, (unsigned long long)globaltimer());
+}
+
+// Activation operand: bf16 weights -> hi/lo bf16 B fragments; fp32 weights -> fp32 rows.
+// `val(n, k)` gives the fp32 activation of column n (n < ncols) at input index k.
+template <int WT, class F>
+__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, F val) {
+  const int tid = threadIdx.x;
+  if (WT == MCD_WEIGHT_BF16) {
+    uint4* bf = reinterpret_cast<uint4*>(c.sm.bfrag);
+    const int total = (Kdim / 16) * 32;
+    for (int idx = tid; idx < total; idx += kConsumerThreads) {
+      const int kt = idx >> 5, ln = idx & 31, n = ln >> 2, t = ln & 3;
+      uint4 o = make_uint4(0u, 0u, 0u, 0u);
+      if (n < ncols) {
+        const int k0 = kt * 16 + 2 * t;
+        uint32_t h0, l0, h1, l1, h2, l2, h3, l3;
+        split_bf16(val(n, k0), h0, l0);
+        split_bf16(val(n, k0 + 1), h1, l1);
+        split_bf16(val(n, k0 + 8), h2, l2);
+        split_bf16(val(n, k0 + 9), h3, l3);
+        o.x = h0 | (h1 << 16);
+        o.y = h2 | (h3 << 16);
+        o.z = l0 | (l1 << 16);
+        o.w = l2 | (l3 << 16);
+      }
+      bf[idx] = o;
+    }
+  } else {
+    float* xs = reinterpret_cast<float*>(c.sm.bfrag);
+    const int total = kMaxRows * Kdim;
+    for (int idx = tid; idx < total; idx += kConsumerThreads) {
+      const int n = idx / Kdim, k = idx - n * Kdim;
+      xs[idx] = n < ncols ? val(n, k) : 0.0f;
+    }
+  }
+  consumer_sync();
+}
+
+// Multiply the unit in ring slot `slot` with the prepared operand; partial sums of every
+// (m-tile, k-group) land in the reduction buffer in mma C-fragment order.
+template <int WT>
+__device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_t* slotp, int Kdim) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Mu = g.Mu, Ku = g.Ku;
+  const int Gk = kConsumerWarps / Mu;
+  const int mi = warp % Mu, kg = warp / Mu, kts = Ku / Gk;
+  float4* red = reinterpret_cast<float4*>(c.sm.red + c.buf * (kRedBytes / 4));
+  if (WT == MCD_WEIGHT_BF16) {
+    const uint4* A = reinterpret_cast<const uint4*>(slotp) + (size_t)(mi * Ku + kg * kts) * 32 + lane;
+    const uint4* B = reinterpret_cast<const uint4*>(c.sm.bfrag) + (size_t)(kg * kts) * 32 + lane;
+    float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+    for (int t = 0; t < kts; ++t) {
+      const uint4 a = A[t * 32];
+      const uint4 b = B[t * 32];
+      mma_bf16_16816(a0, a, b.x, b.y);
+      mma_bf16_16816(a1, a, b.z, b.w);
+    }
+    red[(kg * Mu + mi) * 32 + lane] = make_float4(a0[0] + a1[0], a0[1] + a1[1], a0[2] + a1[2], a0[3] + a1[3]);
+  } else {
+    const int rr = lane & 15, kh = lane >> 4;
+    const float* xs = reinterpret_cast<const float*>(c.sm.bfrag);
+    const float4* A = reinterpret_cast<const float4*>(slotp) + (size_t)(mi * Ku + kg * kts) * 64 + lane * 2;
+    float acc[kMaxRows];
+#pragma unroll
+    for (int n = 0; n < kMaxRows; ++n) acc[n] = 0.f;
+    for (int t = 0; t < kts; ++t) {
+      const float4 w0 = A[t * 64], w1 = A[t * 64 + 1];
+      const int col = (kg * kts + t) * 16 + kh * 8;
+#pragma unroll
+      for (int n = 0; n < kMaxRows; ++n) {
+        const float4 x0 = *reinterpret_cast<const float4*>(xs + n * Kdim + col);
+        const float4 x1 = *reinterpret_cast<const float4*>(xs + n * Kdim + col + 4);
+        acc[n] += w0.x * x0.x + w0.y * x0.y + w0.z * x0.z + w0.w * x0.w + w1.x * x1.x + w1.y * x1.y +
+                  w1.z * x1.z + w1.w * x1.w;
+      }
+    }
+#pragma unroll
+    for (int n = 0; n < kMaxRows; ++n) acc[n] += __shfl_xor_sync(0xFFFFFFFFu, acc[n], 16);
+    if (lane < 16) {
+      float* rf = reinterpret_cast<float*>(red + (kg * Mu + mi) * 32);
+#pragma unroll
+      for (int n = 0; n < kMaxRows; ++n) rf[((rr & 7) * 4 + (n >> 1)) * 4 + (rr >> 3) * 2 + (n & 1)] = acc[n];
+    }
+  }
+}
+
+// Sum of the k-group partials of output (mi, row rr, column n) of the current unit.
+__device__ __forceinline__ float red_get(const Cons& c, const MatGeom& g, int mi, int rr, int n) {
+  const int Gk = kConsumerWarps / g.Mu;
+  const float* red = c.sm.red + c.buf * (kRedBytes / 4);
+  const int ln = (rr & 7) * 4 + (n >> 1), idx = (rr >> 3) * 2 + (n & 1);
+  float v = 0.f;
+  for (int kg = 0; kg < Gk; ++kg) v += red[((kg * g.Mu + mi) * 32 + ln) * 4 + idx];
+  return v;
+}
+
+// Run every unit of stage `si` assigned to this CTA.  prep(u) prepares the operand for
+// unit u when needed; epi(u, mi, rr, n, value) consumes outputs.
+template <int WT, class Prep, class Epi>
+__device__ __forceinline__ void run_stage(Cons& c, int si, int n_units, int Kdim, Prep prep, Epi epi,
+                                          bool pairs_rows = false, int call = 0) {
+  const FrameParams& p = c.p;
+  const MatGeom& g = p.g[stage_kind(si, p.L)];
+  const int lane = threadIdx.x & 31;
+  timeline(c, call, 8 + 4 * si);
+  bool first = true;
+  for (int u = first_unit(blockIdx.x, c.rot, p.n_cta); u < n_units; u += p.n_cta) {
+    prep(u);
+    const uint32_t slot = c.seq % kNumSlots;
+    if (!wait_mbar(&c.sm.full[slot], (c.seq / kNumSlots) & 1u, p.err, p.wait_ns, nullptr)) {
+      c.sm.flags[1] = 1;
+    }
+    if (first) timeline(c, call, 9 + 4 * si);
+    first = false;
+    consumer_sync();
+    if (*(volatile int*)&c.sm.flags[1]) {
+      c.abort_ = true;
+      return;
+    }
+    unit_mma<WT>(c, g, c.sm.ring + (size_t)slot * kSlotBytes, Kdim);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&c.sm.empty[slot]);
+    ++c.seq;
+    consumer_sync();
+    const int outs = g.Mu * (pairs_rows ? 64 : 128);
+    for (int o = threadIdx.x; o < outs; o += kConsumerThreads) {
+      const int per = pairs_rows ? 64 : 128;
+      const int mi = o / per, r = o % per;
+      const int rr = r >> 3, n = r & 7;
+      epi(u, mi, rr, n);
+    }
+    c.buf ^= 1;
+  }
+  c.rot = (c.rot + n_units) % p.n_cta;
+}
+
+__device__ __forceinline__ float bf16_or_f32(const uint8_t* base, long long idx, int wdtype) {
+  if (wdtype == MCD_WEIGHT_BF16) return bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(base)[idx]);
+  return reinterpret_cast<const float*>(base)[idx];
+}
+
+// Rows of the residual stream into act[n][H] and per-row 1/rms into inv_rms.
+__device__ __forceinline__ void rows_rms(Cons& c, int n_rows, int H) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp < n_rows) {
+    float ss = 0.f;
+    for (int k = lane; k < H; k += 32) {
+      const float v = c.sm.act[warp * H + k];
+      ss += v * v;
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
+    if (lane == 0) c.sm.inv_rms[warp] = rsqrtf(ss / (float)H + c.p.eps);
+  }
+  consumer_sync();
+}
+
+// Copy n_rows rows of `len` floats (src row stride `ld`) into dst[n][len] with 16-byte
+// loads, four in flight per thread (every address is independent: one L2 round trip).
+__device__ __forceinline__ void g2s_rows(float* dst, const float* src, int n_rows, int len, long long ld) {
+  const int per = len >> 2, n4 = n_rows * per;
+  float4* d = reinterpret_cast<float4*>(dst);
+  for (int i = threadIdx.x; i < n4; i += 4 * kConsumerThreads) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = i + u * kConsumerThreads;
+      if (j < n4) v[u] = __ldcg(reinterpret_cast<const float4*>(src + (long long)(j / per) * ld) + (j % per));
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = i + u * kConsumerThreads;
+      if (j < n4) d[j] = v[u];
+    }
+  }
+}
+
+// Read-only vector (weights) into shared memory; no barrier (the caller syncs later).
+__device__ __forceinline__ void g2s_vec(float* dst, const float* src, int n) {
+  const int n4 = n >> 2;
+  for (int i = threadIdx.x; i < n4; i += kConsumerThreads)
+    reinterpret_cast<float4*>(dst)[i] = __ldg(reinterpret_cast<const float4*>(src) + i);
+}
+
+__device__ __forceinline__ void load_x(Cons& c, int n_rows) {
+  g2s_rows(c.sm.act, c.p.x, n_rows, c.p.H, c.p.H);
+  consumer_sync();
+}
+
+// Layer-0 input rows of the call: [cond, c0] on the first call, else embeddings of
+// [c_a, d_{a+1}, ...] (table of position a+i).  CTA 0 also seeds the residual stream.
+__device__ void gather_inputs(Cons& c) {
+  const FrameParams& p = c.p;
+  const int* ci = c.sm.call_info;
+  const int n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
+  const int H = p.H, per = H / 8;      // 8 elements (16 B of bf16 or 2x16 B of fp32) per item
+  for (int it = threadIdx.x; it < n_rows * per; it += kConsumerThreads) {
+    const int n = it / per, k0 = (it - n * per) * 8;
+    const int pos = pos0 + n;
+    float v[8];
+    if (pos == 0 || (pos == 1 && p.C0V == 0)) {
+      const float4* src = reinterpret_cast<const float4*>((pos == 0 ? p.cond : p.c0emb) + k0);
+      const float4 a = __ldg(src), b = __ldg(src + 1);
+      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    } else {
+      const int table = pos - 1;
+      int id = ci[CI_IDS + n];
+      if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {  // a c0 outside table 0: fail the frame
+        if (k0 == 0) atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
+        id = 0;
+      }
+      const uint8_t* row = p.embed + (long long)table * p.embed_stride;
+      if (p.wdtype == MCD_WEIGHT_BF16) {
+        const uint4 w = __ldg(reinterpret_cast<const uint4*>(row + ((long long)id * H + k0) * 2));
+        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          v[2 * e] = bf16_bits_to_f32(ww[e] & 0xFFFFu);
+          v[2 * e + 1] = bf16_bits_to_f32(ww[e] >> 16);
+        }
+      } else {
+        const float4* src = reinterpret_cast<const float4*>(row + ((long long)id * H + k0) * 4);
+        const float4 a = __ldg(src), b = __ldg(src + 1);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+      }
+    }
+    float4* dst = reinterpret_cast<float4*>(c.sm.act + n * H + k0);
+    dst[0] = make_float4(v[0], v[1], v[2], v[3]);
+    dst[1] = make_float4(v[4], v[5], v[6], v[7]);
+    if (blockIdx.x == 0) {
+      float4* gx = reinterpret_cast<float4*>(p.x + (size_t)n * H + k0);
+      gx[0] = dst[0];
+      gx[1] = dst[1];
+    }
+  }
+  consumer_sync();
+}
+
+// Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
+// per-frame cache plus the new rows).  Scratch spans act + bfrag (64 KB): the kv head's
+// cached rows are staged in shared memory first, so every dot product reads smem.  The o
+// rows land in act[0..n_rows) x D; the new K/V rows are written to the cache if write_kv.
+__device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
+  const FrameParams& p = c.p;
+  const int* ci = c.sm.call_info;
+  const int n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
+  const int D = p.D, group = p.NH / p.NKV, g = h / group;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int npos_all = pos0 + n_rows;          // keys 0..pos0+n_rows-1
+  float* o = c.sm.act;                         // [8][D]
+  float* qs = o + kMaxRows * 128;              // [8][D]
+  float* ks = qs + kMaxRows * 128;             // [kMaxPos][D]: cached rows, then the new rows
+  float* vs = ks + kMaxPos * 128;              // [kMaxPos][D]
+  float* pr = vs + kMaxPos * 128;              // [8][kMaxPos]
+  float* nrm = pr + kMaxRows * kMaxPos;        // [16]
+  float* gq = nrm + 16;                        // [D]
+  float* gk = gq + 128;                        // [D]
+  const float* kc = p.kcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const float* vc = p.vcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
+  // one round of independent 16-byte loads: q/k/v of the call, cached K/V, QK-norm gains
+  {
+    const int per = D >> 2;
+    const int nq = n_rows * per, nc = pos0 * per;
+    const int total = 3 * nq + 2 * nc + (p.qk_norm ? 2 * per : 0);
+    for (int i = tid; i < total; i += kConsumerThreads) {
+      float4 v;
+      float* dst;
+      if (i < 3 * nq) {
+        const int w = i / nq, r = i - w * nq, n = r / per, d4 = r - n * per;
+        const float* row = p.qkv + (size_t)n * p.qkv_dim + (w == 0 ? qoff : w == 1 ? koff : voff);
+        v = __ldcg(reinterpret_cast<const float4*>(row) + d4);
+        dst = (w == 0 ? qs + n * D : w == 1 ? ks + (pos0 + n) * D : vs + (pos0 + n) * D) + 4 * d4;
+      } else if (i < 3 * nq + 2 * nc) {
+        const int r = i - 3 * nq, w = r / nc, rr = r - w * nc, j = rr / per, d4 = rr - j * per;
+        v = __ldcg(reinterpret_cast<const float4*>((w == 0 ? kc : vc) + (size_t)j * D) + d4);
+        dst = (w == 0 ? ks : vs) + j * D + 4 * d4;
+      } else {
+        const int r = i - 3 * nq - 2 * nc, w = r / per, d4 = r - w * per;
+        v = __ldg(reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D) + d4);
+        dst = (w == 0 ? gq : gk) + 4 * d4;
+      }
+      *reinterpret_cast<float4*>(dst) = v;
+    }
+  }
+  consumer_sync();
+  float* knew = ks + pos0 * D;
+  float* vnew = vs + pos0 * D;
+  if (p.qk_norm) {
+    for (int vi = warp; vi < 2 * n_rows; vi += kConsumerWarps) {
+      const float* v = vi < n_rows ? qs + vi * D : knew + (vi - n_rows) * D;
+      float ss = 0.f;
+      for (int d = lane; d < D; d += 32) ss += v[d] * v[d];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+      if (lane == 0) nrm[vi] = rsqrtf(ss / (float)D + p.eps);
+    }
+    consumer_sync();
+  }
+  // QK-norm gain and RoPE (rotate-half pairs (d, d + D/2)) on the new rows
+  const int half = D / 2;
+  for (int idx = tid; idx < 2 * n_rows * half; idx += kConsumerThreads) {
+    const int vi = idx / half, d = idx - vi * half;
+    const bool isq = vi < n_rows;
+    const int n = isq ? vi : vi - n_rows;
+    float* v = isq ? qs + n * D : knew + n * D;
+    float a = v[d], b = v[d + half];
+    if (p.qk_norm) {
+      const float sc = nrm[vi];
+      const float* gg = isq ? gq : gk;
+      a = a * sc * gg[d];
+      b = b * sc * gg[d + half];
+    }
+    const float2 cs = p.rope[(pos0 + n) * half + d];
+    v[d] = a * cs.x - b * cs.y;
+    v[d + half] = b * cs.x + a * cs.y;
+  }
+  consumer_sync();
+  if (write_kv) {
+    float* kcw = p.kcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+    float* vcw = p.vcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+    const int n4 = n_rows * D / 4;
+    for (int i = tid; i < 2 * n4; i += kConsumerThreads) {
+      const int w = i / n4, r = i - w * n4;
+      float4* dst = reinterpret_cast<float4*>((w ? vcw : kcw) + (size_t)pos0 * D) + r;
+      *dst = reinterpret_cast<const float4*>(w ? vnew : knew)[r];
+    }
+  }
+  // scores: warp n; lane = (key group kq, dim quarter dq)
+  const float scale = rsqrtf((float)D);
+  if (warp < n_rows) {
+    const int n = warp, npos = pos0 + n + 1;
+    const int kq = lane >> 2, dq = lane & 3, dl = D / 4;
+    const float* qv = qs + n * D + dq * dl;
+    float sc[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int j = kq + 8 * i;
+      float acc = 0.f;
+      if (j < npos) {
+        const float* kv = ks + j * D + dq * dl;
+        for (int d = 0; d < dl; ++d) acc += qv[d] * kv[d];
+      }
+      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
+      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 2);
+      sc[i] = j < npos ? acc * scale : -INFINITY;
+    }
+    float m = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+#pragma unroll
+    for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
+    float e[4], sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      e[i] = (kq + 8 * i) < npos ? __expf(sc[i] - m) : 0.f;
+      sum += (dq == 0) ? e[i] : 0.f;
+    }
+#pragma unroll
+    for (int off = 16; off; off >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, off);
+    if (dq == 0) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) pr[n * kMaxPos + kq + 8 * i] = e[i] / sum;
+    }
+    __syncwarp();
+    for (int d = lane; d < D; d += 32) {
+      float acc = 0.f;
+      for (int j = 0; j < npos; ++j) acc += pr[n * kMaxPos + j] * vs[j * D + d];
+      o[n * D + d] = acc;
+    }
+  }
+  (void)npos_all;
+  consumer_sync();
+}
+
+// Columns (row n, offset j) that LM head P reads in this call, in increasing row order.
+__device__ __forceinline__ int head_columns(const FrameParams& p, const int* ci, int P, int* cn, int* cj) {
+  const int fr = ci[CI_FR], n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
+  int nc = 0;
+  for (int n = fr; n < n_rows; ++n) {
+    const int j = P - (pos0 + n);
+    if (j >= 0 && j <= p.K && nc < kMaxRows) {
+      cn[nc] = n;
+      cj[nc] = j;
+      ++nc;
+    }
+  }
+  return nc;
+}
+
+// ------------------------------------------------------------------------------------
+// One call
+// ------------------------------------------------------------------------------------
+template <int WT>
+__device__ void run_call(Cons& c, int call) {
+  const FrameParams& p = c.p;
+  Smem& sm = c.sm;
+  int* ci = sm.call_info;
+  const int L = p.L, H = p.H, D = p.D, F = p.F;
+  unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
+  const int n_rows = ci[CI_NROWS];
+  const unsigned N = (unsigned)p.n_cta;
+
+  for (int l = 0; l < L; ++l) {
+    // ---- S1: RMSNorm -> QKV -------------------------------------------------------
+    g2s_vec(sm.vec, p.attn_norm + (size_t)l * H, H);      // independent of the wait below
+    if (l == 0) {
+      gather_inputs(c);
+    } else {
+      if (!cons_wait(c, ctr + ctr_stage(l - 1, 3), N)) return;
+      load_x(c, n_rows);
+    }
+    rows_rms(c, n_rows, H);
+    prep_operand<WT>(c, n_rows, H, [&](int n, int k) { return sm.act[n * H + k] * sm.inv_rms[n] * sm.vec[k]; });
+    run_stage<WT>(
+        c, 4 * l + 0, p.g[MAT_QKV].n_units, H, [&](int) {},
+        [&](int u, int mi, int rr, int n) {
+          const MatGeom& g = p.g[MAT_QKV];
+          const float v = red_get(c, g, mi, rr, n);
+          const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+          if (n < n_rows) p.qkv[(size_t)n * p.qkv_dim + row] = v;
+        },
+        false, call);
+    if (c.abort_) return;
+    cons_signal(c, ctr + ctr_stage(l, 0), call, 10 + 4 * (4 * l + 0));
+
+    // ---- S2: attention (per query head) -> Wo + residual ---------------------------
+    if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
+    {
+      const MatGeom& g = p.g[MAT_WO];
+      const int group = p.NH / p.NKV;
+      sm.flags[3] = -1;
+      consumer_sync();
+      run_stage<WT>(
+          c, 4 * l + 1, g.n_units, D,
+          [&](int u) {
+            const int h = u / g.n_mb, mb = u % g.n_mb;
+            if (sm.flags[3] != h) {
+              consumer_sync();
+              attention_head(c, l, h, (h % group) == 0 && mb == 0);
+              prep_operand<WT>(c, n_rows, D, [&](int n, int k) { return sm.act[n * D + k]; });
+              if (threadIdx.x == 0) sm.flags[3] = h;
+            } else if ((h % group) == 0 && mb == 0) {
+              // a CTA meets head h's m-block 0 first, so this branch only guards the
+              // invariant that the KV writer always recomputes its rows
+              consumer_sync();
+              attention_head(c, l, h, true);
+              prep_operand<WT>(c, n_rows, D, [&](int n, int k) { return sm.act[n * D + k]; });
+            }
+          },
+          [&](int u, int mi, int rr, int n) {
+            const float v = red_get(c, g, mi, rr, n);
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+            if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
+          },
+          false, call);
+      if (c.abort_) return;
+    }
+    cons_signal(c, ctr + ctr_stage(l, 1), call, 10 + 4 * (4 * l + 1));
+
+    // ---- S3: RMSNorm -> gate/up -> SwiGLU ------------------------------------------
+    g2s_vec(sm.vec, p.ffn_norm + (size_t)l * H, H);
+    if (!cons_wait(c, ctr + ctr_stage(l, 1), N)) return;
+    load_x(c, n_rows);
+    rows_rms(c, n_rows, H);
+    {
+      prep_operand<WT>(c, n_rows, H, [&](int n, int k) { return sm.act[n * H + k] * sm.inv_rms[n] * sm.vec[k]; });
+      const MatGeom& g = p.g[MAT_GU];
+      run_stage<WT>(
+          c, 4 * l + 2, g.n_units, H, [&](int) {},
+          [&](int u, int mi, int rr, int n) {
+            // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
+            const float gt = red_get(c, g, mi, rr, n);
+            const float up = red_get(c, g, mi, rr + 8, n);
+            const int tile = (u % g.n_mb) * g.Mu + mi;
+            const int j = tile * 8 + rr;
+            if (n < n_rows) p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * up;
+          },
+          true, call);
+      if (c.abort_) return;
+    }
+    cons_signal(c, ctr + ctr_stage(l, 2), call, 10 + 4 * (4 * l + 2));
+
+    // ---- S4: down + residual --------------------------------------------------------
+    if (!cons_wait(c, ctr + ctr_stage(l, 2), N)) return;
+    {
+      const MatGeom& g = p.g[MAT_WD];
+      const int Kc = g.Ku * 16;
+      sm.flags[3] = -1;
+      consumer_sync();
+      run_stage<WT>(
+          c, 4 * l + 3, g.n_units, Kc,
+          [&](int u) {
+            const int kc = u / g.n_mb;
+            if (sm.flags[3] != kc) {
+              consumer_sync();
+              g2s_rows(sm.act, p.mbuf + (size_t)kc * Kc, n_rows, Kc, F);
+              consumer_sync();
+              prep_operand<WT>(c, n_rows, Kc, [&](int n, int k) { return sm.act[n * Kc + k]; });
+              if (threadIdx.x == 0) sm.flags[3] = kc;
+            }
+          },
+          [&](int u, int mi, int rr, int n) {
+            const float v = red_get(c, g, mi, rr, n);
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+            if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
+          },
+          false, call);
+      if (c.abort_) return;
+    }
+    cons_signal(c, ctr + ctr_stage(l, 3), call, 10 + 4 * (4 * l + 3));
+  }
+
+  // ---- S5: final RMSNorm -> verify and draft heads -------------------------------------
+  // vec = [final norm | b_1 .. b_min(K,5)]; offsets beyond the fifth are read through L1
+  const int k_sm = min(p.K, kVecFloats / H - 1);
+  g2s_vec(sm.vec, p.final_norm, H);
+  g2s_vec(sm.vec + H, p.offsets, k_sm * H);
+  for (int i = threadIdx.x * 32; i < (p.K - k_sm) * H; i += kConsumerThreads * 32)
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(p.offsets + (size_t)k_sm * H + i));
+  if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
+  load_x(c, n_rows);
+  rows_rms(c, n_rows, H);
+  for (int idx = threadIdx.x; idx < n_rows * H; idx += kConsumerThreads) {
+    const int n = idx / H, k = idx - n * H;
+    sm.act[idx] = sm.act[idx] * sm.inv_rms[n] * sm.vec[k];
+  }
+  consumer_sync();
+  {
+    const MatGeom& g = p.g[MAT_HEAD];
+    const int p_lo = ci[CI_PLO], n_heads = ci[CI_PHI] - ci[CI_PLO] + 1;
+    __shared__ int cn[kMaxRows], cj[kMaxRows], ncols_sh;
+    sm.flags[3] = -1;
+    consumer_sync();
+    run_stage<WT>(
+        c, 4 * L, n_heads * g.n_units, H,
+        [&](int u) {
+          const int hi = u / g.n_units;
+          if (sm.flags[3] != hi) {
+            consumer_sync();
+            if (threadIdx.x == 0) {
+              ncols_sh = head_columns(p, ci, p_lo + hi, cn, cj);
+              sm.flags[3] = hi;
+            }
+            consumer_sync();
+            prep_operand<WT>(c, ncols_sh, H, [&](int col, int k) {
+              const int j = cj[col];
+              float v = sm.act[cn[col] * H + k];
+              if (j > 0) v += j <= k_sm ? sm.vec[j * H + k] : __ldg(p.offsets + (size_t)(j - 1) * H + k);
+              return v;
+            });
+          }
+        },
+        [&](int u, int mi, int rr, int n) {
+          if (n < ncols_sh) {
+            const float v = red_get(c, g, mi, rr, n);
+            const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
+            p.logits[((size_t)cn[n] * (kMaxDraft + 1) + cj[n]) * p.V + id] = v;
+          }
+        },
+        false, call);
+    if (c.abort_) return;
+  }
+  cons_signal(c, ctr + ctr_heads(L), call, 10 + 4 * (4 * L));
+
+  // ---- S6: top-k / temperature softmax of every logits row -----------------------------
+  if (!cons_wait(c, ctr + ctr_heads(L), N)) return;
+  timeline(c, call, 1);
+  {
+    const int fr = ci[CI_FR], pos0 = ci[CI_POS0];
+    TopkScratch& ts = *reinterpret_cast<TopkScratch*>(sm.act);
+    TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
+    int pair = 0;
+    for (int n = fr; n < n_rows; ++n) {
+      const int kn = min(p.K, p.P - (pos0 + n));
+      for (int j = 0; j <= kn; ++j, ++pair) {
+        if (pair % p.n_cta != (int)blockIdx.x) continue;
+        const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
+        block_topk(p.logits + ((size_t)n * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
+                   recs + n * (kMaxDraft + 1) + j);
+        consumer_sync();
+      }
+    }
+  }
+  consumer_sync();
+  timeline(c, call, 2);
+  timeline_max(c, call, 3);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned old = atomicAdd(ctr + ctr_topk(L), 1u);
+    sm.flags[2] = (old == N - 1u) ? 1 : 0;
+    if (sm.flags[2]) __threadfence();
+  }
+  consumer_sync();
+}
+
+// Copy distribution records into shared memory with independent word loads: the header,
+// ids[0..k) and e[0..k) of each (k = top_k; entries past a record's n are never read).
+template <class Src>
+__device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src) {
+  constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kEWord = offsetof(TopkRec, e) / 4;
+  const int words = kIdsWord + 3 * k;
+  for (int i = threadIdx.x; i < nrec * words; i += kConsumerThreads) {
+    const int r = i / words, w = i - r * words;
+    const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kEWord + (w - kIdsWord - k));
+    reinterpret_cast<int*>(dst + r)[off] = __ldcg(reinterpret_cast<const int*>(src(r)) + off);
+  }
+}
+
+// Acceptance step and next drafts (run by the CTA that finished top-k last).  Every record
+// it reads is first staged in shared memory (act + bfrag, 64 KB).
+__device__ void accept_step(Cons& c, int call) {
+  const FrameParams& p = c.p;
+  Smem& sm = c.sm;
+  const int* ci = sm.call_info;
+  const int a = ci[CI_A], n_d = ci[CI_ND], pos0 = ci[CI_POS0], n_rows = ci[CI_NROWS];
+  const int qrow = ci[CI_QROW];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
+  const TopkRec* prev = p.topk + (size_t)((call + 1) & 1) * kMaxRows * (kMaxDraft + 1);
+  TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // [n_p + n_d] staged records
+  const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
+  ResidualScratch& rs = *reinterpret_cast<ResidualScratch*>(srec + 2 * kMaxRows);
+  __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
+  timeline(c, call, 4, true);
+  stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
+    return r < n_p ? cur + (a + 1 + r - pos0) * (kMaxDraft + 1) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p);
+  });
+  consumer_sync();
+  timeline(c, call, 5, true);
+  if (warp == 0) {
+    int drafts[kMaxDraft + 1];
+    for (int i = 0; i < n_d; ++i) drafts[i] = ci[CI_IDS + 1 + i];
+    AcceptResult r = warp_accept(
+        a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(srec + i); },
+        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, call, rs);
+    if (lane == 0) {
+      for (int t = 0; t < r.n_emit; ++t) s_emit[t] = r.emitted[t];
+      s_nemit = r.n_emit;
+      s_nacc = r.n_acc;
+    }
+  }
+  consumer_sync();
+  timeline(c, call, 6, true);
+  const int a_new = a + s_nemit;
+  const int m = a_new - pos0;
+  const int n_next = min(p.K, p.P - a_new);
+  // draft records of row m (the row whose head emitted the last code)
+  stage_records(srec, n_next, p.top_k, [&](int r) { return cur + m * (kMaxDraft + 1) + 1 + r; });
+  consumer_sync();
+  if (threadIdx.x == 0) {
+    for (int j = 1; j <= n_next; ++j) {
+      const double u = uniform_u(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
+      s_next[j - 1] = seq_draw(srec + j - 1, u);
+    }
+    s_nnext = n_next;
+    DevState* st = p.st;
+    for (int t = 0; t < s_nemit; ++t) {
+      st->codes[a + 1 + t] = s_emit[t];
+      if (p.codes_out) p.codes_out[a + t] = s_emit[t];
+    }
+    for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
+    for (int t = 0; t < s_nemit; ++t) st->emitted_last[t] = s_emit[t];
+    st->n_emit_last = s_nemit;
+    st->n_acc_last = s_nacc;
+    st->a = a_new;
+    st->n_d = n_next;
+    st->pos0 = a_new + 1;
+    st->n_rows = min(n_next + 1, p.P - a_new);
+    st->first_head_row = 0;
+    const int calls = ci[CI_CALLS] + 1, heads = ci[CI_HEADS] + ci[CI_PHI] - ci[CI_PLO] + 1;
+    const int kvr = ci[CI_KVROWS] + pos0 + n_rows, rf = ci[CI_ROWSFED] + n_rows;
+    const int drafted = ci[CI_DRAFTED] + n_d, accepted = ci[CI_ACCEPTED] + s_nacc;
+    st->calls = calls;
+    st->heads_read = heads;
+    st->kv_rows = kvr;
+    st->rows_fed = rf;
+    st->drafted = drafted;
+    st->accepted = accepted;
+    st->call = call + 1;
+    st->done = a_new >= p.P ? 1 : 0;
+    st->q_row = m;  // q of the next call's drafts: this call's records of row m
+    if (p.single_call) {
+      if (p.emitted_out)
+        for (int t = 0; t < s_nemit; ++t) p.emitted_out[t] = s_emit[t];
+      if (p.n_emitted_out) *p.n_emitted_out = s_nemit;
+    }
+    if (a_new >= p.P && p.stats) {
+      p.stats->calls = calls;
+      p.stats->codes = a_new;
+      p.stats->drafted = drafted;
+      p.stats->accepted = accepted;
+      p.stats->status = 0;
+      p.stats->heads_read = heads;
+      p.stats->kv_rows = kvr;
+      p.stats->rows_fed = rf;
+    }
+  }
+  consumer_sync();
+  // optional outputs: trace and stepwise logits
+  const int fr = ci[CI_FR];
+  if (p.trace) {
+    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(p.trace) + call;
+    if (threadIdx.x == 0) {
+      tr->a = a;
+      tr->n_rows = n_rows;
+      tr->pos0 = pos0;
+      tr->n_drafts = n_d;
+      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci[CI_IDS + n] : -1;
+      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? ci[CI_IDS + 1 + i] : -1;
+      tr->n_acc = s_nacc;
+      tr->n_emit = s_nemit;
+      for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < s_nemit ? s_emit[t] : -1;
+      tr->n_next = s_nnext;
+      for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = j < s_nnext ? s_next[j] : -1;
+      tr->draft_row = m;
+    }
+    float* vlog = reinterpret_cast<float*>(p.trace + sizeof(mcd_call_trace) * kMaxCalls);
+    float* dlog = vlog + (size_t)kMaxCalls * kMaxRows * p.V;
+    for (int idx = threadIdx.x; idx < kMaxRows * p.V; idx += kConsumerThreads) {
+      const int n = idx / p.V, v = idx - n * p.V;
+      if (n >= fr && n < n_rows)
+        vlog[((size_t)call * kMaxRows + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+      if (n < s_nnext)
+        dlog[((size_t)call * kMaxRows + n) * p.V + v] =
+            __ldcg(p.logits + ((size_t)m * (kMaxDraft + 1) + n + 1) * p.V + v);
+    }
+  }
+  if (p.single_call && p.logits_out) {
+    for (int idx = threadIdx.x; idx < (n_rows - fr) * p.V; idx += kConsumerThreads) {
+      const int n = fr + idx / p.V, v = idx % p.V;
+      p.logits_out[idx] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+    }
+  }
+  consumer_sync();
+  timeline(c, call, 7, true);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+  }
+}
+
+__device__ bool read_call_state(Cons& c, int call, bool first) {
+  const FrameParams& p = c.p;
+  Smem& sm = c.sm;
+  if (!first) {
+    if (!cons_wait(c, p.ctr + (size_t)call * p.ctr_stride + ctr_ready(p.L), 1u)) return false;
+  }
+  // one parallel read of the whole state (sizeof(DevState) / 4 words) into the act region
+  constexpr int kWords = sizeof(DevState) / 4;
+  int* stw = reinterpret_cast<int*>(sm.act);
+  for (int i = threadIdx.x; i < kWords; i += kConsumerThreads) stw[i] = __ldcg(reinterpret_cast<const int*>(p.st) + i);
+  consumer_sync();
+  if (threadIdx.x == 0) {
+    const DevState* st = reinterpret_cast<const DevState*>(stw);
+    int* ci = sm.call_info;
+    ci[CI_CALL] = call;
+    ci[CI_A] = st->a;
+    ci[CI_ND] = st->n_d;
+    ci[CI_POS0] = st->pos0;
+    ci[CI_NROWS] = st->n_rows;
+    ci[CI_FR] = st->first_head_row;
+    ci[CI_DONE] = st->done;
+    ci[CI_QROW] = st->q_row;
+    ci[CI_CALLS] = st->calls;
+    ci[CI_HEADS] = st->heads_read;
+    ci[CI_KVROWS] = st->kv_rows;
+    ci[CI_ROWSFED] = st->rows_fed;
+    ci[CI_DRAFTED] = st->drafted;
+    ci[CI_ACCEPTED] = st->accepted;
+    int plo, phi;
+    head_range(p, ci[CI_A], ci[CI_POS0], ci[CI_NROWS], plo, phi);
+    ci[CI_PLO] = plo;
+    ci[CI_PHI] = phi;
+    // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft i-1
+    const int a = ci[CI_A];
+    for (int i = 0; i < kMaxDraft; ++i) ci[CI_IDS + 1 + i] = st->drafts[i];
+    if (ci[CI_POS0] == 0) {
+      ci[CI_IDS + 0] = -1;
+      ci[CI_IDS + 1] = st->codes[0];
+    } else {
+      ci[CI_IDS + 0] = st->codes[a];
+    }
+  }
+  consumer_sync();
+  timeline(c, call, 0);
+  return true;
+}
+
+template <int WT>
+__global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constant__ FrameParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  Smem sm = smem_layout(smem_raw);
+  const int tid = threadIdx.x, warp = tid >> 5;
+  if (tid == 0) {
+    for (int s = 0; s < kNumSlots; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kConsumerWarps);
+    }
+    sm.flags[0] = 0;
+    sm.flags[1] = 0;
+    sm.flags[2] = 0;
+    sm.flags[3] = -1;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  const int call0 = __ldcg(&p.st->call);
+  if (warp == kConsumerWarps) {
+    if ((tid & 31) == 0) producer_loop(p, sm, call0);
+  } else {
+    Cons c(p, sm);
+    for (int call = call0; call < kMaxCalls; ++call) {
+      if (!read_call_state(c, call, call == call0)) break;
+      if (sm.call_info[CI_DONE]) break;
+      run_call<WT>(c, call);
+      if (c.abort_) break;
+      if (sm.flags[2]) accept_step(c, call);
+      if (p.single_call) break;
+    }
+    if (tid == 0) sm.flags[0] = 1;  // stop the producer
+  }
+  __syncthreads();
+  if (tid == 0 && *(volatile int*)p.err != 0 && p.stats) p.stats->status = *(volatile int*)p.err;
+}
+
+// host-side launcher ------------------------------------------------------------------
+cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream) {
+  void* args[] = {const_cast<FrameParams*>(&p)};
+  if (p.wdtype == MCD_WEIGHT_BF16)
+    return cudaLaunchCooperativeKernel((void*)frame_kernel<MCD_WEIGHT_BF16>, dim3(p.n_cta), dim3(kThreads), args,
+                                       (size_t)kSmemBytes, stream);
+  return cudaLaunchCooperativeKernel((void*)frame_kernel<MCD_WEIGHT_F32>, dim3(p.n_cta), dim3(kThreads), args,
+                                     (size_t)kSmemBytes, stream);
+}
+
+cudaError_t prepare_frame_kernel(int* max_ctas_per_sm) {
+  cudaError_t e = cudaFuncSetAttribute((void*)frame_kernel<MCD_WEIGHT_BF16>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute((void*)frame_kernel<MCD_WEIGHT_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kSmemBytes);
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(max_ctas_per_sm, (void*)frame_kernel<MCD_WEIGHT_BF16>,
+                                                       kThreads, kSmemBytes);
+}
+
+int frame_smem_bytes() { return kSmemBytes; }
+
+}  // namespace mcd

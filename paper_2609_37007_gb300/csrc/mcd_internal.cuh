@@ -1,0 +1,289 @@
+// Internal definitions of libmcd: device-side structures, limits and PTX helpers.
+//
+// Data layout in HBM (one context = one stream's model + state):
+//   * Weight matrices of the hot path are stored as "units": a unit is Mu x Ku tiles of
+//     16 x 16 elements, contiguous, so one bulk copy moves one unit into a shared-memory
+//     ring slot.  A bf16 tile is 512 B in the A-fragment order of mma.m16n8k16 (lane l
+//     holds rows l/4 and l/4+8, columns 2(l%4)+{0,1} and +8), an fp32 tile is 1 KB with
+//     lane l holding row l%16, columns 8*(l/16)..+7.  Units of a matrix are ordered
+//     [k-chunk][m-block]; tiles inside a unit [m-tile][k-tile].
+//   * Embedding tables stay row-major [vocab, hidden] in the weight dtype (row gather).
+//   * Norm gains and offsets are fp32.  Activations, KV cache and logits are fp32.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+#include "../../include/mcd.h"
+
+namespace mcd {
+
+constexpr int kMaxRows = 8;          // rows of one call (K+1 <= 8; first call uses 2)
+constexpr int kMaxDraft = 7;         // K
+constexpr int kMaxTopK = 256;
+constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
+constexpr int kMaxCalls = 16;        // calls per frame (15 positions, first call emits 1)
+constexpr int kMaxVocab = 4096;
+constexpr int kConsumerWarps = 8;
+constexpr int kConsumerThreads = kConsumerWarps * 32;
+constexpr int kThreads = kConsumerThreads + 32;   // + one producer warp
+constexpr int kSlotBytes = 32768;
+constexpr int kNumSlots = 4;
+constexpr int kActBytes = 32768;     // fp32 activation rows / attention / top-k scratch
+constexpr int kBfragBytes = 32768;   // B operand (activations) of the unit GEMMs
+constexpr int kRedBytes = 4096;      // one cross-warp reduction buffer (x2)
+
+enum MatKind { MAT_QKV = 0, MAT_WO = 1, MAT_GU = 2, MAT_WD = 3, MAT_HEAD = 4, MAT_COUNT = 5 };
+
+struct MatGeom {
+  int M, K;            // logical rows / columns
+  int Mu, Ku;          // m-tiles and k-tiles per unit
+  int n_mb, n_kc;      // m-blocks, k-chunks
+  int n_units;         // n_mb * n_kc
+  int unit_bytes;
+  long long stride;    // bytes between consecutive matrices of this kind (layer / head)
+};
+
+// Per-call state shared by all CTAs, rewritten by the CTA that runs the acceptance step.
+struct DevState {
+  int call;            // index of the next call
+  int a;               // codes emitted so far
+  int done;
+  int n_d;             // pending drafts (positions a+1..a+n_d)
+  int pos0;            // sequence position of the next call's first row
+  int n_rows;          // rows of the next call
+  int first_head_row;  // first row that reads an LM head (1 in the first call)
+  int n_acc_last;
+  int q_row;           // row of the previous call whose draft records are pending
+  int codes[kMaxPos];  // codes[0] = c0 id (or -1), codes[s] = c_s
+  int drafts[kMaxDraft + 1];
+  int emitted_last[kMaxRows];
+  int n_emit_last;
+  int calls, drafted, accepted;
+  int heads_read;      // LM heads streamed, summed over the frame's calls
+  int kv_rows;         // sum over calls of (pos0 + n_rows): KV positions read or written
+  int rows_fed;        // sum over calls of n_rows
+  int err;
+};
+
+// One top-k / temperature distribution.
+struct TopkRec {
+  int n;
+  int pad;
+  double S;
+  int ids[kMaxTopK];
+  double e[kMaxTopK];
+};
+
+struct FrameParams {
+  // configuration
+  int L, H, NH, NKV, D, F, P, V, C0V, K, top_k, qk_norm, wdtype, draft_mode;
+  float eps, T, sigma;
+  unsigned long long seed;
+  // geometry
+  MatGeom g[MAT_COUNT];
+  int qkv_dim;                 // NH*D + 2*NKV*D
+  // weights
+  const uint8_t* w_qkv;        // + l * g[MAT_QKV].stride
+  const uint8_t* w_wo;
+  const uint8_t* w_gu;
+  const uint8_t* w_wd;
+  const uint8_t* w_head;       // + (P-1) * g[MAT_HEAD].stride
+  const float* attn_norm;      // [L][H]
+  const float* ffn_norm;       // [L][H]
+  const float* q_norm;         // [L][D]
+  const float* k_norm;         // [L][D]
+  const float* final_norm;     // [H]
+  const float* offsets;        // [K][H]
+  const uint8_t* embed;        // table i at embed + i * embed_stride (row-major, weight dtype)
+  long long embed_stride;
+  const float2* rope;          // [kMaxPos][D/2] (cos, sin)
+  // buffers
+  float* x;                    // [kMaxRows][H]
+  float* qkv;                  // [kMaxRows][qkv_dim]
+  float* mbuf;                 // [kMaxRows][F]
+  float* logits;               // [kMaxRows][kMaxDraft+1][V]
+  float* kcache;               // [L][NKV][kMaxPos][D]
+  float* vcache;
+  TopkRec* topk;               // [kMaxRows][kMaxDraft+1]
+  TopkRec* draftq;             // [kMaxDraft] pending drafts' q
+  DevState* st;
+  unsigned* ctr;               // [kMaxCalls][ctr_stride]
+  int ctr_stride;
+  int* err;                    // context-wide error word
+  uint8_t* trace;              // optional
+  // frame inputs
+  const float* cond;
+  const int* c0;
+  const float* c0emb;
+  unsigned stream_id, frame_idx;
+  int* codes_out;
+  mcd_frame_stats* stats;
+  float* logits_out;           // stepwise: verify logits of the single call
+  int* emitted_out;
+  int* n_emitted_out;
+  unsigned long long* timeline;  // optional [kMaxCalls][32] %globaltimer stamps (CTA 0)
+  int single_call;             // 1 = run exactly one call (stepwise API)
+  int n_cta;
+  unsigned long long wait_ns;  // bound of every device-side wait
+};
+
+// Counter slots of one call (per layer 4 stages, then heads, top-k, call ready).
+__host__ __device__ inline int ctr_stage(int layer, int s) { return layer * 4 + s; }
+__host__ __device__ inline int ctr_heads(int L) { return L * 4; }
+__host__ __device__ inline int ctr_topk(int L) { return L * 4 + 1; }
+__host__ __device__ inline int ctr_ready(int L) { return L * 4 + 2; }
+
+// ---------------------------------------------------------------------------------------
+// PTX helpers
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// 1-D bulk copy global -> shared, completion counted on `bar` (16-B aligned, size % 16 == 0).
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                         uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint32_t ld_acquire(const unsigned* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint4& a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b0), "r"(b1));
+}
+
+// fp32 -> (hi, lo) bf16 pair with x ~= hi + lo (round-to-nearest-even on both).
+__device__ __forceinline__ uint32_t bf16_rn_bits(float x) {
+  uint32_t u = __float_as_uint(x);
+  uint32_t bias = ((u >> 16) & 1u) + 0x7FFFu;
+  return (u + bias) >> 16;
+}
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t b) { return __uint_as_float(b << 16); }
+__device__ __forceinline__ void split_bf16(float x, uint32_t& hi, uint32_t& lo) {
+  hi = bf16_rn_bits(x);
+  lo = bf16_rn_bits(x - bf16_bits_to_f32(hi));
+}
+
+// ---------------------------------------------------------------------------------------
+// Philox4x32-10 (Salmon et al., SC'11) and the counter contract of mcd.h
+// ---------------------------------------------------------------------------------------
+__host__ __device__ inline void philox4x32_10(uint32_t c[4], uint32_t k0, uint32_t k1) {
+  const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u, W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += W0;
+      k1 += W1;
+    }
+    uint64_t p0 = (uint64_t)M0 * c[0];
+    uint64_t p1 = (uint64_t)M1 * c[2];
+    uint32_t n0 = (uint32_t)(p1 >> 32) ^ c[1] ^ k0;
+    uint32_t n2 = (uint32_t)(p0 >> 32) ^ c[3] ^ k1;
+    c[0] = n0;
+    c[1] = (uint32_t)p1;
+    c[2] = n2;
+    c[3] = (uint32_t)p0;
+  }
+}
+__host__ __device__ inline double res53(uint32_t w0, uint32_t w1) {
+  return ((double)(w0 >> 5) * 67108864.0 + (double)(w1 >> 6)) * (1.0 / 9007199254740992.0);
+}
+__host__ __device__ inline void philox_block(unsigned long long seed, uint32_t stream, uint32_t frame, int call,
+                                             int pos, uint32_t purpose, uint32_t out[4]) {
+  out[0] = stream;
+  out[1] = frame;
+  out[2] = ((uint32_t)call << 8) | (uint32_t)pos;
+  out[3] = purpose;
+  philox4x32_10(out, (uint32_t)(seed & 0xFFFFFFFFull), (uint32_t)(seed >> 32));
+}
+__host__ __device__ inline double uniform_u(unsigned long long seed, uint32_t stream, uint32_t frame, int call,
+                                            int pos, uint32_t purpose) {
+  uint32_t w[4];
+  philox_block(seed, stream, frame, call, pos, purpose, w);
+  return res53(w[0], w[1]);
+}
+
+enum { PURPOSE_TARGET = 0, PURPOSE_ACCEPT = 1, PURPOSE_DRAFT = 2, PURPOSE_NOISE = 3 };
+
+// ---------------------------------------------------------------------------------------
+// Bounded waits: every spin gives up after wait_ns and records MCD_ERR_TIMEOUT.
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ bool wait_counter(const unsigned* p, unsigned target, int* err,
+                                             unsigned long long wait_ns) {
+  if (ld_acquire(p) >= target) return true;
+  uint64_t t0 = globaltimer();
+  uint32_t it = 0;
+  while (ld_acquire(p) < target) {
+    if ((++it & 63u) == 0) {
+      if (*(volatile int*)err != 0) return false;
+      if (globaltimer() - t0 > wait_ns) {
+        atomicCAS(err, 0, (int)MCD_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+  return true;
+}
+
+__device__ __forceinline__ bool wait_mbar(uint64_t* bar, uint32_t parity, int* err, unsigned long long wait_ns,
+                                          const volatile int* stop) {
+  if (mbar_try_wait(bar, parity)) return true;
+  uint64_t t0 = globaltimer();
+  uint32_t it = 0;
+  while (!mbar_try_wait(bar, parity)) {
+    if ((++it & 15u) == 0) {
+      if (stop && *stop) return false;
+      if (*(volatile int*)err != 0) return false;
+      if (globaltimer() - t0 > wait_ns) {
+        atomicCAS(err, 0, (int)MCD_ERR_TIMEOUT);
+        return false;
+      }
+    }
+  }
+  return true;
+}
+
+}  // namespace mcd

@@ -1,0 +1,229 @@
+"""Thin ctypes binding of libmcd.so (include/mcd.h); argument marshalling only.
+
+Every function has the name of the C entry point it wraps.  Device buffers are torch CUDA
+tensors (their data_ptr() is passed through); weights are numpy arrays.  Nothing here
+computes any part of the decoding path, and there is no fallback: if the library is
+missing, loading it raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Optional
+
+import numpy as np
+
+from .synth import MCDConfig
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmcd.so")
+_lib: Optional[ctypes.CDLL] = None
+
+MCD_OK = 0
+STATUS_NAMES = {0: "MCD_OK", 1: "MCD_ERR_INVALID_ARG", 2: "MCD_ERR_STATE", 3: "MCD_ERR_CUDA",
+                4: "MCD_ERR_OOM", 5: "MCD_ERR_TIMEOUT", 6: "MCD_ERR_WEIGHTS", 7: "MCD_ERR_UNSUPPORTED"}
+
+MAX_CALLS = 16
+MAX_ROWS = 8
+
+
+class McdConfig(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32),
+                ("n_pos", ctypes.c_int32), ("vocab", ctypes.c_int32), ("c0_vocab", ctypes.c_int32),
+                ("rms_eps", ctypes.c_float), ("rope_base", ctypes.c_float),
+                ("qk_norm", ctypes.c_int32), ("weight_dtype", ctypes.c_int32),
+                ("draft_len", ctypes.c_int32), ("top_k", ctypes.c_int32),
+                ("temperature", ctypes.c_float), ("draft_mode", ctypes.c_int32),
+                ("noise_sigma", ctypes.c_float), ("seed", ctypes.c_uint64)]
+
+
+CALL_TRACE_DTYPE = np.dtype([("a", "<i4"), ("n_rows", "<i4"), ("pos0", "<i4"), ("n_drafts", "<i4"),
+                             ("input_ids", "<i4", 8), ("drafts", "<i4", 8), ("n_acc", "<i4"),
+                             ("n_emit", "<i4"), ("emitted", "<i4", 8), ("n_next", "<i4"),
+                             ("next_drafts", "<i4", 8), ("draft_row", "<i4"), ("reserved", "<i4", 24)])
+assert CALL_TRACE_DTYPE.itemsize == 256
+
+
+class MCDError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)}")
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load_library() -> ctypes.CDLL:
+    """Load the in-tree libmcd.so (built by __graft_entry__.build()); raises if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise RuntimeError(f"{_LIB_PATH} is missing: build it with __graft_entry__.build()")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, I32, I64, U32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    sig = {
+        "mcd_create": (I32, [ctypes.POINTER(McdConfig), P, ctypes.POINTER(P)]),
+        "mcd_load_weights": (I32, [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(P),
+                                   ctypes.POINTER(I64)]),
+        "mcd_decode_frame": (I32, [P, U32, U32, P, P, P, P, P]),
+        "mcd_begin_frame": (I32, [P, U32, U32, P, P, P]),
+        "mcd_verify_accept": (I32, [P, P, P, P]),
+        "mcd_draft": (I32, [P, I32, I32, P, P, P, P, P]),
+        "mcd_accept_from_logits": (I32, [P, I32, I32, I32, P, P, P, P, P]),
+        "mcd_topk_softmax": (I32, [P, I32, P, P, P]),
+        "mcd_trace_bytes": (I64, [P]),
+        "mcd_set_trace": (I32, [P, P]),
+        "mcd_set_timeline": (I32, [P, P]),
+        "mcd_sync": (I32, [P]),
+        "mcd_call_weight_bytes": (I64, [P, I32]),
+        "mcd_num_ctas": (I32, [P]),
+        "mcd_destroy": (None, [P]),
+        "mcd_status_str": (ctypes.c_char_p, [I32]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(fn: str, status: int):
+    if status != MCD_OK:
+        raise MCDError(fn, status)
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("device buffers must be CUDA tensors")
+    return t.data_ptr()
+
+
+def config_struct(cfg: MCDConfig) -> McdConfig:
+    return McdConfig(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn,
+                     cfg.n_pos, cfg.vocab, cfg.c0_vocab, cfg.rms_eps, cfg.rope_base, cfg.qk_norm,
+                     cfg.weight_dtype, cfg.draft_len, cfg.top_k, cfg.temperature, cfg.draft_mode,
+                     cfg.noise_sigma, cfg.sample_seed)
+
+
+# ---- one wrapper per entry point ------------------------------------------------------
+def mcd_create(cfg: MCDConfig, stream=None) -> ctypes.c_void_p:
+    lib = load_library()
+    c = config_struct(cfg)
+    out = ctypes.c_void_p()
+    s = ctypes.c_void_p(stream.cuda_stream if stream is not None else None)
+    _check("mcd_create", lib.mcd_create(ctypes.byref(c), s, ctypes.byref(out)))
+    return out
+
+
+def mcd_load_weights(ctx, weights: Dict[str, np.ndarray]):
+    lib = load_library()
+    names = list(weights)
+    arrs = [np.ascontiguousarray(weights[k]) for k in names]
+    n = len(names)
+    c_names = (ctypes.c_char_p * n)(*[k.encode() for k in names])
+    c_ptrs = (ctypes.c_void_p * n)(*[a.ctypes.data for a in arrs])
+    c_sz = (ctypes.c_int64 * n)(*[a.nbytes for a in arrs])
+    _check("mcd_load_weights", lib.mcd_load_weights(ctx, n, c_names, c_ptrs, c_sz))
+
+
+def mcd_decode_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):
+    _check("mcd_decode_frame", load_library().mcd_decode_frame(
+        ctx, stream_id, frame_idx, _ptr(cond), _ptr(c0), _ptr(c0_emb), _ptr(codes_out), _ptr(stats)))
+
+
+def mcd_begin_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb):
+    _check("mcd_begin_frame", load_library().mcd_begin_frame(
+        ctx, stream_id, frame_idx, _ptr(cond), _ptr(c0), _ptr(c0_emb)))
+
+
+def mcd_verify_accept(ctx, emitted, n_emitted, logits_out=None):
+    _check("mcd_verify_accept", load_library().mcd_verify_accept(
+        ctx, _ptr(emitted), _ptr(n_emitted), _ptr(logits_out)))
+
+
+def mcd_draft(ctx, pos_k: int, call_idx: int, h_k, draft_ids, q_ids=None, q_probs=None, z_out=None):
+    _check("mcd_draft", load_library().mcd_draft(
+        ctx, pos_k, call_idx, _ptr(h_k), _ptr(draft_ids), _ptr(q_ids), _ptr(q_probs), _ptr(z_out)))
+
+
+def mcd_accept_from_logits(ctx, a: int, n_drafts: int, call_idx: int, p_logits, q_logits, draft_ids,
+                           emitted, out2):
+    _check("mcd_accept_from_logits", load_library().mcd_accept_from_logits(
+        ctx, a, n_drafts, call_idx, _ptr(p_logits), _ptr(q_logits), _ptr(draft_ids), _ptr(emitted),
+        _ptr(out2)))
+
+
+def mcd_topk_softmax(ctx, n_rows: int, logits, ids, probs):
+    _check("mcd_topk_softmax", load_library().mcd_topk_softmax(ctx, n_rows, _ptr(logits), _ptr(ids),
+                                                                _ptr(probs)))
+
+
+def mcd_trace_bytes(ctx) -> int:
+    return int(load_library().mcd_trace_bytes(ctx))
+
+
+def mcd_set_trace(ctx, trace):
+    _check("mcd_set_trace", load_library().mcd_set_trace(ctx, _ptr(trace)))
+
+
+def mcd_set_timeline(ctx, timeline):
+    _check("mcd_set_timeline", load_library().mcd_set_timeline(ctx, _ptr(timeline)))
+
+
+def mcd_sync(ctx):
+    _check("mcd_sync", load_library().mcd_sync(ctx))
+
+
+def mcd_call_weight_bytes(ctx, n_heads: int) -> int:
+    return int(load_library().mcd_call_weight_bytes(ctx, n_heads))
+
+
+def mcd_num_ctas(ctx) -> int:
+    return int(load_library().mcd_num_ctas(ctx))
+
+
+def mcd_destroy(ctx):
+    load_library().mcd_destroy(ctx)
+
+
+def mcd_status_str(status: int) -> str:
+    return load_library().mcd_status_str(status).decode()
+
+
+def parse_trace(buf: np.ndarray, vocab: int):
+    """Split a trace buffer (uint8, mcd_trace_bytes long) into (records, verify, draft)."""
+    rec_bytes = CALL_TRACE_DTYPE.itemsize * MAX_CALLS
+    recs = buf[:rec_bytes].view(CALL_TRACE_DTYPE)
+    logits = buf[rec_bytes:].view(np.float32)
+    n = MAX_CALLS * MAX_ROWS * vocab
+    return recs, logits[:n].reshape(MAX_CALLS, MAX_ROWS, vocab), logits[n:2 * n].reshape(
+        MAX_CALLS, MAX_ROWS, vocab)
+
+
+class Decoder:
+    """Owns one context: weights, per-frame state and the stream it runs on."""
+
+    def __init__(self, cfg: MCDConfig, weights: Optional[Dict[str, np.ndarray]] = None, stream=None):
+        import torch
+        self.cfg = cfg
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        self.ctx = mcd_create(cfg, self.stream)
+        if weights is not None:
+            mcd_load_weights(self.ctx, weights)
+
+    def close(self):
+        if self.ctx:
+            mcd_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

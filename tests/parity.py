@@ -1,0 +1,77 @@
+"""Parity helpers: replay a GPU frame trace through the CPU oracle.
+
+A traced frame records, for every model call, the rows the GPU fed, the fp32 logits it
+computed (verify rows and the draft rows it used) and every decision it took.  The
+oracle then (1) recomputes each call's rows in fp64 from the same inputs and compares
+the logits, and (2) runs its own sampler on the GPU's fp32 logits with the same Philox
+counters; accept decisions, emitted codes and drafts must be identical.  Together this
+shows that the GPU frame is the oracle's model composed with the oracle's sampler.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from paper_2609_37007_gb300 import mcd
+from oracle.frame import Sampling, sample_drafts, verify_round
+
+
+def check_trace_against_oracle(cfg, model, fr, stream_id, frame_idx, trace_u8, codes, n_calls,
+                               logit_tol, draft_mode=None):
+    recs, vlog, dlog = mcd.parse_trace(np.asarray(trace_u8, dtype=np.uint8), cfg.vocab)
+    S = Sampling(cfg, stream_id, frame_idx, draft_mode)
+    P, K = cfg.n_pos, cfg.draft_len
+    kv = model.new_kv()
+    max_err = 0.0
+    prev_q = []
+    prev_next = []
+    emitted_all = []
+    for c in range(n_calls):
+        r = recs[c]
+        a, n_rows, pos0, n_d = int(r["a"]), int(r["n_rows"]), int(r["pos0"]), int(r["n_drafts"])
+        assert a == len(emitted_all), (c, a)
+        if c == 0:
+            assert pos0 == 0 and n_rows == 2 and n_d == 0
+            rows = [(0, np.asarray(fr.cond, dtype=np.float64)), (1, model.c0_row(fr.c0, fr.c0_emb))]
+            first = 1
+        else:
+            ids = [int(v) for v in r["input_ids"][:n_rows]]
+            assert pos0 == a + 1 and n_rows == min(n_d + 1, P - a), (c, pos0, n_rows, n_d)
+            assert ids[0] == emitted_all[-1]
+            assert ids[1:] == prev_next[: n_rows - 1]
+            assert [int(v) for v in r["drafts"][:n_d]] == prev_next[:n_d]
+            rows = [(pos0 + n, model.code_row(pos0 + n - 1, ids[n])) for n in range(n_rows)]
+            first = 0
+        h = {pos: model.row(kv, x, pos) for pos, x in rows}
+        p_rows = []
+        for n in range(first, n_rows):
+            pos = pos0 + n
+            ref = model.verify_logits(pos, h[pos])
+            got = vlog[c, n].astype(np.float64)
+            err = float(np.max(np.abs(got - ref)))
+            max_err = max(max_err, err)
+            assert err <= logit_tol, f"call {c} row {n}: verify logits differ by {err}"
+            p_rows.append(vlog[c, n].copy())
+        drafts = list(zip([int(v) for v in r["drafts"][:n_d]], prev_q))
+        n_acc, emitted = verify_round(S, c, a, P, p_rows, drafts)
+        assert n_acc == int(r["n_acc"]), (c, n_acc, int(r["n_acc"]))
+        assert emitted == [int(v) for v in r["emitted"][: int(r["n_emit"])]], (c, emitted, r["emitted"])
+        a_new = a + len(emitted)
+        assert int(r["draft_row"]) == a_new - pos0
+        n_next = int(r["n_next"])
+        assert n_next == min(K, P - a_new)
+        z_rows = []
+        for j in range(1, n_next + 1):
+            ref = model.draft_logits(a_new, j, h[a_new])
+            got = dlog[c, j - 1].astype(np.float64)
+            err = float(np.max(np.abs(got - ref)))
+            max_err = max(max_err, err)
+            assert err <= logit_tol, f"call {c} draft {j}: logits differ by {err}"
+            z_rows.append(dlog[c, j - 1].copy())
+        nd = sample_drafts(S, c, a_new, z_rows)
+        prev_next = [d for d, _ in nd]
+        assert prev_next == [int(v) for v in r["next_drafts"][:n_next]], (c, prev_next, r["next_drafts"])
+        prev_q = [q for _, q in nd]
+        emitted_all += emitted
+    assert len(emitted_all) == P
+    assert emitted_all == [int(v) for v in codes], (emitted_all, list(codes))
+    return max_err

@@ -1,0 +1,320 @@
+"""GPU parity of libmcd against the CPU oracle (all calls go through the C ABI).
+
+  * sampler: top-k sets/order bit-exact, probabilities to the last bits, accept decisions,
+    emitted codes and drafts bit-exact when fed the same fp32 logits and counters;
+  * frames: every call's logits within tolerance of the oracle at the same inputs
+    (1e-5 fp32 model, 2e-2 bf16 model) and every decision identical (tests/parity.py);
+  * distribution: chi-square of GPU-emitted codes against the exact law.
+"""
+import math
+from collections import Counter
+
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2609_37007_gb300 import build as _build  # noqa: E402
+from paper_2609_37007_gb300 import mcd  # noqa: E402
+from paper_2609_37007_gb300.synth import (DRAFT_GREEDY, MCD, TINY, make_frame,  # noqa: E402
+                                          make_weights, random_logits, weights_as_f32)
+from oracle.enumeration import PrefixModel, ar_distribution, spec_distribution  # noqa: E402
+from oracle.frame import Sampling, decode_frame, verify_round  # noqa: E402
+from oracle.model import Model  # noqa: E402
+from oracle.sampler import topk_dist  # noqa: E402
+from parity import check_trace_against_oracle  # noqa: E402
+
+DEV = torch.device("cuda:0")
+_build.build()
+
+
+def t(x, dtype=None):
+    return torch.from_numpy(np.ascontiguousarray(x)).to(DEV) if dtype is None else \
+        torch.from_numpy(np.ascontiguousarray(x)).to(device=DEV, dtype=dtype)
+
+
+class Env:
+    def __init__(self, cfg, weights=None):
+        self.cfg = cfg
+        self.w = make_weights(cfg) if weights is None else weights
+        self.dec = mcd.Decoder(cfg, self.w)
+        self._model = None
+
+    @property
+    def model(self):
+        if self._model is None:
+            self._model = Model(self.cfg, weights_as_f32(self.cfg, self.w))
+        return self._model
+
+    def frame_inputs(self, fr):
+        cond = t(fr.cond)
+        c0 = t(np.array([fr.c0], dtype=np.int32)) if self.cfg.c0_vocab > 0 else None
+        emb = t(fr.c0_emb) if self.cfg.c0_vocab == 0 else None
+        return cond, c0, emb
+
+    def decode(self, fr, frame_idx, stream_id=0, trace=False):
+        cond, c0, emb = self.frame_inputs(fr)
+        codes = torch.full((self.cfg.n_pos,), -1, dtype=torch.int32, device=DEV)
+        stats = torch.zeros(8, dtype=torch.int32, device=DEV)
+        tr = None
+        if trace:
+            tr = torch.zeros(mcd.mcd_trace_bytes(self.dec.ctx), dtype=torch.uint8, device=DEV)
+        mcd.mcd_set_trace(self.dec.ctx, tr)
+        mcd.mcd_decode_frame(self.dec.ctx, stream_id, frame_idx, cond, c0, emb, codes, stats)
+        mcd.mcd_sync(self.dec.ctx)
+        mcd.mcd_set_trace(self.dec.ctx, None)
+        return codes.cpu().numpy(), stats.cpu().numpy(), (tr.cpu().numpy() if trace else None)
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    return Env(TINY)
+
+
+@pytest.fixture(scope="module")
+def big():
+    return Env(MCD)
+
+
+# ---------------------------------------------------------------- sampler ----------
+@pytest.mark.parametrize("V,k,T,ties", [(2048, 50, 0.9, 0.0), (2048, 50, 0.9, 0.6), (64, 8, 1.0, 0.5),
+                                        (64, 64, 1.0, 0.3), (2048, 256, 0.7, 0.2), (3072, 1, 1.3, 0.9)])
+def test_topk_softmax_matches_oracle(V, k, T, ties):
+    cfg = TINY.replace(vocab=V, top_k=k, temperature=T)
+    dec = mcd.Decoder(cfg)                     # sampler entry points need no weights
+    rng = np.random.default_rng(V + k)
+    rows = 24
+    logits = random_logits(rng, rows, V, scale=0.7, tie_frac=ties)
+    logits[0] = 0.0                            # all equal: lowest ids win
+    logits[1, ::2] = -0.0                      # signed zeros tie
+    ids = torch.zeros((rows, k), dtype=torch.int32, device=DEV)
+    probs = torch.zeros((rows, k), dtype=torch.float64, device=DEV)
+    mcd.mcd_topk_softmax(dec.ctx, rows, t(logits), ids, probs)
+    mcd.mcd_sync(dec.ctx)
+    ids, probs = ids.cpu().numpy(), probs.cpu().numpy()
+    for r in range(rows):
+        d = topk_dist(logits[r], k, T)
+        assert ids[r].tolist() == d.ids, r
+        ref = np.array([d.prob(x) for x in d.ids])
+        # each side calls its own double exp (CUDA vs libm): a few ulps apart at most
+        assert np.allclose(probs[r], ref, rtol=8 * np.finfo(np.float64).eps, atol=0), \
+            (r, np.max(np.abs(probs[r] - ref) / ref))
+    assert ids[0].tolist() == list(range(k))
+    dec.close()
+
+
+def _begin(dec, cfg, stream_id=0, frame_idx=0):
+    fr = make_frame(cfg, 0)
+    cond = t(fr.cond)
+    c0 = t(np.array([max(fr.c0, 0)], dtype=np.int32))
+    emb = t(fr.c0_emb) if fr.c0_emb is not None else None
+    mcd.mcd_begin_frame(dec.ctx, stream_id, frame_idx, cond, c0, emb)
+
+
+@pytest.mark.parametrize("cfg,mode", [(MCD, 0), (TINY, 0), (TINY.replace(draft_len=7, n_pos=15), 0),
+                                      (MCD, DRAFT_GREEDY)])
+def test_accept_from_logits_is_bit_exact(cfg, mode):
+    cfg = cfg.replace(draft_mode=mode)
+    dec = mcd.Decoder(cfg)
+    rng = np.random.default_rng(11 + mode)
+    V, K, P = cfg.vocab, cfg.draft_len, cfg.n_pos
+    emitted = torch.zeros(8, dtype=torch.int32, device=DEV)
+    out2 = torch.zeros(2, dtype=torch.int32, device=DEV)
+    n_cases, n_acc_total = 120, 0
+    for case in range(n_cases):
+        stream_id, frame_idx, call = int(rng.integers(0, 4)), int(rng.integers(0, 1000)), int(rng.integers(1, 15))
+        _begin(dec, cfg, stream_id, frame_idx)
+        a = int(rng.integers(1, P))
+        n_d = int(rng.integers(0, min(K, P - a) + 1))
+        n_p = n_d + 1 if a + 1 + n_d <= P else n_d
+        p = random_logits(rng, max(n_p, 1), V, scale=1.0, tie_frac=0.1)
+        noise = [0.0, 0.05, 0.5, 3.0][case % 4]     # from q == p (all kept) to unrelated q
+        q = (p[:max(n_d, 1)] + noise * rng.standard_normal((max(n_d, 1), V))).astype(np.float32)
+        S = Sampling(cfg, stream_id, frame_idx, mode)
+        drafts = []
+        for i in range(n_d):
+            qd = S.dist(q[i]) if mode != DRAFT_GREEDY else None
+            from oracle.sampler import greedy_dist, draw
+            qd = greedy_dist(q[i]) if mode == DRAFT_GREEDY else qd
+            drafts.append((draw(qd, float(rng.random())), qd))
+        ref_acc, ref_emit = verify_round(S, call, a, P, list(p[:n_p]), drafts)
+        mcd.mcd_accept_from_logits(dec.ctx, a, n_d, call, t(p), t(q),
+                                   t(np.array([d for d, _ in drafts] or [0], dtype=np.int32)), emitted, out2)
+        mcd.mcd_sync(dec.ctx)
+        o = out2.cpu().numpy()
+        assert int(o[0]) == ref_acc and int(o[1]) == len(ref_emit), (case, o, ref_acc, ref_emit)
+        assert emitted.cpu().numpy()[: o[1]].tolist() == ref_emit, case
+        n_acc_total += ref_acc
+    assert n_acc_total > 0
+    dec.close()
+
+
+# ---------------------------------------------------------------- frames -----------
+def test_tiny_frames_trace_parity(tiny):
+    cfg = tiny.cfg
+    worst = 0.0
+    for f in range(12):
+        fr = make_frame(cfg, f)
+        codes, st, tr = tiny.decode(fr, f, stream_id=f % 3, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        worst = max(worst, check_trace_against_oracle(cfg, tiny.model, fr, f % 3, f, tr, codes, int(st[0]),
+                                                      logit_tol=1e-5))
+    print("tiny max |dlogit|", worst)
+
+
+def test_tiny_codes_equal_oracle_end_to_end(tiny):
+    cfg = tiny.cfg
+    same = 0
+    n = 40
+    for f in range(n):
+        fr = make_frame(cfg, 100 + f)
+        codes, st, _ = tiny.decode(fr, 100 + f)
+        ref = decode_frame(tiny.model, fr, frame_idx=100 + f)
+        same += list(codes) == ref.codes
+        if list(codes) == ref.codes:
+            assert int(st[0]) == ref.calls
+    assert same >= n - 1, f"{n - same} of {n} frames differ from the oracle"
+
+
+def test_mcd_frame_trace_parity_full_size(big):
+    cfg = big.cfg
+    for f in (0, 1):
+        fr = make_frame(cfg, f)
+        codes, st, tr = big.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        err = check_trace_against_oracle(cfg, big.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=2e-2)
+        print("bf16 max |dlogit|", err)
+
+
+def test_mcd_frames_are_complete_and_bounded(big):
+    cfg = big.cfg
+    frames = 50
+    calls = 0
+    for f in range(frames):
+        codes, st, _ = big.decode(make_frame(cfg, f), f)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        assert (codes >= 0).all() and (codes < cfg.vocab).all()
+        assert 1 + math.ceil((cfg.n_pos - 1) / (cfg.draft_len + 1)) <= st[0] <= cfg.n_pos
+        assert st[3] <= st[2]
+        calls += int(st[0])
+    assert calls <= frames * cfg.n_pos
+
+
+@pytest.mark.parametrize("variant", ["ar", "k7", "greedy", "topk_all"])
+def test_tiny_variants_trace_parity(variant):
+    cfg = {"ar": TINY.replace(draft_len=0), "k7": TINY.replace(draft_len=7, n_pos=12),
+           "greedy": TINY.replace(draft_mode=DRAFT_GREEDY), "topk_all": TINY.replace(top_k=64)}[variant]
+    env = Env(cfg)
+    for f in range(4):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        check_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=1e-5,
+                                   draft_mode=cfg.draft_mode)
+        if variant == "ar":
+            assert int(st[0]) == cfg.n_pos
+    env.dec.close()
+
+
+def test_stepwise_api_matches_decode_frame(tiny):
+    cfg = tiny.cfg
+    dec = tiny.dec
+    fr = make_frame(cfg, 7)
+    ref, st, _ = tiny.decode(fr, 7)
+    cond, c0, emb = tiny.frame_inputs(fr)
+    mcd.mcd_begin_frame(dec.ctx, 0, 7, cond, c0, emb)
+    emitted = torch.zeros(8, dtype=torch.int32, device=DEV)
+    n_em = torch.zeros(1, dtype=torch.int32, device=DEV)
+    logits = torch.zeros((8, cfg.vocab), dtype=torch.float32, device=DEV)
+    got = []
+    for call in range(cfg.n_pos + 1):
+        mcd.mcd_verify_accept(dec.ctx, emitted, n_em, logits)
+        mcd.mcd_sync(dec.ctx)
+        k = int(n_em.item())
+        if k == 0:
+            break
+        got += emitted.cpu().numpy()[:k].tolist()
+    assert got == list(ref)
+    assert call == int(st[0])
+
+
+def test_draft_api_matches_oracle(tiny):
+    cfg = tiny.cfg
+    dec = tiny.dec
+    m = tiny.model
+    _begin(dec, cfg, 2, 5)
+    rng = np.random.default_rng(3)
+    h = rng.standard_normal(cfg.hidden).astype(np.float32)
+    K = cfg.draft_len
+    ids = torch.zeros(K, dtype=torch.int32, device=DEV)
+    q_ids = torch.zeros((K, cfg.top_k), dtype=torch.int32, device=DEV)
+    q_probs = torch.zeros((K, cfg.top_k), dtype=torch.float64, device=DEV)
+    z = torch.zeros((K, cfg.vocab), dtype=torch.float32, device=DEV)
+    S = Sampling(cfg, 2, 5)
+    for k_pos in (1, 2):
+        mcd.mcd_draft(dec.ctx, k_pos, 4, t(h), ids, q_ids, q_probs, z)
+        mcd.mcd_sync(dec.ctx)
+        n_j = min(K, cfg.n_pos - k_pos)
+        zz = z.cpu().numpy()
+        for j in range(1, n_j + 1):
+            ref = m.draft_logits(k_pos, j, h.astype(np.float64))
+            assert np.max(np.abs(zz[j - 1] - ref)) < 1e-5
+            q = S.dist(zz[j - 1])
+            from oracle.sampler import draw
+            assert int(ids[j - 1]) == draw(q, S.u(4, k_pos + j, 2))
+            assert q_ids.cpu().numpy()[j - 1].tolist() == q.ids
+
+
+def test_bad_c0_fails_the_frame_without_faulting(big):
+    cfg = big.cfg
+    fr = make_frame(cfg, 0)
+    cond = t(fr.cond)
+    c0 = t(np.array([cfg.c0_vocab + 5], dtype=np.int32))
+    codes = torch.zeros(cfg.n_pos, dtype=torch.int32, device=DEV)
+    mcd.mcd_decode_frame(big.dec.ctx, 0, 0, cond, c0, None, codes, None)
+    with pytest.raises(mcd.MCDError) as e:
+        mcd.mcd_sync(big.dec.ctx)
+    assert e.value.status == 1
+    # the context stays usable
+    codes2, st, _ = big.decode(fr, 0)
+    assert st[4] == 0 and st[1] == cfg.n_pos
+
+
+# ---------------------------------------------------------------- distribution -----
+def test_chi_square_of_gpu_codes_against_exact_law(tiny):
+    cfg = tiny.cfg
+    pm = PrefixModel(tiny.model, make_frame(cfg, 0))
+    ar = ar_distribution(pm, cfg.n_pos)
+    _, exp_calls = spec_distribution(pm, cfg.n_pos, cfg.draft_len)
+    fr = make_frame(cfg, 0)
+    cond, c0, emb = tiny.frame_inputs(fr)
+    n = 20000
+    codes = torch.zeros((n, cfg.n_pos), dtype=torch.int32, device=DEV)
+    stats = torch.zeros((n, 8), dtype=torch.int32, device=DEV)
+    for i in range(n):
+        mcd.mcd_decode_frame(tiny.dec.ctx, 1, 10_000 + i, cond, c0, emb, codes[i], stats[i])
+    mcd.mcd_sync(tiny.dec.ctx)
+    codes, stats = codes.cpu().numpy(), stats.cpu().numpy()
+    assert (stats[:, 4] == 0).all()
+    from scipy import stats as ss
+    for cells in ((0,), (1,), (2,), (3,), (0, 1)):
+        law = Counter()
+        for seq, pr in ar.items():
+            law[tuple(seq[c] for c in cells)] += pr
+        obs = Counter(tuple(row[list(cells)]) for row in codes)
+        keys = sorted(law)
+        e = np.array([law[k] * n for k in keys])
+        o = np.array([obs.get(k, 0) for k in keys])
+        assert sum(obs.values()) == o.sum() == n, cells           # nothing outside the support
+        big_ = e >= 5
+        o2 = np.append(o[big_], o[~big_].sum())
+        e2 = np.append(e[big_], e[~big_].sum())
+        if e2[-1] == 0:
+            o2, e2 = o2[:-1], e2[:-1]
+        p = ss.chisquare(o2, e2 * o2.sum() / e2.sum()).pvalue
+        assert p > 1e-4, (cells, p)
+    mean_calls = stats[:, 0].mean()
+    assert abs(mean_calls - exp_calls) < 4 * stats[:, 0].std() / math.sqrt(n) + 1e-3, (mean_calls, exp_calls)
