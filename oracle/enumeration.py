@@ -3,8 +3,9 @@ TEST INFRASTRUCTURE ONLY.
 
 The paper's correctness claim (Abstract; Sec. 3.2) is that the speculative decoder is
 distributionally lossless under the deployed top-k sampling: the law of the emitted
-codes c1..c_P equals the autoregressive law prod_s p_s(c_s | c_<s).  On a small model
-both laws can be written out exactly in fp64:
+codes c1..c_P equals the autoregressive law prod_s p_s(c_s | c_<s).  The sampler's
+distributions are integer weights (oracle.sampler R-S2), so on a small model both laws
+can be written out exactly as rationals (fractions.Fraction):
 
   * AR: product of the top-k/temperature probabilities along every sequence.
   * speculative: the procedure of oracle.frame, with every random choice replaced by
@@ -19,6 +20,7 @@ from __future__ import annotations
 
 import itertools
 from collections import defaultdict
+from fractions import Fraction
 from typing import Dict, Tuple
 
 import numpy as np
@@ -78,8 +80,8 @@ class PrefixModel:
         return self._q[key]
 
 
-def ar_distribution(pm: PrefixModel, n_pos: int) -> Dict[Tuple[int, ...], float]:
-    out: Dict[Tuple[int, ...], float] = {}
+def ar_distribution(pm: PrefixModel, n_pos: int) -> Dict[Tuple[int, ...], Fraction]:
+    out: Dict[Tuple[int, ...], Fraction] = {}
 
     def rec(prefix, pr):
         if len(prefix) == n_pos:
@@ -87,15 +89,15 @@ def ar_distribution(pm: PrefixModel, n_pos: int) -> Dict[Tuple[int, ...], float]
             return
         p = pm.target(prefix)
         for x in p.ids:
-            rec(prefix + (x,), pr * p.prob(x))
+            rec(prefix + (x,), pr * p.frac(x))
 
-    rec((), 1.0)
+    rec((), Fraction(1))
     return out
 
 
 def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
     """(law of c1..c_P, expected model calls per frame) of the speculative procedure."""
-    memo: Dict[Tuple[int, ...], Tuple[Dict[Tuple[int, ...], float], float]] = {}
+    memo: Dict[Tuple[int, ...], Tuple[Dict[Tuple[int, ...], Fraction], Fraction]] = {}
 
     def add(res, calls, head, sub, w):
         sub_law, sub_calls = sub
@@ -108,29 +110,29 @@ def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
         if prefix in memo:
             return memo[prefix]
         a = len(prefix)
-        res: Dict[Tuple[int, ...], float] = defaultdict(float)
-        calls = 1.0
+        res: Dict[Tuple[int, ...], Fraction] = defaultdict(Fraction)
+        calls = Fraction(1)
         if a == n_pos:
-            memo[prefix] = ({(): 1.0}, 0.0)
+            memo[prefix] = ({(): Fraction(1)}, Fraction(0))
             return memo[prefix]
         n_d = min(draft_len, n_pos - a)
         qs = [pm.draft(prefix, j) for j in range(1, n_d + 1)]
         for dt in itertools.product(*[q.ids for q in qs]):
-            pr = 1.0
+            pr = Fraction(1)
             for q, d in zip(qs, dt):
-                pr *= q.prob(d)
+                pr *= q.frac(d)
             cur = prefix
             for i in range(n_d):
                 p, q, d = pm.target(cur), qs[i], dt[i]
-                alpha = min(1.0, p.prob(d) / q.prob(d))
-                if alpha < 1.0:
+                alpha = min(Fraction(1), p.frac(d) / q.frac(d))
+                if alpha < 1:
                     xs, r, R = residual_weights(p, q)
                     for x, rx in zip(xs, r):
-                        if rx > 0.0:
+                        if rx > 0:
                             calls = add(res, calls, cur[a:] + (x,), from_state(cur + (x,)),
-                                        pr * (1.0 - alpha) * rx / R)
+                                        pr * (1 - alpha) * Fraction(rx, R))
                 pr *= alpha
-                if pr == 0.0:
+                if pr == 0:
                     break
                 cur = cur + (d,)
             else:
@@ -138,7 +140,7 @@ def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
                     p = pm.target(cur)
                     for x in p.ids:
                         calls = add(res, calls, cur[a:] + (x,), from_state(cur + (x,)),
-                                    pr * p.prob(x))
+                                    pr * p.frac(x))
                 else:
                     res[cur[a:]] += pr
         memo[prefix] = (dict(res), calls)
@@ -146,13 +148,13 @@ def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
 
     # first call: rows (cond, c0), emits c1 from LM head 1 -- plain AR
     p1 = pm.target(())
-    law: Dict[Tuple[int, ...], float] = defaultdict(float)
-    calls = 1.0
+    law: Dict[Tuple[int, ...], Fraction] = defaultdict(Fraction)
+    calls = Fraction(1)
     for x in p1.ids:
-        calls = add(law, calls, (x,), from_state((x,)), p1.prob(x))
+        calls = add(law, calls, (x,), from_state((x,)), p1.frac(x))
     return dict(law), calls
 
 
-def alpha(p: Dist, q: Dist) -> float:
+def alpha(p: Dist, q: Dist) -> Fraction:
     """Acceptance probability of one draft: sum_x min(p(x), q(x))."""
-    return sum(min(p.prob(x), q.prob(x)) for x in set(p.ids) | set(q.ids))
+    return sum((min(p.frac(x), q.frac(x)) for x in set(p.ids) | set(q.ids)), Fraction(0))

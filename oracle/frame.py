@@ -77,8 +77,9 @@ class Sampling:
         self.mode = cfg.draft_mode if draft_mode is None else draft_mode
         self.sigma = cfg.noise_sigma if noise_sigma is None else noise_sigma
 
-    def u(self, rnd: int, pos: int, purpose: int) -> float:
-        return philox.uniform(self.seed, self.stream, self.frame, rnd, pos, purpose)
+    def u(self, rnd: int, pos: int, purpose: int) -> int:
+        """The 53-bit integer uniform of a decision (oracle.sampler R-S3..R-S5)."""
+        return philox.uniform_int(self.seed, self.stream, self.frame, rnd, pos, purpose)
 
     def dist(self, logits) -> Dist:
         return topk_dist(logits, self.k, self.T)

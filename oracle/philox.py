@@ -14,7 +14,8 @@ counter contract so that two independent implementations can be compared draw by
   purpose 3 + v//2: Gaussian pair for vocabulary entries (v, v+1) of a noisy draft row
 
 A uniform in [0, 1) uses words 0 and 1 of the block: ((w0 >> 5) * 2^26 + (w1 >> 6)) * 2^-53,
-the 53-bit construction of Matsumoto and Nishimura's genrand_res53.
+the 53-bit construction of Matsumoto and Nishimura's genrand_res53; the sampler's decisions
+use its integer numerator U directly.
 """
 from __future__ import annotations
 
@@ -57,9 +58,20 @@ def res53(w0: int, w1: int) -> float:
     return ((w0 >> 5) * 67108864.0 + (w1 >> 6)) * (1.0 / 9007199254740992.0)
 
 
+def int53(w0: int, w1: int) -> int:
+    """The 53-bit integer U behind res53: res53(w0, w1) == U / 2^53 exactly."""
+    return ((w0 >> 5) << 26) | (w1 >> 6)
+
+
 def uniform(seed: int, stream: int, frame: int, rnd: int, position: int, purpose: int) -> float:
     w = philox4x32_10(counter(stream, frame, rnd, position, purpose), key_of(seed))
     return res53(w[0], w[1])
+
+
+def uniform_int(seed: int, stream: int, frame: int, rnd: int, position: int, purpose: int) -> int:
+    """The decision uniform as its 53-bit integer (u = U / 2^53)."""
+    w = philox4x32_10(counter(stream, frame, rnd, position, purpose), key_of(seed))
+    return int53(w[0], w[1])
 
 
 def normal_pair(seed: int, stream: int, frame: int, rnd: int, position: int, pair: int):

@@ -26,6 +26,13 @@ def test_res53_endpoints_and_exactness():
     assert philox.res53(0, 1 << 6) == 2.0 ** -53
 
 
+def test_integer_uniform_is_the_res53_numerator():
+    for w0, w1 in ((0, 0), (0xFFFFFFFF, 0xFFFFFFFF), (0x12345678, 0x9ABCDEF0), (1 << 31, 1 << 6)):
+        assert philox.int53(w0, w1) / 2.0 ** 53 == philox.res53(w0, w1)
+        assert 0 <= philox.int53(w0, w1) < 2 ** 53
+    assert philox.uniform_int(1, 2, 3, 4, 5, 0) / 2.0 ** 53 == philox.uniform(1, 2, 3, 4, 5, 0)
+
+
 def test_counter_layout_separates_decisions():
     seen = set()
     for rnd in range(3):

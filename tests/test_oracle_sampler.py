@@ -1,7 +1,10 @@
-"""Pins of oracle.sampler: top-k order, softmax closed forms, and the acceptance rule's
-losslessness (Sec. 2.2 / Sec. 3.2: keep d with prob min(1, p/q), else resample from
-norm(max(0, p - q)); the emitted code is then distributed exactly as p)."""
+"""Pins of oracle.sampler: the fp32 exponential, top-k order, integer-weight softmax, and
+the acceptance rule's losslessness (Sec. 2.2 / Sec. 3.2: keep d with prob min(1, p/q),
+else resample from norm(max(0, p - q)); the emitted code is then distributed exactly as p).
+"""
 import math
+import struct
+from fractions import Fraction
 
 import numpy as np
 import pytest
@@ -9,10 +12,38 @@ from scipy import stats
 
 from oracle import philox
 from oracle.enumeration import alpha
-from oracle.sampler import (Dist, accept, draw, greedy_dist, residual_draw,
+from oracle.sampler import (TAYLOR, Dist, accept, draw, exp32, greedy_dist, residual_draw,
                             residual_weights, topk_dist, topk_order)
 
 
+def bits(f):
+    return struct.unpack("<I", struct.pack("<f", float(np.float32(f))))[0]
+
+
+# ---- exp32 (Cody-Waite range reduction + Taylor polynomial) ---------------------------
+def test_exp32_constants_are_the_rounded_taylor_coefficients():
+    # the CUDA implementation hard-codes these fp32 bit patterns
+    assert [bits(c) for c in TAYLOR] == [0x39500D01, 0x3AB60B61, 0x3C088889, 0x3D2AAAAB,
+                                          0x3E2AAAAB, 0x3F000000, 0x3F800000, 0x3F800000]
+
+
+def test_exp32_matches_libm_within_a_few_ulp():
+    xs = np.concatenate([-np.logspace(-8, math.log10(87), 4000), np.linspace(-87, 0, 4001)]).astype(np.float32)
+    for x in xs:
+        got = float(exp32(x))
+        ref = math.exp(float(x))
+        assert abs(got - ref) <= 4 * 2.0 ** -24 * ref, (x, got, ref)
+    assert exp32(np.float32(0)) == np.float32(1)
+    assert exp32(np.float32(-88)) == 0 and exp32(np.float32(-1000)) == 0
+
+
+def test_exp32_special_values():
+    # exact powers of two: d = -n ln2 reduces to r ~ 0
+    assert abs(float(exp32(np.float32(-math.log(2)))) - 0.5) <= 2 ** -24
+    assert abs(float(exp32(np.float32(-10 * math.log(2)))) - 2.0 ** -10) <= 2 ** -33
+
+
+# ---- top-k order -----------------------------------------------------------------------
 def test_topk_ties_go_to_lower_id():
     l = np.array([1.0, 3.0, 3.0, 2.0, 3.0], dtype=np.float32)
     assert topk_order(l, 2) == [1, 2]
@@ -35,69 +66,81 @@ def test_topk_matches_lexsort_brute_force():
         assert topk_order(l, k) == [int(i) for i in ref]
 
 
-def test_softmax_two_entry_closed_form():
+# ---- integer-weight softmax ------------------------------------------------------------
+def test_weights_two_entry_closed_form():
     l = np.array([0.25, 1.5], dtype=np.float32)
     T = 0.9
     d = topk_dist(l, 2, T)
     Tf = float(np.float32(T))
-    p1 = 1.0 / (1.0 + math.exp((0.25 - 1.5) / Tf))
     assert d.ids == [1, 0]
-    assert math.isclose(d.prob(1), p1, rel_tol=1e-15)
-    assert math.isclose(d.prob(0), 1.0 - p1, rel_tol=1e-14)
-    assert d.prob(7) == 0.0
+    assert d.W[0] == 2 ** 24                                 # the maximum has e = 1 exactly
+    p1 = 1.0 / (1.0 + math.exp((0.25 - 1.5) / Tf))
+    assert abs(d.prob(1) - p1) < 1e-6
+    assert d.frac(0) + d.frac(1) == 1 and d.frac(7) == 0
 
 
-def test_softmax_temperature_and_truncation():
+def test_weights_follow_temperature_softmax():
     rng = np.random.default_rng(1)
     l = rng.standard_normal(64).astype(np.float32)
     d = topk_dist(l, 8, 0.5)
     ids = np.argsort(-l.astype(np.float64), kind="stable")[:8]
     w = np.exp((l[ids].astype(np.float64) - l[ids[0]]) / float(np.float32(0.5)))
-    ref = w / w.sum()
     assert d.ids == list(ids)
-    assert np.allclose([d.prob(i) for i in ids], ref, rtol=1e-13, atol=0)
-    assert math.isclose(sum(d.prob(i) for i in range(64)), 1.0, rel_tol=1e-14)
+    assert np.allclose([d.prob(i) for i in ids], w / w.sum(), rtol=2e-6, atol=0)
+    assert sum(d.frac(i) for i in range(64)) == 1
 
 
-def test_draw_endpoints_and_frequencies():
-    d = Dist(ids=[4, 2, 9], e=[0.5, 0.3, 0.2], S=1.0)
-    assert draw(d, 0.0) == 4
-    assert draw(d, 0.4999999) == 4 and draw(d, 0.5) == 2
-    assert draw(d, 1.0 - 2.0 ** -53) == 9
+def test_weights_are_floor_of_scaled_exp32():
+    l = np.array([3.0, 1.0, -2.0, 0.5], dtype=np.float32)
+    d = topk_dist(l, 4, 1.3)
+    T = np.float32(1.3)
+    z = [l[i] / T for i in d.ids]
+    assert d.W == [math.floor(float(exp32(zi - z[0])) * 2 ** 24) for zi in z]
+
+
+# ---- draws and acceptance ---------------------------------------------------------------
+def test_draw_boundaries_are_exact():
+    d = Dist(ids=[4, 2, 9], W=[5, 3, 2])                     # p = 1/2, 3/10, 1/5
+    top = 2 ** 53
+    assert draw(d, 0) == 4
+    assert draw(d, top // 2 - 1) == 4 and draw(d, top // 2) == 2
+    assert draw(d, (top * 8) // 10 - 1) == 2 and draw(d, -(-top * 8 // 10)) == 9
+    assert draw(d, top - 1) == 9
     n = 20000
     c = {4: 0, 2: 0, 9: 0}
     for i in range(n):
-        c[draw(d, philox.uniform(2, 0, i, 0, 1, 0))] += 1
-    chi = stats.chisquare([c[4], c[2], c[9]], [n * 0.5, n * 0.3, n * 0.2])
-    assert chi.pvalue > 1e-4
+        c[draw(d, philox.uniform_int(2, 0, i, 0, 1, 0))] += 1
+    assert stats.chisquare([c[4], c[2], c[9]], [n * 0.5, n * 0.3, n * 0.2]).pvalue > 1e-4
 
 
 def test_greedy_is_one_hot_on_argmax():
     l = np.array([0.0, 2.0, 2.0, 1.0], dtype=np.float32)
     g = greedy_dist(l)
-    assert g.ids == [1] and g.prob(1) == 1.0 and g.prob(2) == 0.0
+    assert g.ids == [1] and g.frac(1) == 1 and g.frac(2) == 0
 
 
 def test_accept_rule_special_cases():
-    p = Dist(ids=[0, 1], e=[0.6, 0.4], S=1.0)
-    q = Dist(ids=[0, 2], e=[0.5, 0.5], S=1.0)
-    # p(0) >= q(0): always kept, even at the largest uniform
-    assert accept(p, q, 0, 1.0 - 2.0 ** -53)
-    # p(2) = 0: never kept, even at u = 0 (strict comparison)
-    assert not accept(p, q, 2, 0.0)
+    p = Dist(ids=[0, 1], W=[6, 4])
+    q = Dist(ids=[0, 2], W=[5, 5])
+    assert accept(p, q, 0, 2 ** 53 - 1)          # p(0) >= q(0): always kept
+    assert not accept(p, q, 2, 0)                # p(2) = 0: never kept (strict)
+    # keep probability exactly p/q: 0.4/0.5 = 4/5 of the uniform range
+    p2 = Dist(ids=[0, 5], W=[4, 6])
+    edge = -(-(2 ** 53 * 4) // 5)                # ceil(0.8 * 2^53): first rejected U
+    assert accept(p2, q, 0, edge - 1) and not accept(p2, q, 0, edge)
 
 
 def _emission_law(p: Dist, q: Dist):
     """Exact law of the code emitted for one draft: q(d) min(1,p/q) on accept + residual."""
     law = {}
-    a = 0.0
+    a = Fraction(0)
     for d in q.ids:
-        keep = min(1.0, p.prob(d) / q.prob(d))
-        law[d] = law.get(d, 0.0) + q.prob(d) * keep
-        a += q.prob(d) * keep
+        keep = min(Fraction(1), p.frac(d) / q.frac(d))
+        law[d] = law.get(d, Fraction(0)) + q.frac(d) * keep
+        a += q.frac(d) * keep
     xs, r, R = residual_weights(p, q)
     for x, rx in zip(xs, r):
-        law[x] = law.get(x, 0.0) + (1.0 - a) * rx / R
+        law[x] = law.get(x, Fraction(0)) + (1 - a) * Fraction(rx, R)
     return law, a
 
 
@@ -114,8 +157,8 @@ def test_acceptance_rule_is_lossless_exactly(V, k):
         p, q = _random_pair(rng, V, k)
         law, a = _emission_law(p, q)
         for x in range(V):
-            assert abs(law.get(x, 0.0) - p.prob(x)) < 1e-15
-        assert math.isclose(a, alpha(p, q), rel_tol=1e-13, abs_tol=1e-15)
+            assert law.get(x, Fraction(0)) == p.frac(x)
+        assert a == alpha(p, q)
 
 
 def test_acceptance_rule_is_lossless_statistically():
@@ -125,27 +168,27 @@ def test_acceptance_rule_is_lossless_statistically():
     counts = np.zeros(8)
     kept = 0
     for i in range(n):
-        d = draw(q, philox.uniform(4, 0, i, 0, 2, philox.PURPOSE_DRAFT))
-        if accept(p, q, d, philox.uniform(4, 0, i, 0, 2, philox.PURPOSE_ACCEPT)):
+        d = draw(q, philox.uniform_int(4, 0, i, 0, 2, philox.PURPOSE_DRAFT))
+        if accept(p, q, d, philox.uniform_int(4, 0, i, 0, 2, philox.PURPOSE_ACCEPT)):
             counts[d] += 1
             kept += 1
         else:
-            counts[residual_draw(p, q, philox.uniform(4, 0, i, 0, 2, philox.PURPOSE_TARGET))] += 1
+            counts[residual_draw(p, q, philox.uniform_int(4, 0, i, 0, 2, philox.PURPOSE_TARGET))] += 1
     exp = np.array([p.prob(x) for x in range(8)]) * n
     m = exp > 0
     assert counts[~m].sum() == 0
-    assert stats.chisquare(counts[m], exp[m]).pvalue > 1e-4
-    a = alpha(p, q)
+    assert stats.chisquare(counts[m], exp[m] * counts[m].sum() / exp[m].sum()).pvalue > 1e-4
+    a = float(alpha(p, q))
     assert abs(kept / n - a) < 4 * math.sqrt(a * (1 - a) / n) + 1e-9
 
 
 def test_residual_support_is_where_p_exceeds_q():
-    p = Dist(ids=[0, 1, 2], e=[0.5, 0.3, 0.2], S=1.0)
-    q = Dist(ids=[0, 3], e=[0.9, 0.1], S=1.0)
+    p = Dist(ids=[0, 1, 2], W=[5, 3, 2])
+    q = Dist(ids=[0, 3], W=[9, 1])
     xs, r, R = residual_weights(p, q)
     assert xs == [0, 1, 2]
-    assert r[0] == 0.0 and r[1] == 0.3 and r[2] == 0.2
-    assert residual_draw(p, q, 0.0) == 1
-    assert residual_draw(p, q, 0.99) == 2
-    # p == q: R = 0 falls back to p (the accept test keeps every draft then)
-    assert residual_draw(p, p, 0.0) == 0
+    # N_x = S_p S_q max(0, p - q): S_p = S_q = 10
+    assert r == [0, 30, 20] and R == 50
+    assert residual_draw(p, q, 0) == 1
+    assert residual_draw(p, q, 2 ** 53 - 1) == 2
+    assert residual_draw(p, p, 0) == 0           # p == q: R = 0 falls back to p
