@@ -26,7 +26,13 @@
  * counter = (stream id, frame index, (call index << 8) | position, purpose); purpose
  * 0 = target / residual / bonus sample, 1 = accept test, 2 = draft sample,
  * 3 + v/2 = Gaussian pair for vocabulary entries (v, v+1) of a noisy draft row.
- * A uniform is ((w0 >> 5) * 2^26 + (w1 >> 6)) * 2^-53 from words 0 and 1.
+ * A decision uses U = (w0 >> 5) * 2^26 + (w1 >> 6) from words 0 and 1 (u = U / 2^53).
+ *
+ * Distributions: the top-k set of a logits row in order (fp32 logit desc, id asc) with
+ * integer weights W_i = floor(2^24 * exp32(z_i - z_max)), z = fp32 logit / fp32 T, where
+ * exp32 is an fp32 exponential (Cody-Waite range reduction, degree-7 Taylor polynomial);
+ * p(x) = W_x / S, S = sum W.  Draws, accept tests (u < p(d)/q(d)) and residual draws
+ * (normalised max(0, p - q)) are exact integer comparisons.
  */
 #ifndef MCD_H
 #define MCD_H
@@ -55,7 +61,7 @@ enum { MCD_DRAFT_SAMPLE = 0, MCD_DRAFT_GREEDY = 1, MCD_DRAFT_NOISY_TARGET = 2 };
 
 /* Model and sampling configuration.  Limits: hidden, ffn multiples of 128; head_dim 64
  * or 128; n_q_heads multiple of n_kv_heads; vocab multiple of 16 and <= 4096;
- * n_pos <= 15; draft_len (K) <= 7; top_k in 1..256 and <= vocab; c0_vocab <= 4096. */
+ * n_pos <= 15; draft_len (K) <= 7; top_k in 1..128 and <= vocab; c0_vocab <= 4096. */
 typedef struct {
   int32_t n_layers, hidden, n_q_heads, n_kv_heads, head_dim, ffn;
   int32_t n_pos;        /* residual positions c1..c_{n_pos} (15 in the paper)           */
@@ -149,10 +155,11 @@ mcd_status mcd_verify_accept(mcd_ctx* ctx, int32_t* emitted, int32_t* n_emitted,
  * z_j = LMH_{k+j}(h_k + b_j); q_j = top-k/temperature softmax of z_j; d_j ~ q_j with the
  * draft-purpose uniform of (call_idx, k+j) under the frame set by mcd_begin_frame.
  *   h_k      dev float [hidden], the post-norm hidden state read by LM head k (1 <= k < n_pos)
- *   draft_ids dev int32 [K]; q_ids dev int32 [K, top_k]; q_probs dev double [K, top_k]
- *   z_out    dev float [K, vocab], optional.  Unused rows are left untouched. */
+ *   draft_ids dev int32 [K]; q_ids dev int32 [K, top_k] and q_weights dev uint32
+ *   [K, top_k] (optional): the draft distributions; z_out dev float [K, vocab], optional.
+ *   Unused rows are left untouched. */
 mcd_status mcd_draft(mcd_ctx* ctx, int32_t pos_k, int32_t call_idx, const float* h_k,
-                     int32_t* draft_ids, int32_t* q_ids, double* q_probs, float* z_out);
+                     int32_t* draft_ids, int32_t* q_ids, uint32_t* q_weights, float* z_out);
 
 /* Sampler on given fp32 logits (parity hook for the acceptance rule).  p_logits dev
  * float [n_drafts+1, vocab] are the verify rows of positions a+1..a+1+n_drafts (the last
@@ -165,11 +172,12 @@ mcd_status mcd_accept_from_logits(mcd_ctx* ctx, int32_t a, int32_t n_drafts, int
                                   const float* p_logits, const float* q_logits,
                                   const int32_t* draft_ids, int32_t* emitted, int32_t* out2);
 
-/* Top-k / temperature softmax of n_rows fp32 logits rows (dev float [n_rows, vocab]):
- * ids (dev int32 [n_rows, top_k]) in sampling order (logit desc, id asc), probs
- * (dev double [n_rows, top_k]) = exp(z_i - z_max) / S with z = logit / temperature. */
+/* Top-k / temperature distributions of n_rows fp32 logits rows (dev float [n_rows,
+ * vocab], n_rows <= 128): ids (dev int32 [n_rows, top_k]) in sampling order (logit desc,
+ * id asc), weights (dev uint32 [n_rows, top_k]) and sums (dev uint64 [n_rows]); any
+ * output may be NULL. */
 mcd_status mcd_topk_softmax(mcd_ctx* ctx, int32_t n_rows, const float* logits,
-                            int32_t* ids, double* probs);
+                            int32_t* ids, uint32_t* weights, uint64_t* sums);
 
 /* Tracing for parity tests: while `trace` (dev, mcd_trace_bytes() bytes) is set, frame
  * decoding writes one mcd_call_trace per call followed, after 16 records, by float

@@ -124,7 +124,8 @@ __global__ void zero_emitted_kernel(const DevState* st, int* n_emitted) {
 
 // Top-k of n rows (one CTA of 256 threads per row).
 __global__ void __launch_bounds__(kConsumerThreads) topk_rows_kernel(const float* logits, int V, int k, float T,
-                                                                     TopkRec* recs, int32_t* ids, double* probs) {
+                                                                     TopkRec* recs, int32_t* ids, uint32_t* weights,
+                                                                     unsigned long long* sums) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
   TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
   const int row = blockIdx.x;
@@ -134,8 +135,9 @@ __global__ void __launch_bounds__(kConsumerThreads) topk_rows_kernel(const float
   __threadfence_block();
   for (int i = threadIdx.x; i < k; i += kConsumerThreads) {
     if (ids) ids[(size_t)row * k + i] = r->ids[i];
-    if (probs) probs[(size_t)row * k + i] = r->e[i] / r->S;
+    if (weights) weights[(size_t)row * k + i] = r->W[i];
   }
+  if (threadIdx.x == 0 && sums) sums[row] = r->S;
 }
 
 // Acceptance on given logits: rows 0..n_d of p, rows 0..n_d-1 of q, one CTA.
@@ -192,7 +194,7 @@ __global__ void draft_logits_kernel(FrameParams p, int pos_k, int n_j, const flo
 
 __global__ void __launch_bounds__(kConsumerThreads) draft_sample_kernel(FrameParams p, int pos_k, int call,
                                                                         const float* z, TopkRec* recs, int* draft_ids,
-                                                                        int* q_ids, double* q_probs) {
+                                                                        int* q_ids, uint32_t* q_weights) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
   TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
   const int j = blockIdx.x + 1;
@@ -201,12 +203,12 @@ __global__ void __launch_bounds__(kConsumerThreads) draft_sample_kernel(FramePar
   consumer_sync();
   __threadfence_block();
   if (threadIdx.x == 0) {
-    const double u = uniform_u(p.seed, p.stream_id, p.frame_idx, call, pos_k + j, PURPOSE_DRAFT);
-    draft_ids[j - 1] = seq_draw(r, u);
+    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, pos_k + j, PURPOSE_DRAFT);
+    draft_ids[j - 1] = seq_draw(r, U);
   }
   for (int i = threadIdx.x; i < p.top_k; i += kConsumerThreads) {
     if (q_ids) q_ids[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->ids[i] : -1;
-    if (q_probs) q_probs[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->e[i] / r->S : 0.0;
+    if (q_weights) q_weights[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->W[i] : 0u;
   }
 }
 
@@ -642,7 +644,7 @@ mcd_status mcd_verify_accept(mcd_ctx* c, int32_t* emitted, int32_t* n_emitted, f
 }
 
 mcd_status mcd_draft(mcd_ctx* c, int32_t pos_k, int32_t call_idx, const float* h_k, int32_t* draft_ids,
-                     int32_t* q_ids, double* q_probs, float* z_out) {
+                     int32_t* q_ids, uint32_t* q_weights, float* z_out) {
   if (!c || !h_k || !draft_ids) return MCD_ERR_INVALID_ARG;
   if (!c->weights_loaded || !c->frame_begun) return MCD_ERR_STATE;
   FrameParams& p = c->fp;
@@ -653,7 +655,7 @@ mcd_status mcd_draft(mcd_ctx* c, int32_t pos_k, int32_t call_idx, const float* h
   const int warps = n_j * p.V;
   draft_logits_kernel<<<(warps * 32 + 255) / 256, 256, 0, c->stream>>>(p, pos_k, n_j, h_k, z);
   draft_sample_kernel<<<n_j, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(p, pos_k, call_idx, z, p.topk,
-                                                                                  draft_ids, q_ids, q_probs);
+                                                                                  draft_ids, q_ids, q_weights);
   MCD_CHECK(cudaGetLastError());
   return MCD_OK;
 }
@@ -672,13 +674,14 @@ mcd_status mcd_accept_from_logits(mcd_ctx* c, int32_t a, int32_t n_drafts, int32
   return MCD_OK;
 }
 
-mcd_status mcd_topk_softmax(mcd_ctx* c, int32_t n_rows, const float* logits, int32_t* ids, double* probs) {
+mcd_status mcd_topk_softmax(mcd_ctx* c, int32_t n_rows, const float* logits, int32_t* ids, uint32_t* weights,
+                            uint64_t* sums) {
   if (!c || !logits || n_rows < 0) return MCD_ERR_INVALID_ARG;
   if (n_rows == 0) return MCD_OK;
   FrameParams& p = c->fp;
   if (n_rows > 2 * kMaxRows * (kMaxDraft + 1)) return MCD_ERR_UNSUPPORTED;
-  topk_rows_kernel<<<n_rows, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(logits, p.V, p.top_k, p.T, p.topk,
-                                                                                  ids, probs);
+  topk_rows_kernel<<<n_rows, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(
+      logits, p.V, p.top_k, p.T, p.topk, ids, weights, reinterpret_cast<unsigned long long*>(sums));
   MCD_CHECK(cudaGetLastError());
   return MCD_OK;
 }

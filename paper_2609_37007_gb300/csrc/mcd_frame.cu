@@ -811,14 +811,14 @@ __device__ void run_call(Cons& c, int call) {
 }
 
 // Copy distribution records into shared memory with independent word loads: the header,
-// ids[0..k) and e[0..k) of each (k = top_k; entries past a record's n are never read).
+// ids[0..k) and W[0..k) of each (k = top_k; entries past a record's n are never read).
 template <class Src>
 __device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src) {
-  constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kEWord = offsetof(TopkRec, e) / 4;
-  const int words = kIdsWord + 3 * k;
+  constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kWWord = offsetof(TopkRec, W) / 4;
+  const int words = kIdsWord + 2 * k;
   for (int i = threadIdx.x; i < nrec * words; i += kConsumerThreads) {
     const int r = i / words, w = i - r * words;
-    const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kEWord + (w - kIdsWord - k));
+    const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kWWord + (w - kIdsWord - k));
     reinterpret_cast<int*>(dst + r)[off] = __ldcg(reinterpret_cast<const int*>(src(r)) + off);
   }
 }
@@ -866,8 +866,8 @@ __device__ void accept_step(Cons& c, int call) {
   consumer_sync();
   if (threadIdx.x == 0) {
     for (int j = 1; j <= n_next; ++j) {
-      const double u = uniform_u(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
-      s_next[j - 1] = seq_draw(srec + j - 1, u);
+      const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
+      s_next[j - 1] = seq_draw(srec + j - 1, U);
     }
     s_nnext = n_next;
     DevState* st = p.st;

@@ -18,7 +18,7 @@ namespace mcd {
 
 constexpr int kMaxRows = 8;          // rows of one call (K+1 <= 8; first call uses 2)
 constexpr int kMaxDraft = 7;         // K
-constexpr int kMaxTopK = 256;
+constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
 constexpr int kMaxCalls = 16;        // calls per frame (15 positions, first call emits 1)
 constexpr int kMaxVocab = 4096;
@@ -64,13 +64,13 @@ struct DevState {
   int err;
 };
 
-// One top-k / temperature distribution.
+// One top-k / temperature distribution as integer weights: p(ids[i]) = W[i] / S.
 struct TopkRec {
   int n;
   int pad;
-  double S;
+  unsigned long long S;
   int ids[kMaxTopK];
-  double e[kMaxTopK];
+  uint32_t W[kMaxTopK];
 };
 
 struct FrameParams {
@@ -239,11 +239,12 @@ __host__ __device__ inline void philox_block(unsigned long long seed, uint32_t s
   out[3] = purpose;
   philox4x32_10(out, (uint32_t)(seed & 0xFFFFFFFFull), (uint32_t)(seed >> 32));
 }
-__host__ __device__ inline double uniform_u(unsigned long long seed, uint32_t stream, uint32_t frame, int call,
-                                            int pos, uint32_t purpose) {
+// The 53-bit integer uniform of a decision: u = U / 2^53 = res53(w0, w1).
+__host__ __device__ inline unsigned long long uniform_U(unsigned long long seed, uint32_t stream, uint32_t frame,
+                                                        int call, int pos, uint32_t purpose) {
   uint32_t w[4];
   philox_block(seed, stream, frame, call, pos, purpose, w);
-  return res53(w[0], w[1]);
+  return ((unsigned long long)(w[0] >> 5) << 26) | (unsigned long long)(w[1] >> 6);
 }
 
 enum { PURPOSE_TARGET = 0, PURPOSE_ACCEPT = 1, PURPOSE_DRAFT = 2, PURPOSE_NOISE = 3 };

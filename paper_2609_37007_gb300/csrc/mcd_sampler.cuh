@@ -1,16 +1,17 @@
-// Top-k / temperature softmax, categorical draw, acceptance test and residual resampling
+// Top-k / temperature sampling, categorical draw, acceptance test and residual resampling
 // on the device (Abstract and Sec. 3.2: the deployed top-k sampling is kept and drafts are
 // verified with the standard lossless rule: keep d with probability min(1, p(d)/q(d)),
 // otherwise resample from max(0, p - q) renormalised).
 //
-// Fixed so that the GPU and the CPU oracle take every integer decision from the same fp32
-// logits and the same uniforms:
+// A distribution is a list of integer weights (ids in sampling order, W, S = sum W):
 //   * top-k set and order: (fp32 logit desc, id asc); -0 and +0 compare equal;
-//   * z = double(logit) / double(T), e_i = exp(z_i - z_max), S = sequential sum in order;
-//   * draw: first i with u*S < e_0 + ... + e_i;
-//   * accept: u * q(d) < p(d) with p(x) = e_x / S (0 outside the top-k);
-//   * residual: r(x) = max(0, p(x) - q(x)) over p's support in ascending id order, drawn
-//     like a categorical with R = sequential sum of r; R == 0 draws from p.
+//   * z = fp32 logit / fp32 T; W_i = floor(2^24 * exp32(z_i - z_max)); p(x) = W_x / S;
+//   * draw with a 53-bit integer uniform U: first i with U*S < 2^53 * (W_0 + .. + W_i);
+//   * accept draft d iff U * Wq_d * S_p < 2^53 * Wp_d * S_q  (u < p(d)/q(d));
+//   * residual: N_x = max(0, Wp_x S_q - Wq_x S_p) over p's support in ascending id order,
+//     first x with U * R < 2^53 * (N_1 + .. + N_x), R = sum N; R == 0 draws from p.
+// Every decision is an exact integer comparison, so a CPU implementation that computes the
+// same fp32 exp32 agrees bit for bit; sums are order-free and need no fp64 arithmetic.
 #pragma once
 #include "mcd_internal.cuh"
 
@@ -21,16 +22,55 @@ struct TopkScratch {
   uint32_t hist[256];
   uint32_t cand_key[kMaxTopK];
   int cand_id[kMaxTopK];
-  double e[kMaxTopK];
+  unsigned long long wsum[kConsumerWarps];
   int misc[8];
   int warp_tot[kConsumerWarps];
 };
 static_assert(sizeof(TopkScratch) <= kActBytes, "top-k scratch must fit the activation region");
 
 struct ResidualScratch {
-  double r[kMaxTopK];
+  unsigned long long n[kMaxTopK];
   int x[kMaxTopK];
 };
+
+// fp32 exponential of d <= 0: Cody-Waite range reduction (Cody and Waite, "Software Manual
+// for the Elementary Functions", 1980) with ln 2 = C1 + C2, then e^r by the degree-7 Taylor
+// polynomial in Horner form and a scale by 2^n.  Every step is one IEEE single-precision
+// operation with round-to-nearest (no contraction into fused multiply-add), constants are
+// the fp32 roundings of log2(e), C1 = 0.693359375, C2 = ln 2 - C1 and 1/k!.
+__device__ __forceinline__ float exp32_cw(float d) {
+  if (d < -87.0f) return 0.0f;
+  const float n = rintf(__fmul_rn(d, __int_as_float(0x3fb8aa3b)));
+  const float r = __fsub_rn(__fsub_rn(d, __fmul_rn(n, __int_as_float(0x3f318000))),
+                            __fmul_rn(n, __int_as_float(0xb95e8083)));
+  float p = __int_as_float(0x39500d01);                        // 1/7!
+  p = __fadd_rn(__fmul_rn(p, r), __int_as_float(0x3ab60b61));  // 1/6!
+  p = __fadd_rn(__fmul_rn(p, r), __int_as_float(0x3c088889));  // 1/5!
+  p = __fadd_rn(__fmul_rn(p, r), __int_as_float(0x3d2aaaab));  // 1/4!
+  p = __fadd_rn(__fmul_rn(p, r), __int_as_float(0x3e2aaaab));  // 1/3!
+  p = __fadd_rn(__fmul_rn(p, r), 0.5f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  p = __fadd_rn(__fmul_rn(p, r), 1.0f);
+  return __fmul_rn(p, __int_as_float(((int)n + 127) << 23));
+}
+
+__device__ __forceinline__ uint32_t weight24(float e) { return __float2uint_rd(__fmul_rn(e, 16777216.0f)); }
+
+// ---- exact 128-bit helpers -------------------------------------------------------------
+struct U128 {
+  unsigned long long lo, hi;
+};
+__device__ __forceinline__ U128 mul64(unsigned long long a, unsigned long long b) {
+  return U128{a * b, __umul64hi(a, b)};
+}
+// (a * b) for a product known to fit in 128 bits
+__device__ __forceinline__ U128 mul128x64(U128 a, unsigned long long b) {
+  U128 r = mul64(a.lo, b);
+  r.hi += a.hi * b;
+  return r;
+}
+__device__ __forceinline__ U128 shl53(unsigned long long x) { return U128{x << 53, x >> 11}; }
+__device__ __forceinline__ bool lt128(U128 a, U128 b) { return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo); }
 
 __device__ __forceinline__ uint32_t f32_key(float v) {
   uint32_t u = __float_as_uint(v);
@@ -41,12 +81,12 @@ __device__ __forceinline__ float key_f32(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k ^ 0x80000000u) : ~k);
 }
 
-// Block-wide (256 consumer threads) top-k of one fp32 row.  `greedy` replaces the
-// distribution by the one-hot of its first entry.  Result written to `out` (global).
+// Block-wide (256 consumer threads) top-k of one fp32 row into `out` (global or shared).
+// `greedy` replaces the distribution by the one-hot of its first entry.
 static __device__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
-                           TopkScratch& s, TopkRec* out) {
+                                  TopkScratch& s, TopkRec* out) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int i = tid; i < (V >> 2); i += 2 * kConsumerThreads) {   // V % 16 == 0: 16-byte loads, two in flight
+  for (int i = tid; i < (V >> 2); i += 2 * kConsumerThreads) {   // V % 16 == 0: two 16-byte loads in flight
     const int i2 = i + kConsumerThreads;
     const float4 a = __ldcg(reinterpret_cast<const float4*>(logits) + i);
     float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -62,6 +102,7 @@ static __device__ void block_topk(const float* __restrict__ logits, int V, int k
       s.keys[4 * i2 + 3] = f32_key(b.w);
     }
   }
+  // radix select of the k-th largest key, 8 bits per pass
   uint32_t prefix = 0, mask = 0;
   int krem = k;
   int count_eq = 0;
@@ -170,88 +211,92 @@ static __device__ void block_topk(const float* __restrict__ logits, int V, int k
     s.cand_id[rank] = mid;
   }
   consumer_sync();
+  // integer weights and their (order-free) sum
+  uint32_t w = 0;
   if (tid < k) {
-    const double Td = (double)T;
-    const double m = (double)key_f32(s.cand_key[0]) / Td;
-    const double z = (double)key_f32(s.cand_key[tid]) / Td;
-    const double e = exp(z - m);
-    s.e[tid] = e;
+    const float z0 = __fdiv_rn(key_f32(s.cand_key[0]), T);
+    const float z = __fdiv_rn(key_f32(s.cand_key[tid]), T);
+    w = greedy ? (tid == 0 ? 1u : 0u) : weight24(exp32_cw(__fsub_rn(z, z0)));
     out->ids[tid] = s.cand_id[tid];
-    out->e[tid] = greedy ? (tid == 0 ? 1.0 : 0.0) : e;
+    out->W[tid] = w;
   }
+  unsigned long long ws = w;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) ws += __shfl_xor_sync(0xFFFFFFFFu, ws, o);
+  if (lane == 0) s.wsum[warp] = ws;
   consumer_sync();
   if (tid == 0) {
-    double S = 0.0;
-    for (int j = 0; j < k; ++j) S += s.e[j];
-    out->S = greedy ? 1.0 : S;
+    unsigned long long S = 0;
+#pragma unroll
+    for (int w2 = 0; w2 < kConsumerWarps; ++w2) S += s.wsum[w2];
+    out->S = S;
     out->n = greedy ? 1 : k;
   }
 }
 
-// The helpers below read records through generic pointers: the frame kernel stages them in
-// shared memory, the standalone sampler kernels read the global copies their own CTA wrote.
+// The record helpers read through generic pointers: the frame kernel stages records in
+// shared memory, the standalone sampler kernels read the copies their own CTA wrote.
 
-// p(x) of a distribution record, evaluated by a full warp (same value on every lane).
-__device__ __forceinline__ double warp_prob(const TopkRec* r, int x) {
+// W_x of a record (0 outside it), evaluated by a full warp (same value on every lane).
+__device__ __forceinline__ uint32_t warp_weight(const TopkRec* r, int x) {
   const int lane = threadIdx.x & 31;
   const int n = r->n;
   int found = -1;
   for (int i = lane; i < n; i += 32)
     if (r->ids[i] == x) found = i;
   const unsigned b = __ballot_sync(0xFFFFFFFFu, found >= 0);
-  if (!b) return 0.0;
+  if (!b) return 0u;
   const int idx = __shfl_sync(0xFFFFFFFFu, found, __ffs(b) - 1);
-  return r->e[idx] / r->S;
+  return r->W[idx];
 }
 
-// Sequential inverse-CDF draw (one thread).
-__device__ __forceinline__ int seq_draw(const TopkRec* r, double u) {
+// Inverse-CDF draw (one thread).
+__device__ __forceinline__ int seq_draw(const TopkRec* r, unsigned long long U) {
   const int n = r->n;
-  const double t = u * r->S;
-  double c = 0.0;
+  const U128 lhs = mul64(U, r->S);
+  unsigned long long c = 0;
   for (int i = 0; i < n; ++i) {
-    c += r->e[i];
-    if (t < c) return r->ids[i];
+    c += r->W[i];
+    if (lt128(lhs, shl53(c))) return r->ids[i];
   }
   return r->ids[n - 1];
 }
 
 // Residual draw from normalise(max(0, p - q)), evaluated by a full warp.
-static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, double u, ResidualScratch& rs) {
+static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U, ResidualScratch& rs) {
   const int lane = threadIdx.x & 31;
   const int np = p->n, nq = q->n;
-  const double Sp = p->S, Sq = q->S;
+  const unsigned long long Sp = p->S, Sq = q->S;
   for (int i = lane; i < np; i += 32) {
     const int x = p->ids[i];
-    const double px = p->e[i] / Sp;
-    double qx = 0.0;
+    unsigned long long wq = 0;
     for (int j = 0; j < nq; ++j)
       if (q->ids[j] == x) {
-        qx = q->e[j] / Sq;
+        wq = q->W[j];
         break;
       }
+    const unsigned long long a = (unsigned long long)p->W[i] * Sq, b = wq * Sp;
     int rank = 0;
     for (int j = 0; j < np; ++j) rank += (p->ids[j] < x);
-    rs.r[rank] = fmax(0.0, px - qx);
+    rs.n[rank] = a > b ? a - b : 0ull;
     rs.x[rank] = x;
   }
   __syncwarp();
   int out = 0;
   if (lane == 0) {
-    double R = 0.0;
-    for (int i = 0; i < np; ++i) R += rs.r[i];
-    if (R == 0.0) {
-      out = seq_draw(p, u);
+    unsigned long long R = 0;
+    for (int i = 0; i < np; ++i) R += rs.n[i];
+    if (R == 0) {
+      out = seq_draw(p, U);
     } else {
-      const double t = u * R;
-      double c = 0.0;
-      out = rs.x[np - 1];
+      const U128 lhs = mul64(U, R);
+      unsigned long long c = 0;
       int last = rs.x[np - 1];
       bool hit = false;
       for (int i = 0; i < np && !hit; ++i) {
-        c += rs.r[i];
-        if (rs.r[i] > 0.0) last = rs.x[i];
-        if (t < c) {
+        c += rs.n[i];
+        if (rs.n[i] > 0) last = rs.x[i];
+        if (lt128(lhs, shl53(c))) {
           out = rs.x[i];
           hit = true;
         }
@@ -285,24 +330,23 @@ __device__ AcceptResult warp_accept(int a, int n_d, int n_pos, const int* drafts
     const TopkRec* pr = p_row(i);
     const TopkRec* qr = q_rec(i);
     const int d = drafts[i];
-    const double pd = warp_prob(pr, d);
-    const double qd = warp_prob(qr, d);
-    const double u = uniform_u(seed, stream, frame, call, s, PURPOSE_ACCEPT);
-    if (u * qd < pd) {
+    const unsigned long long wp = warp_weight(pr, d), wq = warp_weight(qr, d);
+    const unsigned long long U = uniform_U(seed, stream, frame, call, s, PURPOSE_ACCEPT);
+    if (lt128(mul128x64(mul64(U, wq), pr->S), shl53(wp * qr->S))) {
       res.emitted[res.n_emit++] = d;
       res.n_acc++;
     } else {
-      const double u2 = uniform_u(seed, stream, frame, call, s, PURPOSE_TARGET);
-      res.emitted[res.n_emit++] = warp_residual(pr, qr, u2, rs);
+      const unsigned long long U2 = uniform_U(seed, stream, frame, call, s, PURPOSE_TARGET);
+      res.emitted[res.n_emit++] = warp_residual(pr, qr, U2, rs);
       rejected = true;
     }
   }
   if (!rejected) {
     const int s = a + 1 + n_d;
     if (s <= n_pos) {
-      const double u = uniform_u(seed, stream, frame, call, s, PURPOSE_TARGET);
+      const unsigned long long U = uniform_U(seed, stream, frame, call, s, PURPOSE_TARGET);
       int x = 0;
-      if ((threadIdx.x & 31) == 0) x = seq_draw(p_row(n_d), u);
+      if ((threadIdx.x & 31) == 0) x = seq_draw(p_row(n_d), U);
       res.emitted[res.n_emit++] = __shfl_sync(0xFFFFFFFFu, x, 0);
     }
   }

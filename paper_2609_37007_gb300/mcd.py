@@ -73,7 +73,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_verify_accept": (I32, [P, P, P, P]),
         "mcd_draft": (I32, [P, I32, I32, P, P, P, P, P]),
         "mcd_accept_from_logits": (I32, [P, I32, I32, I32, P, P, P, P, P]),
-        "mcd_topk_softmax": (I32, [P, I32, P, P, P]),
+        "mcd_topk_softmax": (I32, [P, I32, P, P, P, P]),
         "mcd_trace_bytes": (I64, [P]),
         "mcd_set_trace": (I32, [P, P]),
         "mcd_set_timeline": (I32, [P, P]),
@@ -147,9 +147,9 @@ def mcd_verify_accept(ctx, emitted, n_emitted, logits_out=None):
         ctx, _ptr(emitted), _ptr(n_emitted), _ptr(logits_out)))
 
 
-def mcd_draft(ctx, pos_k: int, call_idx: int, h_k, draft_ids, q_ids=None, q_probs=None, z_out=None):
+def mcd_draft(ctx, pos_k: int, call_idx: int, h_k, draft_ids, q_ids=None, q_weights=None, z_out=None):
     _check("mcd_draft", load_library().mcd_draft(
-        ctx, pos_k, call_idx, _ptr(h_k), _ptr(draft_ids), _ptr(q_ids), _ptr(q_probs), _ptr(z_out)))
+        ctx, pos_k, call_idx, _ptr(h_k), _ptr(draft_ids), _ptr(q_ids), _ptr(q_weights), _ptr(z_out)))
 
 
 def mcd_accept_from_logits(ctx, a: int, n_drafts: int, call_idx: int, p_logits, q_logits, draft_ids,
@@ -159,9 +159,9 @@ def mcd_accept_from_logits(ctx, a: int, n_drafts: int, call_idx: int, p_logits, 
         _ptr(out2)))
 
 
-def mcd_topk_softmax(ctx, n_rows: int, logits, ids, probs):
+def mcd_topk_softmax(ctx, n_rows: int, logits, ids, weights=None, sums=None):
     _check("mcd_topk_softmax", load_library().mcd_topk_softmax(ctx, n_rows, _ptr(logits), _ptr(ids),
-                                                                _ptr(probs)))
+                                                                _ptr(weights), _ptr(sums)))
 
 
 def mcd_trace_bytes(ctx) -> int:
