@@ -17,7 +17,7 @@ weights, so that each decision is an exact rational comparison:
        in the sorted order with U * S < 2^53 * (W_0 + ... + W_i).
   R-S4 accept test: keep draft d iff U * Wq_d * S_p < 2^53 * Wp_d * S_q, i.e. u < p(d)/q(d).
   R-S5 residual: N_x = max(0, Wp_x * S_q - Wq_x * S_p) = S_p S_q max(0, p(x) - q(x)) over
-       p's support in ascending id order, R = sum N; draw the first x with
+       p's support in p's sampling order (R-S1), R = sum N; draw the first x with
        U * R < 2^53 * (N_1 + ... + N_x); R == 0 draws from p.
   R-S6 greedy drafts: q is one-hot at the first id of the sorted order (W = [1]).
   R-S7 exp32: fp32 exponential by Cody and Waite's range reduction ("Software Manual for
@@ -122,8 +122,8 @@ def accept(p: Dist, q: Dist, d: int, U: int) -> bool:
 
 
 def residual_weights(p: Dist, q: Dist):
-    """R-S5 weights: (ids ascending, N_x, R) with N_x / R = normalise(max(0, p - q))."""
-    xs = sorted(p.ids)
+    """R-S5 weights: (p's ids in sampling order, N_x, R), N_x / R = normalise(max(0, p - q))."""
+    xs = list(p.ids)
     n = [max(0, p.weight(x) * q.S - q.weight(x) * p.S) for x in xs]
     return xs, n, sum(n)
 

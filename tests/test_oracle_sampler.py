@@ -186,9 +186,13 @@ def test_residual_support_is_where_p_exceeds_q():
     p = Dist(ids=[0, 1, 2], W=[5, 3, 2])
     q = Dist(ids=[0, 3], W=[9, 1])
     xs, r, R = residual_weights(p, q)
-    assert xs == [0, 1, 2]
+    assert xs == [0, 1, 2]                       # p's sampling order
     # N_x = S_p S_q max(0, p - q): S_p = S_q = 10
     assert r == [0, 30, 20] and R == 50
     assert residual_draw(p, q, 0) == 1
     assert residual_draw(p, q, 2 ** 53 - 1) == 2
     assert residual_draw(p, p, 0) == 0           # p == q: R = 0 falls back to p
+    # the walk follows p's sampling order, not id order
+    p3 = Dist(ids=[7, 1], W=[2, 2])
+    q3 = Dist(ids=[5], W=[1])
+    assert residual_draw(p3, q3, 0) == 7
