@@ -9,17 +9,17 @@ it (readings R-S1..R-S7 of the design notes).  Every distribution is a list of i
 weights, so that each decision is an exact rational comparison:
 
   R-S1 top-k set: sort by (fp32 logit descending, id ascending), keep the first k;
-       k >= V keeps every id.
+       k >= V keeps every id.  A distribution lists its set in ascending id order.
   R-S2 weights: z_i = fp32(logit_i) / fp32(T) and d_i = z_i - z_max in fp32,
        e_i = exp32(d_i) (below), W_i = floor(2^24 * e_i); S = sum of W.  The
        distribution is p(x) = W_x / S exactly (p(x) = 0 outside the top-k).
   R-S3 categorical draw with a 53-bit integer uniform U (u = U / 2^53): the first entry i
-       in the sorted order with U * S < 2^53 * (W_0 + ... + W_i).
+       in ascending id order with U * S < 2^53 * (W_0 + ... + W_i).
   R-S4 accept test: keep draft d iff U * Wq_d * S_p < 2^53 * Wp_d * S_q, i.e. u < p(d)/q(d).
   R-S5 residual: N_x = max(0, Wp_x * S_q - Wq_x * S_p) = S_p S_q max(0, p(x) - q(x)) over
-       p's support in p's sampling order (R-S1), R = sum N; draw the first x with
+       p's support in ascending id order, R = sum N; draw the first x with
        U * R < 2^53 * (N_1 + ... + N_x); R == 0 draws from p.
-  R-S6 greedy drafts: q is one-hot at the first id of the sorted order (W = [1]).
+  R-S6 greedy drafts: q is one-hot at the largest logit, ties to the lowest id (W = [1]).
   R-S7 exp32: fp32 exponential by Cody and Waite's range reduction ("Software Manual for
        the Elementary Functions", 1980): n = rint(d * log2 e), r = (d - n*C1) - n*C2 with
        ln 2 = C1 + C2 split so that n*C1 is exact, then e^r by the degree-7 Taylor
@@ -60,7 +60,7 @@ def exp32(d) -> np.float32:
 
 @dataclass
 class Dist:
-    """A top-k / temperature distribution: ids in sampling order, integer weights W, S = sum W."""
+    """A top-k / temperature distribution: ids in draw order, integer weights W, S = sum W."""
     ids: List[int]
     W: List[int]
     S: int = 0
@@ -93,10 +93,11 @@ def topk_order(logits: Sequence[float], k: int) -> List[int]:
 def topk_dist(logits: Sequence[float], k: int, temperature: float) -> Dist:
     """R-S1, R-S2 on an fp32 logits row; the temperature is taken as its fp32 value."""
     l32 = np.asarray(logits, dtype=np.float32)
-    ids = topk_order(l32, k)
+    top = topk_order(l32, k)
     T = F32(temperature)
-    z = [l32[i] / T for i in ids]
-    W = [int(math.floor(float(exp32(zi - z[0])) * 2.0 ** WEIGHT_BITS)) for zi in z]
+    z_max = l32[top[0]] / T
+    ids = sorted(top)
+    W = [int(math.floor(float(exp32(l32[i] / T - z_max)) * 2.0 ** WEIGHT_BITS)) for i in ids]
     return Dist(ids=ids, W=W)
 
 
@@ -106,7 +107,7 @@ def greedy_dist(logits: Sequence[float]) -> Dist:
 
 
 def draw(d: Dist, U: int) -> int:
-    """R-S3: inverse-CDF draw over the sorted order with a 53-bit integer uniform."""
+    """R-S3: inverse-CDF draw over the listed order with a 53-bit integer uniform."""
     lhs = U * d.S
     c = 0
     for x, w in zip(d.ids, d.W):
@@ -122,7 +123,7 @@ def accept(p: Dist, q: Dist, d: int, U: int) -> bool:
 
 
 def residual_weights(p: Dist, q: Dist):
-    """R-S5 weights: (p's ids in sampling order, N_x, R), N_x / R = normalise(max(0, p - q))."""
+    """R-S5 weights: (p's ids in its listed order, N_x, R), N_x / R = normalise(max(0, p - q))."""
     xs = list(p.ids)
     n = [max(0, p.weight(x) * q.S - q.weight(x) * p.S) for x in xs]
     return xs, n, sum(n)

@@ -72,8 +72,8 @@ def test_weights_two_entry_closed_form():
     T = 0.9
     d = topk_dist(l, 2, T)
     Tf = float(np.float32(T))
-    assert d.ids == [1, 0]
-    assert d.W[0] == 2 ** 24                                 # the maximum has e = 1 exactly
+    assert d.ids == [0, 1]                                   # listed in ascending id order
+    assert d.weight(1) == 2 ** 24                            # the maximum has e = 1 exactly
     p1 = 1.0 / (1.0 + math.exp((0.25 - 1.5) / Tf))
     assert abs(d.prob(1) - p1) < 1e-6
     assert d.frac(0) + d.frac(1) == 1 and d.frac(7) == 0
@@ -85,7 +85,7 @@ def test_weights_follow_temperature_softmax():
     d = topk_dist(l, 8, 0.5)
     ids = np.argsort(-l.astype(np.float64), kind="stable")[:8]
     w = np.exp((l[ids].astype(np.float64) - l[ids[0]]) / float(np.float32(0.5)))
-    assert d.ids == list(ids)
+    assert d.ids == sorted(int(i) for i in ids)
     assert np.allclose([d.prob(i) for i in ids], w / w.sum(), rtol=2e-6, atol=0)
     assert sum(d.frac(i) for i in range(64)) == 1
 
@@ -94,8 +94,12 @@ def test_weights_are_floor_of_scaled_exp32():
     l = np.array([3.0, 1.0, -2.0, 0.5], dtype=np.float32)
     d = topk_dist(l, 4, 1.3)
     T = np.float32(1.3)
-    z = [l[i] / T for i in d.ids]
-    assert d.W == [math.floor(float(exp32(zi - z[0])) * 2 ** 24) for zi in z]
+    assert d.ids == [0, 1, 2, 3]
+    z_max = l[0] / T
+    assert d.W == [math.floor(float(exp32(l[i] / T - z_max)) * 2 ** 24) for i in d.ids]
+    # ties at the boundary: the lower ids are kept, then listed ascending
+    t = topk_dist(np.array([1.0, 2.0, 1.0, 1.0, 0.0], dtype=np.float32), 3, 1.0)
+    assert t.ids == [0, 1, 2]
 
 
 # ---- draws and acceptance ---------------------------------------------------------------
