@@ -79,6 +79,23 @@ __global__ void to_f32_kernel(const uint8_t* src, int wdtype, long long n, float
                                        : reinterpret_cast<const float*>(src)[i];
 }
 
+// LMH_P b_j for j = 1..K from the row-major head (one warp per output): the offsets'
+// additive share of the draft logits, LMH_P (h + b_j) = LMH_P h + LMH_P b_j.
+__global__ void head_bias_kernel(const uint8_t* head, const float* offsets, int K, int V, int H, int wdtype,
+                                 float* out) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= K * V) return;
+  const int j = warp / V, id = warp % V;
+  float acc = 0.f;
+  for (int k = lane; k < H; k += 32) {
+    const float w = wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(head)[(size_t)id * H + k])
+                                              : reinterpret_cast<const float*>(head)[(size_t)id * H + k];
+    acc += w * offsets[(size_t)j * H + k];
+  }
+  for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+  if (lane == 0) out[(size_t)j * V + id] = acc;
+}
+
 __global__ void rope_kernel(float2* rope, int D, double base) {
   const int half = D / 2;
   for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < kMaxPos * half; idx += gridDim.x * blockDim.x) {
@@ -159,13 +176,12 @@ __global__ void __launch_bounds__(kConsumerThreads) accept_logits_kernel(FramePa
   }
   __threadfence();
   consumer_sync();
-  ResidualScratch& rs = *reinterpret_cast<ResidualScratch*>(smem_raw);
   if (threadIdx.x < 32) {
     int drafts[kMaxDraft + 1];
     for (int i = 0; i < n_d; ++i) drafts[i] = draft_ids[i];
     AcceptResult r = warp_accept(
         a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(recs + i); },
-        [&](int i) { return (const TopkRec*)(recs + kMaxRows + i); }, p.seed, p.stream_id, p.frame_idx, call, rs);
+        [&](int i) { return (const TopkRec*)(recs + kMaxRows + i); }, p.seed, p.stream_id, p.frame_idx, call);
     if (threadIdx.x == 0) {
       for (int t = 0; t < r.n_emit; ++t) emitted[t] = r.emitted[t];
       out2[0] = r.n_acc;
@@ -202,9 +218,10 @@ __global__ void __launch_bounds__(kConsumerThreads) draft_sample_kernel(FramePar
   block_topk(z + (size_t)(j - 1) * p.V, p.V, p.top_k, p.T, p.draft_mode == MCD_DRAFT_GREEDY, ts, r);
   consumer_sync();
   __threadfence_block();
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {
     const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, pos_k + j, PURPOSE_DRAFT);
-    draft_ids[j - 1] = seq_draw(r, U);
+    const int d = warp_draw(r, U);
+    if (threadIdx.x == 0) draft_ids[j - 1] = d;
   }
   for (int i = threadIdx.x; i < p.top_k; i += kConsumerThreads) {
     if (q_ids) q_ids[(size_t)(j - 1) * p.top_k + i] = i < r->n ? r->ids[i] : -1;
@@ -408,6 +425,9 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.final_norm = p.k_norm + (size_t)p.L * p.D;
   p.offsets = p.final_norm + p.H;
 
+  float* head_bias = nullptr;
+  if ((e = ctx_alloc(c, &head_bias, sizeof(float) * (size_t)p.P * Kd * p.V)) != cudaSuccess) return fail(cuda_status(e));
+  p.head_bias = head_bias;
   float2* rope = nullptr;
   if ((e = ctx_alloc(c, &rope, sizeof(float2) * kMaxPos * (p.D / 2))) != cudaSuccess) return fail(cuda_status(e));
   p.rope = rope;
@@ -560,6 +580,12 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
   }
   conv("final_norm", H, p.final_norm);
   for (int j = 1; j <= Kd; ++j) conv("offset." + std::to_string(j), H, p.offsets + (size_t)(j - 1) * H);
+  for (int P = 1; P <= p.P && p.K > 0; ++P) {
+    const int warps = p.K * p.V;
+    head_bias_kernel<<<(warps * 32 + 255) / 256, 256, 0, c->stream>>>(
+        S("head." + std::to_string(P)), p.offsets, p.K, p.V, p.H, p.wdtype,
+        const_cast<float*>(p.head_bias) + (size_t)(P - 1) * p.K * p.V);
+  }
   for (int P = 1; P <= p.P; ++P) {
     RowSrc rh{};
     rh.seg[0] = S("head." + std::to_string(P));

@@ -5,21 +5,22 @@
 // Per call (a "round"): the rows [c_a, d_{a+1}, ..., d_{a+n}] (first call: [cond, c0]) go
 // through the MultiCodeDecoder (5 pre-norm layers: RMSNorm -> QKV -> QK-norm -> RoPE ->
 // causal GQA attention over the per-frame KV cache -> Wo + residual -> RMSNorm ->
-// gate/up -> SwiGLU -> down + residual), the final RMSNorm gives h, LM head a+1+i reads
-// row i (verify) and LM head s+j reads h_s + b_j (draft of position s+j from row s).  Then
-// top-k/temperature softmax of every row, the acceptance step and the next drafts.
+// gate/up -> SwiGLU -> down + residual), the final RMSNorm gives h, LM head s reads row s
+// (verify) and LM head s+j reads h_s + b_j (draft of position s+j).  Then the top-k /
+// temperature distribution of every row, the acceptance step and the next drafts.
 //
 // Work split.  Weight matrices are cut into units of <= 32 KB (see mcd_internal.cuh).
-// Unit u of the call's k-th stage goes to CTA (u + rot) mod n_cta, rot being the number of
-// units of all earlier stages, so every CTA streams about the same bytes.  In each CTA a
+// Unit u of a backbone stage goes to CTA (u + rot) mod n_cta, rot being the number of units
+// of all earlier stages, so every CTA streams about the same bytes; the LM-head stage hands
+// each CTA a contiguous block of units so that a CTA mostly reads one head.  In each CTA a
 // producer warp issues 1-D bulk copies (cp.async.bulk, evict-first) of its units into a
 // 4-slot shared-memory ring as fast as slots free up -- across stage and call boundaries --
 // while 8 consumer warps wait for the stage's inputs (a global counter reaching n_cta),
-// turn the fp32 activations into bf16 hi/lo mma operands and multiply each unit with
-// mma.m16n8k16 (weights as the 16-row A side, up to 8 activation columns as B).
-// Dependencies between stages are per-call counters; every wait is bounded by wait_ns.
-#include <cooperative_groups.h>
-
+// turn the activations into bf16 hi/lo mma operands in one pass from global memory and
+// multiply each unit with mma.m16n8k16 (weights as the 16-row A side, up to 8 activation
+// columns as B).  RMSNorm is applied as a per-column scale in the epilogue: W (x . g) / rms.
+// The draft offsets enter as precomputed logit biases: LMH_P (h + b_j) = LMH_P h + LMH_P b_j,
+// so every LM head multiplies the same operand (all rows' h).  Every wait is bounded.
 #include "mcd_internal.cuh"
 #include "mcd_sampler.cuh"
 
@@ -30,12 +31,13 @@ struct Smem {
   float* act;
   uint8_t* bfrag;
   float* red;
-  float* vec;     // norm gains / final norm + offsets of the current stage
+  float* vec;      // the current stage's norm gain
+  float* part;     // [kConsumerWarps][kMaxRows] partial sums of squares
   uint64_t* full;
   uint64_t* empty;
-  int* flags;     // [0] stop, [1] abort, [2] last-arriver, [3] cur head/chunk
-  float* inv_rms; // [kMaxRows]
-  int* call_info; // snapshot of the call's state
+  int* flags;      // [0] stop, [1] abort, [2] last-arriver, [3] current head / chunk
+  float* inv_rms;  // [kMaxRows]
+  int* call_info;  // snapshot of the call's state
 };
 
 constexpr int kRingOff = 0;
@@ -43,8 +45,9 @@ constexpr int kActOff = kRingOff + kNumSlots * kSlotBytes;
 constexpr int kBfragOff = kActOff + kActBytes;
 constexpr int kRedOff = kBfragOff + kBfragBytes;
 constexpr int kVecOff = kRedOff + 2 * kRedBytes;
-constexpr int kVecFloats = 6 * 1024;   // final norm + up to 5 offset vectors of hidden <= 1024
-constexpr int kBarOff = kVecOff + kVecFloats * 4;
+constexpr int kVecFloats = 1024;
+constexpr int kPartOff = kVecOff + kVecFloats * 4;
+constexpr int kBarOff = kPartOff + kConsumerWarps * kMaxRows * 4;
 constexpr int kFlagOff = kBarOff + 2 * kNumSlots * 8;
 constexpr int kRmsOff = kFlagOff + 64;
 constexpr int kInfoOff = kRmsOff + 64;
@@ -62,6 +65,7 @@ __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   s.bfrag = base + kBfragOff;
   s.red = reinterpret_cast<float*>(base + kRedOff);
   s.vec = reinterpret_cast<float*>(base + kVecOff);
+  s.part = reinterpret_cast<float*>(base + kPartOff);
   s.full = reinterpret_cast<uint64_t*>(base + kBarOff);
   s.empty = s.full + kNumSlots;
   s.flags = reinterpret_cast<int*>(base + kFlagOff);
@@ -93,10 +97,18 @@ __device__ __forceinline__ const uint8_t* unit_src(const FrameParams& p, int si,
   return base + (long long)layer * g.stride + (long long)u * g.unit_bytes;
 }
 
-__device__ __forceinline__ int first_unit(int cta, int rot, int n_cta) {
-  int f = cta - rot;
-  f %= n_cta;
-  return f < 0 ? f + n_cta : f;
+// Units [first, end) step `step` of stage si for this CTA: strided with rotation for the
+// backbone, one contiguous block for the LM heads.
+struct UnitRange {
+  int first, end, step;
+};
+__device__ __forceinline__ UnitRange unit_range(int si, int L, int n, int cta, int rot, int n_cta) {
+  if (stage_kind(si, L) == MAT_HEAD) {
+    return UnitRange{(int)(((long long)cta * n) / n_cta), (int)(((long long)(cta + 1) * n) / n_cta), 1};
+  }
+  int f = (cta - rot) % n_cta;
+  if (f < 0) f += n_cta;
+  return UnitRange{f, n, n_cta};
 }
 
 // heads touched by a call: P_lo = a+1, P_hi = min(n_pos, last row position + K)
@@ -138,7 +150,8 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
       }
       const int n = stage_units(p, si, n_heads);
       const uint32_t bytes = (uint32_t)p.g[stage_kind(si, p.L)].unit_bytes;
-      for (int u = first_unit(cta, rot, n_cta); u < n; u += n_cta) {
+      const UnitRange ur = unit_range(si, p.L, n, cta, rot, n_cta);
+      for (int u = ur.first; u < ur.end; u += ur.step) {
         const uint32_t slot = issued % kNumSlots;
         if (issued >= (uint32_t)kNumSlots) {
           if (!wait_mbar(&sm.empty[slot], ((issued / kNumSlots) - 1u) & 1u, p.err, p.wait_ns, stop)) {
@@ -181,27 +194,6 @@ struct Cons {
   __device__ Cons(const FrameParams& pp, Smem& s) : p(pp), sm(s), seq(0), buf(0), rot(0), abort_(false) {}
 };
 
-__device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned target) {
-  if (threadIdx.x == 0) {
-    bool ok = wait_counter(ctr, target, c.p.err, c.p.wait_ns);
-    if (!ok) c.sm.flags[1] = 1;
-  }
-  consumer_sync();
-  if (*(volatile int*)&c.sm.flags[1]) c.abort_ = true;
-  return !c.abort_;
-}
-
-__device__ __forceinline__ void timeline_max(const Cons& c, int call, int idx);
-__device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call = 0, int slot = -1) {
-  consumer_sync();
-  if (slot >= 0) timeline_max(c, call, slot);
-  if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(ctr, 1u);
-  }
-  if (slot >= 0) timeline_max(c, call, slot + 1);
-}
-
 // Optional profiling stamps (%globaltimer, ns), 128 per call.  Slots: 0 call start;
 // 1 top-k inputs ready; 2 top-k done (CTA 0); 3 top-k done (last CTA); 4..7 acceptance
 // start / records staged / decided / end.  Stage s (0..4L, 4l+k = layer l step k, 4L =
@@ -217,43 +209,100 @@ __device__ __forceinline__ void timeline_max(const Cons& c, int call, int idx) {
     atomicMax(c.p.timeline + call * kTimelineSlots + idx, (unsigned long long)globaltimer());
 }
 
-// Activation operand: bf16 weights -> hi/lo bf16 B fragments; fp32 weights -> fp32 rows.
-// `val(n, k)` gives the fp32 activation of column n (n < ncols) at input index k.
-template <int WT, class F>
-__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, F val) {
-  const int tid = threadIdx.x;
-  if (WT == MCD_WEIGHT_BF16) {
-    uint4* bf = reinterpret_cast<uint4*>(c.sm.bfrag);
-    const int total = (Kdim / 16) * 32;
-    for (int idx = tid; idx < total; idx += kConsumerThreads) {
-      const int kt = idx >> 5, ln = idx & 31, n = ln >> 2, t = ln & 3;
-      uint4 o = make_uint4(0u, 0u, 0u, 0u);
-      if (n < ncols) {
-        const int k0 = kt * 16 + 2 * t;
-        uint32_t h0, l0, h1, l1, h2, l2, h3, l3;
-        split_bf16(val(n, k0), h0, l0);
-        split_bf16(val(n, k0 + 1), h1, l1);
-        split_bf16(val(n, k0 + 8), h2, l2);
-        split_bf16(val(n, k0 + 9), h3, l3);
-        o.x = h0 | (h1 << 16);
-        o.y = h2 | (h3 << 16);
-        o.z = l0 | (l1 << 16);
-        o.w = l2 | (l3 << 16);
-      }
-      bf[idx] = o;
-    }
-  } else {
-    float* xs = reinterpret_cast<float*>(c.sm.bfrag);
-    const int total = kMaxRows * Kdim;
-    for (int idx = tid; idx < total; idx += kConsumerThreads) {
-      const int n = idx / Kdim, k = idx - n * Kdim;
-      xs[idx] = n < ncols ? val(n, k) : 0.0f;
-    }
+__device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned target) {
+  if (threadIdx.x == 0) {
+    bool ok = wait_counter(ctr, target, c.p.err, c.p.wait_ns);
+    if (!ok) c.sm.flags[1] = 1;
   }
   consumer_sync();
+  if (*(volatile int*)&c.sm.flags[1]) c.abort_ = true;
+  return !c.abort_;
 }
 
-// Multiply the unit in ring slot `slot` with the prepared operand; partial sums of every
+__device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call, int slot) {
+  consumer_sync();
+  timeline_max(c, call, slot);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(ctr, 1u);
+  }
+  timeline_max(c, call, slot + 1);
+}
+
+// Activation operand in one pass.  `ld(n, k)` returns elements (k, k+1) of column n
+// (n < ncols) from global or shared memory; `gain` (shared, may be null) multiplies them
+// per input index; with want_ss the per-column 1/rms of the raw values lands in inv_rms.
+// bf16 weights get hi/lo bf16 B fragments of mma.m16n8k16 (entry (kt, lane): column
+// lane/4, inputs kt*16 + 2(lane%4) + {0,1,8,9}); fp32 weights get fp32 rows [8][Kdim].
+// Every load of a thread is issued before any of its stores (one memory round trip).
+template <int WT, class Ld>
+__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, const float* gain, bool want_ss, Ld ld) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int n = lane >> 2, t = lane & 3;
+  const int total = (Kdim / 16) * 32;              // entries; Kdim <= 1024 -> at most 8 per thread
+  constexpr int kE = 8;
+  float2 va[kE], vb[kE];
+#pragma unroll
+  for (int e = 0; e < kE; ++e) {
+    const int idx = tid + e * kConsumerThreads;
+    if (idx < total && n < ncols) {
+      const int k0 = (idx >> 5) * 16 + 2 * t;
+      va[e] = ld(n, k0);
+      vb[e] = ld(n, k0 + 8);
+    } else {
+      va[e] = make_float2(0.f, 0.f);
+      vb[e] = make_float2(0.f, 0.f);
+    }
+  }
+  float ss = 0.f;
+#pragma unroll
+  for (int e = 0; e < kE; ++e) {
+    const int idx = tid + e * kConsumerThreads;
+    if (idx < total) {
+      const int k0 = (idx >> 5) * 16 + 2 * t;
+      float x0 = va[e].x, x1 = va[e].y, x2 = vb[e].x, x3 = vb[e].y;
+      ss += x0 * x0 + x1 * x1 + x2 * x2 + x3 * x3;
+      if (gain) {
+        x0 *= gain[k0];
+        x1 *= gain[k0 + 1];
+        x2 *= gain[k0 + 8];
+        x3 *= gain[k0 + 9];
+      }
+      if (WT == MCD_WEIGHT_BF16) {
+        uint32_t h0, l0, h1, l1, h2, l2, h3, l3;
+        split_bf16(x0, h0, l0);
+        split_bf16(x1, h1, l1);
+        split_bf16(x2, h2, l2);
+        split_bf16(x3, h3, l3);
+        reinterpret_cast<uint4*>(c.sm.bfrag)[idx] =
+            make_uint4(h0 | (h1 << 16), h2 | (h3 << 16), l0 | (l1 << 16), l2 | (l3 << 16));
+      } else {
+        float* xs = reinterpret_cast<float*>(c.sm.bfrag) + n * Kdim + k0;
+        xs[0] = x0;
+        xs[1] = x1;
+        xs[8] = x2;
+        xs[9] = x3;
+      }
+    }
+  }
+  if (want_ss) {
+    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 1);
+    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 2);
+    if (t == 0) c.sm.part[warp * kMaxRows + n] = ss;
+  }
+  consumer_sync();
+  if (want_ss) {
+    if (tid < kMaxRows) {
+      float s = 0.f;
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; ++w) s += c.sm.part[w * kMaxRows + tid];  // fixed order
+      c.sm.inv_rms[tid] = rsqrtf(s / (float)Kdim + c.p.eps);
+    }
+    consumer_sync();
+  }
+}
+
+// Multiply the unit in ring slot `slotp` with the prepared operand; partial sums of every
 // (m-tile, k-group) land in the reduction buffer in mma C-fragment order.
 template <int WT>
 __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_t* slotp, int Kdim) {
@@ -308,26 +357,26 @@ __device__ __forceinline__ float red_get(const Cons& c, const MatGeom& g, int mi
   const float* red = c.sm.red + c.buf * (kRedBytes / 4);
   const int ln = (rr & 7) * 4 + (n >> 1), idx = (rr >> 3) * 2 + (n & 1);
   float v = 0.f;
+#pragma unroll 8
   for (int kg = 0; kg < Gk; ++kg) v += red[((kg * g.Mu + mi) * 32 + ln) * 4 + idx];
   return v;
 }
 
-// Run every unit of stage `si` assigned to this CTA.  prep(u) prepares the operand for
-// unit u when needed; epi(u, mi, rr, n, value) consumes outputs.
+// Run every unit of stage `si` assigned to this CTA.  prep(u) runs before the unit's
+// weights are awaited (operand changes, prefetches); epi(u, mi, rr, n) consumes outputs.
 template <int WT, class Prep, class Epi>
-__device__ __forceinline__ void run_stage(Cons& c, int si, int n_units, int Kdim, Prep prep, Epi epi,
-                                          bool pairs_rows = false, int call = 0) {
+__device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, Prep prep, Epi epi,
+                                          bool pairs_rows = false) {
   const FrameParams& p = c.p;
   const MatGeom& g = p.g[stage_kind(si, p.L)];
   const int lane = threadIdx.x & 31;
   timeline(c, call, 8 + 4 * si);
   bool first = true;
-  for (int u = first_unit(blockIdx.x, c.rot, p.n_cta); u < n_units; u += p.n_cta) {
+  const UnitRange ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
+  for (int u = ur.first; u < ur.end; u += ur.step) {
     prep(u);
     const uint32_t slot = c.seq % kNumSlots;
-    if (!wait_mbar(&c.sm.full[slot], (c.seq / kNumSlots) & 1u, p.err, p.wait_ns, nullptr)) {
-      c.sm.flags[1] = 1;
-    }
+    if (!wait_mbar(&c.sm.full[slot], (c.seq / kNumSlots) & 1u, p.err, p.wait_ns, nullptr)) c.sm.flags[1] = 1;
     if (first) timeline(c, call, 9 + 4 * si);
     first = false;
     consumer_sync();
@@ -340,73 +389,29 @@ __device__ __forceinline__ void run_stage(Cons& c, int si, int n_units, int Kdim
     if (lane == 0) mbar_arrive(&c.sm.empty[slot]);
     ++c.seq;
     consumer_sync();
-    const int outs = g.Mu * (pairs_rows ? 64 : 128);
-    for (int o = threadIdx.x; o < outs; o += kConsumerThreads) {
-      const int per = pairs_rows ? 64 : 128;
+    const int per = pairs_rows ? 64 : 128;
+    for (int o = threadIdx.x; o < g.Mu * per; o += kConsumerThreads) {
       const int mi = o / per, r = o % per;
-      const int rr = r >> 3, n = r & 7;
-      epi(u, mi, rr, n);
+      epi(u, mi, r >> 3, r & 7);
     }
     c.buf ^= 1;
   }
   c.rot = (c.rot + n_units) % p.n_cta;
 }
 
-__device__ __forceinline__ float bf16_or_f32(const uint8_t* base, long long idx, int wdtype) {
-  if (wdtype == MCD_WEIGHT_BF16) return bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(base)[idx]);
-  return reinterpret_cast<const float*>(base)[idx];
-}
-
-// Rows of the residual stream into act[n][H] and per-row 1/rms into inv_rms.
-__device__ __forceinline__ void rows_rms(Cons& c, int n_rows, int H) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (warp < n_rows) {
-    float ss = 0.f;
-    for (int k = lane; k < H; k += 32) {
-      const float v = c.sm.act[warp * H + k];
-      ss += v * v;
-    }
-#pragma unroll
-    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, o);
-    if (lane == 0) c.sm.inv_rms[warp] = rsqrtf(ss / (float)H + c.p.eps);
-  }
-  consumer_sync();
-}
-
-// Copy n_rows rows of `len` floats (src row stride `ld`) into dst[n][len] with 16-byte
-// loads, four in flight per thread (every address is independent: one L2 round trip).
-__device__ __forceinline__ void g2s_rows(float* dst, const float* src, int n_rows, int len, long long ld) {
-  const int per = len >> 2, n4 = n_rows * per;
-  float4* d = reinterpret_cast<float4*>(dst);
-  for (int i = threadIdx.x; i < n4; i += 4 * kConsumerThreads) {
-    float4 v[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = i + u * kConsumerThreads;
-      if (j < n4) v[u] = __ldcg(reinterpret_cast<const float4*>(src + (long long)(j / per) * ld) + (j % per));
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = i + u * kConsumerThreads;
-      if (j < n4) d[j] = v[u];
-    }
-  }
-}
-
-// Read-only vector (weights) into shared memory; no barrier (the caller syncs later).
+// Read-only vector (weights) into shared memory; no barrier (a later barrier orders it).
 __device__ __forceinline__ void g2s_vec(float* dst, const float* src, int n) {
   const int n4 = n >> 2;
   for (int i = threadIdx.x; i < n4; i += kConsumerThreads)
     reinterpret_cast<float4*>(dst)[i] = __ldg(reinterpret_cast<const float4*>(src) + i);
 }
 
-__device__ __forceinline__ void load_x(Cons& c, int n_rows) {
-  g2s_rows(c.sm.act, c.p.x, n_rows, c.p.H, c.p.H);
-  consumer_sync();
-}
+__device__ __forceinline__ float2 ld_global2(const float* q) { return __ldcg(reinterpret_cast<const float2*>(q)); }
+__device__ __forceinline__ float2 ld_shared2(const float* q) { return *reinterpret_cast<const float2*>(q); }
 
-// Layer-0 input rows of the call: [cond, c0] on the first call, else embeddings of
-// [c_a, d_{a+1}, ...] (table of position a+i).  CTA 0 also seeds the residual stream.
+// Layer-0 input rows of the call into act[n][H]: [cond, c0] on the first call, else the
+// embeddings of [c_a, d_{a+1}, ...] (table of position a+i).  CTA 0 also seeds the residual
+// stream x in global memory.
 __device__ void gather_inputs(Cons& c) {
   const FrameParams& p = c.p;
   const int* ci = c.sm.call_info;
@@ -456,15 +461,15 @@ __device__ void gather_inputs(Cons& c) {
 
 // Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
 // per-frame cache plus the new rows).  Scratch spans act + bfrag (64 KB): the kv head's
-// cached rows are staged in shared memory first, so every dot product reads smem.  The o
-// rows land in act[0..n_rows) x D; the new K/V rows are written to the cache if write_kv.
+// cached rows are staged in shared memory with all loads in flight at once, so every dot
+// product reads shared memory.  The o rows land in act[0..n_rows) x D; the new K/V rows are
+// written to the cache if write_kv.
 __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const FrameParams& p = c.p;
   const int* ci = c.sm.call_info;
   const int n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
   const int D = p.D, group = p.NH / p.NKV, g = h / group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int npos_all = pos0 + n_rows;          // keys 0..pos0+n_rows-1
   float* o = c.sm.act;                         // [8][D]
   float* qs = o + kMaxRows * 128;              // [8][D]
   float* ks = qs + kMaxRows * 128;             // [kMaxPos][D]: cached rows, then the new rows
@@ -476,30 +481,35 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const float* kc = p.kcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
   const float* vc = p.vcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
-  // one round of independent 16-byte loads: q/k/v of the call, cached K/V, QK-norm gains
   {
     const int per = D >> 2;
     const int nq = n_rows * per, nc = pos0 * per;
-    const int total = 3 * nq + 2 * nc + (p.qk_norm ? 2 * per : 0);
-    for (int i = tid; i < total; i += kConsumerThreads) {
-      float4 v;
-      float* dst;
+    const int total = 3 * nq + 2 * nc + (p.qk_norm ? 2 * per : 0);   // <= 8 per thread
+    constexpr int kL = 8;
+    float4 v[kL];
+    float* dst[kL];
+#pragma unroll
+    for (int u = 0; u < kL; ++u) {
+      const int i = tid + u * kConsumerThreads;
+      dst[u] = nullptr;
       if (i < 3 * nq) {
         const int w = i / nq, r = i - w * nq, n = r / per, d4 = r - n * per;
         const float* row = p.qkv + (size_t)n * p.qkv_dim + (w == 0 ? qoff : w == 1 ? koff : voff);
-        v = __ldcg(reinterpret_cast<const float4*>(row) + d4);
-        dst = (w == 0 ? qs + n * D : w == 1 ? ks + (pos0 + n) * D : vs + (pos0 + n) * D) + 4 * d4;
+        v[u] = __ldcg(reinterpret_cast<const float4*>(row) + d4);
+        dst[u] = (w == 0 ? qs + n * D : w == 1 ? ks + (pos0 + n) * D : vs + (pos0 + n) * D) + 4 * d4;
       } else if (i < 3 * nq + 2 * nc) {
         const int r = i - 3 * nq, w = r / nc, rr = r - w * nc, j = rr / per, d4 = rr - j * per;
-        v = __ldcg(reinterpret_cast<const float4*>((w == 0 ? kc : vc) + (size_t)j * D) + d4);
-        dst = (w == 0 ? ks : vs) + j * D + 4 * d4;
-      } else {
+        v[u] = __ldcg(reinterpret_cast<const float4*>((w == 0 ? kc : vc) + (size_t)j * D) + d4);
+        dst[u] = (w == 0 ? ks : vs) + j * D + 4 * d4;
+      } else if (i < total) {
         const int r = i - 3 * nq - 2 * nc, w = r / per, d4 = r - w * per;
-        v = __ldg(reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D) + d4);
-        dst = (w == 0 ? gq : gk) + 4 * d4;
+        v[u] = __ldg(reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D) + d4);
+        dst[u] = (w == 0 ? gq : gk) + 4 * d4;
       }
-      *reinterpret_cast<float4*>(dst) = v;
     }
+#pragma unroll
+    for (int u = 0; u < kL; ++u)
+      if (dst[u]) *reinterpret_cast<float4*>(dst[u]) = v[u];
   }
   consumer_sync();
   float* knew = ks + pos0 * D;
@@ -549,15 +559,19 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   if (warp < n_rows) {
     const int n = warp, npos = pos0 + n + 1;
     const int kq = lane >> 2, dq = lane & 3, dl = D / 4;
-    const float* qv = qs + n * D + dq * dl;
+    const float4* qv = reinterpret_cast<const float4*>(qs + n * D + dq * dl);
     float sc[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int j = kq + 8 * i;
       float acc = 0.f;
       if (j < npos) {
-        const float* kv = ks + j * D + dq * dl;
-        for (int d = 0; d < dl; ++d) acc += qv[d] * kv[d];
+        const float4* kv = reinterpret_cast<const float4*>(ks + j * D + dq * dl);
+#pragma unroll 8
+        for (int d = 0; d < dl / 4; ++d) {
+          const float4 a = qv[d], b = kv[d];
+          acc += a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w;
+        }
       }
       acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
       acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 2);
@@ -579,29 +593,21 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
       for (int i = 0; i < 4; ++i) pr[n * kMaxPos + kq + 8 * i] = e[i] / sum;
     }
     __syncwarp();
-    for (int d = lane; d < D; d += 32) {
-      float acc = 0.f;
-      for (int j = 0; j < npos; ++j) acc += pr[n * kMaxPos + j] * vs[j * D + d];
-      o[n * D + d] = acc;
+    // o[n] = sum_j pr_j v_j: lane owns D/32 consecutive dims
+    const int dpl = D / 32;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int j = 0; j < npos; ++j) {
+      const float a = pr[n * kMaxPos + j];
+      const float* vr = vs + j * D + lane * dpl;
+#pragma unroll
+      for (int d = 0; d < 4; ++d)
+        if (d < dpl) acc[d] += a * vr[d];
     }
+#pragma unroll
+    for (int d = 0; d < 4; ++d)
+      if (d < dpl) o[n * D + lane * dpl + d] = acc[d];
   }
-  (void)npos_all;
   consumer_sync();
-}
-
-// Columns (row n, offset j) that LM head P reads in this call, in increasing row order.
-__device__ __forceinline__ int head_columns(const FrameParams& p, const int* ci, int P, int* cn, int* cj) {
-  const int fr = ci[CI_FR], n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
-  int nc = 0;
-  for (int n = fr; n < n_rows; ++n) {
-    const int j = P - (pos0 + n);
-    if (j >= 0 && j <= p.K && nc < kMaxRows) {
-      cn[nc] = n;
-      cj[nc] = j;
-      ++nc;
-    }
-  }
-  return nc;
 }
 
 // ------------------------------------------------------------------------------------
@@ -616,103 +622,95 @@ __device__ void run_call(Cons& c, int call) {
   unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
   const int n_rows = ci[CI_NROWS];
   const unsigned N = (unsigned)p.n_cta;
+  const float* x = p.x;
+  auto from_x = [&](int n, int k) { return ld_global2(x + (size_t)n * H + k); };
 
   for (int l = 0; l < L; ++l) {
-    // ---- S1: RMSNorm -> QKV -------------------------------------------------------
+    // ---- S1: RMSNorm -> QKV  (q, k, v = W (x . g) / rms) -------------------------------
     g2s_vec(sm.vec, p.attn_norm + (size_t)l * H, H);      // independent of the wait below
     if (l == 0) {
       gather_inputs(c);
+      prep_operand<WT>(c, n_rows, H, sm.vec, true, [&](int n, int k) { return ld_shared2(sm.act + n * H + k); });
     } else {
       if (!cons_wait(c, ctr + ctr_stage(l - 1, 3), N)) return;
-      load_x(c, n_rows);
+      prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
     }
-    rows_rms(c, n_rows, H);
-    prep_operand<WT>(c, n_rows, H, [&](int n, int k) { return sm.act[n * H + k] * sm.inv_rms[n] * sm.vec[k]; });
-    run_stage<WT>(
-        c, 4 * l + 0, p.g[MAT_QKV].n_units, H, [&](int) {},
-        [&](int u, int mi, int rr, int n) {
-          const MatGeom& g = p.g[MAT_QKV];
-          const float v = red_get(c, g, mi, rr, n);
-          const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-          if (n < n_rows) p.qkv[(size_t)n * p.qkv_dim + row] = v;
-        },
-        false, call);
-    if (c.abort_) return;
+    {
+      const MatGeom& g = p.g[MAT_QKV];
+      run_stage<WT>(c, call, 4 * l + 0, g.n_units, H, [&](int) {}, [&](int u, int mi, int rr, int n) {
+        const float v = red_get(c, g, mi, rr, n) * sm.inv_rms[n];
+        const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+        if (n < n_rows) p.qkv[(size_t)n * p.qkv_dim + row] = v;
+      });
+      if (c.abort_) return;
+    }
     cons_signal(c, ctr + ctr_stage(l, 0), call, 10 + 4 * (4 * l + 0));
 
-    // ---- S2: attention (per query head) -> Wo + residual ---------------------------
+    // ---- S2: attention (per query head) -> Wo + residual --------------------------------
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
     {
       const MatGeom& g = p.g[MAT_WO];
       const int group = p.NH / p.NKV;
-      sm.flags[3] = -1;
+      if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
       run_stage<WT>(
-          c, 4 * l + 1, g.n_units, D,
+          c, call, 4 * l + 1, g.n_units, D,
           [&](int u) {
             const int h = u / g.n_mb, mb = u % g.n_mb;
-            if (sm.flags[3] != h) {
+            const bool writer = (h % group) == 0 && mb == 0;
+            if (sm.flags[3] != h || writer) {   // a CTA meets m-block 0 of a head first
               consumer_sync();
-              attention_head(c, l, h, (h % group) == 0 && mb == 0);
-              prep_operand<WT>(c, n_rows, D, [&](int n, int k) { return sm.act[n * D + k]; });
+              attention_head(c, l, h, writer);
+              prep_operand<WT>(c, n_rows, D, nullptr, false, [&](int n, int k) { return ld_shared2(sm.act + n * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
-            } else if ((h % group) == 0 && mb == 0) {
-              // a CTA meets head h's m-block 0 first, so this branch only guards the
-              // invariant that the KV writer always recomputes its rows
-              consumer_sync();
-              attention_head(c, l, h, true);
-              prep_operand<WT>(c, n_rows, D, [&](int n, int k) { return sm.act[n * D + k]; });
             }
           },
           [&](int u, int mi, int rr, int n) {
             const float v = red_get(c, g, mi, rr, n);
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
             if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
-          },
-          false, call);
+          });
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 1), call, 10 + 4 * (4 * l + 1));
 
-    // ---- S3: RMSNorm -> gate/up -> SwiGLU ------------------------------------------
+    // ---- S3: RMSNorm -> gate/up -> SwiGLU --------------------------------------------------
     g2s_vec(sm.vec, p.ffn_norm + (size_t)l * H, H);
     if (!cons_wait(c, ctr + ctr_stage(l, 1), N)) return;
-    load_x(c, n_rows);
-    rows_rms(c, n_rows, H);
+    prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
     {
-      prep_operand<WT>(c, n_rows, H, [&](int n, int k) { return sm.act[n * H + k] * sm.inv_rms[n] * sm.vec[k]; });
       const MatGeom& g = p.g[MAT_GU];
       run_stage<WT>(
-          c, 4 * l + 2, g.n_units, H, [&](int) {},
+          c, call, 4 * l + 2, g.n_units, H, [&](int) {},
           [&](int u, int mi, int rr, int n) {
             // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
-            const float gt = red_get(c, g, mi, rr, n);
-            const float up = red_get(c, g, mi, rr + 8, n);
-            const int tile = (u % g.n_mb) * g.Mu + mi;
-            const int j = tile * 8 + rr;
+            const float s = sm.inv_rms[n];
+            const float gt = red_get(c, g, mi, rr, n) * s;
+            const float up = red_get(c, g, mi, rr + 8, n) * s;
+            const int j = ((u % g.n_mb) * g.Mu + mi) * 8 + rr;
             if (n < n_rows) p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * up;
           },
-          true, call);
+          true);
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 2), call, 10 + 4 * (4 * l + 2));
 
-    // ---- S4: down + residual --------------------------------------------------------
+    // ---- S4: down + residual -------------------------------------------------------------
     if (!cons_wait(c, ctr + ctr_stage(l, 2), N)) return;
     {
       const MatGeom& g = p.g[MAT_WD];
       const int Kc = g.Ku * 16;
-      sm.flags[3] = -1;
+      if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
       run_stage<WT>(
-          c, 4 * l + 3, g.n_units, Kc,
+          c, call, 4 * l + 3, g.n_units, Kc,
           [&](int u) {
             const int kc = u / g.n_mb;
             if (sm.flags[3] != kc) {
               consumer_sync();
-              g2s_rows(sm.act, p.mbuf + (size_t)kc * Kc, n_rows, Kc, F);
-              consumer_sync();
-              prep_operand<WT>(c, n_rows, Kc, [&](int n, int k) { return sm.act[n * Kc + k]; });
+              const float* m = p.mbuf + (size_t)kc * Kc;
+              prep_operand<WT>(c, n_rows, Kc, nullptr, false,
+                               [&](int n, int k) { return ld_global2(m + (size_t)n * F + k); });
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
           },
@@ -720,66 +718,47 @@ __device__ void run_call(Cons& c, int call) {
             const float v = red_get(c, g, mi, rr, n);
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
             if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
-          },
-          false, call);
+          });
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 3), call, 10 + 4 * (4 * l + 3));
   }
 
-  // ---- S5: final RMSNorm -> verify and draft heads -------------------------------------
-  // vec = [final norm | b_1 .. b_min(K,5)]; offsets beyond the fifth are read through L1
-  const int k_sm = min(p.K, kVecFloats / H - 1);
+  // ---- S5: final RMSNorm -> verify and draft heads ---------------------------------------
+  // Column n of the operand is row n (h_n before its 1/rms); LM head P's output for row n
+  // is verify logits (j = 0) or the draft logits of offset j = P - (pos0 + n) (1 <= j <= K),
+  // whose LMH_P b_j term comes from the precomputed bias table.
   g2s_vec(sm.vec, p.final_norm, H);
-  g2s_vec(sm.vec + H, p.offsets, k_sm * H);
-  for (int i = threadIdx.x * 32; i < (p.K - k_sm) * H; i += kConsumerThreads * 32)
-    asm volatile("prefetch.global.L1 [%0];" ::"l"(p.offsets + (size_t)k_sm * H + i));
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
-  load_x(c, n_rows);
-  rows_rms(c, n_rows, H);
-  for (int idx = threadIdx.x; idx < n_rows * H; idx += kConsumerThreads) {
-    const int n = idx / H, k = idx - n * H;
-    sm.act[idx] = sm.act[idx] * sm.inv_rms[n] * sm.vec[k];
-  }
-  consumer_sync();
+  prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
   {
     const MatGeom& g = p.g[MAT_HEAD];
     const int p_lo = ci[CI_PLO], n_heads = ci[CI_PHI] - ci[CI_PLO] + 1;
-    __shared__ int cn[kMaxRows], cj[kMaxRows], ncols_sh;
-    sm.flags[3] = -1;
-    consumer_sync();
+    const int fr = ci[CI_FR], pos0 = ci[CI_POS0];
+    float bias = 0.f;   // this thread's output of the next unit: (row rr, column n) = (tid>>3, tid&7)
     run_stage<WT>(
-        c, 4 * L, n_heads * g.n_units, H,
+        c, call, 4 * L, n_heads * g.n_units, H,
         [&](int u) {
-          const int hi = u / g.n_units;
-          if (sm.flags[3] != hi) {
-            consumer_sync();
-            if (threadIdx.x == 0) {
-              ncols_sh = head_columns(p, ci, p_lo + hi, cn, cj);
-              sm.flags[3] = hi;
-            }
-            consumer_sync();
-            prep_operand<WT>(c, ncols_sh, H, [&](int col, int k) {
-              const int j = cj[col];
-              float v = sm.act[cn[col] * H + k];
-              if (j > 0) v += j <= k_sm ? sm.vec[j * H + k] : __ldg(p.offsets + (size_t)(j - 1) * H + k);
-              return v;
-            });
+          bias = 0.f;
+          const int P = p_lo + u / g.n_units, n = threadIdx.x & 7, j = P - (pos0 + n);
+          if (threadIdx.x < 128 && j >= 1 && j <= p.K && n < n_rows && n >= fr) {
+            const int id = (u % g.n_units) * g.Mu * 16 + (threadIdx.x >> 3);
+            bias = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
           }
         },
         [&](int u, int mi, int rr, int n) {
-          if (n < ncols_sh) {
-            const float v = red_get(c, g, mi, rr, n);
+          const int P = p_lo + u / g.n_units, j = P - (pos0 + n);
+          if (n >= fr && n < n_rows && j >= 0 && j <= p.K) {
+            const float v = red_get(c, g, mi, rr, n) * sm.inv_rms[n] + bias;
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
-            p.logits[((size_t)cn[n] * (kMaxDraft + 1) + cj[n]) * p.V + id] = v;
+            p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] = v;
           }
-        },
-        false, call);
+        });
     if (c.abort_) return;
   }
   cons_signal(c, ctr + ctr_heads(L), call, 10 + 4 * (4 * L));
 
-  // ---- S6: top-k / temperature softmax of every logits row -----------------------------
+  // ---- S6: top-k / temperature distribution of every logits row --------------------------
   if (!cons_wait(c, ctr + ctr_heads(L), N)) return;
   timeline(c, call, 1);
   {
@@ -834,9 +813,8 @@ __device__ void accept_step(Cons& c, int call) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
   const TopkRec* prev = p.topk + (size_t)((call + 1) & 1) * kMaxRows * (kMaxDraft + 1);
-  TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // [n_p + n_d] staged records
+  TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // staged records
   const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
-  ResidualScratch& rs = *reinterpret_cast<ResidualScratch*>(srec + 2 * kMaxRows);
   __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
   timeline(c, call, 4, true);
   stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
@@ -849,7 +827,7 @@ __device__ void accept_step(Cons& c, int call) {
     for (int i = 0; i < n_d; ++i) drafts[i] = ci[CI_IDS + 1 + i];
     AcceptResult r = warp_accept(
         a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(srec + i); },
-        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, call, rs);
+        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, call);
     if (lane == 0) {
       for (int t = 0; t < r.n_emit; ++t) s_emit[t] = r.emitted[t];
       s_nemit = r.n_emit;
@@ -861,14 +839,16 @@ __device__ void accept_step(Cons& c, int call) {
   const int a_new = a + s_nemit;
   const int m = a_new - pos0;
   const int n_next = min(p.K, p.P - a_new);
-  // draft records of row m (the row whose head emitted the last code)
+  // draft records of row m (the row whose head emitted the last code): one warp each
   stage_records(srec, n_next, p.top_k, [&](int r) { return cur + m * (kMaxDraft + 1) + 1 + r; });
   consumer_sync();
+  for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
+    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
+    const int d = warp_draw(srec + j - 1, U);
+    if (lane == 0) s_next[j - 1] = d;
+  }
+  consumer_sync();
   if (threadIdx.x == 0) {
-    for (int j = 1; j <= n_next; ++j) {
-      const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
-      s_next[j - 1] = seq_draw(srec + j - 1, U);
-    }
     s_nnext = n_next;
     DevState* st = p.st;
     for (int t = 0; t < s_nemit; ++t) {
@@ -877,6 +857,9 @@ __device__ void accept_step(Cons& c, int call) {
     }
     for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
     for (int t = 0; t < s_nemit; ++t) st->emitted_last[t] = s_emit[t];
+    const int calls = ci[CI_CALLS] + 1, heads = ci[CI_HEADS] + ci[CI_PHI] - ci[CI_PLO] + 1;
+    const int kvr = ci[CI_KVROWS] + pos0 + n_rows, rf = ci[CI_ROWSFED] + n_rows;
+    const int drafted = ci[CI_DRAFTED] + n_d, accepted = ci[CI_ACCEPTED] + s_nacc;
     st->n_emit_last = s_nemit;
     st->n_acc_last = s_nacc;
     st->a = a_new;
@@ -884,9 +867,6 @@ __device__ void accept_step(Cons& c, int call) {
     st->pos0 = a_new + 1;
     st->n_rows = min(n_next + 1, p.P - a_new);
     st->first_head_row = 0;
-    const int calls = ci[CI_CALLS] + 1, heads = ci[CI_HEADS] + ci[CI_PHI] - ci[CI_PLO] + 1;
-    const int kvr = ci[CI_KVROWS] + pos0 + n_rows, rf = ci[CI_ROWSFED] + n_rows;
-    const int drafted = ci[CI_DRAFTED] + n_d, accepted = ci[CI_ACCEPTED] + s_nacc;
     st->calls = calls;
     st->heads_read = heads;
     st->kv_rows = kvr;

@@ -93,6 +93,7 @@ struct FrameParams {
   const float* k_norm;         // [L][D]
   const float* final_norm;     // [H]
   const float* offsets;        // [K][H]
+  const float* head_bias;      // [n_pos][K][V]: LMH_P b_j, the offsets' share of the draft logits
   const uint8_t* embed;        // table i at embed + i * embed_stride (row-major, weight dtype)
   long long embed_stride;
   const float2* rope;          // [kMaxPos][D/2] (cos, sin)

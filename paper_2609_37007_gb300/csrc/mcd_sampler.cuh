@@ -4,7 +4,7 @@
 // otherwise resample from max(0, p - q) renormalised).
 //
 // A distribution is a list of integer weights (ids in sampling order, W, S = sum W):
-//   * top-k set and order: (fp32 logit desc, id asc); -0 and +0 compare equal;
+//   * top-k set: (fp32 logit desc, id asc); -0 and +0 compare equal; listed by ascending id;
 //   * z = fp32 logit / fp32 T; W_i = floor(2^24 * exp32(z_i - z_max)); p(x) = W_x / S;
 //   * draw with a 53-bit integer uniform U: first i with U*S < 2^53 * (W_0 + .. + W_i);
 //   * accept draft d iff U * Wq_d * S_p < 2^53 * Wp_d * S_q  (u < p(d)/q(d));
@@ -18,20 +18,11 @@
 namespace mcd {
 
 struct TopkScratch {
-  uint32_t keys[kMaxVocab];
-  uint32_t hist[256];
-  uint32_t cand_key[kMaxTopK];
-  int cand_id[kMaxTopK];
+  uint32_t part[2][kConsumerWarps][8];   // per-warp counts of the threshold search (double-buffered)
+  uint32_t wred[2][kConsumerWarps];      // per-warp maxima / scan totals (double-buffered)
   unsigned long long wsum[kConsumerWarps];
-  int misc[8];
-  int warp_tot[kConsumerWarps];
 };
 static_assert(sizeof(TopkScratch) <= kActBytes, "top-k scratch must fit the activation region");
-
-struct ResidualScratch {
-  unsigned long long n[kMaxTopK];
-  int x[kMaxTopK];
-};
 
 // fp32 exponential of d <= 0: Cody-Waite range reduction (Cody and Waite, "Software Manual
 // for the Elementary Functions", 1980) with ln 2 = C1 + C2, then e^r by the degree-7 Taylor
@@ -81,157 +72,209 @@ __device__ __forceinline__ float key_f32(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k ^ 0x80000000u) : ~k);
 }
 
-// Block-wide (256 consumer threads) top-k of one fp32 row into `out` (global or shared).
-// `greedy` replaces the distribution by the one-hot of its first entry.
-static __device__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
-                                  TopkScratch& s, TopkRec* out) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  for (int i = tid; i < (V >> 2); i += 2 * kConsumerThreads) {   // V % 16 == 0: two 16-byte loads in flight
-    const int i2 = i + kConsumerThreads;
-    const float4 a = __ldcg(reinterpret_cast<const float4*>(logits) + i);
-    float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (i2 < (V >> 2)) b = __ldcg(reinterpret_cast<const float4*>(logits) + i2);
-    s.keys[4 * i] = f32_key(a.x);
-    s.keys[4 * i + 1] = f32_key(a.y);
-    s.keys[4 * i + 2] = f32_key(a.z);
-    s.keys[4 * i + 3] = f32_key(a.w);
-    if (i2 < (V >> 2)) {
-      s.keys[4 * i2] = f32_key(b.x);
-      s.keys[4 * i2 + 1] = f32_key(b.y);
-      s.keys[4 * i2 + 2] = f32_key(b.z);
-      s.keys[4 * i2 + 3] = f32_key(b.w);
-    }
+// Exclusive scan of v over the 256 consumer threads in thread order; returns the prefix
+// and writes the block total to *total.  One barrier (buf selects the scratch half).
+__device__ __forceinline__ uint32_t block_exscan(uint32_t v, TopkScratch& s, int buf, uint32_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += t;
   }
-  // radix select of the k-th largest key, 8 bits per pass
-  uint32_t prefix = 0, mask = 0;
-  int krem = k;
-  int count_eq = 0;
-  for (int pass = 3; pass >= 0; --pass) {
-    const int shift = pass * 8;
-    s.hist[tid] = 0;
-    consumer_sync();
-    for (int i = tid; i < V; i += kConsumerThreads) {
-      const uint32_t key = s.keys[i];
-      if ((key & mask) == prefix) atomicAdd(&s.hist[(key >> shift) & 255u], 1u);
+  if (lane == 31) s.wred[buf][warp] = incl;
+  consumer_sync();
+  uint32_t before = 0, tot = 0;
+#pragma unroll
+  for (int w = 0; w < kConsumerWarps; ++w) {
+    const uint32_t t = s.wred[buf][w];
+    before += (w < warp) ? t : 0u;
+    tot += t;
+  }
+  *total = tot;
+  return before + incl - v;
+}
+
+// Block-wide (256 consumer threads) top-k of one fp32 row (V % 16 == 0, V <= 4096) into `out`
+// (global or shared), listed in ascending id order.  Thread t holds the keys of ids
+// 4t + 1024j + c (j < 4, c < 4) in registers.  The k-th largest key is found by a counting
+// search, 3 bits per step (seven thresholds per step, counts reduced with redux.sync, one
+// barrier per step); the set is then compacted in id order (ties at the threshold keep the
+// lowest ids).  `greedy` replaces the distribution by the one-hot of the argmax.  `dbg`, when
+// not null, receives clock64() stamps at the six phase boundaries (profiling only).
+static __device__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
+                                  TopkScratch& s, TopkRec* out, long long* dbg = nullptr) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+#define MCD_TOPK_STAMP(i) \
+  if (dbg && tid == 0) dbg[i] = clock64();
+  MCD_TOPK_STAMP(0)
+  constexpr int kJ = kMaxVocab / 1024;
+  uint32_t key[4 * kJ];
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) {
+    const int i4 = tid + kConsumerThreads * j;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    const bool ok = 4 * i4 < V;
+    if (ok) v = __ldcg(reinterpret_cast<const float4*>(logits) + i4);
+    key[4 * j + 0] = ok ? f32_key(v.x) : 0u;   // key 0 (a NaN pattern) is never counted
+    key[4 * j + 1] = ok ? f32_key(v.y) : 0u;
+    key[4 * j + 2] = ok ? f32_key(v.z) : 0u;
+    key[4 * j + 3] = ok ? f32_key(v.w) : 0u;
+  }
+  // block maximum
+  uint32_t kmax = 0;
+#pragma unroll
+  for (int e = 0; e < 4 * kJ; ++e) kmax = max(kmax, key[e]);
+  kmax = __reduce_max_sync(0xFFFFFFFFu, kmax);
+  if (lane == 0) s.wred[0][warp] = kmax;
+  consumer_sync();
+#pragma unroll
+  for (int w = 0; w < kConsumerWarps; ++w) kmax = max(kmax, s.wred[0][w]);
+  MCD_TOPK_STAMP(1)
+  // counting search: T = largest t with #(key >= t) >= k, i.e. the k-th largest key
+  // Thresholds lo + i 2^sb stay below 2^32 for every i < nthr (lo is a multiple of 2^(sb+3));
+  // the unused ones (i >= nthr in the last step) may wrap and are ignored.
+  const int nj = (V + 1023) >> 10;
+  uint32_t lo = 0;
+  int bits = 32, buf = 0;
+  while (bits > 0) {
+    const int sb = bits >= 3 ? bits - 3 : 0;
+    const int nthr = bits >= 3 ? 7 : (1 << bits) - 1;
+    uint32_t cnt[7];
+#pragma unroll
+    for (int i = 0; i < 7; ++i) {
+      const uint32_t t = lo + ((uint32_t)(i + 1) << sb);
+      uint32_t c = 0;
+#pragma unroll
+      for (int e = 0; e < 4 * kJ; ++e)
+        if ((e >> 2) < nj) c += key[e] >= t ? 1u : 0u;
+      cnt[i] = __reduce_add_sync(0xFFFFFFFFu, c);
+    }
+    if (lane < 7) {
+      uint32_t mine = cnt[0];
+#pragma unroll
+      for (int i = 1; i < 7; ++i) mine = lane == i ? cnt[i] : mine;
+      s.part[buf][warp][lane] = mine;
     }
     consumer_sync();
-    if (warp == 0) {
-      int cnt[8], tot = 0;
+    uint32_t tot = 0;
+    if (lane < nthr)
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        cnt[j] = (int)s.hist[255 - 8 * lane - j];
-        tot += cnt[j];
-      }
-      int incl = tot;
+      for (int w = 0; w < kConsumerWarps; ++w) tot += s.part[buf][w][lane];
+    const unsigned ok = __ballot_sync(0xFFFFFFFFu, lane < nthr && tot >= (uint32_t)k);
+    lo += (uint32_t)__popc(ok) << sb;
+    bits = sb;
+    buf ^= 1;
+  }
+  const uint32_t Tk = lo;
+  MCD_TOPK_STAMP(2)
+  // counts above and at the threshold
+  uint32_t c_gt = 0, c_eq = 0;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        int n = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-        if (lane >= o) incl += n;
-      }
-      int c = incl - tot;
-      if (c < krem && krem <= c + tot) {
+  for (int e = 0; e < 4 * kJ; ++e) {
+    c_gt += key[e] > Tk ? 1u : 0u;
+    c_eq += key[e] == Tk ? 1u : 0u;
+  }
+  c_gt = __reduce_add_sync(0xFFFFFFFFu, c_gt);
+  c_eq = __reduce_add_sync(0xFFFFFFFFu, c_eq);
+  if (lane == 0) {
+    s.part[buf][warp][0] = c_gt;
+    s.part[buf][warp][1] = c_eq;
+  }
+  consumer_sync();
+  uint32_t n_gt = 0, n_eq = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          if (c < krem && krem <= c + cnt[j]) {
-            s.misc[0] = 255 - 8 * lane - j;
-            s.misc[1] = c;
-            s.misc[2] = cnt[j];
-          }
-          c += cnt[j];
+  for (int w = 0; w < kConsumerWarps; ++w) {
+    n_gt += s.part[buf][w][0];
+    n_eq += s.part[buf][w][1];
+  }
+  const uint32_t krem = (uint32_t)k - n_gt;      // >= 1 threshold keys to keep, lowest ids first
+  const bool all_eq = n_eq == krem;
+  MCD_TOPK_STAMP(3)
+  // id-ordered compaction with weights
+  const float Td = T;
+  const float zmax = __fdiv_rn(key_f32(kmax), Td);
+  uint32_t base = 0, tie_base = 0;
+  unsigned long long wsum = 0;
+  int sbuf = 1;
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) {
+    if (1024 * j >= V) break;                    // block-uniform
+    bool inc[4];
+    uint32_t n_inc = 0, n_tie = 0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) n_tie += key[4 * j + c] == Tk ? 1u : 0u;
+    uint32_t tie_pre = 0;
+    if (!all_eq) {
+      uint32_t tot;
+      tie_pre = tie_base + block_exscan(n_tie, s, sbuf, &tot);
+      sbuf ^= 1;
+      tie_base += tot;
+    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const uint32_t kv = key[4 * j + c];
+      const bool eq = kv == Tk;
+      inc[c] = kv > Tk || (eq && (all_eq || tie_pre < krem));
+      tie_pre += eq ? 1u : 0u;
+      n_inc += inc[c] ? 1u : 0u;
+    }
+    uint32_t tot;
+    uint32_t pos = base + block_exscan(n_inc, s, sbuf, &tot);
+    sbuf ^= 1;
+    base += tot;
+    if (!greedy) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        if (inc[c]) {
+          const float z = __fdiv_rn(key_f32(key[4 * j + c]), Td);
+          const uint32_t w = weight24(exp32_cw(__fsub_rn(z, zmax)));
+          out->ids[pos] = 4 * (tid + kConsumerThreads * j) + c;
+          out->W[pos] = w;
+          wsum += w;
+          ++pos;
         }
       }
     }
-    consumer_sync();
-    prefix |= (uint32_t)s.misc[0] << shift;
-    mask |= 255u << shift;
-    krem -= s.misc[1];
-    count_eq = s.misc[2];
-    consumer_sync();
   }
-  const uint32_t Tk = prefix;
-  const int n_gt = k - krem;
-  if (tid == 0) {
-    s.misc[4] = 0;
-    s.misc[5] = 0;
-  }
-  consumer_sync();
-  const bool take_all_eq = (count_eq == krem);
-  for (int i = tid; i < V; i += kConsumerThreads) {
-    const uint32_t key = s.keys[i];
-    if (key > Tk) {
-      const int slot = atomicAdd(&s.misc[4], 1);
-      s.cand_key[slot] = key;
-      s.cand_id[slot] = i;
-    } else if (key == Tk && take_all_eq) {
-      const int slot = n_gt + atomicAdd(&s.misc[5], 1);
-      s.cand_key[slot] = key;
-      s.cand_id[slot] = i;
-    }
-  }
-  if (!take_all_eq) {  // the krem lowest ids among the keys equal to the threshold
-    int base = 0;
-    for (int c0 = 0; c0 < V && base < krem; c0 += kConsumerThreads) {
-      const int i = c0 + tid;
-      const bool eq = (i < V) && (s.keys[i] == Tk);
-      const unsigned bal = __ballot_sync(0xFFFFFFFFu, eq);
-      if (lane == 0) s.warp_tot[warp] = __popc(bal);
-      consumer_sync();
-      int before = 0, total = 0;
+  MCD_TOPK_STAMP(4)
+  if (greedy) {
+    // argmax, ties to the lowest id
+    uint32_t best = 0xFFFFFFFFu;
 #pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) {
-        const int t = s.warp_tot[w];
-        before += (w < warp) ? t : 0;
-        total += t;
+    for (int j = 0; j < kJ; ++j)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const uint32_t id = 4 * (tid + kConsumerThreads * j) + c;
+        if (key[4 * j + c] == kmax && (int)id < V) best = min(best, id);
       }
-      const int rank = base + before + __popc(bal & ((1u << lane) - 1u));
-      if (eq && rank < krem) {
-        s.cand_key[n_gt + rank] = Tk;
-        s.cand_id[n_gt + rank] = i;
-      }
-      base += total;
-      consumer_sync();
+    best = __reduce_min_sync(0xFFFFFFFFu, best);
+    if (lane == 0) s.wred[sbuf][warp] = best;
+    consumer_sync();
+    if (tid == 0) {
+      uint32_t b = 0xFFFFFFFFu;
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; ++w) b = min(b, s.wred[sbuf][w]);
+      out->ids[0] = (int)b;
+      out->W[0] = 1u;
+      out->S = 1ull;
+      out->n = 1;
+    }
+  } else {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) wsum += __shfl_xor_sync(0xFFFFFFFFu, wsum, o);
+    if (lane == 0) s.wsum[warp] = wsum;
+    consumer_sync();
+    if (tid == 0) {
+      unsigned long long S = 0;
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; ++w) S += s.wsum[w];
+      out->S = S;
+      out->n = k;
     }
   }
-  consumer_sync();
-  // rank sort by (key desc, id asc)
-  uint32_t mk = 0;
-  int mid = 0, rank = 0;
-  if (tid < k) {
-    mk = s.cand_key[tid];
-    mid = s.cand_id[tid];
-    for (int j = 0; j < k; ++j) {
-      const uint32_t kj = s.cand_key[j];
-      const int ij = s.cand_id[j];
-      rank += (kj > mk) || (kj == mk && ij < mid);
-    }
-  }
-  consumer_sync();
-  if (tid < k) {
-    s.cand_key[rank] = mk;
-    s.cand_id[rank] = mid;
-  }
-  consumer_sync();
-  // integer weights and their (order-free) sum
-  uint32_t w = 0;
-  if (tid < k) {
-    const float z0 = __fdiv_rn(key_f32(s.cand_key[0]), T);
-    const float z = __fdiv_rn(key_f32(s.cand_key[tid]), T);
-    w = greedy ? (tid == 0 ? 1u : 0u) : weight24(exp32_cw(__fsub_rn(z, z0)));
-    out->ids[tid] = s.cand_id[tid];
-    out->W[tid] = w;
-  }
-  unsigned long long ws = w;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) ws += __shfl_xor_sync(0xFFFFFFFFu, ws, o);
-  if (lane == 0) s.wsum[warp] = ws;
-  consumer_sync();
-  if (tid == 0) {
-    unsigned long long S = 0;
-#pragma unroll
-    for (int w2 = 0; w2 < kConsumerWarps; ++w2) S += s.wsum[w2];
-    out->S = S;
-    out->n = greedy ? 1 : k;
-  }
+  MCD_TOPK_STAMP(5)
+#undef MCD_TOPK_STAMP
 }
 
 // The record helpers read through generic pointers: the frame kernel stages records in
@@ -250,62 +293,80 @@ __device__ __forceinline__ uint32_t warp_weight(const TopkRec* r, int x) {
   return r->W[idx];
 }
 
-// Inverse-CDF draw (one thread).
-__device__ __forceinline__ int seq_draw(const TopkRec* r, unsigned long long U) {
-  const int n = r->n;
-  const U128 lhs = mul64(U, r->S);
-  unsigned long long c = 0;
-  for (int i = 0; i < n; ++i) {
-    c += r->W[i];
-    if (lt128(lhs, shl53(c))) return r->ids[i];
+// Warp-parallel inverse-CDF draw: entry i (0 <= i < n) has value v (lane L holds entries
+// 4L..4L+3 in v[0..3]); returns the first i with U * S < 2^53 * (v_0 + ... + v_i).  The
+// prefix sums are exact integers, so the result equals the sequential walk's.
+constexpr int kDrawPerLane = kMaxTopK / 32;
+__device__ __forceinline__ int warp_draw_lanes(const unsigned long long (&v)[kDrawPerLane], int n,
+                                               unsigned long long S, unsigned long long U) {
+  const int lane = threadIdx.x & 31;
+  unsigned long long tot = 0;
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) tot += v[e];
+  unsigned long long incl = tot;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long t = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane >= o) incl += t;
   }
-  return r->ids[n - 1];
+  unsigned long long c = incl - tot;
+  const U128 lhs = mul64(U, S);
+  int hit = -1;
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    c += v[e];
+    const int i = lane * kDrawPerLane + e;
+    if (hit < 0 && i < n && lt128(lhs, shl53(c))) hit = i;
+  }
+  const unsigned b = __ballot_sync(0xFFFFFFFFu, hit >= 0);
+  if (!b) return n - 1;
+  return __shfl_sync(0xFFFFFFFFu, hit, __ffs(b) - 1);
 }
 
-// Residual draw from normalise(max(0, p - q)), evaluated by a full warp.
-static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U, ResidualScratch& rs) {
+// Categorical draw from a record, evaluated by a full warp.
+__device__ __forceinline__ int warp_draw(const TopkRec* r, unsigned long long U) {
+  const int lane = threadIdx.x & 31, n = r->n;
+  unsigned long long v[kDrawPerLane];
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    const int i = lane * kDrawPerLane + e;
+    v[e] = i < n ? r->W[i] : 0ull;
+  }
+  return r->ids[warp_draw_lanes(v, n, r->S, U)];
+}
+
+// Residual draw from normalise(max(0, p - q)) over p's entries in p's order, by a full warp.
+static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U) {
   const int lane = threadIdx.x & 31;
   const int np = p->n, nq = q->n;
   const unsigned long long Sp = p->S, Sq = q->S;
-  for (int i = lane; i < np; i += 32) {
-    const int x = p->ids[i];
-    unsigned long long wq = 0;
-    for (int j = 0; j < nq; ++j)
-      if (q->ids[j] == x) {
-        wq = q->W[j];
-        break;
-      }
-    const unsigned long long a = (unsigned long long)p->W[i] * Sq, b = wq * Sp;
-    int rank = 0;
-    for (int j = 0; j < np; ++j) rank += (p->ids[j] < x);
-    rs.n[rank] = a > b ? a - b : 0ull;
-    rs.x[rank] = x;
+  int id[kDrawPerLane];
+  unsigned long long wq[kDrawPerLane], v[kDrawPerLane];
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    const int i = lane * kDrawPerLane + e;
+    id[e] = i < np ? p->ids[i] : -1;
+    wq[e] = 0;
   }
-  __syncwarp();
-  int out = 0;
-  if (lane == 0) {
-    unsigned long long R = 0;
-    for (int i = 0; i < np; ++i) R += rs.n[i];
-    if (R == 0) {
-      out = seq_draw(p, U);
-    } else {
-      const U128 lhs = mul64(U, R);
-      unsigned long long c = 0;
-      int last = rs.x[np - 1];
-      bool hit = false;
-      for (int i = 0; i < np && !hit; ++i) {
-        c += rs.n[i];
-        if (rs.n[i] > 0) last = rs.x[i];
-        if (lt128(lhs, shl53(c))) {
-          out = rs.x[i];
-          hit = true;
-        }
-      }
-      if (!hit) out = last;
-    }
+  for (int j = 0; j < nq; ++j) {       // q's entries broadcast to every lane
+    const int qid = q->ids[j];
+    const unsigned long long qw = q->W[j];
+#pragma unroll
+    for (int e = 0; e < kDrawPerLane; ++e)
+      if (id[e] == qid) wq[e] = qw;
   }
-  __syncwarp();
-  return __shfl_sync(0xFFFFFFFFu, out, 0);
+  unsigned long long R = 0;
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    const int i = lane * kDrawPerLane + e;
+    const unsigned long long a = i < np ? (unsigned long long)p->W[i] * Sq : 0ull, b = wq[e] * Sp;
+    v[e] = a > b ? a - b : 0ull;
+    R += v[e];
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) R += __shfl_xor_sync(0xFFFFFFFFu, R, o);
+  if (R == 0) return warp_draw(p, U);
+  return p->ids[warp_draw_lanes(v, np, R, U)];
 }
 
 struct AcceptResult {
@@ -319,8 +380,7 @@ struct AcceptResult {
 //   q_rec(i): draft distribution of draft i (position a+1+i), drafts[i] its id
 template <class PRow, class QRec>
 __device__ AcceptResult warp_accept(int a, int n_d, int n_pos, const int* drafts, PRow p_row, QRec q_rec,
-                                    unsigned long long seed, uint32_t stream, uint32_t frame, int call,
-                                    ResidualScratch& rs) {
+                                    unsigned long long seed, uint32_t stream, uint32_t frame, int call) {
   AcceptResult res;
   res.n_acc = 0;
   res.n_emit = 0;
@@ -337,7 +397,7 @@ __device__ AcceptResult warp_accept(int a, int n_d, int n_pos, const int* drafts
       res.n_acc++;
     } else {
       const unsigned long long U2 = uniform_U(seed, stream, frame, call, s, PURPOSE_TARGET);
-      res.emitted[res.n_emit++] = warp_residual(pr, qr, U2, rs);
+      res.emitted[res.n_emit++] = warp_residual(pr, qr, U2);
       rejected = true;
     }
   }
@@ -345,9 +405,7 @@ __device__ AcceptResult warp_accept(int a, int n_d, int n_pos, const int* drafts
     const int s = a + 1 + n_d;
     if (s <= n_pos) {
       const unsigned long long U = uniform_U(seed, stream, frame, call, s, PURPOSE_TARGET);
-      int x = 0;
-      if ((threadIdx.x & 31) == 0) x = seq_draw(p_row(n_d), U);
-      res.emitted[res.n_emit++] = __shfl_sync(0xFFFFFFFFu, x, 0);
+      res.emitted[res.n_emit++] = warp_draw(p_row(n_d), U);
     }
   }
   return res;
