@@ -28,8 +28,9 @@
  * 3 + v/2 = Gaussian pair for vocabulary entries (v, v+1) of a noisy draft row.
  * A decision uses U = (w0 >> 5) * 2^26 + (w1 >> 6) from words 0 and 1 (u = U / 2^53).
  *
- * Distributions: the top-k set of a logits row in order (fp32 logit desc, id asc) with
- * integer weights W_i = floor(2^24 * exp32(z_i - z_max)), z = fp32 logit / fp32 T, where
+ * Distributions: the top-k set of a logits row (ranked by fp32 logit desc, then id asc,
+ * and listed in ascending id order, the order draws walk) with integer weights
+ * W_i = floor(2^24 * exp32(z_i - z_max)), z = fp32 logit / fp32 T, where
  * exp32 is an fp32 exponential (Cody-Waite range reduction, degree-7 Taylor polynomial);
  * p(x) = W_x / S, S = sum W.  Draws, accept tests (u < p(d)/q(d)) and residual draws
  * (normalised max(0, p - q)) are exact integer comparisons.
@@ -138,6 +139,16 @@ mcd_status mcd_decode_frame(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx
                             const float* cond, const int32_t* c0, const float* c0_emb,
                             int32_t* codes_out, mcd_frame_stats* stats);
 
+/* mcd_decode_frame on host buffers: cond (host float [hidden]), c0 (host int32 [1]) or
+ * c0_emb (host float [hidden]) are copied to the context's device staging area, the
+ * frame is decoded, codes_out (host int32 [n_pos]) and stats (host, optional) are copied
+ * back, and the call waits for the stream before returning (pinned host memory makes the
+ * copies cheaper; pageable memory also works).  Returns the first device-side failure
+ * like mcd_sync.  The per-frame entry point of a host-driven TTS loop. */
+mcd_status mcd_decode_frame_host(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx,
+                                 const float* cond, const int32_t* c0, const float* c0_emb,
+                                 int32_t* codes_out, mcd_frame_stats* stats);
+
 /* Stepwise use of the same kernels.  mcd_begin_frame resets the per-frame state and
  * selects the (stream id, frame index) of the Philox counters; it needs no weights, so
  * the sampler hooks below can run on a context without them;
@@ -172,10 +183,12 @@ mcd_status mcd_accept_from_logits(mcd_ctx* ctx, int32_t a, int32_t n_drafts, int
                                   const float* p_logits, const float* q_logits,
                                   const int32_t* draft_ids, int32_t* emitted, int32_t* out2);
 
-/* Top-k / temperature distributions of n_rows fp32 logits rows (dev float [n_rows,
- * vocab], n_rows <= 128): ids (dev int32 [n_rows, top_k]) in sampling order (logit desc,
- * id asc), weights (dev uint32 [n_rows, top_k]) and sums (dev uint64 [n_rows]); any
- * output may be NULL. */
+/* Top-k / temperature distributions (Abstract and Sec. 3.1: the deployed top-k sampling)
+ * of n_rows fp32 logits rows (dev float [n_rows, vocab], n_rows <= 128): ids (dev int32
+ * [n_rows, top_k]) in ascending id order (the sampling order), weights (dev uint32
+ * [n_rows, top_k]) and sums (dev uint64 [n_rows]); any output may be NULL.  With
+ * draft_mode GREEDY the rows are still full top-k distributions (greedy applies to
+ * drafts only). */
 mcd_status mcd_topk_softmax(mcd_ctx* ctx, int32_t n_rows, const float* logits,
                             int32_t* ids, uint32_t* weights, uint64_t* sums);
 

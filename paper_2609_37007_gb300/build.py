@@ -18,6 +18,21 @@ FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-cudart", "sh
          "-I" + os.path.join(ROOT, "include")]
 
 
+FRAME_KERNEL_SOURCES = ["mcd_frame.cu", "mcd_internal.cuh", "mcd_sampler.cuh"]
+
+
+def source_digest(files=FRAME_KERNEL_SOURCES) -> str:
+    """sha256 over the sources the frame kernel is compiled from (names and contents):
+    identifies the kernel build that a stored profile was taken from."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in files:
+        h.update(f.encode())
+        with open(os.path.join(CSRC, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def nvcc() -> str:
     path = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
     if not os.path.exists(path):

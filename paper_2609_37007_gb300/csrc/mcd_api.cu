@@ -246,6 +246,7 @@ struct mcd_ctx {
   size_t w_bytes = 0;
   size_t off_qkv = 0, off_wo = 0, off_gu = 0, off_wd = 0, off_head = 0, off_embed = 0;
   float* f32_arena = nullptr;   // norms + offsets
+  uint8_t* host_stage = nullptr;  // device staging for mcd_decode_frame_host
   bool weights_loaded = false;
   bool frame_begun = false;
   int h_err = 0;                 // host-side sticky CUDA error
@@ -334,6 +335,14 @@ const char* mcd_status_str(mcd_status s) {
   }
   return "unknown status";
 }
+
+// Staging area of mcd_decode_frame_host: cond [H] | c0_emb [H] | c0 | codes [n_pos] | stats.
+static size_t stage_cond(const FrameParams&) { return 0; }
+static size_t stage_emb(const FrameParams& p) { return (size_t)p.H * 4; }
+static size_t stage_c0(const FrameParams& p) { return (size_t)p.H * 8; }
+static size_t stage_codes(const FrameParams& p) { return (size_t)p.H * 8 + 16; }
+static size_t stage_stats(const FrameParams& p) { return stage_codes(p) + 64; }
+static size_t host_stage_bytes(const FrameParams& p) { return stage_stats(p) + sizeof(mcd_frame_stats); }
 
 mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if (!out) return MCD_ERR_INVALID_ARG;
@@ -446,6 +455,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxCalls * p.ctr_stride)) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &c->host_stage, host_stage_bytes(p))) != cudaSuccess) return fail(cuda_status(e));
   if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.vcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -644,6 +654,32 @@ mcd_status mcd_decode_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, 
   p.n_emitted_out = nullptr;
   MCD_CHECK(launch_frame_kernel(p, c->stream));
   return MCD_OK;
+}
+
+mcd_status mcd_decode_frame_host(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
+                                 const int32_t* c0, const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats) {
+  if (!c || !codes_out || !cond) return MCD_ERR_INVALID_ARG;
+  if (!c->weights_loaded) return MCD_ERR_STATE;
+  const FrameParams& p = c->fp;
+  if (p.C0V > 0 && !c0) return MCD_ERR_INVALID_ARG;
+  if (p.C0V == 0 && !c0_emb) return MCD_ERR_INVALID_ARG;
+  uint8_t* st = c->host_stage;
+  float* d_cond = reinterpret_cast<float*>(st + stage_cond(p));
+  float* d_emb = reinterpret_cast<float*>(st + stage_emb(p));
+  int32_t* d_c0 = reinterpret_cast<int32_t*>(st + stage_c0(p));
+  int32_t* d_codes = reinterpret_cast<int32_t*>(st + stage_codes(p));
+  mcd_frame_stats* d_stats = reinterpret_cast<mcd_frame_stats*>(st + stage_stats(p));
+  MCD_CHECK(cudaMemcpyAsync(d_cond, cond, (size_t)p.H * 4, cudaMemcpyHostToDevice, c->stream));
+  if (p.C0V > 0)
+    MCD_CHECK(cudaMemcpyAsync(d_c0, c0, 4, cudaMemcpyHostToDevice, c->stream));
+  else
+    MCD_CHECK(cudaMemcpyAsync(d_emb, c0_emb, (size_t)p.H * 4, cudaMemcpyHostToDevice, c->stream));
+  mcd_status s = mcd_decode_frame(c, stream_id, frame_idx, d_cond, p.C0V > 0 ? d_c0 : nullptr,
+                                  p.C0V > 0 ? nullptr : d_emb, d_codes, d_stats);
+  if (s != MCD_OK) return s;
+  MCD_CHECK(cudaMemcpyAsync(codes_out, d_codes, (size_t)p.P * 4, cudaMemcpyDeviceToHost, c->stream));
+  if (stats) MCD_CHECK(cudaMemcpyAsync(stats, d_stats, sizeof(mcd_frame_stats), cudaMemcpyDeviceToHost, c->stream));
+  return mcd_sync(c);
 }
 
 mcd_status mcd_begin_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond, const int32_t* c0,

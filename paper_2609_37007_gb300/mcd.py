@@ -69,6 +69,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_load_weights": (I32, [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(P),
                                    ctypes.POINTER(I64)]),
         "mcd_decode_frame": (I32, [P, U32, U32, P, P, P, P, P]),
+        "mcd_decode_frame_host": (I32, [P, U32, U32, P, P, P, P, P]),
         "mcd_begin_frame": (I32, [P, U32, U32, P, P, P]),
         "mcd_verify_accept": (I32, [P, P, P, P]),
         "mcd_draft": (I32, [P, I32, I32, P, P, P, P, P]),
@@ -104,6 +105,19 @@ def _ptr(t) -> Optional[int]:
     return t.data_ptr()
 
 
+def _hptr(a) -> Optional[int]:
+    """Host buffer address: a C-contiguous numpy array or CPU torch tensor."""
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        if not a.flags["C_CONTIGUOUS"]:
+            raise ValueError("host buffers must be C-contiguous")
+        return a.ctypes.data
+    if a.is_cuda or not a.is_contiguous():
+        raise ValueError("host buffers must be contiguous CPU tensors")
+    return a.data_ptr()
+
+
 def config_struct(cfg: MCDConfig) -> McdConfig:
     return McdConfig(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn,
                      cfg.n_pos, cfg.vocab, cfg.c0_vocab, cfg.rms_eps, cfg.rope_base, cfg.qk_norm,
@@ -135,6 +149,12 @@ def mcd_load_weights(ctx, weights: Dict[str, np.ndarray]):
 def mcd_decode_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):
     _check("mcd_decode_frame", load_library().mcd_decode_frame(
         ctx, stream_id, frame_idx, _ptr(cond), _ptr(c0), _ptr(c0_emb), _ptr(codes_out), _ptr(stats)))
+
+
+def mcd_decode_frame_host(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):
+    """Host buffers (numpy arrays or CPU tensors, pinned or pageable); returns when done."""
+    _check("mcd_decode_frame_host", load_library().mcd_decode_frame_host(
+        ctx, stream_id, frame_idx, _hptr(cond), _hptr(c0), _hptr(c0_emb), _hptr(codes_out), _hptr(stats)))
 
 
 def mcd_begin_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb):
