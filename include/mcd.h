@@ -192,6 +192,32 @@ mcd_status mcd_accept_from_logits(mcd_ctx* ctx, int32_t a, int32_t n_drafts, int
 mcd_status mcd_topk_softmax(mcd_ctx* ctx, int32_t n_rows, const float* logits,
                             int32_t* ids, uint32_t* weights, uint64_t* sums);
 
+/* No-allocation variant of mcd_topk_softmax (the paper has no counterpart: it is a
+ * deployment convenience).  Some callers cannot allocate device memory when they need a
+ * distribution: a host that hands all device memory to its own pool up front, or a
+ * real-time audio thread that must not enter the CUDA allocator, which can block on
+ * locks shared with other threads.  This call needs no mcd_ctx (creating one allocates)
+ * and allocates nothing: its per-row scratch is a fixed array of
+ * MCD_STATIC_TOPK_MAX_ROWS records in the library's own device memory, so it takes at
+ * most that many rows per call.
+ *   logits   dev float [n_rows, vocab], 16-byte aligned; vocab a multiple of 16, <= 4096
+ *   ids      dev int32 [n_rows, top_k], ascending id order; weights dev uint32
+ *            [n_rows, top_k]; sums dev uint64 [n_rows]; any output may be NULL
+ *   top_k in 1..min(128, vocab); temperature > 0; cuda_stream a cudaStream_t (NULL = legacy
+ *   default stream).  Results are the ones mcd_topk_softmax gives for the same rows.
+ * Errors: MCD_ERR_INVALID_ARG for a bad pointer, alignment, vocab, top_k or temperature;
+ * MCD_ERR_UNSUPPORTED for n_rows > MCD_STATIC_TOPK_MAX_ROWS (nothing is launched) or
+ * vocab > 4096; MCD_ERR_CUDA if the set-up or the launch fails.
+ * The first call on each device (made with that device current) does a one-time set-up
+ * that looks up the scratch's device address; make it before any stream capture begins.
+ * Nothing in the scratch needs to start at zero.  The scratch is shared by every call on
+ * a device: calls whose work can overlap (other streams, other host threads) race on it,
+ * so serialise them, e.g. on one stream. */
+#define MCD_STATIC_TOPK_MAX_ROWS 128
+mcd_status mcd_topk_softmax_static(int32_t n_rows, int32_t vocab, int32_t top_k, float temperature,
+                                   const float* logits, int32_t* ids, uint32_t* weights,
+                                   uint64_t* sums, void* cuda_stream);
+
 /* Tracing for parity tests: while `trace` (dev, mcd_trace_bytes() bytes) is set, frame
  * decoding writes one mcd_call_trace per call followed, after 16 records, by float
  * logits [16 calls][8 rows][vocab] (verify rows) and [16 calls][8 drafts][vocab] (the

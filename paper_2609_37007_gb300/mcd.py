@@ -24,6 +24,7 @@ STATUS_NAMES = {0: "MCD_OK", 1: "MCD_ERR_INVALID_ARG", 2: "MCD_ERR_STATE", 3: "M
 
 MAX_CALLS = 16
 MAX_ROWS = 8
+STATIC_TOPK_MAX_ROWS = 128     # MCD_STATIC_TOPK_MAX_ROWS
 
 
 class McdConfig(ctypes.Structure):
@@ -75,6 +76,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_draft": (I32, [P, I32, I32, P, P, P, P, P]),
         "mcd_accept_from_logits": (I32, [P, I32, I32, I32, P, P, P, P, P]),
         "mcd_topk_softmax": (I32, [P, I32, P, P, P, P]),
+        "mcd_topk_softmax_static": (I32, [I32, I32, I32, ctypes.c_float, P, P, P, P, P]),
         "mcd_trace_bytes": (I64, [P]),
         "mcd_set_trace": (I32, [P, P]),
         "mcd_set_timeline": (I32, [P, P]),
@@ -182,6 +184,13 @@ def mcd_accept_from_logits(ctx, a: int, n_drafts: int, call_idx: int, p_logits, 
 def mcd_topk_softmax(ctx, n_rows: int, logits, ids, weights=None, sums=None):
     _check("mcd_topk_softmax", load_library().mcd_topk_softmax(ctx, n_rows, _ptr(logits), _ptr(ids),
                                                                 _ptr(weights), _ptr(sums)))
+
+
+def mcd_topk_softmax_static(n_rows: int, vocab: int, top_k: int, temperature: float, logits, ids,
+                            weights=None, sums=None, stream=None):
+    _check("mcd_topk_softmax_static", load_library().mcd_topk_softmax_static(
+        n_rows, vocab, top_k, temperature, _ptr(logits), _ptr(ids), _ptr(weights), _ptr(sums),
+        ctypes.c_void_p(stream.cuda_stream if stream is not None else None)))
 
 
 def mcd_trace_bytes(ctx) -> int:
