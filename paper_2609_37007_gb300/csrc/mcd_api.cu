@@ -1,6 +1,7 @@
 // C ABI of libmcd (declared in include/mcd.h): context management, weight loading and
 // re-tiling, frame decoding through the persistent frame kernel, the stepwise API and
 // the sampler parity hooks.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>

@@ -44,7 +44,7 @@ constexpr int kRingOff = 0;
 constexpr int kActOff = kRingOff + kNumSlots * kSlotBytes;
 constexpr int kBfragOff = kActOff + kActBytes;
 constexpr int kRedOff = kBfragOff + kBfragBytes;
-constexpr int kVecOff = kRedOff + 2 * kRedBytes;
+constexpr int kVecOff = kRedOff + kChunk * kRedBytes;
 constexpr int kVecFloats = 1024;
 constexpr int kPartOff = kVecOff + kVecFloats * 4;
 constexpr int kBarOff = kPartOff + kConsumerWarps * kMaxRows * 4;
@@ -188,10 +188,9 @@ struct Cons {
   const FrameParams& p;
   Smem& sm;
   uint32_t seq;   // units consumed (ring sequence)
-  int buf;        // reduction buffer parity
   int rot;
   bool abort_;
-  __device__ Cons(const FrameParams& pp, Smem& s) : p(pp), sm(s), seq(0), buf(0), rot(0), abort_(false) {}
+  __device__ Cons(const FrameParams& pp, Smem& s) : p(pp), sm(s), seq(0), rot(0), abort_(false) {}
 };
 
 // Optional profiling stamps (%globaltimer, ns), 128 per call.  Slots: 0 call start;
@@ -229,70 +228,75 @@ __device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call, in
   timeline_max(c, call, slot + 1);
 }
 
-// Activation operand in one pass.  `ld(n, k)` returns elements (k, k+1) of column n
-// (n < ncols) from global or shared memory; `gain` (shared, may be null) multiplies them
-// per input index; with want_ss the per-column 1/rms of the raw values lands in inv_rms.
-// bf16 weights get hi/lo bf16 B fragments of mma.m16n8k16 (entry (kt, lane): column
-// lane/4, inputs kt*16 + 2(lane%4) + {0,1,8,9}); fp32 weights get fp32 rows [8][Kdim].
+// Activation operand in one pass.  `ld(n, k)` returns elements (k, k+1) of column n from
+// global or shared memory; `gain` (shared, may be null) multiplies them per input index;
+// with want_ss the per-column 1/rms of the raw values lands in inv_rms.  bf16 weights get
+// hi/lo bf16 B fragments of mma.m16n8k16 (entry (kt0 + kt, lane): column lane/4, inputs
+// kt*16 + 2(lane%4) + {0,1,8,9}); fp32 weights get fp32 rows [8][ldk] from column kt0*16.  Only the first
+// ncp = 2^ceil(log2 ncols) columns are written (columns >= ncols as zeros): an mma output
+// column depends only on its own B column and columns >= ncols are never read back.
 // Every load of a thread is issued before any of its stores (one memory round trip).
 template <int WT, class Ld>
-__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, const float* gain, bool want_ss, Ld ld) {
+__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
+                                             bool want_ss, Ld ld) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int n = lane >> 2, t = lane & 3;
-  const int total = (Kdim / 16) * 32;              // entries; Kdim <= 1024 -> at most 8 per thread
+  const int lg = ncols <= 1 ? 0 : ncols <= 2 ? 1 : ncols <= 4 ? 2 : 3;
+  const int n = (tid >> 2) & ((1 << lg) - 1), t = tid & 3;
+  const bool live = n < ncols;
+  const int items = (Kdim >> 4) << (2 + lg);       // (k-tile, column, t)
   constexpr int kE = 8;
+  float ss = 0.f;
+  for (int base = 0; base < items; base += kE * kConsumerThreads) {
   float2 va[kE], vb[kE];
 #pragma unroll
   for (int e = 0; e < kE; ++e) {
-    const int idx = tid + e * kConsumerThreads;
-    if (idx < total && n < ncols) {
-      const int k0 = (idx >> 5) * 16 + 2 * t;
+    const int i = base + tid + e * kConsumerThreads;
+    va[e] = make_float2(0.f, 0.f);
+    vb[e] = make_float2(0.f, 0.f);
+    if (i < items && live) {
+      const int k0 = ((i >> (2 + lg)) << 4) + 2 * t;
       va[e] = ld(n, k0);
       vb[e] = ld(n, k0 + 8);
-    } else {
-      va[e] = make_float2(0.f, 0.f);
-      vb[e] = make_float2(0.f, 0.f);
     }
   }
-  float ss = 0.f;
 #pragma unroll
   for (int e = 0; e < kE; ++e) {
-    const int idx = tid + e * kConsumerThreads;
-    if (idx < total) {
-      const int k0 = (idx >> 5) * 16 + 2 * t;
-      float x0 = va[e].x, x1 = va[e].y, x2 = vb[e].x, x3 = vb[e].y;
-      ss += x0 * x0 + x1 * x1 + x2 * x2 + x3 * x3;
+    const int i = base + tid + e * kConsumerThreads;
+    if (i < items) {
+      const int kt = i >> (2 + lg), k0 = (kt << 4) + 2 * t;
+      float2 x01 = va[e], x89 = vb[e];
+      ss += x01.x * x01.x + x01.y * x01.y + x89.x * x89.x + x89.y * x89.y;
       if (gain) {
-        x0 *= gain[k0];
-        x1 *= gain[k0 + 1];
-        x2 *= gain[k0 + 8];
-        x3 *= gain[k0 + 9];
+        const float2 g01 = *reinterpret_cast<const float2*>(gain + k0);
+        const float2 g89 = *reinterpret_cast<const float2*>(gain + k0 + 8);
+        x01.x *= g01.x;
+        x01.y *= g01.y;
+        x89.x *= g89.x;
+        x89.y *= g89.y;
       }
       if (WT == MCD_WEIGHT_BF16) {
-        uint32_t h0, l0, h1, l1, h2, l2, h3, l3;
-        split_bf16(x0, h0, l0);
-        split_bf16(x1, h1, l1);
-        split_bf16(x2, h2, l2);
-        split_bf16(x3, h3, l3);
-        reinterpret_cast<uint4*>(c.sm.bfrag)[idx] =
-            make_uint4(h0 | (h1 << 16), h2 | (h3 << 16), l0 | (l1 << 16), l2 | (l3 << 16));
+        const uint32_t h01 = pack_bf16x2(x01.x, x01.y), h89 = pack_bf16x2(x89.x, x89.y);
+        const uint32_t l01 = pack_bf16x2(x01.x - bf16_lo_f32(h01), x01.y - bf16_hi_f32(h01));
+        const uint32_t l89 = pack_bf16x2(x89.x - bf16_lo_f32(h89), x89.y - bf16_hi_f32(h89));
+        reinterpret_cast<uint4*>(c.sm.bfrag)[(kt0 + kt) * 32 + 4 * n + t] = make_uint4(h01, h89, l01, l89);
       } else {
-        float* xs = reinterpret_cast<float*>(c.sm.bfrag) + n * Kdim + k0;
-        xs[0] = x0;
-        xs[1] = x1;
-        xs[8] = x2;
-        xs[9] = x3;
+        float* xs = reinterpret_cast<float*>(c.sm.bfrag) + n * ldk + kt0 * 16 + k0;
+        *reinterpret_cast<float2*>(xs) = x01;
+        *reinterpret_cast<float2*>(xs + 8) = x89;
       }
     }
   }
+  }
   if (want_ss) {
-    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 1);
-    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 2);
-    if (t == 0) c.sm.part[warp * kMaxRows + n] = ss;
+    // lanes of one column: t (bits 0-1) and the k-tile bits above the column bits
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1)
+      if (off < 4 || off >= (4 << lg)) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+    if (lane < (4 << lg) && t == 0) c.sm.part[warp * kMaxRows + n] = ss;
   }
   consumer_sync();
   if (want_ss) {
-    if (tid < kMaxRows) {
+    if (tid < ncols) {
       float s = 0.f;
 #pragma unroll
       for (int w = 0; w < kConsumerWarps; ++w) s += c.sm.part[w * kMaxRows + tid];  // fixed order
@@ -302,27 +306,31 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, const
   }
 }
 
-// Multiply the unit in ring slot `slotp` with the prepared operand; partial sums of every
-// (m-tile, k-group) land in the reduction buffer in mma C-fragment order.
+// Multiply the unit in ring slot `slotp` with the prepared operand of k-chunk kc; the
+// warp's partial tile (its m-tile over its k-group) lands in red[r] in C-fragment order.
+// `b` caches the warp's bf16 B fragments across the units of a chunk (same k-range).
 template <int WT>
-__device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_t* slotp, int Kdim) {
+__device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_t* slotp, int Kdim, int kc, int r,
+                                         uint4 (&b)[8], bool load_b) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Mu = g.Mu, Ku = g.Ku;
   const int Gk = kConsumerWarps / Mu;
   const int mi = warp % Mu, kg = warp / Mu, kts = Ku / Gk;
-  float4* red = reinterpret_cast<float4*>(c.sm.red + c.buf * (kRedBytes / 4));
+  float4* red = reinterpret_cast<float4*>(c.sm.red + r * (kRedBytes / 4));
   if (WT == MCD_WEIGHT_BF16) {
     const uint4* A = reinterpret_cast<const uint4*>(slotp) + (size_t)(mi * Ku + kg * kts) * 32 + lane;
-    const uint4* B = reinterpret_cast<const uint4*>(c.sm.bfrag) + (size_t)(kg * kts) * 32 + lane;
+    (void)b;
+    (void)load_b;
+    const uint4* B = reinterpret_cast<const uint4*>(c.sm.bfrag) + (size_t)(kc * Ku + kg * kts) * 32 + lane;
     float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 8
     for (int t = 0; t < kts; ++t) {
       const uint4 a = A[t * 32];
-      const uint4 b = B[t * 32];
-      mma_bf16_16816(a0, a, b.x, b.y);
-      mma_bf16_16816(a1, a, b.z, b.w);
+      const uint4 bb = B[t * 32];
+      mma_bf16_16816(a0, a, bb.x, bb.y);
+      mma_bf16_16816(a1, a, bb.z, bb.w);
     }
-    red[(kg * Mu + mi) * 32 + lane] = make_float4(a0[0] + a1[0], a0[1] + a1[1], a0[2] + a1[2], a0[3] + a1[3]);
+    red[warp * 32 + lane] = make_float4(a0[0] + a1[0], a0[1] + a1[1], a0[2] + a1[2], a0[3] + a1[3]);
   } else {
     const int rr = lane & 15, kh = lane >> 4;
     const float* xs = reinterpret_cast<const float*>(c.sm.bfrag);
@@ -332,7 +340,7 @@ __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_
     for (int n = 0; n < kMaxRows; ++n) acc[n] = 0.f;
     for (int t = 0; t < kts; ++t) {
       const float4 w0 = A[t * 64], w1 = A[t * 64 + 1];
-      const int col = (kg * kts + t) * 16 + kh * 8;
+      const int col = (kc * Ku + kg * kts + t) * 16 + kh * 8;
 #pragma unroll
       for (int n = 0; n < kMaxRows; ++n) {
         const float4 x0 = *reinterpret_cast<const float4*>(xs + n * Kdim + col);
@@ -344,57 +352,81 @@ __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_
 #pragma unroll
     for (int n = 0; n < kMaxRows; ++n) acc[n] += __shfl_xor_sync(0xFFFFFFFFu, acc[n], 16);
     if (lane < 16) {
-      float* rf = reinterpret_cast<float*>(red + (kg * Mu + mi) * 32);
+      float* rf = reinterpret_cast<float*>(red + warp * 32);
 #pragma unroll
       for (int n = 0; n < kMaxRows; ++n) rf[((rr & 7) * 4 + (n >> 1)) * 4 + (rr >> 3) * 2 + (n & 1)] = acc[n];
     }
   }
 }
 
-// Sum of the k-group partials of output (mi, row rr, column n) of the current unit.
-__device__ __forceinline__ float red_get(const Cons& c, const MatGeom& g, int mi, int rr, int n) {
+// Sum over the k-group warps of output (row rr of m-tile mi, column n) of chunk unit r.
+__device__ __forceinline__ float red_sum(const Cons& c, const MatGeom& g, int r, int mi, int rr, int n) {
   const int Gk = kConsumerWarps / g.Mu;
-  const float* red = c.sm.red + c.buf * (kRedBytes / 4);
+  const float* red = c.sm.red + r * (kRedBytes / 4);
   const int ln = (rr & 7) * 4 + (n >> 1), idx = (rr >> 3) * 2 + (n & 1);
   float v = 0.f;
-#pragma unroll 8
-  for (int kg = 0; kg < Gk; ++kg) v += red[((kg * g.Mu + mi) * 32 + ln) * 4 + idx];
+#pragma unroll
+  for (int kg = 0; kg < kConsumerWarps; ++kg)
+    if (kg < Gk) v += red[((kg * g.Mu + mi) * 32 + ln) * 4 + idx];
   return v;
 }
 
-// Run every unit of stage `si` assigned to this CTA.  prep(u) runs before the unit's
-// weights are awaited (operand changes, prefetches); epi(u, mi, rr, n) consumes outputs.
-template <int WT, class Prep, class Epi>
-__device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, Prep prep, Epi epi,
-                                          bool pairs_rows = false) {
+// Run every unit of stage si assigned to this CTA.  Units are taken in chunks of up to
+// kChunk consecutive units that share one operand (opkey(u): the k-chunk / head whose B
+// operand they multiply; prep(u0, cnt, step) builds it for the chunk).  Each chunk: wait
+// for its units' weights, multiply them all, one barrier, then one epilogue pass
+// epi(u, mi, rr, n, v, v8) over the live outputs (columns n < ncols; v8 = row rr + 8 for
+// gate/up pairs).
+template <int WT, class Key, class Prep, class Epi>
+__device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, int ncols, Key opkey,
+                                          Prep prep, Epi epi, bool pairs_rows = false) {
   const FrameParams& p = c.p;
   const MatGeom& g = p.g[stage_kind(si, p.L)];
-  const int lane = threadIdx.x & 31;
   timeline(c, call, 8 + 4 * si);
-  bool first = true;
   const UnitRange ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
-  for (int u = ur.first; u < ur.end; u += ur.step) {
-    prep(u);
-    const uint32_t slot = c.seq % kNumSlots;
-    if (!wait_mbar(&c.sm.full[slot], (c.seq / kNumSlots) & 1u, p.err, p.wait_ns, nullptr)) c.sm.flags[1] = 1;
-    if (first) timeline(c, call, 9 + 4 * si);
-    first = false;
+  const int lgm = g.Mu == 1 ? 0 : g.Mu == 2 ? 1 : g.Mu == 4 ? 2 : 3;
+  const int lgn = ncols <= 1 ? 0 : ncols <= 2 ? 1 : ncols <= 4 ? 2 : 3;
+  const int lg_unit = lgm + (pairs_rows ? 3 : 4) + lgn;       // outputs per unit (log2)
+  bool first_chunk = true;
+  for (int u0 = ur.first; u0 < ur.end;) {
+    const int key = opkey(u0);
+    int cnt = 1;
+    while (cnt < kChunk && u0 + cnt * ur.step < ur.end && opkey(u0 + cnt * ur.step) == key) ++cnt;
+    prep(u0, cnt, ur.step);
+    uint4 b[8];
+#pragma unroll
+    for (int r = 0; r < kChunk; ++r) {
+      if (r < cnt) {
+        const uint32_t slot = (c.seq + r) % kNumSlots;
+        if (!wait_mbar(&c.sm.full[slot], ((c.seq + r) / kNumSlots) & 1u, p.err, p.wait_ns, nullptr))
+          c.sm.flags[1] = 1;
+        if (first_chunk && r == 0) timeline(c, call, 9 + 4 * si);
+        const int u = u0 + r * ur.step;
+        (void)u;
+        unit_mma<WT>(c, g, c.sm.ring + (size_t)slot * kSlotBytes, Kdim, 0, r, b, r == 0);
+        __syncwarp();
+        if ((threadIdx.x & 31) == 0) mbar_arrive(&c.sm.empty[slot]);
+      }
+    }
+    c.seq += cnt;
     consumer_sync();
     if (*(volatile int*)&c.sm.flags[1]) {
       c.abort_ = true;
       return;
     }
-    unit_mma<WT>(c, g, c.sm.ring + (size_t)slot * kSlotBytes, Kdim);
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&c.sm.empty[slot]);
-    ++c.seq;
-    consumer_sync();
-    const int per = pairs_rows ? 64 : 128;
-    for (int o = threadIdx.x; o < g.Mu * per; o += kConsumerThreads) {
-      const int mi = o / per, r = o % per;
-      epi(u, mi, r >> 3, r & 7);
+    for (int o = threadIdx.x; o < (cnt << lg_unit); o += kConsumerThreads) {
+      const int r = o >> lg_unit, q = o & ((1 << lg_unit) - 1);
+      const int row = q >> lgn, n = q & ((1 << lgn) - 1);
+      if (n < ncols) {
+        const int mi = row >> (pairs_rows ? 3 : 4), rr = row & (pairs_rows ? 7 : 15);
+        const float v = red_sum(c, g, r, mi, rr, n);
+        const float v8 = pairs_rows ? red_sum(c, g, r, mi, rr + 8, n) : 0.f;
+        epi(u0 + r * ur.step, mi, rr, n, v, v8);
+      }
     }
-    c.buf ^= 1;
+    u0 += cnt * ur.step;
+    first_chunk = false;
+    if (u0 < ur.end) consumer_sync();
   }
   c.rot = (c.rot + n_units) % p.n_cta;
 }
@@ -464,148 +496,167 @@ __device__ void gather_inputs(Cons& c) {
 // cached rows are staged in shared memory with all loads in flight at once, so every dot
 // product reads shared memory.  The o rows land in act[0..n_rows) x D; the new K/V rows are
 // written to the cache if write_kv.
+// Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
+// per-frame cache plus the new rows).  Scratch spans act + bfrag (64 KB): the kv head's
+// cached rows are staged in shared memory with all loads in flight at once, so every dot
+// product reads shared memory.  The o rows land in act[0..n_rows) x D; the new K/V rows are
+// written to the cache if write_kv.
+// Attention of query head h for the call's rows, output o[n][D] in act.  Three phases
+// separated by barriers: (A) every input row (q, new k / v, cached k / v, RoPE rows, QK-norm
+// gains) is loaded as independent 16-byte chunks; (B) one warp per new q / k vector applies
+// QK-norm and RoPE in registers (lane holds dims l + 32i, so each rotate-half pair
+// (d, d + D/2) sits in one lane) and, for the KV writer, stores k / v rows to the cache;
+// (C) one warp per query row: lane j scores key j (rows padded to D + 4 floats so the
+// lanes' 16-byte reads hit distinct banks), softmax across lanes, then P.V with lane-owned
+// output dims.
 __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const FrameParams& p = c.p;
   const int* ci = c.sm.call_info;
-  const int n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
-  const int D = p.D, group = p.NH / p.NKV, g = h / group;
+  const int nr = ci[CI_NROWS], pos0 = ci[CI_POS0];
+  const int D = p.D, half = D >> 1, g = h / (p.NH / p.NKV);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  float* o = c.sm.act;                         // [8][D]
-  float* qs = o + kMaxRows * 128;              // [8][D]
-  float* ks = qs + kMaxRows * 128;             // [kMaxPos][D]: cached rows, then the new rows
-  float* vs = ks + kMaxPos * 128;              // [kMaxPos][D]
-  float* pr = vs + kMaxPos * 128;              // [8][kMaxPos]
-  float* nrm = pr + kMaxRows * kMaxPos;        // [16]
-  float* gq = nrm + 16;                        // [D]
-  float* gk = gq + 128;                        // [D]
-  const float* kc = p.kcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
-  const float* vc = p.vcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const int cs_shift = D == 128 ? 5 : 4;           // 16-byte chunks per row = D / 4
+  const int cpr = 1 << cs_shift;
+  const int KS = D + 4;                            // padded key-row stride (floats)
+  float* o = c.sm.act;                             // [8][D]
+  float* qs = o + kMaxRows * 128;                  // [8][KS]
+  float* ks = qs + kMaxRows * 132;                 // [kMaxPos][KS]
+  float* vs = ks + kMaxPos * 132;                  // [kMaxPos][D]
+  float2* cs = reinterpret_cast<float2*>(vs + kMaxPos * 128);   // [8][D/2] (cos, sin)
+  float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
+  float* gk = gq + 128;                                          // [D]
+  const size_t cache_off = ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
+  // ---- (A) loads ----------------------------------------------------------------------
   {
-    const int per = D >> 2;
-    const int nq = n_rows * per, nc = pos0 * per;
-    const int total = 3 * nq + 2 * nc + (p.qk_norm ? 2 * per : 0);   // <= 8 per thread
-    constexpr int kL = 8;
+    const int n_new = nr << cs_shift, n_old = pos0 << cs_shift;
+    const int e_q = n_new, e_k = 2 * n_new, e_v = 3 * n_new, e_kc = e_v + n_old, e_vc = e_kc + n_old;
+    const int e_cs = e_vc + n_new, e_g = e_cs + (p.qk_norm ? 2 * cpr : 0);
+    constexpr int kL = 10;
     float4 v[kL];
-    float* dst[kL];
+    float4* dst[kL];
 #pragma unroll
     for (int u = 0; u < kL; ++u) {
       const int i = tid + u * kConsumerThreads;
       dst[u] = nullptr;
-      if (i < 3 * nq) {
-        const int w = i / nq, r = i - w * nq, n = r / per, d4 = r - n * per;
-        const float* row = p.qkv + (size_t)n * p.qkv_dim + (w == 0 ? qoff : w == 1 ? koff : voff);
-        v[u] = __ldcg(reinterpret_cast<const float4*>(row) + d4);
-        dst[u] = (w == 0 ? qs + n * D : w == 1 ? ks + (pos0 + n) * D : vs + (pos0 + n) * D) + 4 * d4;
-      } else if (i < 3 * nq + 2 * nc) {
-        const int r = i - 3 * nq, w = r / nc, rr = r - w * nc, j = rr / per, d4 = rr - j * per;
-        v[u] = __ldcg(reinterpret_cast<const float4*>((w == 0 ? kc : vc) + (size_t)j * D) + d4);
-        dst[u] = (w == 0 ? ks : vs) + j * D + 4 * d4;
-      } else if (i < total) {
-        const int r = i - 3 * nq - 2 * nc, w = r / per, d4 = r - w * per;
-        v[u] = __ldg(reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D) + d4);
-        dst[u] = (w == 0 ? gq : gk) + 4 * d4;
+      if (i < e_g) {
+        const float4* src;
+        if (i < e_v) {
+          const int seg = i < e_q ? 0 : (i < e_k ? 1 : 2);
+          const int r = i - seg * n_new, n = r >> cs_shift, ch = r & (cpr - 1);
+          src = reinterpret_cast<const float4*>(qkv + (size_t)n * p.qkv_dim + (seg == 0 ? qoff : seg == 1 ? koff : voff)) + ch;
+          dst[u] = reinterpret_cast<float4*>(seg == 0 ? qs + n * KS : seg == 1 ? ks + (pos0 + n) * KS : vs + (pos0 + n) * D) + ch;
+        } else if (i < e_vc) {
+          const bool isk = i < e_kc;
+          const int r = i - (isk ? e_v : e_kc), j = r >> cs_shift, ch = r & (cpr - 1);
+          src = reinterpret_cast<const float4*>((isk ? p.kcache : p.vcache) + cache_off + (size_t)j * D) + ch;
+          dst[u] = reinterpret_cast<float4*>(isk ? ks + j * KS : vs + j * D) + ch;
+        } else if (i < e_cs) {
+          const int r = i - e_vc, n = r >> cs_shift, ch = r & (cpr - 1);
+          src = reinterpret_cast<const float4*>(p.rope + (size_t)(pos0 + n) * half) + ch;
+          dst[u] = reinterpret_cast<float4*>(cs + n * 64) + ch;
+        } else {
+          const int r = i - e_cs, w = r >> cs_shift, ch = r & (cpr - 1);
+          src = reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D) + ch;
+          dst[u] = reinterpret_cast<float4*>(w == 0 ? gq : gk) + ch;
+        }
+        v[u] = __ldcg(src);
       }
     }
 #pragma unroll
     for (int u = 0; u < kL; ++u)
-      if (dst[u]) *reinterpret_cast<float4*>(dst[u]) = v[u];
+      if (dst[u]) *dst[u] = v[u];
   }
   consumer_sync();
-  float* knew = ks + pos0 * D;
-  float* vnew = vs + pos0 * D;
-  if (p.qk_norm) {
-    for (int vi = warp; vi < 2 * n_rows; vi += kConsumerWarps) {
-      const float* v = vi < n_rows ? qs + vi * D : knew + (vi - n_rows) * D;
+  // ---- (B) QK-norm + RoPE of the new q / k rows; KV writer stores k / v ---------------
+  const int nd = D >> 5;   // dims per lane: 4 (D = 128) or 2 (D = 64)
+  for (int vi = warp; vi < 2 * nr; vi += kConsumerWarps) {
+    const bool isq = vi < nr;
+    const int n = isq ? vi : vi - nr;
+    float* row = isq ? qs + n * KS : ks + (pos0 + n) * KS;
+    float x[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = i < nd ? row[lane + 32 * i] : 0.f;
+    if (p.qk_norm) {
       float ss = 0.f;
-      for (int d = lane; d < D; d += 32) ss += v[d] * v[d];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ss += x[i] * x[i];
 #pragma unroll
       for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
-      if (lane == 0) nrm[vi] = rsqrtf(ss / (float)D + p.eps);
-    }
-    consumer_sync();
-  }
-  // QK-norm gain and RoPE (rotate-half pairs (d, d + D/2)) on the new rows
-  const int half = D / 2;
-  for (int idx = tid; idx < 2 * n_rows * half; idx += kConsumerThreads) {
-    const int vi = idx / half, d = idx - vi * half;
-    const bool isq = vi < n_rows;
-    const int n = isq ? vi : vi - n_rows;
-    float* v = isq ? qs + n * D : knew + n * D;
-    float a = v[d], b = v[d + half];
-    if (p.qk_norm) {
-      const float sc = nrm[vi];
+      const float sc = rsqrtf(ss / (float)D + p.eps);
       const float* gg = isq ? gq : gk;
-      a = a * sc * gg[d];
-      b = b * sc * gg[d + half];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) x[i] = x[i] * sc * gg[lane + 32 * i];
     }
-    const float2 cs = p.rope[(pos0 + n) * half + d];
-    v[d] = a * cs.x - b * cs.y;
-    v[d + half] = b * cs.x + a * cs.y;
+    // rotate-half pairs: dims (lane + 32 i, lane + 32 i + D/2) for i < nd / 2
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if (i < nd / 2) {
+        const float2 r = cs[n * 64 + lane + 32 * i];
+        const float a = x[i], b = x[i + nd / 2];
+        x[i] = a * r.x - b * r.y;
+        x[i + nd / 2] = b * r.x + a * r.y;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < nd) row[lane + 32 * i] = x[i];
+    if (write_kv) {
+      float* kdst = p.kcache + cache_off + (size_t)(pos0 + n) * D;
+      float* vdst = p.vcache + cache_off + (size_t)(pos0 + n) * D;
+      if (!isq) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (i < nd) kdst[lane + 32 * i] = x[i];
+      } else {
+        const float* vrow = vs + (pos0 + n) * D;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (i < nd) vdst[lane + 32 * i] = vrow[lane + 32 * i];
+      }
+    }
   }
   consumer_sync();
-  if (write_kv) {
-    float* kcw = p.kcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
-    float* vcw = p.vcache + ((size_t)layer * p.NKV + g) * kMaxPos * D;
-    const int n4 = n_rows * D / 4;
-    for (int i = tid; i < 2 * n4; i += kConsumerThreads) {
-      const int w = i / n4, r = i - w * n4;
-      float4* dst = reinterpret_cast<float4*>((w ? vcw : kcw) + (size_t)pos0 * D) + r;
-      *dst = reinterpret_cast<const float4*>(w ? vnew : knew)[r];
-    }
-  }
-  // scores: warp n; lane = (key group kq, dim quarter dq)
-  const float scale = rsqrtf((float)D);
-  if (warp < n_rows) {
-    const int n = warp, npos = pos0 + n + 1;
-    const int kq = lane >> 2, dq = lane & 3, dl = D / 4;
-    const float4* qv = reinterpret_cast<const float4*>(qs + n * D + dq * dl);
-    float sc[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int j = kq + 8 * i;
-      float acc = 0.f;
-      if (j < npos) {
-        const float4* kv = reinterpret_cast<const float4*>(ks + j * D + dq * dl);
+  // ---- (C) scores, softmax, P.V: warp n --------------------------------------------------
+  if (warp < nr) {
+    const int n = warp, npos = pos0 + n + 1;       // causal: keys 0..pos0+n (<= 32)
+    const float scale = rsqrtf((float)D);
+    float s = -INFINITY;
+    if (lane < npos) {
+      const float4* q4 = reinterpret_cast<const float4*>(qs + n * KS);
+      const float4* k4 = reinterpret_cast<const float4*>(ks + lane * KS);
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll 8
-        for (int d = 0; d < dl / 4; ++d) {
-          const float4 a = qv[d], b = kv[d];
-          acc += a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w;
-        }
+      for (int ch = 0; ch < cpr; ++ch) {
+        const float4 q = q4[ch], k = k4[ch];
+        a0 += q.x * k.x;
+        a1 += q.y * k.y;
+        a2 += q.z * k.z;
+        a3 += q.w * k.w;
       }
-      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
-      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 2);
-      sc[i] = j < npos ? acc * scale : -INFINITY;
+      s = ((a0 + a1) + (a2 + a3)) * scale;
     }
-    float m = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+    float m = s;
 #pragma unroll
     for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
-    float e[4], sum = 0.f;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      e[i] = (kq + 8 * i) < npos ? __expf(sc[i] - m) : 0.f;
-      sum += (dq == 0) ? e[i] : 0.f;
-    }
+    const float e = lane < npos ? __expf(s - m) : 0.f;
+    float sum = e;
 #pragma unroll
     for (int off = 16; off; off >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, off);
-    if (dq == 0) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) pr[n * kMaxPos + kq + 8 * i] = e[i] / sum;
-    }
-    __syncwarp();
-    // o[n] = sum_j pr_j v_j: lane owns D/32 consecutive dims
-    const int dpl = D / 32;
+    const float pj = e / sum;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int j = 0; j < npos; ++j) {
-      const float a = pr[n * kMaxPos + j];
-      const float* vr = vs + j * D + lane * dpl;
+      const float a = __shfl_sync(0xFFFFFFFFu, pj, j);
+      const float* vr = vs + j * D + lane;
 #pragma unroll
-      for (int d = 0; d < 4; ++d)
-        if (d < dpl) acc[d] += a * vr[d];
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) acc[i] += a * vr[32 * i];
     }
 #pragma unroll
-    for (int d = 0; d < 4; ++d)
-      if (d < dpl) o[n * D + lane * dpl + d] = acc[d];
+    for (int i = 0; i < 4; ++i)
+      if (i < nd) o[n * D + lane + 32 * i] = acc[i];
   }
   consumer_sync();
 }
@@ -625,28 +676,32 @@ __device__ void run_call(Cons& c, int call) {
   const float* x = p.x;
   auto from_x = [&](int n, int k) { return ld_global2(x + (size_t)n * H + k); };
 
+  auto no_key = [](int) { return 0; };
+  auto no_prep = [](int, int, int) {};
   for (int l = 0; l < L; ++l) {
     // ---- S1: RMSNorm -> QKV  (q, k, v = W (x . g) / rms) -------------------------------
     g2s_vec(sm.vec, p.attn_norm + (size_t)l * H, H);      // independent of the wait below
     if (l == 0) {
       gather_inputs(c);
-      prep_operand<WT>(c, n_rows, H, sm.vec, true, [&](int n, int k) { return ld_shared2(sm.act + n * H + k); });
+      prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, [&](int n, int k) { return ld_shared2(sm.act + n * H + k); });
     } else {
       if (!cons_wait(c, ctr + ctr_stage(l - 1, 3), N)) return;
-      prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
+      prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
     }
     {
       const MatGeom& g = p.g[MAT_QKV];
-      run_stage<WT>(c, call, 4 * l + 0, g.n_units, H, [&](int) {}, [&](int u, int mi, int rr, int n) {
-        const float v = red_get(c, g, mi, rr, n) * sm.inv_rms[n];
-        const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-        if (n < n_rows) p.qkv[(size_t)n * p.qkv_dim + row] = v;
-      });
+      run_stage<WT>(c, call, 4 * l + 0, g.n_units, H, n_rows, no_key, no_prep,
+                    [&](int u, int mi, int rr, int n, float v, float) {
+                      const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+                      p.qkv[(size_t)n * p.qkv_dim + row] = v * sm.inv_rms[n];
+                    });
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 0), call, 10 + 4 * (4 * l + 0));
 
     // ---- S2: attention (per query head) -> Wo + residual --------------------------------
+    // Unit u of Wo covers m-block u % n_mb of query head h = u / n_mb (its k-chunk); its B
+    // operand is head h's attention output.
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
     {
       const MatGeom& g = p.g[MAT_WO];
@@ -654,21 +709,21 @@ __device__ void run_call(Cons& c, int call) {
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
       run_stage<WT>(
-          c, call, 4 * l + 1, g.n_units, D,
-          [&](int u) {
-            const int h = u / g.n_mb, mb = u % g.n_mb;
-            const bool writer = (h % group) == 0 && mb == 0;
-            if (sm.flags[3] != h || writer) {   // a CTA meets m-block 0 of a head first
-              consumer_sync();
+          c, call, 4 * l + 1, g.n_units, D, n_rows, [&](int u) { return u / g.n_mb; },
+          [&](int u, int cnt, int step) {
+            const int h = u / g.n_mb;
+            bool writer = false;      // the CTA holding m-block 0 of a group's first head writes K / V
+            for (int r = 0; r < cnt; ++r) writer |= (h % group) == 0 && (u + r * step) % g.n_mb == 0;
+            if (sm.flags[3] != h || writer) {
               attention_head(c, l, h, writer);
-              prep_operand<WT>(c, n_rows, D, nullptr, false, [&](int n, int k) { return ld_shared2(sm.act + n * D + k); });
+              prep_operand<WT>(c, n_rows, D, 0, D, nullptr, false,
+                               [&](int n, int k) { return ld_shared2(sm.act + n * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
-          [&](int u, int mi, int rr, int n) {
-            const float v = red_get(c, g, mi, rr, n);
+          [&](int u, int mi, int rr, int n, float v, float) {
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
+            atomicAdd(p.x + (size_t)n * H + row, v);
           });
       if (c.abort_) return;
     }
@@ -677,25 +732,24 @@ __device__ void run_call(Cons& c, int call) {
     // ---- S3: RMSNorm -> gate/up -> SwiGLU --------------------------------------------------
     g2s_vec(sm.vec, p.ffn_norm + (size_t)l * H, H);
     if (!cons_wait(c, ctr + ctr_stage(l, 1), N)) return;
-    prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
+    prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
     {
       const MatGeom& g = p.g[MAT_GU];
+      // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
       run_stage<WT>(
-          c, call, 4 * l + 2, g.n_units, H, [&](int) {},
-          [&](int u, int mi, int rr, int n) {
-            // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
+          c, call, 4 * l + 2, g.n_units, H, n_rows, no_key, no_prep,
+          [&](int u, int mi, int rr, int n, float gate, float up) {
             const float s = sm.inv_rms[n];
-            const float gt = red_get(c, g, mi, rr, n) * s;
-            const float up = red_get(c, g, mi, rr + 8, n) * s;
+            const float gt = gate * s;
             const int j = ((u % g.n_mb) * g.Mu + mi) * 8 + rr;
-            if (n < n_rows) p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * up;
+            p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * (up * s);
           },
           true);
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 2), call, 10 + 4 * (4 * l + 2));
 
-    // ---- S4: down + residual -------------------------------------------------------------
+    // ---- S4: down + residual (k-chunks of F) ---------------------------------------------
     if (!cons_wait(c, ctr + ctr_stage(l, 2), N)) return;
     {
       const MatGeom& g = p.g[MAT_WD];
@@ -703,21 +757,19 @@ __device__ void run_call(Cons& c, int call) {
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
       run_stage<WT>(
-          c, call, 4 * l + 3, g.n_units, Kc,
-          [&](int u) {
+          c, call, 4 * l + 3, g.n_units, Kc, n_rows, [&](int u) { return u / g.n_mb; },
+          [&](int u, int, int) {
             const int kc = u / g.n_mb;
             if (sm.flags[3] != kc) {
-              consumer_sync();
               const float* m = p.mbuf + (size_t)kc * Kc;
-              prep_operand<WT>(c, n_rows, Kc, nullptr, false,
+              prep_operand<WT>(c, n_rows, Kc, 0, Kc, nullptr, false,
                                [&](int n, int k) { return ld_global2(m + (size_t)n * F + k); });
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
           },
-          [&](int u, int mi, int rr, int n) {
-            const float v = red_get(c, g, mi, rr, n);
+          [&](int u, int mi, int rr, int n, float v, float) {
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            if (n < n_rows) atomicAdd(p.x + (size_t)n * H + row, v);
+            atomicAdd(p.x + (size_t)n * H + row, v);
           });
       if (c.abort_) return;
     }
@@ -727,31 +779,39 @@ __device__ void run_call(Cons& c, int call) {
   // ---- S5: final RMSNorm -> verify and draft heads ---------------------------------------
   // Column n of the operand is row n (h_n before its 1/rms); LM head P's output for row n
   // is verify logits (j = 0) or the draft logits of offset j = P - (pos0 + n) (1 <= j <= K),
-  // whose LMH_P b_j term comes from the precomputed bias table.
+  // whose LMH_P b_j term comes from the precomputed bias table (staged per chunk in `vec`,
+  // which is free once the operand is built).
   g2s_vec(sm.vec, p.final_norm, H);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
-  prep_operand<WT>(c, n_rows, H, sm.vec, true, from_x);
+  prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
   {
     const MatGeom& g = p.g[MAT_HEAD];
     const int p_lo = ci[CI_PLO], n_heads = ci[CI_PHI] - ci[CI_PLO] + 1;
     const int fr = ci[CI_FR], pos0 = ci[CI_POS0];
-    float bias = 0.f;   // this thread's output of the next unit: (row rr, column n) = (tid>>3, tid&7)
+    float* bias_s = sm.vec;   // [kChunk][16 rows][8 columns]
+    int chunk_u0 = 0;
     run_stage<WT>(
-        c, call, 4 * L, n_heads * g.n_units, H,
-        [&](int u) {
-          bias = 0.f;
-          const int P = p_lo + u / g.n_units, n = threadIdx.x & 7, j = P - (pos0 + n);
-          if (threadIdx.x < 128 && j >= 1 && j <= p.K && n < n_rows && n >= fr) {
-            const int id = (u % g.n_units) * g.Mu * 16 + (threadIdx.x >> 3);
-            bias = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
+        c, call, 4 * L, n_heads * g.n_units, H, n_rows, no_key,
+        [&](int u0, int cnt, int step) {
+          chunk_u0 = u0;
+          for (int o = threadIdx.x; o < cnt * 128; o += kConsumerThreads) {
+            const int r = o >> 7, rr = (o >> 3) & 15, n = o & 7;
+            const int u = u0 + r * step;
+            const int P = p_lo + u / g.n_units, j = P - (pos0 + n);
+            float bv = 0.f;
+            if (j >= 1 && j <= p.K && n < n_rows && n >= fr) {
+              const int id = (u % g.n_units) * 16 + rr;
+              bv = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
+            }
+            bias_s[o] = bv;
           }
         },
-        [&](int u, int mi, int rr, int n) {
+        [&](int u, int mi, int rr, int n, float v, float) {
           const int P = p_lo + u / g.n_units, j = P - (pos0 + n);
-          if (n >= fr && n < n_rows && j >= 0 && j <= p.K) {
-            const float v = red_get(c, g, mi, rr, n) * sm.inv_rms[n] + bias;
+          if (n >= fr && j >= 0 && j <= p.K) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
-            p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] = v;
+            p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
+                v * sm.inv_rms[n] + bias_s[(u - chunk_u0) * 128 + rr * 8 + n];
           }
         });
     if (c.abort_) return;

@@ -27,6 +27,7 @@ constexpr int kConsumerThreads = kConsumerWarps * 32;
 constexpr int kThreads = kConsumerThreads + 32;   // + one producer warp
 constexpr int kSlotBytes = 32768;
 constexpr int kNumSlots = 4;
+constexpr int kChunk = 3;            // units of one stage multiplied before one epilogue pass (<= kNumSlots)
 constexpr int kActBytes = 32768;     // fp32 activation rows / attention / top-k scratch
 constexpr int kBfragBytes = 32768;   // B operand (activations) of the unit GEMMs
 constexpr int kRedBytes = 4096;      // one cross-warp reduction buffer (x2)
@@ -204,6 +205,14 @@ __device__ __forceinline__ uint32_t bf16_rn_bits(float x) {
   return (u + bias) >> 16;
 }
 __device__ __forceinline__ float bf16_bits_to_f32(uint32_t b) { return __uint_as_float(b << 16); }
+// Two fp32 values rounded to nearest-even bf16 in one packed word: `lo` in bits 0-15.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+__device__ __forceinline__ float bf16_lo_f32(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi_f32(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ void split_bf16(float x, uint32_t& hi, uint32_t& lo) {
   hi = bf16_rn_bits(x);
   lo = bf16_rn_bits(x - bf16_bits_to_f32(hi));
