@@ -97,13 +97,14 @@ __device__ __forceinline__ const uint8_t* unit_src(const FrameParams& p, int si,
   return base + (long long)layer * g.stride + (long long)u * g.unit_bytes;
 }
 
-// Units [first, end) step `step` of stage si for this CTA: strided with rotation for the
-// backbone, one contiguous block for the LM heads.
+// Units [first, end) step `step` of stage si for this CTA: strided with rotation for most
+// backbone stages; one contiguous block for the LM heads (a CTA mostly reads one head) and
+// for the down projection (a CTA's units mostly share one k-chunk, so one operand).
 struct UnitRange {
   int first, end, step;
 };
 __device__ __forceinline__ UnitRange unit_range(int si, int L, int n, int cta, int rot, int n_cta) {
-  if (stage_kind(si, L) == MAT_HEAD) {
+  if (stage_kind(si, L) == MAT_HEAD || stage_kind(si, L) == MAT_WD) {
     return UnitRange{(int)(((long long)cta * n) / n_cta), (int)(((long long)(cta + 1) * n) / n_cta), 1};
   }
   int f = (cta - rot) % n_cta;
@@ -492,23 +493,14 @@ __device__ void gather_inputs(Cons& c) {
 }
 
 // Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
-// per-frame cache plus the new rows).  Scratch spans act + bfrag (64 KB): the kv head's
-// cached rows are staged in shared memory with all loads in flight at once, so every dot
-// product reads shared memory.  The o rows land in act[0..n_rows) x D; the new K/V rows are
-// written to the cache if write_kv.
-// Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
-// per-frame cache plus the new rows).  Scratch spans act + bfrag (64 KB): the kv head's
-// cached rows are staged in shared memory with all loads in flight at once, so every dot
-// product reads shared memory.  The o rows land in act[0..n_rows) x D; the new K/V rows are
-// written to the cache if write_kv.
-// Attention of query head h for the call's rows, output o[n][D] in act.  Three phases
-// separated by barriers: (A) every input row (q, new k / v, cached k / v, RoPE rows, QK-norm
-// gains) is loaded as independent 16-byte chunks; (B) one warp per new q / k vector applies
-// QK-norm and RoPE in registers (lane holds dims l + 32i, so each rotate-half pair
-// (d, d + D/2) sits in one lane) and, for the KV writer, stores k / v rows to the cache;
-// (C) one warp per query row: lane j scores key j (rows padded to D + 4 floats so the
-// lanes' 16-byte reads hit distinct banks), softmax across lanes, then P.V with lane-owned
-// output dims.
+// per-frame cache plus the new rows); output o[n][D] in act.  Scratch spans act + bfrag
+// (< 64 KB).  Phases, separated by barriers: (A) every input row (q, new k / v, cached
+// k / v, RoPE rows, QK-norm gains) is loaded as independent 16-byte chunks, all in flight at
+// once; (B) one warp per new q / k vector applies QK-norm and RoPE in registers (lane holds
+// dims l + 32i, so each rotate-half pair (d, d + D/2) sits in one lane) and, for the KV
+// writer, stores the new k / v rows to the cache; (C1) two threads per (row, key) score it
+// over interleaved 16-byte chunks (rows padded to D + 8 floats: conflict-free reads); (C2)
+// one warp per row takes the softmax; (C3) one thread per (row, dim pair) sums P.V.
 __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const FrameParams& p = c.p;
   const int* ci = c.sm.call_info;
@@ -517,11 +509,11 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cs_shift = D == 128 ? 5 : 4;           // 16-byte chunks per row = D / 4
   const int cpr = 1 << cs_shift;
-  const int KS = D + 4;                            // padded key-row stride (floats)
+  const int KS = D + 8;                            // padded row stride (floats) of q and k rows
   float* o = c.sm.act;                             // [8][D]
   float* qs = o + kMaxRows * 128;                  // [8][KS]
-  float* ks = qs + kMaxRows * 132;                 // [kMaxPos][KS]
-  float* vs = ks + kMaxPos * 132;                  // [kMaxPos][D]
+  float* ks = qs + kMaxRows * 136;                 // [kMaxPos][KS]
+  float* vs = ks + kMaxPos * 136;                  // [kMaxPos][D]
   float2* cs = reinterpret_cast<float2*>(vs + kMaxPos * 128);   // [8][D/2] (cos, sin)
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
   float* gk = gq + 128;                                          // [D]
@@ -619,47 +611,74 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
     }
   }
   consumer_sync();
-  // ---- (C) scores, softmax, P.V: warp n --------------------------------------------------
-  if (warp < nr) {
-    const int n = warp, npos = pos0 + n + 1;       // causal: keys 0..pos0+n (<= 32)
+  // ---- (C1) scores: thread pair (n, j) splits the dot product over interleaved chunks ---
+  float* sc = gk + 128;                            // [8][32] scores, then probabilities
+  {
     const float scale = rsqrtf((float)D);
-    float s = -INFINITY;
-    if (lane < npos) {
-      const float4* q4 = reinterpret_cast<const float4*>(qs + n * KS);
-      const float4* k4 = reinterpret_cast<const float4*>(ks + lane * KS);
+    for (int t = tid; t < (nr << 6); t += kConsumerThreads) {
+      const int n = t >> 6, j = (t >> 1) & 31, hf = t & 1;
+      const bool live = j <= pos0 + n;               // causal: keys 0..pos0+n
       float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+      if (live) {
+        const float4* q4 = reinterpret_cast<const float4*>(qs + n * KS) + hf;
+        const float4* k4 = reinterpret_cast<const float4*>(ks + j * KS) + hf;
 #pragma unroll 8
-      for (int ch = 0; ch < cpr; ++ch) {
-        const float4 q = q4[ch], k = k4[ch];
-        a0 += q.x * k.x;
-        a1 += q.y * k.y;
-        a2 += q.z * k.z;
-        a3 += q.w * k.w;
+        for (int ch = 0; ch < (cpr >> 1); ++ch) {
+          const float4 q = q4[2 * ch], k = k4[2 * ch];
+          a0 += q.x * k.x;
+          a1 += q.y * k.y;
+          a2 += q.z * k.z;
+          a3 += q.w * k.w;
+        }
       }
-      s = ((a0 + a1) + (a2 + a3)) * scale;
+      float acc = (a0 + a1) + (a2 + a3);
+      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
+      if (hf == 0) sc[n * 32 + j] = live ? acc * scale : -INFINITY;
     }
+  }
+  consumer_sync();
+  // ---- (C2) softmax over the keys of row n: warp n ------------------------------------
+  if (warp < nr) {
+    const float s = sc[warp * 32 + lane];
     float m = s;
 #pragma unroll
     for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
-    const float e = lane < npos ? __expf(s - m) : 0.f;
+    const float e = lane <= pos0 + warp ? __expf(s - m) : 0.f;
     float sum = e;
 #pragma unroll
     for (int off = 16; off; off >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, off);
-    const float pj = e / sum;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int j = 0; j < npos; ++j) {
-      const float a = __shfl_sync(0xFFFFFFFFu, pj, j);
-      const float* vr = vs + j * D + lane;
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (i < nd) acc[i] += a * vr[32 * i];
+    sc[warp * 32 + lane] = e / sum;
+  }
+  consumer_sync();
+  // ---- (C3) o[n][d..d+1] = sum_j p_j v_j[d..d+1]: one thread per (row, dim pair) --------
+  {
+    const int lgh = D == 128 ? 6 : 5;              // dim pairs per row
+    for (int t = tid; t < (nr << lgh); t += kConsumerThreads) {
+      const int n = t >> lgh, d = 2 * (t & ((1 << lgh) - 1)), npos = pos0 + n + 1;
+      const float* pr = sc + n * 32;
+      float2 c0 = make_float2(0.f, 0.f), c1 = make_float2(0.f, 0.f);
+      int j = 0;
+      for (; j + 1 < npos; j += 2) {
+        const float p0 = pr[j], p1 = pr[j + 1];
+        const float2 v0 = *reinterpret_cast<const float2*>(vs + j * D + d);
+        const float2 v1 = *reinterpret_cast<const float2*>(vs + (j + 1) * D + d);
+        c0.x += p0 * v0.x;
+        c0.y += p0 * v0.y;
+        c1.x += p1 * v1.x;
+        c1.y += p1 * v1.y;
+      }
+      if (j < npos) {
+        const float p0 = pr[j];
+        const float2 v0 = *reinterpret_cast<const float2*>(vs + j * D + d);
+        c0.x += p0 * v0.x;
+        c0.y += p0 * v0.y;
+      }
+      *reinterpret_cast<float2*>(o + n * D + d) = make_float2(c0.x + c1.x, c0.y + c1.y);
     }
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (i < nd) o[n * D + lane + 32 * i] = acc[i];
   }
   consumer_sync();
 }
+
 
 // ------------------------------------------------------------------------------------
 // One call

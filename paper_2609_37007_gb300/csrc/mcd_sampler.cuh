@@ -121,29 +121,42 @@ static __device__ __forceinline__ void block_topk(const float* __restrict__ logi
     key[4 * j + 2] = ok ? f32_key(v.z) : 0u;
     key[4 * j + 3] = ok ? f32_key(v.w) : 0u;
   }
-  // block maximum
-  uint32_t kmax = 0;
+  // block maximum and minimum (padding keys: 0 never wins the maximum, ~0 never the minimum)
+  const int nj = (V + 1023) >> 10;
+  uint32_t kmax = 0, kmin = 0xFFFFFFFFu;
 #pragma unroll
-  for (int e = 0; e < 4 * kJ; ++e) kmax = max(kmax, key[e]);
+  for (int e = 0; e < 4 * kJ; ++e) {
+    if ((e >> 2) < nj) {
+      kmax = max(kmax, key[e]);
+      kmin = min(kmin, key[e]);
+    }
+  }
   kmax = __reduce_max_sync(0xFFFFFFFFu, kmax);
-  if (lane == 0) s.wred[0][warp] = kmax;
+  kmin = __reduce_min_sync(0xFFFFFFFFu, kmin);
+  if (lane == 0) {
+    s.wred[0][warp] = kmax;
+    s.wred[1][warp] = kmin;
+  }
   consumer_sync();
 #pragma unroll
-  for (int w = 0; w < kConsumerWarps; ++w) kmax = max(kmax, s.wred[0][w]);
+  for (int w = 0; w < kConsumerWarps; ++w) {
+    kmax = max(kmax, s.wred[0][w]);
+    kmin = min(kmin, s.wred[1][w]);
+  }
   MCD_TOPK_STAMP(1)
-  // counting search: T = largest t with #(key >= t) >= k, i.e. the k-th largest key
-  // Thresholds lo + i 2^sb stay below 2^32 for every i < nthr (lo is a multiple of 2^(sb+3));
-  // the unused ones (i >= nthr in the last step) may wrap and are ignored.
-  const int nj = (V + 1023) >> 10;
-  uint32_t lo = 0;
-  int bits = 32, buf = 0;
-  while (bits > 0) {
-    const int sb = bits >= 3 ? bits - 3 : 0;
-    const int nthr = bits >= 3 ? 7 : (1 << bits) - 1;
+  // Counting search for the k-th largest key.  Invariant: #(key >= lo) >= k > #(key >= hi).
+  // Each step counts 7 thresholds splitting [lo, hi) into eighths (one barrier); it stops
+  // early when a threshold has exactly k keys at or above it (then that set is the answer
+  // and no tie needs splitting), else when hi = lo + 1 (lo is the k-th largest key).
+  uint32_t lo = kmin;
+  unsigned long long hi = (unsigned long long)kmax + 1ull;
+  int buf = 0;
+  while (hi - lo > 1ull) {
+    const unsigned long long span = hi - lo;
     uint32_t cnt[7];
 #pragma unroll
     for (int i = 0; i < 7; ++i) {
-      const uint32_t t = lo + ((uint32_t)(i + 1) << sb);
+      const uint32_t t = lo + (uint32_t)((span * (unsigned long long)(i + 1)) >> 3);
       uint32_t c = 0;
 #pragma unroll
       for (int e = 0; e < 4 * kJ; ++e)
@@ -158,13 +171,23 @@ static __device__ __forceinline__ void block_topk(const float* __restrict__ logi
     }
     consumer_sync();
     uint32_t tot = 0;
-    if (lane < nthr)
+    if (lane < 7)
 #pragma unroll
       for (int w = 0; w < kConsumerWarps; ++w) tot += s.part[buf][w][lane];
-    const unsigned ok = __ballot_sync(0xFFFFFFFFu, lane < nthr && tot >= (uint32_t)k);
-    lo += (uint32_t)__popc(ok) << sb;
-    bits = sb;
+    const uint32_t my_t = lo + (uint32_t)((span * (unsigned long long)(lane + 1)) >> 3);
+    const unsigned ge = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot >= (uint32_t)k);
+    const unsigned eq = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot == (uint32_t)k);
     buf ^= 1;
+    if (eq) {                                           // exactly k keys >= that threshold
+      lo = __shfl_sync(0xFFFFFFFFu, my_t, __ffs(eq) - 1);
+      break;
+    }
+    // thresholds are increasing in lane, counts decreasing: ge is a prefix of lanes 0..6
+    const int nge = __popc(ge);
+    const uint32_t new_lo = __shfl_sync(0xFFFFFFFFu, my_t, max(nge - 1, 0));
+    const uint32_t new_hi = __shfl_sync(0xFFFFFFFFu, my_t, min(nge, 6));
+    if (nge > 0) lo = new_lo;
+    if (nge < 7) hi = new_hi;
   }
   const uint32_t Tk = lo;
   MCD_TOPK_STAMP(2)
