@@ -74,8 +74,12 @@ typedef struct {
   int32_t draft_len;    /* K; 0 = plain autoregressive decoding                         */
   int32_t top_k;
   float temperature;
-  int32_t draft_mode;   /* MCD_DRAFT_*                                                   */
-  float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only                                  */
+  int32_t draft_mode;   /* MCD_DRAFT_*: SAMPLE = position-aware offset drafter (Sec. 2.2),
+                         * GREEDY = its argmax, NOISY_TARGET = controlled-acceptance drafts:
+                         * q for position s is the target's own fp32 logits of s given the
+                         * drafted prefix (one extra one-row pass per draft, run inside the
+                         * same frame launch) plus noise_sigma * N(0,1) per entry            */
+  float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only (>= 0)                            */
   uint64_t seed;        /* Philox key                                                    */
 } mcd_config;
 
@@ -91,9 +95,10 @@ typedef struct {
   int32_t rows_fed;  /* sum over calls of rows fed                                  */
 } mcd_frame_stats;
 
-/* Per-call record written when tracing is on (mcd_set_trace).  One record per call, in
- * call order; logits of record r live in the trace buffer after all records (see
- * mcd_trace_bytes for the layout). */
+/* Per-call record written when tracing is on (mcd_set_trace).  One record per verify
+ * call, in call order; logits of record r live in the trace buffer after all records (see
+ * mcd_trace_bytes for the layout).  With NOISY_TARGET drafts the draft rows of record r are
+ * the noisy rows its drafts were drawn from. */
 typedef struct {
   int32_t a;              /* codes emitted before this call                           */
   int32_t n_rows;         /* rows fed                                                 */
@@ -152,7 +157,8 @@ mcd_status mcd_decode_frame_host(mcd_ctx* ctx, uint32_t stream_id, uint32_t fram
 /* Stepwise use of the same kernels.  mcd_begin_frame resets the per-frame state and
  * selects the (stream id, frame index) of the Philox counters; it needs no weights, so
  * the sampler hooks below can run on a context without them;
- * mcd_verify_accept runs exactly one model call (the first call feeds cond and c0),
+ * mcd_verify_accept runs exactly one verify call (the first call feeds cond and c0) and,
+ * with NOISY_TARGET drafts, the one-row passes that draft for the next call,
  * writing the codes it emitted to emitted (dev int32 [K+1]) and their count to
  * n_emitted (dev int32 [1]); a call after the frame is complete emits 0 codes.
  * logits_out (dev float [K+1, vocab], optional) receives the verify logits of the

@@ -118,6 +118,10 @@ __global__ void begin_frame_kernel(DevState* st, unsigned* ctr, int n_ctr, const
     st->first_head_row = 1;
     st->n_acc_last = 0;
     st->q_row = 0;
+    st->round = 0;
+    st->emu = 0;
+    st->emu_n = 0;
+    st->emu_in = -1;
     for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
     st->codes[0] = C0V > 0 ? c0[0] : -1;
     for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
@@ -128,12 +132,12 @@ __global__ void begin_frame_kernel(DevState* st, unsigned* ctr, int n_ctr, const
 }
 
 // Reset counters of a single stepwise call (the call index of the state).
+// Counters of the slots one stepwise launch can use (a verify call, its noisy-target
+// drafting passes, and the next slot whose ready flag it raises).
 __global__ void reset_call_counters_kernel(const DevState* st, unsigned* ctr, int stride) {
-  const int call = st->call;
-  if (call < kMaxCalls)
-    for (int i = threadIdx.x; i < stride; i += blockDim.x) ctr[call * stride + i] = 0u;
-  if (call + 1 < kMaxCalls)
-    for (int i = threadIdx.x; i < stride; i += blockDim.x) ctr[(call + 1) * stride + i] = 0u;
+  const int first = st->call;
+  for (int sl = first; sl < min(first + kMaxDraft + 2, kMaxSlots); ++sl)
+    for (int i = threadIdx.x; i < stride; i += blockDim.x) ctr[sl * stride + i] = 0u;
 }
 
 __global__ void zero_emitted_kernel(const DevState* st, int* n_emitted) {
@@ -316,7 +320,7 @@ static mcd_status validate_config(const mcd_config& c) {
   if (!(c.temperature > 0.f) || !(c.rms_eps > 0.f) || !(c.rope_base > 1.f)) return MCD_ERR_INVALID_ARG;
   if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
-  if (c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;  // see mcd.h
+  if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
   if ((long long)c.n_q_heads * c.head_dim + 2LL * c.n_kv_heads * c.head_dim > 8192) return MCD_ERR_UNSUPPORTED;
   return MCD_OK;
 }
@@ -453,7 +457,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.draftq, sizeof(TopkRec) * (kMaxDraft + 1))) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.st, sizeof(DevState))) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxCalls * p.ctr_stride)) != cudaSuccess)
+  if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxSlots * p.ctr_stride)) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &c->host_stage, host_stage_bytes(p))) != cudaSuccess) return fail(cuda_status(e));
@@ -634,7 +638,7 @@ static mcd_status launch_begin(mcd_ctx* c, uint32_t stream_id, uint32_t frame_id
   p.c0emb = c0_emb;
   p.stream_id = stream_id;
   p.frame_idx = frame_idx;
-  begin_frame_kernel<<<1, 256, 0, c->stream>>>(p.st, p.ctr, kMaxCalls * p.ctr_stride, c0, p.C0V);
+  begin_frame_kernel<<<1, 256, 0, c->stream>>>(p.st, p.ctr, kMaxSlots * p.ctr_stride, c0, p.C0V);
   MCD_CHECK(cudaGetLastError());
   c->frame_begun = true;
   return MCD_OK;

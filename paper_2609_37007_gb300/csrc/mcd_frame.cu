@@ -56,7 +56,7 @@ constexpr int kSmemBytes = kInfoOff + kInfoInts * 4;
 
 // call_info slots
 enum { CI_CALL = 0, CI_A, CI_ND, CI_POS0, CI_NROWS, CI_FR, CI_DONE, CI_QROW, CI_PLO, CI_PHI, CI_IDS = 16,
-       CI_CALLS = 24, CI_HEADS, CI_KVROWS, CI_ROWSFED, CI_DRAFTED, CI_ACCEPTED };
+       CI_CALLS = 24, CI_HEADS, CI_KVROWS, CI_ROWSFED, CI_DRAFTED, CI_ACCEPTED, CI_ROUND, CI_EMU, CI_EMUN };
 
 __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   Smem s;
@@ -112,11 +112,17 @@ __device__ __forceinline__ UnitRange unit_range(int si, int L, int n, int cta, i
   return UnitRange{f, n, n_cta};
 }
 
-// heads touched by a call: P_lo = a+1, P_hi = min(n_pos, last row position + K)
-__device__ __forceinline__ void head_range(const FrameParams& p, int a, int pos0, int n_rows, int& p_lo,
+// LM heads a pass reads.  Verify call: P_lo = a+1 up to the last row's position plus K
+// (its draft heads), or up to the last row's position when the drafts come from
+// noisy-target passes.  Noisy-target pass (one row at position s): head s only.
+__device__ __forceinline__ void head_range(const FrameParams& p, int a, int pos0, int n_rows, int emu, int& p_lo,
                                            int& p_hi) {
+  if (emu) {
+    p_lo = p_hi = pos0;
+    return;
+  }
   p_lo = a + 1;
-  p_hi = min(p.P, pos0 + n_rows - 1 + p.K);
+  p_hi = p.draft_mode == MCD_DRAFT_NOISY_TARGET ? pos0 + n_rows - 1 : min(p.P, pos0 + n_rows - 1 + p.K);
 }
 
 // ------------------------------------------------------------------------------------
@@ -129,7 +135,7 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
   int rot = 0;
   volatile int* stop = sm.flags;
   bool halt = false;
-  for (int call = call0; call < kMaxCalls && !halt; ++call) {
+  for (int call = call0; call < kMaxSlots && !halt; ++call) {
     int p_lo = 0, p_hi = -1;
     for (int si = 0; si < n_stages(p) && !halt; ++si) {
       int n_heads = 0;
@@ -142,11 +148,12 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
         }
         const int4 s0 = __ldcg(reinterpret_cast<const int4*>(p.st));        // call, a, done, n_d
         const int2 s1 = __ldcg(reinterpret_cast<const int2*>(p.st) + 2);    // pos0, n_rows
+        const int emu = __ldcg(&p.st->emu);
         if (s0.z) {
           halt = true;
           break;
         }
-        head_range(p, s0.y, s1.x, s1.y, p_lo, p_hi);
+        head_range(p, s0.y, s1.x, s1.y, emu, p_lo, p_hi);
         n_heads = p_hi - p_lo + 1;
       }
       const int n = stage_units(p, si, n_heads);
@@ -166,7 +173,11 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
       }
       rot = (rot + n) % n_cta;
     }
-    if (p.single_call) break;
+    if (p.single_call && !halt) {
+      // a stepwise launch runs one verify call and the noisy-target passes that follow it
+      if (!wait_counter(p.ctr + (call + 1) * p.ctr_stride + ctr_ready(p.L), 1u, p.err, p.wait_ns)) break;
+      if (__ldcg(&p.st->emu) == 0 || __ldcg(&p.st->done)) break;
+    }
   }
   // Drain: every issued copy must land before the CTA may exit.
   const uint32_t first = issued > (uint32_t)kNumSlots ? issued - kNumSlots : 0u;
@@ -200,13 +211,17 @@ struct Cons {
 // heads) at 8+4s: +0 inputs ready (CTA 0), +1 first unit's weights in smem (CTA 0),
 // +2 last epilogue done and +3 signalled (latest CTA).
 constexpr int kTimelineSlots = 128;
-__device__ __forceinline__ void timeline(const Cons& c, int call, int idx, bool any_cta = false) {
-  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots)
-    c.p.timeline[call * kTimelineSlots + idx] = globaltimer();
+// (Indexed by verify round; noisy-target passes are not stamped.)
+__device__ __forceinline__ void timeline(const Cons& c, int, int idx, bool any_cta = false) {
+  const int* ci = c.sm.call_info;
+  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots && !ci[CI_EMU] &&
+      ci[CI_ROUND] < kMaxCalls)
+    c.p.timeline[ci[CI_ROUND] * kTimelineSlots + idx] = globaltimer();
 }
-__device__ __forceinline__ void timeline_max(const Cons& c, int call, int idx) {
-  if (c.p.timeline && threadIdx.x == 0 && idx < kTimelineSlots)
-    atomicMax(c.p.timeline + call * kTimelineSlots + idx, (unsigned long long)globaltimer());
+__device__ __forceinline__ void timeline_max(const Cons& c, int, int idx) {
+  const int* ci = c.sm.call_info;
+  if (c.p.timeline && threadIdx.x == 0 && idx < kTimelineSlots && !ci[CI_EMU] && ci[CI_ROUND] < kMaxCalls)
+    atomicMax(c.p.timeline + ci[CI_ROUND] * kTimelineSlots + idx, (unsigned long long)globaltimer());
 }
 
 __device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned target) {
@@ -841,18 +856,44 @@ __device__ void run_call(Cons& c, int call) {
   if (!cons_wait(c, ctr + ctr_heads(L), N)) return;
   timeline(c, call, 1);
   {
-    const int fr = ci[CI_FR], pos0 = ci[CI_POS0];
+    const int fr = ci[CI_FR], pos0 = ci[CI_POS0], emu = ci[CI_EMU];
     TopkScratch& ts = *reinterpret_cast<TopkScratch*>(sm.act);
-    TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
-    int pair = 0;
-    for (int n = fr; n < n_rows; ++n) {
-      const int kn = min(p.K, p.P - (pos0 + n));
-      for (int j = 0; j <= kn; ++j, ++pair) {
-        if (pair % p.n_cta != (int)blockIdx.x) continue;
-        const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
-        block_topk(p.logits + ((size_t)n * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
-                   recs + n * (kMaxDraft + 1) + j);
+    if (emu) {
+      // noisy-target pass j = emu: q = fp32(target logits + sigma N(0,1)) of position pos0
+      // (Box-Muller pairs of purpose 3 + v/2 under the verify round's counters)
+      if (blockIdx.x == 0) {
+        const float* lg = p.logits;                                   // row 0, j = 0
+        float* zq = p.logits + (size_t)1 * p.V;                        // row 0, slot j = 1
+        for (int pr = threadIdx.x; pr < (p.V >> 1); pr += kConsumerThreads) {
+          const double2 nz = normal_pair(p.seed, p.stream_id, p.frame_idx, ci[CI_ROUND], pos0, pr);
+          const float2 l = __ldcg(reinterpret_cast<const float2*>(lg) + pr);
+          const float2 z = make_float2((float)((double)l.x + (double)p.sigma * nz.x),
+                                       (float)((double)l.y + (double)p.sigma * nz.y));
+          reinterpret_cast<float2*>(zq)[pr] = z;
+          if (p.trace && ci[CI_ROUND] < kMaxCalls) {
+            float* dlog = reinterpret_cast<float*>(p.trace + sizeof(mcd_call_trace) * kMaxCalls) +
+                          (size_t)kMaxCalls * kMaxRows * p.V;
+            reinterpret_cast<float2*>(dlog + ((size_t)ci[CI_ROUND] * kMaxRows + (emu - 1)) * p.V)[pr] = z;
+          }
+        }
+        __threadfence();
         consumer_sync();
+        block_topk(zq, p.V, p.top_k, p.T, 0, ts, p.draftq + (emu - 1));
+        consumer_sync();
+      }
+    } else {
+      TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
+      const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
+      int pair = 0;
+      for (int n = fr; n < n_rows; ++n) {
+        const int kn = noisy ? 0 : min(p.K, p.P - (pos0 + n));
+        for (int j = 0; j <= kn; ++j, ++pair) {
+          if (pair % p.n_cta != (int)blockIdx.x) continue;
+          const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
+          block_topk(p.logits + ((size_t)n * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
+                     recs + n * (kMaxDraft + 1) + j);
+          consumer_sync();
+        }
       }
     }
   }
@@ -888,7 +929,8 @@ __device__ void accept_step(Cons& c, int call) {
   Smem& sm = c.sm;
   const int* ci = sm.call_info;
   const int a = ci[CI_A], n_d = ci[CI_ND], pos0 = ci[CI_POS0], n_rows = ci[CI_NROWS];
-  const int qrow = ci[CI_QROW];
+  const int qrow = ci[CI_QROW], round = ci[CI_ROUND];
+  const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
   const TopkRec* prev = p.topk + (size_t)((call + 1) & 1) * kMaxRows * (kMaxDraft + 1);
@@ -896,8 +938,11 @@ __device__ void accept_step(Cons& c, int call) {
   const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
   __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
   timeline(c, call, 4, true);
+  // p of positions a+1..: this call's verify records; q of the drafts: the previous call's
+  // records of its row qrow, or the noisy-target passes' records
   stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
-    return r < n_p ? cur + (a + 1 + r - pos0) * (kMaxDraft + 1) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p);
+    return r < n_p ? cur + (a + 1 + r - pos0) * (kMaxDraft + 1)
+                   : (noisy ? p.draftq + (r - n_p) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p));
   });
   consumer_sync();
   timeline(c, call, 5, true);
@@ -906,7 +951,7 @@ __device__ void accept_step(Cons& c, int call) {
     for (int i = 0; i < n_d; ++i) drafts[i] = ci[CI_IDS + 1 + i];
     AcceptResult r = warp_accept(
         a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(srec + i); },
-        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, call);
+        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, round);
     if (lane == 0) {
       for (int t = 0; t < r.n_emit; ++t) s_emit[t] = r.emitted[t];
       s_nemit = r.n_emit;
@@ -918,15 +963,18 @@ __device__ void accept_step(Cons& c, int call) {
   const int a_new = a + s_nemit;
   const int m = a_new - pos0;
   const int n_next = min(p.K, p.P - a_new);
-  // draft records of row m (the row whose head emitted the last code): one warp each
-  stage_records(srec, n_next, p.top_k, [&](int r) { return cur + m * (kMaxDraft + 1) + 1 + r; });
-  consumer_sync();
-  for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
-    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, a_new + j, PURPOSE_DRAFT);
-    const int d = warp_draw(srec + j - 1, U);
-    if (lane == 0) s_next[j - 1] = d;
+  // draft records of row m (the row whose head emitted the last code): one warp each (the
+  // noisy-target passes that follow draw their drafts themselves)
+  if (!noisy) {
+    stage_records(srec, n_next, p.top_k, [&](int r) { return cur + m * (kMaxDraft + 1) + 1 + r; });
+    consumer_sync();
+    for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
+      const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, round, a_new + j, PURPOSE_DRAFT);
+      const int d = warp_draw(srec + j - 1, U);
+      if (lane == 0) s_next[j - 1] = d;
+    }
+    consumer_sync();
   }
-  consumer_sync();
   if (threadIdx.x == 0) {
     s_nnext = n_next;
     DevState* st = p.st;
@@ -934,7 +982,8 @@ __device__ void accept_step(Cons& c, int call) {
       st->codes[a + 1 + t] = s_emit[t];
       if (p.codes_out) p.codes_out[a + t] = s_emit[t];
     }
-    for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
+    if (!noisy)
+      for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
     for (int t = 0; t < s_nemit; ++t) st->emitted_last[t] = s_emit[t];
     const int calls = ci[CI_CALLS] + 1, heads = ci[CI_HEADS] + ci[CI_PHI] - ci[CI_PLO] + 1;
     const int kvr = ci[CI_KVROWS] + pos0 + n_rows, rf = ci[CI_ROWSFED] + n_rows;
@@ -942,9 +991,19 @@ __device__ void accept_step(Cons& c, int call) {
     st->n_emit_last = s_nemit;
     st->n_acc_last = s_nacc;
     st->a = a_new;
-    st->n_d = n_next;
-    st->pos0 = a_new + 1;
-    st->n_rows = min(n_next + 1, p.P - a_new);
+    if (noisy && n_next > 0) {           // next: noisy-target pass 1 (row c_a' at position a'+1)
+      st->n_d = 0;
+      st->pos0 = a_new + 1;
+      st->n_rows = 1;
+      st->emu = 1;
+      st->emu_n = n_next;
+      st->emu_in = s_emit[s_nemit - 1];
+    } else {
+      st->n_d = n_next;
+      st->pos0 = a_new + 1;
+      st->n_rows = min(n_next + 1, p.P - a_new);
+      st->round = round + 1;
+    }
     st->first_head_row = 0;
     st->calls = calls;
     st->heads_read = heads;
@@ -975,7 +1034,7 @@ __device__ void accept_step(Cons& c, int call) {
   // optional outputs: trace and stepwise logits
   const int fr = ci[CI_FR];
   if (p.trace) {
-    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(p.trace) + call;
+    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(p.trace) + round;
     if (threadIdx.x == 0) {
       tr->a = a;
       tr->n_rows = n_rows;
@@ -987,7 +1046,7 @@ __device__ void accept_step(Cons& c, int call) {
       tr->n_emit = s_nemit;
       for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < s_nemit ? s_emit[t] : -1;
       tr->n_next = s_nnext;
-      for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = j < s_nnext ? s_next[j] : -1;
+      for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = (j < s_nnext && !noisy) ? s_next[j] : -1;
       tr->draft_row = m;
     }
     float* vlog = reinterpret_cast<float*>(p.trace + sizeof(mcd_call_trace) * kMaxCalls);
@@ -995,9 +1054,9 @@ __device__ void accept_step(Cons& c, int call) {
     for (int idx = threadIdx.x; idx < kMaxRows * p.V; idx += kConsumerThreads) {
       const int n = idx / p.V, v = idx - n * p.V;
       if (n >= fr && n < n_rows)
-        vlog[((size_t)call * kMaxRows + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
-      if (n < s_nnext)
-        dlog[((size_t)call * kMaxRows + n) * p.V + v] =
+        vlog[((size_t)round * kMaxRows + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+      if (n < s_nnext && !noisy)
+        dlog[((size_t)round * kMaxRows + n) * p.V + v] =
             __ldcg(p.logits + ((size_t)m * (kMaxDraft + 1) + n + 1) * p.V + v);
     }
   }
@@ -1010,6 +1069,49 @@ __device__ void accept_step(Cons& c, int call) {
   consumer_sync();
   timeline(c, call, 7, true);
   if (threadIdx.x == 0) {
+    __threadfence();
+    atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+  }
+}
+
+// Draft step of noisy-target pass j (run by the CTA that finished top-k last): draw the
+// draft of position pos0 from the pass's noisy distribution with the draft-purpose uniform
+// of the verify round, then set up pass j+1 or, after the last pass, the verify call.
+__device__ void emu_step(Cons& c, int call) {
+  const FrameParams& p = c.p;
+  Smem& sm = c.sm;
+  const int* ci = sm.call_info;
+  const int j = ci[CI_EMU], n = ci[CI_EMUN], round = ci[CI_ROUND], pos0 = ci[CI_POS0], a = ci[CI_A];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);
+  __shared__ int s_d;
+  stage_records(srec, 1, p.top_k, [&](int) { return p.draftq + (j - 1); });
+  consumer_sync();
+  if (warp == 0) {
+    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, round, pos0, PURPOSE_DRAFT);
+    const int d = warp_draw(srec, U);
+    if (lane == 0) s_d = d;
+  }
+  consumer_sync();
+  if (threadIdx.x == 0) {
+    DevState* st = p.st;
+    const int d = s_d;
+    st->drafts[j - 1] = d;
+    if (j < n) {
+      st->emu = j + 1;
+      st->emu_in = d;
+      st->pos0 = pos0 + 1;
+      st->n_rows = 1;
+    } else {
+      st->emu = 0;
+      st->emu_n = 0;
+      st->n_d = n;
+      st->pos0 = a + 1;
+      st->n_rows = min(n + 1, p.P - a);
+      st->round = round + 1;
+    }
+    st->call = call + 1;
+    if (p.trace && round < kMaxCalls) reinterpret_cast<mcd_call_trace*>(p.trace)[round].next_drafts[j - 1] = d;
     __threadfence();
     atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
   }
@@ -1043,14 +1145,20 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
     ci[CI_ROWSFED] = st->rows_fed;
     ci[CI_DRAFTED] = st->drafted;
     ci[CI_ACCEPTED] = st->accepted;
+    ci[CI_ROUND] = st->round;
+    ci[CI_EMU] = st->emu;
+    ci[CI_EMUN] = st->emu_n;
     int plo, phi;
-    head_range(p, ci[CI_A], ci[CI_POS0], ci[CI_NROWS], plo, phi);
+    head_range(p, ci[CI_A], ci[CI_POS0], ci[CI_NROWS], ci[CI_EMU], plo, phi);
     ci[CI_PLO] = plo;
     ci[CI_PHI] = phi;
-    // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft i-1
+    // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft i-1;
+    // a noisy-target pass feeds its one code
     const int a = ci[CI_A];
     for (int i = 0; i < kMaxDraft; ++i) ci[CI_IDS + 1 + i] = st->drafts[i];
-    if (ci[CI_POS0] == 0) {
+    if (ci[CI_EMU]) {
+      ci[CI_IDS + 0] = st->emu_in;
+    } else if (ci[CI_POS0] == 0) {
       ci[CI_IDS + 0] = -1;
       ci[CI_IDS + 1] = st->codes[0];
     } else {
@@ -1084,13 +1192,19 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
     if ((tid & 31) == 0) producer_loop(p, sm, call0);
   } else {
     Cons c(p, sm);
-    for (int call = call0; call < kMaxCalls; ++call) {
+    for (int call = call0; call < kMaxSlots; ++call) {
       if (!read_call_state(c, call, call == call0)) break;
       if (sm.call_info[CI_DONE]) break;
+      // a stepwise launch runs one verify call and the noisy-target passes that follow it
+      if (p.single_call && call != call0 && !sm.call_info[CI_EMU]) break;
       run_call<WT>(c, call);
       if (c.abort_) break;
-      if (sm.flags[2]) accept_step(c, call);
-      if (p.single_call) break;
+      if (sm.flags[2]) {
+        if (sm.call_info[CI_EMU])
+          emu_step(c, call);
+        else
+          accept_step(c, call);
+      }
     }
     if (tid == 0) sm.flags[0] = 1;  // stop the producer
   }

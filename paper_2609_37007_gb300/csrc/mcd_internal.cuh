@@ -20,7 +20,8 @@ constexpr int kMaxRows = 8;          // rows of one call (K+1 <= 8; first call u
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
-constexpr int kMaxCalls = 16;        // calls per frame (15 positions, first call emits 1)
+constexpr int kMaxCalls = 16;        // verify calls per frame (15 positions, first call emits 1)
+constexpr int kMaxSlots = 128;       // passes per frame: verify calls + noisy-target drafting passes
 constexpr int kMaxVocab = 4096;
 constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
@@ -45,7 +46,8 @@ struct MatGeom {
 
 // Per-call state shared by all CTAs, rewritten by the CTA that runs the acceptance step.
 struct DevState {
-  int call;            // index of the next call
+  int call;            // slot (counter set) of the next pass: every verify call and every
+                       // noisy-target drafting pass takes one
   int a;               // codes emitted so far
   int done;
   int n_d;             // pending drafts (positions a+1..a+n_d)
@@ -63,6 +65,10 @@ struct DevState {
   int kv_rows;         // sum over calls of (pos0 + n_rows): KV positions read or written
   int rows_fed;        // sum over calls of n_rows
   int err;
+  int round;           // verify round of the next pass (Philox round, trace index)
+  int emu;             // 0: the next pass is a verify call; j >= 1: noisy-target pass j
+  int emu_n;           // drafts the noisy-target passes make for the next verify call
+  int emu_in;          // code fed to the next noisy-target pass
 };
 
 // One top-k / temperature distribution as integer weights: p(ids[i]) = W[i] / S.
@@ -258,6 +264,22 @@ __host__ __device__ inline unsigned long long uniform_U(unsigned long long seed,
 }
 
 enum { PURPOSE_TARGET = 0, PURPOSE_ACCEPT = 1, PURPOSE_DRAFT = 2, PURPOSE_NOISE = 3 };
+
+// Two N(0,1) draws for vocabulary entries (2 pair, 2 pair + 1) of a noisy draft row: the
+// Box-Muller transform (Box and Muller, 1958) of the 53-bit uniforms of words (0,1) and
+// (2,3) of purpose 3 + pair, radius sqrt(-2 ln(1 - u1)), angle 2 pi u2, in fp64.
+__device__ inline double2 normal_pair(unsigned long long seed, uint32_t stream, uint32_t frame, int round,
+                                      int position, int pair) {
+  uint32_t c[4] = {stream, frame, ((uint32_t)round << 8) | (uint32_t)position, (uint32_t)(PURPOSE_NOISE + pair)};
+  philox4x32_10(c, (uint32_t)seed, (uint32_t)(seed >> 32));
+  const double u1 = ((double)(c[0] >> 5) * 67108864.0 + (double)(c[1] >> 6)) * (1.0 / 9007199254740992.0);
+  const double u2 = ((double)(c[2] >> 5) * 67108864.0 + (double)(c[3] >> 6)) * (1.0 / 9007199254740992.0);
+  const double r = sqrt(-2.0 * log(1.0 - u1));
+  const double t = 2.0 * 3.141592653589793 * u2;
+  double sn, cs;
+  sincos(t, &sn, &cs);
+  return make_double2(r * cs, r * sn);
+}
 
 // ---------------------------------------------------------------------------------------
 // Bounded waits: every spin gives up after wait_ns and records MCD_ERR_TIMEOUT.

@@ -12,7 +12,8 @@ from __future__ import annotations
 import numpy as np
 
 from paper_2609_37007_gb300 import mcd
-from oracle.frame import Sampling, sample_drafts, verify_round
+from paper_2609_37007_gb300.synth import DRAFT_NOISY_TARGET
+from oracle.frame import Sampling, sample_drafts, to_f32, verify_round
 
 
 def check_trace_against_oracle(cfg, model, fr, stream_id, frame_idx, trace_u8, codes, n_calls,
@@ -60,13 +61,30 @@ def check_trace_against_oracle(cfg, model, fr, stream_id, frame_idx, trace_u8, c
         n_next = int(r["n_next"])
         assert n_next == min(K, P - a_new)
         z_rows = []
-        for j in range(1, n_next + 1):
-            ref = model.draft_logits(a_new, j, h[a_new])
-            got = dlog[c, j - 1].astype(np.float64)
-            err = float(np.max(np.abs(got - ref)))
-            max_err = max(max_err, err)
-            assert err <= logit_tol, f"call {c} draft {j}: logits differ by {err}"
-            z_rows.append(dlog[c, j - 1].copy())
+        gpu_next = [int(v) for v in r["next_drafts"][:n_next]]
+        if S.mode == DRAFT_NOISY_TARGET:
+            # noisy-target rows: one-row passes on a copy of the KV cache, fed the GPU's
+            # drafts (Sec. 2.2 chain), plus the counter-based Gaussian noise
+            kv2 = kv.copy()
+            prev = emitted[-1]
+            for j in range(1, n_next + 1):
+                s = a_new + j
+                hs = model.row(kv2, model.code_row(s - 1, prev), s)
+                ref = S.noisy(to_f32(model.verify_logits(s, hs)), c, s).astype(np.float64)
+                got = dlog[c, j - 1].astype(np.float64)
+                err = float(np.max(np.abs(got - ref)))
+                max_err = max(max_err, err)
+                assert err <= logit_tol, f"call {c} noisy draft {j}: logits differ by {err}"
+                z_rows.append(dlog[c, j - 1].copy())
+                prev = gpu_next[j - 1]
+        else:
+            for j in range(1, n_next + 1):
+                ref = model.draft_logits(a_new, j, h[a_new])
+                got = dlog[c, j - 1].astype(np.float64)
+                err = float(np.max(np.abs(got - ref)))
+                max_err = max(max_err, err)
+                assert err <= logit_tol, f"call {c} draft {j}: logits differ by {err}"
+                z_rows.append(dlog[c, j - 1].copy())
         nd = sample_drafts(S, c, a_new, z_rows)
         prev_next = [d for d, _ in nd]
         assert prev_next == [int(v) for v in r["next_drafts"][:n_next]], (c, prev_next, r["next_drafts"])

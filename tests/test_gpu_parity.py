@@ -20,10 +20,11 @@ if not torch.cuda.is_available():
 
 from paper_2609_37007_gb300 import build as _build  # noqa: E402
 from paper_2609_37007_gb300 import mcd  # noqa: E402
-from paper_2609_37007_gb300.synth import (DRAFT_GREEDY, MCD, TINY, make_frame,  # noqa: E402
+from paper_2609_37007_gb300.synth import (DRAFT_GREEDY, DRAFT_NOISY_TARGET, MCD, TINY, make_frame,  # noqa: E402
                                           make_weights, random_logits, weights_as_f32)
 from oracle.enumeration import PrefixModel, ar_distribution, spec_distribution  # noqa: E402
 from oracle.frame import Sampling, decode_frame, verify_round  # noqa: E402
+from oracle import accounting  # noqa: E402
 from oracle.model import Model  # noqa: E402
 from oracle.sampler import topk_dist  # noqa: E402
 from parity import check_trace_against_oracle  # noqa: E402
@@ -221,6 +222,48 @@ def test_tiny_variants_trace_parity(variant):
     env.dec.close()
 
 
+# ------------------------------------------------- noisy-target drafts (K sweep) ------
+@pytest.mark.parametrize("K,sigma", [(1, 0.5), (2, 1.0), (3, 0.25), (7, 2.0)])
+def test_tiny_noisy_target_trace_parity(K, sigma):
+    """Drafts from the target's own logits plus counter-based Gaussian noise (the controlled-
+    acceptance workload): every verify row and every noisy draft row within 1e-5 of the
+    oracle, every decision identical."""
+    cfg = TINY.replace(draft_len=K, n_pos=12 if K > 3 else TINY.n_pos, draft_mode=DRAFT_NOISY_TARGET,
+                       noise_sigma=sigma)
+    env = Env(cfg)
+    for f in range(4):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        check_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=1e-5,
+                                   draft_mode=cfg.draft_mode)
+    env.dec.close()
+
+
+def test_noise_free_target_drafts_are_all_kept_on_gpu():
+    cfg = TINY.replace(draft_len=2, draft_mode=DRAFT_NOISY_TARGET, noise_sigma=0.0)
+    env = Env(cfg)
+    for f in range(3):
+        codes, st, _ = env.decode(make_frame(cfg, f), f)
+        assert int(st[0]) == accounting.chain_calls_per_frame_all_accepted(2, cfg.n_pos)
+        assert int(st[3]) == int(st[2])            # accepted == drafted
+        ref = decode_frame(env.model, make_frame(cfg, f), frame_idx=f)
+        assert list(codes) == ref.codes
+    env.dec.close()
+
+
+def test_mcd_noisy_target_trace_parity_full_size():
+    cfg = MCD.replace(draft_mode=DRAFT_NOISY_TARGET, noise_sigma=1.0)
+    env = Env(cfg)
+    fr = make_frame(cfg, 3)
+    codes, st, tr = env.decode(fr, 3, trace=True)
+    assert st[4] == 0 and st[1] == cfg.n_pos
+    err = check_trace_against_oracle(cfg, env.model, fr, 0, 3, tr, codes, int(st[0]), logit_tol=2e-2,
+                                     draft_mode=cfg.draft_mode)
+    print("mcd noisy max |dlogit|", err)
+    env.dec.close()
+
+
 def test_stepwise_api_matches_decode_frame(tiny):
     cfg = tiny.cfg
     dec = tiny.dec
@@ -241,6 +284,28 @@ def test_stepwise_api_matches_decode_frame(tiny):
         got += emitted.cpu().numpy()[:k].tolist()
     assert got == list(ref)
     assert call == int(st[0])
+
+
+def test_stepwise_api_runs_noisy_target_passes():
+    cfg = TINY.replace(draft_len=2, draft_mode=DRAFT_NOISY_TARGET, noise_sigma=0.5)
+    env = Env(cfg)
+    fr = make_frame(cfg, 5)
+    ref, st, _ = env.decode(fr, 5)
+    cond, c0, emb = env.frame_inputs(fr)
+    mcd.mcd_begin_frame(env.dec.ctx, 0, 5, cond, c0, emb)
+    emitted = torch.zeros(8, dtype=torch.int32, device=DEV)
+    n_em = torch.zeros(1, dtype=torch.int32, device=DEV)
+    got = []
+    for call in range(cfg.n_pos + 1):
+        mcd.mcd_verify_accept(env.dec.ctx, emitted, n_em, None)   # a verify call + its drafting passes
+        mcd.mcd_sync(env.dec.ctx)
+        k = int(n_em.item())
+        if k == 0:
+            break
+        got += emitted.cpu().numpy()[:k].tolist()
+    assert got == list(ref)
+    assert call == int(st[0])
+    env.dec.close()
 
 
 def test_draft_api_matches_oracle(tiny):
