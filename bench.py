@@ -191,6 +191,58 @@ def run_reference(args, cfg, weights):
 
 
 # ----------------------------------------------------------------------------------------
+def run_sweep(args, weights):
+    """Controlled-acceptance sweep: draft length K = 1..7 x noise sigma.  Acceptance (tokens
+    per verify call) comes from frames whose drafts are the target's own logits plus
+    sigma * N(0,1) (noisy-target drafting passes); microseconds per verify call come from
+    timed frames with the position-aware drafter at the same K (the same verify shapes).
+    Prints one JSON line per (K, sigma)."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    from paper_2609_37007_gb300.synth import DRAFT_NOISY_TARGET, MCD, make_frames
+    _build.build()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    n = args.sweep_frames
+    cond_h, c0_h, _ = make_frames(MCD, n + 3, first=2_000_000)
+    cond = torch.from_numpy(cond_h).to(dev)
+    c0 = torch.from_numpy(c0_h).to(dev)
+    codes = torch.zeros((n + 3, MCD.n_pos), dtype=torch.int32, device=dev)
+    stats = torch.zeros((n + 3, 8), dtype=torch.int32, device=dev)
+
+    def frames(dec):
+        for i in range(3):
+            mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+        mcd.mcd_sync(dec.ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(3, n + 3):
+            mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mcd.mcd_sync(dec.ctx)
+        st = stats.cpu().numpy()[3:]
+        assert (st[:, 4] == 0).all() and (st[:, 1] == MCD.n_pos).all()
+        return e0.elapsed_time(e1) * 1e3, int(st[:, 0].sum()), int(st[:, 1].sum())
+
+    for K in range(1, 8):
+        dec = mcd.Decoder(MCD.replace(draft_len=K), weights, stream)
+        t_us, calls, toks = frames(dec)
+        dec.close()
+        us_per_call = t_us / calls
+        for sigma in args.sigmas:
+            dec = mcd.Decoder(MCD.replace(draft_len=K, draft_mode=DRAFT_NOISY_TARGET, noise_sigma=sigma), weights,
+                              stream)
+            _, ncalls, ntoks = frames(dec)
+            dec.close()
+            tpc = ntoks / ncalls
+            print(json.dumps({"sweep": "noisy-target draft length x sigma", "K": K, "sigma": sigma,
+                              "tokens_per_call": tpc, "us_per_verify_call": us_per_call,
+                              "tokens_per_s": tpc / us_per_call * 1e6, "frames": n,
+                              "us_per_call_from": "position-aware drafter frames at the same K"}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -201,6 +253,9 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--ar-frames", type=int, default=200)
     ap.add_argument("--stats-out", default=None, help="write per-frame stats and algorithmic bytes (JSON)")
+    ap.add_argument("--sweep", action="store_true", help="noisy-target K x sigma sweep instead of the bench line")
+    ap.add_argument("--sweep-frames", type=int, default=100)
+    ap.add_argument("--sigmas", type=float, nargs="+", default=[0.05, 0.1, 0.25, 0.5, 1.0, 2.0])
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -209,6 +264,9 @@ def main():
     weights = make_weights(cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, weights)
+    if args.sweep:
+        # one weight set with offsets b_1..b_7 serves every K (extra tensors are ignored)
+        return run_sweep(args, make_weights(cfg.replace(draft_len=7)))
 
     import torch
     from paper_2609_37007_gb300 import build as _build
