@@ -81,6 +81,8 @@ typedef struct {
                          * same frame launch) plus noise_sigma * N(0,1) per entry            */
   float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only (>= 0)                            */
   uint64_t seed;        /* Philox key                                                    */
+  int32_t max_streams;  /* streams one mcd_decode_frames call may decode together (1..8;
+                         * max_streams * max(K + 1, 2) <= 8; NOISY_TARGET needs 1)       */
 } mcd_config;
 
 /* Per-frame counters written by the device (device memory, caller-owned). */
@@ -143,6 +145,24 @@ mcd_status mcd_load_weights(mcd_ctx* ctx, int32_t n, const char* const* names,
 mcd_status mcd_decode_frame(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx,
                             const float* cond, const int32_t* c0, const float* c0_emb,
                             int32_t* codes_out, mcd_frame_stats* stats);
+
+/* Batched streams: decode one frame for each of n_streams (1..max_streams) independent
+ * streams in one launch.  The streams advance in lock step, one call at a time; every
+ * call packs the rows of every stream whose frame is not complete into one operand
+ * (re-packed each call, since streams accept different numbers of drafts), streams the
+ * backbone once and the union of the LM heads the streams need, and runs each stream's
+ * acceptance on its own CTA.  Stream s uses the Philox counters of (stream_ids[s],
+ * frame_idx[s]) and its own KV cache, so its codes are those a single-stream
+ * mcd_decode_frame would emit from the same logits.
+ *   stream_ids, frame_idx  host uint32 [n_streams]
+ *   cond      dev float [n_streams, hidden] (16-byte aligned rows)
+ *   c0        dev int32 [n_streams] (c0_vocab > 0) or c0_emb dev float [n_streams, hidden]
+ *   codes_out dev int32 [n_streams, n_pos]; stats dev mcd_frame_stats [n_streams], optional.
+ * Tracing (mcd_set_trace) records every stream: stream s's block starts at byte
+ * s * mcd_trace_bytes() / max_streams. */
+mcd_status mcd_decode_frames(mcd_ctx* ctx, int32_t n_streams, const uint32_t* stream_ids,
+                             const uint32_t* frame_idx, const float* cond, const int32_t* c0,
+                             const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats);
 
 /* mcd_decode_frame on host buffers: cond (host float [hidden]), c0 (host int32 [1]) or
  * c0_emb (host float [hidden]) are copied to the context's device staging area, the

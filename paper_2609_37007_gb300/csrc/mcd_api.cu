@@ -106,9 +106,10 @@ __global__ void rope_kernel(float2* rope, int D, double base) {
   }
 }
 
-__global__ void begin_frame_kernel(DevState* st, unsigned* ctr, int n_ctr, const int* c0, int C0V) {
+__global__ void begin_frame_kernel(DevState* sts, unsigned* ctr, int n_ctr, const int* c0, int C0V, int S) {
   for (int i = threadIdx.x; i < n_ctr; i += blockDim.x) ctr[i] = 0u;
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < S) {
+    DevState* st = sts + threadIdx.x;
     st->call = 0;
     st->a = 0;
     st->done = 0;
@@ -123,7 +124,7 @@ __global__ void begin_frame_kernel(DevState* st, unsigned* ctr, int n_ctr, const
     st->emu_n = 0;
     st->emu_in = -1;
     for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
-    st->codes[0] = C0V > 0 ? c0[0] : -1;
+    st->codes[0] = C0V > 0 ? c0[threadIdx.x] : -1;
     for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
     st->n_emit_last = 0;
     st->calls = st->drafted = st->accepted = 0;
@@ -186,7 +187,7 @@ __global__ void __launch_bounds__(kConsumerThreads) accept_logits_kernel(FramePa
     for (int i = 0; i < n_d; ++i) drafts[i] = draft_ids[i];
     AcceptResult r = warp_accept(
         a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(recs + i); },
-        [&](int i) { return (const TopkRec*)(recs + kMaxRows + i); }, p.seed, p.stream_id, p.frame_idx, call);
+        [&](int i) { return (const TopkRec*)(recs + kMaxRows + i); }, p.seed, p.stream_ids[0], p.frame_ids[0], call);
     if (threadIdx.x == 0) {
       for (int t = 0; t < r.n_emit; ++t) emitted[t] = r.emitted[t];
       out2[0] = r.n_acc;
@@ -224,7 +225,7 @@ __global__ void __launch_bounds__(kConsumerThreads) draft_sample_kernel(FramePar
   consumer_sync();
   __threadfence_block();
   if (threadIdx.x < 32) {
-    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, call, pos_k + j, PURPOSE_DRAFT);
+    const unsigned long long U = uniform_U(p.seed, p.stream_ids[0], p.frame_ids[0], call, pos_k + j, PURPOSE_DRAFT);
     const int d = warp_draw(r, U);
     if (threadIdx.x == 0) draft_ids[j - 1] = d;
   }
@@ -321,6 +322,10 @@ static mcd_status validate_config(const mcd_config& c) {
   if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
+  if (c.max_streams < 1 || c.max_streams > kMaxStreams) return MCD_ERR_UNSUPPORTED;
+  // every stream's rows of one call are packed into one operand of kMaxRows columns
+  if (c.max_streams * std::max(c.draft_len + 1, 2) > kMaxRows) return MCD_ERR_UNSUPPORTED;
+  if (c.max_streams > 1 && c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;
   if ((long long)c.n_q_heads * c.head_dim + 2LL * c.n_kv_heads * c.head_dim > 8192) return MCD_ERR_UNSUPPORTED;
   return MCD_OK;
 }
@@ -395,6 +400,8 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.qkv_dim = p.NH * p.D + 2 * p.NKV * p.D;
   p.n_cta = n_sm;
   p.wait_ns = 2000000000ull;  // 2 s
+  p.S = 1;
+  p.trace_stride = (long long)sizeof(mcd_call_trace) * kMaxCalls + (long long)2 * kMaxCalls * kMaxRows * p.V * 4;
   const char* wn = getenv("MCD_WAIT_NS");
   if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
 
@@ -450,13 +457,14 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxRows * p.F)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxRows * (kMaxDraft + 1) * p.V)) != cudaSuccess)
     return fail(cuda_status(e));
-  const size_t kvsz = sizeof(float) * (size_t)p.L * p.NKV * kMaxPos * p.D;
+  p.kv_stride = (long long)p.L * p.NKV * kMaxPos * p.D;
+  const size_t kvsz = sizeof(float) * (size_t)p.kv_stride * k.max_streams;
   if ((e = ctx_alloc(c, &p.kcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.vcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * 2 * kMaxRows * (kMaxDraft + 1))) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.draftq, sizeof(TopkRec) * (kMaxDraft + 1))) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.st, sizeof(DevState))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.st, sizeof(DevState) * k.max_streams)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxSlots * p.ctr_stride)) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
@@ -464,7 +472,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.vcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
-  if (cudaMemsetAsync(p.st, 0, sizeof(DevState), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaMemsetAsync(p.st, 0, sizeof(DevState) * k.max_streams, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base);
   if (cudaGetLastError() != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -624,10 +632,11 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
   return s;
 }
 
-static mcd_status launch_begin(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
-                               const int32_t* c0, const float* c0_emb) {
+static mcd_status launch_begin(mcd_ctx* c, int n, const uint32_t* stream_ids, const uint32_t* frame_ids,
+                               const float* cond, const int32_t* c0, const float* c0_emb) {
   FrameParams& p = c->fp;
-  if (!cond) return MCD_ERR_INVALID_ARG;
+  if (!cond || n < 1 || !stream_ids || !frame_ids) return MCD_ERR_INVALID_ARG;
+  if (n > c->cfg.max_streams) return MCD_ERR_INVALID_ARG;
   // the kernel reads these rows with 16-byte loads
   if ((reinterpret_cast<uintptr_t>(cond) & 15u) || (reinterpret_cast<uintptr_t>(c0_emb) & 15u))
     return MCD_ERR_INVALID_ARG;
@@ -636,19 +645,23 @@ static mcd_status launch_begin(mcd_ctx* c, uint32_t stream_id, uint32_t frame_id
   p.cond = cond;
   p.c0 = c0;
   p.c0emb = c0_emb;
-  p.stream_id = stream_id;
-  p.frame_idx = frame_idx;
-  begin_frame_kernel<<<1, 256, 0, c->stream>>>(p.st, p.ctr, kMaxSlots * p.ctr_stride, c0, p.C0V);
+  p.S = n;
+  for (int s = 0; s < kMaxStreams; ++s) {
+    p.stream_ids[s] = s < n ? stream_ids[s] : 0u;
+    p.frame_ids[s] = s < n ? frame_ids[s] : 0u;
+  }
+  begin_frame_kernel<<<1, 256, 0, c->stream>>>(p.st, p.ctr, kMaxSlots * p.ctr_stride, c0, p.C0V, n);
   MCD_CHECK(cudaGetLastError());
   c->frame_begun = true;
   return MCD_OK;
 }
 
-mcd_status mcd_decode_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
-                            const int32_t* c0, const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats) {
+mcd_status mcd_decode_frames(mcd_ctx* c, int32_t n_streams, const uint32_t* stream_ids, const uint32_t* frame_idx,
+                             const float* cond, const int32_t* c0, const float* c0_emb, int32_t* codes_out,
+                             mcd_frame_stats* stats) {
   if (!c || !codes_out) return MCD_ERR_INVALID_ARG;
   if (!c->weights_loaded) return MCD_ERR_STATE;
-  mcd_status s = launch_begin(c, stream_id, frame_idx, cond, c0, c0_emb);
+  mcd_status s = launch_begin(c, n_streams, stream_ids, frame_idx, cond, c0, c0_emb);
   if (s != MCD_OK) return s;
   FrameParams p = c->fp;
   p.codes_out = codes_out;
@@ -659,6 +672,11 @@ mcd_status mcd_decode_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, 
   p.n_emitted_out = nullptr;
   MCD_CHECK(launch_frame_kernel(p, c->stream));
   return MCD_OK;
+}
+
+mcd_status mcd_decode_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
+                            const int32_t* c0, const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats) {
+  return mcd_decode_frames(c, 1, &stream_id, &frame_idx, cond, c0, c0_emb, codes_out, stats);
 }
 
 mcd_status mcd_decode_frame_host(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond,
@@ -690,7 +708,7 @@ mcd_status mcd_decode_frame_host(mcd_ctx* c, uint32_t stream_id, uint32_t frame_
 mcd_status mcd_begin_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond, const int32_t* c0,
                            const float* c0_emb) {
   if (!c) return MCD_ERR_INVALID_ARG;
-  return launch_begin(c, stream_id, frame_idx, cond, c0, c0_emb);
+  return launch_begin(c, 1, &stream_id, &frame_idx, cond, c0, c0_emb);
 }
 
 mcd_status mcd_verify_accept(mcd_ctx* c, int32_t* emitted, int32_t* n_emitted, float* logits_out) {
@@ -755,7 +773,7 @@ mcd_status mcd_topk_softmax(mcd_ctx* c, int32_t n_rows, const float* logits, int
 
 int64_t mcd_trace_bytes(const mcd_ctx* c) {
   if (!c) return 0;
-  return (int64_t)sizeof(mcd_call_trace) * kMaxCalls + (int64_t)2 * kMaxCalls * kMaxRows * c->fp.V * 4;
+  return c->fp.trace_stride * c->cfg.max_streams;
 }
 
 mcd_status mcd_set_trace(mcd_ctx* c, void* trace) {

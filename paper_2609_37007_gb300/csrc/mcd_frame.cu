@@ -2,6 +2,11 @@
 // speculative decoding (arXiv 2609.37007, Sec. 2.2 and Fig. 3) in a single cooperative
 // launch with one CTA per SM.
 //
+// A launch decodes one frame for each of S streams (S = 1 for single-stream decoding); the
+// streams advance in lock step, one call (round) at a time, and every call packs the rows of
+// every stream whose frame is not finished into one operand (re-packed each round, since
+// streams accept different numbers of drafts).
+//
 // Per call (a "round"): the rows [c_a, d_{a+1}, ..., d_{a+n}] (first call: [cond, c0]) go
 // through the MultiCodeDecoder (5 pre-norm layers: RMSNorm -> QKV -> QK-norm -> RoPE ->
 // causal GQA attention over the per-frame KV cache -> Wo + residual -> RMSNorm ->
@@ -26,6 +31,26 @@
 
 namespace mcd {
 
+// Snapshot of one call: the packed rows and every stream's state.
+struct CallInfo {
+  int call;                    // slot (counter set) of this pass
+  int M;                       // packed rows
+  int n_act;                   // streams with rows in this call
+  int n_heads;                 // LM heads streamed
+  int heads[16];               // their positions P
+  int emu, round0;             // noisy-target pass flag, stream 0's verify round (S = 1)
+  int all_done;
+  // packed rows
+  int r_s[kMaxRows], r_n[kMaxRows], r_pos[kMaxRows], r_id[kMaxRows];
+  // per stream (index = stream)
+  int act[kMaxStreams];        // active streams in packing order
+  int a[kMaxStreams], nd[kMaxStreams], pos0[kMaxStreams], nrows[kMaxStreams], fr[kMaxStreams];
+  int done[kMaxStreams], qrow[kMaxStreams], base[kMaxStreams], round[kMaxStreams], emu_n[kMaxStreams];
+  int plo[kMaxStreams], phi[kMaxStreams];
+  int calls[kMaxStreams], heads_rd[kMaxStreams], kvrows[kMaxStreams], rowsfed[kMaxStreams];
+  int drafted[kMaxStreams], accepted[kMaxStreams], drafts[kMaxStreams][kMaxDraft], code_a[kMaxStreams];
+};
+
 struct Smem {
   uint8_t* ring;
   float* act;
@@ -37,7 +62,7 @@ struct Smem {
   uint64_t* empty;
   int* flags;      // [0] stop, [1] abort, [2] last-arriver, [3] current head / chunk
   float* inv_rms;  // [kMaxRows]
-  int* call_info;  // snapshot of the call's state
+  CallInfo* ci;    // snapshot of the call's state
 };
 
 constexpr int kRingOff = 0;
@@ -51,12 +76,7 @@ constexpr int kBarOff = kPartOff + kConsumerWarps * kMaxRows * 4;
 constexpr int kFlagOff = kBarOff + 2 * kNumSlots * 8;
 constexpr int kRmsOff = kFlagOff + 64;
 constexpr int kInfoOff = kRmsOff + 64;
-constexpr int kInfoInts = 48;
-constexpr int kSmemBytes = kInfoOff + kInfoInts * 4;
-
-// call_info slots
-enum { CI_CALL = 0, CI_A, CI_ND, CI_POS0, CI_NROWS, CI_FR, CI_DONE, CI_QROW, CI_PLO, CI_PHI, CI_IDS = 16,
-       CI_CALLS = 24, CI_HEADS, CI_KVROWS, CI_ROWSFED, CI_DRAFTED, CI_ACCEPTED, CI_ROUND, CI_EMU, CI_EMUN };
+constexpr int kSmemBytes = kInfoOff + (int)((sizeof(CallInfo) + 15) / 16 * 16);
 
 __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   Smem s;
@@ -70,7 +90,7 @@ __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   s.empty = s.full + kNumSlots;
   s.flags = reinterpret_cast<int*>(base + kFlagOff);
   s.inv_rms = reinterpret_cast<float*>(base + kRmsOff);
-  s.call_info = reinterpret_cast<int*>(base + kInfoOff);
+  s.ci = reinterpret_cast<CallInfo*>(base + kInfoOff);
   return s;
 }
 
@@ -85,12 +105,13 @@ __device__ __forceinline__ int stage_units(const FrameParams& p, int si, int n_h
   return kind == MAT_HEAD ? n_heads * p.g[MAT_HEAD].n_units : p.g[kind].n_units;
 }
 
-__device__ __forceinline__ const uint8_t* unit_src(const FrameParams& p, int si, int u, int p_lo) {
+// `heads` lists the positions P of the LM heads the call streams (heads stage only).
+__device__ __forceinline__ const uint8_t* unit_src(const FrameParams& p, int si, int u, const int* heads) {
   const int kind = stage_kind(si, p.L);
   const MatGeom& g = p.g[kind];
   if (kind == MAT_HEAD) {
     const int hi = u / g.n_units, uu = u % g.n_units;
-    return p.w_head + (long long)(p_lo + hi - 1) * g.stride + (long long)uu * g.unit_bytes;
+    return p.w_head + (long long)(heads[hi] - 1) * g.stride + (long long)uu * g.unit_bytes;
   }
   const int layer = si >> 2;
   const uint8_t* base = kind == MAT_QKV ? p.w_qkv : kind == MAT_WO ? p.w_wo : kind == MAT_GU ? p.w_gu : p.w_wd;
@@ -125,6 +146,20 @@ __device__ __forceinline__ void head_range(const FrameParams& p, int a, int pos0
   p_hi = p.draft_mode == MCD_DRAFT_NOISY_TARGET ? pos0 + n_rows - 1 : min(p.P, pos0 + n_rows - 1 + p.K);
 }
 
+// LM heads one call streams: the union over the streams with rows in the call, as a bit
+// mask over positions (bit P).
+__device__ __forceinline__ unsigned call_heads_mask(const FrameParams& p) {
+  unsigned mask = 0;
+  for (int s = 0; s < p.S; ++s) {
+    const DevState* st = p.st + s;
+    if (__ldcg(&st->done)) continue;
+    int lo, hi;
+    head_range(p, __ldcg(&st->a), __ldcg(&st->pos0), __ldcg(&st->n_rows), __ldcg(&st->emu), lo, hi);
+    for (int P = lo; P <= hi; ++P) mask |= 1u << P;
+  }
+  return mask;
+}
+
 // ------------------------------------------------------------------------------------
 // Producer: one thread streams this CTA's units into the ring.
 // ------------------------------------------------------------------------------------
@@ -136,7 +171,7 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
   volatile int* stop = sm.flags;
   bool halt = false;
   for (int call = call0; call < kMaxSlots && !halt; ++call) {
-    int p_lo = 0, p_hi = -1;
+    int heads[16];
     for (int si = 0; si < n_stages(p) && !halt; ++si) {
       int n_heads = 0;
       if (stage_kind(si, p.L) == MAT_HEAD) {
@@ -146,15 +181,15 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
             break;
           }
         }
-        const int4 s0 = __ldcg(reinterpret_cast<const int4*>(p.st));        // call, a, done, n_d
-        const int2 s1 = __ldcg(reinterpret_cast<const int2*>(p.st) + 2);    // pos0, n_rows
-        const int emu = __ldcg(&p.st->emu);
-        if (s0.z) {
+        unsigned mask = call_heads_mask(p);
+        if (!mask) {                       // every stream's frame is complete
           halt = true;
           break;
         }
-        head_range(p, s0.y, s1.x, s1.y, emu, p_lo, p_hi);
-        n_heads = p_hi - p_lo + 1;
+        while (mask) {
+          heads[n_heads++] = __ffs(mask) - 1;
+          mask &= mask - 1;
+        }
       }
       const int n = stage_units(p, si, n_heads);
       const uint32_t bytes = (uint32_t)p.g[stage_kind(si, p.L)].unit_bytes;
@@ -168,7 +203,7 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
           }
         }
         mbar_arrive_expect_tx(&sm.full[slot], bytes);
-        bulk_g2s(sm.ring + (size_t)slot * kSlotBytes, unit_src(p, si, u, p_lo), bytes, &sm.full[slot], pol);
+        bulk_g2s(sm.ring + (size_t)slot * kSlotBytes, unit_src(p, si, u, heads), bytes, &sm.full[slot], pol);
         ++issued;
       }
       rot = (rot + n) % n_cta;
@@ -213,15 +248,15 @@ struct Cons {
 constexpr int kTimelineSlots = 128;
 // (Indexed by verify round; noisy-target passes are not stamped.)
 __device__ __forceinline__ void timeline(const Cons& c, int, int idx, bool any_cta = false) {
-  const int* ci = c.sm.call_info;
-  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots && !ci[CI_EMU] &&
-      ci[CI_ROUND] < kMaxCalls)
-    c.p.timeline[ci[CI_ROUND] * kTimelineSlots + idx] = globaltimer();
+  const CallInfo* ci = c.sm.ci;
+  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots && !ci->emu &&
+      ci->round0 < kMaxCalls)
+    c.p.timeline[ci->round0 * kTimelineSlots + idx] = globaltimer();
 }
 __device__ __forceinline__ void timeline_max(const Cons& c, int, int idx) {
-  const int* ci = c.sm.call_info;
-  if (c.p.timeline && threadIdx.x == 0 && idx < kTimelineSlots && !ci[CI_EMU] && ci[CI_ROUND] < kMaxCalls)
-    atomicMax(c.p.timeline + ci[CI_ROUND] * kTimelineSlots + idx, (unsigned long long)globaltimer());
+  const CallInfo* ci = c.sm.ci;
+  if (c.p.timeline && threadIdx.x == 0 && idx < kTimelineSlots && !ci->emu && ci->round0 < kMaxCalls)
+    atomicMax(c.p.timeline + ci->round0 * kTimelineSlots + idx, (unsigned long long)globaltimer());
 }
 
 __device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned target) {
@@ -457,25 +492,25 @@ __device__ __forceinline__ void g2s_vec(float* dst, const float* src, int n) {
 __device__ __forceinline__ float2 ld_global2(const float* q) { return __ldcg(reinterpret_cast<const float2*>(q)); }
 __device__ __forceinline__ float2 ld_shared2(const float* q) { return *reinterpret_cast<const float2*>(q); }
 
-// Layer-0 input rows of the call into act[n][H]: [cond, c0] on the first call, else the
-// embeddings of [c_a, d_{a+1}, ...] (table of position a+i).  CTA 0 also seeds the residual
-// stream x in global memory.
-__device__ void gather_inputs(Cons& c) {
+// Layer-0 input rows of the call into act[r][H] (packed row r of stream s): [cond, c0] on a
+// stream's first call, else the embeddings of [c_a, d_{a+1}, ...] (table of position a+i).
+// CTA 0 also seeds the residual stream x in global memory.
+__device__ __forceinline__ void gather_inputs(Cons& c) {
   const FrameParams& p = c.p;
-  const int* ci = c.sm.call_info;
-  const int n_rows = ci[CI_NROWS], pos0 = ci[CI_POS0];
+  const CallInfo* ci = c.sm.ci;
+  const int M = ci->M;
   const int H = p.H, per = H / 8;      // 8 elements (16 B of bf16 or 2x16 B of fp32) per item
-  for (int it = threadIdx.x; it < n_rows * per; it += kConsumerThreads) {
-    const int n = it / per, k0 = (it - n * per) * 8;
-    const int pos = pos0 + n;
+  for (int it = threadIdx.x; it < M * per; it += kConsumerThreads) {
+    const int r = it / per, k0 = (it - r * per) * 8;
+    const int s = ci->r_s[r], pos = ci->r_pos[r];
     float v[8];
     if (pos == 0 || (pos == 1 && p.C0V == 0)) {
-      const float4* src = reinterpret_cast<const float4*>((pos == 0 ? p.cond : p.c0emb) + k0);
+      const float4* src = reinterpret_cast<const float4*>((pos == 0 ? p.cond : p.c0emb) + (size_t)s * H + k0);
       const float4 a = __ldg(src), b = __ldg(src + 1);
       v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
     } else {
       const int table = pos - 1;
-      int id = ci[CI_IDS + n];
+      int id = ci->r_id[r];
       if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {  // a c0 outside table 0: fail the frame
         if (k0 == 0) atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
         id = 0;
@@ -495,11 +530,11 @@ __device__ void gather_inputs(Cons& c) {
         v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
       }
     }
-    float4* dst = reinterpret_cast<float4*>(c.sm.act + n * H + k0);
+    float4* dst = reinterpret_cast<float4*>(c.sm.act + r * H + k0);
     dst[0] = make_float4(v[0], v[1], v[2], v[3]);
     dst[1] = make_float4(v[4], v[5], v[6], v[7]);
     if (blockIdx.x == 0) {
-      float4* gx = reinterpret_cast<float4*>(p.x + (size_t)n * H + k0);
+      float4* gx = reinterpret_cast<float4*>(p.x + (size_t)r * H + k0);
       gx[0] = dst[0];
       gx[1] = dst[1];
     }
@@ -507,8 +542,9 @@ __device__ void gather_inputs(Cons& c) {
   consumer_sync();
 }
 
-// Attention of query head h for the call's rows (QK-norm, RoPE, causal softmax over the
-// per-frame cache plus the new rows); output o[n][D] in act.  Scratch spans act + bfrag
+// Attention of query head h for the nr rows of stream s (packed rows base..base+nr-1; QK-norm,
+// RoPE, causal softmax over the stream's per-frame cache plus the new rows); output
+// o[base + n][D] in act.  Scratch spans act + bfrag
 // (< 64 KB).  Phases, separated by barriers: (A) every input row (q, new k / v, cached
 // k / v, RoPE rows, QK-norm gains) is loaded as independent 16-byte chunks, all in flight at
 // once; (B) one warp per new q / k vector applies QK-norm and RoPE in registers (lane holds
@@ -516,10 +552,8 @@ __device__ void gather_inputs(Cons& c) {
 // writer, stores the new k / v rows to the cache; (C1) two threads per (row, key) score it
 // over interleaved 16-byte chunks (rows padded to D + 8 floats: conflict-free reads); (C2)
 // one warp per row takes the softmax; (C3) one thread per (row, dim pair) sums P.V.
-__device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
+__device__ void attention_stream(Cons& c, int layer, int h, bool write_kv, int nr, int pos0, int base, int s) {
   const FrameParams& p = c.p;
-  const int* ci = c.sm.call_info;
-  const int nr = ci[CI_NROWS], pos0 = ci[CI_POS0];
   const int D = p.D, half = D >> 1, g = h / (p.NH / p.NKV);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cs_shift = D == 128 ? 5 : 4;           // 16-byte chunks per row = D / 4
@@ -532,7 +566,7 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   float2* cs = reinterpret_cast<float2*>(vs + kMaxPos * 128);   // [8][D/2] (cos, sin)
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
   float* gk = gq + 128;                                          // [D]
-  const size_t cache_off = ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
   const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
   // ---- (A) loads ----------------------------------------------------------------------
@@ -552,7 +586,8 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
         if (i < e_v) {
           const int seg = i < e_q ? 0 : (i < e_k ? 1 : 2);
           const int r = i - seg * n_new, n = r >> cs_shift, ch = r & (cpr - 1);
-          src = reinterpret_cast<const float4*>(qkv + (size_t)n * p.qkv_dim + (seg == 0 ? qoff : seg == 1 ? koff : voff)) + ch;
+          src = reinterpret_cast<const float4*>(qkv + (size_t)(base + n) * p.qkv_dim +
+                                                (seg == 0 ? qoff : seg == 1 ? koff : voff)) + ch;
           dst[u] = reinterpret_cast<float4*>(seg == 0 ? qs + n * KS : seg == 1 ? ks + (pos0 + n) * KS : vs + (pos0 + n) * D) + ch;
         } else if (i < e_vc) {
           const bool isk = i < e_kc;
@@ -688,12 +723,22 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
         c0.x += p0 * v0.x;
         c0.y += p0 * v0.y;
       }
-      *reinterpret_cast<float2*>(o + n * D + d) = make_float2(c0.x + c1.x, c0.y + c1.y);
+      *reinterpret_cast<float2*>(o + (base + n) * D + d) = make_float2(c0.x + c1.x, c0.y + c1.y);
     }
   }
   consumer_sync();
 }
 
+
+// Attention of query head h for every stream with rows in the call (outputs at the
+// streams' packed rows).
+__device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
+  const CallInfo* ci = c.sm.ci;
+  for (int i = 0; i < ci->n_act; ++i) {
+    const int s = ci->act[i];
+    attention_stream(c, layer, h, write_kv, ci->nrows[s], ci->pos0[s], ci->base[s], s);
+  }
+}
 
 // ------------------------------------------------------------------------------------
 // One call
@@ -702,10 +747,10 @@ template <int WT>
 __device__ void run_call(Cons& c, int call) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
-  int* ci = sm.call_info;
+  const CallInfo* ci = sm.ci;
   const int L = p.L, H = p.H, D = p.D, F = p.F;
   unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
-  const int n_rows = ci[CI_NROWS];
+  const int n_rows = ci->M;                 // packed rows of every stream in the call
   const unsigned N = (unsigned)p.n_cta;
   const float* x = p.x;
   auto from_x = [&](int n, int k) { return ld_global2(x + (size_t)n * H + k); };
@@ -811,38 +856,40 @@ __device__ void run_call(Cons& c, int call) {
   }
 
   // ---- S5: final RMSNorm -> verify and draft heads ---------------------------------------
-  // Column n of the operand is row n (h_n before its 1/rms); LM head P's output for row n
-  // is verify logits (j = 0) or the draft logits of offset j = P - (pos0 + n) (1 <= j <= K),
-  // whose LMH_P b_j term comes from the precomputed bias table (staged per chunk in `vec`,
-  // which is free once the operand is built).
+  // Operand column r is packed row r (h before its 1/rms).  LM head P's output for row r at
+  // position pos is its verify logits (j = P - pos = 0) or the draft logits of offset j
+  // (1 <= j <= K), whose LMH_P b_j term comes from the precomputed bias table (staged per
+  // chunk in `vec`, which is free once the operand is built).  The call streams the union
+  // of the heads its streams need.
   g2s_vec(sm.vec, p.final_norm, H);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
   prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
   {
     const MatGeom& g = p.g[MAT_HEAD];
-    const int p_lo = ci[CI_PLO], n_heads = ci[CI_PHI] - ci[CI_PLO] + 1;
-    const int fr = ci[CI_FR], pos0 = ci[CI_POS0];
     float* bias_s = sm.vec;   // [kChunk][16 rows][8 columns]
     int chunk_u0 = 0;
     run_stage<WT>(
-        c, call, 4 * L, n_heads * g.n_units, H, n_rows, no_key,
+        c, call, 4 * L, ci->n_heads * g.n_units, H, n_rows, no_key,
         [&](int u0, int cnt, int step) {
           chunk_u0 = u0;
           for (int o = threadIdx.x; o < cnt * 128; o += kConsumerThreads) {
             const int r = o >> 7, rr = (o >> 3) & 15, n = o & 7;
             const int u = u0 + r * step;
-            const int P = p_lo + u / g.n_units, j = P - (pos0 + n);
+            const int P = ci->heads[u / g.n_units];
             float bv = 0.f;
-            if (j >= 1 && j <= p.K && n < n_rows && n >= fr) {
-              const int id = (u % g.n_units) * 16 + rr;
-              bv = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
+            if (n < n_rows) {
+              const int j = P - ci->r_pos[n];
+              if (j >= 1 && j <= p.K && ci->r_pos[n] >= 1) {
+                const int id = (u % g.n_units) * 16 + rr;
+                bv = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
+              }
             }
             bias_s[o] = bv;
           }
         },
         [&](int u, int mi, int rr, int n, float v, float) {
-          const int P = p_lo + u / g.n_units, j = P - (pos0 + n);
-          if (n >= fr && j >= 0 && j <= p.K) {
+          const int P = ci->heads[u / g.n_units], pos = ci->r_pos[n], j = P - pos;
+          if (pos >= 1 && j >= 0 && j <= p.K) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
             p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
                 v * sm.inv_rms[n] + bias_s[(u - chunk_u0) * 128 + rr * 8 + n];
@@ -856,24 +903,24 @@ __device__ void run_call(Cons& c, int call) {
   if (!cons_wait(c, ctr + ctr_heads(L), N)) return;
   timeline(c, call, 1);
   {
-    const int fr = ci[CI_FR], pos0 = ci[CI_POS0], emu = ci[CI_EMU];
     TopkScratch& ts = *reinterpret_cast<TopkScratch*>(sm.act);
-    if (emu) {
-      // noisy-target pass j = emu: q = fp32(target logits + sigma N(0,1)) of position pos0
-      // (Box-Muller pairs of purpose 3 + v/2 under the verify round's counters)
+    if (ci->emu) {
+      // noisy-target pass j = emu (one stream): q = fp32(target logits + sigma N(0,1)) of
+      // position pos0 (Box-Muller pairs of purpose 3 + v/2 under the verify round's counters)
       if (blockIdx.x == 0) {
+        const int emu = ci->emu, pos0 = ci->pos0[0], round = ci->round[0];
         const float* lg = p.logits;                                   // row 0, j = 0
         float* zq = p.logits + (size_t)1 * p.V;                        // row 0, slot j = 1
         for (int pr = threadIdx.x; pr < (p.V >> 1); pr += kConsumerThreads) {
-          const double2 nz = normal_pair(p.seed, p.stream_id, p.frame_idx, ci[CI_ROUND], pos0, pr);
+          const double2 nz = normal_pair(p.seed, p.stream_ids[0], p.frame_ids[0], round, pos0, pr);
           const float2 l = __ldcg(reinterpret_cast<const float2*>(lg) + pr);
           const float2 z = make_float2((float)((double)l.x + (double)p.sigma * nz.x),
                                        (float)((double)l.y + (double)p.sigma * nz.y));
           reinterpret_cast<float2*>(zq)[pr] = z;
-          if (p.trace && ci[CI_ROUND] < kMaxCalls) {
+          if (p.trace && round < kMaxCalls) {
             float* dlog = reinterpret_cast<float*>(p.trace + sizeof(mcd_call_trace) * kMaxCalls) +
                           (size_t)kMaxCalls * kMaxRows * p.V;
-            reinterpret_cast<float2*>(dlog + ((size_t)ci[CI_ROUND] * kMaxRows + (emu - 1)) * p.V)[pr] = z;
+            reinterpret_cast<float2*>(dlog + ((size_t)round * kMaxRows + (emu - 1)) * p.V)[pr] = z;
           }
         }
         __threadfence();
@@ -885,13 +932,15 @@ __device__ void run_call(Cons& c, int call) {
       TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
       const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
       int pair = 0;
-      for (int n = fr; n < n_rows; ++n) {
-        const int kn = noisy ? 0 : min(p.K, p.P - (pos0 + n));
+      for (int r = 0; r < n_rows; ++r) {
+        const int pos = ci->r_pos[r];
+        if (pos < 1) continue;                        // the conditioning row reads no head
+        const int kn = noisy ? 0 : min(p.K, p.P - pos);
         for (int j = 0; j <= kn; ++j, ++pair) {
           if (pair % p.n_cta != (int)blockIdx.x) continue;
           const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
-          block_topk(p.logits + ((size_t)n * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
-                     recs + n * (kMaxDraft + 1) + j);
+          block_topk(p.logits + ((size_t)r * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
+                     recs + r * (kMaxDraft + 1) + j);
           consumer_sync();
         }
       }
@@ -900,13 +949,25 @@ __device__ void run_call(Cons& c, int call) {
   consumer_sync();
   timeline(c, call, 2);
   timeline_max(c, call, 3);
+  // Every CTA's records must be visible before an acceptance step reads them.  One stream:
+  // the CTA that arrives last runs its acceptance.  Several: CTA b runs the acceptance of
+  // the b-th stream in the call once every CTA has arrived.
   if (threadIdx.x == 0) {
     __threadfence();
     const unsigned old = atomicAdd(ctr + ctr_topk(L), 1u);
-    sm.flags[2] = (old == N - 1u) ? 1 : 0;
-    if (sm.flags[2]) __threadfence();
+    int mine = -1;
+    if (p.S == 1) {
+      if (old == N - 1u) mine = 0;
+    } else if ((int)blockIdx.x < ci->n_act) {
+      if (wait_counter(ctr + ctr_topk(L), N, p.err, p.wait_ns)) mine = ci->act[blockIdx.x];
+      else sm.flags[1] = 1;
+    }
+    if (mine >= 0) __threadfence();
+    sm.flags[2] = mine >= 0 ? 1 : 0;
+    sm.flags[4] = mine;
   }
   consumer_sync();
+  if (*(volatile int*)&sm.flags[1]) c.abort_ = true;
 }
 
 // Copy distribution records into shared memory with independent word loads: the header,
@@ -924,12 +985,13 @@ __device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src
 
 // Acceptance step and next drafts (run by the CTA that finished top-k last).  Every record
 // it reads is first staged in shared memory (act + bfrag, 64 KB).
-__device__ void accept_step(Cons& c, int call) {
+__device__ void accept_step(Cons& c, int call, int s) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
-  const int* ci = sm.call_info;
-  const int a = ci[CI_A], n_d = ci[CI_ND], pos0 = ci[CI_POS0], n_rows = ci[CI_NROWS];
-  const int qrow = ci[CI_QROW], round = ci[CI_ROUND];
+  const CallInfo* ci = sm.ci;
+  const int a = ci->a[s], n_d = ci->nd[s], pos0 = ci->pos0[s], n_rows = ci->nrows[s];
+  const int qrow = ci->qrow[s], round = ci->round[s], base = ci->base[s];
+  const unsigned sid = p.stream_ids[s], fid = p.frame_ids[s];
   const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
@@ -937,21 +999,21 @@ __device__ void accept_step(Cons& c, int call) {
   TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // staged records
   const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
   __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
-  timeline(c, call, 4, true);
-  // p of positions a+1..: this call's verify records; q of the drafts: the previous call's
-  // records of its row qrow, or the noisy-target passes' records
+  if (s == 0) timeline(c, call, 4, true);
+  // p of positions a+1..: this call's verify records (packed rows base + ...); q of the
+  // drafts: the previous call's records of its packed row qrow, or the noisy-target passes'
   stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
-    return r < n_p ? cur + (a + 1 + r - pos0) * (kMaxDraft + 1)
+    return r < n_p ? cur + (base + a + 1 + r - pos0) * (kMaxDraft + 1)
                    : (noisy ? p.draftq + (r - n_p) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p));
   });
   consumer_sync();
-  timeline(c, call, 5, true);
+  if (s == 0) timeline(c, call, 5, true);
   if (warp == 0) {
     int drafts[kMaxDraft + 1];
-    for (int i = 0; i < n_d; ++i) drafts[i] = ci[CI_IDS + 1 + i];
+    for (int i = 0; i < n_d; ++i) drafts[i] = ci->drafts[s][i];
     AcceptResult r = warp_accept(
         a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(srec + i); },
-        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, p.stream_id, p.frame_idx, round);
+        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, sid, fid, round);
     if (lane == 0) {
       for (int t = 0; t < r.n_emit; ++t) s_emit[t] = r.emitted[t];
       s_nemit = r.n_emit;
@@ -959,17 +1021,17 @@ __device__ void accept_step(Cons& c, int call) {
     }
   }
   consumer_sync();
-  timeline(c, call, 6, true);
+  if (s == 0) timeline(c, call, 6, true);
   const int a_new = a + s_nemit;
   const int m = a_new - pos0;
   const int n_next = min(p.K, p.P - a_new);
   // draft records of row m (the row whose head emitted the last code): one warp each (the
   // noisy-target passes that follow draw their drafts themselves)
   if (!noisy) {
-    stage_records(srec, n_next, p.top_k, [&](int r) { return cur + m * (kMaxDraft + 1) + 1 + r; });
+    stage_records(srec, n_next, p.top_k, [&](int r) { return cur + (base + m) * (kMaxDraft + 1) + 1 + r; });
     consumer_sync();
     for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
-      const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, round, a_new + j, PURPOSE_DRAFT);
+      const unsigned long long U = uniform_U(p.seed, sid, fid, round, a_new + j, PURPOSE_DRAFT);
       const int d = warp_draw(srec + j - 1, U);
       if (lane == 0) s_next[j - 1] = d;
     }
@@ -977,17 +1039,18 @@ __device__ void accept_step(Cons& c, int call) {
   }
   if (threadIdx.x == 0) {
     s_nnext = n_next;
-    DevState* st = p.st;
+    DevState* st = p.st + s;
+    int* codes_out = p.codes_out ? p.codes_out + (size_t)s * p.P : nullptr;
     for (int t = 0; t < s_nemit; ++t) {
       st->codes[a + 1 + t] = s_emit[t];
-      if (p.codes_out) p.codes_out[a + t] = s_emit[t];
+      if (codes_out) codes_out[a + t] = s_emit[t];
     }
     if (!noisy)
       for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
     for (int t = 0; t < s_nemit; ++t) st->emitted_last[t] = s_emit[t];
-    const int calls = ci[CI_CALLS] + 1, heads = ci[CI_HEADS] + ci[CI_PHI] - ci[CI_PLO] + 1;
-    const int kvr = ci[CI_KVROWS] + pos0 + n_rows, rf = ci[CI_ROWSFED] + n_rows;
-    const int drafted = ci[CI_DRAFTED] + n_d, accepted = ci[CI_ACCEPTED] + s_nacc;
+    const int calls = ci->calls[s] + 1, heads = ci->heads_rd[s] + ci->phi[s] - ci->plo[s] + 1;
+    const int kvr = ci->kvrows[s] + pos0 + n_rows, rf = ci->rowsfed[s] + n_rows;
+    const int drafted = ci->drafted[s] + n_d, accepted = ci->accepted[s] + s_nacc;
     st->n_emit_last = s_nemit;
     st->n_acc_last = s_nacc;
     st->a = a_new;
@@ -1013,35 +1076,37 @@ __device__ void accept_step(Cons& c, int call) {
     st->accepted = accepted;
     st->call = call + 1;
     st->done = a_new >= p.P ? 1 : 0;
-    st->q_row = m;  // q of the next call's drafts: this call's records of row m
+    st->q_row = base + m;  // q of the next call's drafts: this call's records of packed row base + m
     if (p.single_call) {
       if (p.emitted_out)
         for (int t = 0; t < s_nemit; ++t) p.emitted_out[t] = s_emit[t];
       if (p.n_emitted_out) *p.n_emitted_out = s_nemit;
     }
     if (a_new >= p.P && p.stats) {
-      p.stats->calls = calls;
-      p.stats->codes = a_new;
-      p.stats->drafted = drafted;
-      p.stats->accepted = accepted;
-      p.stats->status = 0;
-      p.stats->heads_read = heads;
-      p.stats->kv_rows = kvr;
-      p.stats->rows_fed = rf;
+      mcd_frame_stats* fs = p.stats + s;
+      fs->calls = calls;
+      fs->codes = a_new;
+      fs->drafted = drafted;
+      fs->accepted = accepted;
+      fs->status = 0;
+      fs->heads_read = heads;
+      fs->kv_rows = kvr;
+      fs->rows_fed = rf;
     }
   }
   consumer_sync();
   // optional outputs: trace and stepwise logits
-  const int fr = ci[CI_FR];
-  if (p.trace) {
-    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(p.trace) + round;
+  const int fr = ci->fr[s];
+  if (p.trace && round < kMaxCalls) {
+    uint8_t* tb = p.trace + (size_t)s * p.trace_stride;
+    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(tb) + round;
     if (threadIdx.x == 0) {
       tr->a = a;
       tr->n_rows = n_rows;
       tr->pos0 = pos0;
       tr->n_drafts = n_d;
-      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci[CI_IDS + n] : -1;
-      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? ci[CI_IDS + 1 + i] : -1;
+      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci->r_id[base + n] : -1;
+      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? ci->drafts[s][i] : -1;
       tr->n_acc = s_nacc;
       tr->n_emit = s_nemit;
       for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < s_nemit ? s_emit[t] : -1;
@@ -1049,28 +1114,34 @@ __device__ void accept_step(Cons& c, int call) {
       for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = (j < s_nnext && !noisy) ? s_next[j] : -1;
       tr->draft_row = m;
     }
-    float* vlog = reinterpret_cast<float*>(p.trace + sizeof(mcd_call_trace) * kMaxCalls);
+    float* vlog = reinterpret_cast<float*>(tb + sizeof(mcd_call_trace) * kMaxCalls);
     float* dlog = vlog + (size_t)kMaxCalls * kMaxRows * p.V;
     for (int idx = threadIdx.x; idx < kMaxRows * p.V; idx += kConsumerThreads) {
       const int n = idx / p.V, v = idx - n * p.V;
       if (n >= fr && n < n_rows)
-        vlog[((size_t)round * kMaxRows + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+        vlog[((size_t)round * kMaxRows + n) * p.V + v] =
+            __ldcg(p.logits + ((size_t)(base + n) * (kMaxDraft + 1)) * p.V + v);
       if (n < s_nnext && !noisy)
         dlog[((size_t)round * kMaxRows + n) * p.V + v] =
-            __ldcg(p.logits + ((size_t)m * (kMaxDraft + 1) + n + 1) * p.V + v);
+            __ldcg(p.logits + ((size_t)(base + m) * (kMaxDraft + 1) + n + 1) * p.V + v);
     }
   }
   if (p.single_call && p.logits_out) {
     for (int idx = threadIdx.x; idx < (n_rows - fr) * p.V; idx += kConsumerThreads) {
       const int n = fr + idx / p.V, v = idx % p.V;
-      p.logits_out[idx] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+      p.logits_out[idx] = __ldcg(p.logits + ((size_t)(base + n) * (kMaxDraft + 1)) * p.V + v);
     }
   }
   consumer_sync();
-  timeline(c, call, 7, true);
+  if (s == 0) timeline(c, call, 7, true);
   if (threadIdx.x == 0) {
+    // the last acceptance of the call releases the next call
     __threadfence();
-    atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+    unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
+    if (atomicAdd(ctr + ctr_accept(p.L), 1u) == (unsigned)ci->n_act - 1u) {
+      __threadfence();
+      atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+    }
   }
 }
 
@@ -1080,15 +1151,15 @@ __device__ void accept_step(Cons& c, int call) {
 __device__ void emu_step(Cons& c, int call) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
-  const int* ci = sm.call_info;
-  const int j = ci[CI_EMU], n = ci[CI_EMUN], round = ci[CI_ROUND], pos0 = ci[CI_POS0], a = ci[CI_A];
+  const CallInfo* ci = sm.ci;
+  const int j = ci->emu, n = ci->emu_n[0], round = ci->round[0], pos0 = ci->pos0[0], a = ci->a[0];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);
   __shared__ int s_d;
   stage_records(srec, 1, p.top_k, [&](int) { return p.draftq + (j - 1); });
   consumer_sync();
   if (warp == 0) {
-    const unsigned long long U = uniform_U(p.seed, p.stream_id, p.frame_idx, round, pos0, PURPOSE_DRAFT);
+    const unsigned long long U = uniform_U(p.seed, p.stream_ids[0], p.frame_ids[0], round, pos0, PURPOSE_DRAFT);
     const int d = warp_draw(srec, U);
     if (lane == 0) s_d = d;
   }
@@ -1123,46 +1194,65 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
   if (!first) {
     if (!cons_wait(c, p.ctr + (size_t)call * p.ctr_stride + ctr_ready(p.L), 1u)) return false;
   }
-  // one parallel read of the whole state (sizeof(DevState) / 4 words) into the act region
+  // one parallel read of every stream's state into the act region
   constexpr int kWords = sizeof(DevState) / 4;
   int* stw = reinterpret_cast<int*>(sm.act);
-  for (int i = threadIdx.x; i < kWords; i += kConsumerThreads) stw[i] = __ldcg(reinterpret_cast<const int*>(p.st) + i);
+  for (int i = threadIdx.x; i < p.S * kWords; i += kConsumerThreads)
+    stw[i] = __ldcg(reinterpret_cast<const int*>(p.st) + i);
   consumer_sync();
   if (threadIdx.x == 0) {
-    const DevState* st = reinterpret_cast<const DevState*>(stw);
-    int* ci = sm.call_info;
-    ci[CI_CALL] = call;
-    ci[CI_A] = st->a;
-    ci[CI_ND] = st->n_d;
-    ci[CI_POS0] = st->pos0;
-    ci[CI_NROWS] = st->n_rows;
-    ci[CI_FR] = st->first_head_row;
-    ci[CI_DONE] = st->done;
-    ci[CI_QROW] = st->q_row;
-    ci[CI_CALLS] = st->calls;
-    ci[CI_HEADS] = st->heads_read;
-    ci[CI_KVROWS] = st->kv_rows;
-    ci[CI_ROWSFED] = st->rows_fed;
-    ci[CI_DRAFTED] = st->drafted;
-    ci[CI_ACCEPTED] = st->accepted;
-    ci[CI_ROUND] = st->round;
-    ci[CI_EMU] = st->emu;
-    ci[CI_EMUN] = st->emu_n;
-    int plo, phi;
-    head_range(p, ci[CI_A], ci[CI_POS0], ci[CI_NROWS], ci[CI_EMU], plo, phi);
-    ci[CI_PLO] = plo;
-    ci[CI_PHI] = phi;
-    // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft i-1;
-    // a noisy-target pass feeds its one code
-    const int a = ci[CI_A];
-    for (int i = 0; i < kMaxDraft; ++i) ci[CI_IDS + 1 + i] = st->drafts[i];
-    if (ci[CI_EMU]) {
-      ci[CI_IDS + 0] = st->emu_in;
-    } else if (ci[CI_POS0] == 0) {
-      ci[CI_IDS + 0] = -1;
-      ci[CI_IDS + 1] = st->codes[0];
-    } else {
-      ci[CI_IDS + 0] = st->codes[a];
+    CallInfo* ci = sm.ci;
+    const DevState* sts = reinterpret_cast<const DevState*>(stw);
+    ci->call = call;
+    ci->M = 0;
+    ci->n_act = 0;
+    ci->all_done = 1;
+    ci->emu = sts[0].emu;
+    ci->round0 = sts[0].round;
+    unsigned mask = 0;
+    for (int s = 0; s < p.S; ++s) {
+      const DevState* st = sts + s;
+      ci->done[s] = st->done;
+      ci->a[s] = st->a;
+      ci->nd[s] = st->n_d;
+      ci->pos0[s] = st->pos0;
+      ci->nrows[s] = st->n_rows;
+      ci->fr[s] = st->first_head_row;
+      ci->qrow[s] = st->q_row;
+      ci->round[s] = st->round;
+      ci->emu_n[s] = st->emu_n;
+      ci->calls[s] = st->calls;
+      ci->heads_rd[s] = st->heads_read;
+      ci->kvrows[s] = st->kv_rows;
+      ci->rowsfed[s] = st->rows_fed;
+      ci->drafted[s] = st->drafted;
+      ci->accepted[s] = st->accepted;
+      for (int i = 0; i < kMaxDraft; ++i) ci->drafts[s][i] = st->drafts[i];
+      ci->code_a[s] = st->codes[st->a];
+      if (st->done) continue;
+      ci->all_done = 0;
+      ci->act[ci->n_act++] = s;
+      ci->base[s] = ci->M;
+      int lo, hi;
+      head_range(p, st->a, st->pos0, st->n_rows, st->emu, lo, hi);
+      ci->plo[s] = lo;
+      ci->phi[s] = hi;
+      for (int P = lo; P <= hi; ++P) mask |= 1u << P;
+      // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft
+      // i-1; a noisy-target pass feeds its one code
+      for (int n = 0; n < st->n_rows && ci->M < kMaxRows; ++n) {
+        const int r = ci->M++;
+        ci->r_s[r] = s;
+        ci->r_n[r] = n;
+        ci->r_pos[r] = st->pos0 + n;
+        ci->r_id[r] = st->emu ? st->emu_in
+                              : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+      }
+    }
+    ci->n_heads = 0;
+    while (mask) {
+      ci->heads[ci->n_heads++] = __ffs(mask) - 1;
+      mask &= mask - 1;
     }
   }
   consumer_sync();
@@ -1194,22 +1284,23 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
     Cons c(p, sm);
     for (int call = call0; call < kMaxSlots; ++call) {
       if (!read_call_state(c, call, call == call0)) break;
-      if (sm.call_info[CI_DONE]) break;
+      if (sm.ci->all_done) break;
       // a stepwise launch runs one verify call and the noisy-target passes that follow it
-      if (p.single_call && call != call0 && !sm.call_info[CI_EMU]) break;
+      if (p.single_call && call != call0 && !sm.ci->emu) break;
       run_call<WT>(c, call);
       if (c.abort_) break;
       if (sm.flags[2]) {
-        if (sm.call_info[CI_EMU])
+        if (sm.ci->emu)
           emu_step(c, call);
         else
-          accept_step(c, call);
+          accept_step(c, call, sm.flags[4]);
       }
     }
     if (tid == 0) sm.flags[0] = 1;  // stop the producer
   }
   __syncthreads();
-  if (tid == 0 && *(volatile int*)p.err != 0 && p.stats) p.stats->status = *(volatile int*)p.err;
+  if (tid == 0 && *(volatile int*)p.err != 0 && p.stats)
+    for (int s = 0; s < p.S; ++s) p.stats[s].status = *(volatile int*)p.err;
 }
 
 // host-side launcher ------------------------------------------------------------------

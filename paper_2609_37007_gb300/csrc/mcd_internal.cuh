@@ -16,7 +16,8 @@
 
 namespace mcd {
 
-constexpr int kMaxRows = 8;          // rows of one call (K+1 <= 8; first call uses 2)
+constexpr int kMaxRows = 8;          // rows of one call over all streams (packed operand columns)
+constexpr int kMaxStreams = 8;       // streams decoded together by one launch
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
@@ -109,22 +110,25 @@ struct FrameParams {
   float* qkv;                  // [kMaxRows][qkv_dim]
   float* mbuf;                 // [kMaxRows][F]
   float* logits;               // [kMaxRows][kMaxDraft+1][V]
-  float* kcache;               // [L][NKV][kMaxPos][D]
+  float* kcache;               // [S][L][NKV][kMaxPos][D]
   float* vcache;
   TopkRec* topk;               // [kMaxRows][kMaxDraft+1]
   TopkRec* draftq;             // [kMaxDraft] pending drafts' q
-  DevState* st;
+  DevState* st;                // [S]
   unsigned* ctr;               // [kMaxCalls][ctr_stride]
   int ctr_stride;
   int* err;                    // context-wide error word
   uint8_t* trace;              // optional
   // frame inputs
-  const float* cond;
-  const int* c0;
-  const float* c0emb;
-  unsigned stream_id, frame_idx;
-  int* codes_out;
-  mcd_frame_stats* stats;
+  const float* cond;           // [S][H]
+  const int* c0;               // [S]
+  const float* c0emb;          // [S][H]
+  int S;                       // streams of this launch
+  unsigned stream_ids[kMaxStreams], frame_ids[kMaxStreams];
+  int* codes_out;              // [S][n_pos]
+  mcd_frame_stats* stats;      // [S]
+  long long kv_stride;         // floats between streams' KV caches
+  long long trace_stride;      // bytes between streams' trace blocks
   float* logits_out;           // stepwise: verify logits of the single call
   int* emitted_out;
   int* n_emitted_out;
@@ -139,6 +143,7 @@ __host__ __device__ inline int ctr_stage(int layer, int s) { return layer * 4 + 
 __host__ __device__ inline int ctr_heads(int L) { return L * 4; }
 __host__ __device__ inline int ctr_topk(int L) { return L * 4 + 1; }
 __host__ __device__ inline int ctr_ready(int L) { return L * 4 + 2; }
+__host__ __device__ inline int ctr_accept(int L) { return L * 4 + 3; }
 
 // ---------------------------------------------------------------------------------------
 // PTX helpers

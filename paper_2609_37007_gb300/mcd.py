@@ -36,7 +36,7 @@ class McdConfig(ctypes.Structure):
                 ("qk_norm", ctypes.c_int32), ("weight_dtype", ctypes.c_int32),
                 ("draft_len", ctypes.c_int32), ("top_k", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("draft_mode", ctypes.c_int32),
-                ("noise_sigma", ctypes.c_float), ("seed", ctypes.c_uint64)]
+                ("noise_sigma", ctypes.c_float), ("seed", ctypes.c_uint64), ("max_streams", ctypes.c_int32)]
 
 
 CALL_TRACE_DTYPE = np.dtype([("a", "<i4"), ("n_rows", "<i4"), ("pos0", "<i4"), ("n_drafts", "<i4"),
@@ -71,6 +71,7 @@ def load_library() -> ctypes.CDLL:
                                    ctypes.POINTER(I64)]),
         "mcd_decode_frame": (I32, [P, U32, U32, P, P, P, P, P]),
         "mcd_decode_frame_host": (I32, [P, U32, U32, P, P, P, P, P]),
+        "mcd_decode_frames": (I32, [P, I32, P, P, P, P, P, P, P]),
         "mcd_begin_frame": (I32, [P, U32, U32, P, P, P]),
         "mcd_verify_accept": (I32, [P, P, P, P]),
         "mcd_draft": (I32, [P, I32, I32, P, P, P, P, P]),
@@ -124,7 +125,7 @@ def config_struct(cfg: MCDConfig) -> McdConfig:
     return McdConfig(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn,
                      cfg.n_pos, cfg.vocab, cfg.c0_vocab, cfg.rms_eps, cfg.rope_base, cfg.qk_norm,
                      cfg.weight_dtype, cfg.draft_len, cfg.top_k, cfg.temperature, cfg.draft_mode,
-                     cfg.noise_sigma, cfg.sample_seed)
+                     cfg.noise_sigma, cfg.sample_seed, cfg.max_streams)
 
 
 # ---- one wrapper per entry point ------------------------------------------------------
@@ -151,6 +152,15 @@ def mcd_load_weights(ctx, weights: Dict[str, np.ndarray]):
 def mcd_decode_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):
     _check("mcd_decode_frame", load_library().mcd_decode_frame(
         ctx, stream_id, frame_idx, _ptr(cond), _ptr(c0), _ptr(c0_emb), _ptr(codes_out), _ptr(stats)))
+
+
+def mcd_decode_frames(ctx, stream_ids, frame_idx, cond, c0, c0_emb, codes_out, stats=None):
+    """Several streams' frames in one launch; stream_ids / frame_idx are host integer lists."""
+    n = len(stream_ids)
+    sid = (ctypes.c_uint32 * n)(*[int(v) for v in stream_ids])
+    fid = (ctypes.c_uint32 * n)(*[int(v) for v in frame_idx])
+    _check("mcd_decode_frames", load_library().mcd_decode_frames(
+        ctx, n, sid, fid, _ptr(cond), _ptr(c0), _ptr(c0_emb), _ptr(codes_out), _ptr(stats)))
 
 
 def mcd_decode_frame_host(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):

@@ -57,6 +57,7 @@ class MCDConfig:
     weight_seed: int = 0
     sample_seed: int = 1
     frames: int = 1
+    max_streams: int = 1  # streams one launch may decode together
 
     def replace(self, **kw) -> "MCDConfig":
         return dataclasses.replace(self, **kw)

@@ -222,6 +222,65 @@ def test_tiny_variants_trace_parity(variant):
     env.dec.close()
 
 
+# ------------------------------------------------- batched streams ---------------------
+def decode_many(env, frames, frame_idx, stream_ids):
+    """One mcd_decode_frames launch over len(frames) streams, traced."""
+    cfg = env.cfg
+    n = len(frames)
+    ins = [env.frame_inputs(fr) for fr in frames]
+    cond = torch.stack([c for c, _, _ in ins])
+    c0 = torch.cat([c for _, c, _ in ins]) if cfg.c0_vocab else None
+    emb = torch.stack([e for _, _, e in ins]) if not cfg.c0_vocab else None
+    codes = torch.full((n, cfg.n_pos), -1, dtype=torch.int32, device=DEV)
+    stats = torch.zeros((n, 8), dtype=torch.int32, device=DEV)
+    tr = torch.zeros(mcd.mcd_trace_bytes(env.dec.ctx), dtype=torch.uint8, device=DEV)
+    mcd.mcd_set_trace(env.dec.ctx, tr)
+    mcd.mcd_decode_frames(env.dec.ctx, stream_ids, frame_idx, cond, c0, emb, codes, stats)
+    mcd.mcd_sync(env.dec.ctx)
+    mcd.mcd_set_trace(env.dec.ctx, None)
+    per = tr.numel() // cfg.max_streams
+    trh = tr.cpu().numpy()
+    return codes.cpu().numpy(), stats.cpu().numpy(), [trh[i * per:(i + 1) * per] for i in range(n)]
+
+
+@pytest.mark.parametrize("cfg", [TINY.replace(max_streams=2), TINY.replace(draft_len=0, max_streams=4),
+                                 TINY.replace(draft_len=1, max_streams=4)])
+def test_batched_streams_trace_parity(cfg):
+    """Several streams in one launch, rows re-packed every call: each stream's calls match
+    the oracle decoding that stream alone (its own counters and KV cache)."""
+    env = Env(cfg)
+    for rep in range(3):
+        n = cfg.max_streams - (rep % 2)            # also a launch with fewer streams than allowed
+        fidx = [10 * rep + s for s in range(n)]
+        sids = [7 + s for s in range(n)]
+        frames = [make_frame(cfg, f) for f in fidx]
+        codes, st, trs = decode_many(env, frames, fidx, sids)
+        for s in range(n):
+            assert st[s, 4] == 0 and st[s, 1] == cfg.n_pos
+            check_trace_against_oracle(cfg, env.model, frames[s], sids[s], fidx[s], trs[s], codes[s], int(st[s, 0]),
+                                       logit_tol=1e-5)
+    env.dec.close()
+
+
+def test_batched_streams_full_size():
+    cfg = MCD.replace(max_streams=2)
+    env = Env(cfg)
+    fidx, sids = [4, 9], [3, 5]
+    frames = [make_frame(cfg, f) for f in fidx]
+    codes, st, trs = decode_many(env, frames, fidx, sids)
+    for s in range(2):
+        assert st[s, 4] == 0 and st[s, 1] == cfg.n_pos
+        err = check_trace_against_oracle(cfg, env.model, frames[s], sids[s], fidx[s], trs[s], codes[s],
+                                         int(st[s, 0]), logit_tol=2e-2)
+        print("batched stream", s, "max |dlogit|", err)
+    env.dec.close()
+
+
+def test_batched_streams_reject_too_many_rows():
+    with pytest.raises(mcd.MCDError):
+        mcd.Decoder(MCD.replace(max_streams=3))       # 3 x (K + 1) > 8 packed rows
+
+
 # ------------------------------------------------- noisy-target drafts (K sweep) ------
 @pytest.mark.parametrize("K,sigma", [(1, 0.5), (2, 1.0), (3, 0.25), (7, 2.0)])
 def test_tiny_noisy_target_trace_parity(K, sigma):
