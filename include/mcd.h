@@ -82,7 +82,7 @@ typedef struct {
   float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only (>= 0)                            */
   uint64_t seed;        /* Philox key                                                    */
   int32_t max_streams;  /* streams one mcd_decode_frames call may decode together (1..8;
-                         * max_streams * max(K + 1, 2) <= 8; NOISY_TARGET needs 1)       */
+                         * max_streams * max(K + 1, 2) <= 32; NOISY_TARGET needs 1)      */
 } mcd_config;
 
 /* Per-frame counters written by the device (device memory, caller-owned). */

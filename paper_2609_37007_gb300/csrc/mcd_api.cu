@@ -323,8 +323,8 @@ static mcd_status validate_config(const mcd_config& c) {
   if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
   if (c.max_streams < 1 || c.max_streams > kMaxStreams) return MCD_ERR_UNSUPPORTED;
-  // every stream's rows of one call are packed into one operand of kMaxRows columns
-  if (c.max_streams * std::max(c.draft_len + 1, 2) > kMaxRows) return MCD_ERR_UNSUPPORTED;
+  // every stream's rows of one call are packed into one operand of kMaxCols columns
+  if (c.max_streams * std::max(c.draft_len + 1, 2) > kMaxCols) return MCD_ERR_UNSUPPORTED;
   if (c.max_streams > 1 && c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;
   if ((long long)c.n_q_heads * c.head_dim + 2LL * c.n_kv_heads * c.head_dim > 8192) return MCD_ERR_UNSUPPORTED;
   return MCD_OK;
@@ -452,16 +452,16 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   float2* rope = nullptr;
   if ((e = ctx_alloc(c, &rope, sizeof(float2) * kMaxPos * (p.D / 2))) != cudaSuccess) return fail(cuda_status(e));
   p.rope = rope;
-  if ((e = ctx_alloc(c, &p.x, sizeof(float) * kMaxRows * p.H)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.qkv, sizeof(float) * kMaxRows * p.qkv_dim)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxRows * p.F)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxRows * (kMaxDraft + 1) * p.V)) != cudaSuccess)
+  if ((e = ctx_alloc(c, &p.x, sizeof(float) * kMaxCols * p.H)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.qkv, sizeof(float) * kMaxCols * p.qkv_dim)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxCols * p.F)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxCols * (kMaxDraft + 1) * p.V)) != cudaSuccess)
     return fail(cuda_status(e));
   p.kv_stride = (long long)p.L * p.NKV * kMaxPos * p.D;
   const size_t kvsz = sizeof(float) * (size_t)p.kv_stride * k.max_streams;
   if ((e = ctx_alloc(c, &p.kcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.vcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * 2 * kMaxRows * (kMaxDraft + 1))) != cudaSuccess)
+  if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * 2 * kMaxCols * (kMaxDraft + 1))) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.draftq, sizeof(TopkRec) * (kMaxDraft + 1))) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.st, sizeof(DevState) * k.max_streams)) != cudaSuccess) return fail(cuda_status(e));
@@ -764,7 +764,7 @@ mcd_status mcd_topk_softmax(mcd_ctx* c, int32_t n_rows, const float* logits, int
   if (!c || !logits || n_rows < 0) return MCD_ERR_INVALID_ARG;
   if (n_rows == 0) return MCD_OK;
   FrameParams& p = c->fp;
-  if (n_rows > 2 * kMaxRows * (kMaxDraft + 1)) return MCD_ERR_UNSUPPORTED;
+  if (n_rows > 128) return MCD_ERR_UNSUPPORTED;   // the documented limit
   topk_rows_kernel<<<n_rows, kConsumerThreads, sizeof(TopkScratch), c->stream>>>(
       logits, p.V, p.top_k, p.T, p.topk, ids, weights, reinterpret_cast<unsigned long long*>(sums));
   MCD_CHECK(cudaGetLastError());

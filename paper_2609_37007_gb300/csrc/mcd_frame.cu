@@ -40,8 +40,9 @@ struct CallInfo {
   int heads[16];               // their positions P
   int emu, round0;             // noisy-target pass flag, stream 0's verify round (S = 1)
   int all_done;
-  // packed rows
-  int r_s[kMaxRows], r_n[kMaxRows], r_pos[kMaxRows], r_id[kMaxRows];
+  // packed rows: stream, row within the stream, position, code fed, layer-0 input row
+  int r_s[kMaxCols], r_n[kMaxCols], r_pos[kMaxCols], r_id[kMaxCols], r_f32[kMaxCols];
+  const uint8_t* r_src[kMaxCols];
   // per stream (index = stream)
   int act[kMaxStreams];        // active streams in packing order
   int a[kMaxStreams], nd[kMaxStreams], pos0[kMaxStreams], nrows[kMaxStreams], fr[kMaxStreams];
@@ -57,11 +58,11 @@ struct Smem {
   uint8_t* bfrag;
   float* red;
   float* vec;      // the current stage's norm gain
-  float* part;     // [kConsumerWarps][kMaxRows] partial sums of squares
+  float* part;     // [kConsumerWarps][kMaxCols] partial sums of squares
   uint64_t* full;
   uint64_t* empty;
   int* flags;      // [0] stop, [1] abort, [2] last-arriver, [3] current head / chunk
-  float* inv_rms;  // [kMaxRows]
+  float* inv_rms;  // [kMaxCols]
   CallInfo* ci;    // snapshot of the call's state
 };
 
@@ -69,14 +70,15 @@ constexpr int kRingOff = 0;
 constexpr int kActOff = kRingOff + kNumSlots * kSlotBytes;
 constexpr int kBfragOff = kActOff + kActBytes;
 constexpr int kRedOff = kBfragOff + kBfragBytes;
-constexpr int kVecOff = kRedOff + kChunk * kRedBytes;
-constexpr int kVecFloats = 1024;
+constexpr int kVecOff = kRedOff + kRedBytes;
+constexpr int kVecFloats = 2048;     // norm gain (H <= 1024) or the heads' bias tiles
 constexpr int kPartOff = kVecOff + kVecFloats * 4;
-constexpr int kBarOff = kPartOff + kConsumerWarps * kMaxRows * 4;
+constexpr int kBarOff = kPartOff + kConsumerWarps * kMaxCols * 4;
 constexpr int kFlagOff = kBarOff + 2 * kNumSlots * 8;
 constexpr int kRmsOff = kFlagOff + 64;
-constexpr int kInfoOff = kRmsOff + 64;
+constexpr int kInfoOff = kRmsOff + kMaxCols * 4;
 constexpr int kSmemBytes = kInfoOff + (int)((sizeof(CallInfo) + 15) / 16 * 16);
+static_assert(kSmemBytes <= 227 * 1024, "frame kernel shared memory exceeds the per-CTA limit");
 
 __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   Smem s;
@@ -237,8 +239,13 @@ struct Cons {
   uint32_t seq;   // units consumed (ring sequence)
   int rot;
   bool abort_;
-  __device__ Cons(const FrameParams& pp, Smem& s) : p(pp), sm(s), seq(0), rot(0), abort_(false) {}
+  uint8_t* op;    // B operand of the current stage (in the 64 KB work region act + bfrag)
+  __device__ Cons(const FrameParams& pp, Smem& s)
+      : p(pp), sm(s), seq(0), rot(0), abort_(false), op(reinterpret_cast<uint8_t*>(s.act)) {}
 };
+
+// Offset of the Wo operand in the work region: past the attention scratch (< 48 KB).
+constexpr int kWoOperandOff = 48 * 1024;
 
 // Optional profiling stamps (%globaltimer, ns), 128 per call.  Slots: 0 call start;
 // 1 top-k inputs ready; 2 top-k done (CTA 0); 3 top-k done (last CTA); 4..7 acceptance
@@ -279,185 +286,256 @@ __device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call, in
   timeline_max(c, call, slot + 1);
 }
 
+// Operand geometry of a call with ncols packed columns: ncp = 2^ceil(log2 ncols) columns
+// are written (columns >= ncols as zeros); NT = ncp / 8 n-tiles (at least 1).  Up to 16
+// columns the activations are a bf16 hi + lo pair (16 B per fragment entry, about 16
+// mantissa bits); beyond that a single bf16 (8 B per entry).
+__device__ __forceinline__ int col_log2(int ncols) {
+  return ncols <= 1 ? 0 : ncols <= 2 ? 1 : ncols <= 4 ? 2 : ncols <= 8 ? 3 : ncols <= 16 ? 4 : 5;
+}
+__device__ __forceinline__ int n_tiles(int ncols) { return max(1, (1 << col_log2(ncols)) >> 3); }
+__device__ __forceinline__ bool hilo_operand(int ncols) { return ncols <= 16; }
+
 // Activation operand in one pass.  `ld(n, k)` returns elements (k, k+1) of column n from
 // global or shared memory; `gain` (shared, may be null) multiplies them per input index;
-// with want_ss the per-column 1/rms of the raw values lands in inv_rms.  bf16 weights get
-// hi/lo bf16 B fragments of mma.m16n8k16 (entry (kt0 + kt, lane): column lane/4, inputs
-// kt*16 + 2(lane%4) + {0,1,8,9}); fp32 weights get fp32 rows [8][ldk] from column kt0*16.  Only the first
-// ncp = 2^ceil(log2 ncols) columns are written (columns >= ncols as zeros): an mma output
-// column depends only on its own B column and columns >= ncols are never read back.
-// Every load of a thread is issued before any of its stores (one memory round trip).
-template <int WT, class Ld>
+// with want_ss the per-column 1/rms of the raw values lands in inv_rms; store_raw (may be
+// null) receives the raw values as fp32 rows [ncols][ldk].  bf16 weights get B fragments of
+// mma.m16n8k16: entry ((kt0 + kt) * NT + nt, lane) holds column nt*8 + lane/4, inputs
+// kt*16 + 2(lane%4) + {0,1,8,9}; fp32 weights get fp32 rows [ncols][ldk] from column kt0*16.
+// Only the first ncp columns are written: an mma output column depends only on its own B
+// column and columns >= ncols are never read back.  Every load of a batch is issued before
+// any of its stores (one memory round trip per 2048 entries).
+template <int WT, bool WIDE, class Ld>
 __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
-                                             bool want_ss, Ld ld) {
+                                             bool want_ss, Ld ld, float* store_raw = nullptr) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int lg = ncols <= 1 ? 0 : ncols <= 2 ? 1 : ncols <= 4 ? 2 : 3;
+  const int lg = col_log2(ncols), NT = WIDE ? n_tiles(ncols) : 1;
+  const bool hilo = WIDE ? hilo_operand(ncols) : true;
   const int n = (tid >> 2) & ((1 << lg) - 1), t = tid & 3;
   const bool live = n < ncols;
   const int items = (Kdim >> 4) << (2 + lg);       // (k-tile, column, t)
   constexpr int kE = 8;
   float ss = 0.f;
   for (int base = 0; base < items; base += kE * kConsumerThreads) {
-  float2 va[kE], vb[kE];
+    float2 va[kE], vb[kE];
 #pragma unroll
-  for (int e = 0; e < kE; ++e) {
-    const int i = base + tid + e * kConsumerThreads;
-    va[e] = make_float2(0.f, 0.f);
-    vb[e] = make_float2(0.f, 0.f);
-    if (i < items && live) {
-      const int k0 = ((i >> (2 + lg)) << 4) + 2 * t;
-      va[e] = ld(n, k0);
-      vb[e] = ld(n, k0 + 8);
-    }
-  }
-#pragma unroll
-  for (int e = 0; e < kE; ++e) {
-    const int i = base + tid + e * kConsumerThreads;
-    if (i < items) {
-      const int kt = i >> (2 + lg), k0 = (kt << 4) + 2 * t;
-      float2 x01 = va[e], x89 = vb[e];
-      ss += x01.x * x01.x + x01.y * x01.y + x89.x * x89.x + x89.y * x89.y;
-      if (gain) {
-        const float2 g01 = *reinterpret_cast<const float2*>(gain + k0);
-        const float2 g89 = *reinterpret_cast<const float2*>(gain + k0 + 8);
-        x01.x *= g01.x;
-        x01.y *= g01.y;
-        x89.x *= g89.x;
-        x89.y *= g89.y;
-      }
-      if (WT == MCD_WEIGHT_BF16) {
-        const uint32_t h01 = pack_bf16x2(x01.x, x01.y), h89 = pack_bf16x2(x89.x, x89.y);
-        const uint32_t l01 = pack_bf16x2(x01.x - bf16_lo_f32(h01), x01.y - bf16_hi_f32(h01));
-        const uint32_t l89 = pack_bf16x2(x89.x - bf16_lo_f32(h89), x89.y - bf16_hi_f32(h89));
-        reinterpret_cast<uint4*>(c.sm.bfrag)[(kt0 + kt) * 32 + 4 * n + t] = make_uint4(h01, h89, l01, l89);
-      } else {
-        float* xs = reinterpret_cast<float*>(c.sm.bfrag) + n * ldk + kt0 * 16 + k0;
-        *reinterpret_cast<float2*>(xs) = x01;
-        *reinterpret_cast<float2*>(xs + 8) = x89;
+    for (int e = 0; e < kE; ++e) {
+      const int i = base + tid + e * kConsumerThreads;
+      va[e] = make_float2(0.f, 0.f);
+      vb[e] = make_float2(0.f, 0.f);
+      if (i < items && live) {
+        const int k0 = ((i >> (2 + lg)) << 4) + 2 * t;
+        va[e] = ld(n, k0);
+        vb[e] = ld(n, k0 + 8);
       }
     }
-  }
+#pragma unroll
+    for (int e = 0; e < kE; ++e) {
+      const int i = base + tid + e * kConsumerThreads;
+      if (i < items) {
+        const int kt = i >> (2 + lg), k0 = (kt << 4) + 2 * t;
+        float2 x01 = va[e], x89 = vb[e];
+        ss += x01.x * x01.x + x01.y * x01.y + x89.x * x89.x + x89.y * x89.y;
+        if (store_raw && live) {
+          *reinterpret_cast<float2*>(store_raw + (size_t)n * ldk + k0) = x01;
+          *reinterpret_cast<float2*>(store_raw + (size_t)n * ldk + k0 + 8) = x89;
+        }
+        if (gain) {
+          const float2 g01 = *reinterpret_cast<const float2*>(gain + k0);
+          const float2 g89 = *reinterpret_cast<const float2*>(gain + k0 + 8);
+          x01.x *= g01.x;
+          x01.y *= g01.y;
+          x89.x *= g89.x;
+          x89.y *= g89.y;
+        }
+        if (WT == MCD_WEIGHT_BF16) {
+          const int entry = ((kt0 + kt) * NT + (n >> 3)) * 32 + 4 * (n & 7) + t;
+          const uint32_t h01 = pack_bf16x2(x01.x, x01.y), h89 = pack_bf16x2(x89.x, x89.y);
+          if (hilo) {
+            const uint32_t l01 = pack_bf16x2(x01.x - bf16_lo_f32(h01), x01.y - bf16_hi_f32(h01));
+            const uint32_t l89 = pack_bf16x2(x89.x - bf16_lo_f32(h89), x89.y - bf16_hi_f32(h89));
+            reinterpret_cast<uint4*>(c.op)[entry] = make_uint4(h01, h89, l01, l89);
+          } else {
+            reinterpret_cast<uint2*>(c.op)[entry] = make_uint2(h01, h89);
+          }
+        } else {
+          float* xs = reinterpret_cast<float*>(c.op) + n * ldk + kt0 * 16 + k0;
+          *reinterpret_cast<float2*>(xs) = x01;
+          *reinterpret_cast<float2*>(xs + 8) = x89;
+        }
+      }
+    }
   }
   if (want_ss) {
     // lanes of one column: t (bits 0-1) and the k-tile bits above the column bits
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1)
       if (off < 4 || off >= (4 << lg)) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
-    if (lane < (4 << lg) && t == 0) c.sm.part[warp * kMaxRows + n] = ss;
+    if (lane < (4 << lg) && t == 0) c.sm.part[warp * kMaxCols + n] = ss;
   }
   consumer_sync();
   if (want_ss) {
     if (tid < ncols) {
+      // warp w holds columns 8w .. 8w+7 (mod ncp): only those warps' partials exist
+      const int ncp = 1 << lg, own = (tid & ~7) & (ncp - 1);
       float s = 0.f;
 #pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) s += c.sm.part[w * kMaxRows + tid];  // fixed order
+      for (int w = 0; w < kConsumerWarps; ++w)
+        if (((8 * w) & (ncp - 1)) == own) s += c.sm.part[w * kMaxCols + tid];  // fixed order
       c.sm.inv_rms[tid] = rsqrtf(s / (float)Kdim + c.p.eps);
     }
     consumer_sync();
   }
 }
 
+// Warp roles in a unit: m-tile mi of Mu, n-tile group gn of Gn (ntpw n-tiles each) and
+// k-group kg of Gk, with Mu * Gn * Gk = 8 warps.  bf16 weights spread the n-tiles over the
+// warps (short reduction buffer); fp32 weights keep Gn = 1 so each warp's fp32 sums stay
+// as short as with one n-tile (the reduction order does not depend on the column count).
+struct WarpRole {
+  int Gn, ntpw, lg_ntpw, Gk, kts, mi, gn, kg;
+};
+__device__ __forceinline__ WarpRole warp_role(const MatGeom& g, int NT, int warp, bool split_n) {
+  WarpRole w;
+  w.Gn = split_n ? min(NT, kConsumerWarps / g.Mu) : 1;
+  w.ntpw = NT / w.Gn;
+  w.lg_ntpw = w.ntpw == 1 ? 0 : w.ntpw == 2 ? 1 : 2;
+  w.Gk = kConsumerWarps / (g.Mu * w.Gn);
+  w.kts = g.Ku / w.Gk;
+  w.mi = warp % g.Mu;
+  const int rest = warp / g.Mu;
+  w.gn = rest % w.Gn;
+  w.kg = rest / w.Gn;
+  return w;
+}
+
 // Multiply the unit in ring slot `slotp` with the prepared operand of k-chunk kc; the
-// warp's partial tile (its m-tile over its k-group) lands in red[r] in C-fragment order.
-// `b` caches the warp's bf16 B fragments across the units of a chunk (same k-range).
-template <int WT>
-__device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const uint8_t* slotp, int Kdim, int kc, int r,
-                                         uint4 (&b)[8], bool load_b) {
+// warp's partial tiles (its m-tile, its n-tiles, over its k-group) land in the reduction
+// buffer of chunk unit r in mma C-fragment order.
+template <int WT, bool WIDE>
+__device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const WarpRole& w, int NT, bool hilo,
+                                         const uint8_t* slotp, int Kdim, int kc, int r) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int Mu = g.Mu, Ku = g.Ku;
-  const int Gk = kConsumerWarps / Mu;
-  const int mi = warp % Mu, kg = warp / Mu, kts = Ku / Gk;
-  float4* red = reinterpret_cast<float4*>(c.sm.red + r * (kRedBytes / 4));
+  const int Ku = g.Ku, kt0 = kc * Ku + w.kg * w.kts;
+  float4* red = reinterpret_cast<float4*>(c.sm.red) + ((size_t)r * kConsumerWarps + warp) * w.ntpw * 32;
   if (WT == MCD_WEIGHT_BF16) {
-    const uint4* A = reinterpret_cast<const uint4*>(slotp) + (size_t)(mi * Ku + kg * kts) * 32 + lane;
-    (void)b;
-    (void)load_b;
-    const uint4* B = reinterpret_cast<const uint4*>(c.sm.bfrag) + (size_t)(kc * Ku + kg * kts) * 32 + lane;
-    float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint4* A = reinterpret_cast<const uint4*>(slotp) + (size_t)(w.mi * Ku + w.kg * w.kts) * 32 + lane;
+    const int ntpw = WIDE ? w.ntpw : 1;
+    for (int ntl = 0; ntl < ntpw; ++ntl) {
+      const int nt = WIDE ? w.gn * w.ntpw + ntl : 0;
+      float a0[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f};
+      if (!WIDE || hilo) {
+        const uint4* B = reinterpret_cast<const uint4*>(c.op) + ((size_t)kt0 * NT + nt) * 32 + lane;
 #pragma unroll 8
-    for (int t = 0; t < kts; ++t) {
-      const uint4 a = A[t * 32];
-      const uint4 bb = B[t * 32];
-      mma_bf16_16816(a0, a, bb.x, bb.y);
-      mma_bf16_16816(a1, a, bb.z, bb.w);
-    }
-    red[warp * 32 + lane] = make_float4(a0[0] + a1[0], a0[1] + a1[1], a0[2] + a1[2], a0[3] + a1[3]);
-  } else {
-    const int rr = lane & 15, kh = lane >> 4;
-    const float* xs = reinterpret_cast<const float*>(c.sm.bfrag);
-    const float4* A = reinterpret_cast<const float4*>(slotp) + (size_t)(mi * Ku + kg * kts) * 64 + lane * 2;
-    float acc[kMaxRows];
-#pragma unroll
-    for (int n = 0; n < kMaxRows; ++n) acc[n] = 0.f;
-    for (int t = 0; t < kts; ++t) {
-      const float4 w0 = A[t * 64], w1 = A[t * 64 + 1];
-      const int col = (kc * Ku + kg * kts + t) * 16 + kh * 8;
-#pragma unroll
-      for (int n = 0; n < kMaxRows; ++n) {
-        const float4 x0 = *reinterpret_cast<const float4*>(xs + n * Kdim + col);
-        const float4 x1 = *reinterpret_cast<const float4*>(xs + n * Kdim + col + 4);
-        acc[n] += w0.x * x0.x + w0.y * x0.y + w0.z * x0.z + w0.w * x0.w + w1.x * x1.x + w1.y * x1.y +
-                  w1.z * x1.z + w1.w * x1.w;
+        for (int t = 0; t < w.kts; ++t) {
+          const uint4 a = A[t * 32];
+          const uint4 bb = B[(size_t)t * NT * 32];
+          mma_bf16_16816(a0, a, bb.x, bb.y);
+          mma_bf16_16816(a1, a, bb.z, bb.w);
+        }
+      } else {
+        const uint2* B = reinterpret_cast<const uint2*>(c.op) + ((size_t)kt0 * NT + nt) * 32 + lane;
+#pragma unroll 8
+        for (int t = 0; t < w.kts; t += 2) {
+          const uint4 a = A[t * 32];
+          const uint2 bb = B[(size_t)t * NT * 32];
+          mma_bf16_16816(a0, a, bb.x, bb.y);
+          if (t + 1 < w.kts) {
+            const uint4 a2 = A[(t + 1) * 32];
+            const uint2 b2 = B[(size_t)(t + 1) * NT * 32];
+            mma_bf16_16816(a1, a2, b2.x, b2.y);
+          }
+        }
       }
+      red[ntl * 32 + lane] = make_float4(a0[0] + a1[0], a0[1] + a1[1], a0[2] + a1[2], a0[3] + a1[3]);
     }
+  } else {
+    // fp32 weights: lane = (row rr, k-half kh) holds 8 consecutive inputs of a tile row
+    const int rr = lane & 15, kh = lane >> 4;
+    const float* xs = reinterpret_cast<const float*>(c.op);
+    const float4* A = reinterpret_cast<const float4*>(slotp) + (size_t)(w.mi * Ku + w.kg * w.kts) * 64 + lane * 2;
+    const int ntpw = WIDE ? w.ntpw : 1;
+    for (int ntl = 0; ntl < ntpw; ++ntl) {
+      const int n0 = (WIDE ? w.gn * w.ntpw + ntl : 0) * 8;
+      float acc[8];
 #pragma unroll
-    for (int n = 0; n < kMaxRows; ++n) acc[n] += __shfl_xor_sync(0xFFFFFFFFu, acc[n], 16);
-    if (lane < 16) {
-      float* rf = reinterpret_cast<float*>(red + warp * 32);
+      for (int n = 0; n < 8; ++n) acc[n] = 0.f;
+      for (int t = 0; t < w.kts; ++t) {
+        const float4 w0 = A[t * 64], w1 = A[t * 64 + 1];
+        const int col = (kt0 + t) * 16 + kh * 8;
 #pragma unroll
-      for (int n = 0; n < kMaxRows; ++n) rf[((rr & 7) * 4 + (n >> 1)) * 4 + (rr >> 3) * 2 + (n & 1)] = acc[n];
+        for (int n = 0; n < 8; ++n) {
+          const float4 x0 = *reinterpret_cast<const float4*>(xs + (n0 + n) * Kdim + col);
+          const float4 x1 = *reinterpret_cast<const float4*>(xs + (n0 + n) * Kdim + col + 4);
+          acc[n] += w0.x * x0.x + w0.y * x0.y + w0.z * x0.z + w0.w * x0.w + w1.x * x1.x + w1.y * x1.y +
+                    w1.z * x1.z + w1.w * x1.w;
+        }
+      }
+#pragma unroll
+      for (int n = 0; n < 8; ++n) acc[n] += __shfl_xor_sync(0xFFFFFFFFu, acc[n], 16);
+      if (lane < 16) {
+        float* rf = reinterpret_cast<float*>(red + ntl * 32);
+#pragma unroll
+        for (int n = 0; n < 8; ++n) rf[((rr & 7) * 4 + (n >> 1)) * 4 + (rr >> 3) * 2 + (n & 1)] = acc[n];
+      }
     }
   }
 }
 
-// Sum over the k-group warps of output (row rr of m-tile mi, column n) of chunk unit r.
-__device__ __forceinline__ float red_sum(const Cons& c, const MatGeom& g, int r, int mi, int rr, int n) {
-  const int Gk = kConsumerWarps / g.Mu;
-  const float* red = c.sm.red + r * (kRedBytes / 4);
+// Sum over the k-group warps of output (row rr of m-tile mi, column c) of chunk unit r.
+__device__ __forceinline__ float red_sum(const Cons& c, const MatGeom& g, const WarpRole& w, int r, int mi, int rr,
+                                         int col) {
+  const int nt = col >> 3, n = col & 7, gn = nt >> w.lg_ntpw, ntl = nt & (w.ntpw - 1);
+  const float* red = c.sm.red;
   const int ln = (rr & 7) * 4 + (n >> 1), idx = (rr >> 3) * 2 + (n & 1);
   float v = 0.f;
 #pragma unroll
-  for (int kg = 0; kg < kConsumerWarps; ++kg)
-    if (kg < Gk) v += red[((kg * g.Mu + mi) * 32 + ln) * 4 + idx];
+  for (int kg = 0; kg < kConsumerWarps; ++kg) {
+    if (kg < w.Gk) {
+      const int warp = (kg * w.Gn + gn) * g.Mu + mi;
+      v += red[((((size_t)r * kConsumerWarps + warp) * w.ntpw + ntl) * 32 + ln) * 4 + idx];
+    }
+  }
   return v;
 }
 
 // Run every unit of stage si assigned to this CTA.  Units are taken in chunks of up to
 // kChunk consecutive units that share one operand (opkey(u): the k-chunk / head whose B
-// operand they multiply; prep(u0, cnt, step) builds it for the chunk).  Each chunk: wait
-// for its units' weights, multiply them all, one barrier, then one epilogue pass
-// epi(u, mi, rr, n, v, v8) over the live outputs (columns n < ncols; v8 = row rr + 8 for
-// gate/up pairs).
-template <int WT, class Key, class Prep, class Epi>
+// operand they multiply; prep(u0, cnt, step) builds it for the chunk), as many as the
+// reduction buffer holds.  Each chunk: wait for its units' weights, multiply them all, one
+// barrier, then one epilogue pass epi(u, mi, rr, n, v, v8) over the live outputs (columns
+// n < ncols; v8 = row rr + 8 for gate/up pairs).
+template <int WT, bool WIDE, class Key, class Prep, class Epi>
 __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, int ncols, Key opkey,
                                           Prep prep, Epi epi, bool pairs_rows = false) {
   const FrameParams& p = c.p;
   const MatGeom& g = p.g[stage_kind(si, p.L)];
+  const int lane = threadIdx.x & 31;
   timeline(c, call, 8 + 4 * si);
   const UnitRange ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
+  const int NT = WIDE ? n_tiles(ncols) : 1;
+  const bool hilo = WIDE ? hilo_operand(ncols) : true;
+  const WarpRole role = warp_role(g, NT, threadIdx.x >> 5, WIDE && WT == MCD_WEIGHT_BF16);
+  const int per_unit = kConsumerWarps * role.ntpw * 512;                            // bytes of partials
+  const int cap = max(1, min(kChunk, kRedBytes / per_unit));
   const int lgm = g.Mu == 1 ? 0 : g.Mu == 2 ? 1 : g.Mu == 4 ? 2 : 3;
-  const int lgn = ncols <= 1 ? 0 : ncols <= 2 ? 1 : ncols <= 4 ? 2 : 3;
+  const int lgn = col_log2(ncols);
   const int lg_unit = lgm + (pairs_rows ? 3 : 4) + lgn;       // outputs per unit (log2)
   bool first_chunk = true;
   for (int u0 = ur.first; u0 < ur.end;) {
     const int key = opkey(u0);
     int cnt = 1;
-    while (cnt < kChunk && u0 + cnt * ur.step < ur.end && opkey(u0 + cnt * ur.step) == key) ++cnt;
+    while (cnt < cap && u0 + cnt * ur.step < ur.end && opkey(u0 + cnt * ur.step) == key) ++cnt;
     prep(u0, cnt, ur.step);
-    uint4 b[8];
-#pragma unroll
-    for (int r = 0; r < kChunk; ++r) {
-      if (r < cnt) {
-        const uint32_t slot = (c.seq + r) % kNumSlots;
-        if (!wait_mbar(&c.sm.full[slot], ((c.seq + r) / kNumSlots) & 1u, p.err, p.wait_ns, nullptr))
-          c.sm.flags[1] = 1;
-        if (first_chunk && r == 0) timeline(c, call, 9 + 4 * si);
-        const int u = u0 + r * ur.step;
-        (void)u;
-        unit_mma<WT>(c, g, c.sm.ring + (size_t)slot * kSlotBytes, Kdim, 0, r, b, r == 0);
-        __syncwarp();
-        if ((threadIdx.x & 31) == 0) mbar_arrive(&c.sm.empty[slot]);
-      }
+#pragma unroll 1
+    for (int r = 0; r < cnt; ++r) {
+      const uint32_t slot = (c.seq + r) % kNumSlots;
+      if (!wait_mbar(&c.sm.full[slot], ((c.seq + r) / kNumSlots) & 1u, p.err, p.wait_ns, nullptr))
+        c.sm.flags[1] = 1;
+      if (first_chunk && r == 0) timeline(c, call, 9 + 4 * si);
+      unit_mma<WT, WIDE>(c, g, role, NT, hilo, c.sm.ring + (size_t)slot * kSlotBytes, Kdim, 0, r);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&c.sm.empty[slot]);
     }
     c.seq += cnt;
     consumer_sync();
@@ -470,8 +548,8 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
       const int row = q >> lgn, n = q & ((1 << lgn) - 1);
       if (n < ncols) {
         const int mi = row >> (pairs_rows ? 3 : 4), rr = row & (pairs_rows ? 7 : 15);
-        const float v = red_sum(c, g, r, mi, rr, n);
-        const float v8 = pairs_rows ? red_sum(c, g, r, mi, rr + 8, n) : 0.f;
+        const float v = red_sum(c, g, role, r, mi, rr, n);
+        const float v8 = pairs_rows ? red_sum(c, g, role, r, mi, rr + 8, n) : 0.f;
         epi(u0 + r * ur.step, mi, rr, n, v, v8);
       }
     }
@@ -492,56 +570,6 @@ __device__ __forceinline__ void g2s_vec(float* dst, const float* src, int n) {
 __device__ __forceinline__ float2 ld_global2(const float* q) { return __ldcg(reinterpret_cast<const float2*>(q)); }
 __device__ __forceinline__ float2 ld_shared2(const float* q) { return *reinterpret_cast<const float2*>(q); }
 
-// Layer-0 input rows of the call into act[r][H] (packed row r of stream s): [cond, c0] on a
-// stream's first call, else the embeddings of [c_a, d_{a+1}, ...] (table of position a+i).
-// CTA 0 also seeds the residual stream x in global memory.
-__device__ __forceinline__ void gather_inputs(Cons& c) {
-  const FrameParams& p = c.p;
-  const CallInfo* ci = c.sm.ci;
-  const int M = ci->M;
-  const int H = p.H, per = H / 8;      // 8 elements (16 B of bf16 or 2x16 B of fp32) per item
-  for (int it = threadIdx.x; it < M * per; it += kConsumerThreads) {
-    const int r = it / per, k0 = (it - r * per) * 8;
-    const int s = ci->r_s[r], pos = ci->r_pos[r];
-    float v[8];
-    if (pos == 0 || (pos == 1 && p.C0V == 0)) {
-      const float4* src = reinterpret_cast<const float4*>((pos == 0 ? p.cond : p.c0emb) + (size_t)s * H + k0);
-      const float4 a = __ldg(src), b = __ldg(src + 1);
-      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-    } else {
-      const int table = pos - 1;
-      int id = ci->r_id[r];
-      if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {  // a c0 outside table 0: fail the frame
-        if (k0 == 0) atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
-        id = 0;
-      }
-      const uint8_t* row = p.embed + (long long)table * p.embed_stride;
-      if (p.wdtype == MCD_WEIGHT_BF16) {
-        const uint4 w = __ldg(reinterpret_cast<const uint4*>(row + ((long long)id * H + k0) * 2));
-        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          v[2 * e] = bf16_bits_to_f32(ww[e] & 0xFFFFu);
-          v[2 * e + 1] = bf16_bits_to_f32(ww[e] >> 16);
-        }
-      } else {
-        const float4* src = reinterpret_cast<const float4*>(row + ((long long)id * H + k0) * 4);
-        const float4 a = __ldg(src), b = __ldg(src + 1);
-        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-      }
-    }
-    float4* dst = reinterpret_cast<float4*>(c.sm.act + r * H + k0);
-    dst[0] = make_float4(v[0], v[1], v[2], v[3]);
-    dst[1] = make_float4(v[4], v[5], v[6], v[7]);
-    if (blockIdx.x == 0) {
-      float4* gx = reinterpret_cast<float4*>(p.x + (size_t)r * H + k0);
-      gx[0] = dst[0];
-      gx[1] = dst[1];
-    }
-  }
-  consumer_sync();
-}
-
 // Attention of query head h for the nr rows of stream s (packed rows base..base+nr-1; QK-norm,
 // RoPE, causal softmax over the stream's per-frame cache plus the new rows); output
 // o[base + n][D] in act.  Scratch spans act + bfrag
@@ -559,11 +587,12 @@ __device__ void attention_stream(Cons& c, int layer, int h, bool write_kv, int n
   const int cs_shift = D == 128 ? 5 : 4;           // 16-byte chunks per row = D / 4
   const int cpr = 1 << cs_shift;
   const int KS = D + 8;                            // padded row stride (floats) of q and k rows
-  float* o = c.sm.act;                             // [8][D]
-  float* qs = o + kMaxRows * 128;                  // [8][KS]
-  float* ks = qs + kMaxRows * 136;                 // [kMaxPos][KS]
-  float* vs = ks + kMaxPos * 136;                  // [kMaxPos][D]
-  float2* cs = reinterpret_cast<float2*>(vs + kMaxPos * 128);   // [8][D/2] (cos, sin)
+  constexpr int kAttnPos = 16;                     // sequence positions 0..15 (c15 is never fed)
+  float* o = c.sm.act;                             // [kMaxCols][D]: every stream's packed rows
+  float* qs = o + kMaxCols * 128;                  // [8][KS]
+  float* ks = qs + kMaxRows * 136;                 // [kAttnPos][KS]
+  float* vs = ks + kAttnPos * 136;                 // [kAttnPos][D]
+  float2* cs = reinterpret_cast<float2*>(vs + kAttnPos * 128);  // [8][D/2] (cos, sin)
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
   float* gk = gq + 128;                                          // [D]
   const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
@@ -743,7 +772,7 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
 // ------------------------------------------------------------------------------------
 // One call
 // ------------------------------------------------------------------------------------
-template <int WT>
+template <int WT, bool WIDE>
 __device__ void run_call(Cons& c, int call) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
@@ -761,15 +790,25 @@ __device__ void run_call(Cons& c, int call) {
     // ---- S1: RMSNorm -> QKV  (q, k, v = W (x . g) / rms) -------------------------------
     g2s_vec(sm.vec, p.attn_norm + (size_t)l * H, H);      // independent of the wait below
     if (l == 0) {
-      gather_inputs(c);
-      prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, [&](int n, int k) { return ld_shared2(sm.act + n * H + k); });
+      // layer-0 rows straight from their sources (cond / c0 vector / embedding rows); CTA 0
+      // also seeds the residual stream x
+      consumer_sync();                     // the gain is in shared memory
+      prep_operand<WT, WIDE>(
+          c, n_rows, H, 0, H, sm.vec, true,
+          [&](int n, int k) {
+            const uint8_t* src = ci->r_src[n];
+            if (ci->r_f32[n]) return __ldg(reinterpret_cast<const float2*>(src) + (k >> 1));
+            const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(src) + (k >> 1));
+            return make_float2(bf16_bits_to_f32(w & 0xFFFFu), bf16_bits_to_f32(w >> 16));
+          },
+          blockIdx.x == 0 ? p.x : nullptr);
     } else {
       if (!cons_wait(c, ctr + ctr_stage(l - 1, 3), N)) return;
-      prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
+      prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
     }
     {
       const MatGeom& g = p.g[MAT_QKV];
-      run_stage<WT>(c, call, 4 * l + 0, g.n_units, H, n_rows, no_key, no_prep,
+      run_stage<WT, WIDE>(c, call, 4 * l + 0, g.n_units, H, n_rows, no_key, no_prep,
                     [&](int u, int mi, int rr, int n, float v, float) {
                       const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
                       p.qkv[(size_t)n * p.qkv_dim + row] = v * sm.inv_rms[n];
@@ -787,7 +826,7 @@ __device__ void run_call(Cons& c, int call) {
       const int group = p.NH / p.NKV;
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
-      run_stage<WT>(
+      run_stage<WT, WIDE>(
           c, call, 4 * l + 1, g.n_units, D, n_rows, [&](int u) { return u / g.n_mb; },
           [&](int u, int cnt, int step) {
             const int h = u / g.n_mb;
@@ -795,7 +834,8 @@ __device__ void run_call(Cons& c, int call) {
             for (int r = 0; r < cnt; ++r) writer |= (h % group) == 0 && (u + r * step) % g.n_mb == 0;
             if (sm.flags[3] != h || writer) {
               attention_head(c, l, h, writer);
-              prep_operand<WT>(c, n_rows, D, 0, D, nullptr, false,
+              c.op = reinterpret_cast<uint8_t*>(sm.act) + kWoOperandOff;
+              prep_operand<WT, WIDE>(c, n_rows, D, 0, D, nullptr, false,
                                [&](int n, int k) { return ld_shared2(sm.act + n * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
@@ -806,16 +846,17 @@ __device__ void run_call(Cons& c, int call) {
           });
       if (c.abort_) return;
     }
+    c.op = reinterpret_cast<uint8_t*>(sm.act);
     cons_signal(c, ctr + ctr_stage(l, 1), call, 10 + 4 * (4 * l + 1));
 
     // ---- S3: RMSNorm -> gate/up -> SwiGLU --------------------------------------------------
     g2s_vec(sm.vec, p.ffn_norm + (size_t)l * H, H);
     if (!cons_wait(c, ctr + ctr_stage(l, 1), N)) return;
-    prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
+    prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
     {
       const MatGeom& g = p.g[MAT_GU];
       // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
-      run_stage<WT>(
+      run_stage<WT, WIDE>(
           c, call, 4 * l + 2, g.n_units, H, n_rows, no_key, no_prep,
           [&](int u, int mi, int rr, int n, float gate, float up) {
             const float s = sm.inv_rms[n];
@@ -835,13 +876,13 @@ __device__ void run_call(Cons& c, int call) {
       const int Kc = g.Ku * 16;
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
-      run_stage<WT>(
+      run_stage<WT, WIDE>(
           c, call, 4 * l + 3, g.n_units, Kc, n_rows, [&](int u) { return u / g.n_mb; },
           [&](int u, int, int) {
             const int kc = u / g.n_mb;
             if (sm.flags[3] != kc) {
               const float* m = p.mbuf + (size_t)kc * Kc;
-              prep_operand<WT>(c, n_rows, Kc, 0, Kc, nullptr, false,
+              prep_operand<WT, WIDE>(c, n_rows, Kc, 0, Kc, nullptr, false,
                                [&](int n, int k) { return ld_global2(m + (size_t)n * F + k); });
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
@@ -863,17 +904,17 @@ __device__ void run_call(Cons& c, int call) {
   // of the heads its streams need.
   g2s_vec(sm.vec, p.final_norm, H);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
-  prep_operand<WT>(c, n_rows, H, 0, H, sm.vec, true, from_x);
+  prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
   {
     const MatGeom& g = p.g[MAT_HEAD];
-    float* bias_s = sm.vec;   // [kChunk][16 rows][8 columns]
+    float* bias_s = sm.vec;   // [kChunk][16 rows][kMaxCols columns]
     int chunk_u0 = 0;
-    run_stage<WT>(
+    run_stage<WT, WIDE>(
         c, call, 4 * L, ci->n_heads * g.n_units, H, n_rows, no_key,
         [&](int u0, int cnt, int step) {
           chunk_u0 = u0;
-          for (int o = threadIdx.x; o < cnt * 128; o += kConsumerThreads) {
-            const int r = o >> 7, rr = (o >> 3) & 15, n = o & 7;
+          for (int o = threadIdx.x; o < cnt * 16 * kMaxCols; o += kConsumerThreads) {
+            const int r = o / (16 * kMaxCols), rr = (o / kMaxCols) & 15, n = o % kMaxCols;
             const int u = u0 + r * step;
             const int P = ci->heads[u / g.n_units];
             float bv = 0.f;
@@ -892,7 +933,7 @@ __device__ void run_call(Cons& c, int call) {
           if (pos >= 1 && j >= 0 && j <= p.K) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
             p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
-                v * sm.inv_rms[n] + bias_s[(u - chunk_u0) * 128 + rr * 8 + n];
+                v * sm.inv_rms[n] + bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
           }
         });
     if (c.abort_) return;
@@ -929,7 +970,7 @@ __device__ void run_call(Cons& c, int call) {
         consumer_sync();
       }
     } else {
-      TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
+      TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1);
       const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
       int pair = 0;
       for (int r = 0; r < n_rows; ++r) {
@@ -994,8 +1035,8 @@ __device__ void accept_step(Cons& c, int call, int s) {
   const unsigned sid = p.stream_ids[s], fid = p.frame_ids[s];
   const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxRows * (kMaxDraft + 1);
-  const TopkRec* prev = p.topk + (size_t)((call + 1) & 1) * kMaxRows * (kMaxDraft + 1);
+  const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1);
+  const TopkRec* prev = p.topk + (size_t)((call + 1) & 1) * kMaxCols * (kMaxDraft + 1);
   TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // staged records
   const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
   __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
@@ -1240,13 +1281,30 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
       for (int P = lo; P <= hi; ++P) mask |= 1u << P;
       // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft
       // i-1; a noisy-target pass feeds its one code
-      for (int n = 0; n < st->n_rows && ci->M < kMaxRows; ++n) {
+      for (int n = 0; n < st->n_rows && ci->M < kMaxCols; ++n) {
         const int r = ci->M++;
         ci->r_s[r] = s;
         ci->r_n[r] = n;
         ci->r_pos[r] = st->pos0 + n;
-        ci->r_id[r] = st->emu ? st->emu_in
-                              : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+        int id = st->emu ? st->emu_in
+                         : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+        // layer-0 input row: cond (position 0), the c0 embedding vector (position 1 without
+        // a c0 table), else row `id` of table pos - 1
+        const int pos = st->pos0 + n;
+        if (pos == 0 || (pos == 1 && p.C0V == 0)) {
+          ci->r_src[r] = reinterpret_cast<const uint8_t*>((pos == 0 ? p.cond : p.c0emb) + (size_t)s * p.H);
+          ci->r_f32[r] = 1;
+        } else {
+          const int table = pos - 1;
+          if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {   // a c0 outside table 0: fail the frame
+            atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
+            id = 0;
+          }
+          const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+          ci->r_src[r] = p.embed + (long long)table * p.embed_stride + (long long)id * p.H * es;
+          ci->r_f32[r] = p.wdtype == MCD_WEIGHT_BF16 ? 0 : 1;
+        }
+        ci->r_id[r] = id;
       }
     }
     ci->n_heads = 0;
@@ -1260,7 +1318,7 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
   return true;
 }
 
-template <int WT>
+template <int WT, bool WIDE>
 __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constant__ FrameParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   Smem sm = smem_layout(smem_raw);
@@ -1287,7 +1345,7 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
       if (sm.ci->all_done) break;
       // a stepwise launch runs one verify call and the noisy-target passes that follow it
       if (p.single_call && call != call0 && !sm.ci->emu) break;
-      run_call<WT>(c, call);
+      run_call<WT, WIDE>(c, call);
       if (c.abort_) break;
       if (sm.flags[2]) {
         if (sm.ci->emu)
@@ -1304,24 +1362,29 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
 }
 
 // host-side launcher ------------------------------------------------------------------
+// WIDE: the call may pack more than 8 rows (several streams), so the operand has up to 4
+// n-tiles; the narrow instantiation serves single-stream decoding.
+template <int WT, bool WIDE>
+static void* frame_entry() {
+  return (void*)frame_kernel<WT, WIDE>;
+}
+
 cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream) {
   void* args[] = {const_cast<FrameParams*>(&p)};
-  if (p.wdtype == MCD_WEIGHT_BF16)
-    return cudaLaunchCooperativeKernel((void*)frame_kernel<MCD_WEIGHT_BF16>, dim3(p.n_cta), dim3(kThreads), args,
-                                       (size_t)kSmemBytes, stream);
-  return cudaLaunchCooperativeKernel((void*)frame_kernel<MCD_WEIGHT_F32>, dim3(p.n_cta), dim3(kThreads), args,
-                                     (size_t)kSmemBytes, stream);
+  const bool wide = p.S * max(p.K + 1, 2) > kMaxRows;
+  void* fn = p.wdtype == MCD_WEIGHT_BF16 ? (wide ? frame_entry<MCD_WEIGHT_BF16, true>() : frame_entry<MCD_WEIGHT_BF16, false>())
+                                         : (wide ? frame_entry<MCD_WEIGHT_F32, true>() : frame_entry<MCD_WEIGHT_F32, false>());
+  return cudaLaunchCooperativeKernel(fn, dim3(p.n_cta), dim3(kThreads), args, (size_t)kSmemBytes, stream);
 }
 
 cudaError_t prepare_frame_kernel(int* max_ctas_per_sm) {
-  cudaError_t e = cudaFuncSetAttribute((void*)frame_kernel<MCD_WEIGHT_BF16>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute((void*)frame_kernel<MCD_WEIGHT_F32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           kSmemBytes);
-  if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(max_ctas_per_sm, (void*)frame_kernel<MCD_WEIGHT_BF16>,
-                                                       kThreads, kSmemBytes);
+  void* fns[4] = {frame_entry<MCD_WEIGHT_BF16, false>(), frame_entry<MCD_WEIGHT_BF16, true>(),
+                  frame_entry<MCD_WEIGHT_F32, false>(), frame_entry<MCD_WEIGHT_F32, true>()};
+  for (void* fn : fns) {
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(max_ctas_per_sm, fns[0], kThreads, kSmemBytes);
 }
 
 int frame_smem_bytes() { return kSmemBytes; }

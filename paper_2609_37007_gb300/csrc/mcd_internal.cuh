@@ -16,7 +16,8 @@
 
 namespace mcd {
 
-constexpr int kMaxRows = 8;          // rows of one call over all streams (packed operand columns)
+constexpr int kMaxRows = 8;          // rows of one stream in one call (K + 1 <= 8; first call uses 2)
+constexpr int kMaxCols = 32;         // rows of one call over all streams (packed operand columns)
 constexpr int kMaxStreams = 8;       // streams decoded together by one launch
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
@@ -32,7 +33,7 @@ constexpr int kNumSlots = 4;
 constexpr int kChunk = 3;            // units of one stage multiplied before one epilogue pass (<= kNumSlots)
 constexpr int kActBytes = 32768;     // fp32 activation rows / attention / top-k scratch
 constexpr int kBfragBytes = 32768;   // B operand (activations) of the unit GEMMs
-constexpr int kRedBytes = 4096;      // one cross-warp reduction buffer (x2)
+constexpr int kRedBytes = 16384;     // cross-warp partial tiles of a chunk of units
 
 enum MatKind { MAT_QKV = 0, MAT_WO = 1, MAT_GU = 2, MAT_WD = 3, MAT_HEAD = 4, MAT_COUNT = 5 };
 
@@ -106,13 +107,13 @@ struct FrameParams {
   long long embed_stride;
   const float2* rope;          // [kMaxPos][D/2] (cos, sin)
   // buffers
-  float* x;                    // [kMaxRows][H]
-  float* qkv;                  // [kMaxRows][qkv_dim]
-  float* mbuf;                 // [kMaxRows][F]
-  float* logits;               // [kMaxRows][kMaxDraft+1][V]
+  float* x;                    // [kMaxCols][H]
+  float* qkv;                  // [kMaxCols][qkv_dim]
+  float* mbuf;                 // [kMaxCols][F]
+  float* logits;               // [kMaxCols][kMaxDraft+1][V]
   float* kcache;               // [S][L][NKV][kMaxPos][D]
   float* vcache;
-  TopkRec* topk;               // [kMaxRows][kMaxDraft+1]
+  TopkRec* topk;               // [2][kMaxCols][kMaxDraft+1]
   TopkRec* draftq;             // [kMaxDraft] pending drafts' q
   DevState* st;                // [S]
   unsigned* ctr;               // [kMaxCalls][ctr_stride]

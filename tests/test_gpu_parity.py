@@ -244,7 +244,8 @@ def decode_many(env, frames, frame_idx, stream_ids):
 
 
 @pytest.mark.parametrize("cfg", [TINY.replace(max_streams=2), TINY.replace(draft_len=0, max_streams=4),
-                                 TINY.replace(draft_len=1, max_streams=4)])
+                                 TINY.replace(draft_len=1, max_streams=4), TINY.replace(draft_len=3, max_streams=8),
+                                 TINY.replace(draft_len=3, max_streams=3)])
 def test_batched_streams_trace_parity(cfg):
     """Several streams in one launch, rows re-packed every call: each stream's calls match
     the oracle decoding that stream alone (its own counters and KV cache)."""
@@ -262,13 +263,15 @@ def test_batched_streams_trace_parity(cfg):
     env.dec.close()
 
 
-def test_batched_streams_full_size():
-    cfg = MCD.replace(max_streams=2)
+@pytest.mark.parametrize("n_streams", [2, 4, 8])
+def test_batched_streams_full_size(n_streams):
+    """Up to 16 packed rows use the bf16 hi/lo operand, 17..32 a single bf16 operand."""
+    cfg = MCD.replace(max_streams=n_streams)
     env = Env(cfg)
-    fidx, sids = [4, 9], [3, 5]
+    fidx, sids = [4 + 5 * s for s in range(n_streams)], [3 + 2 * s for s in range(n_streams)]
     frames = [make_frame(cfg, f) for f in fidx]
     codes, st, trs = decode_many(env, frames, fidx, sids)
-    for s in range(2):
+    for s in range(n_streams):
         assert st[s, 4] == 0 and st[s, 1] == cfg.n_pos
         err = check_trace_against_oracle(cfg, env.model, frames[s], sids[s], fidx[s], trs[s], codes[s],
                                          int(st[s, 0]), logit_tol=2e-2)
@@ -278,7 +281,7 @@ def test_batched_streams_full_size():
 
 def test_batched_streams_reject_too_many_rows():
     with pytest.raises(mcd.MCDError):
-        mcd.Decoder(MCD.replace(max_streams=3))       # 3 x (K + 1) > 8 packed rows
+        mcd.Decoder(MCD.replace(max_streams=8, draft_len=4))       # 8 x (K + 1) > 32 packed rows
 
 
 # ------------------------------------------------- noisy-target drafts (K sweep) ------
