@@ -243,6 +243,53 @@ def run_sweep(args, weights):
                               "us_per_call_from": "position-aware drafter frames at the same K"}), flush=True)
 
 
+def run_streams(args, weights):
+    """Batched independent streams: one mcd_decode_frames launch decodes a frame for each of
+    B streams (rows re-packed every call).  Prints one JSON line per B: aggregate accepted
+    tokens/s over all streams, launches (frame sets) per second, calls per launch."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    from paper_2609_37007_gb300.synth import MCD, make_frames
+    _build.build()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    n = args.stream_launches
+    for B in args.streams:
+        cfg = MCD.replace(max_streams=B)
+        dec = mcd.Decoder(cfg, weights, stream)
+        cond_h, c0_h, _ = make_frames(cfg, B * (n + 3), first=3_000_000)
+        cond = torch.from_numpy(cond_h).to(dev).view(n + 3, B, cfg.hidden)
+        c0 = torch.from_numpy(c0_h).to(dev).view(n + 3, B)
+        codes = torch.zeros((n + 3, B, cfg.n_pos), dtype=torch.int32, device=dev)
+        stats = torch.zeros((n + 3, B, 8), dtype=torch.int32, device=dev)
+        sids = list(range(B))
+
+        def launch(i):
+            mcd.mcd_decode_frames(dec.ctx, sids, [i] * B, cond[i], c0[i], None, codes[i], stats[i])
+
+        for i in range(3):
+            launch(i)
+        mcd.mcd_sync(dec.ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(3, n + 3):
+            launch(i)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mcd.mcd_sync(dec.ctx)
+        st = stats.cpu().numpy()[3:]
+        assert (st[:, :, 4] == 0).all() and (st[:, :, 1] == cfg.n_pos).all()
+        t = e0.elapsed_time(e1) / 1e3
+        toks = int(st[:, :, 1].sum())
+        calls = int(st[:, :, 0].max(axis=1).sum())            # a launch runs until its slowest stream is done
+        print(json.dumps({"streams": B, "tokens_per_s": toks / t, "launches_per_s": n / t,
+                          "us_per_call": 1e6 * t / calls, "calls_per_launch": calls / n,
+                          "tokens_per_call_per_stream": float(st[:, :, 1].sum() / st[:, :, 0].sum()),
+                          "launches": n, "workload": WORKLOAD.replace("single stream", f"{B} streams")}), flush=True)
+        dec.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -256,6 +303,9 @@ def main():
     ap.add_argument("--sweep", action="store_true", help="noisy-target K x sigma sweep instead of the bench line")
     ap.add_argument("--sweep-frames", type=int, default=100)
     ap.add_argument("--sigmas", type=float, nargs="+", default=[0.05, 0.1, 0.25, 0.5, 1.0, 2.0])
+    ap.add_argument("--streams", type=int, nargs="*", default=None,
+                    help="batched-stream runs for these B instead of the bench line (e.g. --streams 1 2 4 8)")
+    ap.add_argument("--stream-launches", type=int, default=100)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -264,6 +314,8 @@ def main():
     weights = make_weights(cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, weights)
+    if args.streams:
+        return run_streams(args, weights)
     if args.sweep:
         # one weight set with offsets b_1..b_7 serves every K (extra tensors are ignored)
         return run_sweep(args, make_weights(cfg.replace(draft_len=7)))
