@@ -415,7 +415,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   ok = ok && make_geom(p.H, p.F, 1, tb, 1024, p.g[MAT_WD]);
   ok = ok && make_geom(p.V, p.H, 1, tb, 1024, p.g[MAT_HEAD]) && p.g[MAT_HEAD].n_kc == 1;
   if (!ok) return fail(MCD_ERR_UNSUPPORTED);
-  p.ctr_stride = ctr_ready(p.L) + 2;
+  p.ctr_stride = ctr_count(p.L);
 
   // weight arena
   const size_t sq = p.g[MAT_QKV].stride, so = p.g[MAT_WO].stride, sg = p.g[MAT_GU].stride, sd = p.g[MAT_WD].stride;
@@ -455,6 +455,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.x, sizeof(float) * kMaxCols * p.H)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.qkv, sizeof(float) * kMaxCols * p.qkv_dim)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxCols * p.F)) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.attn, sizeof(float) * kMaxCols * p.NH * p.D)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxCols * (kMaxDraft + 1) * p.V)) != cudaSuccess)
     return fail(cuda_status(e));
   p.kv_stride = (long long)p.L * p.NKV * kMaxPos * p.D;

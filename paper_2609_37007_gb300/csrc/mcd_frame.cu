@@ -819,9 +819,46 @@ __device__ void run_call(Cons& c, int call) {
 
     // ---- S2: attention (per query head) -> Wo + residual --------------------------------
     // Unit u of Wo covers m-block u % n_mb of query head h = u / n_mb (its k-chunk); its B
-    // operand is head h's attention output.
+    // operand is head h's attention output.  Single stream: the CTAs holding head h's Wo
+    // units compute that attention themselves.  Several streams: first one task per
+    // (stream, query head) spread over the CTAs writes the outputs to global memory, then
+    // Wo reads them.
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
-    {
+    if (WIDE) {
+      const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
+      for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
+        const int i = t / p.NH, h = t - i * p.NH, s = ci->act[i];
+        const int nr = ci->nrows[s], base = ci->base[s];
+        attention_stream(c, l, h, (h % group) == 0, nr, ci->pos0[s], base, s);
+        for (int q = threadIdx.x; q < nr * (D >> 2); q += kConsumerThreads) {
+          const int n = q / (D >> 2), d4 = q - n * (D >> 2);
+          reinterpret_cast<float4*>(p.attn + (size_t)(base + n) * p.NH * D + h * D)[d4] =
+              reinterpret_cast<const float4*>(sm.act + (base + n) * D)[d4];
+        }
+        consumer_sync();
+      }
+      cons_signal(c, ctr + ctr_att(L, l), call, kTimelineSlots);
+      if (!cons_wait(c, ctr + ctr_att(L, l), N)) return;
+      const MatGeom& g = p.g[MAT_WO];
+      if (threadIdx.x == 0) sm.flags[3] = -1;
+      consumer_sync();
+      run_stage<WT, WIDE>(
+          c, call, 4 * l + 1, g.n_units, D, n_rows, [&](int u) { return u / g.n_mb; },
+          [&](int u, int, int) {
+            const int h = u / g.n_mb;
+            if (sm.flags[3] != h) {
+              const float* src = p.attn + h * D;
+              prep_operand<WT, WIDE>(c, n_rows, D, 0, D, nullptr, false,
+                                     [&](int n, int k) { return ld_global2(src + (size_t)n * p.NH * D + k); });
+              if (threadIdx.x == 0) sm.flags[3] = h;
+            }
+          },
+          [&](int u, int mi, int rr, int n, float v, float) {
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
+            atomicAdd(p.x + (size_t)n * H + row, v);
+          });
+      if (c.abort_) return;
+    } else {
       const MatGeom& g = p.g[MAT_WO];
       const int group = p.NH / p.NKV;
       if (threadIdx.x == 0) sm.flags[3] = -1;

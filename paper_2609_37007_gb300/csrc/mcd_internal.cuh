@@ -110,6 +110,7 @@ struct FrameParams {
   float* x;                    // [kMaxCols][H]
   float* qkv;                  // [kMaxCols][qkv_dim]
   float* mbuf;                 // [kMaxCols][F]
+  float* attn;                 // [kMaxCols][NH*D] attention outputs (batched calls)
   float* logits;               // [kMaxCols][kMaxDraft+1][V]
   float* kcache;               // [S][L][NKV][kMaxPos][D]
   float* vcache;
@@ -145,6 +146,8 @@ __host__ __device__ inline int ctr_heads(int L) { return L * 4; }
 __host__ __device__ inline int ctr_topk(int L) { return L * 4 + 1; }
 __host__ __device__ inline int ctr_ready(int L) { return L * 4 + 2; }
 __host__ __device__ inline int ctr_accept(int L) { return L * 4 + 3; }
+__host__ __device__ inline int ctr_att(int L, int layer) { return L * 4 + 4 + layer; }   // batched attention
+__host__ __device__ inline int ctr_count(int L) { return L * 5 + 4; }
 
 // ---------------------------------------------------------------------------------------
 // PTX helpers
