@@ -43,13 +43,10 @@ struct CallInfo {
   // packed rows: stream, row within the stream, position, code fed, layer-0 input row
   int r_s[kMaxCols], r_n[kMaxCols], r_pos[kMaxCols], r_id[kMaxCols], r_f32[kMaxCols];
   const uint8_t* r_src[kMaxCols];
-  // per stream (index = stream)
+  // per stream (index = stream): its state and the derived packing
+  DevState st[kMaxStreams];
   int act[kMaxStreams];        // active streams in packing order
-  int a[kMaxStreams], nd[kMaxStreams], pos0[kMaxStreams], nrows[kMaxStreams], fr[kMaxStreams];
-  int done[kMaxStreams], qrow[kMaxStreams], base[kMaxStreams], round[kMaxStreams], emu_n[kMaxStreams];
-  int plo[kMaxStreams], phi[kMaxStreams];
-  int calls[kMaxStreams], heads_rd[kMaxStreams], kvrows[kMaxStreams], rowsfed[kMaxStreams];
-  int drafted[kMaxStreams], accepted[kMaxStreams], drafts[kMaxStreams][kMaxDraft], code_a[kMaxStreams];
+  int base[kMaxStreams], plo[kMaxStreams], phi[kMaxStreams];
 };
 
 struct Smem {
@@ -765,7 +762,7 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const CallInfo* ci = c.sm.ci;
   for (int i = 0; i < ci->n_act; ++i) {
     const int s = ci->act[i];
-    attention_stream(c, layer, h, write_kv, ci->nrows[s], ci->pos0[s], ci->base[s], s);
+    attention_stream(c, layer, h, write_kv, ci->st[s].n_rows, ci->st[s].pos0, ci->base[s], s);
   }
 }
 
@@ -828,8 +825,8 @@ __device__ void run_call(Cons& c, int call) {
       const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
       for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
         const int i = t / p.NH, h = t - i * p.NH, s = ci->act[i];
-        const int nr = ci->nrows[s], base = ci->base[s];
-        attention_stream(c, l, h, (h % group) == 0, nr, ci->pos0[s], base, s);
+        const int nr = ci->st[s].n_rows, base = ci->base[s];
+        attention_stream(c, l, h, (h % group) == 0, nr, ci->st[s].pos0, base, s);
         for (int q = threadIdx.x; q < nr * (D >> 2); q += kConsumerThreads) {
           const int n = q / (D >> 2), d4 = q - n * (D >> 2);
           reinterpret_cast<float4*>(p.attn + (size_t)(base + n) * p.NH * D + h * D)[d4] =
@@ -986,7 +983,7 @@ __device__ void run_call(Cons& c, int call) {
       // noisy-target pass j = emu (one stream): q = fp32(target logits + sigma N(0,1)) of
       // position pos0 (Box-Muller pairs of purpose 3 + v/2 under the verify round's counters)
       if (blockIdx.x == 0) {
-        const int emu = ci->emu, pos0 = ci->pos0[0], round = ci->round[0];
+        const int emu = ci->emu, pos0 = ci->st[0].pos0, round = ci->st[0].round;
         const float* lg = p.logits;                                   // row 0, j = 0
         float* zq = p.logits + (size_t)1 * p.V;                        // row 0, slot j = 1
         for (int pr = threadIdx.x; pr < (p.V >> 1); pr += kConsumerThreads) {
@@ -1067,8 +1064,8 @@ __device__ void accept_step(Cons& c, int call, int s) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
   const CallInfo* ci = sm.ci;
-  const int a = ci->a[s], n_d = ci->nd[s], pos0 = ci->pos0[s], n_rows = ci->nrows[s];
-  const int qrow = ci->qrow[s], round = ci->round[s], base = ci->base[s];
+  const int a = ci->st[s].a, n_d = ci->st[s].n_d, pos0 = ci->st[s].pos0, n_rows = ci->st[s].n_rows;
+  const int qrow = ci->st[s].q_row, round = ci->st[s].round, base = ci->base[s];
   const unsigned sid = p.stream_ids[s], fid = p.frame_ids[s];
   const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1080,23 +1077,61 @@ __device__ void accept_step(Cons& c, int call, int s) {
   if (s == 0) timeline(c, call, 4, true);
   // p of positions a+1..: this call's verify records (packed rows base + ...); q of the
   // drafts: the previous call's records of its packed row qrow, or the noisy-target passes'
-  stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
+  const int n_pq = n_p + n_d;
+  const bool pre = false;   // staging every row's draft records up front measured slower
+  const int n_dr = pre ? n_rows * p.K : 0;
+  stage_records(srec, n_pq + n_dr, p.top_k, [&](int r) {
+    if (r >= n_pq) {
+      const int rr = (r - n_pq) / p.K, j = 1 + (r - n_pq) % p.K;
+      return (const TopkRec*)(cur + (base + rr) * (kMaxDraft + 1) + j);
+    }
     return r < n_p ? cur + (base + a + 1 + r - pos0) * (kMaxDraft + 1)
                    : (noisy ? p.draftq + (r - n_p) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p));
   });
   consumer_sync();
   if (s == 0) timeline(c, call, 5, true);
-  if (warp == 0) {
-    int drafts[kMaxDraft + 1];
-    for (int i = 0; i < n_d; ++i) drafts[i] = ci->drafts[s][i];
-    AcceptResult r = warp_accept(
-        a, n_d, p.P, drafts, [&](int i) { return (const TopkRec*)(srec + i); },
-        [&](int i) { return (const TopkRec*)(srec + n_p + i); }, p.seed, sid, fid, round);
-    if (lane == 0) {
-      for (int t = 0; t < r.n_emit; ++t) s_emit[t] = r.emitted[t];
-      s_nemit = r.n_emit;
-      s_nacc = r.n_acc;
+  // The acceptance rule of every draft in parallel, warp i for draft i (its accept test and
+  // the residual draw it would take if it were the first rejection) and warp n_d for the
+  // bonus draw; then the chain is read off in order: drafts kept up to the first rejection,
+  // whose residual code ends the call, else the bonus code (same decisions as testing the
+  // drafts one after another).
+  __shared__ int s_ok[kMaxDraft + 1], s_alt[kMaxDraft + 1];
+  if (warp <= n_d) {
+    const int i = warp, pos = a + 1 + i;
+    if (i < n_d) {
+      const TopkRec* pr = srec + i;
+      const TopkRec* qr = srec + n_p + i;
+      const int d = ci->st[s].drafts[i];
+      const unsigned long long wp = warp_weight(pr, d), wq = warp_weight(qr, d);
+      const unsigned long long U = uniform_U(p.seed, sid, fid, round, pos, PURPOSE_ACCEPT);
+      const bool ok = lt128(mul128x64(mul64(U, wq), pr->S), shl53(wp * qr->S));
+      int alt = -1;
+      if (!ok) alt = warp_residual(pr, qr, uniform_U(p.seed, sid, fid, round, pos, PURPOSE_TARGET));
+      if (lane == 0) {
+        s_ok[i] = ok ? 1 : 0;
+        s_alt[i] = alt;
+      }
+    } else if (pos <= p.P) {
+      const int b = warp_draw(srec + n_d, uniform_U(p.seed, sid, fid, round, pos, PURPOSE_TARGET));
+      if (lane == 0) s_alt[i] = b;
     }
+  }
+  consumer_sync();
+  if (threadIdx.x == 0) {
+    int ne = 0, na = 0;
+    bool rejected = false;
+    for (int i = 0; i < n_d && !rejected; ++i) {
+      if (s_ok[i]) {
+        s_emit[ne++] = ci->st[s].drafts[i];
+        ++na;
+      } else {
+        s_emit[ne++] = s_alt[i];
+        rejected = true;
+      }
+    }
+    if (!rejected && a + 1 + n_d <= p.P) s_emit[ne++] = s_alt[n_d];
+    s_nemit = ne;
+    s_nacc = na;
   }
   consumer_sync();
   if (s == 0) timeline(c, call, 6, true);
@@ -1106,11 +1141,14 @@ __device__ void accept_step(Cons& c, int call, int s) {
   // draft records of row m (the row whose head emitted the last code): one warp each (the
   // noisy-target passes that follow draw their drafts themselves)
   if (!noisy) {
-    stage_records(srec, n_next, p.top_k, [&](int r) { return cur + (base + m) * (kMaxDraft + 1) + 1 + r; });
-    consumer_sync();
+    if (!pre) {        // too many rows x drafts to stage up front: row m's records now
+      stage_records(srec + n_pq, n_next, p.top_k, [&](int r) { return cur + (base + m) * (kMaxDraft + 1) + 1 + r; });
+      consumer_sync();
+    }
+    const TopkRec* drec = srec + n_pq + (pre ? m * p.K : 0);
     for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
       const unsigned long long U = uniform_U(p.seed, sid, fid, round, a_new + j, PURPOSE_DRAFT);
-      const int d = warp_draw(srec + j - 1, U);
+      const int d = warp_draw(drec + (j - 1), U);
       if (lane == 0) s_next[j - 1] = d;
     }
     consumer_sync();
@@ -1126,9 +1164,9 @@ __device__ void accept_step(Cons& c, int call, int s) {
     if (!noisy)
       for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
     for (int t = 0; t < s_nemit; ++t) st->emitted_last[t] = s_emit[t];
-    const int calls = ci->calls[s] + 1, heads = ci->heads_rd[s] + ci->phi[s] - ci->plo[s] + 1;
-    const int kvr = ci->kvrows[s] + pos0 + n_rows, rf = ci->rowsfed[s] + n_rows;
-    const int drafted = ci->drafted[s] + n_d, accepted = ci->accepted[s] + s_nacc;
+    const int calls = ci->st[s].calls + 1, heads = ci->st[s].heads_read + ci->phi[s] - ci->plo[s] + 1;
+    const int kvr = ci->st[s].kv_rows + pos0 + n_rows, rf = ci->st[s].rows_fed + n_rows;
+    const int drafted = ci->st[s].drafted + n_d, accepted = ci->st[s].accepted + s_nacc;
     st->n_emit_last = s_nemit;
     st->n_acc_last = s_nacc;
     st->a = a_new;
@@ -1174,7 +1212,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
   }
   consumer_sync();
   // optional outputs: trace and stepwise logits
-  const int fr = ci->fr[s];
+  const int fr = ci->st[s].first_head_row;
   if (p.trace && round < kMaxCalls) {
     uint8_t* tb = p.trace + (size_t)s * p.trace_stride;
     mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(tb) + round;
@@ -1184,7 +1222,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
       tr->pos0 = pos0;
       tr->n_drafts = n_d;
       for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci->r_id[base + n] : -1;
-      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? ci->drafts[s][i] : -1;
+      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? ci->st[s].drafts[i] : -1;
       tr->n_acc = s_nacc;
       tr->n_emit = s_nemit;
       for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < s_nemit ? s_emit[t] : -1;
@@ -1216,8 +1254,8 @@ __device__ void accept_step(Cons& c, int call, int s) {
     // the last acceptance of the call releases the next call
     __threadfence();
     unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
-    if (atomicAdd(ctr + ctr_accept(p.L), 1u) == (unsigned)ci->n_act - 1u) {
-      __threadfence();
+    if (ci->n_act == 1 || atomicAdd(ctr + ctr_accept(p.L), 1u) == (unsigned)ci->n_act - 1u) {
+      if (ci->n_act > 1) __threadfence();
       atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
     }
   }
@@ -1230,7 +1268,7 @@ __device__ void emu_step(Cons& c, int call) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
   const CallInfo* ci = sm.ci;
-  const int j = ci->emu, n = ci->emu_n[0], round = ci->round[0], pos0 = ci->pos0[0], a = ci->a[0];
+  const int j = ci->emu, n = ci->st[0].emu_n, round = ci->st[0].round, pos0 = ci->st[0].pos0, a = ci->st[0].a;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);
   __shared__ int s_d;
@@ -1272,83 +1310,72 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
   if (!first) {
     if (!cons_wait(c, p.ctr + (size_t)call * p.ctr_stride + ctr_ready(p.L), 1u)) return false;
   }
-  // one parallel read of every stream's state into the act region
+  // one parallel read of every stream's state straight into the call snapshot
   constexpr int kWords = sizeof(DevState) / 4;
-  int* stw = reinterpret_cast<int*>(sm.act);
+  CallInfo* ci = sm.ci;
+  int* stw = reinterpret_cast<int*>(ci->st);
   for (int i = threadIdx.x; i < p.S * kWords; i += kConsumerThreads)
     stw[i] = __ldcg(reinterpret_cast<const int*>(p.st) + i);
   consumer_sync();
+  const DevState* sts = ci->st;
+  // packing order, row bases and the union of heads (one thread)
   if (threadIdx.x == 0) {
-    CallInfo* ci = sm.ci;
-    const DevState* sts = reinterpret_cast<const DevState*>(stw);
     ci->call = call;
-    ci->M = 0;
-    ci->n_act = 0;
-    ci->all_done = 1;
     ci->emu = sts[0].emu;
     ci->round0 = sts[0].round;
+    int M = 0, n_act = 0;
     unsigned mask = 0;
     for (int s = 0; s < p.S; ++s) {
-      const DevState* st = sts + s;
-      ci->done[s] = st->done;
-      ci->a[s] = st->a;
-      ci->nd[s] = st->n_d;
-      ci->pos0[s] = st->pos0;
-      ci->nrows[s] = st->n_rows;
-      ci->fr[s] = st->first_head_row;
-      ci->qrow[s] = st->q_row;
-      ci->round[s] = st->round;
-      ci->emu_n[s] = st->emu_n;
-      ci->calls[s] = st->calls;
-      ci->heads_rd[s] = st->heads_read;
-      ci->kvrows[s] = st->kv_rows;
-      ci->rowsfed[s] = st->rows_fed;
-      ci->drafted[s] = st->drafted;
-      ci->accepted[s] = st->accepted;
-      for (int i = 0; i < kMaxDraft; ++i) ci->drafts[s][i] = st->drafts[i];
-      ci->code_a[s] = st->codes[st->a];
-      if (st->done) continue;
-      ci->all_done = 0;
-      ci->act[ci->n_act++] = s;
-      ci->base[s] = ci->M;
+      ci->base[s] = M;
+      if (sts[s].done) continue;
+      ci->act[n_act++] = s;
+      M = min(M + sts[s].n_rows, kMaxCols);
       int lo, hi;
-      head_range(p, st->a, st->pos0, st->n_rows, st->emu, lo, hi);
+      head_range(p, sts[s].a, sts[s].pos0, sts[s].n_rows, sts[s].emu, lo, hi);
       ci->plo[s] = lo;
       ci->phi[s] = hi;
-      for (int P = lo; P <= hi; ++P) mask |= 1u << P;
-      // ids fed at each row: first call [cond, c0]; later calls row 0 = c_a, row i = draft
-      // i-1; a noisy-target pass feeds its one code
-      for (int n = 0; n < st->n_rows && ci->M < kMaxCols; ++n) {
-        const int r = ci->M++;
-        ci->r_s[r] = s;
-        ci->r_n[r] = n;
-        ci->r_pos[r] = st->pos0 + n;
-        int id = st->emu ? st->emu_in
-                         : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
-        // layer-0 input row: cond (position 0), the c0 embedding vector (position 1 without
-        // a c0 table), else row `id` of table pos - 1
-        const int pos = st->pos0 + n;
-        if (pos == 0 || (pos == 1 && p.C0V == 0)) {
-          ci->r_src[r] = reinterpret_cast<const uint8_t*>((pos == 0 ? p.cond : p.c0emb) + (size_t)s * p.H);
-          ci->r_f32[r] = 1;
-        } else {
-          const int table = pos - 1;
-          if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {   // a c0 outside table 0: fail the frame
-            atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
-            id = 0;
-          }
-          const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
-          ci->r_src[r] = p.embed + (long long)table * p.embed_stride + (long long)id * p.H * es;
-          ci->r_f32[r] = p.wdtype == MCD_WEIGHT_BF16 ? 0 : 1;
-        }
-        ci->r_id[r] = id;
-      }
+      mask |= (hi >= lo) ? ((2u << hi) - (1u << lo)) : 0u;     // bits lo..hi
     }
-    ci->n_heads = 0;
+    ci->M = M;
+    ci->n_act = n_act;
+    ci->all_done = n_act == 0;
+    int nh = 0;
     while (mask) {
-      ci->heads[ci->n_heads++] = __ffs(mask) - 1;
+      ci->heads[nh++] = __ffs(mask) - 1;
       mask &= mask - 1;
     }
+    ci->n_heads = nh;
+  }
+  consumer_sync();
+  // (3) one thread per packed row: stream, position, code fed, layer-0 input row
+  if (threadIdx.x < ci->M) {
+    const int r = threadIdx.x;
+    int s = 0;
+    for (int i = 0; i < ci->n_act; ++i)
+      if (ci->base[ci->act[i]] <= r) s = ci->act[i];
+    const DevState* st = sts + s;
+    const int n = r - ci->base[s], pos = st->pos0 + n;
+    int id = st->emu ? st->emu_in
+                     : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+    // layer-0 input row: cond (position 0), the c0 embedding vector (position 1 without a
+    // c0 table), else row `id` of table pos - 1
+    if (pos == 0 || (pos == 1 && p.C0V == 0)) {
+      ci->r_src[r] = reinterpret_cast<const uint8_t*>((pos == 0 ? p.cond : p.c0emb) + (size_t)s * p.H);
+      ci->r_f32[r] = 1;
+    } else {
+      const int table = pos - 1;
+      if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {   // a c0 outside table 0: fail the frame
+        atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
+        id = 0;
+      }
+      const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+      ci->r_src[r] = p.embed + (long long)table * p.embed_stride + (long long)id * p.H * es;
+      ci->r_f32[r] = p.wdtype == MCD_WEIGHT_BF16 ? 0 : 1;
+    }
+    ci->r_s[r] = s;
+    ci->r_n[r] = n;
+    ci->r_pos[r] = pos;
+    ci->r_id[r] = id;
   }
   consumer_sync();
   timeline(c, call, 0);
