@@ -1078,16 +1078,15 @@ __device__ void accept_step(Cons& c, int call, int s) {
   // p of positions a+1..: this call's verify records (packed rows base + ...); q of the
   // drafts: the previous call's records of its packed row qrow, or the noisy-target passes'
   const int n_pq = n_p + n_d;
-  const bool pre = false;   // staging every row's draft records up front measured slower
-  const int n_dr = pre ? n_rows * p.K : 0;
-  stage_records(srec, n_pq + n_dr, p.top_k, [&](int r) {
-    if (r >= n_pq) {
-      const int rr = (r - n_pq) / p.K, j = 1 + (r - n_pq) % p.K;
-      return (const TopkRec*)(cur + (base + rr) * (kMaxDraft + 1) + j);
-    }
+  stage_records(srec, n_pq, p.top_k, [&](int r) {
     return r < n_p ? cur + (base + a + 1 + r - pos0) * (kMaxDraft + 1)
                    : (noisy ? p.draftq + (r - n_p) : prev + qrow * (kMaxDraft + 1) + 1 + (r - n_p));
   });
+  // The row m whose head drafts the next call is known only after acceptance, so the warps
+  // that take no part in it stage every row's draft records meanwhile (if they fit).
+  const int idle0 = (n_d + 1) * 32;
+  const bool pre = !noisy && idle0 < kConsumerThreads &&
+                   (size_t)(n_pq + n_rows * p.K) * sizeof(TopkRec) <= (size_t)(kActBytes + kBfragBytes);
   consumer_sync();
   if (s == 0) timeline(c, call, 5, true);
   // The acceptance rule of every draft in parallel, warp i for draft i (its accept test and
@@ -1096,6 +1095,16 @@ __device__ void accept_step(Cons& c, int call, int s) {
   // whose residual code ends the call, else the bonus code (same decisions as testing the
   // drafts one after another).
   __shared__ int s_ok[kMaxDraft + 1], s_alt[kMaxDraft + 1];
+  if (pre && (int)threadIdx.x >= idle0) {
+    constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kWWord = offsetof(TopkRec, W) / 4;
+    const int words = kIdsWord + 2 * p.top_k, nrec = n_rows * p.K;
+    for (int i = threadIdx.x - idle0; i < nrec * words; i += kConsumerThreads - idle0) {
+      const int r = i / words, w = i - r * words;
+      const int off = w < kIdsWord ? w : (w < kIdsWord + p.top_k ? w : kWWord + (w - kIdsWord - p.top_k));
+      const TopkRec* src = cur + (base + r / p.K) * (kMaxDraft + 1) + 1 + r % p.K;
+      reinterpret_cast<int*>(srec + n_pq + r)[off] = __ldcg(reinterpret_cast<const int*>(src) + off);
+    }
+  }
   if (warp <= n_d) {
     const int i = warp, pos = a + 1 + i;
     if (i < n_d) {
