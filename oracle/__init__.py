@@ -15,6 +15,8 @@ Modules:
   sampler      top-k / temperature / softmax, categorical draw, accept test, residual.
   model        fp64 MultiCodeDecoder rows with a per-frame KV cache.
   frame        autoregressive and speculative frame procedures.
+  codedecoder  the outer CodeDecoder (one call per frame, emits c0) and the full frame
+               pipeline of Fig. 1 (prompt prefill, c0, MultiCodeDecoder, input sum).
   enumeration  exact output distributions of both procedures (losslessness pin).
   accounting   the paper's real-time call arithmetic.
 

@@ -71,6 +71,10 @@ class Model:
         c = self.cfg
         return np.zeros((c.n_layers, 2, c.n_kv_heads, c.n_pos + 2, c.head_dim))
 
+    def kv_store(self, v: np.ndarray) -> np.ndarray:
+        """Values as the KV cache keeps them (the MultiCodeDecoder's cache is exact)."""
+        return v
+
     # ---- one row --------------------------------------------------------------------
     def row(self, kv: np.ndarray, x_in: np.ndarray, pos: int) -> np.ndarray:
         """Run the row at sequence position `pos`; writes its K/V, returns post-norm h."""
@@ -89,8 +93,8 @@ class Model:
                 k = np.stack([rmsnorm(k[h], w[p + "k_norm"], c.rms_eps) for h in range(Hkv)])
             q = rope(q, pos, c.rope_base)
             k = rope(k, pos, c.rope_base)
-            kv[l, 0, :, pos] = k
-            kv[l, 1, :, pos] = v
+            kv[l, 0, :, pos] = self.kv_store(k)
+            kv[l, 1, :, pos] = self.kv_store(v)
             o = np.empty((Hq, D))
             for h in range(Hq):
                 g = h // group

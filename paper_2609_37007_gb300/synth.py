@@ -175,3 +175,108 @@ def random_logits(rng: np.random.Generator, rows: int, vocab: int, scale: float 
         m = rng.random((rows, vocab)) < tie_frac
         x[m] = np.round(x[m] * 4.0).astype(np.float32) / np.float32(4.0)
     return x
+
+
+# ---------------------------------------------------------------------------------------
+# Outer CodeDecoder (full frame pipeline, Fig. 1): one decoder call per 80 ms frame emits
+# the seed code c0; its hidden state and c0 start the MultiCodeDecoder's frame.
+# ---------------------------------------------------------------------------------------
+@dataclasses.dataclass(frozen=True)
+class OuterConfig:
+    """Shape and sampling configuration of the outer CodeDecoder of a frame pipeline."""
+    name: str
+    n_layers: int
+    hidden: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    ffn: int
+    c0_vocab: int         # rows of the c0 table and of the c0 head
+    text_vocab: int       # rows of the text-token table
+    rms_eps: float
+    rope_base: float
+    qk_norm: int
+    weight_dtype: int     # WEIGHT_F32 or WEIGHT_BF16; the KV cache is kept in this dtype
+    top_k: int
+    temperature: float
+    prompt_len: int       # text tokens prefilled before frame 0
+    frames: int           # frames of one utterance
+    weight_seed: int = 0
+    sample_seed: int = 1
+
+    @property
+    def max_tokens(self) -> int:
+        """KV positions one utterance fills: the prompt plus one row per frame after the first."""
+        return self.prompt_len + self.frames - 1
+
+    def replace(self, **kw) -> "OuterConfig":
+        return dataclasses.replace(self, **kw)
+
+
+# Tiny fp32 pipeline for brute-force checks (inner model: TINY, which takes the c0
+# embedding vector from the outer model).
+OUTER_TINY = OuterConfig(name="outer_tiny_fp32", n_layers=2, hidden=256, n_q_heads=4, n_kv_heads=2,
+                         head_dim=64, ffn=768, c0_vocab=96, text_vocab=512, rms_eps=1e-6,
+                         rope_base=10000.0, qk_norm=1, weight_dtype=WEIGHT_F32, top_k=8,
+                         temperature=1.0, prompt_len=12, frames=8)
+
+# CodeDecoder-shaped bf16 model: 28 layers, hidden 1024, 16q/8kv x 128, FFN 3072, c0 vocab
+# 3072, text vocab 151936, 256-token text prompt, 375 frames (30 s), top-k 50, T = 0.9.
+OUTER = OuterConfig(name="codedecoder_bf16", n_layers=28, hidden=1024, n_q_heads=16, n_kv_heads=8,
+                    head_dim=128, ffn=3072, c0_vocab=3072, text_vocab=151936, rms_eps=1e-6,
+                    rope_base=10000.0, qk_norm=1, weight_dtype=WEIGHT_BF16, top_k=50,
+                    temperature=0.9, prompt_len=256, frames=375)
+
+# The MultiCodeDecoder of the pipeline: config-2 shapes, c0 embedding supplied by the outer model.
+PIPE_INNER = MCD.replace(name="mcd_bf16_pipeline", c0_vocab=0)
+PIPELINES = {"tiny": (OUTER_TINY, TINY), "full": (OUTER, PIPE_INNER)}
+
+
+def outer_tensor_specs(cfg: OuterConfig, inner: MCDConfig) -> List[Tuple[str, Tuple[int, ...], str]]:
+    """Tensors of the outer model: its layers (same names as the inner model's), final norm,
+    c0 head and c0 table, the text table, and the table of the inner model's last code
+    c_{n_pos}, which only the outer model's input sum reads."""
+    H, D = cfg.hidden, cfg.head_dim
+    qd, kd = cfg.n_q_heads * D, cfg.n_kv_heads * D
+    specs: List[Tuple[str, Tuple[int, ...], str]] = []
+    for l in range(cfg.n_layers):
+        p = f"layers.{l}."
+        specs += [(p + "attn_norm", (H,), "gain"),
+                  (p + "wq", (qd, H), "mat"), (p + "wk", (kd, H), "mat"), (p + "wv", (kd, H), "mat")]
+        if cfg.qk_norm:
+            specs += [(p + "q_norm", (D,), "gain"), (p + "k_norm", (D,), "gain")]
+        specs += [(p + "wo", (H, qd), "mat"), (p + "ffn_norm", (H,), "gain"),
+                  (p + "wg", (cfg.ffn, H), "mat"), (p + "wu", (cfg.ffn, H), "mat"),
+                  (p + "wd", (H, cfg.ffn), "mat")]
+    specs += [("final_norm", (H,), "gain"), ("c0_head", (cfg.c0_vocab, H), "mat"),
+              ("c0_embed", (cfg.c0_vocab, H), "mat"), ("text_embed", (cfg.text_vocab, H), "mat"),
+              (f"code_embed.{inner.n_pos}", (inner.vocab, H), "mat")]
+    return specs
+
+
+def make_outer_weights(cfg: OuterConfig, inner: MCDConfig) -> Dict[str, np.ndarray]:
+    """Outer-model weights, drawn like make_weights but from streams (seed, 5, index) so
+    that they never repeat the inner model's."""
+    out: Dict[str, np.ndarray] = {}
+    for idx, (name, shape, kind) in enumerate(outer_tensor_specs(cfg, inner)):
+        rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([cfg.weight_seed, 5, idx])))
+        draw = rng.standard_normal(shape, dtype=np.float32)
+        if kind == "gain":
+            vals = (1.0 + 0.1 * draw.astype(np.float64)).astype(np.float32)
+        else:
+            vals = (0.02 * draw.astype(np.float64)).astype(np.float32)
+        out[name] = round_to_bf16_bits(vals) if cfg.weight_dtype == WEIGHT_BF16 else vals
+    return out
+
+
+def outer_weights_as_f32(cfg: OuterConfig, w: Dict[str, np.ndarray]) -> Dict[str, np.ndarray]:
+    if cfg.weight_dtype == WEIGHT_BF16:
+        return {k: bf16_bits_to_f32(v) for k, v in w.items()}
+    return dict(w)
+
+
+def make_prompt(cfg: OuterConfig, utterance: int = 0, seed: int | None = None) -> np.ndarray:
+    """Text-token ids of one utterance's prompt, uniform over [0, text_vocab)."""
+    s = cfg.weight_seed if seed is None else seed
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([s, 11, utterance])))
+    return rng.integers(0, cfg.text_vocab, size=cfg.prompt_len).astype(np.int32)
