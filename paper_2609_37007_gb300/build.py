@@ -12,13 +12,13 @@ CSRC = os.path.join(PKG, "csrc")
 ROOT = os.path.dirname(PKG)
 LIB = os.path.join(PKG, "libmcd.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu"]
+SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu", "mcd_outer.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-cudart", "shared",
          "-I" + os.path.join(ROOT, "include")]
 
 
-FRAME_KERNEL_SOURCES = ["mcd_frame.cu", "mcd_internal.cuh", "mcd_sampler.cuh"]
+FRAME_KERNEL_SOURCES = ["mcd_frame.cu", "mcd_stage.cuh", "mcd_internal.cuh", "mcd_sampler.cuh"]
 
 
 def source_digest(files=FRAME_KERNEL_SOURCES) -> str:
@@ -50,7 +50,7 @@ def _stale(out: str, deps) -> bool:
 def build(verbose: bool = False, force: bool = False, extra=()) -> str:
     os.makedirs(BUILD_DIR, exist_ok=True)
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
-    headers.append(os.path.join(ROOT, "include", "mcd.h"))
+    headers += [os.path.join(ROOT, "include", f) for f in ("mcd.h", "mcd_pipeline.h")]
     objs, jobs = [], []
     for src in SOURCES:
         s = os.path.join(CSRC, src)

@@ -12,6 +12,7 @@
 
 #include "mcd_internal.cuh"
 #include "mcd_sampler.cuh"
+#include "mcd_host.cuh"
 
 namespace mcd {
 cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream);
@@ -21,32 +22,6 @@ int frame_smem_bytes();
 // ------------------------------------------------------------------------------------
 // Auxiliary kernels
 // ------------------------------------------------------------------------------------
-struct RowSrc {
-  const uint8_t* seg[3];
-  int seg_rows[3];
-  int nseg;
-  int interleave_gu;  // 1: logical tile t = [gate rows 8t..8t+7 ; up rows 8t..8t+7]
-  int src_cols;       // elements per source row
-};
-
-// Logical element (r, c) -> offset (in elements) inside the tiled matrix.
-__host__ __device__ inline long long tiled_offset(const MatGeom& g, int r, int c, int wdtype) {
-  const int kc = c / (g.Ku * 16), kt = (c % (g.Ku * 16)) / 16;
-  const int mb = r / (g.Mu * 16), mi = (r % (g.Mu * 16)) / 16;
-  const long long u = (long long)kc * g.n_mb + mb;
-  const long long tile = (u * g.Mu + mi) * g.Ku + kt;
-  const int rr = r & 15, cc = c & 15;
-  int pos;
-  if (wdtype == MCD_WEIGHT_BF16) {
-    const int lane = (rr & 7) * 4 + ((cc & 7) >> 1);
-    const int reg = (rr >> 3) + 2 * (cc >> 3);
-    pos = lane * 8 + reg * 2 + (cc & 1);
-  } else {
-    pos = (rr + 16 * (cc >> 3)) * 8 + (cc & 7);
-  }
-  return tile * 256 + pos;
-}
-
 __global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst) {
   const long long total = (long long)g.M * g.K;
   const int es = wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
@@ -97,9 +72,9 @@ __global__ void head_bias_kernel(const uint8_t* head, const float* offsets, int 
   if (lane == 0) out[(size_t)j * V + id] = acc;
 }
 
-__global__ void rope_kernel(float2* rope, int D, double base) {
+__global__ void rope_kernel(float2* rope, int D, double base, int n_pos) {
   const int half = D / 2;
-  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < kMaxPos * half; idx += gridDim.x * blockDim.x) {
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < n_pos * half; idx += gridDim.x * blockDim.x) {
     const int pos = idx / half, i = idx % half;
     const double ang = (double)pos * pow(base, -2.0 * (double)i / (double)D);
     rope[idx] = make_float2((float)cos(ang), (float)sin(ang));
@@ -258,21 +233,15 @@ struct mcd_ctx {
   int h_err = 0;                 // host-side sticky CUDA error
 };
 
-static mcd_status cuda_status(cudaError_t e) {
+mcd_status mcd::cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return MCD_OK;
   if (e == cudaErrorMemoryAllocation) return MCD_ERR_OOM;
   return MCD_ERR_CUDA;
 }
 
-#define MCD_CHECK(call)                                 \
-  do {                                                  \
-    cudaError_t e__ = (call);                           \
-    if (e__ != cudaSuccess) {                           \
-      if (getenv("MCD_DEBUG"))                          \
-        fprintf(stderr, "mcd: %s failed: %s (%s:%d)\n", #call, cudaGetErrorString(e__), __FILE__, __LINE__); \
-      return cuda_status(e__);                          \
-    }                                                   \
-  } while (0)
+const FrameParams& mcd::ctx_params(const mcd_ctx* c) { return c->fp; }
+cudaStream_t mcd::ctx_stream(const mcd_ctx* c) { return c->stream; }
+bool mcd::ctx_weights_loaded(const mcd_ctx* c) { return c->weights_loaded; }
 
 template <class T>
 static cudaError_t ctx_alloc(mcd_ctx* c, T** p, size_t bytes) {
@@ -284,7 +253,7 @@ static cudaError_t ctx_alloc(mcd_ctx* c, T** p, size_t bytes) {
   return cudaSuccess;
 }
 
-static bool make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeom& g) {
+bool mcd::make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeom& g) {
   const int Gk = kConsumerWarps / Mu;
   if (M % (Mu * 16) || K % 16) return false;
   const int kt = K / 16;
@@ -306,6 +275,63 @@ static bool make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeo
   g.unit_bytes = Mu * Ku * tile_bytes;
   g.stride = (long long)g.n_units * g.unit_bytes;
   return true;
+}
+
+bool mcd::backbone_geom(FrameParams& p, int head_rows) {
+  const int tb = p.wdtype == MCD_WEIGHT_BF16 ? 512 : 1024;
+  bool ok = make_geom(p.qkv_dim, p.H, 1, tb, 1024, p.g[MAT_QKV]) && p.g[MAT_QKV].n_kc == 1;
+  int mu_o = 8;
+  while (mu_o > 1 && (mu_o * (p.D / 16) * tb > kSlotBytes || p.H % (mu_o * 16))) mu_o >>= 1;
+  ok = ok && make_geom(p.H, p.NH * p.D, mu_o, tb, p.D, p.g[MAT_WO]) && p.g[MAT_WO].Ku * 16 == p.D;
+  ok = ok && make_geom(2 * p.F, p.H, 1, tb, 1024, p.g[MAT_GU]) && p.g[MAT_GU].n_kc == 1;
+  ok = ok && make_geom(p.H, p.F, 1, tb, 1024, p.g[MAT_WD]);
+  ok = ok && make_geom(head_rows, p.H, 1, tb, 1024, p.g[MAT_HEAD]) && p.g[MAT_HEAD].n_kc == 1;
+  return ok;
+}
+
+void mcd::load_layer(const FrameParams& p, cudaStream_t stream, const LayerSrc& src, int l) {
+  const int H = p.H, D = p.D, F = p.F, qd = p.NH * D, kd = p.NKV * D;
+  auto tile = [&](RowSrc rs, const MatGeom& g, const uint8_t* dst) {
+    tile_kernel<<<1024, 256, 0, stream>>>(rs, g, p.wdtype, const_cast<uint8_t*>(dst));
+  };
+  auto conv = [&](const uint8_t* from, int64_t count, const float* dst) {
+    to_f32_kernel<<<64, 256, 0, stream>>>(from, p.wdtype, count, const_cast<float*>(dst));
+  };
+  RowSrc rs{};
+  rs.seg[0] = src.wq;
+  rs.seg[1] = src.wk;
+  rs.seg[2] = src.wv;
+  rs.seg_rows[0] = qd;
+  rs.seg_rows[1] = kd;
+  rs.seg_rows[2] = kd;
+  rs.nseg = 3;
+  rs.src_cols = H;
+  tile(rs, p.g[MAT_QKV], p.w_qkv + (size_t)l * p.g[MAT_QKV].stride);
+  RowSrc ro{};
+  ro.seg[0] = src.wo;
+  ro.seg_rows[0] = H;
+  ro.nseg = 1;
+  ro.src_cols = qd;
+  tile(ro, p.g[MAT_WO], p.w_wo + (size_t)l * p.g[MAT_WO].stride);
+  RowSrc rg{};
+  rg.seg[0] = src.wg;
+  rg.seg[1] = src.wu;
+  rg.nseg = 2;
+  rg.interleave_gu = 1;
+  rg.src_cols = H;
+  tile(rg, p.g[MAT_GU], p.w_gu + (size_t)l * p.g[MAT_GU].stride);
+  RowSrc rd{};
+  rd.seg[0] = src.wd;
+  rd.seg_rows[0] = H;
+  rd.nseg = 1;
+  rd.src_cols = F;
+  tile(rd, p.g[MAT_WD], p.w_wd + (size_t)l * p.g[MAT_WD].stride);
+  conv(src.attn_norm, H, p.attn_norm + (size_t)l * H);
+  conv(src.ffn_norm, H, p.ffn_norm + (size_t)l * H);
+  if (p.qk_norm) {
+    conv(src.q_norm, D, p.q_norm + (size_t)l * D);
+    conv(src.k_norm, D, p.k_norm + (size_t)l * D);
+  }
 }
 
 static mcd_status validate_config(const mcd_config& c) {
@@ -405,15 +431,8 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   const char* wn = getenv("MCD_WAIT_NS");
   if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
 
-  const int tb = k.weight_dtype == MCD_WEIGHT_BF16 ? 512 : 1024;
   const int es = k.weight_dtype == MCD_WEIGHT_BF16 ? 2 : 4;
-  bool ok = make_geom(p.qkv_dim, p.H, 1, tb, 1024, p.g[MAT_QKV]) && p.g[MAT_QKV].n_kc == 1;
-  int mu_o = 8;
-  while (mu_o > 1 && (mu_o * (p.D / 16) * tb > kSlotBytes || p.H % (mu_o * 16))) mu_o >>= 1;
-  ok = ok && make_geom(p.H, p.NH * p.D, mu_o, tb, p.D, p.g[MAT_WO]) && p.g[MAT_WO].Ku * 16 == p.D;
-  ok = ok && make_geom(2 * p.F, p.H, 1, tb, 1024, p.g[MAT_GU]) && p.g[MAT_GU].n_kc == 1;
-  ok = ok && make_geom(p.H, p.F, 1, tb, 1024, p.g[MAT_WD]);
-  ok = ok && make_geom(p.V, p.H, 1, tb, 1024, p.g[MAT_HEAD]) && p.g[MAT_HEAD].n_kc == 1;
+  const bool ok = backbone_geom(p, p.V);
   if (!ok) return fail(MCD_ERR_UNSUPPORTED);
   p.ctr_stride = ctr_count(p.L);
 
@@ -474,7 +493,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.vcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.st, 0, sizeof(DevState) * k.max_streams, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
-  rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base);
+  rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base, kMaxPos);
   if (cudaGetLastError() != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   *out = c;
@@ -566,41 +585,10 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
   };
   for (int l = 0; l < p.L; ++l) {
     const std::string pre = "layers." + std::to_string(l) + ".";
-    RowSrc rs{};
-    rs.seg[0] = S(pre + "wq");
-    rs.seg[1] = S(pre + "wk");
-    rs.seg[2] = S(pre + "wv");
-    rs.seg_rows[0] = (int)qd;
-    rs.seg_rows[1] = (int)kd;
-    rs.seg_rows[2] = (int)kd;
-    rs.nseg = 3;
-    rs.src_cols = (int)H;
-    tile(rs, p.g[MAT_QKV], c->w_arena + c->off_qkv + (size_t)l * p.g[MAT_QKV].stride);
-    RowSrc ro{};
-    ro.seg[0] = S(pre + "wo");
-    ro.seg_rows[0] = (int)H;
-    ro.nseg = 1;
-    ro.src_cols = (int)qd;
-    tile(ro, p.g[MAT_WO], c->w_arena + c->off_wo + (size_t)l * p.g[MAT_WO].stride);
-    RowSrc rg{};
-    rg.seg[0] = S(pre + "wg");
-    rg.seg[1] = S(pre + "wu");
-    rg.nseg = 2;
-    rg.interleave_gu = 1;
-    rg.src_cols = (int)H;
-    tile(rg, p.g[MAT_GU], c->w_arena + c->off_gu + (size_t)l * p.g[MAT_GU].stride);
-    RowSrc rd{};
-    rd.seg[0] = S(pre + "wd");
-    rd.seg_rows[0] = (int)H;
-    rd.nseg = 1;
-    rd.src_cols = (int)F;
-    tile(rd, p.g[MAT_WD], c->w_arena + c->off_wd + (size_t)l * p.g[MAT_WD].stride);
-    conv(pre + "attn_norm", H, p.attn_norm + (size_t)l * H);
-    conv(pre + "ffn_norm", H, p.ffn_norm + (size_t)l * H);
-    if (p.qk_norm) {
-      conv(pre + "q_norm", D, p.q_norm + (size_t)l * D);
-      conv(pre + "k_norm", D, p.k_norm + (size_t)l * D);
-    }
+    LayerSrc ls{S(pre + "wq"), S(pre + "wk"), S(pre + "wv"), S(pre + "wo"), S(pre + "wg"), S(pre + "wu"),
+                S(pre + "wd"), S(pre + "attn_norm"), S(pre + "ffn_norm"),
+                p.qk_norm ? S(pre + "q_norm") : nullptr, p.qk_norm ? S(pre + "k_norm") : nullptr};
+    load_layer(p, c->stream, ls, l);
   }
   conv("final_norm", H, p.final_norm);
   for (int j = 1; j <= Kd; ++j) conv("offset." + std::to_string(j), H, p.offsets + (size_t)(j - 1) * H);

@@ -13,7 +13,7 @@ from typing import Dict, Optional
 
 import numpy as np
 
-from .synth import MCDConfig
+from .synth import MCDConfig, OuterConfig
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmcd.so")
 _lib: Optional[ctypes.CDLL] = None
@@ -37,6 +37,17 @@ class McdConfig(ctypes.Structure):
                 ("draft_len", ctypes.c_int32), ("top_k", ctypes.c_int32),
                 ("temperature", ctypes.c_float), ("draft_mode", ctypes.c_int32),
                 ("noise_sigma", ctypes.c_float), ("seed", ctypes.c_uint64), ("max_streams", ctypes.c_int32)]
+
+
+class McdOuterConfig(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("hidden", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32),
+                ("c0_vocab", ctypes.c_int32), ("text_vocab", ctypes.c_int32),
+                ("max_tokens", ctypes.c_int32), ("rms_eps", ctypes.c_float),
+                ("rope_base", ctypes.c_float), ("qk_norm", ctypes.c_int32),
+                ("weight_dtype", ctypes.c_int32), ("top_k", ctypes.c_int32),
+                ("temperature", ctypes.c_float), ("seed", ctypes.c_uint64)]
 
 
 CALL_TRACE_DTYPE = np.dtype([("a", "<i4"), ("n_rows", "<i4"), ("pos0", "<i4"), ("n_drafts", "<i4"),
@@ -86,6 +97,19 @@ def load_library() -> ctypes.CDLL:
         "mcd_num_ctas": (I32, [P]),
         "mcd_destroy": (None, [P]),
         "mcd_status_str": (ctypes.c_char_p, [I32]),
+        "mcd_outer_create": (I32, [ctypes.POINTER(McdOuterConfig), P, ctypes.POINTER(P)]),
+        "mcd_outer_destroy": (None, [P]),
+        "mcd_outer_load_weights": (I32, [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(P),
+                                         ctypes.POINTER(I64)]),
+        "mcd_outer_prefill": (I32, [P, U32, I32, P]),
+        "mcd_outer_step": (I32, [P, P, I32]),
+        "mcd_outer_frame_inputs": (I32, [P, ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(P),
+                                         ctypes.POINTER(U32)]),
+        "mcd_pipeline_frames": (I32, [P, I32, P, P, P]),
+        "mcd_outer_trace_floats": (I64, [P]),
+        "mcd_outer_set_trace": (I32, [P, P, I32]),
+        "mcd_outer_sync": (I32, [P]),
+        "mcd_outer_step_weight_bytes": (I64, [P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -138,15 +162,19 @@ def mcd_create(cfg: MCDConfig, stream=None) -> ctypes.c_void_p:
     return out
 
 
-def mcd_load_weights(ctx, weights: Dict[str, np.ndarray]):
-    lib = load_library()
+def _weight_args(weights: Dict[str, np.ndarray]):
     names = list(weights)
     arrs = [np.ascontiguousarray(weights[k]) for k in names]
     n = len(names)
     c_names = (ctypes.c_char_p * n)(*[k.encode() for k in names])
     c_ptrs = (ctypes.c_void_p * n)(*[a.ctypes.data for a in arrs])
     c_sz = (ctypes.c_int64 * n)(*[a.nbytes for a in arrs])
-    _check("mcd_load_weights", lib.mcd_load_weights(ctx, n, c_names, c_ptrs, c_sz))
+    return n, c_names, c_ptrs, c_sz, arrs
+
+
+def mcd_load_weights(ctx, weights: Dict[str, np.ndarray]):
+    n, c_names, c_ptrs, c_sz, _keep = _weight_args(weights)
+    _check("mcd_load_weights", load_library().mcd_load_weights(ctx, n, c_names, c_ptrs, c_sz))
 
 
 def mcd_decode_frame(ctx, stream_id: int, frame_idx: int, cond, c0, c0_emb, codes_out, stats=None):
@@ -260,6 +288,96 @@ class Decoder:
         if self.ctx:
             mcd_destroy(self.ctx)
             self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# ---- outer CodeDecoder and the frame pipeline (include/mcd_pipeline.h) ------------------
+def outer_config_struct(cfg: OuterConfig) -> McdOuterConfig:
+    return McdOuterConfig(cfg.n_layers, cfg.hidden, cfg.n_q_heads, cfg.n_kv_heads, cfg.head_dim, cfg.ffn,
+                          cfg.c0_vocab, cfg.text_vocab, cfg.max_tokens, cfg.rms_eps, cfg.rope_base,
+                          cfg.qk_norm, cfg.weight_dtype, cfg.top_k, cfg.temperature, cfg.sample_seed)
+
+
+def mcd_outer_create(cfg: OuterConfig, inner_ctx) -> ctypes.c_void_p:
+    c = outer_config_struct(cfg)
+    out = ctypes.c_void_p()
+    _check("mcd_outer_create", load_library().mcd_outer_create(ctypes.byref(c), inner_ctx, ctypes.byref(out)))
+    return out
+
+
+def mcd_outer_destroy(o):
+    load_library().mcd_outer_destroy(o)
+
+
+def mcd_outer_load_weights(o, weights: Dict[str, np.ndarray]):
+    n, c_names, c_ptrs, c_sz, _keep = _weight_args(weights)
+    _check("mcd_outer_load_weights", load_library().mcd_outer_load_weights(o, n, c_names, c_ptrs, c_sz))
+
+
+def mcd_outer_prefill(o, stream_id: int, text_ids):
+    _check("mcd_outer_prefill", load_library().mcd_outer_prefill(o, stream_id, int(text_ids.numel()),
+                                                                  _ptr(text_ids)))
+
+
+def mcd_outer_step(o, prev_codes, text_id: int = -1):
+    _check("mcd_outer_step", load_library().mcd_outer_step(o, _ptr(prev_codes), int(text_id)))
+
+
+def mcd_outer_frame_inputs(o):
+    """Device addresses (cond, c0_emb, c0) and the frame index of the current frame."""
+    cond, emb, c0 = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+    fi = ctypes.c_uint32()
+    _check("mcd_outer_frame_inputs", load_library().mcd_outer_frame_inputs(
+        o, ctypes.byref(cond), ctypes.byref(emb), ctypes.byref(c0), ctypes.byref(fi)))
+    return cond.value, emb.value, c0.value, fi.value
+
+
+def mcd_pipeline_frames(o, n_frames: int, codes_out, text_ids=None, stats=None):
+    tid = None
+    if text_ids is not None:
+        tid = (ctypes.c_int32 * n_frames)(*[int(v) for v in text_ids])
+    _check("mcd_pipeline_frames", load_library().mcd_pipeline_frames(o, n_frames, tid, _ptr(codes_out),
+                                                                      _ptr(stats)))
+
+
+def mcd_outer_trace_floats(o) -> int:
+    return int(load_library().mcd_outer_trace_floats(o))
+
+
+def mcd_outer_set_trace(o, trace, n_frames: int):
+    _check("mcd_outer_set_trace", load_library().mcd_outer_set_trace(o, _ptr(trace), n_frames))
+
+
+def mcd_outer_sync(o):
+    _check("mcd_outer_sync", load_library().mcd_outer_sync(o))
+
+
+def mcd_outer_step_weight_bytes(o) -> int:
+    return int(load_library().mcd_outer_step_weight_bytes(o))
+
+
+class Pipeline:
+    """An inner Decoder plus the outer CodeDecoder on top of it (one utterance at a time)."""
+
+    def __init__(self, outer_cfg: OuterConfig, inner_cfg: MCDConfig,
+                 outer_weights: Optional[Dict[str, np.ndarray]] = None,
+                 inner_weights: Optional[Dict[str, np.ndarray]] = None, stream=None):
+        self.inner = Decoder(inner_cfg, inner_weights, stream)
+        self.cfg = outer_cfg
+        self.o = mcd_outer_create(outer_cfg, self.inner.ctx)
+        if outer_weights is not None:
+            mcd_outer_load_weights(self.o, outer_weights)
+
+    def close(self):
+        if self.o:
+            mcd_outer_destroy(self.o)
+            self.o = None
+        self.inner.close()
 
     def __del__(self):
         try:

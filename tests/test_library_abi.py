@@ -1,5 +1,6 @@
 """CPU-side checks of the C ABI: the library builds, loads, exports every function that
-include/mcd.h declares, and its structs have the layout the binding assumes.  No GPU."""
+include/*.h declares, and its structs have the layout the binding assumes.  No GPU."""
+import glob
 import ctypes
 import os
 import re
@@ -9,7 +10,7 @@ import pytest
 
 from conftest import ROOT
 
-HEADER = os.path.join(ROOT, "include", "mcd.h")
+HEADERS = sorted(glob.glob(os.path.join(ROOT, "include", "*.h")))
 
 
 @pytest.fixture(scope="module")
@@ -20,15 +21,18 @@ def lib():
 
 
 def declared_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(mcd_[a-z_0-9]+)\s*\(", text)))
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(mcd_[a-z_0-9]+)\s*\(", text))
+    return sorted(names)
 
 
 def test_header_declares_the_boundary():
     fns = declared_functions()
     for need in ("mcd_create", "mcd_load_weights", "mcd_draft", "mcd_verify_accept", "mcd_decode_frame",
-                 "mcd_accept_from_logits", "mcd_destroy", "mcd_status_str"):
+                 "mcd_accept_from_logits", "mcd_destroy", "mcd_status_str", "mcd_outer_create",
+                 "mcd_outer_prefill", "mcd_pipeline_frames"):
         assert need in fns
 
 
@@ -40,13 +44,17 @@ def test_every_declared_symbol_is_exported(lib):
 def test_struct_layouts_match_the_binding(tmp_path):
     from paper_2609_37007_gb300 import mcd
     src = tmp_path / "sz.c"
-    src.write_text('#include "mcd.h"\n#include <stdio.h>\n#include <stddef.h>\nint main(void){printf("%zu %zu %zu %zu",'
+    src.write_text('#include "mcd_pipeline.h"\n#include <stdio.h>\n#include <stddef.h>\n'
+                   'int main(void){printf("%zu %zu %zu %zu %zu %zu",'
                    ' sizeof(mcd_config), sizeof(mcd_call_trace), sizeof(mcd_frame_stats),'
-                   ' offsetof(mcd_config, seed));return 0;}\n')
+                   ' offsetof(mcd_config, seed), sizeof(mcd_outer_config), offsetof(mcd_outer_config, seed));'
+                   'return 0;}\n')
     exe = tmp_path / "sz"
     subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
-    cfg_sz, trace_sz, stats_sz, seed_off = map(int, out)
+    cfg_sz, trace_sz, stats_sz, seed_off, ocfg_sz, oseed_off = map(int, out)
+    assert ocfg_sz == ctypes.sizeof(mcd.McdOuterConfig)
+    assert oseed_off == mcd.McdOuterConfig.seed.offset
     assert cfg_sz == ctypes.sizeof(mcd.McdConfig)
     assert seed_off == mcd.McdConfig.seed.offset
     assert trace_sz == mcd.CALL_TRACE_DTYPE.itemsize
