@@ -290,6 +290,172 @@ def run_streams(args, weights):
         dec.close()
 
 
+PIPE_METRIC = "sustained frames/s of the full frame pipeline"
+PIPE_UNIT = "frames/s"
+PIPE_WORKLOAD = ("CodeDecoder bf16, 28 layers, hidden 1024, 16q/8kv x 128, SwiGLU 3072, c0 vocab 3072, text vocab "
+                 "151936, 256-token prompt, 375 frames (30 s of audio), c0 top-k 50 T 0.9; each frame feeds the "
+                 "MultiCodeDecoder bf16 workload (K=3 drafts, top-k 50, T 0.9); single stream")
+REALTIME_FPS = 12.5       # one frame per 80 ms
+
+
+def outer_step_bytes(ocfg, weights: int, pos: int) -> int:
+    """Bytes one CodeDecoder row at position pos must move: its weights (backbone and c0
+    head) once, the bf16 K/V of the pos cached positions read and its own row written, and
+    the 16 code-embedding rows of its input plus the c0 embedding row it hands on."""
+    kv_row = ocfg.n_layers * 2 * ocfg.n_kv_heads * ocfg.head_dim * 2
+    return weights + (pos + 1) * kv_row + 17 * ocfg.hidden * 2
+
+
+def cpu_pipeline_baseline(ocfg, icfg, ow, iw, budget_s: float):
+    """The oracle as it stands: the prompt prefill, then whole frames until budget_s."""
+    from paper_2609_37007_gb300.synth import make_prompt, outer_weights_as_f32, weights_as_f32
+    from oracle.codedecoder import CodeDecoder, Pipeline
+    from oracle.model import Model
+    oc = CodeDecoder(ocfg, outer_weights_as_f32(ocfg, ow), Model(icfg, weights_as_f32(icfg, iw)))
+    pl = Pipeline(oc)
+    t0 = time.perf_counter()
+    pl.prefill(make_prompt(ocfg))
+    t_pre = time.perf_counter() - t0
+    frames, prev = 0, None
+    t1 = time.perf_counter()
+    while frames < 2 or time.perf_counter() - t0 < budget_s:
+        prev = pl.run_frame(prev_codes=prev).codes
+        frames += 1
+    dt = time.perf_counter() - t1
+    return {"value": frames / dt, "unit": PIPE_UNIT, "cores": blas_threads(), "kind": "oracle",
+            "sample": f"the 256-token prompt prefill ({t_pre:.1f} s, not in the value) and the first {frames} "
+                      f"frames of the utterance in {dt:.1f} s, fp64 numpy oracle"}
+
+
+def run_pipeline(args):
+    """Full frame pipeline (CodeDecoder + speculative MultiCodeDecoder): one JSON line with
+    sustained frames/s over whole utterances, the per-frame split between the two kernels,
+    the real-time factor against 12.5 frames/s, and both kernels' rooflines."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    from paper_2609_37007_gb300.synth import OUTER, PIPE_INNER, make_outer_weights, make_prompt, make_weights
+    _build.build()
+    ocfg, icfg = OUTER, PIPE_INNER
+    iw, ow = make_weights(icfg), make_outer_weights(ocfg, icfg)
+    cpu = None if args.no_cpu else cpu_pipeline_baseline(ocfg, icfg, ow, iw, args.cpu_budget)
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    pl = mcd.Pipeline(ocfg, icfg, ow, iw, stream)
+    o, ictx = pl.o, pl.inner.ctx
+    F, W = ocfg.frames, icfg.n_pos + 1
+    prompt_h = make_prompt(ocfg)
+    prompt = torch.from_numpy(prompt_h).to(dev)
+    U = max(1, args.utterances)
+    codes = torch.zeros((U, F, W), dtype=torch.int32, device=dev)
+    stats = torch.zeros((U, F, 8), dtype=torch.int32, device=dev)
+    for _ in range(max(1, args.warmup // 3)):                      # warm-up utterances
+        mcd.mcd_outer_prefill(o, 0, prompt)
+        mcd.mcd_pipeline_frames(o, F, codes[0], stats=stats[0])
+    mcd.mcd_outer_sync(o)
+    mcd.mcd_sync(ictx)
+
+    # ---- timed: U whole utterances through mcd_pipeline_frames ---------------------------
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * U + 1)]
+    clocks = Clocks(0)
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    ev[0].record(stream)
+    for u in range(U):
+        mcd.mcd_outer_prefill(o, u, prompt)
+        ev[2 * u + 1].record(stream)
+        mcd.mcd_pipeline_frames(o, F, codes[u], stats=stats[u])
+        ev[2 * u + 2].record(stream)
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    mcd.mcd_outer_sync(o)
+    mcd.mcd_sync(ictx)
+    t_pre = sum(ev[2 * u].elapsed_time(ev[2 * u + 1]) for u in range(U)) / 1e3
+    t_frames = sum(ev[2 * u + 1].elapsed_time(ev[2 * u + 2]) for u in range(U)) / 1e3
+    st = stats.cpu().numpy().reshape(U * F, 8)
+    assert (st[:, 4] == 0).all() and (st[:, 1] == icfg.n_pos).all(), "device-side failure"
+
+    # ---- split per frame: outer row and inner frame timed apart (same launches) --------------
+    lib = mcd.load_library()
+    cb = torch.zeros((F, W), dtype=torch.int32, device=dev)
+    sb = torch.zeros((F, 8), dtype=torch.int32, device=dev)
+    eo = [torch.cuda.Event(enable_timing=True) for _ in range(3 * F)]
+    mcd.mcd_outer_prefill(o, 7, prompt, cb[0, 0:1])          # frame 0's c0 comes from the prompt
+    for f in range(F):
+        eo[3 * f].record(stream)
+        if f > 0:
+            mcd.mcd_outer_step(o, cb[f - 1], -1, cb[f, 0:1])
+        eo[3 * f + 1].record(stream)
+        cond_p, emb_p, _, fi = mcd.mcd_outer_frame_inputs(o)
+        mcd._check("mcd_decode_frame", lib.mcd_decode_frame(ictx, 7, fi, cond_p, None, emb_p,
+                                                            cb[f, 1:].data_ptr(), sb[f].data_ptr()))
+        eo[3 * f + 2].record(stream)
+    torch.cuda.synchronize(dev)
+    mcd.mcd_outer_sync(o)
+    t_outer = [eo[3 * f].elapsed_time(eo[3 * f + 1]) * 1e3 for f in range(1, F)]      # us
+    t_inner = [eo[3 * f + 1].elapsed_time(eo[3 * f + 2]) * 1e3 for f in range(F)]
+    s_split = sb.cpu().numpy()
+    w_outer = mcd.mcd_outer_step_weight_bytes(o)
+    pos = [ocfg.prompt_len - 1 + f for f in range(1, F)]
+    b_outer = [outer_step_bytes(ocfg, w_outer, q) for q in pos]
+    peak, peak_kind = read_peaks()
+    ach_outer = statistics.mean(b_outer) / (statistics.mean(t_outer) / 1e6) / 1e9
+    backbone = mcd.mcd_call_weight_bytes(ictx, 0)
+    head = mcd.mcd_call_weight_bytes(ictx, 1) - backbone
+    b_inner = algorithmic_bytes(icfg, s_split, backbone, head) / F
+    ach_inner = b_inner / (statistics.mean(t_inner) / 1e6) / 1e9
+
+    # ---- end to end through the C ABI: prompt ids from pinned host memory, each frame's
+    # codes read back to pinned host memory as soon as it is done (streaming) -------------------
+    prompt_pin = torch.from_numpy(prompt_h).pin_memory()
+    host_codes = torch.zeros((F, W), dtype=torch.int32).pin_memory()
+    dprompt = torch.zeros_like(prompt)
+    dcodes = torch.zeros((F, W), dtype=torch.int32, device=dev)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    dprompt.copy_(prompt_pin, non_blocking=True)
+    mcd.mcd_outer_prefill(o, 9, dprompt)
+    for f in range(F):
+        mcd.mcd_pipeline_frames(o, 1, dcodes[f])
+        host_codes[f].copy_(dcodes[f], non_blocking=True)
+        stream.synchronize()
+    t_e2e = time.perf_counter() - t0
+    mcd.mcd_outer_sync(o)
+    assert (host_codes.numpy() >= 0).all()
+
+    frames_all = U * F
+    prefill_launches = -(-ocfg.prompt_len // 16)
+    line = {
+        "metric": PIPE_METRIC, "value": frames_all / t_frames, "unit": PIPE_UNIT, "n_gpus": 1,
+        "steps": frames_all, "warmup": max(1, args.warmup // 3) * F, "ms_per_step": 1e3 * t_frames / frames_all,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": PIPE_WORKLOAD, "utterances": U, "step": "one frame (c0..c15)",
+                   "l2": "inputs larger than L2: 887 MB of CodeDecoder weights per frame"},
+        "realtime_factor": frames_all / t_frames / REALTIME_FPS,
+        "frames_per_s_with_prefill": frames_all / (t_frames + t_pre),
+        "prefill_ms": 1e3 * t_pre / U,
+        "per_frame_us": {"outer_row": statistics.mean(t_outer), "inner_frame": statistics.mean(t_inner),
+                         "inner_calls_per_frame": float(s_split[:, 0].mean())},
+        "tokens_per_s": float(st[:, 1].sum() + frames_all) / t_frames,
+        "roofline": {"bound": "hbm", "achieved": ach_inner, "peak": peak, "unit": "GB/s", "frac": ach_inner / peak,
+                     "traffic": None, "peak_kind": peak_kind, "kernel": "frame_kernel<bf16> (inner frame)",
+                     "bytes_per_launch": b_inner, "launch_us": statistics.mean(t_inner)},
+        "roofline_outer": {"bound": "hbm", "achieved": ach_outer, "peak": peak, "unit": "GB/s",
+                           "frac": ach_outer / peak, "traffic": None, "peak_kind": peak_kind,
+                           "kernel": "outer_kernel<bf16> (one CodeDecoder row)",
+                           "bytes_per_launch": statistics.mean(b_outer), "launch_us": statistics.mean(t_outer)},
+        "cpu_baseline": cpu,
+        "e2e": {"value": F / t_e2e, "unit": PIPE_UNIT, "h2d_bytes_per_step": ocfg.prompt_len * 4 / F,
+                "d2h_bytes_per_step": W * 4, "api": "mcd_outer_prefill + mcd_pipeline_frames per frame, codes "
+                                                   "read back to the host after every frame (host clock)"},
+        "gpu_launches": U * (2 * prefill_launches + 4 * (F - 1) + 2),
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    pl.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -306,6 +472,9 @@ def main():
     ap.add_argument("--streams", type=int, nargs="*", default=None,
                     help="batched-stream runs for these B instead of the bench line (e.g. --streams 1 2 4 8)")
     ap.add_argument("--stream-launches", type=int, default=100)
+    ap.add_argument("--pipeline", action="store_true",
+                    help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
+    ap.add_argument("--utterances", type=int, default=2)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -316,6 +485,8 @@ def main():
         return run_reference(args, cfg, weights)
     if args.streams:
         return run_streams(args, weights)
+    if args.pipeline:
+        return run_pipeline(args)
     if args.sweep:
         # one weight set with offsets b_1..b_7 serves every K (extra tensors are ignored)
         return run_sweep(args, make_weights(cfg.replace(draft_len=7)))

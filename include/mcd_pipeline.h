@@ -76,16 +76,19 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
 
 /* Start an utterance of stream `stream_id`: reset the KV cache and run the prompt rows
  * text_ids[0..n_tokens) (device int32) at positions 0..n_tokens-1, up to 16 rows per
- * launch; the last row gives frame 0's c0 and inner inputs.  Errors: MCD_ERR_INVALID_ARG,
- * MCD_ERR_STATE (weights not loaded), MCD_ERR_UNSUPPORTED (n_tokens > max_tokens); an id
- * outside the text table is reported by mcd_outer_sync as MCD_ERR_INVALID_ARG. */
-mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens, const int32_t* text_ids);
+ * launch; the last row gives frame 0's c0 and inner inputs (c0_out, device int32,
+ * optional, also receives c0).  Errors: MCD_ERR_INVALID_ARG, MCD_ERR_STATE (weights not
+ * loaded), MCD_ERR_UNSUPPORTED (n_tokens > max_tokens); an id outside the text table is
+ * reported by mcd_outer_sync as MCD_ERR_INVALID_ARG. */
+mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens, const int32_t* text_ids,
+                             int32_t* c0_out);
 
 /* One CodeDecoder row for the next frame: input = the sum above over prev_codes (device
  * int32 [n_pos + 1]: c0..c_P of the previous frame) and text row text_id (-1: none).
- * Produces the frame's c0 and inner inputs (mcd_outer_frame_inputs).  MCD_ERR_STATE
- * before a prefill or when the KV cache is full. */
-mcd_status mcd_outer_step(mcd_outer* o, const int32_t* prev_codes, int32_t text_id);
+ * Produces the frame's c0 and inner inputs (mcd_outer_frame_inputs); c0_out (device
+ * int32, optional) also receives c0.  MCD_ERR_STATE before a prefill or when the KV cache
+ * is full. */
+mcd_status mcd_outer_step(mcd_outer* o, const int32_t* prev_codes, int32_t text_id, int32_t* c0_out);
 
 /* Device pointers to the current frame's inner inputs (cond [H] fp32, c0 embedding [H]
  * fp32, c0 [1] int32) and its frame index; valid until the next prefill / step. */

@@ -905,7 +905,8 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
   return s;
 }
 
-mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens, const int32_t* text_ids) {
+mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens, const int32_t* text_ids,
+                             int32_t* c0_out) {
   if (!o || !text_ids || n_tokens < 1) return MCD_ERR_INVALID_ARG;
   if (!o->weights_loaded) return MCD_ERR_STATE;
   if (n_tokens > o->st.cap) return MCD_ERR_UNSUPPORTED;
@@ -920,7 +921,7 @@ mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens,
     s.text_ids = text_ids + s0;
     s.prev_codes = nullptr;
     s.text_id = -1;
-    s.c0_out2 = nullptr;
+    s.c0_out2 = s.head ? c0_out : nullptr;
     s.frame_id = 0;
     s.trace = (o->trace && o->trace_frames > 0) ? o->trace : nullptr;
     mcd_status r = outer_launch(o, s);
@@ -932,10 +933,10 @@ mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens,
   return MCD_OK;
 }
 
-mcd_status mcd_outer_step(mcd_outer* o, const int32_t* prev_codes, int32_t text_id) {
+mcd_status mcd_outer_step(mcd_outer* o, const int32_t* prev_codes, int32_t text_id, int32_t* c0_out) {
   if (!o) return MCD_ERR_INVALID_ARG;
   if (!o->weights_loaded) return MCD_ERR_STATE;
-  return outer_step_launch(o, prev_codes, text_id, nullptr);
+  return outer_step_launch(o, prev_codes, text_id, c0_out);
 }
 
 mcd_status mcd_outer_frame_inputs(const mcd_outer* o, const float** cond, const float** c0_emb, const int32_t** c0,

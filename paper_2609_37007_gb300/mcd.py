@@ -101,8 +101,8 @@ def load_library() -> ctypes.CDLL:
         "mcd_outer_destroy": (None, [P]),
         "mcd_outer_load_weights": (I32, [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(P),
                                          ctypes.POINTER(I64)]),
-        "mcd_outer_prefill": (I32, [P, U32, I32, P]),
-        "mcd_outer_step": (I32, [P, P, I32]),
+        "mcd_outer_prefill": (I32, [P, U32, I32, P, P]),
+        "mcd_outer_step": (I32, [P, P, I32, P]),
         "mcd_outer_frame_inputs": (I32, [P, ctypes.POINTER(P), ctypes.POINTER(P), ctypes.POINTER(P),
                                          ctypes.POINTER(U32)]),
         "mcd_pipeline_frames": (I32, [P, I32, P, P, P]),
@@ -319,13 +319,13 @@ def mcd_outer_load_weights(o, weights: Dict[str, np.ndarray]):
     _check("mcd_outer_load_weights", load_library().mcd_outer_load_weights(o, n, c_names, c_ptrs, c_sz))
 
 
-def mcd_outer_prefill(o, stream_id: int, text_ids):
+def mcd_outer_prefill(o, stream_id: int, text_ids, c0_out=None):
     _check("mcd_outer_prefill", load_library().mcd_outer_prefill(o, stream_id, int(text_ids.numel()),
-                                                                  _ptr(text_ids)))
+                                                                  _ptr(text_ids), _ptr(c0_out)))
 
 
-def mcd_outer_step(o, prev_codes, text_id: int = -1):
-    _check("mcd_outer_step", load_library().mcd_outer_step(o, _ptr(prev_codes), int(text_id)))
+def mcd_outer_step(o, prev_codes, text_id: int = -1, c0_out=None):
+    _check("mcd_outer_step", load_library().mcd_outer_step(o, _ptr(prev_codes), int(text_id), _ptr(c0_out)))
 
 
 def mcd_outer_frame_inputs(o):

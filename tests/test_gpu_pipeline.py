@@ -125,6 +125,30 @@ def test_tiny_pipeline_repeatable_and_restartable(tiny_pipe):
     assert [list(x[0]) for x in a] == [list(x[0]) for x in b]
 
 
+def test_stepwise_outer_api_matches_pipeline_call(tiny_pipe):
+    """mcd_outer_prefill / mcd_outer_step + mcd_outer_frame_inputs + mcd_decode_frame, driven
+    by the caller, give the codes mcd_pipeline_frames gives."""
+    env = tiny_pipe
+    o, ictx = env.pl.o, env.pl.inner.ctx
+    W, n = TINY.n_pos + 1, 5
+    prompt = torch.from_numpy(make_prompt(env.ocfg, utterance=2)).to(DEV)
+    ref = torch.full((n, W), -1, dtype=torch.int32, device=DEV)
+    mcd.mcd_outer_prefill(o, 4, prompt)
+    mcd.mcd_pipeline_frames(o, n, ref)
+    got = torch.full((n, W), -1, dtype=torch.int32, device=DEV)
+    lib = mcd.load_library()
+    mcd.mcd_outer_prefill(o, 4, prompt, got[0, 0:1])
+    for f in range(n):
+        if f > 0:
+            mcd.mcd_outer_step(o, got[f - 1], -1, got[f, 0:1])
+        cond, emb, _, fi = mcd.mcd_outer_frame_inputs(o)
+        assert fi == f
+        mcd._check("mcd_decode_frame", lib.mcd_decode_frame(ictx, 4, fi, cond, None, emb, got[f, 1:].data_ptr(), None))
+    mcd.mcd_outer_sync(o)
+    mcd.mcd_sync(ictx)
+    assert torch.equal(got, ref)
+
+
 @pytest.mark.parametrize("variant", ["mha", "one_row_prompt", "ar_inner", "text_rows", "bf16"])
 def test_tiny_pipeline_variants(variant):
     ocfg, icfg = OUTER_TINY, TINY
