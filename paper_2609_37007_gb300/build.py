@@ -12,7 +12,7 @@ CSRC = os.path.join(PKG, "csrc")
 ROOT = os.path.dirname(PKG)
 LIB = os.path.join(PKG, "libmcd.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu", "mcd_outer.cu"]
+SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu", "mcd_outer.cu", "mcd_batch.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-cudart", "shared",
          "-I" + os.path.join(ROOT, "include")]

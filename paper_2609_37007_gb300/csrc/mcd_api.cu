@@ -83,28 +83,7 @@ __global__ void rope_kernel(float2* rope, int D, double base, int n_pos) {
 
 __global__ void begin_frame_kernel(DevState* sts, unsigned* ctr, int n_ctr, const int* c0, int C0V, int S) {
   for (int i = threadIdx.x; i < n_ctr; i += blockDim.x) ctr[i] = 0u;
-  if (threadIdx.x < S) {
-    DevState* st = sts + threadIdx.x;
-    st->call = 0;
-    st->a = 0;
-    st->done = 0;
-    st->n_d = 0;
-    st->pos0 = 0;
-    st->n_rows = 2;
-    st->first_head_row = 1;
-    st->n_acc_last = 0;
-    st->q_row = 0;
-    st->round = 0;
-    st->emu = 0;
-    st->emu_n = 0;
-    st->emu_in = -1;
-    for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
-    st->codes[0] = C0V > 0 ? c0[threadIdx.x] : -1;
-    for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
-    st->n_emit_last = 0;
-    st->calls = st->drafted = st->accepted = 0;
-    st->heads_read = st->kv_rows = st->rows_fed = 0;
-  }
+  if (threadIdx.x < S) init_stream_state(sts + threadIdx.x, C0V > 0 ? c0[threadIdx.x] : -1);
 }
 
 // Reset counters of a single stepwise call (the call index of the state).
@@ -231,6 +210,7 @@ struct mcd_ctx {
   bool weights_loaded = false;
   bool frame_begun = false;
   int h_err = 0;                 // host-side sticky CUDA error
+  mcd::BatchState* batch = nullptr;   // GEMM path for calls with more than kMaxCols packed rows
 };
 
 mcd_status mcd::cuda_status(cudaError_t e) {
@@ -348,10 +328,15 @@ static mcd_status validate_config(const mcd_config& c) {
   if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
-  if (c.max_streams < 1 || c.max_streams > kMaxStreams) return MCD_ERR_UNSUPPORTED;
-  // every stream's rows of one call are packed into one operand of kMaxCols columns
-  if (c.max_streams * std::max(c.draft_len + 1, 2) > kMaxCols) return MCD_ERR_UNSUPPORTED;
+  if (c.max_streams < 1 || c.max_streams > kMaxBatchStreams) return MCD_ERR_UNSUPPORTED;
   if (c.max_streams > 1 && c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;
+  // beyond kMaxCols packed rows per call (or kMaxStreams streams) calls run on the batched
+  // GEMM path: bf16 weights, at most kMaxBatchRows rows, 16 query vectors per (stream, KV head)
+  const int rows = c.max_streams * std::max(c.draft_len + 1, 2);
+  if (rows > kMaxCols || c.max_streams > kMaxStreams) {
+    if (c.weight_dtype != MCD_WEIGHT_BF16 || rows > kMaxBatchRows) return MCD_ERR_UNSUPPORTED;
+    if (std::max(c.draft_len + 1, 2) * (c.n_q_heads / c.n_kv_heads) > 16) return MCD_ERR_UNSUPPORTED;
+  }
   if ((long long)c.n_q_heads * c.head_dim + 2LL * c.n_kv_heads * c.head_dim > 8192) return MCD_ERR_UNSUPPORTED;
   return MCD_OK;
 }
@@ -496,6 +481,10 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base, kMaxPos);
   if (cudaGetLastError() != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (k.max_streams > kMaxStreams || batch_rows(p, k.max_streams) > kMaxCols) {
+    mcd_status bs = batch_create(p, k.max_streams, &c->batch);
+    if (bs != MCD_OK) return fail(bs);
+  }
   *out = c;
   return MCD_OK;
 }
@@ -503,6 +492,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
 void mcd_destroy(mcd_ctx* c) {
   if (!c) return;
   cudaStreamSynchronize(c->stream);
+  batch_destroy(c->batch);
   for (void* q : c->allocs) cudaFree(q);
   delete c;
 }
@@ -650,6 +640,17 @@ mcd_status mcd_decode_frames(mcd_ctx* c, int32_t n_streams, const uint32_t* stre
                              mcd_frame_stats* stats) {
   if (!c || !codes_out) return MCD_ERR_INVALID_ARG;
   if (!c->weights_loaded) return MCD_ERR_STATE;
+  if (n_streams > kMaxStreams || batch_rows(c->fp, n_streams) > kMaxCols) {
+    // many streams: the batched GEMM path (one CUDA graph launch per frame)
+    const FrameParams& p = c->fp;
+    if (!c->batch || n_streams > c->cfg.max_streams) return MCD_ERR_INVALID_ARG;
+    if (!cond || !stream_ids || !frame_idx) return MCD_ERR_INVALID_ARG;
+    if (p.C0V > 0 && !c0) return MCD_ERR_INVALID_ARG;
+    if (p.C0V == 0 && !c0_emb) return MCD_ERR_INVALID_ARG;
+    c->frame_begun = false;
+    return batch_decode(c->batch, p, c->stream, n_streams, stream_ids, frame_idx, cond, c0, c0_emb, codes_out, stats,
+                        p.trace);
+  }
   mcd_status s = launch_begin(c, n_streams, stream_ids, frame_idx, cond, c0, c0_emb);
   if (s != MCD_OK) return s;
   FrameParams p = c->fp;

@@ -1,0 +1,900 @@
+// Batched decoding of many independent streams (up to 128 streams, 512 packed rows per
+// call): the per-frame draft-and-verify loop of arXiv 2609.37007 (Sec. 2.2, Fig. 3) for
+// every stream at once, with the rows of all unfinished streams re-packed every call.
+//
+// With hundreds of rows per call the weight matrices are multiplied as real GEMMs, so this
+// path is a sequence of grid-wide kernels per call instead of the persistent frame kernel:
+//
+//   pack -> embed -> 5 x [QKV GEMM -> attention -> Wo GEMM (+residual) -> gate/up GEMM
+//   (SwiGLU) -> down GEMM (+residual)] -> LM-head GEMM (grouped by head) -> top-k -> accept
+//
+// captured once per context as a CUDA graph holding n_pos call bodies (a call never emits
+// fewer than one code, so n_pos calls always finish a frame; bodies after the last active
+// call find no rows and return at once).  RMSNorm never gets its own pass: the kernels that
+// write the residual stream also accumulate each row's sum of squares, and the next GEMM
+// scales its operand rows by gain / rms while staging them.  The GEMMs take the weights in
+// the same tiled unit layout as the frame kernel (each 16 x 16 tile in mma.m16n8k16
+// A-fragment order), stream them with cp.async through a 4-stage shared-memory pipeline and
+// multiply 128 weight rows x 64 packed rows per CTA with mma.sync (bf16 operands, fp32
+// accumulation).  Sampling and acceptance use the same integer sampler as the frame kernel.
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+#include "mcd_host.cuh"
+#include "mcd_internal.cuh"
+#include "mcd_sampler.cuh"
+
+namespace mcd {
+
+constexpr int kGM = 128;                 // weight rows per GEMM tile (8 m-tiles)
+constexpr int kGN = 64;                  // packed rows per GEMM tile (8 n-tiles)
+constexpr int kGK = 64;                  // k per pipeline stage (4 k-tiles)
+constexpr int kGStages = 4;
+constexpr int kGBStride = kGK + 8;       // bf16 per staged operand row (144 B: conflict-free ldmatrix)
+constexpr int kGAStage = 32 * 512;       // 8 m-tiles x 4 k-tiles of 512 B
+constexpr int kGBStage = kGN * kGBStride * 2;
+constexpr int kGemmSmem = kGStages * (kGAStage + kGBStage);
+constexpr int kRecSlots = kMaxDraft + 1;   // distributions per packed row (verify + drafts)
+constexpr int kBatchQVec = 16;             // query vectors per attention CTA: rows x (q heads per KV head)
+
+enum BSrc { BSRC_NORM = 0, BSRC_BF16 = 1 };
+enum Epi { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_HEADS = 3 };
+
+struct BatchRow {
+  int s, n, pos, id;
+  const uint8_t* src;     // layer-0 input row
+  int f32;                // src is fp32 (else bf16)
+};
+
+struct BatchInfo {
+  int M;                  // packed rows of the call
+  int n_pairs;            // (row, j) distributions of the call
+  int head_rows[16];      // rows reading LM head P (entries in head_list)
+  int head_off[16];
+};
+
+// Per-frame arguments, copied to the device before each graph launch.
+struct BatchFrame {
+  int S;
+  unsigned stream_ids[kMaxBatchStreams];
+  unsigned frame_ids[kMaxBatchStreams];
+  const float* cond;
+  const int* c0;
+  const float* c0emb;
+  int* codes_out;
+  mcd_frame_stats* stats;
+  uint8_t* trace;
+};
+
+struct BatchBufs {
+  int R;                  // packed-row capacity
+  BatchInfo* info;
+  BatchFrame* frame;
+  BatchRow* rows;         // [R]
+  int* sbase;             // [kMaxBatchStreams] first packed row of each stream (-1: inactive)
+  int* pairs;             // [R * kRecSlots] (row << 3) | j
+  int* head_list;         // [R * kRecSlots] grouped by head
+  float* X;               // [R][H] residual stream
+  float* ss;              // [2L + 1][R] per-row sums of squares of X after each residual write
+  float* qkv;             // [R][qkv_dim]
+  uint16_t* att;          // [R][NH * D] bf16 attention outputs
+  uint16_t* act;          // [R][F] bf16 SwiGLU outputs
+  float* logits;          // [R][kRecSlots][V]
+  TopkRec* recs;          // [2][R][kRecSlots]
+};
+
+// ------------------------------------------------------------------------------------
+// small helpers
+// ------------------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ uint16_t f32_to_bf16(float x) { return (uint16_t)bf16_rn_bits(x); }
+
+// Offset (bytes) of 16 x 16 tile (m-tile mt, k-tile kt) in a tiled bf16 matrix.
+__device__ __forceinline__ size_t tile_byte_offset(const MatGeom& g, int mt, int kt) {
+  const int kcu = kt / g.Ku, ktl = kt - kcu * g.Ku, mbu = mt / g.Mu, mi = mt - mbu * g.Mu;
+  const long long u = (long long)kcu * g.n_mb + mbu;
+  return (size_t)(((u * g.Mu + mi) * g.Ku) + ktl) * 512;
+}
+
+// ------------------------------------------------------------------------------------
+// pack: the call's rows, distributions and head groups from every stream's state
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) batch_pack_kernel(FrameParams p, BatchBufs b) {
+  __shared__ int s_cnt[256], s_pc[256], s_head[16], s_hcur[16];
+  const BatchFrame* fa = b.frame;
+  const int S = fa->S, tid = threadIdx.x;
+  const int L = p.L;
+  for (int i = tid; i < (2 * L + 1) * b.R; i += blockDim.x) b.ss[i] = 0.f;
+  if (tid < 16) s_head[tid] = 0;
+  int nr = 0, np = 0;
+  DevState st;
+  if (tid < S) {
+    st = p.st[tid];
+    if (!st.done) {
+      nr = st.n_rows;
+      for (int n = 0; n < nr; ++n) {
+        const int pos = st.pos0 + n;
+        if (pos >= 1) np += min(p.K, p.P - pos) + 1;
+      }
+    }
+  }
+  s_cnt[tid] = nr;
+  s_pc[tid] = np;
+  __syncthreads();
+  for (int off = 1; off < 256; off <<= 1) {      // inclusive scans (Hillis-Steele)
+    const int a = tid >= off ? s_cnt[tid - off] : 0, c = tid >= off ? s_pc[tid - off] : 0;
+    __syncthreads();
+    s_cnt[tid] += a;
+    s_pc[tid] += c;
+    __syncthreads();
+  }
+  const int base = s_cnt[tid] - nr, pbase = s_pc[tid] - np;
+  if (tid < S && nr > 0) {
+    for (int n = 0; n < nr; ++n) {
+      const int pos = st.pos0 + n, r = base + n;
+      int id = st.pos0 == 0 ? (n == 0 ? -1 : st.codes[0]) : (n == 0 ? st.codes[st.a] : st.drafts[n - 1]);
+      BatchRow row;
+      row.s = tid;
+      row.n = n;
+      row.pos = pos;
+      if (pos == 0 || (pos == 1 && p.C0V == 0)) {
+        row.src = reinterpret_cast<const uint8_t*>((pos == 0 ? fa->cond : fa->c0emb) + (size_t)tid * p.H);
+        row.f32 = 1;
+      } else {
+        const int table = pos - 1;
+        if (id < 0 || id >= (table == 0 ? p.C0V : p.V)) {
+          atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
+          id = 0;
+        }
+        row.src = p.embed + (long long)table * p.embed_stride + (long long)id * p.H * 2;
+        row.f32 = 0;
+      }
+      row.id = id;
+      b.rows[r] = row;
+      if (pos >= 1) {
+        const int kn = min(p.K, p.P - pos);
+        for (int j = 0; j <= kn; ++j) atomicAdd(&s_head[pos + j], 1);
+      }
+    }
+  }
+  if (tid < kMaxBatchStreams) b.sbase[tid] = (tid < S && nr > 0) ? base : -1;
+  __syncthreads();
+  if (tid == 0) {
+    int off = 0;
+    for (int P = 0; P < 16; ++P) {
+      b.info->head_rows[P] = s_head[P];
+      b.info->head_off[P] = off;
+      s_hcur[P] = off;
+      off += s_head[P];
+    }
+    b.info->M = s_cnt[255];
+    b.info->n_pairs = s_pc[255];
+  }
+  __syncthreads();
+  if (tid < S && nr > 0) {
+    int pi = pbase;
+    for (int n = 0; n < nr; ++n) {
+      const int pos = st.pos0 + n, r = base + n;
+      if (pos < 1) continue;
+      const int kn = min(p.K, p.P - pos);
+      for (int j = 0; j <= kn; ++j) {
+        b.pairs[pi++] = (r << 3) | j;
+        b.head_list[atomicAdd(&s_hcur[pos + j], 1)] = (r << 3) | j;
+      }
+    }
+  }
+}
+
+// embed: X[r] = the row's input vector; ss[0][r] = sum of squares.
+__global__ void __launch_bounds__(256) batch_embed_kernel(FrameParams p, BatchBufs b) {
+  const int r = blockIdx.x;
+  if (r >= b.info->M) return;
+  const BatchRow row = b.rows[r];
+  float s = 0.f;
+  for (int k = threadIdx.x; k < p.H; k += blockDim.x) {
+    const float v = row.f32 ? __ldg(reinterpret_cast<const float*>(row.src) + k)
+                            : bf16_bits_to_f32(__ldg(reinterpret_cast<const uint16_t*>(row.src) + k));
+    b.X[(size_t)r * p.H + k] = v;
+    s += v * v;
+  }
+  for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+  __shared__ float sw[8];
+  if ((threadIdx.x & 31) == 0) sw[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += sw[w];
+    b.ss[r] = t;
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// GEMM: C[o][row] = sum_k W[o][k] X[row][k] over 128 weight rows x 64 packed rows per CTA
+// ------------------------------------------------------------------------------------
+struct GemmArgs {
+  const uint8_t* W;       // tiled bf16 matrix (heads: head 1; head P at + (P-1) * g.stride)
+  MatGeom g;
+  // operand rows
+  const float* X;         // BSRC_NORM: fp32 rows [R][ldx], scaled by gain[k] / rms(row)
+  const float* gain;
+  const float* ss;        // per-row sums of squares of X
+  const uint16_t* Xb;     // BSRC_BF16: bf16 rows [R][ldx]
+  int ldx;
+  // outputs
+  float* out;             // EPI_QKV: [R][ld]; EPI_RESID: the residual X [R][ld]
+  float* ss_out;          // EPI_RESID: sums of squares of the updated rows
+  uint16_t* act;          // EPI_SWIGLU: [R][ld]
+  int ld;
+  float* logits;          // EPI_HEADS: [R][kRecSlots][V]
+  const float* head_bias; // EPI_HEADS: [n_pos][K][V]
+  int K, V;
+  const BatchInfo* info;
+  const int* head_list;
+  float eps;
+};
+
+template <int BSRC, int EPI>
+__global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__ GemmArgs a) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ int s_row[kGN];
+  __shared__ int s_j[kGN];
+  __shared__ float s_inv[kGN];
+  __shared__ float s_ss[kGN];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const BatchInfo* info = a.info;
+  int n_rows;
+  const int* rlist = nullptr;
+  const uint8_t* W = a.W;
+  int P = 0;
+  if (EPI == EPI_HEADS) {
+    P = blockIdx.z + 1;
+    n_rows = info->head_rows[P];
+    rlist = a.head_list + info->head_off[P];
+    W += (size_t)(P - 1) * a.g.stride;
+  } else {
+    n_rows = info->M;
+  }
+  const int r0 = blockIdx.y * kGN;
+  if (r0 >= n_rows) return;
+  const MatGeom& g = a.g;
+  const int mt0 = blockIdx.x * (kGM / 16);                 // first m-tile of the CTA
+  const int n_mt = g.M >> 4;
+  const int Kdim = g.K, n_kc = Kdim / kGK;
+  if (tid < kGN) {
+    const int i = r0 + tid;
+    int r = -1, j = 0;
+    if (i < n_rows) {
+      if (rlist) {
+        const int e = rlist[i];
+        r = e >> 3;
+        j = e & 7;
+      } else {
+        r = i;
+      }
+    }
+    s_row[tid] = r;
+    s_j[tid] = j;
+    if (BSRC == BSRC_NORM) s_inv[tid] = r >= 0 ? rsqrtf(a.ss[r] / (float)Kdim + a.eps) : 0.f;
+    s_ss[tid] = 0.f;
+  }
+  __syncthreads();
+  uint8_t* sA = smem;
+  uint16_t* sB = reinterpret_cast<uint16_t*>(smem + kGStages * kGAStage);
+
+  // ---- stage loaders ------------------------------------------------------------------------
+  auto load_A = [&](int kc, int st) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int c = tid + 256 * i, t = c >> 5, part = c & 31;
+      const int mt = mt0 + (t >> 2), kt = kc * 4 + (t & 3);
+      uint8_t* dst = sA + st * kGAStage + t * 512 + part * 16;
+      const bool ok = mt < n_mt;
+      const uint8_t* src = W + (ok ? tile_byte_offset(g, mt, kt) : 0) + part * 16;
+      cp_async16(dst, src, ok ? 16 : 0);
+    }
+  };
+  float4 breg[4];
+  auto fetch_B = [&](int kc) {           // BSRC_NORM: fp32 rows into registers
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int c = tid + 256 * i, rr = c >> 4, q = c & 15;
+      const int r = s_row[rr];
+      breg[i] = r >= 0 ? __ldcg(reinterpret_cast<const float4*>(a.X + (size_t)r * a.ldx + kc * kGK) + q)
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  };
+  auto store_B = [&](int kc, int st) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int c = tid + 256 * i, rr = c >> 4, q = c & 15, k = kc * kGK + 4 * q;
+      const float4 gg = __ldg(reinterpret_cast<const float4*>(a.gain + k));
+      const float s = s_inv[rr];
+      const uint32_t lo = pack_bf16x2(breg[i].x * gg.x * s, breg[i].y * gg.y * s);
+      const uint32_t hi = pack_bf16x2(breg[i].z * gg.z * s, breg[i].w * gg.w * s);
+      *reinterpret_cast<uint2*>(sB + (size_t)st * (kGN * kGBStride) + rr * kGBStride + 4 * q) = make_uint2(lo, hi);
+    }
+  };
+  auto load_B16 = [&](int kc, int st) {   // BSRC_BF16: cp.async
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int c = tid + 256 * i, rr = c >> 3, ch = c & 7;
+      const int r = s_row[rr];
+      const uint16_t* src = a.Xb + (size_t)(r >= 0 ? r : 0) * a.ldx + kc * kGK + ch * 8;
+      cp_async16(sB + (size_t)st * (kGN * kGBStride) + rr * kGBStride + ch * 8, src, r >= 0 ? 16 : 0);
+    }
+  };
+
+  // ---- main loop ------------------------------------------------------------------------------
+  const int wm = (warp & 3) * 2;          // the warp's first m-tile within the CTA tile
+  const int wn = (warp >> 2) * 4;         // its first n-tile
+  float acc[2][4][4];
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[i][j][e] = 0.f;
+
+#pragma unroll
+  for (int st = 0; st < kGStages - 1; ++st) {
+    if (st < n_kc) {
+      load_A(st, st);
+      if (BSRC == BSRC_BF16) {
+        load_B16(st, st);
+      } else {
+        fetch_B(st);
+        store_B(st, st);
+      }
+    }
+    cp_async_commit();
+  }
+  for (int kc = 0; kc < n_kc; ++kc) {
+    const int st = kc % kGStages;
+    const int nk = kc + kGStages - 1;
+    if (BSRC == BSRC_NORM && nk < n_kc) fetch_B(nk);
+    cp_async_wait<kGStages - 2>();
+    __syncthreads();
+    const uint8_t* A = sA + st * kGAStage;
+    const uint16_t* B = sB + (size_t)st * (kGN * kGBStride);
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt) {
+      const uint4 a0 = *reinterpret_cast<const uint4*>(A + ((wm + 0) * 4 + kt) * 512 + lane * 16);
+      const uint4 a1 = *reinterpret_cast<const uint4*>(A + ((wm + 1) * 4 + kt) * 512 + lane * 16);
+#pragma unroll
+      for (int hp = 0; hp < 2; ++hp) {
+        uint32_t bf[4];
+        const int row = (wn + 2 * hp + (lane >> 4)) * 8 + (lane & 7);
+        const int kk = kt * 16 + ((lane >> 3) & 1) * 8;
+        ldmatrix_x4(bf, B + row * kGBStride + kk);
+        mma_bf16_16816(acc[0][2 * hp], a0, bf[0], bf[1]);
+        mma_bf16_16816(acc[0][2 * hp + 1], a0, bf[2], bf[3]);
+        mma_bf16_16816(acc[1][2 * hp], a1, bf[0], bf[1]);
+        mma_bf16_16816(acc[1][2 * hp + 1], a1, bf[2], bf[3]);
+      }
+    }
+    // stage nk % kGStages was last read in iteration kc - 1, which every warp has left
+    if (nk < n_kc) {
+      const int sn = nk % kGStages;
+      load_A(nk, sn);
+      if (BSRC == BSRC_BF16)
+        load_B16(nk, sn);
+      else
+        store_B(nk, sn);
+    }
+    cp_async_commit();
+  }
+  cp_async_wait<0>();
+
+  // ---- epilogue ----------------------------------------------------------------------------
+  // acc[i][j]: m-tile wm + i, n-tile wn + j; c0/c1 -> weight row +lane/4, packed rows
+  // 2(lane%4) + {0,1}; c2/c3 -> weight row +lane/4 + 8.
+  float ssp[4][2];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) ssp[j][0] = ssp[j][1] = 0.f;
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int mt = mt0 + wm + i;
+    if (mt >= n_mt) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {      // packed row 2(lane%4) + h
+        const int rr = (wn + j) * 8 + 2 * (lane & 3) + h;
+        const int r = s_row[rr];
+        if (r < 0) continue;
+        const float v_lo = acc[i][j][h], v_hi = acc[i][j][2 + h];   // weight rows +lane/4, +lane/4 + 8
+        const int o = mt * 16 + (lane >> 2);
+        if (EPI == EPI_QKV) {
+          a.out[(size_t)r * a.ld + o] = v_lo;
+          a.out[(size_t)r * a.ld + o + 8] = v_hi;
+        } else if (EPI == EPI_RESID) {
+          float* xr = a.out + (size_t)r * a.ld;
+          const float n0 = xr[o] + v_lo, n1 = xr[o + 8] + v_hi;
+          xr[o] = n0;
+          xr[o + 8] = n1;
+          ssp[j][h] += n0 * n0 + n1 * n1;
+        } else if (EPI == EPI_SWIGLU) {
+          const int jj = mt * 8 + (lane >> 2);       // gate row (tile row lane/4), up row (+8)
+          const float gt = v_lo;
+          a.act[(size_t)r * a.ld + jj] = f32_to_bf16(gt / (1.0f + __expf(-gt)) * v_hi);
+        } else {
+          const int jd = s_j[rr];
+          float* lg = a.logits + ((size_t)r * kRecSlots + jd) * a.V;
+          float b0 = 0.f, b1 = 0.f;
+          if (jd >= 1) {
+            const float* bias = a.head_bias + ((size_t)(P - 1) * a.K + (jd - 1)) * a.V;
+            b0 = __ldg(bias + o);
+            b1 = __ldg(bias + o + 8);
+          }
+          lg[o] = v_lo + b0;
+          lg[o + 8] = v_hi + b1;
+        }
+      }
+    }
+  }
+  if (EPI == EPI_RESID) {
+    // per packed row: sum over the lanes sharing it (lane/4 varies) and the warps' m-tiles
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float v = ssp[j][h];
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 4);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 8);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 16);
+        if (lane < 4) atomicAdd(&s_ss[(wn + j) * 8 + 2 * lane + h], v);
+      }
+    __syncthreads();
+    if (tid < kGN && s_row[tid] >= 0) atomicAdd(a.ss_out + s_row[tid], s_ss[tid]);
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// attention: one CTA per (stream, KV head)
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBufs b, int layer) {
+  const int s = blockIdx.x, g = blockIdx.y;
+  if (s >= b.frame->S) return;
+  const int base = b.sbase[s];
+  if (base < 0) return;
+  const DevState* st = p.st + s;
+  const int nr = st->n_rows, pos0 = st->pos0;
+  const int D = p.D, half = D >> 1, group = p.NH / p.NKV, nq = nr * group;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  __shared__ float qs[kBatchQVec][132];        // nr x group query vectors
+  __shared__ float ks[kMaxPos][132];
+  __shared__ float vs[kMaxPos][128];
+  __shared__ float sc[kBatchQVec][kMaxPos];
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const int nk = pos0 + nr;
+  // loads: queries, new keys / values, cached keys / values
+  for (int i = tid; i < nq * D; i += blockDim.x) {
+    const int qi = i / D, d = i - qi * D, n = qi / group, h = g * group + qi % group;
+    qs[qi][d] = __ldcg(b.qkv + (size_t)(base + n) * p.qkv_dim + h * D + d);
+  }
+  for (int i = tid; i < nk * D; i += blockDim.x) {
+    const int j = i / D, d = i - j * D;
+    if (j < pos0) {
+      ks[j][d] = __ldcg(p.kcache + cache_off + (size_t)j * D + d);
+      vs[j][d] = __ldcg(p.vcache + cache_off + (size_t)j * D + d);
+    } else {
+      const size_t rb = (size_t)(base + j - pos0) * p.qkv_dim;
+      ks[j][d] = __ldcg(b.qkv + rb + p.NH * D + g * D + d);
+      vs[j][d] = __ldcg(b.qkv + rb + p.NH * D + p.NKV * D + g * D + d);
+    }
+  }
+  __syncthreads();
+  // QK-norm + RoPE of the queries and the new keys (one warp per vector); new K / V cached
+  const int nd = D >> 5;
+  for (int vi = warp; vi < nq + nr; vi += 8) {
+    const bool isq = vi < nq;
+    const int n = isq ? vi / group : vi - nq;
+    float* row = isq ? qs[vi] : ks[pos0 + n];
+    float x[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = i < nd ? row[lane + 32 * i] : 0.f;
+    if (p.qk_norm) {
+      float ss = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ss += x[i] * x[i];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+      const float scl = rsqrtf(ss / (float)D + p.eps);
+      const float* gg = (isq ? p.q_norm : p.k_norm) + (size_t)layer * D;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) x[i] = x[i] * scl * __ldg(gg + lane + 32 * i);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if (i < nd / 2) {
+        const float2 r = __ldg(p.rope + (size_t)(pos0 + n) * half + lane + 32 * i);
+        const float a0 = x[i], b0 = x[i + nd / 2];
+        x[i] = a0 * r.x - b0 * r.y;
+        x[i + nd / 2] = b0 * r.x + a0 * r.y;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < nd) row[lane + 32 * i] = x[i];
+    if (!isq) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) {
+          p.kcache[cache_off + (size_t)(pos0 + n) * D + lane + 32 * i] = x[i];
+          p.vcache[cache_off + (size_t)(pos0 + n) * D + lane + 32 * i] = vs[pos0 + n][lane + 32 * i];
+        }
+    }
+  }
+  __syncthreads();
+  // scores (one thread per (query, key)), softmax (one warp per query), P.V
+  const float scale = rsqrtf((float)D);
+  for (int t = tid; t < nq * nk; t += blockDim.x) {
+    const int qi = t / nk, j = t - qi * nk, n = qi / group;
+    float acc = 0.f;
+    if (j <= pos0 + n)
+      for (int d = 0; d < D; ++d) acc += qs[qi][d] * ks[j][d];
+    sc[qi][j] = j <= pos0 + n ? acc * scale : -INFINITY;
+  }
+  __syncthreads();
+  for (int qi = warp; qi < nq; qi += 8) {
+    const float v = lane < nk ? sc[qi][lane] : -INFINITY;
+    float m = v;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
+    const float e = v == -INFINITY ? 0.f : __expf(v - m);
+    float l = e;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, off);
+    if (lane < nk) sc[qi][lane] = e / l;
+  }
+  __syncthreads();
+  for (int t = tid; t < nq * D; t += blockDim.x) {
+    const int qi = t / D, d = t - qi * D, n = qi / group, h = g * group + qi % group;
+    float acc = 0.f;
+    for (int j = 0; j <= pos0 + n; ++j) acc += sc[qi][j] * vs[j][d];
+    b.att[(size_t)(base + n) * p.NH * D + h * D + d] = f32_to_bf16(acc);
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// top-k of every (row, j) distribution of the call; then the acceptance per stream
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kConsumerThreads) batch_topk_kernel(FrameParams p, BatchBufs b, int call) {
+  __shared__ __align__(16) uint8_t smem_raw[sizeof(TopkScratch)];
+  TopkScratch& ts = *reinterpret_cast<TopkScratch*>(smem_raw);
+  if ((int)blockIdx.x >= b.info->n_pairs) return;
+  const int e = b.pairs[blockIdx.x], r = e >> 3, j = e & 7;
+  const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
+  TopkRec* recs = b.recs + (size_t)(call & 1) * b.R * kRecSlots;
+  block_topk(b.logits + ((size_t)r * kRecSlots + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
+             recs + (size_t)r * kRecSlots + j);
+}
+
+__global__ void __launch_bounds__(kConsumerThreads) batch_accept_kernel(FrameParams p, BatchBufs b, int call) {
+  const int s = blockIdx.x;
+  const BatchFrame* fa = b.frame;
+  if (s >= fa->S) return;
+  const int base = b.sbase[s];
+  if (base < 0) return;
+  DevState* st = p.st + s;
+  __shared__ AcceptResult s_res;
+  __shared__ int s_next[kMaxDraft], s_old[kMaxDraft + 1];
+  const int a = st->a, n_d = st->n_d, pos0 = st->pos0, n_rows = st->n_rows, qrow = st->q_row;
+  const int fr = st->first_head_row;
+  if (threadIdx.x <= kMaxDraft) s_old[threadIdx.x] = (int)threadIdx.x < n_d ? st->drafts[threadIdx.x] : -1;
+  __syncthreads();
+  const unsigned sid = fa->stream_ids[s], fid = fa->frame_ids[s];
+  const TopkRec* cur = b.recs + (size_t)(call & 1) * b.R * kRecSlots;
+  const TopkRec* prev = b.recs + (size_t)((call + 1) & 1) * b.R * kRecSlots;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp == 0) {
+    const AcceptResult r = warp_accept(
+        a, n_d, p.P, s_old, [&](int i) { return cur + (size_t)(base + a + 1 + i - pos0) * kRecSlots; },
+        [&](int i) { return prev + (size_t)qrow * kRecSlots + 1 + i; }, p.seed, sid, fid, call);
+    if (lane == 0) s_res = r;
+  }
+  __syncthreads();
+  const int n_emit = s_res.n_emit, n_acc = s_res.n_acc;
+  const int a_new = a + n_emit, m = a_new - pos0, n_next = min(p.K, p.P - a_new);
+  // next drafts from the draft distributions of row m, whose head emitted the last code
+  for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
+    const unsigned long long U = uniform_U(p.seed, sid, fid, call, a_new + j, PURPOSE_DRAFT);
+    const int d = warp_draw(cur + (size_t)(base + m) * kRecSlots + j, U);
+    if (lane == 0) s_next[j - 1] = d;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int* codes_out = fa->codes_out ? fa->codes_out + (size_t)s * p.P : nullptr;
+    for (int t = 0; t < n_emit; ++t) {
+      st->codes[a + 1 + t] = s_res.emitted[t];
+      if (codes_out) codes_out[a + t] = s_res.emitted[t];
+    }
+    for (int j = 0; j < n_next; ++j) st->drafts[j] = s_next[j];
+    for (int t = 0; t < n_emit; ++t) st->emitted_last[t] = s_res.emitted[t];
+    const int p_lo = a + 1, p_hi = min(p.P, pos0 + n_rows - 1 + p.K);
+    const int calls = st->calls + 1, heads = st->heads_read + p_hi - p_lo + 1;
+    const int kvr = st->kv_rows + pos0 + n_rows, rf = st->rows_fed + n_rows;
+    const int drafted = st->drafted + n_d, accepted = st->accepted + n_acc;
+    st->n_emit_last = n_emit;
+    st->n_acc_last = n_acc;
+    st->a = a_new;
+    st->n_d = n_next;
+    st->pos0 = a_new + 1;
+    st->n_rows = min(n_next + 1, p.P - a_new);
+    st->round = call + 1;
+    st->first_head_row = 0;
+    st->calls = calls;
+    st->heads_read = heads;
+    st->kv_rows = kvr;
+    st->rows_fed = rf;
+    st->drafted = drafted;
+    st->accepted = accepted;
+    st->call = call + 1;
+    st->done = a_new >= p.P ? 1 : 0;
+    st->q_row = base + m;     // the next call's q: this call's records of packed row base + m
+    if (a_new >= p.P && fa->stats) {
+      mcd_frame_stats* fs = fa->stats + s;
+      fs->calls = calls;
+      fs->codes = a_new;
+      fs->drafted = drafted;
+      fs->accepted = accepted;
+      fs->status = *(volatile int*)p.err;
+      fs->heads_read = heads;
+      fs->kv_rows = kvr;
+      fs->rows_fed = rf;
+    }
+  }
+  // optional trace, in the frame kernel's layout
+  if (fa->trace && call < kMaxCalls) {
+    uint8_t* tb = fa->trace + (size_t)s * p.trace_stride;
+    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(tb) + call;
+    if (threadIdx.x == 0) {
+      tr->a = a;
+      tr->n_rows = n_rows;
+      tr->pos0 = pos0;
+      tr->n_drafts = n_d;
+      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? b.rows[base + n].id : -1;
+      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = i < n_d ? s_old[i] : -1;
+      tr->n_acc = n_acc;
+      tr->n_emit = n_emit;
+      for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < n_emit ? s_res.emitted[t] : -1;
+      tr->n_next = n_next;
+      for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = j < n_next ? s_next[j] : -1;
+      tr->draft_row = m;
+    }
+    float* vlog = reinterpret_cast<float*>(tb + sizeof(mcd_call_trace) * kMaxCalls);
+    float* dlog = vlog + (size_t)kMaxCalls * kMaxRows * p.V;
+    for (int idx = threadIdx.x; idx < kMaxRows * p.V; idx += blockDim.x) {
+      const int n = idx / p.V, v = idx - n * p.V;
+      if (n >= fr && n < n_rows)
+        vlog[((size_t)call * kMaxRows + n) * p.V + v] = __ldcg(b.logits + ((size_t)(base + n) * kRecSlots) * p.V + v);
+      if (n < n_next)
+        dlog[((size_t)call * kMaxRows + n) * p.V + v] =
+            __ldcg(b.logits + ((size_t)(base + m) * kRecSlots + n + 1) * p.V + v);
+    }
+  }
+}
+
+__global__ void batch_begin_kernel(FrameParams p, BatchBufs b) {
+  const BatchFrame* fa = b.frame;
+  for (int s = threadIdx.x; s < fa->S; s += blockDim.x) init_stream_state(p.st + s, p.C0V > 0 ? fa->c0[s] : -1);
+}
+
+}  // namespace mcd
+
+// ------------------------------------------------------------------------------------
+// Host side: buffers, the per-context graph, one launch per frame
+// ------------------------------------------------------------------------------------
+namespace mcd {
+
+struct BatchState {
+  BatchBufs b;
+  BatchFrame host_frame;
+  int max_streams = 0;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  cudaStream_t cap = nullptr;
+  std::vector<void*> allocs;
+};
+
+template <class T>
+static cudaError_t batch_alloc(BatchState* bs, T** p, size_t bytes) {
+  void* q = nullptr;
+  cudaError_t e = cudaMalloc(&q, bytes < 256 ? 256 : bytes);
+  if (e != cudaSuccess) return e;
+  bs->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return cudaSuccess;
+}
+
+void batch_destroy(BatchState* bs) {
+  if (!bs) return;
+  if (bs->exec) cudaGraphExecDestroy(bs->exec);
+  if (bs->graph) cudaGraphDestroy(bs->graph);
+  if (bs->cap) cudaStreamDestroy(bs->cap);
+  for (void* q : bs->allocs) cudaFree(q);
+  delete bs;
+}
+
+int batch_rows(const FrameParams& p, int max_streams) { return max_streams * std::max(p.K + 1, 2); }
+
+mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out) {
+  *out = nullptr;
+  BatchState* bs = new BatchState();
+  bs->max_streams = max_streams;
+  auto fail = [&](mcd_status s) {
+    batch_destroy(bs);
+    return s;
+  };
+  BatchBufs& b = bs->b;
+  const int R = (batch_rows(p, max_streams) + kGN - 1) / kGN * kGN;
+  b.R = R;
+  cudaError_t e;
+#define BATCH_ALLOC(ptr, bytes)                                                        \
+  do {                                                                                 \
+    if ((e = batch_alloc(bs, &(ptr), (bytes))) != cudaSuccess) return fail(cuda_status(e)); \
+  } while (0)
+  BATCH_ALLOC(b.info, sizeof(BatchInfo));
+  BATCH_ALLOC(b.frame, sizeof(BatchFrame));
+  BATCH_ALLOC(b.rows, sizeof(BatchRow) * R);
+  BATCH_ALLOC(b.sbase, sizeof(int) * kMaxBatchStreams);
+  BATCH_ALLOC(b.pairs, sizeof(int) * R * kRecSlots);
+  BATCH_ALLOC(b.head_list, sizeof(int) * R * kRecSlots);
+  BATCH_ALLOC(b.X, sizeof(float) * R * p.H);
+  BATCH_ALLOC(b.ss, sizeof(float) * (2 * p.L + 1) * R);
+  BATCH_ALLOC(b.qkv, sizeof(float) * R * p.qkv_dim);
+  BATCH_ALLOC(b.att, sizeof(uint16_t) * R * p.NH * p.D);
+  BATCH_ALLOC(b.act, sizeof(uint16_t) * R * p.F);
+  BATCH_ALLOC(b.logits, sizeof(float) * R * kRecSlots * p.V);
+  BATCH_ALLOC(b.recs, sizeof(TopkRec) * 2 * R * kRecSlots);
+#undef BATCH_ALLOC
+  if (cudaMemset(b.info, 0, sizeof(BatchInfo)) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  if (cudaStreamCreateWithFlags(&bs->cap, cudaStreamNonBlocking) != cudaSuccess) return fail(MCD_ERR_CUDA);
+  void* gemms[] = {(void*)batch_gemm_kernel<BSRC_NORM, EPI_QKV>, (void*)batch_gemm_kernel<BSRC_BF16, EPI_RESID>,
+                   (void*)batch_gemm_kernel<BSRC_NORM, EPI_SWIGLU>, (void*)batch_gemm_kernel<BSRC_NORM, EPI_HEADS>};
+  for (void* fn : gemms)
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem) != cudaSuccess)
+      return fail(MCD_ERR_CUDA);
+  *out = bs;
+  return MCD_OK;
+}
+
+static GemmArgs gemm_args(const FrameParams& p, const BatchBufs& b) {
+  GemmArgs a;
+  memset(&a, 0, sizeof(a));
+  a.info = b.info;
+  a.head_list = b.head_list;
+  a.eps = p.eps;
+  a.K = p.K;
+  a.V = p.V;
+  return a;
+}
+
+// Every kernel of one frame, in stream order on `s` (captured into the graph).
+static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cudaStream_t s) {
+  const BatchBufs& b = bs->b;
+  const int R = b.R, L = p.L, H = p.H;
+  const dim3 blk(256);
+  batch_begin_kernel<<<1, 256, 0, s>>>(p, b);
+  for (int call = 0; call < p.P; ++call) {
+    batch_pack_kernel<<<1, 256, 0, s>>>(p, b);
+    batch_embed_kernel<<<R, 256, 0, s>>>(p, b);
+    for (int l = 0; l < L; ++l) {
+      {   // RMSNorm -> QKV
+        GemmArgs a = gemm_args(p, b);
+        a.W = p.w_qkv + (size_t)l * p.g[MAT_QKV].stride;
+        a.g = p.g[MAT_QKV];
+        a.X = b.X;
+        a.ldx = H;
+        a.gain = p.attn_norm + (size_t)l * H;
+        a.ss = b.ss + (size_t)(2 * l) * R;
+        a.out = b.qkv;
+        a.ld = p.qkv_dim;
+        batch_gemm_kernel<BSRC_NORM, EPI_QKV><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+      }
+      batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);
+      {   // Wo + residual
+        GemmArgs a = gemm_args(p, b);
+        a.W = p.w_wo + (size_t)l * p.g[MAT_WO].stride;
+        a.g = p.g[MAT_WO];
+        a.Xb = b.att;
+        a.ldx = p.NH * p.D;
+        a.out = b.X;
+        a.ld = H;
+        a.ss_out = b.ss + (size_t)(2 * l + 1) * R;
+        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+      }
+      {   // RMSNorm -> gate/up -> SwiGLU
+        GemmArgs a = gemm_args(p, b);
+        a.W = p.w_gu + (size_t)l * p.g[MAT_GU].stride;
+        a.g = p.g[MAT_GU];
+        a.X = b.X;
+        a.ldx = H;
+        a.gain = p.ffn_norm + (size_t)l * H;
+        a.ss = b.ss + (size_t)(2 * l + 1) * R;
+        a.act = b.act;
+        a.ld = p.F;
+        batch_gemm_kernel<BSRC_NORM, EPI_SWIGLU><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+      }
+      {   // down + residual
+        GemmArgs a = gemm_args(p, b);
+        a.W = p.w_wd + (size_t)l * p.g[MAT_WD].stride;
+        a.g = p.g[MAT_WD];
+        a.Xb = b.act;
+        a.ldx = p.F;
+        a.out = b.X;
+        a.ld = H;
+        a.ss_out = b.ss + (size_t)(2 * l + 2) * R;
+        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+      }
+    }
+    {   // final RMSNorm -> LM heads, one grid slice per head
+      GemmArgs a = gemm_args(p, b);
+      a.W = p.w_head;
+      a.g = p.g[MAT_HEAD];
+      a.X = b.X;
+      a.ldx = H;
+      a.gain = p.final_norm;
+      a.ss = b.ss + (size_t)(2 * L) * R;
+      a.logits = b.logits;
+      a.head_bias = p.head_bias;
+      batch_gemm_kernel<BSRC_NORM, EPI_HEADS>
+          <<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN, p.P), blk, kGemmSmem, s>>>(a);
+    }
+    batch_topk_kernel<<<R * (p.K + 1), kConsumerThreads, 0, s>>>(p, b, call);
+    batch_accept_kernel<<<bs->max_streams, kConsumerThreads, 0, s>>>(p, b, call);
+  }
+  return cudaGetLastError();
+}
+
+mcd_status batch_decode(BatchState* bs, const FrameParams& p, cudaStream_t stream, int n, const uint32_t* stream_ids,
+                        const uint32_t* frame_ids, const float* cond, const int32_t* c0, const float* c0_emb,
+                        int32_t* codes_out, mcd_frame_stats* stats, uint8_t* trace) {
+  if (n < 1 || n > bs->max_streams) return MCD_ERR_INVALID_ARG;
+  if (!bs->exec) {
+    cudaStream_t s = bs->cap;
+    MCD_CHECK(cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal));
+    cudaError_t e = enqueue_frame(p, bs, s);
+    cudaGraph_t g = nullptr;
+    cudaError_t e2 = cudaStreamEndCapture(s, &g);
+    if (e != cudaSuccess || e2 != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      return cuda_status(e != cudaSuccess ? e : e2);
+    }
+    bs->graph = g;
+    MCD_CHECK(cudaGraphInstantiate(&bs->exec, g, 0));
+  }
+  BatchFrame& f = bs->host_frame;
+  memset(&f, 0, sizeof(f));
+  f.S = n;
+  for (int i = 0; i < n; ++i) {
+    f.stream_ids[i] = stream_ids[i];
+    f.frame_ids[i] = frame_ids[i];
+  }
+  f.cond = cond;
+  f.c0 = c0;
+  f.c0emb = c0_emb;
+  f.codes_out = codes_out;
+  f.stats = stats;
+  f.trace = trace;
+  MCD_CHECK(cudaMemcpyAsync(bs->b.frame, &f, sizeof(f), cudaMemcpyHostToDevice, stream));
+  MCD_CHECK(cudaGraphLaunch(bs->exec, stream));
+  return MCD_OK;
+}
+
+}  // namespace mcd

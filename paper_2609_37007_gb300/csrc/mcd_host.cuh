@@ -54,6 +54,15 @@ void load_layer(const FrameParams& p, cudaStream_t stream, const LayerSrc& src, 
 
 mcd_status cuda_status(cudaError_t e);
 
+// Batched decoding of many streams (GEMM path, mcd_batch.cu).
+struct BatchState;
+int batch_rows(const FrameParams& p, int max_streams);
+mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out);
+void batch_destroy(BatchState* bs);
+mcd_status batch_decode(BatchState* bs, const FrameParams& p, cudaStream_t stream, int n, const uint32_t* stream_ids,
+                        const uint32_t* frame_ids, const float* cond, const int32_t* c0, const float* c0_emb,
+                        int32_t* codes_out, mcd_frame_stats* stats, uint8_t* trace);
+
 // The inner (MultiCodeDecoder) context's parameters and stream.
 const FrameParams& ctx_params(const mcd_ctx* c);
 cudaStream_t ctx_stream(const mcd_ctx* c);

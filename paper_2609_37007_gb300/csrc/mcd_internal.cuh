@@ -18,7 +18,9 @@ namespace mcd {
 
 constexpr int kMaxRows = 8;          // rows of one stream in one call (K + 1 <= 8; first call uses 2)
 constexpr int kMaxCols = 32;         // rows of one call over all streams (packed operand columns)
-constexpr int kMaxStreams = 8;       // streams decoded together by one launch
+constexpr int kMaxStreams = 8;       // streams decoded together by one launch of the frame kernel
+constexpr int kMaxBatchStreams = 128;  // streams of one batched decode (GEMM path)
+constexpr int kMaxBatchRows = 512;     // packed rows of one batched call
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
@@ -72,6 +74,29 @@ struct DevState {
   int emu_n;           // drafts the noisy-target passes make for the next verify call
   int emu_in;          // code fed to the next noisy-target pass
 };
+
+// State of a stream at the start of a frame: the first call feeds [cond, c0] (positions 0, 1).
+__device__ inline void init_stream_state(DevState* st, int c0) {
+  st->call = 0;
+  st->a = 0;
+  st->done = 0;
+  st->n_d = 0;
+  st->pos0 = 0;
+  st->n_rows = 2;
+  st->first_head_row = 1;
+  st->n_acc_last = 0;
+  st->q_row = 0;
+  st->round = 0;
+  st->emu = 0;
+  st->emu_n = 0;
+  st->emu_in = -1;
+  for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
+  st->codes[0] = c0;
+  for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
+  st->n_emit_last = 0;
+  st->calls = st->drafted = st->accepted = 0;
+  st->heads_read = st->kv_rows = st->rows_fed = 0;
+}
 
 // One top-k / temperature distribution as integer weights: p(ids[i]) = W[i] / S.
 struct TopkRec {

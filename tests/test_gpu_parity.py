@@ -279,9 +279,60 @@ def test_batched_streams_full_size(n_streams):
     env.dec.close()
 
 
-def test_batched_streams_reject_too_many_rows():
-    with pytest.raises(mcd.MCDError):
-        mcd.Decoder(MCD.replace(max_streams=8, draft_len=4))       # 8 x (K + 1) > 32 packed rows
+def test_batched_streams_reject_shapes_beyond_the_gemm_path():
+    for cfg in (MCD.replace(max_streams=128, draft_len=4),         # 640 packed rows > 512
+                MCD.replace(max_streams=129),                      # more than 128 streams
+                TINY.replace(max_streams=16)):                     # fp32 weights beyond 32 packed rows
+        with pytest.raises(mcd.MCDError) as e:
+            mcd.Decoder(cfg)
+        assert e.value.status == 7
+
+
+# ------------------------------------------------- batched GEMM path (> 32 rows) ------
+TINY_BF16 = TINY.replace(weight_dtype=1)
+
+
+@pytest.mark.parametrize("cfg", [TINY_BF16.replace(max_streams=16), TINY_BF16.replace(max_streams=24, draft_len=3),
+                                 TINY_BF16.replace(max_streams=40, draft_len=1),
+                                 TINY_BF16.replace(max_streams=12, draft_len=0, n_pos=6)])
+def test_gemm_path_trace_parity_tiny_bf16(cfg):
+    """More than 32 packed rows per call: the batched GEMM path (one graph launch per frame).
+    Every stream's calls match the oracle decoding that stream alone."""
+    env = Env(cfg)
+    for rep in range(2):
+        n = cfg.max_streams - 3 * rep             # also fewer streams than the context allows
+        fidx = [100 * rep + 3 * s for s in range(n)]
+        sids = [11 + s for s in range(n)]
+        frames = [make_frame(cfg, f) for f in fidx]
+        codes, st, trs = decode_many(env, frames, fidx, sids)
+        worst = 0.0
+        for s in range(n):
+            assert st[s, 4] == 0 and st[s, 1] == cfg.n_pos, (s, st[s])
+            worst = max(worst, check_trace_against_oracle(cfg, env.model, frames[s], sids[s], fidx[s], trs[s],
+                                                          codes[s], int(st[s, 0]), logit_tol=2e-2))
+        print(cfg.max_streams, "streams: max |dlogit|", worst)
+    env.dec.close()
+
+
+@pytest.mark.parametrize("n_streams,checked", [(32, (0, 13, 31)), (128, (0, 77, 127))])
+def test_gemm_path_full_size(n_streams, checked):
+    """MultiCodeDecoder bf16 at B = 32 and 128 streams (128 and 512 packed rows): every
+    stream finishes its frame; sampled streams replay exactly against the oracle."""
+    cfg = MCD.replace(max_streams=n_streams)
+    env = Env(cfg)
+    fidx, sids = [7 + s for s in range(n_streams)], [1000 + s for s in range(n_streams)]
+    frames = [make_frame(cfg, f) for f in fidx]
+    codes, st, trs = decode_many(env, frames, fidx, sids)
+    assert (st[:, 4] == 0).all() and (st[:, 1] == cfg.n_pos).all()
+    assert ((codes >= 0) & (codes < cfg.vocab)).all()
+    for s in checked:
+        err = check_trace_against_oracle(cfg, env.model, frames[s], sids[s], fidx[s], trs[s], codes[s],
+                                         int(st[s, 0]), logit_tol=2e-2)
+        print("gemm path stream", s, "of", n_streams, "max |dlogit|", err)
+    # a second frame on the same context (the graph is reused)
+    codes2, st2, _ = decode_many(env, frames, [f + 1 for f in fidx], sids)
+    assert (st2[:, 1] == cfg.n_pos).all()
+    env.dec.close()
 
 
 # ------------------------------------------------- noisy-target drafts (K sweep) ------
