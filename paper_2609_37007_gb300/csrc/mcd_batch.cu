@@ -35,10 +35,14 @@ constexpr int kGBStride = kGK + 8;       // bf16 per staged operand row (144 B: 
 constexpr int kGAStage = 32 * 512;       // 8 m-tiles x 4 k-tiles of 512 B
 constexpr int kGBStage = kGN * kGBStride * 2;
 constexpr int kGemmSmem = kGStages * (kGAStage + kGBStage);
+constexpr int kGemmSmemHilo = kGStages * (kGAStage + 2 * kGBStage);   // B as a bf16 hi + lo pair
 constexpr int kRecSlots = kMaxDraft + 1;   // distributions per packed row (verify + drafts)
 constexpr int kBatchQVec = 16;             // query vectors per attention CTA: rows x (q heads per KV head)
 
-enum BSrc { BSRC_NORM = 0, BSRC_BF16 = 1 };
+// Operand rows: fp32 rows normalised while staged (as one bf16, or as a bf16 hi + lo pair
+// carrying about 16 mantissa bits, for the QKV and LM-head products whose errors the
+// attention softmax and the sampler see directly), or rows already in bf16.
+enum BSrc { BSRC_NORM = 0, BSRC_BF16 = 1, BSRC_NORM_HILO = 2 };
 enum Epi { EPI_QKV = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_HEADS = 3 };
 
 struct BatchRow {
@@ -236,7 +240,6 @@ struct GemmArgs {
   int ldx;
   // outputs
   float* out;             // EPI_QKV: [R][ld]; EPI_RESID: the residual X [R][ld]
-  float* ss_out;          // EPI_RESID: sums of squares of the updated rows
   uint16_t* act;          // EPI_SWIGLU: [R][ld]
   int ld;
   float* logits;          // EPI_HEADS: [R][kRecSlots][V]
@@ -249,6 +252,7 @@ struct GemmArgs {
 
 template <int BSRC, int EPI>
 __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__ GemmArgs a) {
+  constexpr bool kNorm = BSRC != BSRC_BF16, kHilo = BSRC == BSRC_NORM_HILO;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_row[kGN];
   __shared__ int s_j[kGN];
@@ -273,7 +277,16 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
   const MatGeom& g = a.g;
   const int mt0 = blockIdx.x * (kGM / 16);                 // first m-tile of the CTA
   const int n_mt = g.M >> 4;
-  const int Kdim = g.K, n_kc = Kdim / kGK;
+  const int Kdim = g.K;
+  // k-chunks of this CTA: all of them, or (residual GEMMs) slice blockIdx.z of gridDim.z
+  int kc0 = 0, kc1 = Kdim / kGK;
+  if (EPI != EPI_HEADS && gridDim.z > 1) {
+    const int per = (kc1 + gridDim.z - 1) / gridDim.z;
+    kc0 = blockIdx.z * per;
+    kc1 = min(kc1, kc0 + per);
+    if (kc0 >= kc1) return;
+  }
+  const int n_kc = kc1 - kc0;
   if (tid < kGN) {
     const int i = r0 + tid;
     int r = -1, j = 0;
@@ -288,12 +301,13 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
     }
     s_row[tid] = r;
     s_j[tid] = j;
-    if (BSRC == BSRC_NORM) s_inv[tid] = r >= 0 ? rsqrtf(a.ss[r] / (float)Kdim + a.eps) : 0.f;
+    if (kNorm) s_inv[tid] = r >= 0 ? rsqrtf(a.ss[r] / (float)Kdim + a.eps) : 0.f;
     s_ss[tid] = 0.f;
   }
   __syncthreads();
   uint8_t* sA = smem;
   uint16_t* sB = reinterpret_cast<uint16_t*>(smem + kGStages * kGAStage);
+  uint16_t* sBl = sB + (size_t)kGStages * kGN * kGBStride;   // lo parts (hi/lo operand)
 
   // ---- stage loaders ------------------------------------------------------------------------
   auto load_A = [&](int kc, int st) {
@@ -323,9 +337,16 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
       const int c = tid + 256 * i, rr = c >> 4, q = c & 15, k = kc * kGK + 4 * q;
       const float4 gg = __ldg(reinterpret_cast<const float4*>(a.gain + k));
       const float s = s_inv[rr];
-      const uint32_t lo = pack_bf16x2(breg[i].x * gg.x * s, breg[i].y * gg.y * s);
-      const uint32_t hi = pack_bf16x2(breg[i].z * gg.z * s, breg[i].w * gg.w * s);
-      *reinterpret_cast<uint2*>(sB + (size_t)st * (kGN * kGBStride) + rr * kGBStride + 4 * q) = make_uint2(lo, hi);
+      const float x0 = breg[i].x * gg.x * s, x1 = breg[i].y * gg.y * s, x2 = breg[i].z * gg.z * s,
+                  x3 = breg[i].w * gg.w * s;
+      const uint32_t h01 = pack_bf16x2(x0, x1), h23 = pack_bf16x2(x2, x3);
+      const size_t off = (size_t)st * (kGN * kGBStride) + rr * kGBStride + 4 * q;
+      *reinterpret_cast<uint2*>(sB + off) = make_uint2(h01, h23);
+      if (kHilo) {
+        const uint32_t l01 = pack_bf16x2(x0 - bf16_lo_f32(h01), x1 - bf16_hi_f32(h01));
+        const uint32_t l23 = pack_bf16x2(x2 - bf16_lo_f32(h23), x3 - bf16_hi_f32(h23));
+        *reinterpret_cast<uint2*>(sBl + off) = make_uint2(l01, l23);
+      }
     }
   };
   auto load_B16 = [&](int kc, int st) {   // BSRC_BF16: cp.async
@@ -352,24 +373,25 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
 #pragma unroll
   for (int st = 0; st < kGStages - 1; ++st) {
     if (st < n_kc) {
-      load_A(st, st);
-      if (BSRC == BSRC_BF16) {
-        load_B16(st, st);
+      load_A(kc0 + st, st);
+      if (!kNorm) {
+        load_B16(kc0 + st, st);
       } else {
-        fetch_B(st);
-        store_B(st, st);
+        fetch_B(kc0 + st);
+        store_B(kc0 + st, st);
       }
     }
     cp_async_commit();
   }
-  for (int kc = 0; kc < n_kc; ++kc) {
-    const int st = kc % kGStages;
-    const int nk = kc + kGStages - 1;
-    if (BSRC == BSRC_NORM && nk < n_kc) fetch_B(nk);
+  for (int it = 0; it < n_kc; ++it) {
+    const int st = it % kGStages;
+    const int nk = it + kGStages - 1;
+    if (kNorm && nk < n_kc) fetch_B(kc0 + nk);
     cp_async_wait<kGStages - 2>();
     __syncthreads();
     const uint8_t* A = sA + st * kGAStage;
     const uint16_t* B = sB + (size_t)st * (kGN * kGBStride);
+    const uint16_t* Bl = sBl + (size_t)st * (kGN * kGBStride);
 #pragma unroll
     for (int kt = 0; kt < 4; ++kt) {
       const uint4 a0 = *reinterpret_cast<const uint4*>(A + ((wm + 0) * 4 + kt) * 512 + lane * 16);
@@ -384,16 +406,23 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
         mma_bf16_16816(acc[0][2 * hp + 1], a0, bf[2], bf[3]);
         mma_bf16_16816(acc[1][2 * hp], a1, bf[0], bf[1]);
         mma_bf16_16816(acc[1][2 * hp + 1], a1, bf[2], bf[3]);
+        if (kHilo) {
+          ldmatrix_x4(bf, Bl + row * kGBStride + kk);
+          mma_bf16_16816(acc[0][2 * hp], a0, bf[0], bf[1]);
+          mma_bf16_16816(acc[0][2 * hp + 1], a0, bf[2], bf[3]);
+          mma_bf16_16816(acc[1][2 * hp], a1, bf[0], bf[1]);
+          mma_bf16_16816(acc[1][2 * hp + 1], a1, bf[2], bf[3]);
+        }
       }
     }
-    // stage nk % kGStages was last read in iteration kc - 1, which every warp has left
+    // stage nk % kGStages was last read in iteration it - 1, which every warp has left
     if (nk < n_kc) {
       const int sn = nk % kGStages;
-      load_A(nk, sn);
-      if (BSRC == BSRC_BF16)
-        load_B16(nk, sn);
+      load_A(kc0 + nk, sn);
+      if (!kNorm)
+        load_B16(kc0 + nk, sn);
       else
-        store_B(nk, sn);
+        store_B(kc0 + nk, sn);
     }
     cp_async_commit();
   }
@@ -402,9 +431,6 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
   // ---- epilogue ----------------------------------------------------------------------------
   // acc[i][j]: m-tile wm + i, n-tile wn + j; c0/c1 -> weight row +lane/4, packed rows
   // 2(lane%4) + {0,1}; c2/c3 -> weight row +lane/4 + 8.
-  float ssp[4][2];
-#pragma unroll
-  for (int j = 0; j < 4; ++j) ssp[j][0] = ssp[j][1] = 0.f;
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int mt = mt0 + wm + i;
@@ -421,12 +447,10 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
         if (EPI == EPI_QKV) {
           a.out[(size_t)r * a.ld + o] = v_lo;
           a.out[(size_t)r * a.ld + o + 8] = v_hi;
-        } else if (EPI == EPI_RESID) {
+        } else if (EPI == EPI_RESID) {   // k-slices of several CTAs add into the residual
           float* xr = a.out + (size_t)r * a.ld;
-          const float n0 = xr[o] + v_lo, n1 = xr[o + 8] + v_hi;
-          xr[o] = n0;
-          xr[o + 8] = n1;
-          ssp[j][h] += n0 * n0 + n1 * n1;
+          atomicAdd(xr + o, v_lo);
+          atomicAdd(xr + o + 8, v_hi);
         } else if (EPI == EPI_SWIGLU) {
           const int jj = mt * 8 + (lane >> 2);       // gate row (tile row lane/4), up row (+8)
           const float gt = v_lo;
@@ -446,21 +470,22 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
       }
     }
   }
-  if (EPI == EPI_RESID) {
-    // per packed row: sum over the lanes sharing it (lane/4 varies) and the warps' m-tiles
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        float v = ssp[j][h];
-        v += __shfl_xor_sync(0xFFFFFFFFu, v, 4);
-        v += __shfl_xor_sync(0xFFFFFFFFu, v, 8);
-        v += __shfl_xor_sync(0xFFFFFFFFu, v, 16);
-        if (lane < 4) atomicAdd(&s_ss[(wn + j) * 8 + 2 * lane + h], v);
-      }
-    __syncthreads();
-    if (tid < kGN && s_row[tid] >= 0) atomicAdd(a.ss_out + s_row[tid], s_ss[tid]);
+}
+
+// Per-row sums of squares of the residual stream after a residual GEMM (one warp per row):
+// the next RMSNorm's 1/rms, applied while the next GEMM stages its operand.
+__global__ void __launch_bounds__(256) batch_rowss_kernel(const float* X, int H, float* ss, const BatchInfo* info) {
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= info->M) return;
+  const float4* x = reinterpret_cast<const float4*>(X + (size_t)r * H);
+  float s = 0.f;
+  for (int i = lane; i < (H >> 2); i += 32) {
+    const float4 v = __ldcg(x + i);
+    s += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+  if (lane == 0) ss[r] = s;
 }
 
 // ------------------------------------------------------------------------------------
@@ -765,10 +790,10 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
 #undef BATCH_ALLOC
   if (cudaMemset(b.info, 0, sizeof(BatchInfo)) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamCreateWithFlags(&bs->cap, cudaStreamNonBlocking) != cudaSuccess) return fail(MCD_ERR_CUDA);
-  void* gemms[] = {(void*)batch_gemm_kernel<BSRC_NORM, EPI_QKV>, (void*)batch_gemm_kernel<BSRC_BF16, EPI_RESID>,
-                   (void*)batch_gemm_kernel<BSRC_NORM, EPI_SWIGLU>, (void*)batch_gemm_kernel<BSRC_NORM, EPI_HEADS>};
+  void* gemms[] = {(void*)batch_gemm_kernel<BSRC_NORM_HILO, EPI_QKV>, (void*)batch_gemm_kernel<BSRC_BF16, EPI_RESID>,
+                   (void*)batch_gemm_kernel<BSRC_NORM, EPI_SWIGLU>, (void*)batch_gemm_kernel<BSRC_NORM_HILO, EPI_HEADS>};
   for (void* fn : gemms)
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem) != cudaSuccess)
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmemHilo) != cudaSuccess)
       return fail(MCD_ERR_CUDA);
   *out = bs;
   return MCD_OK;
@@ -783,6 +808,14 @@ static GemmArgs gemm_args(const FrameParams& p, const BatchBufs& b) {
   a.K = p.K;
   a.V = p.V;
   return a;
+}
+
+// k-slices of a residual GEMM: enough CTAs for about two per SM, at least 4 k-chunks each.
+static int split_k(dim3 grid, int K, int n_sm) {
+  const int ctas = (int)(grid.x * grid.y), chunks = K / kGK;
+  int z = 1;
+  while (ctas * z < 2 * n_sm && chunks / (2 * z) >= 4) z *= 2;
+  return z;
 }
 
 // Every kernel of one frame, in stream order on `s` (captured into the graph).
@@ -805,7 +838,8 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
         a.ss = b.ss + (size_t)(2 * l) * R;
         a.out = b.qkv;
         a.ld = p.qkv_dim;
-        batch_gemm_kernel<BSRC_NORM, EPI_QKV><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+        batch_gemm_kernel<BSRC_NORM_HILO, EPI_QKV>
+            <<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmemHilo, s>>>(a);
       }
       batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);
       {   // Wo + residual
@@ -816,8 +850,9 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
         a.ldx = p.NH * p.D;
         a.out = b.X;
         a.ld = H;
-        a.ss_out = b.ss + (size_t)(2 * l + 1) * R;
-        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+        const dim3 grid(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN);
+        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(grid.x, grid.y, split_k(grid, a.g.K, p.n_cta)), blk, kGemmSmem, s>>>(a);
+        batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 1) * R, b.info);
       }
       {   // RMSNorm -> gate/up -> SwiGLU
         GemmArgs a = gemm_args(p, b);
@@ -839,8 +874,9 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
         a.ldx = p.F;
         a.out = b.X;
         a.ld = H;
-        a.ss_out = b.ss + (size_t)(2 * l + 2) * R;
-        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN), blk, kGemmSmem, s>>>(a);
+        const dim3 grid(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN);
+        batch_gemm_kernel<BSRC_BF16, EPI_RESID><<<dim3(grid.x, grid.y, split_k(grid, a.g.K, p.n_cta)), blk, kGemmSmem, s>>>(a);
+        batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 2) * R, b.info);
       }
     }
     {   // final RMSNorm -> LM heads, one grid slice per head
@@ -853,8 +889,8 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       a.ss = b.ss + (size_t)(2 * L) * R;
       a.logits = b.logits;
       a.head_bias = p.head_bias;
-      batch_gemm_kernel<BSRC_NORM, EPI_HEADS>
-          <<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN, p.P), blk, kGemmSmem, s>>>(a);
+      batch_gemm_kernel<BSRC_NORM_HILO, EPI_HEADS>
+          <<<dim3(a.g.M / kGM + (a.g.M % kGM != 0), R / kGN, p.P), blk, kGemmSmemHilo, s>>>(a);
     }
     batch_topk_kernel<<<R * (p.K + 1), kConsumerThreads, 0, s>>>(p, b, call);
     batch_accept_kernel<<<bs->max_streams, kConsumerThreads, 0, s>>>(p, b, call);
