@@ -34,10 +34,12 @@ constexpr int kGStages = 4;
 constexpr int kGBStride = kGK + 8;       // bf16 per staged operand row (144 B: conflict-free ldmatrix)
 constexpr int kGAStage = 32 * 512;       // 8 m-tiles x 4 k-tiles of 512 B
 constexpr int kGBStage = kGN * kGBStride * 2;
+constexpr int kGStagesHilo = 3;          // with the hi + lo operand: two CTAs per SM still fit
 constexpr int kGemmSmem = kGStages * (kGAStage + kGBStage);
-constexpr int kGemmSmemHilo = kGStages * (kGAStage + 2 * kGBStage);   // B as a bf16 hi + lo pair
+constexpr int kGemmSmemHilo = kGStagesHilo * (kGAStage + 2 * kGBStage);
 constexpr int kRecSlots = kMaxDraft + 1;   // distributions per packed row (verify + drafts)
 constexpr int kBatchQVec = 16;             // query vectors per attention CTA: rows x (q heads per KV head)
+constexpr int kBatchKeys = 16;             // keys of a frame: positions 0..15 (c15 is never fed)
 
 // Operand rows: fp32 rows normalised while staged (as one bf16, or as a bf16 hi + lo pair
 // carrying about 16 mantissa bits, for the QKV and LM-head products whose errors the
@@ -253,6 +255,7 @@ struct GemmArgs {
 template <int BSRC, int EPI>
 __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__ GemmArgs a) {
   constexpr bool kNorm = BSRC != BSRC_BF16, kHilo = BSRC == BSRC_NORM_HILO;
+  constexpr int kStages = kHilo ? kGStagesHilo : kGStages;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int s_row[kGN];
   __shared__ int s_j[kGN];
@@ -306,8 +309,8 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
   }
   __syncthreads();
   uint8_t* sA = smem;
-  uint16_t* sB = reinterpret_cast<uint16_t*>(smem + kGStages * kGAStage);
-  uint16_t* sBl = sB + (size_t)kGStages * kGN * kGBStride;   // lo parts (hi/lo operand)
+  uint16_t* sB = reinterpret_cast<uint16_t*>(smem + kStages * kGAStage);
+  uint16_t* sBl = sB + (size_t)kStages * kGN * kGBStride;   // lo parts (hi/lo operand)
 
   // ---- stage loaders ------------------------------------------------------------------------
   auto load_A = [&](int kc, int st) {
@@ -371,7 +374,7 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
       for (int e = 0; e < 4; ++e) acc[i][j][e] = 0.f;
 
 #pragma unroll
-  for (int st = 0; st < kGStages - 1; ++st) {
+  for (int st = 0; st < kStages - 1; ++st) {
     if (st < n_kc) {
       load_A(kc0 + st, st);
       if (!kNorm) {
@@ -384,10 +387,10 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
     cp_async_commit();
   }
   for (int it = 0; it < n_kc; ++it) {
-    const int st = it % kGStages;
-    const int nk = it + kGStages - 1;
+    const int st = it % kStages;
+    const int nk = it + kStages - 1;
     if (kNorm && nk < n_kc) fetch_B(kc0 + nk);
-    cp_async_wait<kGStages - 2>();
+    cp_async_wait<kStages - 2>();
     __syncthreads();
     const uint8_t* A = sA + st * kGAStage;
     const uint16_t* B = sB + (size_t)st * (kGN * kGBStride);
@@ -415,9 +418,9 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
         }
       }
     }
-    // stage nk % kGStages was last read in iteration it - 1, which every warp has left
+    // stage nk % kStages was last read in iteration it - 1, which every warp has left
     if (nk < n_kc) {
-      const int sn = nk % kGStages;
+      const int sn = nk % kStages;
       load_A(kc0 + nk, sn);
       if (!kNorm)
         load_B16(kc0 + nk, sn);
@@ -501,9 +504,9 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
   const int D = p.D, half = D >> 1, group = p.NH / p.NKV, nq = nr * group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   __shared__ float qs[kBatchQVec][132];        // nr x group query vectors
-  __shared__ float ks[kMaxPos][132];
-  __shared__ float vs[kMaxPos][128];
-  __shared__ float sc[kBatchQVec][kMaxPos];
+  __shared__ float ks[kBatchKeys][132];
+  __shared__ float vs[kBatchKeys][128];
+  __shared__ float sc[kBatchQVec][kBatchKeys];
   const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
   const int nk = pos0 + nr;
   // loads: queries, new keys / values, cached keys / values
