@@ -223,6 +223,12 @@ __device__ __forceinline__ uint32_t ld_acquire(const unsigned* p) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+// Release-ordered add at GPU scope: every write that precedes it in this thread, or in the
+// CTA's threads before a CTA barrier this thread passed, is visible to a thread that reads
+// the new value with an acquire load.
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 __device__ __forceinline__ uint64_t globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -202,10 +202,7 @@ __device__ __forceinline__ bool cons_wait(Cons& c, const unsigned* ctr, unsigned
 __device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call, int slot) {
   consumer_sync();
   timeline_max(c, call, slot);
-  if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(ctr, 1u);
-  }
+  if (threadIdx.x == 0) red_release_add(ctr, 1u);
   timeline_max(c, call, slot + 1);
 }
 
