@@ -17,7 +17,8 @@ Modules:
   frame        autoregressive and speculative frame procedures.
   codedecoder  the outer CodeDecoder (one call per frame, emits c0) and the full frame
                pipeline of Fig. 1 (prompt prefill, c0, MultiCodeDecoder, input sum).
-  enumeration  exact output distributions of both procedures (losslessness pin).
+  tree         sparse tree drafting and verification (Fig. 2) and the greedy tree growth.
+  enumeration  exact output distributions of the procedures (losslessness pin).
   accounting   the paper's real-time call arithmetic.
 
 Parity status: every function here is pinned by a `-m "not gpu"` test

@@ -158,3 +158,83 @@ def spec_distribution(pm: PrefixModel, n_pos: int, draft_len: int):
 def alpha(p: Dist, q: Dist) -> Fraction:
     """Acceptance probability of one draft: sum_x min(p(x), q(x))."""
     return sum((min(p.frac(x), q.frac(x)) for x in set(p.ids) | set(q.ids)), Fraction(0))
+
+
+def tree_distribution(pm: PrefixModel, n_pos: int, tree, m_need=None):
+    """(law of c1..c_P, expected calls) of tree-drafted decoding (oracle.tree, R-T1..R-T5),
+    written with probabilities: at a node with target p and candidates x_1, x_2, .. (the
+    node's children in rank order), test i keeps x_i with probability p(x_i) / (1 - sum of
+    p over the candidates rejected before it); when none is kept a code is drawn from p
+    restricted to the rejected candidates' complement, renormalised."""
+    from .tree import ranked                               # the candidate ranking (R-T2)
+    K = tree.max_depth
+    m_need = tree.ranks_needed() if m_need is None else m_need
+    memo: Dict[Tuple[int, ...], Tuple[Dict[Tuple[int, ...], Fraction], Fraction]] = {}
+
+    def cands(prefix):
+        a = len(prefix)
+        h = pm.state(prefix[:-1])[1]
+        out = []
+        for d in range(1, min(K, n_pos - a) + 1):
+            z = to_f32(pm.m.draft_logits(a, d, h))
+            out.append(ranked(z, m_need[d - 1]))
+        return out
+
+    def from_state(prefix):
+        if prefix in memo:
+            return memo[prefix]
+        a = len(prefix)
+        if a == n_pos:
+            memo[prefix] = ({(): Fraction(1)}, Fraction(0))
+            return memo[prefix]
+        cand = cands(prefix)
+        res: Dict[Tuple[int, ...], Fraction] = defaultdict(Fraction)
+        calls = [Fraction(1)]
+
+        def visit(node, cur, pr):
+            """Walk at `node` (-1: the call's first row) with codes `cur` emitted so far."""
+            p = pm.target(cur)
+            s = len(cur) + 1
+            left = Fraction(1)
+            rejected = []
+            for ch in tree.children(node):
+                if a + tree.depth[ch] > n_pos:
+                    continue
+                x = cand[tree.depth[ch] - 1][tree.rank[ch]]
+                keep = p.frac(x) / left if left > 0 else Fraction(0)
+                if keep > 0:
+                    if s == n_pos:
+                        res[cur[a:] + (x,)] += pr * keep
+                    else:
+                        visit(ch, cur + (x,), pr * keep)
+                pr *= 1 - keep
+                left -= p.frac(x)
+                rejected.append(x)
+                if pr == 0:
+                    return
+            if s > n_pos:
+                res[cur[a:]] += pr
+                return
+            for x in p.ids:
+                if x in rejected or p.frac(x) == 0:
+                    continue
+                w = pr * p.frac(x) / left
+                sub_law, sub_calls = from_state(cur + (x,))
+                for tail, pv in sub_law.items():
+                    res[cur[a:] + (x,) + tail] += w * pv
+                calls[0] += w * sub_calls
+
+        visit(-1, prefix, Fraction(1))
+        # a walk that ended by keeping the last position's code finishes the frame
+        memo[prefix] = (dict(res), calls[0])
+        return memo[prefix]
+
+    p1 = pm.target(())
+    law: Dict[Tuple[int, ...], Fraction] = defaultdict(Fraction)
+    calls = Fraction(1)
+    for x in p1.ids:
+        sub_law, sub_calls = from_state((x,))
+        for tail, pv in sub_law.items():
+            law[(x,) + tail] += p1.frac(x) * pv
+        calls += p1.frac(x) * sub_calls
+    return dict(law), calls
