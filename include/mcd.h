@@ -58,7 +58,7 @@ typedef enum {
 } mcd_status;
 
 enum { MCD_WEIGHT_F32 = 0, MCD_WEIGHT_BF16 = 1 };
-enum { MCD_DRAFT_SAMPLE = 0, MCD_DRAFT_GREEDY = 1, MCD_DRAFT_NOISY_TARGET = 2 };
+enum { MCD_DRAFT_SAMPLE = 0, MCD_DRAFT_GREEDY = 1, MCD_DRAFT_NOISY_TARGET = 2, MCD_DRAFT_TREE = 3 };
 
 /* Model and sampling configuration.  Limits: hidden, ffn multiples of 128; head_dim 64
  * or 128; n_q_heads multiple of n_kv_heads; vocab multiple of 16 and <= 4096;
@@ -78,11 +78,16 @@ typedef struct {
                          * GREEDY = its argmax, NOISY_TARGET = controlled-acceptance drafts:
                          * q for position s is the target's own fp32 logits of s given the
                          * drafted prefix (one extra one-row pass per draft, run inside the
-                         * same frame launch) plus noise_sigma * N(0,1) per entry            */
+                         * same frame launch) plus noise_sigma * N(0,1) per entry,
+                         * TREE = sparse tree of top-m candidates per drafted position
+                         * (mcd_set_tree; Sec. 2.2 and Fig. 2), verified in one call       */
   float noise_sigma;    /* MCD_DRAFT_NOISY_TARGET only (>= 0)                            */
   uint64_t seed;        /* Philox key                                                    */
-  int32_t max_streams;  /* streams one mcd_decode_frames call may decode together (1..8;
-                         * max_streams * max(K + 1, 2) <= 32; NOISY_TARGET needs 1)      */
+  int32_t max_streams;  /* streams one mcd_decode_frames call may decode together (1..128).
+                         * Up to 8 streams and 32 packed rows (streams x max(K + 1, 2)) a
+                         * frame is one persistent-kernel launch; beyond that calls run on
+                         * the batched GEMM path (bf16 weights, <= 512 packed rows, one
+                         * CUDA graph launch per frame).  NOISY_TARGET and TREE need 1     */
 } mcd_config;
 
 /* Per-frame counters written by the device (device memory, caller-owned). */
@@ -247,9 +252,39 @@ mcd_status mcd_topk_softmax_static(int32_t n_rows, int32_t vocab, int32_t top_k,
 /* Tracing for parity tests: while `trace` (dev, mcd_trace_bytes() bytes) is set, frame
  * decoding writes one mcd_call_trace per call followed, after 16 records, by float
  * logits [16 calls][8 rows][vocab] (verify rows) and [16 calls][8 drafts][vocab] (the
- * draft rows used).  NULL turns tracing off. */
+ * draft rows used).  In TREE mode the block continues with 16 mcd_tree_trace records and
+ * the verify logits of every row, [16 calls][32 rows][vocab].  NULL turns tracing off. */
 int64_t mcd_trace_bytes(const mcd_ctx* ctx);
 mcd_status mcd_set_trace(mcd_ctx* ctx, void* trace);
+
+/* Per-call record of TREE mode (after the mcd_call_trace records; see mcd_set_trace). */
+typedef struct {
+  int32_t n_rows;         /* rows fed: row 0 = the last emitted code, then tree nodes     */
+  int32_t row_node[32];   /* tree node of each row (-1: row 0)                            */
+  int32_t row_id[32];     /* code fed at each row                                         */
+  int32_t path_len;       /* nodes kept                                                   */
+  int32_t path[8];        /* kept nodes, root first                                       */
+  int32_t draft_row;      /* row whose draft logits gave the next call's candidates       */
+  int32_t n_next;         /* candidate depths of the next call                            */
+  int32_t next_cand[8][8];/* [depth - 1][rank] candidate ids of the next call             */
+  int32_t reserved[20];
+} mcd_tree_trace;
+
+/* Sparse tree of TREE mode (Sec. 2.2 "Tree attention ...", Fig. 2): n_nodes <= 31 nodes
+ * in breadth-first order (host arrays); node i has parent[i] (-1: a child of the call's
+ * first row, else an earlier node) and rank[i] < 8 (distinct among siblings), depth =
+ * parent's depth + 1 <= draft_len.  A node of depth d proposes the id of rank rank[i] in
+ * the draft logits of depth d (fp32 logit descending, id ascending) of the row whose LM
+ * head emitted the call's last code; rows attend to the committed prefix, the call's
+ * first row, their ancestors and themselves.  Verification walks from the first row: the
+ * children of a node are tested in rank order, test i keeping its candidate x with
+ * probability p'(x), p' being the node's distribution without the candidates already
+ * rejected there (uniform of counter (call, code position, purpose 1 for i = 0, else
+ * 0x10000 + i)); when none is kept, or the node has no children, a code is drawn from p'
+ * with purpose 0.  The kept nodes' keys and values become the committed cache.  Until
+ * set, the tree is the chain of draft_len rank-0 nodes.  Errors: MCD_ERR_INVALID_ARG
+ * (malformed tree), MCD_ERR_STATE (context not in TREE mode). */
+mcd_status mcd_set_tree(mcd_ctx* ctx, int32_t n_nodes, const int32_t* parent, const int32_t* rank);
 
 /* Profiling hook: while `timeline` (dev, uint64 [16 calls][128], zeroed by the caller)
  * is set, frame decoding writes %globaltimer stamps (ns) per call: slot 0 call start;

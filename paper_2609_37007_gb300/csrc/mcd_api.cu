@@ -326,7 +326,8 @@ static mcd_status validate_config(const mcd_config& c) {
   if (c.top_k < 1 || c.top_k > kMaxTopK || c.top_k > c.vocab) return MCD_ERR_UNSUPPORTED;
   if (!(c.temperature > 0.f) || !(c.rms_eps > 0.f) || !(c.rope_base > 1.f)) return MCD_ERR_INVALID_ARG;
   if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
-  if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_NOISY_TARGET) return MCD_ERR_INVALID_ARG;
+  if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_TREE) return MCD_ERR_INVALID_ARG;
+  if (c.draft_mode == MCD_DRAFT_TREE && (c.max_streams != 1 || c.draft_len < 1)) return MCD_ERR_UNSUPPORTED;
   if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
   if (c.max_streams < 1 || c.max_streams > kMaxBatchStreams) return MCD_ERR_UNSUPPORTED;
   if (c.max_streams > 1 && c.draft_mode == MCD_DRAFT_NOISY_TARGET) return MCD_ERR_UNSUPPORTED;
@@ -413,6 +414,8 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.wait_ns = 2000000000ull;  // 2 s
   p.S = 1;
   p.trace_stride = (long long)sizeof(mcd_call_trace) * kMaxCalls + (long long)2 * kMaxCalls * kMaxRows * p.V * 4;
+  if (k.draft_mode == MCD_DRAFT_TREE)   // + the tree records and every row's verify logits
+    p.trace_stride += (long long)sizeof(mcd_tree_trace) * kMaxCalls + (long long)kMaxCalls * kMaxCols * p.V * 4;
   const char* wn = getenv("MCD_WAIT_NS");
   if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
 
@@ -462,7 +465,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.attn, sizeof(float) * kMaxCols * p.NH * p.D)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxCols * (kMaxDraft + 1) * p.V)) != cudaSuccess)
     return fail(cuda_status(e));
-  p.kv_stride = (long long)p.L * p.NKV * kMaxPos * p.D;
+  p.kv_stride = (long long)p.L * p.NKV * kKVSlots * p.D;
   const size_t kvsz = sizeof(float) * (size_t)p.kv_stride * k.max_streams;
   if ((e = ctx_alloc(c, &p.kcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.vcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
@@ -473,6 +476,18 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxSlots * p.ctr_stride)) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &p.tree_cand, sizeof(int) * kMaxDraft * kMaxTreeRank)) != cudaSuccess)
+    return fail(cuda_status(e));
+  if (k.draft_mode == MCD_DRAFT_TREE) {       // until mcd_set_tree: the chain of K rank-0 nodes
+    p.tree_n = k.draft_len;
+    p.tree_maxd = k.draft_len;
+    for (int i = 0; i < k.draft_len; ++i) {
+      p.tree_parent[i] = (signed char)(i - 1);
+      p.tree_rank[i] = 0;
+      p.tree_depth[i] = (signed char)(i + 1);
+      p.tree_m[i] = 1;
+    }
+  }
   if ((e = ctx_alloc(c, &c->host_stage, host_stage_bytes(p))) != cudaSuccess) return fail(cuda_status(e));
   if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -695,9 +710,37 @@ mcd_status mcd_decode_frame_host(mcd_ctx* c, uint32_t stream_id, uint32_t frame_
   return mcd_sync(c);
 }
 
+mcd_status mcd_set_tree(mcd_ctx* c, int32_t n_nodes, const int32_t* parent, const int32_t* rank) {
+  if (!c) return MCD_ERR_INVALID_ARG;
+  FrameParams& p = c->fp;
+  if (p.draft_mode != MCD_DRAFT_TREE) return MCD_ERR_STATE;
+  if (n_nodes < 1 || n_nodes > kMaxTree || !parent || !rank) return MCD_ERR_INVALID_ARG;
+  int depth[kMaxTree], m[kMaxDraft] = {0}, maxd = 0;
+  for (int i = 0; i < n_nodes; ++i) {
+    if (parent[i] < -1 || parent[i] >= i || rank[i] < 0 || rank[i] >= kMaxTreeRank) return MCD_ERR_INVALID_ARG;
+    depth[i] = parent[i] < 0 ? 1 : depth[parent[i]] + 1;
+    if (depth[i] > p.K || rank[i] >= p.top_k) return MCD_ERR_INVALID_ARG;
+    if (i > 0 && depth[i] < depth[i - 1]) return MCD_ERR_INVALID_ARG;       // breadth-first order
+    for (int j = 0; j < i; ++j)
+      if (parent[j] == parent[i] && rank[j] == rank[i]) return MCD_ERR_INVALID_ARG;
+    m[depth[i] - 1] = std::max(m[depth[i] - 1], rank[i] + 1);
+    maxd = std::max(maxd, depth[i]);
+  }
+  p.tree_n = n_nodes;
+  p.tree_maxd = maxd;
+  for (int i = 0; i < n_nodes; ++i) {
+    p.tree_parent[i] = (signed char)parent[i];
+    p.tree_rank[i] = (signed char)rank[i];
+    p.tree_depth[i] = (signed char)depth[i];
+  }
+  for (int d = 0; d < kMaxDraft; ++d) p.tree_m[d] = m[d];
+  return MCD_OK;
+}
+
 mcd_status mcd_begin_frame(mcd_ctx* c, uint32_t stream_id, uint32_t frame_idx, const float* cond, const int32_t* c0,
                            const float* c0_emb) {
   if (!c) return MCD_ERR_INVALID_ARG;
+  if (c->fp.draft_mode == MCD_DRAFT_TREE) return MCD_ERR_UNSUPPORTED;   // stepwise calls are chain-only
   return launch_begin(c, 1, &stream_id, &frame_idx, cond, c0, c0_emb);
 }
 

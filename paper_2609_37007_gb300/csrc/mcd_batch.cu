@@ -507,7 +507,7 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
   __shared__ float ks[kBatchKeys][132];
   __shared__ float vs[kBatchKeys][128];
   __shared__ float sc[kBatchQVec][kBatchKeys];
-  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
   const int nk = pos0 + nr;
   // loads: queries, new keys / values, cached keys / values
   for (int i = tid; i < nq * D; i += blockDim.x) {
@@ -664,6 +664,7 @@ __global__ void __launch_bounds__(kConsumerThreads) batch_accept_kernel(FramePar
     st->n_d = n_next;
     st->pos0 = a_new + 1;
     st->n_rows = min(n_next + 1, p.P - a_new);
+    st->top_pos = st->pos0 + st->n_rows - 1;
     st->round = call + 1;
     st->first_head_row = 0;
     st->calls = calls;

@@ -23,17 +23,16 @@
 
 namespace mcd {
 
-// LM heads a pass reads.  Verify call: P_lo = a+1 up to the last row's position plus K
-// (its draft heads), or up to the last row's position when the drafts come from
-// noisy-target passes.  Noisy-target pass (one row at position s): head s only.
-__device__ __forceinline__ void head_range(const FrameParams& p, int a, int pos0, int n_rows, int emu, int& p_lo,
-                                           int& p_hi) {
+// LM heads a pass reads, from the largest row position `top` of the pass.  Verify call:
+// P_lo = a+1 up to top plus K (its draft heads), or up to top when the drafts come from
+// noisy-target passes.  Noisy-target pass (one row at position top): head top only.
+__device__ __forceinline__ void head_range(const FrameParams& p, int a, int top, int emu, int& p_lo, int& p_hi) {
   if (emu) {
-    p_lo = p_hi = pos0;
+    p_lo = p_hi = top;
     return;
   }
   p_lo = a + 1;
-  p_hi = p.draft_mode == MCD_DRAFT_NOISY_TARGET ? pos0 + n_rows - 1 : min(p.P, pos0 + n_rows - 1 + p.K);
+  p_hi = p.draft_mode == MCD_DRAFT_NOISY_TARGET ? top : min(p.P, top + p.K);
 }
 
 // LM heads one call streams: the union over the streams with rows in the call, as a bit
@@ -44,7 +43,7 @@ __device__ __forceinline__ unsigned call_heads_mask(const FrameParams& p) {
     const DevState* st = p.st + s;
     if (__ldcg(&st->done)) continue;
     int lo, hi;
-    head_range(p, __ldcg(&st->a), __ldcg(&st->pos0), __ldcg(&st->n_rows), __ldcg(&st->emu), lo, hi);
+    head_range(p, __ldcg(&st->a), __ldcg(&st->top_pos), __ldcg(&st->emu), lo, hi);
     for (int P = lo; P <= hi; ++P) mask |= 1u << P;
   }
   return mask;
@@ -127,7 +126,7 @@ __device__ void attention_stream(Cons& c, int layer, int h, bool write_kv, int n
   float2* cs = reinterpret_cast<float2*>(vs + kAttnPos * 128);  // [8][D/2] (cos, sin)
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
   float* gk = gq + 128;                                          // [D]
-  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kMaxPos * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
   const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
   // ---- (A) loads ----------------------------------------------------------------------
@@ -301,6 +300,186 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   }
 }
 
+// Attention of query head h for rows lo..hi-1 of a tree call (one stream, packed rows from
+// 0).  Keys: the committed positions 0..pos0-1 (cache slots) and the call's rows 0..hi-1,
+// row n seeing row m iff bit m of r_anc[n]; each row is rotated at its own position r_pos
+// (row 0 at pos0, a node of depth d at pos0 + d).  The task of a KV head's first query head
+// stores K / V of rows lo..hi-1: row 0 at its position, node rows at slot kMaxPos + n until
+// the acceptance step commits the kept ones.  Outputs go to p.attn.  Scratch (act + bfrag,
+// 62 KB): k [48][D + 8], v [48][D], q [8][D + 8], RoPE rows by depth [9][D/2], QK-norm
+// gains, scores [8][48].
+__device__ void attention_tree_task(Cons& c, int layer, int h, int lo, int hi, int pos0) {
+  const FrameParams& p = c.p;
+  const CallInfo* ci = c.sm.ci;
+  const int D = p.D, half = D >> 1, group = p.NH / p.NKV, g = h / group;
+  const bool write_kv = (h % group) == 0;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cs_shift = D == 128 ? 5 : 4, cpr = 1 << cs_shift;   // 16-byte chunks per row
+  const int KS = D + 8;
+  constexpr int kKeys = 48, kDepths = 9;
+  float* ks = c.sm.act;
+  float* vs = ks + kKeys * 136;
+  float* qs = vs + kKeys * 128;
+  float2* cs = reinterpret_cast<float2*>(qs + 8 * 136);
+  float* gq = reinterpret_cast<float*>(cs + kDepths * 64);
+  float* gk = gq + 128;
+  float* sc = gk + 128;
+  const size_t cache_off = ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  const float* qkv = p.qkv;
+  const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
+  const int nq = hi - lo, nk = pos0 + hi;
+  const int dmax = ci->r_pos[hi - 1] - pos0;       // rows are in tree order: depth nondecreasing
+  // ---- (A) loads, 16-byte chunks, batches of 8 per thread in flight --------------------------
+  {
+    const int e_q = nq << cs_shift, e_k = e_q + (hi << cs_shift), e_v = e_k + (hi << cs_shift);
+    const int e_kc = e_v + (pos0 << cs_shift), e_vc = e_kc + (pos0 << cs_shift);
+    const int e_cs = e_vc + ((dmax + 1) << cs_shift), e_g = e_cs + (p.qk_norm ? 2 * cpr : 0);
+    for (int base = 0; base < e_g; base += 8 * kConsumerThreads) {
+      float4 v[8];
+      float4* dst[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = base + tid + u * kConsumerThreads;
+        dst[u] = nullptr;
+        if (i >= e_g) continue;
+        const float4* src;
+        const int ch = i & (cpr - 1);
+        if (i < e_q) {
+          const int n = lo + (i >> cs_shift);
+          src = reinterpret_cast<const float4*>(qkv + (size_t)n * p.qkv_dim + qoff);
+          dst[u] = reinterpret_cast<float4*>(qs + (n - lo) * KS) + ch;
+        } else if (i < e_v) {
+          const bool isv = i >= e_k;
+          const int n = (i - (isv ? e_k : e_q)) >> cs_shift;
+          src = reinterpret_cast<const float4*>(qkv + (size_t)n * p.qkv_dim + (isv ? voff : koff));
+          dst[u] = reinterpret_cast<float4*>(isv ? vs + (pos0 + n) * D : ks + (pos0 + n) * KS) + ch;
+        } else if (i < e_vc) {
+          const bool isv = i >= e_kc;
+          const int j = (i - (isv ? e_kc : e_v)) >> cs_shift;
+          src = reinterpret_cast<const float4*>((isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D);
+          dst[u] = reinterpret_cast<float4*>(isv ? vs + j * D : ks + j * KS) + ch;
+        } else if (i < e_cs) {
+          const int d = (i - e_vc) >> cs_shift;
+          src = reinterpret_cast<const float4*>(p.rope + (size_t)(pos0 + d) * half);
+          dst[u] = reinterpret_cast<float4*>(cs + d * 64) + ch;
+        } else {
+          const int w = (i - e_cs) >> cs_shift;
+          src = reinterpret_cast<const float4*>((w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D);
+          dst[u] = reinterpret_cast<float4*>(w == 0 ? gq : gk) + ch;
+        }
+        v[u] = __ldcg(src + ch);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (dst[u]) *dst[u] = v[u];
+    }
+  }
+  consumer_sync();
+  // ---- (B) QK-norm + RoPE of the queries and the new keys; K / V of rows lo..hi-1 stored ------
+  const int nd = D >> 5;
+  for (int vi = warp; vi < nq + hi; vi += kConsumerWarps) {
+    const bool isq = vi < nq;
+    const int n = isq ? lo + vi : vi - nq;
+    float* row = isq ? qs + (n - lo) * KS : ks + (pos0 + n) * KS;
+    const int depth = ci->r_pos[n] - pos0;
+    float x[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = i < nd ? row[lane + 32 * i] : 0.f;
+    if (p.qk_norm) {
+      float ss = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ss += x[i] * x[i];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+      const float scl = rsqrtf(ss / (float)D + p.eps);
+      const float* gg = isq ? gq : gk;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) x[i] = x[i] * scl * gg[lane + 32 * i];
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if (i < nd / 2) {
+        const float2 r = cs[depth * 64 + lane + 32 * i];
+        const float a0 = x[i], b0 = x[i + nd / 2];
+        x[i] = a0 * r.x - b0 * r.y;
+        x[i + nd / 2] = b0 * r.x + a0 * r.y;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < nd) row[lane + 32 * i] = x[i];
+    if (!isq && write_kv && n >= lo) {
+      const int slot = n == 0 ? pos0 : kMaxPos + n;
+      float* kd = p.kcache + cache_off + (size_t)slot * D;
+      float* vd = p.vcache + cache_off + (size_t)slot * D;
+      const float* vrow = vs + (pos0 + n) * D;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) {
+          kd[lane + 32 * i] = x[i];
+          vd[lane + 32 * i] = vrow[lane + 32 * i];
+        }
+    }
+  }
+  consumer_sync();
+  // ---- (C1) scores: two threads per (query, key) over interleaved chunks ----------------------
+  {
+    const float scale = rsqrtf((float)D);
+    for (int t = tid; t < nq * kKeys * 2; t += kConsumerThreads) {
+      const int qi = t / (2 * kKeys), j = (t >> 1) % kKeys, hf = t & 1;
+      const int n = lo + qi;
+      const bool live = j < nk && (j < pos0 || ((ci->r_anc[n] >> (j - pos0)) & 1u));
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+      if (live) {
+        const float4* q4 = reinterpret_cast<const float4*>(qs + qi * KS) + hf;
+        const float4* k4 = reinterpret_cast<const float4*>(ks + j * KS) + hf;
+#pragma unroll 8
+        for (int ch = 0; ch < (cpr >> 1); ++ch) {
+          const float4 q = q4[2 * ch], k = k4[2 * ch];
+          a0 += q.x * k.x;
+          a1 += q.y * k.y;
+          a2 += q.z * k.z;
+          a3 += q.w * k.w;
+        }
+      }
+      float acc = (a0 + a1) + (a2 + a3);
+      acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
+      if (hf == 0) sc[qi * kKeys + j] = live ? acc * scale : -INFINITY;
+    }
+  }
+  consumer_sync();
+  // ---- (C2) softmax: one warp per query, keys lane and lane + 32 ---------------------------------
+  for (int qi = warp; qi < nq; qi += kConsumerWarps) {
+    const float s0 = sc[qi * kKeys + lane];
+    const float s1 = lane + 32 < kKeys ? sc[qi * kKeys + lane + 32] : -INFINITY;
+    float m = fmaxf(s0, s1);
+#pragma unroll
+    for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
+    const float e0 = s0 == -INFINITY ? 0.f : __expf(s0 - m), e1 = s1 == -INFINITY ? 0.f : __expf(s1 - m);
+    float l = e0 + e1;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, off);
+    sc[qi * kKeys + lane] = e0 / l;
+    if (lane + 32 < kKeys) sc[qi * kKeys + lane + 32] = e1 / l;
+  }
+  consumer_sync();
+  // ---- (C3) o = sum_j p_j v_j over keys up to the row itself (ancestors precede it) ------------
+  for (int t = tid; t < nq * half; t += kConsumerThreads) {
+    const int qi = t / half, d = 2 * (t - qi * half), n = lo + qi, npos = pos0 + n + 1;
+    const float* pr = sc + qi * kKeys;
+    float2 acc = make_float2(0.f, 0.f);
+    for (int j = 0; j < npos; ++j) {
+      const float w = pr[j];
+      const float2 v = *reinterpret_cast<const float2*>(vs + j * D + d);
+      acc.x += w * v.x;
+      acc.y += w * v.y;
+    }
+    *reinterpret_cast<float2*>(p.attn + (size_t)n * p.NH * D + h * D + d) = acc;
+  }
+  consumer_sync();
+}
+
 // ------------------------------------------------------------------------------------
 // One call
 // ------------------------------------------------------------------------------------
@@ -357,17 +536,24 @@ __device__ void run_call(Cons& c, int call) {
     // Wo reads them.
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
     if (WIDE) {
-      const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
-      for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
-        const int i = t / p.NH, h = t - i * p.NH, s = ci->act[i];
-        const int nr = ci->st[s].n_rows, base = ci->base[s];
-        attention_stream(c, l, h, (h % group) == 0, nr, ci->st[s].pos0, base, s);
-        for (int q = threadIdx.x; q < nr * (D >> 2); q += kConsumerThreads) {
-          const int n = q / (D >> 2), d4 = q - n * (D >> 2);
-          reinterpret_cast<float4*>(p.attn + (size_t)(base + n) * p.NH * D + h * D)[d4] =
-              reinterpret_cast<const float4*>(sm.act + (base + n) * D)[d4];
+      if (p.draft_mode == MCD_DRAFT_TREE && ci->st[0].pos0 > 0) {
+        // tree call (one stream): one task per (query head, group of 8 rows)
+        const int nr = ci->M, n_rg = (nr + 7) >> 3;
+        for (int t = blockIdx.x; t < p.NH * n_rg; t += p.n_cta)
+          attention_tree_task(c, l, t % p.NH, 8 * (t / p.NH), min(8 * (t / p.NH) + 8, nr), ci->st[0].pos0);
+      } else {
+        const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
+        for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
+          const int i = t / p.NH, h = t - i * p.NH, s = ci->act[i];
+          const int nr = ci->st[s].n_rows, base = ci->base[s];
+          attention_stream(c, l, h, (h % group) == 0, nr, ci->st[s].pos0, base, s);
+          for (int q = threadIdx.x; q < nr * (D >> 2); q += kConsumerThreads) {
+            const int n = q / (D >> 2), d4 = q - n * (D >> 2);
+            reinterpret_cast<float4*>(p.attn + (size_t)(base + n) * p.NH * D + h * D)[d4] =
+                reinterpret_cast<const float4*>(sm.act + (base + n) * D)[d4];
+          }
+          consumer_sync();
         }
-        consumer_sync();
       }
       cons_signal(c, ctr + ctr_att(L, l), call, kTimelineSlots);
       if (!cons_wait(c, ctr + ctr_att(L, l), N)) return;
@@ -718,6 +904,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
       st->n_d = 0;
       st->pos0 = a_new + 1;
       st->n_rows = 1;
+      st->top_pos = a_new + 1;
       st->emu = 1;
       st->emu_n = n_next;
       st->emu_in = s_emit[s_nemit - 1];
@@ -725,6 +912,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
       st->n_d = n_next;
       st->pos0 = a_new + 1;
       st->n_rows = min(n_next + 1, p.P - a_new);
+      st->top_pos = st->pos0 + st->n_rows - 1;
       st->round = round + 1;
     }
     st->first_head_row = 0;
@@ -805,6 +993,237 @@ __device__ void accept_step(Cons& c, int call, int s) {
   }
 }
 
+// Acceptance step of a tree call (one stream; run by the CTA that finished top-k last).
+// One warp walks the tree from the first row: the children of the current node are tested
+// in rank order, test i keeping its candidate x iff U * S' < 2^53 * W_x, S' being the
+// node's weight sum without the candidates rejected so far (one-hot draft distributions);
+// a kept child continues the walk, otherwise a code is drawn from the remainder (purpose 0)
+// and the call ends.  Then: the next call's candidates (the top-m ids by logit of each
+// draft distribution of the last visited row), the kept nodes' K / V moved to their
+// positions, the state update, the trace and the release of the next call.
+__device__ void accept_tree(Cons& c, int call) {
+  const FrameParams& p = c.p;
+  Smem& sm = c.sm;
+  const CallInfo* ci = sm.ci;
+  const DevState& st0 = ci->st[0];
+  const int a = st0.a, pos0 = st0.pos0, n_rows = st0.n_rows, round = st0.round;
+  const unsigned sid = p.stream_ids[0], fid = p.frame_ids[0];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1);
+  __shared__ int t_emit[kMaxDraft + 1], t_path[kMaxDraft + 1], t_path_row[kMaxDraft + 1], t_res[4];
+  __shared__ int t_next[kMaxDraft][kMaxTreeRank];
+  if (warp == 0) {
+    int node = -1, row = st0.first_head_row, n_emit = 0, plen = 0, tests = 0;
+    while (true) {
+      const int s = a + 1 + plen;                     // code position of the node's children
+      const TopkRec* pr = cur + (size_t)row * (kMaxDraft + 1);
+      unsigned long long S_rem = pr->S;
+      int rej[kMaxTreeRank];
+      int n_rej = 0, kept = -1, kx = -1;
+      if (pos0 > 0) {
+        for (int r = 0; r < kMaxTreeRank && kept < 0; ++r) {
+          int ch = -1;
+          for (int k = 0; k < p.tree_n; ++k)
+            if (p.tree_parent[k] == node && p.tree_rank[k] == r) ch = k;
+          if (ch < 0 || a + p.tree_depth[ch] > p.P) continue;
+          const int x = ci->tcand[p.tree_depth[ch] - 1][r];
+          const unsigned long long W = warp_weight(pr, x);
+          const uint32_t purpose = n_rej == 0 ? (uint32_t)PURPOSE_ACCEPT : kPurposeSibling + (uint32_t)n_rej;
+          const unsigned long long U = uniform_U(p.seed, sid, fid, round, s, purpose);
+          ++tests;
+          if (W > 0 && lt128(mul64(U, S_rem), shl53(W))) {
+            kept = ch;
+            kx = x;
+          } else {
+            rej[n_rej++] = x;
+            S_rem -= W;
+          }
+        }
+      }
+      if (kept >= 0) {
+        int kr = -1;
+        for (int r2 = 0; r2 < n_rows; ++r2)
+          if (ci->r_node[r2] == kept) kr = r2;
+        if (lane == 0) {
+          t_emit[n_emit] = kx;
+          t_path[plen] = kept;
+          t_path_row[plen] = kr;
+        }
+        ++n_emit;
+        ++plen;
+        if (s == p.P || kr < 0) break;                // the last position: nothing follows
+        node = kept;
+        row = kr;
+        continue;
+      }
+      if (s <= p.P) {
+        const int x = warp_draw_excluding(pr, rej, n_rej, S_rem, uniform_U(p.seed, sid, fid, round, s, PURPOSE_TARGET));
+        if (lane == 0) t_emit[n_emit] = x;
+        ++n_emit;
+      }
+      break;
+    }
+    if (lane == 0) {
+      t_res[0] = n_emit;
+      t_res[1] = plen;
+      t_res[2] = row;
+      t_res[3] = tests;
+    }
+  }
+  consumer_sync();
+  const int n_emit = t_res[0], plen = t_res[1], drow = t_res[2];
+  const int a_new = a + n_emit, n_next = min(p.tree_maxd, p.P - a_new);
+  // next candidates: warp j - 1 ranks the draft distribution of depth j of row drow (the
+  // record's ids with their fp32 logits; largest logit first, ties to the lower id)
+  for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
+    const TopkRec* dr = cur + (size_t)drow * (kMaxDraft + 1) + j;
+    const float* lg = p.logits + ((size_t)drow * (kMaxDraft + 1) + j) * p.V;
+    unsigned long long key[kDrawPerLane];
+#pragma unroll
+    for (int e = 0; e < kDrawPerLane; ++e) {
+      const int i = lane * kDrawPerLane + e;
+      key[e] = 0ull;
+      if (i < dr->n) {
+        const int id = dr->ids[i];
+        key[e] = ((unsigned long long)f32_key(__ldcg(lg + id)) << 32) | (0xFFFFFFFFu - (uint32_t)id);
+      }
+    }
+    for (int r = 0; r < p.tree_m[j - 1]; ++r) {
+      unsigned long long best = 0ull;
+#pragma unroll
+      for (int e = 0; e < kDrawPerLane; ++e) best = key[e] > best ? key[e] : best;
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(0xFFFFFFFFu, best, off);
+        best = o > best ? o : best;
+      }
+#pragma unroll
+      for (int e = 0; e < kDrawPerLane; ++e)
+        if (key[e] == best) key[e] = 0ull;
+      if (lane == 0) t_next[j - 1][r] = best ? (int)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull)) : -1;
+    }
+  }
+  // the kept nodes' keys and values: slot kMaxPos + row -> position a + 2 + t
+  {
+    int n_mv = 0;
+    for (int t = 0; t < plen; ++t) n_mv += t_path_row[t] >= 0 ? 1 : 0;
+    const int D4 = p.D >> 2, per = p.L * p.NKV * n_mv * D4;
+    for (int i = threadIdx.x; i < 2 * per; i += kConsumerThreads) {
+      const bool isv = i >= per;
+      const int k = isv ? i - per : i;
+      const int d4 = k % D4, t = (k / D4) % n_mv, lg = k / (D4 * n_mv);   // lg = layer * NKV + kv head
+      float* base = (isv ? p.vcache : p.kcache) + (size_t)lg * kKVSlots * p.D;
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(base + (size_t)(kMaxPos + t_path_row[t]) * p.D) + d4);
+      reinterpret_cast<float4*>(base + (size_t)(a + 2 + t) * p.D)[d4] = v;
+    }
+  }
+  consumer_sync();
+  // state of the next call
+  __shared__ int t_nvalid, t_maxd;
+  if (threadIdx.x == 0) {
+    int nv = 0, md = 0;
+    for (int i = 0; i < p.tree_n; ++i) {
+      const int d = p.tree_depth[i];
+      if (d <= n_next && a_new + d < p.P) {
+        ++nv;
+        md = max(md, d);
+      }
+    }
+    t_nvalid = nv;
+    t_maxd = md;
+    DevState* st = p.st;
+    int* codes_out = p.codes_out;
+    for (int t = 0; t < n_emit; ++t) {
+      st->codes[a + 1 + t] = t_emit[t];
+      if (codes_out) codes_out[a + t] = t_emit[t];
+      st->emitted_last[t] = t_emit[t];
+    }
+    const int calls = st0.calls + 1, heads = st0.heads_read + ci->phi[0] - ci->plo[0] + 1;
+    const int kvr = st0.kv_rows + pos0 + n_rows, rf = st0.rows_fed + n_rows;
+    const int drafted = st0.drafted + t_res[3], accepted = st0.accepted + plen;
+    st->n_emit_last = n_emit;
+    st->n_acc_last = plen;
+    st->a = a_new;
+    st->n_d = n_next;
+    st->pos0 = a_new + 1;
+    st->n_rows = 1 + nv;
+    st->top_pos = a_new + 1 + md;
+    st->round = round + 1;
+    st->first_head_row = 0;
+    st->calls = calls;
+    st->heads_read = heads;
+    st->kv_rows = kvr;
+    st->rows_fed = rf;
+    st->drafted = drafted;
+    st->accepted = accepted;
+    st->call = call + 1;
+    st->done = a_new >= p.P ? 1 : 0;
+    if (a_new >= p.P && p.stats) {
+      mcd_frame_stats* fs = p.stats;
+      fs->calls = calls;
+      fs->codes = a_new;
+      fs->drafted = drafted;
+      fs->accepted = accepted;
+      fs->status = 0;
+      fs->heads_read = heads;
+      fs->kv_rows = kvr;
+      fs->rows_fed = rf;
+    }
+  }
+  for (int i = threadIdx.x; i < kMaxDraft * kMaxTreeRank; i += kConsumerThreads) {
+    const int d = i / kMaxTreeRank, r = i % kMaxTreeRank;
+    p.tree_cand[i] = (d < n_next && r < p.tree_m[d]) ? t_next[d][r] : -1;
+  }
+  consumer_sync();
+  // optional trace: the chain record, the draft row's logits, the tree record and every row's
+  // verify logits
+  if (p.trace && round < kMaxCalls) {
+    uint8_t* tb = p.trace;
+    mcd_call_trace* tr = reinterpret_cast<mcd_call_trace*>(tb) + round;
+    float* dlog = reinterpret_cast<float*>(tb + sizeof(mcd_call_trace) * kMaxCalls) +
+                  (size_t)kMaxCalls * kMaxRows * p.V;
+    const size_t chain_bytes = sizeof(mcd_call_trace) * kMaxCalls + (size_t)2 * kMaxCalls * kMaxRows * p.V * 4;
+    mcd_tree_trace* tt = reinterpret_cast<mcd_tree_trace*>(tb + chain_bytes) + round;
+    float* vall = reinterpret_cast<float*>(tb + chain_bytes + sizeof(mcd_tree_trace) * kMaxCalls);
+    if (threadIdx.x == 0) {
+      tr->a = a;
+      tr->n_rows = n_rows;
+      tr->pos0 = pos0;
+      tr->n_drafts = t_res[3];
+      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci->r_id[n] : -1;
+      for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = -1;
+      tr->n_acc = plen;
+      tr->n_emit = n_emit;
+      for (int t = 0; t < kMaxRows; ++t) tr->emitted[t] = t < n_emit ? t_emit[t] : -1;
+      tr->n_next = n_next;
+      for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = j < n_next ? t_next[j][0] : -1;
+      tr->draft_row = drow;
+      tt->n_rows = n_rows;
+      for (int n = 0; n < kMaxCols; ++n) {
+        tt->row_node[n] = n < n_rows ? ci->r_node[n] : -1;
+        tt->row_id[n] = n < n_rows ? ci->r_id[n] : -1;
+      }
+      tt->path_len = plen;
+      for (int t = 0; t < kMaxDraft + 1; ++t) tt->path[t] = t < plen ? t_path[t] : -1;
+      tt->draft_row = drow;
+      tt->n_next = n_next;
+      for (int d = 0; d < kMaxDraft + 1; ++d)
+        for (int r = 0; r < kMaxTreeRank; ++r)
+          tt->next_cand[d][r] = (d < n_next && d < kMaxDraft && r < p.tree_m[d]) ? t_next[d][r] : -1;
+    }
+    for (int idx = threadIdx.x; idx < kMaxCols * p.V; idx += kConsumerThreads) {
+      const int n = idx / p.V, v = idx - n * p.V;
+      if (n < n_rows && ci->r_pos[n] >= 1)
+        vall[((size_t)round * kMaxCols + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+      if (n < n_next)
+        dlog[((size_t)round * kMaxRows + n) * p.V + v] =
+            __ldcg(p.logits + ((size_t)drow * (kMaxDraft + 1) + n + 1) * p.V + v);
+    }
+  }
+  consumer_sync();
+  if (threadIdx.x == 0) red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+}
+
 // Draft step of noisy-target pass j (run by the CTA that finished top-k last): draw the
 // draft of position pos0 from the pass's noisy distribution with the draft-purpose uniform
 // of the verify round, then set up pass j+1 or, after the last pass, the verify call.
@@ -833,12 +1252,14 @@ __device__ void emu_step(Cons& c, int call) {
       st->emu_in = d;
       st->pos0 = pos0 + 1;
       st->n_rows = 1;
+      st->top_pos = pos0 + 1;
     } else {
       st->emu = 0;
       st->emu_n = 0;
       st->n_d = n;
       st->pos0 = a + 1;
       st->n_rows = min(n + 1, p.P - a);
+      st->top_pos = st->pos0 + st->n_rows - 1;
       st->round = round + 1;
     }
     st->call = call + 1;
@@ -848,6 +1269,7 @@ __device__ void emu_step(Cons& c, int call) {
   }
 }
 
+template <bool WIDE>
 __device__ bool read_call_state(Cons& c, int call, bool first) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
@@ -860,8 +1282,15 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
   int* stw = reinterpret_cast<int*>(ci->st);
   for (int i = threadIdx.x; i < p.S * kWords; i += kConsumerThreads)
     stw[i] = __ldcg(reinterpret_cast<const int*>(p.st) + i);
+  const bool tree_mode = WIDE && p.draft_mode == MCD_DRAFT_TREE;    // tree calls run wide
+  if (tree_mode)
+    for (int i = threadIdx.x; i < kMaxDraft * kMaxTreeRank; i += kConsumerThreads)
+      ci->tcand[i / kMaxTreeRank][i % kMaxTreeRank] = __ldcg(p.tree_cand + i);
   consumer_sync();
   const DevState* sts = ci->st;
+  // a tree call (after the first call): row 0 feeds c_a, then the nodes whose candidates
+  // exist and whose code position a + depth < P, in tree order
+  const bool tree_rows = tree_mode && sts[0].pos0 > 0 && !sts[0].done;
   // packing order, row bases and the union of heads (one thread)
   if (threadIdx.x == 0) {
     ci->call = call;
@@ -875,7 +1304,7 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
       ci->act[n_act++] = s;
       M = min(M + sts[s].n_rows, kMaxCols);
       int lo, hi;
-      head_range(p, sts[s].a, sts[s].pos0, sts[s].n_rows, sts[s].emu, lo, hi);
+      head_range(p, sts[s].a, sts[s].top_pos, sts[s].emu, lo, hi);
       ci->plo[s] = lo;
       ci->phi[s] = hi;
       mask |= (hi >= lo) ? ((2u << hi) - (1u << lo)) : 0u;     // bits lo..hi
@@ -889,6 +1318,27 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
       mask &= mask - 1;
     }
     ci->n_heads = nh;
+    if (tree_rows) {
+      const DevState& st = sts[0];
+      int row_of[kMaxTree];
+      int n = 1;
+      ci->r_pos[0] = st.pos0;
+      ci->r_id[0] = st.codes[st.a];
+      ci->r_node[0] = -1;
+      ci->r_anc[0] = 1u;
+      for (int i = 0; i < p.tree_n; ++i) {
+        const int d = p.tree_depth[i];
+        row_of[i] = -1;
+        if (d > st.n_d || st.a + d >= p.P) continue;
+        const int pa = p.tree_parent[i];
+        ci->r_pos[n] = st.pos0 + d;
+        ci->r_id[n] = ci->tcand[d - 1][p.tree_rank[i]];
+        ci->r_node[n] = (signed char)i;
+        ci->r_anc[n] = (pa < 0 ? 1u : ci->r_anc[row_of[pa]]) | (1u << n);
+        row_of[i] = n++;
+      }
+      if (n != ci->M) atomicCAS(p.err, 0, (int)MCD_ERR_STATE);   // the acceptance step counted otherwise
+    }
   }
   consumer_sync();
   // (3) one thread per packed row: stream, position, code fed, layer-0 input row
@@ -898,9 +1348,18 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
     for (int i = 0; i < ci->n_act; ++i)
       if (ci->base[ci->act[i]] <= r) s = ci->act[i];
     const DevState* st = sts + s;
-    const int n = r - ci->base[s], pos = st->pos0 + n;
-    int id = st->emu ? st->emu_in
-                     : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+    const int n = r - ci->base[s];
+    int pos, id;
+    if (tree_rows) {
+      pos = ci->r_pos[r];
+      id = ci->r_id[r];
+    } else {
+      pos = st->pos0 + n;
+      id = st->emu ? st->emu_in
+                   : st->pos0 == 0 ? (n == 0 ? -1 : st->codes[0]) : (n == 0 ? st->codes[st->a] : st->drafts[n - 1]);
+      ci->r_anc[r] = (2u << n) - 1u;          // rows 0..n (n <= 31; 2 << 31 wraps to 0)
+      ci->r_node[r] = -1;
+    }
     // layer-0 input row: cond (position 0), the c0 embedding vector (position 1 without a
     // c0 table), else row `id` of table pos - 1
     if (pos == 0 || (pos == 1 && p.C0V == 0)) {
@@ -949,7 +1408,7 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
   } else {
     Cons c(p, sm);
     for (int call = call0; call < kMaxSlots; ++call) {
-      if (!read_call_state(c, call, call == call0)) break;
+      if (!read_call_state<WIDE>(c, call, call == call0)) break;
       if (sm.ci->all_done) break;
       // a stepwise launch runs one verify call and the noisy-target passes that follow it
       if (p.single_call && call != call0 && !sm.ci->emu) break;
@@ -958,6 +1417,8 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
       if (sm.flags[2]) {
         if (sm.ci->emu)
           emu_step(c, call);
+        else if (WIDE && p.draft_mode == MCD_DRAFT_TREE)
+          accept_tree(c, call);
         else
           accept_step(c, call, sm.flags[4]);
       }
@@ -979,7 +1440,7 @@ static void* frame_entry() {
 
 cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream) {
   void* args[] = {const_cast<FrameParams*>(&p)};
-  const bool wide = p.S * max(p.K + 1, 2) > kMaxRows;
+  const bool wide = p.S * max(p.K + 1, 2) > kMaxRows || p.draft_mode == MCD_DRAFT_TREE;
   void* fn = p.wdtype == MCD_WEIGHT_BF16 ? (wide ? frame_entry<MCD_WEIGHT_BF16, true>() : frame_entry<MCD_WEIGHT_BF16, false>())
                                          : (wide ? frame_entry<MCD_WEIGHT_F32, true>() : frame_entry<MCD_WEIGHT_F32, false>());
   return cudaLaunchCooperativeKernel(fn, dim3(p.n_cta), dim3(kThreads), args, (size_t)kSmemBytes, stream);

@@ -24,6 +24,10 @@ constexpr int kMaxBatchRows = 512;     // packed rows of one batched call
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
+constexpr int kKVSlots = 2 * kMaxPos; // cache entries per (layer, KV head): positions, then the
+                                      // current tree call's node rows (kMaxPos + row)
+constexpr int kMaxTree = 31;         // tree nodes (rows = 1 + nodes <= kMaxCols)
+constexpr int kMaxTreeRank = 8;      // candidates per drafted position
 constexpr int kMaxCalls = 16;        // verify calls per frame (15 positions, first call emits 1)
 constexpr int kMaxSlots = 128;       // passes per frame: verify calls + noisy-target drafting passes
 constexpr int kMaxVocab = 4096;
@@ -73,6 +77,7 @@ struct DevState {
   int emu;             // 0: the next pass is a verify call; j >= 1: noisy-target pass j
   int emu_n;           // drafts the noisy-target passes make for the next verify call
   int emu_in;          // code fed to the next noisy-target pass
+  int top_pos;         // largest row position of the next pass
 };
 
 // State of a stream at the start of a frame: the first call feeds [cond, c0] (positions 0, 1).
@@ -90,6 +95,7 @@ __device__ inline void init_stream_state(DevState* st, int c0) {
   st->emu = 0;
   st->emu_n = 0;
   st->emu_in = -1;
+  st->top_pos = 1;
   for (int i = 0; i < kMaxPos; ++i) st->codes[i] = -1;
   st->codes[0] = c0;
   for (int i = 0; i <= kMaxDraft; ++i) st->drafts[i] = -1;
@@ -137,7 +143,7 @@ struct FrameParams {
   float* mbuf;                 // [kMaxCols][F]
   float* attn;                 // [kMaxCols][NH*D] attention outputs (batched calls)
   float* logits;               // [kMaxCols][kMaxDraft+1][V]
-  float* kcache;               // [S][L][NKV][kMaxPos][D]
+  float* kcache;               // [S][L][NKV][kKVSlots][D]
   float* vcache;
   TopkRec* topk;               // [2][kMaxCols][kMaxDraft+1]
   TopkRec* draftq;             // [kMaxDraft] pending drafts' q
@@ -161,6 +167,11 @@ struct FrameParams {
   int* n_emitted_out;
   unsigned long long* timeline;  // optional [kMaxCalls][32] %globaltimer stamps (CTA 0)
   int single_call;             // 1 = run exactly one call (stepwise API)
+  // sparse tree (TREE mode): nodes in breadth-first order
+  int tree_n, tree_maxd;
+  signed char tree_parent[kMaxTree], tree_rank[kMaxTree], tree_depth[kMaxTree];
+  int tree_m[kMaxDraft];       // candidates needed per depth
+  int* tree_cand;              // [kMaxDraft][kMaxTreeRank] candidates of the next call
   int n_cta;
   unsigned long long wait_ns;  // bound of every device-side wait
 };
@@ -304,6 +315,7 @@ __host__ __device__ inline unsigned long long uniform_U(unsigned long long seed,
 }
 
 enum { PURPOSE_TARGET = 0, PURPOSE_ACCEPT = 1, PURPOSE_DRAFT = 2, PURPOSE_NOISE = 3 };
+constexpr uint32_t kPurposeSibling = 0x10000u;   // + i: test i >= 1 at a tree node
 
 // Two N(0,1) draws for vocabulary entries (2 pair, 2 pair + 1) of a noisy draft row: the
 // Box-Muller transform (Box and Muller, 1958) of the 53-bit uniforms of words (0,1) and

@@ -358,6 +358,26 @@ __device__ __forceinline__ int warp_draw(const TopkRec* r, unsigned long long U)
   return r->ids[warp_draw_lanes(v, n, r->S, U)];
 }
 
+// Draw from p without the ids in ex[0..n_ex) (weights set to zero; S_rem = S minus their
+// weights), by a full warp: the residual of one-hot draft distributions tested in turn.
+__device__ __forceinline__ int warp_draw_excluding(const TopkRec* r, const int* ex, int n_ex, unsigned long long S_rem,
+                                                   unsigned long long U) {
+  const int lane = threadIdx.x & 31, n = r->n;
+  unsigned long long v[kDrawPerLane];
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    const int i = lane * kDrawPerLane + e;
+    v[e] = 0ull;
+    if (i < n) {
+      const int id = r->ids[i];
+      bool out = false;
+      for (int t = 0; t < n_ex; ++t) out |= ex[t] == id;
+      if (!out) v[e] = r->W[i];
+    }
+  }
+  return r->ids[warp_draw_lanes(v, n, S_rem, U)];
+}
+
 // Residual draw from normalise(max(0, p - q)) over p's entries in p's order, by a full warp.
 static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U) {
   const int lane = threadIdx.x & 31;

@@ -32,6 +32,11 @@ struct CallInfo {
   // packed rows: stream, row within the stream, position, code fed, layer-0 input row
   int r_s[kMaxCols], r_n[kMaxCols], r_pos[kMaxCols], r_id[kMaxCols], r_f32[kMaxCols];
   const uint8_t* r_src[kMaxCols];
+  // rows of the same stream visible to packed row r (bit n: the stream's row n): every
+  // earlier row and itself, or for a tree call the first row, its ancestors and itself
+  unsigned r_anc[kMaxCols];
+  signed char r_node[kMaxCols];                  // tree node of the row (-1: none)
+  int tcand[kMaxDraft][kMaxTreeRank];            // tree call: candidates of its nodes
   // per stream (index = stream): its state and the derived packing
   DevState st[kMaxStreams];
   int act[kMaxStreams];        // active streams in packing order

@@ -56,6 +56,11 @@ CALL_TRACE_DTYPE = np.dtype([("a", "<i4"), ("n_rows", "<i4"), ("pos0", "<i4"), (
                              ("next_drafts", "<i4", 8), ("draft_row", "<i4"), ("reserved", "<i4", 24)])
 assert CALL_TRACE_DTYPE.itemsize == 256
 
+TREE_TRACE_DTYPE = np.dtype([("n_rows", "<i4"), ("row_node", "<i4", 32), ("row_id", "<i4", 32),
+                             ("path_len", "<i4"), ("path", "<i4", 8), ("draft_row", "<i4"), ("n_next", "<i4"),
+                             ("next_cand", "<i4", (8, 8)), ("reserved", "<i4", 20)])
+assert TREE_TRACE_DTYPE.itemsize == 640
+
 
 class MCDError(RuntimeError):
     def __init__(self, fn: str, status: int):
@@ -97,6 +102,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_num_ctas": (I32, [P]),
         "mcd_destroy": (None, [P]),
         "mcd_status_str": (ctypes.c_char_p, [I32]),
+        "mcd_set_tree": (I32, [P, I32, P, P]),
         "mcd_outer_create": (I32, [ctypes.POINTER(McdOuterConfig), P, ctypes.POINTER(P)]),
         "mcd_outer_destroy": (None, [P]),
         "mcd_outer_load_weights": (I32, [P, I32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(P),
@@ -271,6 +277,23 @@ def parse_trace(buf: np.ndarray, vocab: int):
     n = MAX_CALLS * MAX_ROWS * vocab
     return recs, logits[:n].reshape(MAX_CALLS, MAX_ROWS, vocab), logits[n:2 * n].reshape(
         MAX_CALLS, MAX_ROWS, vocab)
+
+
+def mcd_set_tree(ctx, parent, rank):
+    """Sparse tree of TREE mode: parent[i] (-1: child of the call's first row), rank[i]."""
+    n = len(parent)
+    pa = (ctypes.c_int32 * n)(*[int(v) for v in parent])
+    rk = (ctypes.c_int32 * n)(*[int(v) for v in rank])
+    _check("mcd_set_tree", load_library().mcd_set_tree(ctx, n, pa, rk))
+
+
+def parse_tree_trace(buf: np.ndarray, vocab: int):
+    """TREE mode: (tree records [16], verify logits of every row [16 calls][32 rows][vocab])."""
+    start = CALL_TRACE_DTYPE.itemsize * MAX_CALLS + 2 * MAX_CALLS * MAX_ROWS * vocab * 4
+    n = TREE_TRACE_DTYPE.itemsize * MAX_CALLS
+    recs = buf[start:start + n].view(TREE_TRACE_DTYPE)
+    vall = buf[start + n:start + n + MAX_CALLS * 32 * vocab * 4].view(np.float32).reshape(MAX_CALLS, 32, vocab)
+    return recs, vall
 
 
 class Decoder:

@@ -30,6 +30,7 @@ WEIGHT_BF16 = 1
 DRAFT_SAMPLE = 0
 DRAFT_GREEDY = 1
 DRAFT_NOISY_TARGET = 2
+DRAFT_TREE = 3
 
 
 @dataclasses.dataclass(frozen=True)

@@ -93,3 +93,90 @@ def check_trace_against_oracle(cfg, model, fr, stream_id, frame_idx, trace_u8, c
     assert len(emitted_all) == P
     assert emitted_all == [int(v) for v in codes], (emitted_all, list(codes))
     return max_err
+
+
+def check_tree_trace_against_oracle(cfg, model, fr, stream_id, frame_idx, trace_u8, codes, n_calls, tree,
+                                    logit_tol):
+    """TREE mode: every call's rows (tree order, ids), every row's verify logits and the draft
+    row's draft logits against the oracle (rows recomputed with the tree attention mask on the
+    oracle's own cache), then the walk, the kept path, the emitted codes and the next
+    candidates identical when the oracle works on the GPU's fp32 logits."""
+    from oracle import philox
+    from oracle.sampler import draw
+    from oracle.tree import ranked, tree_row, walk
+    V, P = cfg.vocab, cfg.n_pos
+    buf = np.asarray(trace_u8, dtype=np.uint8)
+    recs, _, dlog = mcd.parse_trace(buf, V)
+    trecs, vall = mcd.parse_tree_trace(buf, V)
+    S = Sampling(cfg, stream_id, frame_idx)
+    m_need, K = tree.ranks_needed(), tree.max_depth
+    kv = model.new_kv()
+    max_err = 0.0
+
+    def cmp(got, ref, what):
+        nonlocal max_err
+        err = float(np.max(np.abs(np.asarray(got, dtype=np.float64) - ref)))
+        max_err = max(max_err, err)
+        assert err <= logit_tol, f"{what}: logits differ by {err}"
+
+    # call 0: [cond, c0] at positions 0, 1; c1 from LM head 1
+    model.row(kv, np.asarray(fr.cond, dtype=np.float64), 0)
+    h1 = model.row(kv, model.c0_row(fr.c0, fr.c0_emb), 1)
+    t0 = trecs[0]
+    assert int(recs[0]["a"]) == 0 and int(t0["n_rows"]) == 2
+    cmp(vall[0, 1], model.verify_logits(1, h1), "call 0 row 1")
+    c1 = draw(S.dist(vall[0, 1].copy()), S.u(0, 1, philox.PURPOSE_TARGET))
+    assert [c1] == [int(v) for v in recs[0]["emitted"][:int(recs[0]["n_emit"])]]
+    emitted_all = [c1]
+    n_next = int(t0["n_next"])
+    assert n_next == min(K, P - 1)
+    cand = []
+    for d in range(1, n_next + 1):
+        cmp(dlog[0, d - 1], model.draft_logits(1, d, h1), f"call 0 draft {d}")
+        cand.append(ranked(dlog[0, d - 1], m_need[d - 1]))
+        assert cand[-1] == [int(v) for v in t0["next_cand"][d - 1][:m_need[d - 1]]], (cand[-1], t0["next_cand"])
+    for c in range(1, n_calls):
+        r, t = recs[c], trecs[c]
+        a = int(r["a"])
+        assert a == len(emitted_all), (c, a)
+        codes_map = {i + 1: x for i, x in enumerate(emitted_all)}
+        # expected rows: c_a, then the nodes whose candidates exist and a + depth < P
+        rows = [(-1, a + 1, codes_map[a])]
+        row_of_node = {}
+        for i in range(tree.n):
+            d = tree.depth[i]
+            if d <= len(cand) and a + d < P:
+                row_of_node[i] = len(rows)
+                rows.append((i, a + 1 + d, cand[d - 1][tree.rank[i]]))
+        n_rows = int(t["n_rows"])
+        assert n_rows == len(rows), (c, n_rows, len(rows))
+        assert [int(v) for v in t["row_node"][:n_rows]] == [x[0] for x in rows]
+        assert [int(v) for v in t["row_id"][:n_rows]] == [x[2] for x in rows]
+        h, own = {}, {}
+        h[0], own[0] = tree_row(model, kv, a + 1, [], model.code_row(a, codes_map[a]), a + 1)
+        for n in range(1, n_rows):
+            node, pos, x = rows[n]
+            anc = [own[0]] + [own[row_of_node[j]] for j in tree.ancestors(node)[:-1]]
+            h[n], own[n] = tree_row(model, kv, a + 1, anc, model.code_row(pos - 1, x), pos)
+        for n in range(n_rows):
+            cmp(vall[c, n], model.verify_logits(rows[n][1], h[n]), f"call {c} row {n}")
+        emitted, path, drow = walk(S, c, a, P, tree, cand, lambda n: S.dist(vall[c, n].copy()), row_of_node)
+        assert emitted == [int(v) for v in r["emitted"][:int(r["n_emit"])]], (c, emitted, r["emitted"])
+        assert path == [int(v) for v in t["path"][:int(t["path_len"])]], (c, path, t["path"])
+        assert drow == int(t["draft_row"]), (c, drow, int(t["draft_row"]))
+        for i, rr in enumerate([0] + [row_of_node[nn] for nn in path if nn in row_of_node]):
+            for l in range(model.cfg.n_layers):
+                kv[l, 0, :, a + 1 + i] = own[rr][l][0]
+                kv[l, 1, :, a + 1 + i] = own[rr][l][1]
+        emitted_all += emitted
+        a_new = len(emitted_all)
+        n_next = int(t["n_next"])
+        assert n_next == min(K, P - a_new)
+        cand = []
+        for d in range(1, n_next + 1):
+            cmp(dlog[c, d - 1], model.draft_logits(rows[drow][1], d, h[drow]), f"call {c} draft {d}")
+            cand.append(ranked(dlog[c, d - 1], m_need[d - 1]))
+            assert cand[-1] == [int(v) for v in t["next_cand"][d - 1][:m_need[d - 1]]], (c, d, cand[-1])
+    assert len(emitted_all) == P
+    assert emitted_all == [int(v) for v in codes], (emitted_all, list(codes))
+    return max_err

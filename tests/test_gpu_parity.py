@@ -27,7 +27,7 @@ from oracle.frame import Sampling, decode_frame, verify_round  # noqa: E402
 from oracle import accounting  # noqa: E402
 from oracle.model import Model  # noqa: E402
 from oracle.sampler import topk_dist  # noqa: E402
-from parity import check_trace_against_oracle  # noqa: E402
+from parity import check_trace_against_oracle, check_tree_trace_against_oracle  # noqa: E402
 
 DEV = torch.device("cuda:0")
 _build.build()
@@ -333,6 +333,72 @@ def test_gemm_path_full_size(n_streams, checked):
     codes2, st2, _ = decode_many(env, frames, [f + 1 for f in fidx], sids)
     assert (st2[:, 1] == cfg.n_pos).all()
     env.dec.close()
+
+
+# ------------------------------------------------- sparse tree verification (Fig. 2) ---
+def _trees():
+    from oracle.tree import Tree, grow_tree
+    fig2 = Tree(parent=[-1, -1, 0, 0, 1, 2, 4, 4], rank=[0, 1, 0, 1, 0, 0, 0, 1])
+    big = grow_tree([[0.5, 0.3, 0.2, 0.1, 0.05], [0.4, 0.25, 0.1], [0.3, 0.2]], 31)
+    return {"chain3": Tree.chain(3), "fig2": fig2, "wide": Tree(parent=[-1, -1, -1, -1], rank=[0, 1, 2, 3]),
+            "big31": big}
+
+
+@pytest.mark.parametrize("name", ["chain3", "fig2", "wide", "big31"])
+def test_tree_mode_trace_parity_tiny(name):
+    """TREE mode: every call's rows, logits (1e-5), walk, kept path, codes and next candidates
+    against the oracle; the 31-node tree packs 32 rows per call."""
+    tree = _trees()[name]
+    cfg = TINY.replace(draft_mode=3, draft_len=3, n_pos=8)
+    env = Env(cfg)
+    mcd.mcd_set_tree(env.dec.ctx, tree.parent, tree.rank)
+    worst = 0.0
+    for f in range(4):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, stream_id=1, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos, st
+        worst = max(worst, check_tree_trace_against_oracle(cfg, env.model, fr, 1, f, tr, codes, int(st[0]), tree,
+                                                           logit_tol=1e-5))
+    print(name, "max |dlogit|", worst)
+    env.dec.close()
+
+
+def test_chain_tree_equals_greedy_drafts_on_gpu():
+    cfg = TINY.replace(draft_len=3, n_pos=8)
+    tree_env = Env(cfg.replace(draft_mode=3))
+    greedy_env = Env(cfg.replace(draft_mode=DRAFT_GREEDY))
+    for f in range(6):
+        fr = make_frame(cfg, f)
+        a, sa, _ = tree_env.decode(fr, f)
+        b, sb, _ = greedy_env.decode(fr, f)
+        assert list(a) == list(b) and int(sa[0]) == int(sb[0]), f
+    tree_env.dec.close()
+    greedy_env.dec.close()
+
+
+def test_tree_mode_full_size():
+    tree = _trees()["fig2"]
+    cfg = MCD.replace(draft_mode=3, draft_len=3)
+    env = Env(cfg)
+    mcd.mcd_set_tree(env.dec.ctx, tree.parent, tree.rank)
+    for f in (0, 1):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        err = check_tree_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]), tree, logit_tol=2e-2)
+        print("tree full size max |dlogit|", err)
+    env.dec.close()
+
+
+def test_tree_api_rejects_malformed_trees():
+    env = Env(TINY.replace(draft_mode=3, draft_len=2))
+    ctx = env.dec.ctx
+    for parent, rank in (([0], [0]), ([-1, -1], [0, 0]), ([-1, 0, 1], [0, 0, 0]), ([-1], [8])):
+        with pytest.raises(mcd.MCDError):
+            mcd.mcd_set_tree(ctx, parent, rank)
+    env.dec.close()
+    with pytest.raises(mcd.MCDError):
+        mcd.Decoder(TINY.replace(draft_mode=3, max_streams=2))
 
 
 # ------------------------------------------------- noisy-target drafts (K sweep) ------
