@@ -243,6 +243,71 @@ def run_sweep(args, weights):
                               "us_per_call_from": "position-aware drafter frames at the same K"}), flush=True)
 
 
+def run_tree_sweep(args, weights):
+    """Sparse tree verification (Sec. 2.2, Fig. 4): acceptance statistics per (depth, rank)
+    from traced frames of a probe tree, greedy trees of N = 1..31 nodes grown from them,
+    then per N: accepted tokens per call, microseconds per verify call and tokens/s.  One
+    JSON line per N."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    from paper_2609_37007_gb300 import tree as trees
+    from paper_2609_37007_gb300.synth import DRAFT_TREE, MCD, make_frames
+    _build.build()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    cfg = MCD.replace(draft_mode=DRAFT_TREE, draft_len=3)
+    n = args.sweep_frames
+    cond_h, c0_h, _ = make_frames(cfg, n + 3, first=6_000_000)
+    cond = torch.from_numpy(cond_h).to(dev)
+    c0 = torch.from_numpy(c0_h).to(dev)
+    codes = torch.zeros((n + 3, cfg.n_pos), dtype=torch.int32, device=dev)
+    stats = torch.zeros((n + 3, 8), dtype=torch.int32, device=dev)
+    dec = mcd.Decoder(cfg, weights, stream)
+    # statistics from a probe tree (8 candidates at each of 3 depths)
+    depth, ranks = 3, 8
+    mcd.mcd_set_tree(dec.ctx, *trees.probe_tree(depth, ranks))
+    tr = torch.zeros(mcd.mcd_trace_bytes(dec.ctx), dtype=torch.uint8, device=dev)
+    records, frame_codes = [], []
+    mcd.mcd_set_trace(dec.ctx, tr)
+    for i in range(min(n, 60)):
+        mcd.mcd_decode_frame(dec.ctx, 0, 7_000_000 + i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+        mcd.mcd_sync(dec.ctx)
+        buf = tr.cpu().numpy()
+        recs, _, _ = mcd.parse_trace(buf, cfg.vocab)
+        trecs, _ = mcd.parse_tree_trace(buf, cfg.vocab)
+        calls = int(stats[i, 0])
+        records.append([(int(recs[c]["a"]) + int(recs[c]["n_emit"]),
+                         [list(map(int, trecs[c]["next_cand"][d][:ranks])) for d in range(depth)])
+                        for c in range(calls)])
+        frame_codes.append(codes[i].cpu().numpy().tolist())
+    mcd.mcd_set_trace(dec.ctx, None)
+    acc = trees.measure_acceptance(records, frame_codes, depth, ranks, cfg.n_pos)
+    print(json.dumps({"tree_stats": "P(rank-r candidate of depth d is the emitted code)", "acc": acc,
+                      "frames": len(records)}), flush=True)
+    for N in args.tree_sizes:
+        parent, rank = trees.grow_tree(acc, N)
+        mcd.mcd_set_tree(dec.ctx, parent, rank)
+        for i in range(3):
+            mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+        mcd.mcd_sync(dec.ctx)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(3, n + 3):
+            mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        mcd.mcd_sync(dec.ctx)
+        st = stats.cpu().numpy()[3:]
+        assert (st[:, 4] == 0).all() and (st[:, 1] == cfg.n_pos).all()
+        t_us = e0.elapsed_time(e1) * 1e3
+        calls, toks = int(st[:, 0].sum()), int(st[:, 1].sum())
+        print(json.dumps({"tree_nodes": len(parent), "rows_per_call": 1 + len(parent), "tokens_per_call": toks / calls,
+                          "us_per_verify_call": t_us / calls, "tokens_per_s": toks / t_us * 1e6, "frames": n,
+                          "parent": parent, "rank": rank}), flush=True)
+    dec.close()
+
+
 def run_streams(args, weights):
     """Batched independent streams: one mcd_decode_frames launch decodes a frame for each of
     B streams (rows re-packed every call).  Prints one JSON line per B: aggregate accepted
@@ -472,6 +537,9 @@ def main():
     ap.add_argument("--streams", type=int, nargs="*", default=None,
                     help="batched-stream runs for these B instead of the bench line (e.g. --streams 1 2 4 8)")
     ap.add_argument("--stream-launches", type=int, default=100)
+    ap.add_argument("--tree-sweep", action="store_true",
+                    help="sparse tree sizes N (greedy trees from measured statistics) instead of the bench line")
+    ap.add_argument("--tree-sizes", type=int, nargs="+", default=[1, 2, 4, 8, 16, 31])
     ap.add_argument("--pipeline", action="store_true",
                     help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
     ap.add_argument("--utterances", type=int, default=2)
@@ -487,6 +555,8 @@ def main():
         return run_streams(args, weights)
     if args.pipeline:
         return run_pipeline(args)
+    if args.tree_sweep:
+        return run_tree_sweep(args, weights)
     if args.sweep:
         # one weight set with offsets b_1..b_7 serves every K (extra tensors are ignored)
         return run_sweep(args, make_weights(cfg.replace(draft_len=7)))
