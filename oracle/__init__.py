@@ -17,6 +17,7 @@ Modules:
   frame        autoregressive and speculative frame procedures.
   codedecoder  the outer CodeDecoder (one call per frame, emits c0) and the full frame
                pipeline of Fig. 1 (prompt prefill, c0, MultiCodeDecoder, input sum).
+  quant        W8A16 per-row symmetric int8 weights.
   tree         sparse tree drafting and verification (Fig. 2) and the greedy tree growth.
   enumeration  exact output distributions of the procedures (losslessness pin).
   accounting   the paper's real-time call arithmetic.

@@ -26,6 +26,7 @@ import numpy as np
 
 WEIGHT_F32 = 0
 WEIGHT_BF16 = 1
+WEIGHT_INT8 = 2      # W8A16: the library quantises the bf16 matrices it streams at load time
 
 DRAFT_SAMPLE = 0
 DRAFT_GREEDY = 1
@@ -131,13 +132,13 @@ def make_weights(cfg: MCDConfig) -> Dict[str, np.ndarray]:
             vals = (1.0 + 0.1 * draw.astype(np.float64)).astype(np.float32)
         else:
             vals = (0.02 * draw.astype(np.float64)).astype(np.float32)
-        out[name] = round_to_bf16_bits(vals) if cfg.weight_dtype == WEIGHT_BF16 else vals
+        out[name] = round_to_bf16_bits(vals) if cfg.weight_dtype in (WEIGHT_BF16, WEIGHT_INT8) else vals
     return out
 
 
 def weights_as_f32(cfg: MCDConfig, w: Dict[str, np.ndarray]) -> Dict[str, np.ndarray]:
     """The exact values the weights represent, as float32 (bf16 widening is exact)."""
-    if cfg.weight_dtype == WEIGHT_BF16:
+    if cfg.weight_dtype in (WEIGHT_BF16, WEIGHT_INT8):
         return {k: bf16_bits_to_f32(v) for k, v in w.items()}
     return dict(w)
 
