@@ -131,7 +131,11 @@ def cpu_oracle_baseline(cfg, weights, budget_s: float, first_frame: int):
     from paper_2609_37007_gb300.synth import make_frame, weights_as_f32
     from oracle.model import Model
     from oracle.frame import decode_frame
-    model = Model(cfg, weights_as_f32(cfg, weights))
+    w = weights_as_f32(cfg, weights)
+    if cfg.weight_dtype == 2:                    # W8A16: the oracle computes with q * s
+        from oracle.quant import w8a16_weights
+        w = w8a16_weights(w)
+    model = Model(cfg, w)
     t0 = time.perf_counter()
     frames = codes = calls = 0
     while frames < 2 or time.perf_counter() - t0 < budget_s:
@@ -537,6 +541,8 @@ def main():
     ap.add_argument("--streams", type=int, nargs="*", default=None,
                     help="batched-stream runs for these B instead of the bench line (e.g. --streams 1 2 4 8)")
     ap.add_argument("--stream-launches", type=int, default=100)
+    ap.add_argument("--w8a16", action="store_true",
+                    help="the bench line with int8 weights quantised per row at load (W8A16)")
     ap.add_argument("--tree-sweep", action="store_true",
                     help="sparse tree sizes N (greedy trees from measured statistics) instead of the bench line")
     ap.add_argument("--tree-sizes", type=int, nargs="+", default=[1, 2, 4, 8, 16, 31])
@@ -546,8 +552,8 @@ def main():
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
-    from paper_2609_37007_gb300.synth import MCD, make_frames, make_weights
-    cfg = MCD
+    from paper_2609_37007_gb300.synth import MCD, WEIGHT_INT8, make_frames, make_weights
+    cfg = MCD.replace(weight_dtype=WEIGHT_INT8) if args.w8a16 else MCD
     weights = make_weights(cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, weights)
@@ -702,9 +708,11 @@ def main():
     line = {
         "metric": METRIC, "value": tokens_all / elapsed_all, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * elapsed_all / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "w8a16" if args.w8a16 else "bf16",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "frames_per_rank": args.steps,
+        "config": {"workload": WORKLOAD.replace("MultiCodeDecoder bf16", "MultiCodeDecoder W8A16 (int8 weights, "
+                                                "per-row scales)") if args.w8a16 else WORKLOAD,
+                   "frames_per_rank": args.steps,
                    "arithmetic": "bf16 weights x fp32 activations (bf16 hi+lo split), fp32 accumulate; "
                                  "sampler on 24-bit integer weights with exact integer decisions",
                    "l2": "inputs larger than L2: 287 MB of weights per context, ~175-187 MB streamed per call",

@@ -57,7 +57,11 @@ typedef enum {
   MCD_ERR_UNSUPPORTED = 7    /* shape outside the kernels' limits                      */
 } mcd_status;
 
-enum { MCD_WEIGHT_F32 = 0, MCD_WEIGHT_BF16 = 1 };
+/* MCD_WEIGHT_INT8 (W8A16, Sec. 3.3): weights are passed in bf16 like MCD_WEIGHT_BF16 and
+ * the library quantises every streamed matrix (Wq, Wk, Wv, Wo, Wg, Wu, Wd, LM heads) per
+ * output row at load: s = fp32(max |w| / 127), q = clamp(rint(fp32(w / s)), -127, 127),
+ * computing with q * s; embedding tables stay bf16.  Single-stream and up to 32 packed rows. */
+enum { MCD_WEIGHT_F32 = 0, MCD_WEIGHT_BF16 = 1, MCD_WEIGHT_INT8 = 2 };
 enum { MCD_DRAFT_SAMPLE = 0, MCD_DRAFT_GREEDY = 1, MCD_DRAFT_NOISY_TARGET = 2, MCD_DRAFT_TREE = 3 };
 
 /* Model and sampling configuration.  Limits: hidden, ffn multiples of 128; head_dim 64
@@ -70,7 +74,7 @@ typedef struct {
   int32_t c0_vocab;     /* rows of table 0; 0 = frames pass a c0 embedding vector       */
   float rms_eps, rope_base;
   int32_t qk_norm;      /* per-head RMSNorm of q and k before RoPE                      */
-  int32_t weight_dtype; /* MCD_WEIGHT_F32 or MCD_WEIGHT_BF16                            */
+  int32_t weight_dtype; /* MCD_WEIGHT_F32, MCD_WEIGHT_BF16 or MCD_WEIGHT_INT8             */
   int32_t draft_len;    /* K; 0 = plain autoregressive decoding                         */
   int32_t top_k;
   float temperature;

@@ -22,50 +22,79 @@ int frame_smem_bytes();
 // ------------------------------------------------------------------------------------
 // Auxiliary kernels
 // ------------------------------------------------------------------------------------
-__global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst) {
+// Source row of tiled row r.
+__device__ inline const uint8_t* src_row(const RowSrc& rs, int r, int es) {
+  const uint8_t* src;
+  int sr;
+  if (rs.interleave_gu) {
+    const int t = r >> 4, rr = r & 15;
+    src = rs.seg[rr < 8 ? 0 : 1];
+    sr = 8 * t + (rr & 7);
+  } else {
+    int rem = r, s = 0;
+    while (s < rs.nseg - 1 && rem >= rs.seg_rows[s]) rem -= rs.seg_rows[s++];
+    src = rs.seg[s];
+    sr = rem;
+  }
+  return src + (long long)sr * rs.src_cols * es;
+}
+
+// W8A16 quantisation of one element: q = clamp(rint(fp32(w / s)), -127, 127), 0 if s = 0.
+__device__ inline int quantise_w8(float w, float s) {
+  if (!(s > 0.f)) return 0;
+  const float q = rintf(__fdiv_rn(w, s));
+  return (int)fminf(127.f, fmaxf(-127.f, q));
+}
+
+__global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst, const float* scale) {
   const long long total = (long long)g.M * g.K;
-  const int es = wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  const int es = wdtype == MCD_WEIGHT_F32 ? 4 : 2;                        // source element bytes
+  const int ed = wdtype == MCD_WEIGHT_F32 ? 4 : (wdtype == MCD_WEIGHT_INT8 ? 1 : 2);   // tiled element bytes
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
     const int r = (int)(e / g.K), c = (int)(e % g.K);
-    const uint8_t* src;
-    int sr;
-    if (rs.interleave_gu) {
-      const int t = r >> 4, rr = r & 15;
-      src = rs.seg[rr < 8 ? 0 : 1];
-      sr = 8 * t + (rr & 7);
+    const uint8_t* src = src_row(rs, r, es) + (long long)c * es;
+    const long long d = tiled_offset(g, r, c, wdtype) * ed;
+    if (ed == 1) {
+      const float w = bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(src));
+      reinterpret_cast<int8_t*>(dst)[d] = (int8_t)quantise_w8(w, scale[r]);
+    } else if (ed == 2) {
+      *reinterpret_cast<uint16_t*>(dst + d) = *reinterpret_cast<const uint16_t*>(src);
     } else {
-      int rem = r, s = 0;
-      while (s < rs.nseg - 1 && rem >= rs.seg_rows[s]) rem -= rs.seg_rows[s++];
-      src = rs.seg[s];
-      sr = rem;
+      *reinterpret_cast<uint32_t*>(dst + d) = *reinterpret_cast<const uint32_t*>(src);
     }
-    const long long so = ((long long)sr * rs.src_cols + c) * es;
-    const long long d = tiled_offset(g, r, c, wdtype) * es;
-    if (es == 2)
-      *reinterpret_cast<uint16_t*>(dst + d) = *reinterpret_cast<const uint16_t*>(src + so);
-    else
-      *reinterpret_cast<uint32_t*>(dst + d) = *reinterpret_cast<const uint32_t*>(src + so);
   }
+}
+
+// One warp per tiled row: s = fp32(max |w| / 127) over the row's bf16 source values.
+__global__ void row_scale_kernel(RowSrc rs, MatGeom g, float* scale) {
+  const int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (r >= g.M) return;
+  const uint16_t* src = reinterpret_cast<const uint16_t*>(src_row(rs, r, 2));
+  float m = 0.f;
+  for (int c = lane; c < g.K; c += 32) m = fmaxf(m, fabsf(bf16_bits_to_f32(src[c])));
+  for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+  if (lane == 0) scale[r] = __fdiv_rn(m, 127.f);
 }
 
 __global__ void to_f32_kernel(const uint8_t* src, int wdtype, long long n, float* dst) {
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
-    dst[i] = wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(src)[i])
+    dst[i] = wdtype != MCD_WEIGHT_F32 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(src)[i])
                                        : reinterpret_cast<const float*>(src)[i];
 }
 
 // LMH_P b_j for j = 1..K from the row-major head (one warp per output): the offsets'
 // additive share of the draft logits, LMH_P (h + b_j) = LMH_P h + LMH_P b_j.
 __global__ void head_bias_kernel(const uint8_t* head, const float* offsets, int K, int V, int H, int wdtype,
-                                 float* out) {
+                                 const float* scale, float* out) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= K * V) return;
   const int j = warp / V, id = warp % V;
   float acc = 0.f;
   for (int k = lane; k < H; k += 32) {
-    const float w = wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(head)[(size_t)id * H + k])
-                                              : reinterpret_cast<const float*>(head)[(size_t)id * H + k];
+    float w = wdtype != MCD_WEIGHT_F32 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(head)[(size_t)id * H + k])
+                                       : reinterpret_cast<const float*>(head)[(size_t)id * H + k];
+    if (wdtype == MCD_WEIGHT_INT8) w = (float)quantise_w8(w, scale[id]) * scale[id];   // the W8A16 head's value
     acc += w * offsets[(size_t)j * H + k];
   }
   for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
@@ -160,8 +189,10 @@ __global__ void draft_logits_kernel(FrameParams p, int pos_k, int n_j, const flo
   float acc = 0.f;
   for (int k = lane; k < p.H; k += 32) {
     const long long off = tiled_offset(g, id, k, p.wdtype);
-    const float w = p.wdtype == MCD_WEIGHT_BF16 ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(W)[off])
-                                                : reinterpret_cast<const float*>(W)[off];
+    const float w = p.wdtype == MCD_WEIGHT_BF16   ? bf16_bits_to_f32(reinterpret_cast<const uint16_t*>(W)[off])
+                    : p.wdtype == MCD_WEIGHT_INT8 ? (float)reinterpret_cast<const int8_t*>(W)[off] *
+                                                        p.s_head[(size_t)(pos_k + j - 1) * p.V + id]
+                                                  : reinterpret_cast<const float*>(W)[off];
     acc += w * (h[k] + p.offsets[(size_t)(j - 1) * p.H + k]);
   }
   for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
@@ -258,21 +289,28 @@ bool mcd::make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeom&
 }
 
 bool mcd::backbone_geom(FrameParams& p, int head_rows) {
-  const int tb = p.wdtype == MCD_WEIGHT_BF16 ? 512 : 1024;
-  bool ok = make_geom(p.qkv_dim, p.H, 1, tb, 1024, p.g[MAT_QKV]) && p.g[MAT_QKV].n_kc == 1;
+  // bytes per 16 x 16 tile; one-byte W8A16 tiles go two m-tiles per unit to keep units at 32 KB
+  const int tb = p.wdtype == MCD_WEIGHT_BF16 ? 512 : p.wdtype == MCD_WEIGHT_INT8 ? 256 : 1024;
+  const int mu = p.wdtype == MCD_WEIGHT_INT8 ? 2 : 1;
+  auto mu_for = [&](int rows) { return rows % (mu * 16) == 0 ? mu : 1; };
+  bool ok = make_geom(p.qkv_dim, p.H, mu_for(p.qkv_dim), tb, 1024, p.g[MAT_QKV]) && p.g[MAT_QKV].n_kc == 1;
   int mu_o = 8;
   while (mu_o > 1 && (mu_o * (p.D / 16) * tb > kSlotBytes || p.H % (mu_o * 16))) mu_o >>= 1;
   ok = ok && make_geom(p.H, p.NH * p.D, mu_o, tb, p.D, p.g[MAT_WO]) && p.g[MAT_WO].Ku * 16 == p.D;
-  ok = ok && make_geom(2 * p.F, p.H, 1, tb, 1024, p.g[MAT_GU]) && p.g[MAT_GU].n_kc == 1;
-  ok = ok && make_geom(p.H, p.F, 1, tb, 1024, p.g[MAT_WD]);
+  ok = ok && make_geom(2 * p.F, p.H, mu_for(2 * p.F), tb, 1024, p.g[MAT_GU]) && p.g[MAT_GU].n_kc == 1;
+  ok = ok && make_geom(p.H, p.F, mu_for(p.H), tb, 1024, p.g[MAT_WD]);
+  // (heads keep one m-tile per unit: the draft-offset bias tiles are staged per 16 rows)
   ok = ok && make_geom(head_rows, p.H, 1, tb, 1024, p.g[MAT_HEAD]) && p.g[MAT_HEAD].n_kc == 1;
   return ok;
 }
 
 void mcd::load_layer(const FrameParams& p, cudaStream_t stream, const LayerSrc& src, int l) {
   const int H = p.H, D = p.D, F = p.F, qd = p.NH * D, kd = p.NKV * D;
-  auto tile = [&](RowSrc rs, const MatGeom& g, const uint8_t* dst) {
-    tile_kernel<<<1024, 256, 0, stream>>>(rs, g, p.wdtype, const_cast<uint8_t*>(dst));
+  const bool q8 = p.wdtype == MCD_WEIGHT_INT8;
+  auto tile = [&](RowSrc rs, const MatGeom& g, const uint8_t* dst, const float* scale) {
+    float* sc = const_cast<float*>(scale);
+    if (q8) row_scale_kernel<<<(g.M * 32 + 255) / 256, 256, 0, stream>>>(rs, g, sc);
+    tile_kernel<<<1024, 256, 0, stream>>>(rs, g, p.wdtype, const_cast<uint8_t*>(dst), q8 ? sc : nullptr);
   };
   auto conv = [&](const uint8_t* from, int64_t count, const float* dst) {
     to_f32_kernel<<<64, 256, 0, stream>>>(from, p.wdtype, count, const_cast<float*>(dst));
@@ -286,26 +324,26 @@ void mcd::load_layer(const FrameParams& p, cudaStream_t stream, const LayerSrc& 
   rs.seg_rows[2] = kd;
   rs.nseg = 3;
   rs.src_cols = H;
-  tile(rs, p.g[MAT_QKV], p.w_qkv + (size_t)l * p.g[MAT_QKV].stride);
+  tile(rs, p.g[MAT_QKV], p.w_qkv + (size_t)l * p.g[MAT_QKV].stride, q8 ? p.s_qkv + (size_t)l * p.qkv_dim : nullptr);
   RowSrc ro{};
   ro.seg[0] = src.wo;
   ro.seg_rows[0] = H;
   ro.nseg = 1;
   ro.src_cols = qd;
-  tile(ro, p.g[MAT_WO], p.w_wo + (size_t)l * p.g[MAT_WO].stride);
+  tile(ro, p.g[MAT_WO], p.w_wo + (size_t)l * p.g[MAT_WO].stride, q8 ? p.s_wo + (size_t)l * H : nullptr);
   RowSrc rg{};
   rg.seg[0] = src.wg;
   rg.seg[1] = src.wu;
   rg.nseg = 2;
   rg.interleave_gu = 1;
   rg.src_cols = H;
-  tile(rg, p.g[MAT_GU], p.w_gu + (size_t)l * p.g[MAT_GU].stride);
+  tile(rg, p.g[MAT_GU], p.w_gu + (size_t)l * p.g[MAT_GU].stride, q8 ? p.s_gu + (size_t)l * 2 * F : nullptr);
   RowSrc rd{};
   rd.seg[0] = src.wd;
   rd.seg_rows[0] = H;
   rd.nseg = 1;
   rd.src_cols = F;
-  tile(rd, p.g[MAT_WD], p.w_wd + (size_t)l * p.g[MAT_WD].stride);
+  tile(rd, p.g[MAT_WD], p.w_wd + (size_t)l * p.g[MAT_WD].stride, q8 ? p.s_wd + (size_t)l * H : nullptr);
   conv(src.attn_norm, H, p.attn_norm + (size_t)l * H);
   conv(src.ffn_norm, H, p.ffn_norm + (size_t)l * H);
   if (p.qk_norm) {
@@ -325,7 +363,7 @@ static mcd_status validate_config(const mcd_config& c) {
   if (c.draft_len < 0 || c.draft_len > kMaxDraft) return MCD_ERR_UNSUPPORTED;
   if (c.top_k < 1 || c.top_k > kMaxTopK || c.top_k > c.vocab) return MCD_ERR_UNSUPPORTED;
   if (!(c.temperature > 0.f) || !(c.rms_eps > 0.f) || !(c.rope_base > 1.f)) return MCD_ERR_INVALID_ARG;
-  if (c.weight_dtype != MCD_WEIGHT_F32 && c.weight_dtype != MCD_WEIGHT_BF16) return MCD_ERR_INVALID_ARG;
+  if (c.weight_dtype < MCD_WEIGHT_F32 || c.weight_dtype > MCD_WEIGHT_INT8) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode < 0 || c.draft_mode > MCD_DRAFT_TREE) return MCD_ERR_INVALID_ARG;
   if (c.draft_mode == MCD_DRAFT_TREE && (c.max_streams != 1 || c.draft_len < 1)) return MCD_ERR_UNSUPPORTED;
   if (c.draft_mode == MCD_DRAFT_NOISY_TARGET && !(c.noise_sigma >= 0.f)) return MCD_ERR_INVALID_ARG;
@@ -419,7 +457,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   const char* wn = getenv("MCD_WAIT_NS");
   if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
 
-  const int es = k.weight_dtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  const int es = k.weight_dtype == MCD_WEIGHT_F32 ? 4 : 2;     // embedding tables (bf16 for W8A16)
   const bool ok = backbone_geom(p, p.V);
   if (!ok) return fail(MCD_ERR_UNSUPPORTED);
   p.ctr_stride = ctr_count(p.L);
@@ -453,6 +491,16 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.final_norm = p.k_norm + (size_t)p.L * p.D;
   p.offsets = p.final_norm + p.H;
 
+  if (k.weight_dtype == MCD_WEIGHT_INT8) {    // W8A16 row scales
+    const size_t ns = (size_t)p.L * (p.qkv_dim + 2 * p.H + 2 * p.F) + (size_t)p.P * p.V;
+    float* sc = nullptr;
+    if ((e = ctx_alloc(c, &sc, ns * 4)) != cudaSuccess) return fail(cuda_status(e));
+    p.s_qkv = sc;
+    p.s_wo = p.s_qkv + (size_t)p.L * p.qkv_dim;
+    p.s_gu = p.s_wo + (size_t)p.L * p.H;
+    p.s_wd = p.s_gu + (size_t)p.L * 2 * p.F;
+    p.s_head = p.s_wd + (size_t)p.L * p.H;
+  }
   float* head_bias = nullptr;
   if ((e = ctx_alloc(c, &head_bias, sizeof(float) * (size_t)p.P * Kd * p.V)) != cudaSuccess) return fail(cuda_status(e));
   p.head_bias = head_bias;
@@ -517,15 +565,18 @@ int32_t mcd_num_ctas(const mcd_ctx* c) { return c ? c->fp.n_cta : 0; }
 int64_t mcd_call_weight_bytes(const mcd_ctx* c, int32_t n_heads) {
   if (!c) return 0;
   const FrameParams& p = c->fp;
-  return (int64_t)p.L * (p.g[MAT_QKV].stride + p.g[MAT_WO].stride + p.g[MAT_GU].stride + p.g[MAT_WD].stride) +
-         (int64_t)n_heads * p.g[MAT_HEAD].stride;
+  int64_t b = (int64_t)p.L * (p.g[MAT_QKV].stride + p.g[MAT_WO].stride + p.g[MAT_GU].stride + p.g[MAT_WD].stride) +
+              (int64_t)n_heads * p.g[MAT_HEAD].stride;
+  if (p.wdtype == MCD_WEIGHT_INT8)   // + the row scales the epilogues read
+    b += 4LL * p.L * (p.qkv_dim + 2 * p.H + 2 * p.F) + 4LL * n_heads * p.V;
+  return b;
 }
 
 mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, const void* const* host_ptrs,
                             const int64_t* nbytes) {
   if (!c || n <= 0 || !names || !host_ptrs || !nbytes) return MCD_ERR_INVALID_ARG;
   FrameParams& p = c->fp;
-  const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+  const int es = p.wdtype == MCD_WEIGHT_F32 ? 4 : 2;           // source element bytes
   const int Kd = std::max(p.K, 1);
   std::map<std::string, std::pair<const void*, int64_t>> given;
   for (int i = 0; i < n; ++i) {
@@ -582,9 +633,11 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
       return cleanup(MCD_ERR_CUDA);
   }
   auto S = [&](const std::string& name) { return (const uint8_t*)(stage + soff[name]); };
-  auto tile = [&](RowSrc rs, const MatGeom& g, uint8_t* dst) {
-    tile_kernel<<<1024, 256, 0, c->stream>>>(rs, g, p.wdtype, dst);
+  auto tile = [&](RowSrc rs, const MatGeom& g, uint8_t* dst, float* scale) {
+    if (scale) row_scale_kernel<<<(g.M * 32 + 255) / 256, 256, 0, c->stream>>>(rs, g, scale);
+    tile_kernel<<<1024, 256, 0, c->stream>>>(rs, g, p.wdtype, dst, scale);
   };
+  const bool q8 = p.wdtype == MCD_WEIGHT_INT8;
   auto conv = [&](const std::string& name, int64_t count, const float* dst) {
     to_f32_kernel<<<64, 256, 0, c->stream>>>(S(name), p.wdtype, count, const_cast<float*>(dst));
   };
@@ -597,19 +650,21 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
   }
   conv("final_norm", H, p.final_norm);
   for (int j = 1; j <= Kd; ++j) conv("offset." + std::to_string(j), H, p.offsets + (size_t)(j - 1) * H);
-  for (int P = 1; P <= p.P && p.K > 0; ++P) {
-    const int warps = p.K * p.V;
-    head_bias_kernel<<<(warps * 32 + 255) / 256, 256, 0, c->stream>>>(
-        S("head." + std::to_string(P)), p.offsets, p.K, p.V, p.H, p.wdtype,
-        const_cast<float*>(p.head_bias) + (size_t)(P - 1) * p.K * p.V);
-  }
+  // LM heads (W8A16: row scales first, which the draft-offset biases also use)
   for (int P = 1; P <= p.P; ++P) {
     RowSrc rh{};
     rh.seg[0] = S("head." + std::to_string(P));
     rh.seg_rows[0] = p.V;
     rh.nseg = 1;
     rh.src_cols = (int)H;
-    tile(rh, p.g[MAT_HEAD], c->w_arena + c->off_head + (size_t)(P - 1) * p.g[MAT_HEAD].stride);
+    tile(rh, p.g[MAT_HEAD], c->w_arena + c->off_head + (size_t)(P - 1) * p.g[MAT_HEAD].stride,
+         q8 ? const_cast<float*>(p.s_head) + (size_t)(P - 1) * p.V : nullptr);
+  }
+  for (int P = 1; P <= p.P && p.K > 0; ++P) {
+    const int warps = p.K * p.V;
+    head_bias_kernel<<<(warps * 32 + 255) / 256, 256, 0, c->stream>>>(
+        S("head." + std::to_string(P)), p.offsets, p.K, p.V, p.H, p.wdtype, q8 ? p.s_head + (size_t)(P - 1) * p.V : nullptr,
+        const_cast<float*>(p.head_bias) + (size_t)(P - 1) * p.K * p.V);
   }
   if (p.C0V > 0)
     if (cudaMemcpyAsync(c->w_arena + c->off_embed, S("embed.0"), (size_t)p.C0V * H * es, cudaMemcpyDeviceToDevice,

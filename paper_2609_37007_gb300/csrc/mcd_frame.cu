@@ -522,7 +522,7 @@ __device__ void run_call(Cons& c, int call) {
       run_stage<WT, WIDE>(c, call, 4 * l + 0, g.n_units, H, n_rows, no_key, no_prep,
                     [&](int u, int mi, int rr, int n, float v, float) {
                       const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-                      p.qkv[(size_t)n * p.qkv_dim + row] = v * sm.inv_rms[n];
+                      p.qkv[(size_t)n * p.qkv_dim + row] = v * sm.inv_rms[n] * wscale<WT>(p.s_qkv, (size_t)l * p.qkv_dim + row);
                     });
       if (c.abort_) return;
     }
@@ -573,7 +573,7 @@ __device__ void run_call(Cons& c, int call) {
           },
           [&](int u, int mi, int rr, int n, float v, float) {
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v);
+            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wo, (size_t)l * H + row));
           });
       if (c.abort_) return;
     } else {
@@ -597,7 +597,7 @@ __device__ void run_call(Cons& c, int call) {
           },
           [&](int u, int mi, int rr, int n, float v, float) {
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v);
+            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wo, (size_t)l * H + row));
           });
       if (c.abort_) return;
     }
@@ -615,9 +615,11 @@ __device__ void run_call(Cons& c, int call) {
           c, call, 4 * l + 2, g.n_units, H, n_rows, no_key, no_prep,
           [&](int u, int mi, int rr, int n, float gate, float up) {
             const float s = sm.inv_rms[n];
-            const float gt = gate * s;
+            const int t16 = ((u % g.n_mb) * g.Mu + mi) * 16 + rr;      // tiled row of the gate
+            const float gt = gate * s * wscale<WT>(p.s_gu, (size_t)l * 2 * F + t16);
+            const float ut = up * s * wscale<WT>(p.s_gu, (size_t)l * 2 * F + t16 + 8);
             const int j = ((u % g.n_mb) * g.Mu + mi) * 8 + rr;
-            p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * (up * s);
+            p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * ut;
           },
           true);
       if (c.abort_) return;
@@ -644,7 +646,7 @@ __device__ void run_call(Cons& c, int call) {
           },
           [&](int u, int mi, int rr, int n, float v, float) {
             const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v);
+            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wd, (size_t)l * H + row));
           });
       if (c.abort_) return;
     }
@@ -688,7 +690,8 @@ __device__ void run_call(Cons& c, int call) {
           if (pos >= 1 && j >= 0 && j <= p.K) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
             p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
-                v * sm.inv_rms[n] + bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
+                v * sm.inv_rms[n] * wscale<WT>(p.s_head, (size_t)(P - 1) * p.V + id) +
+                bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
           }
         });
     if (c.abort_) return;
@@ -1371,9 +1374,9 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
         atomicCAS(p.err, 0, (int)MCD_ERR_INVALID_ARG);
         id = 0;
       }
-      const int es = p.wdtype == MCD_WEIGHT_BF16 ? 2 : 4;
+      const int es = p.wdtype == MCD_WEIGHT_F32 ? 4 : 2;      // embedding tables: bf16 unless fp32
       ci->r_src[r] = p.embed + (long long)table * p.embed_stride + (long long)id * p.H * es;
-      ci->r_f32[r] = p.wdtype == MCD_WEIGHT_BF16 ? 0 : 1;
+      ci->r_f32[r] = p.wdtype == MCD_WEIGHT_F32 ? 1 : 0;
     }
     ci->r_s[r] = s;
     ci->r_n[r] = n;
@@ -1438,22 +1441,29 @@ static void* frame_entry() {
   return (void*)frame_kernel<WT, WIDE>;
 }
 
+static void* frame_fn(int wdtype, bool wide) {
+  switch (wdtype) {
+    case MCD_WEIGHT_BF16: return wide ? frame_entry<MCD_WEIGHT_BF16, true>() : frame_entry<MCD_WEIGHT_BF16, false>();
+    case MCD_WEIGHT_INT8: return wide ? frame_entry<MCD_WEIGHT_INT8, true>() : frame_entry<MCD_WEIGHT_INT8, false>();
+    default: return wide ? frame_entry<MCD_WEIGHT_F32, true>() : frame_entry<MCD_WEIGHT_F32, false>();
+  }
+}
+
 cudaError_t launch_frame_kernel(const FrameParams& p, cudaStream_t stream) {
   void* args[] = {const_cast<FrameParams*>(&p)};
   const bool wide = p.S * max(p.K + 1, 2) > kMaxRows || p.draft_mode == MCD_DRAFT_TREE;
-  void* fn = p.wdtype == MCD_WEIGHT_BF16 ? (wide ? frame_entry<MCD_WEIGHT_BF16, true>() : frame_entry<MCD_WEIGHT_BF16, false>())
-                                         : (wide ? frame_entry<MCD_WEIGHT_F32, true>() : frame_entry<MCD_WEIGHT_F32, false>());
-  return cudaLaunchCooperativeKernel(fn, dim3(p.n_cta), dim3(kThreads), args, (size_t)kSmemBytes, stream);
+  return cudaLaunchCooperativeKernel(frame_fn(p.wdtype, wide), dim3(p.n_cta), dim3(kThreads), args, (size_t)kSmemBytes,
+                                     stream);
 }
 
 cudaError_t prepare_frame_kernel(int* max_ctas_per_sm) {
-  void* fns[4] = {frame_entry<MCD_WEIGHT_BF16, false>(), frame_entry<MCD_WEIGHT_BF16, true>(),
-                  frame_entry<MCD_WEIGHT_F32, false>(), frame_entry<MCD_WEIGHT_F32, true>()};
-  for (void* fn : fns) {
-    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (e != cudaSuccess) return e;
-  }
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(max_ctas_per_sm, fns[0], kThreads, kSmemBytes);
+  for (int wd : {MCD_WEIGHT_F32, MCD_WEIGHT_BF16, MCD_WEIGHT_INT8})
+    for (bool wide : {false, true}) {
+      cudaError_t e = cudaFuncSetAttribute(frame_fn(wd, wide), cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+      if (e != cudaSuccess) return e;
+    }
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(max_ctas_per_sm, frame_fn(MCD_WEIGHT_BF16, false), kThreads,
+                                                       kSmemBytes);
 }
 
 int frame_smem_bytes() { return kSmemBytes; }

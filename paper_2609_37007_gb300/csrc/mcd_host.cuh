@@ -26,7 +26,7 @@ __host__ __device__ inline long long tiled_offset(const MatGeom& g, int r, int c
   const long long tile = (u * g.Mu + mi) * g.Ku + kt;
   const int rr = r & 15, cc = c & 15;
   int pos;
-  if (wdtype == MCD_WEIGHT_BF16) {
+  if (wdtype != MCD_WEIGHT_F32) {          // bf16 / int8: mma.m16n8k16 A-fragment order
     const int lane = (rr & 7) * 4 + ((cc & 7) >> 1);
     const int reg = (rr >> 3) + 2 * (cc >> 3);
     pos = lane * 8 + reg * 2 + (cc & 1);
@@ -36,7 +36,11 @@ __host__ __device__ inline long long tiled_offset(const MatGeom& g, int r, int c
   return tile * 256 + pos;
 }
 
-__global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst);
+// Re-tile a row-major matrix (source elements: fp32 for MCD_WEIGHT_F32, else bf16); for
+// MCD_WEIGHT_INT8 the elements are quantised with the per-row `scale` (see row_scale_kernel).
+__global__ void tile_kernel(RowSrc rs, MatGeom g, int wdtype, uint8_t* dst, const float* scale);
+// W8A16 row scales of a matrix in tiled row order: scale[r] = fp32(max |w_r| / 127).
+__global__ void row_scale_kernel(RowSrc rs, MatGeom g, float* scale);
 __global__ void to_f32_kernel(const uint8_t* src, int wdtype, long long n, float* dst);
 // (cos, sin) of position pos and frequency i for pos < n_pos: [n_pos][D/2].
 __global__ void rope_kernel(float2* rope, int D, double base, int n_pos);
@@ -45,7 +49,8 @@ bool make_geom(int M, int K, int Mu, int tile_bytes, int max_cols, MatGeom& g);
 // Unit geometry of the backbone matrices and of an LM head with `head_rows` outputs.
 bool backbone_geom(FrameParams& p, int head_rows);
 
-// Device copies of one layer's source tensors (row-major, weight dtype).
+// Device copies of one layer's source tensors (row-major, weight dtype); W8A16 scale arrays
+// of the layer (null unless MCD_WEIGHT_INT8).
 struct LayerSrc {
   const uint8_t *wq, *wk, *wv, *wo, *wg, *wu, *wd, *attn_norm, *ffn_norm, *q_norm, *k_norm;
 };

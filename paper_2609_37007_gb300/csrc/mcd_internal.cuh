@@ -9,6 +9,9 @@
 //     [k-chunk][m-block]; tiles inside a unit [m-tile][k-tile].
 //   * Embedding tables stay row-major [vocab, hidden] in the weight dtype (row gather).
 //   * Norm gains and offsets are fp32.  Activations, KV cache and logits are fp32.
+//   * W8A16 (MCD_WEIGHT_INT8): the same tiles with one byte per element (256 B per tile, in
+//     the bf16 tile's element order) and one fp32 scale per output row; the unit GEMMs widen
+//     the bytes to bf16 in registers and the epilogues apply the row scale.
 #pragma once
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -127,6 +130,12 @@ struct FrameParams {
   const uint8_t* w_gu;
   const uint8_t* w_wd;
   const uint8_t* w_head;       // + (P-1) * g[MAT_HEAD].stride
+  // W8A16: per tiled output row scales (null otherwise)
+  const float* s_qkv;          // [L][qkv_dim]
+  const float* s_wo;           // [L][H]
+  const float* s_gu;           // [L][2F], tiled row order (gate rows 16t..16t+7, up rows +8)
+  const float* s_wd;           // [L][H]
+  const float* s_head;         // [n_pos][V]
   const float* attn_norm;      // [L][H]
   const float* ffn_norm;       // [L][H]
   const float* q_norm;         // [L][D]
@@ -269,6 +278,24 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return d;
 }
 __device__ __forceinline__ float bf16_lo_f32(uint32_t w) { return __uint_as_float(w << 16); }
+// Output-row scale of a W8A16 matrix (1 for 16- and 32-bit weights).
+template <int WT>
+__device__ __forceinline__ float wscale(const float* s, size_t i) {
+  if (WT == MCD_WEIGHT_INT8) return __ldg(s + i);
+  return 1.f;
+}
+
+// Eight signed bytes (an A fragment of a W8A16 tile) as eight bf16 values, exactly
+// (|q| <= 127 needs 7 mantissa bits): bytes 2i, 2i+1 -> bf16 pair i (low half first).
+__device__ __forceinline__ uint4 widen_i8x8(uint2 q) {
+  auto pair = [](uint32_t w, int sh) {
+    const float lo = (float)(int)(signed char)(w >> sh), hi = (float)(int)(signed char)(w >> (sh + 8));
+    uint32_t d;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+    return d;
+  };
+  return make_uint4(pair(q.x, 0), pair(q.x, 16), pair(q.y, 0), pair(q.y, 16));
+}
 __device__ __forceinline__ float bf16_hi_f32(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ void split_bf16(float x, uint32_t& hi, uint32_t& lo) {
   hi = bf16_rn_bits(x);

@@ -644,6 +644,7 @@ static mcd_status validate_outer(const mcd_outer_config& c, const FrameParams& i
   if (c.top_k < 1 || c.top_k > kMaxTopK || c.top_k > c.c0_vocab) return MCD_ERR_UNSUPPORTED;
   if (!(c.temperature > 0.f) || !(c.rms_eps > 0.f) || !(c.rope_base > 1.f)) return MCD_ERR_INVALID_ARG;
   if (c.weight_dtype != ip.wdtype) return MCD_ERR_INVALID_ARG;   // the frame sum reads the inner tables
+  if (c.weight_dtype == MCD_WEIGHT_INT8) return MCD_ERR_UNSUPPORTED;
   if (ip.C0V != 0) return MCD_ERR_INVALID_ARG;                   // the inner model takes the c0 vector
   return MCD_OK;
 }
@@ -888,7 +889,7 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
   rh.seg_rows[0] = p.V;
   rh.nseg = 1;
   rh.src_cols = (int)H;
-  tile_kernel<<<1024, 256, 0, o->stream>>>(rh, p.g[MAT_HEAD], p.wdtype, const_cast<uint8_t*>(p.w_head));
+  tile_kernel<<<1024, 256, 0, o->stream>>>(rh, p.g[MAT_HEAD], p.wdtype, const_cast<uint8_t*>(p.w_head), nullptr);
   to_f32_kernel<<<64, 256, 0, o->stream>>>(at["final_norm"], p.wdtype, H, const_cast<float*>(p.final_norm));
   // row-major tables go straight to their arrays
   auto table = [&](const std::string& name, const uint8_t* dst) {

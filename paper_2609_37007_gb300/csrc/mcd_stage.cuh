@@ -273,7 +273,7 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
           x89.x *= g89.x;
           x89.y *= g89.y;
         }
-        if (WT == MCD_WEIGHT_BF16) {
+        if (WT != MCD_WEIGHT_F32) {
           const int entry = ((kt0 + kt) * NT + (n >> 3)) * 32 + 4 * (n & 7) + t;
           const uint32_t h01 = pack_bf16x2(x01.x, x01.y), h89 = pack_bf16x2(x89.x, x89.y);
           if (hilo) {
@@ -343,8 +343,13 @@ __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const WarpRo
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Ku = g.Ku, kt0 = kc * Ku + w.kg * w.kts;
   float4* red = reinterpret_cast<float4*>(c.sm.red) + ((size_t)r * kConsumerWarps + warp) * w.ntpw * 32;
-  if (WT == MCD_WEIGHT_BF16) {
-    const uint4* A = reinterpret_cast<const uint4*>(slotp) + (size_t)(w.mi * Ku + w.kg * w.kts) * 32 + lane;
+  if (WT != MCD_WEIGHT_F32) {
+    // A fragment of k-tile t: 16 bytes per lane (bf16) or 8 bytes widened to bf16 (W8A16)
+    const size_t a0i = (size_t)(w.mi * Ku + w.kg * w.kts) * 32 + lane;
+    auto load_a = [&](int t) -> uint4 {
+      if (WT == MCD_WEIGHT_BF16) return reinterpret_cast<const uint4*>(slotp)[a0i + (size_t)t * 32];
+      return widen_i8x8(reinterpret_cast<const uint2*>(slotp)[a0i + (size_t)t * 32]);
+    };
     const int ntpw = WIDE ? w.ntpw : 1;
     for (int ntl = 0; ntl < ntpw; ++ntl) {
       const int nt = WIDE ? w.gn * w.ntpw + ntl : 0;
@@ -353,7 +358,7 @@ __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const WarpRo
         const uint4* B = reinterpret_cast<const uint4*>(c.op) + ((size_t)kt0 * NT + nt) * 32 + lane;
 #pragma unroll 8
         for (int t = 0; t < w.kts; ++t) {
-          const uint4 a = A[t * 32];
+          const uint4 a = load_a(t);
           const uint4 bb = B[(size_t)t * NT * 32];
           mma_bf16_16816(a0, a, bb.x, bb.y);
           mma_bf16_16816(a1, a, bb.z, bb.w);
@@ -362,11 +367,11 @@ __device__ __forceinline__ void unit_mma(Cons& c, const MatGeom& g, const WarpRo
         const uint2* B = reinterpret_cast<const uint2*>(c.op) + ((size_t)kt0 * NT + nt) * 32 + lane;
 #pragma unroll 8
         for (int t = 0; t < w.kts; t += 2) {
-          const uint4 a = A[t * 32];
+          const uint4 a = load_a(t);
           const uint2 bb = B[(size_t)t * NT * 32];
           mma_bf16_16816(a0, a, bb.x, bb.y);
           if (t + 1 < w.kts) {
-            const uint4 a2 = A[(t + 1) * 32];
+            const uint4 a2 = load_a(t + 1);
             const uint2 b2 = B[(size_t)(t + 1) * NT * 32];
             mma_bf16_16816(a1, a2, b2.x, b2.y);
           }
@@ -440,7 +445,7 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
   const UnitRange ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
   const int NT = WIDE ? n_tiles(ncols) : 1;
   const bool hilo = WIDE ? hilo_operand(ncols) : true;
-  const WarpRole role = warp_role(g, NT, threadIdx.x >> 5, WIDE && WT == MCD_WEIGHT_BF16);
+  const WarpRole role = warp_role(g, NT, threadIdx.x >> 5, WIDE && WT != MCD_WEIGHT_F32);
   const int per_unit = kConsumerWarps * role.ntpw * 512;                            // bytes of partials
   const int cap = max(1, min(kChunk, kRedBytes / per_unit));
   const int lgm = g.Mu == 1 ? 0 : g.Mu == 2 ? 1 : g.Mu == 4 ? 2 : 3;

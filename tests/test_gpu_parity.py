@@ -48,7 +48,11 @@ class Env:
     @property
     def model(self):
         if self._model is None:
-            self._model = Model(self.cfg, weights_as_f32(self.cfg, self.w))
+            w = weights_as_f32(self.cfg, self.w)
+            if self.cfg.weight_dtype == 2:                 # W8A16: the values the library computes with
+                from oracle.quant import w8a16_weights
+                w = w8a16_weights(w)
+            self._model = Model(self.cfg, w)
         return self._model
 
     def frame_inputs(self, fr):
@@ -513,6 +517,58 @@ def test_draft_api_matches_oracle(tiny):
             assert int(ids[j - 1]) == draw(q, S.u(4, k_pos + j, 2))
             assert q_ids.cpu().numpy()[j - 1].tolist() == q.ids
             assert [int(v) for v in q_w.cpu().numpy().view(np.uint32)[j - 1]] == q.W
+
+
+# ------------------------------------------------- W8A16 weight streaming -------------
+@pytest.mark.parametrize("variant", ["tiny", "tiny_k0", "tiny_greedy"])
+def test_w8a16_trace_parity_tiny(variant):
+    """int8 weights quantised per row at load (R-Q1): every call against the oracle computing
+    with q * s (1e-4: the activations enter the tensor cores as bf16 hi + lo pairs)."""
+    cfg = {"tiny": TINY, "tiny_k0": TINY.replace(draft_len=0),
+           "tiny_greedy": TINY.replace(draft_mode=DRAFT_GREEDY)}[variant].replace(weight_dtype=2)
+    env = Env(cfg)
+    worst = 0.0
+    for f in range(5):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        worst = max(worst, check_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]),
+                                                      logit_tol=1e-4))
+    print(variant, "w8a16 max |dlogit|", worst)
+    env.dec.close()
+
+
+def test_w8a16_heads_are_quantised_like_the_oracle():
+    """mcd_draft reads the int8 LM heads and their row scales directly: its draft logits
+    equal the oracle's with the same q * s heads to fp32 rounding, so every quantised weight
+    of the heads (and the draft offsets' bias) matches R-Q1."""
+    cfg = TINY.replace(weight_dtype=2)
+    env = Env(cfg)
+    _begin(env.dec, cfg, 0, 0)
+    h = np.random.default_rng(8).standard_normal(cfg.hidden).astype(np.float32)
+    K = cfg.draft_len
+    ids = torch.zeros(K, dtype=torch.int32, device=DEV)
+    z = torch.zeros((K, cfg.vocab), dtype=torch.float32, device=DEV)
+    for k_pos in (1, 2):
+        mcd.mcd_draft(env.dec.ctx, k_pos, 0, t(h), ids, None, None, z)
+        mcd.mcd_sync(env.dec.ctx)
+        zz = z.cpu().numpy()
+        for j in range(1, min(K, cfg.n_pos - k_pos) + 1):
+            ref = env.model.draft_logits(k_pos, j, h.astype(np.float64))
+            assert np.max(np.abs(zz[j - 1] - ref)) < 2e-6
+    env.dec.close()
+
+
+def test_w8a16_full_size():
+    cfg = MCD.replace(weight_dtype=2)
+    env = Env(cfg)
+    for f in (0, 1):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        err = check_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=2e-2)
+        print("w8a16 full size max |dlogit|", err)
+    env.dec.close()
 
 
 def test_bad_c0_fails_the_frame_without_faulting(big):
