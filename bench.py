@@ -125,6 +125,25 @@ def stored_traffic(digest: str, bytes_per_launch: float):
     return ratio * bytes_per_launch, f"ncu dram bytes of one captured launch x {ratio:.4f} of algorithmic"
 
 
+# ---- replicas (one stream per rank, no collective on the data path) -------------------------
+def replica_first_frame(rank: int) -> int:
+    """Index of the first synthetic frame of rank `rank`: every replica decodes its own inputs."""
+    return rank * 1_000_000
+
+
+def combine_ranks(elapsed: float, tokens: int, calls: int, dist=None, device=None):
+    """Whole-job figures over the ranks: the slowest rank's timed region, the summed tokens
+    and calls (the only collectives of a multi-GPU run)."""
+    if dist is None:
+        return elapsed, tokens, calls
+    import torch
+    t = torch.tensor([elapsed, tokens, calls], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(mx[0]), int(t[1]), int(t[2])
+
+
 # ----------------------------------------------------------------------------------------
 def cpu_oracle_baseline(cfg, weights, budget_s: float, first_frame: int):
     """The oracle as it stands on the host cores, whole frames until budget_s is spent."""
@@ -596,7 +615,7 @@ def main():
     dec = mcd.Decoder(cfg, weights, stream)
     ctx = dec.ctx
     n_frames = args.warmup + args.steps
-    cond_h, c0_h, _ = make_frames(cfg, n_frames, first=rank * 1_000_000)
+    cond_h, c0_h, _ = make_frames(cfg, n_frames, first=replica_first_frame(rank))
     cond = torch.from_numpy(cond_h).to(dev)
     c0 = torch.from_numpy(c0_h).to(dev)
     codes = torch.zeros((n_frames, cfg.n_pos), dtype=torch.int32, device=dev)
@@ -629,14 +648,7 @@ def main():
     assert (st[:, 4] == 0).all() and (st[:, 1] == cfg.n_pos).all(), "device-side failure"
     tokens = int(st[:, 1].sum())
     calls = int(st[:, 0].sum())
-    if dist:
-        t = torch.tensor([elapsed, tokens, calls], dtype=torch.float64, device=dev)
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        elapsed_all, tokens_all, calls_all = float(mx[0]), int(t[1]), int(t[2])
-    else:
-        elapsed_all, tokens_all, calls_all = elapsed, tokens, calls
+    elapsed_all, tokens_all, calls_all = combine_ranks(elapsed, tokens, calls, dist, dev)
 
     # ---- roofline of the frame kernel ---------------------------------------------------
     backbone = mcd.mcd_call_weight_bytes(ctx, 0)
