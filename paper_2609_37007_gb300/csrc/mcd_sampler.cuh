@@ -18,6 +18,11 @@
 namespace mcd {
 
 struct TopkScratch {
+  static constexpr int kBins = 256;
+  uint32_t hist[kBins];                  // value-range histogram
+  uint32_t cand[32];                     // keys of the threshold bin
+  uint32_t ncand;
+  uint32_t mm[2][kConsumerWarps];        // per-warp maximum / minimum key
   uint32_t part[2][kConsumerWarps][8];   // per-warp counts of the threshold search (double-buffered)
   uint32_t wred[2][kConsumerWarps];      // per-warp maxima / scan totals (double-buffered)
   unsigned long long wsum[kConsumerWarps];
@@ -96,12 +101,20 @@ __device__ __forceinline__ uint32_t block_exscan(uint32_t v, TopkScratch& s, int
 }
 
 // Block-wide (256 consumer threads) top-k of one fp32 row (V % 16 == 0, V <= 4096) into `out`
-// (global or shared), listed in ascending id order.  Thread t holds the keys of ids
-// 4t + 1024j + c (j < 4, c < 4) in registers.  The k-th largest key is found by a counting
-// search, 3 bits per step (seven thresholds per step, counts reduced with redux.sync, one
-// barrier per step); the set is then compacted in id order (ties at the threshold keep the
-// lowest ids).  `greedy` replaces the distribution by the one-hot of the argmax.  `dbg`, when
-// not null, receives clock64() stamps at the six phase boundaries (profiling only).
+// (global or shared), listed in ascending id order.  Thread t holds the keys of the E = 4 nj
+// consecutive ids E t .. E t + E - 1 (nj = ceil(V / 1024)) in registers, so thread order is id
+// order.  Finding the k-th largest key Tk:
+//   (1) block maximum and minimum;
+//   (2) a 256-bin histogram over the value range [min, max] (bin = trunc((v - min) * 256 /
+//       (max - min)), a monotone function of the key, so every bin is an interval of keys);
+//   (3) every warp scans the histogram from the top for the bin B holding the k-th largest
+//       key; when B holds at most 32 keys they are gathered and one warp ranks them exactly;
+//       otherwise (or for a non-finite range) a counting search over key thresholds, 3 bits
+//       per step, finds Tk;
+//   (4) one prefix scan of the packed per-thread counts (keys > Tk, keys == Tk) places the
+//       set in id order (ties at the threshold keep the lowest ids) and gives every weight.
+// `greedy` replaces the distribution by the one-hot of the argmax (ties: lowest id).  `dbg`,
+// when not null, receives clock64() stamps at the phase boundaries (profiling only).
 static __device__ __forceinline__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
                                   TopkScratch& s, TopkRec* out, long long* dbg = nullptr) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -109,24 +122,26 @@ static __device__ __forceinline__ void block_topk(const float* __restrict__ logi
   if (dbg && tid == 0) dbg[i] = clock64();
   MCD_TOPK_STAMP(0)
   constexpr int kJ = kMaxVocab / 1024;
+  constexpr int kBins = TopkScratch::kBins;
+  static_assert(kBins == kConsumerThreads, "one histogram bin per consumer thread");
+  const int nj = (V + 1023) >> 10;                 // float4 chunks per thread
+  const int E = 4 * nj;                            // ids per thread
+  const int n_valid = max(0, min(E, V - E * tid)); // ids E*tid .. E*tid + n_valid - 1 exist
   uint32_t key[4 * kJ];
 #pragma unroll
   for (int j = 0; j < kJ; ++j) {
-    const int i4 = tid + kConsumerThreads * j;
+    const bool ok = 4 * j < n_valid;
     float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    const bool ok = 4 * i4 < V;
-    if (ok) v = __ldcg(reinterpret_cast<const float4*>(logits) + i4);
-    key[4 * j + 0] = ok ? f32_key(v.x) : 0u;   // key 0 (a NaN pattern) is never counted
+    if (ok) v = __ldcg(reinterpret_cast<const float4*>(logits) + (nj * tid + j));
+    key[4 * j + 0] = ok ? f32_key(v.x) : 0u;
     key[4 * j + 1] = ok ? f32_key(v.y) : 0u;
     key[4 * j + 2] = ok ? f32_key(v.z) : 0u;
     key[4 * j + 3] = ok ? f32_key(v.w) : 0u;
   }
-  // block maximum and minimum (padding keys: 0 never wins the maximum, ~0 never the minimum)
-  const int nj = (V + 1023) >> 10;
   uint32_t kmax = 0, kmin = 0xFFFFFFFFu;
 #pragma unroll
   for (int e = 0; e < 4 * kJ; ++e) {
-    if ((e >> 2) < nj) {
+    if (e < n_valid) {
       kmax = max(kmax, key[e]);
       kmin = min(kmin, key[e]);
     }
@@ -134,167 +149,199 @@ static __device__ __forceinline__ void block_topk(const float* __restrict__ logi
   kmax = __reduce_max_sync(0xFFFFFFFFu, kmax);
   kmin = __reduce_min_sync(0xFFFFFFFFu, kmin);
   if (lane == 0) {
-    s.wred[0][warp] = kmax;
-    s.wred[1][warp] = kmin;
+    s.mm[0][warp] = kmax;
+    s.mm[1][warp] = kmin;
   }
+  s.hist[tid] = 0u;
+  if (tid == 0) s.ncand = 0u;
   consumer_sync();
 #pragma unroll
   for (int w = 0; w < kConsumerWarps; ++w) {
-    kmax = max(kmax, s.wred[0][w]);
-    kmin = min(kmin, s.wred[1][w]);
+    kmax = max(kmax, s.mm[0][w]);
+    kmin = min(kmin, s.mm[1][w]);
   }
   MCD_TOPK_STAMP(1)
-  // Counting search for the k-th largest key.  Invariant: #(key >= lo) >= k > #(key >= hi).
-  // Each step counts 7 thresholds splitting [lo, hi) into eighths (one barrier); it stops
-  // early when a threshold has exactly k keys at or above it (then that set is the answer
-  // and no tie needs splitting), else when hi = lo + 1 (lo is the k-th largest key).
-  uint32_t lo = kmin;
-  unsigned long long hi = (unsigned long long)kmax + 1ull;
-  int buf = 0;
-  while (hi - lo > 1ull) {
-    const unsigned long long span = hi - lo;
-    uint32_t cnt[7];
-#pragma unroll
-    for (int i = 0; i < 7; ++i) {
-      const uint32_t t = lo + (uint32_t)((span * (unsigned long long)(i + 1)) >> 3);
-      uint32_t c = 0;
-#pragma unroll
-      for (int e = 0; e < 4 * kJ; ++e)
-        if ((e >> 2) < nj) c += key[e] >= t ? 1u : 0u;
-      cnt[i] = __reduce_add_sync(0xFFFFFFFFu, c);
-    }
-    if (lane < 7) {
-      uint32_t mine = cnt[0];
-#pragma unroll
-      for (int i = 1; i < 7; ++i) mine = lane == i ? cnt[i] : mine;
-      s.part[buf][warp][lane] = mine;
-    }
-    consumer_sync();
-    uint32_t tot = 0;
-    if (lane < 7)
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) tot += s.part[buf][w][lane];
-    const uint32_t my_t = lo + (uint32_t)((span * (unsigned long long)(lane + 1)) >> 3);
-    const unsigned ge = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot >= (uint32_t)k);
-    const unsigned eq = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot == (uint32_t)k);
-    buf ^= 1;
-    if (eq) {                                           // exactly k keys >= that threshold
-      lo = __shfl_sync(0xFFFFFFFFu, my_t, __ffs(eq) - 1);
-      break;
-    }
-    // thresholds are increasing in lane, counts decreasing: ge is a prefix of lanes 0..6
-    const int nge = __popc(ge);
-    const uint32_t new_lo = __shfl_sync(0xFFFFFFFFu, my_t, max(nge - 1, 0));
-    const uint32_t new_hi = __shfl_sync(0xFFFFFFFFu, my_t, min(nge, 6));
-    if (nge > 0) lo = new_lo;
-    if (nge < 7) hi = new_hi;
-  }
-  const uint32_t Tk = lo;
-  MCD_TOPK_STAMP(2)
-  // counts above and at the threshold
-  uint32_t c_gt = 0, c_eq = 0;
-#pragma unroll
-  for (int e = 0; e < 4 * kJ; ++e) {
-    c_gt += key[e] > Tk ? 1u : 0u;
-    c_eq += key[e] == Tk ? 1u : 0u;
-  }
-  c_gt = __reduce_add_sync(0xFFFFFFFFu, c_gt);
-  c_eq = __reduce_add_sync(0xFFFFFFFFu, c_eq);
-  if (lane == 0) {
-    s.part[buf][warp][0] = c_gt;
-    s.part[buf][warp][1] = c_eq;
-  }
-  consumer_sync();
-  uint32_t n_gt = 0, n_eq = 0;
-#pragma unroll
-  for (int w = 0; w < kConsumerWarps; ++w) {
-    n_gt += s.part[buf][w][0];
-    n_eq += s.part[buf][w][1];
-  }
-  const uint32_t krem = (uint32_t)k - n_gt;      // >= 1 threshold keys to keep, lowest ids first
-  const bool all_eq = n_eq == krem;
-  MCD_TOPK_STAMP(3)
-  // id-ordered compaction with weights
-  const float Td = T;
-  const float zmax = __fdiv_rn(key_f32(kmax), Td);
-  uint32_t base = 0, tie_base = 0;
-  unsigned long long wsum = 0;
-  int sbuf = 1;
-#pragma unroll
-  for (int j = 0; j < kJ; ++j) {
-    if (1024 * j >= V) break;                    // block-uniform
-    bool inc[4];
-    uint32_t n_inc = 0, n_tie = 0;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) n_tie += key[4 * j + c] == Tk ? 1u : 0u;
-    uint32_t tie_pre = 0;
-    if (!all_eq) {
-      uint32_t tot;
-      tie_pre = tie_base + block_exscan(n_tie, s, sbuf, &tot);
-      sbuf ^= 1;
-      tie_base += tot;
-    }
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const uint32_t kv = key[4 * j + c];
-      const bool eq = kv == Tk;
-      inc[c] = kv > Tk || (eq && (all_eq || tie_pre < krem));
-      tie_pre += eq ? 1u : 0u;
-      n_inc += inc[c] ? 1u : 0u;
-    }
-    uint32_t tot;
-    uint32_t pos = base + block_exscan(n_inc, s, sbuf, &tot);
-    sbuf ^= 1;
-    base += tot;
-    if (!greedy) {
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        if (inc[c]) {
-          const float z = __fdiv_rn(key_f32(key[4 * j + c]), Td);
-          const uint32_t w = weight24(exp32_cw(__fsub_rn(z, zmax)));
-          out->ids[pos] = 4 * (tid + kConsumerThreads * j) + c;
-          out->W[pos] = w;
-          wsum += w;
-          ++pos;
-        }
-      }
-    }
-  }
-  MCD_TOPK_STAMP(4)
   if (greedy) {
-    // argmax, ties to the lowest id
+    // argmax, ties to the lowest id (thread order is id order)
     uint32_t best = 0xFFFFFFFFu;
 #pragma unroll
-    for (int j = 0; j < kJ; ++j)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const uint32_t id = 4 * (tid + kConsumerThreads * j) + c;
-        if (key[4 * j + c] == kmax && (int)id < V) best = min(best, id);
-      }
+    for (int e = 4 * kJ - 1; e >= 0; --e)
+      if (e < n_valid && key[e] == kmax) best = (uint32_t)(E * tid + e);
     best = __reduce_min_sync(0xFFFFFFFFu, best);
-    if (lane == 0) s.wred[sbuf][warp] = best;
+    if (lane == 0) s.wred[0][warp] = best;
     consumer_sync();
     if (tid == 0) {
       uint32_t b = 0xFFFFFFFFu;
 #pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) b = min(b, s.wred[sbuf][w]);
+      for (int w = 0; w < kConsumerWarps; ++w) b = min(b, s.wred[0][w]);
       out->ids[0] = (int)b;
       out->W[0] = 1u;
       out->S = 1ull;
       out->n = 1;
     }
-  } else {
+    MCD_TOPK_STAMP(5)
+    return;
+  }
+  // ---- the k-th largest key -----------------------------------------------------------------
+  const float vmin = key_f32(kmin), vmax = key_f32(kmax);
+  const float range = __fsub_rn(vmax, vmin);
+  const float scale = __fdiv_rn((float)kBins, range);
+  const bool binned = isfinite(vmin) && isfinite(vmax) && range > 0.f && isfinite(range) && isfinite(scale);
+  auto bin_of = [&](uint32_t kk) {
+    return min(kBins - 1, __float2int_rz(__fmul_rn(__fsub_rn(key_f32(kk), vmin), scale)));
+  };
+  uint32_t Tk = 0;
+  bool found = false;
+  if (binned) {                                                     // block-uniform
 #pragma unroll
-    for (int o = 16; o; o >>= 1) wsum += __shfl_xor_sync(0xFFFFFFFFu, wsum, o);
-    if (lane == 0) s.wsum[warp] = wsum;
+    for (int e = 0; e < 4 * kJ; ++e)
+      if (e < n_valid) atomicAdd(&s.hist[bin_of(key[e])], 1u);
     consumer_sync();
-    if (tid == 0) {
-      unsigned long long S = 0;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) S += s.wsum[w];
-      out->S = S;
-      out->n = k;
+    // lane L holds bins 8L .. 8L + 7; S(b) = #keys in bins >= b; B = the largest b with S(b) >= k
+    uint32_t c8[8];
+    {
+      const uint4 h0 = reinterpret_cast<const uint4*>(s.hist)[2 * lane];
+      const uint4 h1 = reinterpret_cast<const uint4*>(s.hist)[2 * lane + 1];
+      c8[0] = h0.x; c8[1] = h0.y; c8[2] = h0.z; c8[3] = h0.w;
+      c8[4] = h1.x; c8[5] = h1.y; c8[6] = h1.z; c8[7] = h1.w;
     }
+    uint32_t local = 0;
+#pragma unroll
+    for (int b = 0; b < 8; ++b) local += c8[b];
+    uint32_t suf = local;                                // keys in the bins of lanes >= L
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t t = __shfl_down_sync(0xFFFFFFFFu, suf, o);
+      if (lane + o < 32) suf += t;
+    }
+    uint32_t run = suf - local, b_cnt = 0, b_above = 0;
+    int b_sel = -1;
+#pragma unroll
+    for (int b = 7; b >= 0; --b) {
+      if (b_sel < 0 && run + c8[b] >= (uint32_t)k) {
+        b_sel = 8 * lane + b;
+        b_cnt = c8[b];
+        b_above = run;
+      }
+      run += c8[b];
+    }
+    const unsigned has = __ballot_sync(0xFFFFFFFFu, b_sel >= 0);   // a prefix of the lanes
+    const int src = 31 - __clz(has);
+    const int B = __shfl_sync(0xFFFFFFFFu, b_sel, src);
+    const uint32_t cntB = __shfl_sync(0xFFFFFFFFu, b_cnt, src);
+    const uint32_t aboveB = __shfl_sync(0xFFFFFFFFu, b_above, src);
+    if (cntB <= 32u) {                                               // block-uniform
+#pragma unroll
+      for (int e = 0; e < 4 * kJ; ++e)
+        if (e < n_valid && bin_of(key[e]) == B) s.cand[atomicAdd(&s.ncand, 1u)] = key[e];
+      consumer_sync();
+      // the (k - aboveB)-th largest of the bin's keys: gt(i) < need <= ge(i)
+      const uint32_t need = (uint32_t)k - aboveB;
+      const uint32_t kc = lane < (int)cntB ? s.cand[lane] : 0u;
+      uint32_t gt = 0, ge = 0;
+      for (int j = 0; j < (int)cntB; ++j) {
+        const uint32_t kj = __shfl_sync(0xFFFFFFFFu, kc, j);
+        gt += kj > kc ? 1u : 0u;
+        ge += kj >= kc ? 1u : 0u;
+      }
+      const unsigned hit = __ballot_sync(0xFFFFFFFFu, lane < (int)cntB && gt < need && need <= ge);
+      Tk = __shfl_sync(0xFFFFFFFFu, kc, __ffs(hit) - 1);
+      found = true;
+    }
+  }
+  MCD_TOPK_STAMP(2)
+  if (!found) {
+    // Counting search.  Invariant: #(key >= lo) >= k > #(key >= hi).  Each step counts 7
+    // thresholds splitting [lo, hi) into eighths (one barrier); it stops early when a
+    // threshold has exactly k keys at or above it, else when hi = lo + 1.
+    uint32_t lo = kmin;
+    unsigned long long hi = (unsigned long long)kmax + 1ull;
+    int buf = 0;
+    while (hi - lo > 1ull) {
+      const unsigned long long span = hi - lo;
+      uint32_t cnt[7];
+#pragma unroll
+      for (int i = 0; i < 7; ++i) {
+        const uint32_t t = lo + (uint32_t)((span * (unsigned long long)(i + 1)) >> 3);
+        uint32_t c = 0;
+#pragma unroll
+        for (int e = 0; e < 4 * kJ; ++e) c += (e < n_valid && key[e] >= t) ? 1u : 0u;
+        cnt[i] = __reduce_add_sync(0xFFFFFFFFu, c);
+      }
+      if (lane < 7) {
+        uint32_t mine = cnt[0];
+#pragma unroll
+        for (int i = 1; i < 7; ++i) mine = lane == i ? cnt[i] : mine;
+        s.part[buf][warp][lane] = mine;
+      }
+      consumer_sync();
+      uint32_t tot = 0;
+      if (lane < 7)
+#pragma unroll
+        for (int w = 0; w < kConsumerWarps; ++w) tot += s.part[buf][w][lane];
+      const uint32_t my_t = lo + (uint32_t)((span * (unsigned long long)(lane + 1)) >> 3);
+      const unsigned ge = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot >= (uint32_t)k);
+      const unsigned eq = __ballot_sync(0xFFFFFFFFu, lane < 7 && tot == (uint32_t)k);
+      buf ^= 1;
+      if (eq) {
+        lo = __shfl_sync(0xFFFFFFFFu, my_t, __ffs(eq) - 1);
+        break;
+      }
+      // thresholds increase with the lane, counts decrease: ge is a prefix of lanes 0..6
+      const int nge = __popc(ge);
+      const uint32_t new_lo = __shfl_sync(0xFFFFFFFFu, my_t, max(nge - 1, 0));
+      const uint32_t new_hi = __shfl_sync(0xFFFFFFFFu, my_t, min(nge, 6));
+      if (nge > 0) lo = new_lo;
+      if (nge < 7) hi = new_hi;
+    }
+    Tk = lo;
+  }
+  MCD_TOPK_STAMP(3)
+  // ---- id-ordered compaction with weights: one scan of (keys > Tk) | (keys == Tk) << 16 ------
+  uint32_t c_gt = 0, c_eq = 0;
+#pragma unroll
+  for (int e = 0; e < 4 * kJ; ++e) {
+    if (e < n_valid) {
+      c_gt += key[e] > Tk ? 1u : 0u;
+      c_eq += key[e] == Tk ? 1u : 0u;
+    }
+  }
+  uint32_t tot;
+  const uint32_t pre = block_exscan(c_gt | (c_eq << 16), s, 0, &tot);
+  const uint32_t krem = (uint32_t)k - (tot & 0xFFFFu);      // threshold keys to keep (>= 1)
+  uint32_t tie = pre >> 16;
+  uint32_t pos = (pre & 0xFFFFu) + min(tie, krem);
+  const float Td = T;
+  const float zmax = __fdiv_rn(key_f32(kmax), Td);
+  unsigned long long wsum = 0;
+#pragma unroll
+  for (int e = 0; e < 4 * kJ; ++e) {
+    if (e < n_valid) {
+      const uint32_t kv = key[e];
+      const bool eq = kv == Tk;
+      const bool inc = kv > Tk || (eq && tie < krem);
+      tie += eq ? 1u : 0u;
+      if (inc) {
+        const float z = __fdiv_rn(key_f32(kv), Td);
+        const uint32_t w = weight24(exp32_cw(__fsub_rn(z, zmax)));
+        out->ids[pos] = E * tid + e;
+        out->W[pos] = w;
+        wsum += w;
+        ++pos;
+      }
+    }
+  }
+  MCD_TOPK_STAMP(4)
+#pragma unroll
+  for (int o = 16; o; o >>= 1) wsum += __shfl_xor_sync(0xFFFFFFFFu, wsum, o);
+  if (lane == 0) s.wsum[warp] = wsum;
+  consumer_sync();
+  if (tid == 0) {
+    unsigned long long S = 0;
+#pragma unroll
+    for (int w = 0; w < kConsumerWarps; ++w) S += s.wsum[w];
+    out->S = S;
+    out->n = k;
   }
   MCD_TOPK_STAMP(5)
 #undef MCD_TOPK_STAMP

@@ -88,10 +88,12 @@ def big():
 # ---------------------------------------------------------------- sampler ----------
 @pytest.mark.parametrize("V,k,T,ties", [(2048, 50, 0.9, 0.0), (2048, 50, 0.9, 0.6), (64, 8, 1.0, 0.5),
                                         (64, 64, 1.0, 0.3), (2048, 128, 0.7, 0.2), (3072, 1, 1.3, 0.9),
-                                        (2048, 50, 0.05, 0.0)])
+                                        (2048, 50, 0.05, 0.0), (2000, 50, 0.9, 0.1), (4096, 100, 0.9, 0.2)])
 def test_topk_softmax_matches_oracle(V, k, T, ties):
     """Top-k ids, integer weights and their sums are bit-exact (both sides compute the same
-    fp32 exp32 and the same integer arithmetic)."""
+    fp32 exp32 and the same integer arithmetic).  Besides random rows: all-equal, signed
+    zeros, an outlier that crowds the threshold into one histogram bin, a cluster of nearly
+    equal values around the threshold and (T >= 0.7) a value range that overflows fp32."""
     cfg = TINY.replace(vocab=V, top_k=k, temperature=T)
     dec = mcd.Decoder(cfg)                     # sampler entry points need no weights
     rng = np.random.default_rng(V + k)
@@ -99,6 +101,11 @@ def test_topk_softmax_matches_oracle(V, k, T, ties):
     logits = random_logits(rng, rows, V, scale=0.7, tie_frac=ties)
     logits[0] = 0.0                            # all equal: lowest ids win
     logits[1, ::2] = -0.0                      # signed zeros tie
+    logits[2, 3] = 1000.0                      # outlier: coarse histogram bins
+    n_cl = min(V // 4, 300)                    # nearly equal values around the threshold
+    logits[4, :n_cl] = (np.float32(2.0) + np.arange(n_cl, dtype=np.float32) * np.float32(2.0 ** -20))
+    if T >= 0.7:
+        logits[3, 5], logits[3, 9] = 2e38, -2e38   # max - min overflows fp32
     ids = torch.zeros((rows, k), dtype=torch.int32, device=DEV)
     w = torch.zeros((rows, k), dtype=torch.int32, device=DEV)
     sums = torch.zeros(rows, dtype=torch.int64, device=DEV)
