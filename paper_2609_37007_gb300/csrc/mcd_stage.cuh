@@ -119,11 +119,12 @@ struct UnitRange {
 };
 __device__ __forceinline__ UnitRange unit_range(int si, int L, int n, int cta, int rot, int n_cta) {
   if (stage_kind(si, L) == MAT_HEAD || stage_kind(si, L) == MAT_WD) {
-    return UnitRange{(int)(((long long)cta * n) / n_cta), (int)(((long long)(cta + 1) * n) / n_cta), 1};
+    // (cta + 1) * n < 2^32 for every supported shape: 32-bit division
+    const unsigned un = (unsigned)n, uc = (unsigned)n_cta;
+    return UnitRange{(int)(((unsigned)cta * un) / uc), (int)(((unsigned)(cta + 1) * un) / uc), 1};
   }
-  int f = (cta - rot) % n_cta;
-  if (f < 0) f += n_cta;
-  return UnitRange{f, n, n_cta};
+  const int f = cta - rot;                // 0 <= cta, rot < n_cta
+  return UnitRange{f < 0 ? f + n_cta : f, n, n_cta};
 }
 
 // ------------------------------------------------------------------------------------
@@ -309,7 +310,8 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
         if (((8 * w) & (ncp - 1)) == own) s += c.sm.part[w * kMaxCols + tid];  // fixed order
       c.sm.inv_rms[tid] = rsqrtf(s / (float)Kdim + c.p.eps);
     }
-    consumer_sync();
+    // no barrier: inv_rms is read only by epilogues, which follow the chunk barrier of the
+    // stage, and part / inv_rms are rewritten only after the stage's closing barrier
   }
 }
 
@@ -320,17 +322,22 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
 struct WarpRole {
   int Gn, ntpw, lg_ntpw, Gk, kts, mi, gn, kg;
 };
+// (Mu, Ku, NT and the derived counts are powers of two: shifts instead of divisions.)
+__device__ __forceinline__ int ilog2(int v) { return 31 - __clz(v); }
 __device__ __forceinline__ WarpRole warp_role(const MatGeom& g, int NT, int warp, bool split_n) {
   WarpRole w;
-  w.Gn = split_n ? min(NT, kConsumerWarps / g.Mu) : 1;
-  w.ntpw = NT / w.Gn;
-  w.lg_ntpw = w.ntpw == 1 ? 0 : w.ntpw == 2 ? 1 : 2;
-  w.Gk = kConsumerWarps / (g.Mu * w.Gn);
-  w.kts = g.Ku / w.Gk;
-  w.mi = warp % g.Mu;
-  const int rest = warp / g.Mu;
-  w.gn = rest % w.Gn;
-  w.kg = rest / w.Gn;
+  const int lmu = ilog2(g.Mu), lnt = ilog2(NT);
+  const int lgn = split_n ? min(lnt, 3 - lmu) : 0;        // kConsumerWarps = 8
+  w.Gn = 1 << lgn;
+  w.lg_ntpw = lnt - lgn;
+  w.ntpw = 1 << w.lg_ntpw;
+  const int lgk = 3 - lmu - lgn;
+  w.Gk = 1 << lgk;
+  w.kts = g.Ku >> lgk;
+  w.mi = warp & (g.Mu - 1);
+  const int rest = warp >> lmu;
+  w.gn = rest & (w.Gn - 1);
+  w.kg = rest >> lgn;
   return w;
 }
 
@@ -446,8 +453,9 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
   const int NT = WIDE ? n_tiles(ncols) : 1;
   const bool hilo = WIDE ? hilo_operand(ncols) : true;
   const WarpRole role = warp_role(g, NT, threadIdx.x >> 5, WIDE && WT != MCD_WEIGHT_F32);
-  const int per_unit = kConsumerWarps * role.ntpw * 512;                            // bytes of partials
-  const int cap = max(1, min(kChunk, kRedBytes / per_unit));
+  // partials: kConsumerWarps * ntpw * 512 bytes per unit, kRedBytes in all
+  static_assert(kRedBytes == kConsumerWarps * 512 * 4, "chunk capacity below assumes 4 single-n-tile units");
+  const int cap = max(1, min(kChunk, 4 >> role.lg_ntpw));
   const int lgm = g.Mu == 1 ? 0 : g.Mu == 2 ? 1 : g.Mu == 4 ? 2 : 3;
   const int lgn = col_log2(ncols);
   const int lg_unit = lgm + (pairs_rows ? 3 : 4) + lgn;       // outputs per unit (log2)
@@ -487,7 +495,9 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
     first_chunk = false;
     if (u0 < ur.end) consumer_sync();
   }
-  c.rot = (c.rot + n_units) % p.n_cta;
+  int rot = c.rot + n_units;
+  while (rot >= p.n_cta) rot -= p.n_cta;
+  c.rot = rot;
 }
 
 // Read-only vector (weights) into shared memory; no barrier (a later barrier orders it).
