@@ -500,6 +500,7 @@ __device__ void run_call(Cons& c, int call) {
   for (int l = 0; l < L; ++l) {
     // ---- S1: RMSNorm -> QKV  (q, k, v = W (x . g) / rms) -------------------------------
     g2s_vec(sm.vec, p.attn_norm + (size_t)l * H, H);      // independent of the wait below
+    const StagePlan sp_qkv = plan_stage<WT, WIDE>(c, 4 * l + 0, p.g[MAT_QKV].n_units, n_rows, no_key);
     if (l == 0) {
       // layer-0 rows straight from their sources (cond / c0 vector / embedding rows); CTA 0
       // also seeds the residual stream x
@@ -519,7 +520,7 @@ __device__ void run_call(Cons& c, int call) {
     }
     {
       const MatGeom& g = p.g[MAT_QKV];
-      run_stage<WT, WIDE>(c, call, 4 * l + 0, g.n_units, H, n_rows, no_key, no_prep,
+      run_stage<WT, WIDE>(c, call, sp_qkv, H, no_key, no_prep,
                     [&](int u, int mi, int rr, int n, float v, float) {
                       const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
                       p.qkv[(size_t)n * p.qkv_dim + row] = v * sm.inv_rms[n] * wscale<WT>(p.s_qkv, (size_t)l * p.qkv_dim + row);
@@ -534,6 +535,9 @@ __device__ void run_call(Cons& c, int call) {
     // units compute that attention themselves.  Several streams: first one task per
     // (stream, query head) spread over the CTAs writes the outputs to global memory, then
     // Wo reads them.
+    auto wo_key = [&](int u) { return u / p.g[MAT_WO].n_mb; };
+    const StagePlan sp_wo = plan_stage<WT, WIDE>(c, 4 * l + 1, p.g[MAT_WO].n_units, n_rows, wo_key);
+    if (!WIDE && threadIdx.x == 0) sm.flags[3] = -1;     // ordered by the wait's barrier
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
     if (WIDE) {
       if (p.draft_mode == MCD_DRAFT_TREE && ci->st[0].pos0 > 0) {
@@ -561,7 +565,7 @@ __device__ void run_call(Cons& c, int call) {
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
       run_stage<WT, WIDE>(
-          c, call, 4 * l + 1, g.n_units, D, n_rows, [&](int u) { return u / g.n_mb; },
+          c, call, sp_wo, D, wo_key,
           [&](int u, int, int) {
             const int h = u / g.n_mb;
             if (sm.flags[3] != h) {
@@ -579,10 +583,8 @@ __device__ void run_call(Cons& c, int call) {
     } else {
       const MatGeom& g = p.g[MAT_WO];
       const int group = p.NH / p.NKV;
-      if (threadIdx.x == 0) sm.flags[3] = -1;
-      consumer_sync();
       run_stage<WT, WIDE>(
-          c, call, 4 * l + 1, g.n_units, D, n_rows, [&](int u) { return u / g.n_mb; },
+          c, call, sp_wo, D, wo_key,
           [&](int u, int cnt, int step) {
             const int h = u / g.n_mb;
             bool writer = false;      // the CTA holding m-block 0 of a group's first head writes K / V
@@ -606,13 +608,14 @@ __device__ void run_call(Cons& c, int call) {
 
     // ---- S3: RMSNorm -> gate/up -> SwiGLU --------------------------------------------------
     g2s_vec(sm.vec, p.ffn_norm + (size_t)l * H, H);
+    const StagePlan sp_gu = plan_stage<WT, WIDE>(c, 4 * l + 2, p.g[MAT_GU].n_units, n_rows, no_key, true);
     if (!cons_wait(c, ctr + ctr_stage(l, 1), N)) return;
     prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
     {
       const MatGeom& g = p.g[MAT_GU];
       // tile rows 0..7 are gate rows j0..j0+7, rows 8..15 the matching up rows
       run_stage<WT, WIDE>(
-          c, call, 4 * l + 2, g.n_units, H, n_rows, no_key, no_prep,
+          c, call, sp_gu, H, no_key, no_prep,
           [&](int u, int mi, int rr, int n, float gate, float up) {
             const float s = sm.inv_rms[n];
             const int t16 = ((u % g.n_mb) * g.Mu + mi) * 16 + rr;      // tiled row of the gate
@@ -620,21 +623,21 @@ __device__ void run_call(Cons& c, int call) {
             const float ut = up * s * wscale<WT>(p.s_gu, (size_t)l * 2 * F + t16 + 8);
             const int j = ((u % g.n_mb) * g.Mu + mi) * 8 + rr;
             p.mbuf[(size_t)n * F + j] = gt / (1.0f + __expf(-gt)) * ut;
-          },
-          true);
+          });
       if (c.abort_) return;
     }
     cons_signal(c, ctr + ctr_stage(l, 2), call, 10 + 4 * (4 * l + 2));
 
     // ---- S4: down + residual (k-chunks of F) ---------------------------------------------
+    auto wd_key = [&](int u) { return u / p.g[MAT_WD].n_mb; };
+    const StagePlan sp_wd = plan_stage<WT, WIDE>(c, 4 * l + 3, p.g[MAT_WD].n_units, n_rows, wd_key);
+    if (threadIdx.x == 0) sm.flags[3] = -1;     // ordered by the wait's barrier
     if (!cons_wait(c, ctr + ctr_stage(l, 2), N)) return;
     {
       const MatGeom& g = p.g[MAT_WD];
       const int Kc = g.Ku * 16;
-      if (threadIdx.x == 0) sm.flags[3] = -1;
-      consumer_sync();
       run_stage<WT, WIDE>(
-          c, call, 4 * l + 3, g.n_units, Kc, n_rows, [&](int u) { return u / g.n_mb; },
+          c, call, sp_wd, Kc, wd_key,
           [&](int u, int, int) {
             const int kc = u / g.n_mb;
             if (sm.flags[3] != kc) {
@@ -660,6 +663,7 @@ __device__ void run_call(Cons& c, int call) {
   // chunk in `vec`, which is free once the operand is built).  The call streams the union
   // of the heads its streams need.
   g2s_vec(sm.vec, p.final_norm, H);
+  const StagePlan sp_head = plan_stage<WT, WIDE>(c, 4 * L, ci->n_heads * p.g[MAT_HEAD].n_units, n_rows, no_key);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
   prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
   {
@@ -667,7 +671,7 @@ __device__ void run_call(Cons& c, int call) {
     float* bias_s = sm.vec;   // [kChunk][16 rows][kMaxCols columns]
     int chunk_u0 = 0;
     run_stage<WT, WIDE>(
-        c, call, 4 * L, ci->n_heads * g.n_units, H, n_rows, no_key,
+        c, call, sp_head, H, no_key,
         [&](int u0, int cnt, int step) {
           chunk_u0 = u0;
           for (int o = threadIdx.x; o < cnt * 16 * kMaxCols; o += kConsumerThreads) {

@@ -308,7 +308,7 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
 #pragma unroll
       for (int w = 0; w < kConsumerWarps; ++w)
         if (((8 * w) & (ncp - 1)) == own) s += c.sm.part[w * kMaxCols + tid];  // fixed order
-      c.sm.inv_rms[tid] = rsqrtf(s / (float)Kdim + c.p.eps);
+      c.sm.inv_rms[tid] = rsqrtf(__fmul_rn(s, __frcp_rn((float)Kdim)) + c.p.eps);
     }
     // no barrier: inv_rms is read only by epilogues, which follow the chunk barrier of the
     // stage, and part / inv_rms are rewritten only after the stage's closing barrier
@@ -322,7 +322,8 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
 struct WarpRole {
   int Gn, ntpw, lg_ntpw, Gk, kts, mi, gn, kg;
 };
-// (Mu, Ku, NT and the derived counts are powers of two: shifts instead of divisions.)
+// (Mu, NT and the warp-group counts are powers of two and Gk divides Ku: shifts instead of
+// divisions.)
 __device__ __forceinline__ int ilog2(int v) { return 31 - __clz(v); }
 __device__ __forceinline__ WarpRole warp_role(const MatGeom& g, int NT, int warp, bool split_n) {
   WarpRole w;
@@ -436,34 +437,70 @@ __device__ __forceinline__ float red_sum(const Cons& c, const MatGeom& g, const 
   return v;
 }
 
-// Run every unit of stage si assigned to this CTA.  Units are taken in chunks of up to
-// kChunk consecutive units that share one operand (opkey(u): the k-chunk / head whose B
-// operand they multiply; prep(u0, cnt, step) builds it for the chunk), as many as the
-// reduction buffer holds.  Each chunk: wait for its units' weights, multiply them all, one
-// barrier, then one epilogue pass epi(u, mi, rr, n, v, v8) over the live outputs (columns
-// n < ncols; v8 = row rr + 8 for gate/up pairs).
-template <int WT, bool WIDE, class Key, class Prep, class Epi>
-__device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, int ncols, Key opkey,
-                                          Prep prep, Epi epi, bool pairs_rows = false) {
+// A stage's schedule for this CTA: its units, the warp roles and chunking, and the size of
+// the first chunk.  It depends only on the call's shape, so a stage plans before it waits
+// for its inputs and the integer work overlaps the grid barrier.
+struct StagePlan {
+  UnitRange ur;
+  WarpRole role;
+  int si, n_units, ncols, NT, cap, lg_unit, lgn, cnt0;
+  bool hilo, pairs;
+};
+template <int WT, bool WIDE, class Key>
+__device__ __forceinline__ StagePlan plan_stage(const Cons& c, int si, int n_units, int ncols, Key opkey,
+                                                bool pairs_rows = false) {
   const FrameParams& p = c.p;
+  const MatGeom& g = p.g[stage_kind(si, p.L)];
+  StagePlan sp;
+  sp.si = si;
+  sp.n_units = n_units;
+  sp.ncols = ncols;
+  sp.pairs = pairs_rows;
+  sp.ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
+  sp.NT = WIDE ? n_tiles(ncols) : 1;
+  sp.hilo = WIDE ? hilo_operand(ncols) : true;
+  sp.role = warp_role(g, sp.NT, threadIdx.x >> 5, WIDE && WT != MCD_WEIGHT_F32);
+  // partials: kConsumerWarps * ntpw * 512 bytes per unit, kRedBytes in all
+  static_assert(kRedBytes == kConsumerWarps * 512 * 4, "chunk capacity below assumes 4 single-n-tile units");
+  sp.cap = max(1, min(kChunk, 4 >> sp.role.lg_ntpw));
+  sp.lgn = col_log2(ncols);
+  sp.lg_unit = ilog2(g.Mu) + (pairs_rows ? 3 : 4) + sp.lgn;     // outputs per unit (log2)
+  sp.cnt0 = 0;
+  const int u0 = sp.ur.first;
+  if (u0 < sp.ur.end) {
+    const int key = opkey(u0);
+    int cnt = 1;
+    while (cnt < sp.cap && u0 + cnt * sp.ur.step < sp.ur.end && opkey(u0 + cnt * sp.ur.step) == key) ++cnt;
+    sp.cnt0 = cnt;
+  }
+  return sp;
+}
+
+// Run every unit of the planned stage.  Units are taken in chunks of up to kChunk
+// consecutive units that share one operand (opkey(u): the k-chunk / head whose B operand
+// they multiply; prep(u0, cnt, step) builds it for the chunk), as many as the reduction
+// buffer holds.  Each chunk: wait for its units' weights, multiply them all, one barrier,
+// then one epilogue pass epi(u, mi, rr, n, v, v8) over the live outputs (columns n < ncols;
+// v8 = row rr + 8 for gate/up pairs).
+template <int WT, bool WIDE, class Key, class Prep, class Epi>
+__device__ __forceinline__ void run_stage(Cons& c, int call, const StagePlan& sp, int Kdim, Key opkey, Prep prep,
+                                          Epi epi) {
+  const FrameParams& p = c.p;
+  const int si = sp.si;
   const MatGeom& g = p.g[stage_kind(si, p.L)];
   const int lane = threadIdx.x & 31;
   timeline(c, call, 8 + 4 * si);
-  const UnitRange ur = unit_range(si, p.L, n_units, blockIdx.x, c.rot, p.n_cta);
-  const int NT = WIDE ? n_tiles(ncols) : 1;
-  const bool hilo = WIDE ? hilo_operand(ncols) : true;
-  const WarpRole role = warp_role(g, NT, threadIdx.x >> 5, WIDE && WT != MCD_WEIGHT_F32);
-  // partials: kConsumerWarps * ntpw * 512 bytes per unit, kRedBytes in all
-  static_assert(kRedBytes == kConsumerWarps * 512 * 4, "chunk capacity below assumes 4 single-n-tile units");
-  const int cap = max(1, min(kChunk, 4 >> role.lg_ntpw));
-  const int lgm = g.Mu == 1 ? 0 : g.Mu == 2 ? 1 : g.Mu == 4 ? 2 : 3;
-  const int lgn = col_log2(ncols);
-  const int lg_unit = lgm + (pairs_rows ? 3 : 4) + lgn;       // outputs per unit (log2)
+  const UnitRange& ur = sp.ur;
+  const int lgn = sp.lgn, lg_unit = sp.lg_unit, ncols = sp.ncols;
+  const bool pairs_rows = sp.pairs;
   bool first_chunk = true;
   for (int u0 = ur.first; u0 < ur.end;) {
-    const int key = opkey(u0);
-    int cnt = 1;
-    while (cnt < cap && u0 + cnt * ur.step < ur.end && opkey(u0 + cnt * ur.step) == key) ++cnt;
+    int cnt = sp.cnt0;
+    if (!first_chunk) {
+      const int key = opkey(u0);
+      cnt = 1;
+      while (cnt < sp.cap && u0 + cnt * ur.step < ur.end && opkey(u0 + cnt * ur.step) == key) ++cnt;
+    }
     prep(u0, cnt, ur.step);
 #pragma unroll 1
     for (int r = 0; r < cnt; ++r) {
@@ -471,7 +508,7 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
       if (!wait_mbar(&c.sm.full[slot], ((c.seq + r) / kNumSlots) & 1u, p.err, p.wait_ns, nullptr))
         c.sm.flags[1] = 1;
       if (first_chunk && r == 0) timeline(c, call, 9 + 4 * si);
-      unit_mma<WT, WIDE>(c, g, role, NT, hilo, c.sm.ring + (size_t)slot * kSlotBytes, Kdim, 0, r);
+      unit_mma<WT, WIDE>(c, g, sp.role, sp.NT, sp.hilo, c.sm.ring + (size_t)slot * kSlotBytes, Kdim, 0, r);
       __syncwarp();
       if (lane == 0) mbar_arrive(&c.sm.empty[slot]);
     }
@@ -486,8 +523,8 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
       const int row = q >> lgn, n = q & ((1 << lgn) - 1);
       if (n < ncols) {
         const int mi = row >> (pairs_rows ? 3 : 4), rr = row & (pairs_rows ? 7 : 15);
-        const float v = red_sum(c, g, role, r, mi, rr, n);
-        const float v8 = pairs_rows ? red_sum(c, g, role, r, mi, rr + 8, n) : 0.f;
+        const float v = red_sum(c, g, sp.role, r, mi, rr, n);
+        const float v8 = pairs_rows ? red_sum(c, g, sp.role, r, mi, rr + 8, n) : 0.f;
         epi(u0 + r * ur.step, mi, rr, n, v, v8);
       }
     }
@@ -495,9 +532,17 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units
     first_chunk = false;
     if (u0 < ur.end) consumer_sync();
   }
-  int rot = c.rot + n_units;
+  int rot = c.rot + sp.n_units;
   while (rot >= p.n_cta) rot -= p.n_cta;
   c.rot = rot;
+}
+
+// Plan and run in one step (stages whose plan cannot precede a wait).
+template <int WT, bool WIDE, class Key, class Prep, class Epi>
+__device__ __forceinline__ void run_stage(Cons& c, int call, int si, int n_units, int Kdim, int ncols, Key opkey,
+                                          Prep prep, Epi epi, bool pairs_rows = false) {
+  const StagePlan sp = plan_stage<WT, WIDE>(c, si, n_units, ncols, opkey, pairs_rows);
+  run_stage<WT, WIDE>(c, call, sp, Kdim, opkey, prep, epi);
 }
 
 // Read-only vector (weights) into shared memory; no barrier (a later barrier orders it).
