@@ -115,7 +115,7 @@ __device__ __forceinline__ uint32_t block_exscan(uint32_t v, TopkScratch& s, int
 //       set in id order (ties at the threshold keep the lowest ids) and gives every weight.
 // `greedy` replaces the distribution by the one-hot of the argmax (ties: lowest id).  `dbg`,
 // when not null, receives clock64() stamps at the phase boundaries (profiling only).
-static __device__ __forceinline__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
+static __device__ __noinline__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
                                   TopkScratch& s, TopkRec* out, long long* dbg = nullptr) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 #define MCD_TOPK_STAMP(i) \
