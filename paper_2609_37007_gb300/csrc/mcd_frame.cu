@@ -775,14 +775,32 @@ __device__ void run_call(Cons& c, int call) {
 
 // Copy distribution records into shared memory with independent word loads: the header,
 // ids[0..k) and W[0..k) of each (k = top_k; entries past a record's n are never read).
+// Threads t0 .. t0 + nt - 1 take part; each issues a batch of up to 8 loads before its
+// stores, so a copy costs about one memory round trip per batch.
 template <class Src>
-__device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src) {
+__device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src, int t0 = 0,
+                                              int nt = kConsumerThreads) {
   constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kWWord = offsetof(TopkRec, W) / 4;
-  const int words = kIdsWord + 2 * k;
-  for (int i = threadIdx.x; i < nrec * words; i += kConsumerThreads) {
-    const int r = i / words, w = i - r * words;
-    const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kWWord + (w - kIdsWord - k));
-    reinterpret_cast<int*>(dst + r)[off] = __ldcg(reinterpret_cast<const int*>(src(r)) + off);
+  constexpr int kB = 8;
+  const int words = kIdsWord + 2 * k, total = nrec * words, me = (int)threadIdx.x - t0;
+  if (me < 0 || me >= nt) return;
+  for (int b = 0; b < total; b += kB * nt) {
+    int v[kB];
+    int* d[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      const int i = b + me + u * nt;
+      d[u] = nullptr;
+      if (i < total) {
+        const int r = i / words, w = i - r * words;
+        const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kWWord + (w - kIdsWord - k));
+        v[u] = __ldcg(reinterpret_cast<const int*>(src(r)) + off);
+        d[u] = reinterpret_cast<int*>(dst + r) + off;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kB; ++u)
+      if (d[u]) *d[u] = v[u];
   }
 }
 
@@ -823,16 +841,10 @@ __device__ void accept_step(Cons& c, int call, int s) {
   // whose residual code ends the call, else the bonus code (same decisions as testing the
   // drafts one after another).
   __shared__ int s_ok[kMaxDraft + 1], s_alt[kMaxDraft + 1];
-  if (pre && (int)threadIdx.x >= idle0) {
-    constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kWWord = offsetof(TopkRec, W) / 4;
-    const int words = kIdsWord + 2 * p.top_k, nrec = n_rows * p.K;
-    for (int i = threadIdx.x - idle0; i < nrec * words; i += kConsumerThreads - idle0) {
-      const int r = i / words, w = i - r * words;
-      const int off = w < kIdsWord ? w : (w < kIdsWord + p.top_k ? w : kWWord + (w - kIdsWord - p.top_k));
-      const TopkRec* src = cur + (base + r / p.K) * (kMaxDraft + 1) + 1 + r % p.K;
-      reinterpret_cast<int*>(srec + n_pq + r)[off] = __ldcg(reinterpret_cast<const int*>(src) + off);
-    }
-  }
+  if (pre)
+    stage_records(srec + n_pq, n_rows * p.K, p.top_k,
+                  [&](int r) { return cur + (base + r / p.K) * (kMaxDraft + 1) + 1 + r % p.K; }, idle0,
+                  kConsumerThreads - idle0);
   if (warp <= n_d) {
     const int i = warp, pos = a + 1 + i;
     if (i < n_d) {

@@ -438,13 +438,27 @@ static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned
     id[e] = i < np ? p->ids[i] : -1;
     wq[e] = 0;
   }
-  for (int j = 0; j < nq; ++j) {       // q's entries broadcast to every lane
-    const int qid = q->ids[j];
-    const unsigned long long qw = q->W[j];
+  // W_q of each of the lane's ids: binary search of q's ids (records list ascending ids),
+  // the lane's searches interleaved
+  int lo[kDrawPerLane], hi[kDrawPerLane];
 #pragma unroll
-    for (int e = 0; e < kDrawPerLane; ++e)
-      if (id[e] == qid) wq[e] = qw;
+  for (int e = 0; e < kDrawPerLane; ++e) {
+    lo[e] = 0;
+    hi[e] = nq;                          // first index with ids >= id[e] lies in [lo, hi]
   }
+  for (int span = nq; span > 0; span >>= 1) {
+#pragma unroll
+    for (int e = 0; e < kDrawPerLane; ++e) {
+      if (lo[e] < hi[e]) {
+        const int mid = (lo[e] + hi[e]) >> 1;
+        if (q->ids[mid] < id[e]) lo[e] = mid + 1;
+        else hi[e] = mid;
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < kDrawPerLane; ++e)
+    if (id[e] >= 0 && lo[e] < nq && q->ids[lo[e]] == id[e]) wq[e] = q->W[lo[e]];
   unsigned long long R = 0;
 #pragma unroll
   for (int e = 0; e < kDrawPerLane; ++e) {
