@@ -12,7 +12,7 @@ CSRC = os.path.join(PKG, "csrc")
 ROOT = os.path.dirname(PKG)
 LIB = os.path.join(PKG, "libmcd.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu", "mcd_outer.cu", "mcd_batch.cu"]
+SOURCES = ["mcd_api.cu", "mcd_frame.cu", "mcd_static.cu", "mcd_outer.cu", "mcd_batch.cu", "mcd_tcgemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-cudart", "shared",
          "-I" + os.path.join(ROOT, "include")]
@@ -50,7 +50,7 @@ def _stale(out: str, deps) -> bool:
 def build(verbose: bool = False, force: bool = False, extra=()) -> str:
     os.makedirs(BUILD_DIR, exist_ok=True)
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
-    headers += [os.path.join(ROOT, "include", f) for f in ("mcd.h", "mcd_pipeline.h")]
+    headers += [os.path.join(ROOT, "include", f) for f in ("mcd.h", "mcd_pipeline.h", "mcd_tc.h")]
     objs, jobs = [], []
     for src in SOURCES:
         s = os.path.join(CSRC, src)

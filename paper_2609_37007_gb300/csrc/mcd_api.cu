@@ -647,6 +647,7 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
                 S(pre + "wd"), S(pre + "attn_norm"), S(pre + "ffn_norm"),
                 p.qk_norm ? S(pre + "q_norm") : nullptr, p.qk_norm ? S(pre + "k_norm") : nullptr};
     load_layer(p, c->stream, ls, l);
+    if (c->batch && batch_load_layer(c->batch, p, c->stream, ls, l) != MCD_OK) return cleanup(MCD_ERR_CUDA);
   }
   conv("final_norm", H, p.final_norm);
   for (int j = 1; j <= Kd; ++j) conv("offset." + std::to_string(j), H, p.offsets + (size_t)(j - 1) * H);

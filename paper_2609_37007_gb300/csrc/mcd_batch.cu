@@ -24,6 +24,7 @@
 #include "mcd_host.cuh"
 #include "mcd_internal.cuh"
 #include "mcd_sampler.cuh"
+#include "mcd_tcgemm.cuh"
 
 namespace mcd {
 
@@ -88,6 +89,18 @@ struct BatchBufs {
   uint16_t* act;          // [R][F] bf16 SwiGLU outputs
   float* logits;          // [R][kRecSlots][V]
   TopkRec* recs;          // [2][R][kRecSlots]
+  // tensor-core GEMM operands (SW128 tiles of Rtc rows, Rtc = R rounded up to 128)
+  int Rtc;
+  uint8_t* xn_hi;         // normalised rows, bf16 (and the low halves for the QKV product)
+  uint8_t* xn_lo;
+  uint8_t* att_t;         // attention outputs
+  uint8_t* act_t;         // SwiGLU outputs
+};
+
+// Weights of the tensor-core GEMMs: per layer the row-major matrices as SW128 tiles.
+struct TcWeights {
+  uint8_t* arena = nullptr;
+  size_t qkv = 0, g = 0, u = 0, o = 0, d = 0, layer = 0;     // offsets within a layer, layer stride
 };
 
 // ------------------------------------------------------------------------------------
@@ -475,6 +488,101 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
   }
 }
 
+// ---- tensor-core GEMM path (tcgen05, mcd_tcgemm.cuh) ---------------------------------------
+// With all of qkv_dim, F and H multiples of 128 the QKV, Wo, gate/up and down products run on
+// the tcgen05 GEMM; their operand rows are written as SW128 tiles first (normalised rows, the
+// attention outputs) or directly by the producing epilogue (the SwiGLU outputs).
+
+// Normalised operand rows x * gain / rms(x) of the call's packed rows as SW128 tiles (hi; with
+// lo also the bf16 remainder), one 8-element chunk per thread.
+__global__ void __launch_bounds__(256) tc_norm_operand_kernel(const float* __restrict__ X, const float* __restrict__ gain,
+                                                              const float* __restrict__ ss, int H, float eps,
+                                                              const BatchInfo* info, int Rtc, uint8_t* hi, uint8_t* lo) {
+  const int M = info->M, cpr = H / 8;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * cpr; i += gridDim.x * blockDim.x) {
+    const int r = i / cpr, ch = i - r * cpr, k = ch * 8;
+    const float s = rsqrtf(ss[r] / (float)H + eps);
+    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k));
+    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k + 4));
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + k));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + k + 4));
+    const float v[8] = {x0.x * g0.x * s, x0.y * g0.y * s, x0.z * g0.z * s, x0.w * g0.w * s,
+                        x1.x * g1.x * s, x1.y * g1.y * s, x1.z * g1.z * s, x1.w * g1.w * s};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
+    }
+    const size_t off = tc::sw128_offset(Rtc, r, ch >> 3, ch & 7);
+    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+// bf16 rows [M][K] (the call's packed rows) -> SW128 tiles of Rtc rows.
+__global__ void __launch_bounds__(256) tc_rows_operand_kernel(const uint16_t* __restrict__ src, int K,
+                                                              const BatchInfo* info, int Rtc, uint8_t* dst) {
+  const int M = info->M, cpr = K / 8;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * cpr; i += gridDim.x * blockDim.x) {
+    const int r = i / cpr, ch = i - r * cpr;
+    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(Rtc, r, ch >> 3, ch & 7)) =
+        __ldcg(reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8));
+  }
+}
+
+// Row-major bf16 [rows][K] -> rows row0.. of an SW128-tiled matrix of R rows (weight load).
+__global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0,
+                                      uint8_t* __restrict__ dst) {
+  const long long total = (long long)rows * (K / 8);
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+    const int r = (int)(i / (K / 8)), ch = (int)(i % (K / 8));
+    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(R, row0 + r, ch >> 3, ch & 7)) =
+        *reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8);
+  }
+}
+
+constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
+constexpr int kTcBNGU = 64;       // gate/up (two accumulators)
+constexpr int kTcSplit = 4;       // k-splits of the residual products
+
+// q, k, v = W (x . g / rms) with the hi + lo operand.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
+                                                                  const BatchInfo* info) {
+  const int M = __ldg(&info->M);
+  tc::gemm_tile<kTcBN, false, true>(g, [&](int m, int n, float v, float) {
+    if (n < M) out[(size_t)n * ld + m] = v;
+  });
+}
+
+// gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
+// product (element (row n, feature m)).
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
+                                                                 const BatchInfo* info) {
+  const int M = __ldg(&info->M);
+  tc::gemm_tile<kTcBNGU, true, false>(g, [&](int m, int n, float gt, float up) {
+    if (n < M) {
+      const float v = gt / (1.0f + __expf(-gt)) * up;
+      *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
+          f32_to_bf16(v);
+    }
+  });
+}
+
+// Residual products (Wo, down), k split over gridDim.z: partial sums added into X.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* X, int ld,
+                                                                    const BatchInfo* info) {
+  const int M = __ldg(&info->M);
+  tc::gemm_tile<kTcBN, false, false>(g, [&](int m, int n, float v, float) {
+    if (n < M) atomicAdd(X + (size_t)n * ld + m, v);
+  });
+}
+
+bool tc_supported(const FrameParams& p) {
+  return p.wdtype == MCD_WEIGHT_BF16 && p.qkv_dim % 128 == 0 && p.F % 128 == 0 && p.H % 128 == 0 &&
+         (p.NH * p.D) % 64 == 0 && p.H % 64 == 0 && p.F % 64 == 0;
+}
+
 // Per-row sums of squares of the residual stream after a residual GEMM (one warp per row):
 // the next RMSNorm's 1/rms, applied while the next GEMM stages its operand.
 __global__ void __launch_bounds__(256) batch_rowss_kernel(const float* X, int H, float* ss, const BatchInfo* info) {
@@ -735,6 +843,8 @@ struct BatchState {
   BatchBufs b;
   BatchFrame host_frame;
   int max_streams = 0;
+  bool use_tc = false;        // QKV, Wo, gate/up and down on the tcgen05 GEMM
+  TcWeights tw;
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
   cudaStream_t cap = nullptr;
@@ -791,6 +901,24 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
   BATCH_ALLOC(b.act, sizeof(uint16_t) * R * p.F);
   BATCH_ALLOC(b.logits, sizeof(float) * R * kRecSlots * p.V);
   BATCH_ALLOC(b.recs, sizeof(TopkRec) * 2 * R * kRecSlots);
+  bs->use_tc = tc_supported(p);
+  if (bs->use_tc) {
+    const int Rtc = (R + 127) / 128 * 128;
+    b.Rtc = Rtc;
+    BATCH_ALLOC(b.xn_hi, (size_t)Rtc * p.H * 2);
+    BATCH_ALLOC(b.xn_lo, (size_t)Rtc * p.H * 2);
+    BATCH_ALLOC(b.att_t, (size_t)Rtc * p.NH * p.D * 2);
+    BATCH_ALLOC(b.act_t, (size_t)Rtc * p.F * 2);
+    TcWeights& tw = bs->tw;
+    const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
+    tw.qkv = 0;
+    tw.g = tw.qkv + (size_t)p.qkv_dim * H * 2;
+    tw.u = tw.g + F * H * 2;
+    tw.o = tw.u + F * H * 2;
+    tw.d = tw.o + H * qd * 2;
+    tw.layer = tw.d + H * F * 2;
+    BATCH_ALLOC(tw.arena, tw.layer * p.L);
+  }
 #undef BATCH_ALLOC
   if (cudaMemset(b.info, 0, sizeof(BatchInfo)) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamCreateWithFlags(&bs->cap, cudaStreamNonBlocking) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -799,8 +927,35 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
   for (void* fn : gemms)
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmemHilo) != cudaSuccess)
       return fail(MCD_ERR_CUDA);
+  if (bs->use_tc &&
+      (cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                            tc::Layout<kTcBN, false, true>::kSmemBytes) != cudaSuccess ||
+       cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                            tc::Layout<kTcBNGU, true, false>::kSmemBytes) != cudaSuccess ||
+       cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                            tc::Layout<kTcBN, false, false>::kSmemBytes) != cudaSuccess))
+    return fail(MCD_ERR_CUDA);
   *out = bs;
   return MCD_OK;
+}
+
+// The tcgen05 GEMMs' copies of layer l's matrices (row-major bf16 sources, device).
+mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t st, const LayerSrc& src, int l) {
+  if (!bs || !bs->use_tc) return MCD_OK;
+  const TcWeights& tw = bs->tw;
+  uint8_t* base = tw.arena + (size_t)l * tw.layer;
+  const int H = p.H, F = p.F, qd = p.NH * p.D, kd = p.NKV * p.D;
+  auto tile = [&](const uint8_t* s, int rows, int K, int R, int row0, size_t off) {
+    tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(s), rows, K, R, row0, base + off);
+  };
+  tile(src.wq, qd, H, p.qkv_dim, 0, tw.qkv);
+  tile(src.wk, kd, H, p.qkv_dim, qd, tw.qkv);
+  tile(src.wv, kd, H, p.qkv_dim, qd + kd, tw.qkv);
+  tile(src.wg, F, H, F, 0, tw.g);
+  tile(src.wu, F, H, F, 0, tw.u);
+  tile(src.wo, H, qd, H, 0, tw.o);
+  tile(src.wd, H, F, H, 0, tw.d);
+  return cudaGetLastError() == cudaSuccess ? MCD_OK : MCD_ERR_CUDA;
 }
 
 static GemmArgs gemm_args(const FrameParams& p, const BatchBufs& b) {
@@ -831,7 +986,44 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
   for (int call = 0; call < p.P; ++call) {
     batch_pack_kernel<<<1, 256, 0, s>>>(p, b);
     batch_embed_kernel<<<R, 256, 0, s>>>(p, b);
-    for (int l = 0; l < L; ++l) {
+    for (int l = 0; l < L && bs->use_tc; ++l) {
+      const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.layer;
+      const int Rtc = b.Rtc, qd = p.NH * p.D;
+      const dim3 tblk(tc::kThreads);
+      // RMSNorm -> QKV (hi + lo operand)
+      tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm + (size_t)l * H, b.ss + (size_t)(2 * l) * R, H, p.eps,
+                                                b.info, Rtc, b.xn_hi, b.xn_lo);
+      {
+        const tc::GemmArgs g{wl + bs->tw.qkv, nullptr, b.xn_hi, b.xn_lo, p.qkv_dim, Rtc, H, &b.info->M, p.err, p.wait_ns};
+        tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
+            g, b.qkv, p.qkv_dim, b.info);
+      }
+      batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);
+      // Wo + residual
+      tc_rows_operand_kernel<<<256, blk, 0, s>>>(b.att, qd, b.info, Rtc, b.att_t);
+      {
+        const tc::GemmArgs g{wl + bs->tw.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
+        tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+            g, b.X, H, b.info);
+      }
+      batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 1) * R, b.info);
+      // RMSNorm -> gate/up -> SwiGLU (into the down product's operand)
+      tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.ffn_norm + (size_t)l * H, b.ss + (size_t)(2 * l + 1) * R, H,
+                                                p.eps, b.info, Rtc, b.xn_hi, nullptr);
+      {
+        const tc::GemmArgs g{wl + bs->tw.g, wl + bs->tw.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
+        tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
+            g, b.act_t, Rtc, b.info);
+      }
+      // down + residual
+      {
+        const tc::GemmArgs g{wl + bs->tw.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
+        tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+            g, b.X, H, b.info);
+      }
+      batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 2) * R, b.info);
+    }
+    for (int l = 0; l < L && !bs->use_tc; ++l) {
       {   // RMSNorm -> QKV
         GemmArgs a = gemm_args(p, b);
         a.W = p.w_qkv + (size_t)l * p.g[MAT_QKV].stride;

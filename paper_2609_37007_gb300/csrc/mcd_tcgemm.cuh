@@ -1,0 +1,245 @@
+// Tensor-core GEMM on the 5th-generation tensor cores (tcgen05, TMEM accumulators) for the
+// products of the batched path that are real GEMMs: D[m][n] = sum_k A[m][k] B[n][k] with A
+// the weights (bf16, M x K) and B the packed activation rows (bf16, N x K), fp32 accumulation.
+//
+// Operands live in HBM in the "SW128 tile" layout: for every 64-wide k-slice kt, rows in
+// groups of 8 form 1024-byte atoms, row r of an atom is 128 bytes (64 bf16) and its 16-byte
+// chunk c sits at chunk position c ^ (r % 8).  A tile of TR rows (TR % 8 == 0) of one k-slice
+// is then TR * 128 contiguous bytes that one cp.async.bulk copies into shared memory, where it
+// is exactly the canonical K-major layout with 128-byte swizzle that tcgen05.mma reads
+// (8-row groups 1024 bytes apart).  No tensor map is needed.
+//
+// One CTA computes a 128 x BN tile of D (UMMA M = 128, N = BN, K = 16 per instruction): a
+// producer thread streams the k-slices of A and B through a 4-stage ring (mbarrier
+// complete_tx), one thread issues the MMAs and returns each stage with tcgen05.commit, and
+// after the last commit the four warps read the accumulator back from TMEM (warp w owns
+// lanes 32w..32w+31 = rows m of the tile) and hand every value to the epilogue functor.
+// Every wait is bounded (p.wait_ns); on a timeout the CTA records MCD_ERR_TIMEOUT, lets the
+// copies and MMAs it started finish, frees its TMEM and returns.
+#pragma once
+#include "mcd_internal.cuh"
+
+namespace mcd {
+namespace tc {
+
+constexpr int kBM = 128;         // rows of A per tile (UMMA M)
+constexpr int kBK = 64;          // k per stage: one 128-byte swizzled row
+constexpr int kStages = 4;
+constexpr int kThreads = 128;
+
+// Byte offset of (row, 16-byte chunk c) of k-slice kt in the SW128 tile layout of a matrix
+// with R rows.
+__host__ __device__ __forceinline__ size_t sw128_offset(int R, int row, int kt, int c) {
+  return (size_t)kt * R * 128 + (size_t)(row >> 3) * 1024 + (size_t)(row & 7) * 128 + (size_t)((c ^ (row & 7)) << 4);
+}
+
+// kDualA: a second A matrix (same shape) multiplies the same B into a second accumulator
+// (gate and up projections side by side); kDualB: a second B operand (the low bf16 half of
+// a hi + lo split) accumulates into the same accumulator.
+template <int BN, bool kDualA = false, bool kDualB = false>
+struct Layout {
+  static_assert(BN % 16 == 0 && BN >= 32 && BN <= 256 && (BN & (BN - 1)) == 0, "UMMA N / TMEM columns");
+  static constexpr int kABytes = kBM * 128;
+  static constexpr int kBBytes = BN * 128;
+  static constexpr int kStageBytes = (kDualA ? 2 : 1) * kABytes + (kDualB ? 2 : 1) * kBBytes;
+  static constexpr int kTmemCols = (kDualA ? 2 : 1) * BN;
+  static constexpr int kBarOff = kStages * kStageBytes;                 // full[s], empty[s], accum
+  static constexpr int kTmemSlotOff = kBarOff + (2 * kStages + 1) * 8;
+  static constexpr int kFlagOff = kTmemSlotOff + 4;
+  static constexpr int kSmemBytes = kFlagOff + 4 + 1024;               // + alignment slack
+  static_assert(kSmemBytes <= 227 * 1024, "tensor-core GEMM stages exceed shared memory");
+  static_assert(kTmemCols <= 512, "TMEM columns");
+};
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t smem_addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr >> 4) & 0x3FFFu);            // start address
+  d |= (uint64_t)1u << 16;                                 // leading byte offset (unused here)
+  d |= (uint64_t)(1024u >> 4) << 32;                       // stride byte offset
+  d |= (uint64_t)1u << 46;                                 // descriptor version
+  d |= (uint64_t)2u << 61;                                 // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of kind::f16: bf16 A and B (K-major), fp32 D, M = 128, N = BN.
+template <int BN>
+__host__ __device__ constexpr uint32_t idesc_bf16() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, bool accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"((uint32_t)accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+
+// 32 lanes x 16 consecutive fp32 columns of TMEM (lane = this thread's lane of the warp's
+// quarter) into v[0..15].
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// Bounded wait on an mbarrier phase; false (and the error recorded) on a timeout.
+__device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, int* err, unsigned long long wait_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer() - t0 > wait_ns) {
+      atomicCAS(err, 0, (int)MCD_ERR_TIMEOUT);
+      return false;
+    }
+  }
+  return true;
+}
+
+struct GemmArgs {
+  const uint8_t* a;      // A in SW128 tiles, M rows
+  const uint8_t* a2;     // kDualA: the second A (same layout)
+  const uint8_t* b;      // B in SW128 tiles, N rows
+  const uint8_t* b2;     // kDualB: the second B (same layout)
+  int M, N, K;           // M % 128 == 0, N % BN == 0, K % 64 == 0
+  const int* n_active;   // optional (device): columns n >= *n_active are not computed
+  int* err;
+  unsigned long long wait_ns;
+};
+
+// The GEMM body for the tile of rows m0 = blockIdx.y * 128 of A and n0 = blockIdx.x * BN of B
+// over the k-slices of split blockIdx.z of gridDim.z (the CTAs that share an A tile are
+// adjacent in launch order, so the weights stream from HBM about once while the activation
+// tiles stay in L2); epi(m, n, v, v2) for every m and n of the tile (each thread: one m, BN
+// values of n in order; v2 = the second accumulator with kDualA, else 0).  A tile whose
+// first column is at or past *n_active returns at once.
+template <int BN, bool kDualA, bool kDualB, class Epi>
+__device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
+  using L = Layout<BN, kDualA, kDualB>;
+  extern __shared__ uint8_t tc_smem_raw[];
+  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  if (g.n_active && n0 >= __ldg(g.n_active)) return;          // uniform over the CTA
+  const int nk_all = g.K / kBK, per = (nk_all + gridDim.z - 1) / gridDim.z;
+  const int kt0 = blockIdx.z * per, kt1 = min(nk_all, kt0 + per), nk = kt1 - kt0;
+  if (nk <= 0) return;
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
+  uint64_t* empty = full + kStages;
+  uint64_t* accum = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kTmemSlotOff);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kFlagOff);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"((uint32_t)L::kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // producer: k-slice kt of the A tile(s) (rows m0..) and the B tile(s) (rows n0..)
+    const uint64_t pol_a = policy_evict_first(), pol_b = policy_evict_last();
+    int issued = 0;
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % kStages, kt = kt0 + i;
+      if (i >= kStages && !tc_wait(&empty[s], ((i / kStages) - 1) & 1, g.err, g.wait_ns)) {
+        *abort_flag = 1;
+        break;
+      }
+      if (*abort_flag) break;
+      uint8_t* st = smem + s * L::kStageBytes;
+      const size_t ao = (size_t)kt * g.M * 128 + (size_t)m0 * 128, bo = (size_t)kt * g.N * 128 + (size_t)n0 * 128;
+      mbar_arrive_expect_tx(&full[s], L::kStageBytes);
+      bulk_g2s(st, g.a + ao, L::kABytes, &full[s], pol_a);
+      if (kDualA) bulk_g2s(st + L::kABytes, g.a2 + ao, L::kABytes, &full[s], pol_a);
+      uint8_t* sb = st + (kDualA ? 2 : 1) * L::kABytes;
+      bulk_g2s(sb, g.b + bo, L::kBBytes, &full[s], pol_b);
+      if (kDualB) bulk_g2s(sb + L::kBBytes, g.b2 + bo, L::kBBytes, &full[s], pol_b);
+      ++issued;
+    }
+    // every issued copy lands before the CTA may exit
+    for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i)
+      tc_wait(&full[i % kStages], (i / kStages) & 1, g.err, g.wait_ns);
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer
+    constexpr uint32_t idesc = idesc_bf16<BN>();
+    for (int i = 0; i < nk; ++i) {
+      const int s = i % kStages;
+      if (!tc_wait(&full[s], (i / kStages) & 1, g.err, g.wait_ns)) {
+        *abort_flag = 1;
+        break;
+      }
+      if (*abort_flag) break;
+      tc_fence_after();
+      const uint32_t sa = smem_u32(smem + s * L::kStageBytes);
+      const uint32_t sb = sa + (kDualA ? 2 : 1) * L::kABytes;
+#pragma unroll
+      for (int j = 0; j < kBK / 16; ++j) {
+        const bool acc = (i | j) != 0;
+        umma_bf16(tmem, sw128_desc(sa + 32 * j), sw128_desc(sb + 32 * j), idesc, acc);
+        if (kDualB) umma_bf16(tmem, sw128_desc(sa + 32 * j), sw128_desc(sb + L::kBBytes + 32 * j), idesc, true);
+        if (kDualA)
+          umma_bf16(tmem + BN, sw128_desc(sa + L::kABytes + 32 * j), sw128_desc(sb + 32 * j), idesc, acc);
+      }
+      umma_commit(&empty[s]);         // the stage is free once these MMAs have read it
+    }
+    umma_commit(accum);               // every MMA issued so far has completed
+  }
+  // epilogue: all four warps, after the accumulator is complete
+  const bool ok = tc_wait(accum, 0, g.err, g.wait_ns) && !*abort_flag;
+  __syncwarp();                       // the .sync.aligned TMEM loads need whole warps
+  tc_fence_after();
+  if (ok) {
+    const int m = m0 + warp * 32 + lane;
+    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 16) {
+      float v[16], v2[16];
+      tmem_ld16(lane_base + (uint32_t)c0, v);
+      if (kDualA) tmem_ld16(lane_base + (uint32_t)(BN + c0), v2);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) epi(m, n0 + c0 + j, v[j], kDualA ? v2[j] : 0.f);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)L::kTmemCols)
+                 : "memory");
+}
+
+}  // namespace tc
+}  // namespace mcd

@@ -116,6 +116,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_outer_set_trace": (I32, [P, P, I32]),
         "mcd_outer_sync": (I32, [P]),
         "mcd_outer_step_weight_bytes": (I64, [P]),
+        "mcd_tc_gemm": (I32, [I32, I32, I32, I32, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -263,6 +264,13 @@ def mcd_num_ctas(ctx) -> int:
 
 def mcd_destroy(ctx):
     load_library().mcd_destroy(ctx)
+
+
+def mcd_tc_gemm(M: int, N: int, K: int, bn: int, A, B, Y, stream=None):
+    """Y[n][m] = sum_k A[m][k] B[n][k] on the tensor cores (tcgen05): A bf16 [M, K], B bf16
+    [N, K], Y fp32 [N, M], all device tensors (synchronises the stream)."""
+    _check("mcd_tc_gemm", load_library().mcd_tc_gemm(M, N, K, bn, _ptr(A), _ptr(B), _ptr(Y),
+                                                     ctypes.c_void_p(stream.cuda_stream if stream is not None else None)))
 
 
 def mcd_status_str(status: int) -> str:
