@@ -95,6 +95,7 @@ struct BatchBufs {
   uint8_t* xn_lo;
   uint8_t* att_t;         // attention outputs
   uint8_t* act_t;         // SwiGLU outputs
+  float* part;            // [kTcSplit][Rtc][H] k-split partial sums of the residual products
 };
 
 // Weights of the tensor-core GEMMs: per layer the row-major matrices as SW128 tiles.
@@ -490,8 +491,10 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
 
 // ---- tensor-core GEMM path (tcgen05, mcd_tcgemm.cuh) ---------------------------------------
 // With all of qkv_dim, F and H multiples of 128 the QKV, Wo, gate/up and down products run on
-// the tcgen05 GEMM; their operand rows are written as SW128 tiles first (normalised rows, the
-// attention outputs) or directly by the producing epilogue (the SwiGLU outputs).
+// the tcgen05 GEMM.  Their operand rows are written as SW128 tiles by the kernel that produces
+// them: the normalised rows by the pass that also folds the k-split partial sums of the
+// previous residual product into the residual stream, the attention outputs by the attention
+// kernel, the SwiGLU outputs by the gate/up epilogue.
 
 // Normalised operand rows x * gain / rms(x) of the call's packed rows as SW128 tiles (hi; with
 // lo also the bf16 remainder), one 8-element chunk per thread.
@@ -520,17 +523,6 @@ __global__ void __launch_bounds__(256) tc_norm_operand_kernel(const float* __res
   }
 }
 
-// bf16 rows [M][K] (the call's packed rows) -> SW128 tiles of Rtc rows.
-__global__ void __launch_bounds__(256) tc_rows_operand_kernel(const uint16_t* __restrict__ src, int K,
-                                                              const BatchInfo* info, int Rtc, uint8_t* dst) {
-  const int M = info->M, cpr = K / 8;
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * cpr; i += gridDim.x * blockDim.x) {
-    const int r = i / cpr, ch = i - r * cpr;
-    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(Rtc, r, ch >> 3, ch & 7)) =
-        __ldcg(reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8));
-  }
-}
-
 // Row-major bf16 [rows][K] -> rows row0.. of an SW128-tiled matrix of R rows (weight load).
 __global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0,
                                       uint8_t* __restrict__ dst) {
@@ -543,7 +535,7 @@ __global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows
 }
 
 constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
-constexpr int kTcBNGU = 64;       // gate/up (two accumulators)
+constexpr int kTcBNGU = 128;      // gate/up (two accumulators)
 constexpr int kTcSplit = 4;       // k-splits of the residual products
 
 // q, k, v = W (x . g / rms) with the hi + lo operand.
@@ -569,13 +561,74 @@ __global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmAr
   });
 }
 
-// Residual products (Wo, down), k split over gridDim.z: partial sums added into X.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* X, int ld,
+// Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
+// part[z][n][m] (plain stores); tc_resid_norm_kernel adds them into the residual stream.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
                                                                     const BatchInfo* info) {
   const int M = __ldg(&info->M);
+  float* pz = part + (size_t)blockIdx.z * Rtc * ld;
   tc::gemm_tile<kTcBN, false, false>(g, [&](int m, int n, float v, float) {
-    if (n < M) atomicAdd(X + (size_t)n * ld + m, v);
+    if (n < M) pz[(size_t)n * ld + m] = v;
   });
+}
+
+// Per packed row (one CTA, thread t owns elements 8t..8t+7): X += the nz partial sums, the
+// row's sum of squares (the next RMSNorm), and with a gain the next product's normalised
+// operand (hi; with lo also the remainder) as SW128 tiles.
+__global__ void __launch_bounds__(128) tc_resid_norm_kernel(float* X, const float* __restrict__ part, int nz, int Rtc,
+                                                            int H, const BatchInfo* info, float* ss_out,
+                                                            const float* __restrict__ gain, float eps, uint8_t* hi,
+                                                            uint8_t* lo) {
+  const int r = blockIdx.x;
+  if (r >= info->M) return;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const bool live = t < H / 8;
+  __shared__ float red[4];
+  float x[8];
+  float ss = 0.f;
+  if (live) {
+    float4* xr = reinterpret_cast<float4*>(X + (size_t)r * H + 8 * t);
+    float4 a = xr[0], b = xr[1];
+    for (int z = 0; z < nz; ++z) {
+      const float4* pr = reinterpret_cast<const float4*>(part + ((size_t)z * Rtc + r) * H + 8 * t);
+      const float4 u = __ldcg(pr), w = __ldcg(pr + 1);
+      a.x += u.x; a.y += u.y; a.z += u.z; a.w += u.w;
+      b.x += w.x; b.y += w.y; b.z += w.z; b.w += w.w;
+    }
+    xr[0] = a;
+    xr[1] = b;
+    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss += x[i] * x[i];
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  const float tot = red[0] + red[1] + red[2] + red[3];
+  if (t == 0) ss_out[r] = tot;
+  if (gain && live) {
+    const float s = rsqrtf(tot / (float)H + eps);
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t + 4));
+    const float v[8] = {x[0] * g0.x * s, x[1] * g0.y * s, x[2] * g0.z * s, x[3] * g0.w * s,
+                        x[4] * g1.x * s, x[5] * g1.y * s, x[6] * g1.z * s, x[7] * g1.w * s};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
+    }
+    const size_t off = tc::sw128_offset(Rtc, r, t >> 3, t & 7);
+    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+// Non-empty k-splits of a residual product over K (gemm_tile's split of the k-slices).
+static int tc_splits(int K) {
+  const int nk = K / tc::kBK, per = (nk + kTcSplit - 1) / kTcSplit;
+  return (nk + per - 1) / per;
 }
 
 bool tc_supported(const FrameParams& p) {
@@ -703,7 +756,12 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
     const int qi = t / D, d = t - qi * D, n = qi / group, h = g * group + qi % group;
     float acc = 0.f;
     for (int j = 0; j <= pos0 + n; ++j) acc += sc[qi][j] * vs[j][d];
-    b.att[(size_t)(base + n) * p.NH * D + h * D + d] = f32_to_bf16(acc);
+    const int f = h * D + d;
+    if (b.att_t)        // the Wo product's operand, SW128 tiles (tensor-core path)
+      *reinterpret_cast<uint16_t*>(b.att_t + tc::sw128_offset(b.Rtc, base + n, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
+          f32_to_bf16(acc);
+    else
+      b.att[(size_t)(base + n) * p.NH * D + f] = f32_to_bf16(acc);
   }
 }
 
@@ -909,6 +967,7 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
     BATCH_ALLOC(b.xn_lo, (size_t)Rtc * p.H * 2);
     BATCH_ALLOC(b.att_t, (size_t)Rtc * p.NH * p.D * 2);
     BATCH_ALLOC(b.act_t, (size_t)Rtc * p.F * 2);
+    BATCH_ALLOC(b.part, (size_t)kTcSplit * Rtc * p.H * 4);
     TcWeights& tw = bs->tw;
     const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
     tw.qkv = 0;
@@ -990,38 +1049,39 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.layer;
       const int Rtc = b.Rtc, qd = p.NH * p.D;
       const dim3 tblk(tc::kThreads);
-      // RMSNorm -> QKV (hi + lo operand)
-      tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm + (size_t)l * H, b.ss + (size_t)(2 * l) * R, H, p.eps,
-                                                b.info, Rtc, b.xn_hi, b.xn_lo);
+      // RMSNorm -> QKV (hi + lo operand; after layer 0 written by the previous layer's last
+      // residual pass)
+      if (l == 0)
+        tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm, b.ss, H, p.eps, b.info, Rtc, b.xn_hi, b.xn_lo);
       {
         const tc::GemmArgs g{wl + bs->tw.qkv, nullptr, b.xn_hi, b.xn_lo, p.qkv_dim, Rtc, H, &b.info->M, p.err, p.wait_ns};
         tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
             g, b.qkv, p.qkv_dim, b.info);
       }
-      batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);
-      // Wo + residual
-      tc_rows_operand_kernel<<<256, blk, 0, s>>>(b.att, qd, b.info, Rtc, b.att_t);
+      batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);      // -> att_t
+      // Wo (k-split partials) -> residual, ss, the gate/up operand
       {
         const tc::GemmArgs g{wl + bs->tw.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
         tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.X, H, b.info);
+            g, b.part, H, Rtc, b.info);
       }
-      batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 1) * R, b.info);
-      // RMSNorm -> gate/up -> SwiGLU (into the down product's operand)
-      tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.ffn_norm + (size_t)l * H, b.ss + (size_t)(2 * l + 1) * R, H,
-                                                p.eps, b.info, Rtc, b.xn_hi, nullptr);
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, b.info, b.ss + (size_t)(2 * l + 1) * R,
+                                             p.ffn_norm + (size_t)l * H, p.eps, b.xn_hi, nullptr);
+      // gate/up -> SwiGLU (into the down product's operand)
       {
         const tc::GemmArgs g{wl + bs->tw.g, wl + bs->tw.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
         tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
             g, b.act_t, Rtc, b.info);
       }
-      // down + residual
+      // down (k-split partials) -> residual, ss, the next layer's QKV operand
       {
         const tc::GemmArgs g{wl + bs->tw.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
         tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.X, H, b.info);
+            g, b.part, H, Rtc, b.info);
       }
-      batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 2) * R, b.info);
+      const bool last = l + 1 == L;
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(p.F), Rtc, H, b.info, b.ss + (size_t)(2 * l + 2) * R,
+                                             last ? nullptr : p.attn_norm + (size_t)(l + 1) * H, p.eps, b.xn_hi, b.xn_lo);
     }
     for (int l = 0; l < L && !bs->use_tc; ++l) {
       {   // RMSNorm -> QKV
