@@ -660,6 +660,8 @@ mcd_status mcd_load_weights(mcd_ctx* c, int32_t n, const char* const* names, con
     rh.src_cols = (int)H;
     tile(rh, p.g[MAT_HEAD], c->w_arena + c->off_head + (size_t)(P - 1) * p.g[MAT_HEAD].stride,
          q8 ? const_cast<float*>(p.s_head) + (size_t)(P - 1) * p.V : nullptr);
+    if (c->batch && batch_load_head(c->batch, p, c->stream, S("head." + std::to_string(P)), P) != MCD_OK)
+      return cleanup(MCD_ERR_CUDA);
   }
   for (int P = 1; P <= p.P && p.K > 0; ++P) {
     const int warps = p.K * p.V;

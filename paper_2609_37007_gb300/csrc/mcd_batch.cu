@@ -96,12 +96,16 @@ struct BatchBufs {
   uint8_t* att_t;         // attention outputs
   uint8_t* act_t;         // SwiGLU outputs
   float* part;            // [kTcSplit][Rtc][H] k-split partial sums of the residual products
+  int Qcap;               // LM-head operand rows: every (row, j) pair, groups padded per head
+  uint8_t* hq_hi;         // LM-head operand (normalised rows of the pairs, grouped by head)
+  uint8_t* hq_lo;
 };
 
 // Weights of the tensor-core GEMMs: per layer the row-major matrices as SW128 tiles.
 struct TcWeights {
   uint8_t* arena = nullptr;
   size_t qkv = 0, g = 0, u = 0, o = 0, d = 0, layer = 0;     // offsets within a layer, layer stride
+  uint8_t* heads = nullptr;                                   // [n_pos][V x H] SW128 tiles
 };
 
 // ------------------------------------------------------------------------------------
@@ -631,6 +635,85 @@ static int tc_splits(int K) {
   return (nk + per - 1) / per;
 }
 
+// LM heads.  The (row, j) pairs of the call are grouped by head (head_list); group P starts at
+// operand row qoff(P) = the sum of the earlier groups rounded up to the tile width, so every
+// tile of the product belongs to one head.
+__device__ __forceinline__ int tc_head_qoff(const BatchInfo* info, int P) {
+  int o = 0;
+  for (int i = 1; i < P; ++i) o += (info->head_rows[i] + kTcBN - 1) / kTcBN * kTcBN;
+  return o;
+}
+
+// The pairs' normalised rows (final RMSNorm, hi + lo) as SW128 tiles of Qcap rows.
+__global__ void __launch_bounds__(256) tc_heads_operand_kernel(const float* __restrict__ X, const float* __restrict__ gain,
+                                                               const float* __restrict__ ss, int H, float eps,
+                                                               const BatchInfo* info, const int* __restrict__ head_list,
+                                                               int n_pos, int Qcap, uint8_t* hi, uint8_t* lo) {
+  __shared__ int s_off[16], s_rows[16], s_q[16];
+  if (threadIdx.x < 16) {
+    const int P = threadIdx.x;
+    s_off[P] = info->head_off[P];
+    s_rows[P] = P >= 1 && P <= n_pos ? info->head_rows[P] : 0;
+    s_q[P] = P >= 1 && P <= n_pos ? tc_head_qoff(info, P) : 0;
+  }
+  __syncthreads();
+  const int T = info->n_pairs, cpr = H / 8;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T * cpr; i += gridDim.x * blockDim.x) {
+    const int gi = i / cpr, ch = i - gi * cpr, k = ch * 8;
+    int P = 1;
+    while (P < n_pos && !(gi >= s_off[P] && gi < s_off[P] + s_rows[P])) ++P;
+    const int q = s_q[P] + (gi - s_off[P]);
+    const int r = head_list[gi] >> 3;
+    const float s = rsqrtf(ss[r] / (float)H + eps);
+    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k));
+    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k + 4));
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + k));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + k + 4));
+    const float v[8] = {x0.x * g0.x * s, x0.y * g0.y * s, x0.z * g0.z * s, x0.w * g0.w * s,
+                        x1.x * g1.x * s, x1.y * g1.y * s, x1.z * g1.z * s, x1.w * g1.w * s};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      h[t] = pack_bf16x2(v[2 * t], v[2 * t + 1]);
+      l[t] = pack_bf16x2(v[2 * t] - bf16_lo_f32(h[t]), v[2 * t + 1] - bf16_hi_f32(h[t]));
+    }
+    const size_t off = tc::sw128_offset(Qcap, q, ch >> 3, ch & 7);
+    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+// Logits of every pair: tile (blockIdx.x) of head P's group times head P's weights, plus the
+// draft-offset bias for j >= 1.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_heads_kernel(const tc::GemmArgs g, const uint8_t* w_heads,
+                                                                    size_t head_bytes, float* logits,
+                                                                    const float* head_bias, const BatchInfo* info,
+                                                                    const int* head_list, int n_pos, int K, int V) {
+  const int q0 = blockIdx.x * kTcBN;
+  int P = 0, qoff = 0;
+  for (int i = 1, o = 0; i <= n_pos; ++i) {
+    const int span = (info->head_rows[i] + kTcBN - 1) / kTcBN * kTcBN;
+    if (q0 >= o && q0 < o + span) {
+      P = i;
+      qoff = o;
+    }
+    o += span;
+  }
+  if (P == 0) return;                                   // past the last group (uniform per CTA)
+  const int rows = info->head_rows[P], off = info->head_off[P];
+  tc::GemmArgs ga = g;
+  ga.a = w_heads + (size_t)(P - 1) * head_bytes;
+  ga.n_active = nullptr;
+  tc::gemm_tile<kTcBN, false, true>(ga, [&](int m, int n, float v, float) {
+    const int i = n - qoff;
+    if (i < rows) {
+      const int e = head_list[off + i], r = e >> 3, j = e & 7;
+      const float bias = j >= 1 ? __ldg(head_bias + ((size_t)(P - 1) * K + (j - 1)) * V + m) : 0.f;
+      logits[((size_t)r * kRecSlots + j) * V + m] = v + bias;
+    }
+  });
+}
+
 bool tc_supported(const FrameParams& p) {
   return p.wdtype == MCD_WEIGHT_BF16 && p.qkv_dim % 128 == 0 && p.F % 128 == 0 && p.H % 128 == 0 &&
          (p.NH * p.D) % 64 == 0 && p.H % 64 == 0 && p.F % 64 == 0;
@@ -968,6 +1051,12 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
     BATCH_ALLOC(b.att_t, (size_t)Rtc * p.NH * p.D * 2);
     BATCH_ALLOC(b.act_t, (size_t)Rtc * p.F * 2);
     BATCH_ALLOC(b.part, (size_t)kTcSplit * Rtc * p.H * 4);
+    if (p.V % tc::kBM == 0) {
+      b.Qcap = (R * kRecSlots + p.P * (kTcBN - 1) + kTcBN - 1) / kTcBN * kTcBN;
+      BATCH_ALLOC(b.hq_hi, (size_t)b.Qcap * p.H * 2);
+      BATCH_ALLOC(b.hq_lo, (size_t)b.Qcap * p.H * 2);
+      BATCH_ALLOC(bs->tw.heads, (size_t)p.P * p.V * p.H * 2);
+    }
     TcWeights& tw = bs->tw;
     const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
     tw.qkv = 0;
@@ -992,7 +1081,9 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
        cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                             tc::Layout<kTcBNGU, true, false>::kSmemBytes) != cudaSuccess ||
        cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            tc::Layout<kTcBN, false, false>::kSmemBytes) != cudaSuccess))
+                            tc::Layout<kTcBN, false, false>::kSmemBytes) != cudaSuccess ||
+       cudaFuncSetAttribute(tc_heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                            tc::Layout<kTcBN, false, true>::kSmemBytes) != cudaSuccess))
     return fail(MCD_ERR_CUDA);
   *out = bs;
   return MCD_OK;
@@ -1014,6 +1105,14 @@ mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t s
   tile(src.wu, F, H, F, 0, tw.u);
   tile(src.wo, H, qd, H, 0, tw.o);
   tile(src.wd, H, F, H, 0, tw.d);
+  return cudaGetLastError() == cudaSuccess ? MCD_OK : MCD_ERR_CUDA;
+}
+
+// The tcgen05 GEMM's copy of LM head P (row-major bf16 [V][H] source, device).
+mcd_status batch_load_head(BatchState* bs, const FrameParams& p, cudaStream_t st, const uint8_t* src, int P) {
+  if (!bs || !bs->tw.heads) return MCD_OK;
+  tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(src), p.V, p.H, p.V, 0,
+                                             bs->tw.heads + (size_t)(P - 1) * p.V * p.H * 2);
   return cudaGetLastError() == cudaSuccess ? MCD_OK : MCD_ERR_CUDA;
 }
 
@@ -1135,7 +1234,14 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
         batch_rowss_kernel<<<R / 8, blk, 0, s>>>(b.X, H, b.ss + (size_t)(2 * l + 2) * R, b.info);
       }
     }
-    {   // final RMSNorm -> LM heads, one grid slice per head
+    if (bs->tw.heads) {   // final RMSNorm -> LM heads on the tensor cores, tiles grouped by head
+      tc_heads_operand_kernel<<<512, blk, 0, s>>>(b.X, p.final_norm, b.ss + (size_t)(2 * L) * R, H, p.eps, b.info,
+                                                 b.head_list, p.P, b.Qcap, b.hq_hi, b.hq_lo);
+      const tc::GemmArgs g{nullptr, nullptr, b.hq_hi, b.hq_lo, p.V, b.Qcap, H, nullptr, p.err, p.wait_ns};
+      tc_heads_kernel<<<dim3(b.Qcap / kTcBN, p.V / tc::kBM, 1), dim3(tc::kThreads),
+                        tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(g, bs->tw.heads, (size_t)p.V * H * 2, b.logits,
+                                                                        p.head_bias, b.info, b.head_list, p.P, p.K, p.V);
+    } else {   // final RMSNorm -> LM heads, one grid slice per head
       GemmArgs a = gemm_args(p, b);
       a.W = p.w_head;
       a.g = p.g[MAT_HEAD];

@@ -65,6 +65,7 @@ int batch_rows(const FrameParams& p, int max_streams);
 mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out);
 // The batched path's copies of layer l's weights for its tensor-core GEMMs (no-op without).
 mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t st, const LayerSrc& src, int l);
+mcd_status batch_load_head(BatchState* bs, const FrameParams& p, cudaStream_t st, const uint8_t* src, int P);
 void batch_destroy(BatchState* bs);
 mcd_status batch_decode(BatchState* bs, const FrameParams& p, cudaStream_t stream, int n, const uint32_t* stream_ids,
                         const uint32_t* frame_ids, const float* cond, const int32_t* c0, const float* c0_emb,

@@ -305,10 +305,12 @@ TINY_BF16 = TINY.replace(weight_dtype=1)
 
 @pytest.mark.parametrize("cfg", [TINY_BF16.replace(max_streams=16), TINY_BF16.replace(max_streams=24, draft_len=3),
                                  TINY_BF16.replace(max_streams=40, draft_len=1),
-                                 TINY_BF16.replace(max_streams=12, draft_len=0, n_pos=6)])
+                                 TINY_BF16.replace(max_streams=12, draft_len=0, n_pos=6),
+                                 TINY_BF16.replace(max_streams=33, draft_len=3, vocab=256)])
 def test_gemm_path_trace_parity_tiny_bf16(cfg):
-    """More than 32 packed rows per call: the batched GEMM path (one graph launch per frame).
-    Every stream's calls match the oracle decoding that stream alone."""
+    """More than 32 packed rows per call: the batched GEMM path (one graph launch per frame;
+    tensor-core GEMMs for the backbone, and for the LM heads when the vocabulary is a
+    multiple of 128).  Every stream's calls match the oracle decoding that stream alone."""
     env = Env(cfg)
     for rep in range(2):
         n = cfg.max_streams - 3 * rep             # also fewer streams than the context allows
