@@ -747,26 +747,46 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
   const int nr = st->n_rows, pos0 = st->pos0;
   const int D = p.D, half = D >> 1, group = p.NH / p.NKV, nq = nr * group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  __shared__ float qs[kBatchQVec][132];        // nr x group query vectors
-  __shared__ float ks[kBatchKeys][132];
-  __shared__ float vs[kBatchKeys][128];
+  __shared__ __align__(16) float qs[kBatchQVec][132];        // nr x group query vectors
+  __shared__ __align__(16) float ks[kBatchKeys][132];
+  __shared__ __align__(16) float vs[kBatchKeys][128];
   __shared__ float sc[kBatchQVec][kBatchKeys];
   const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
   const int nk = pos0 + nr;
-  // loads: queries, new keys / values, cached keys / values
-  for (int i = tid; i < nq * D; i += blockDim.x) {
-    const int qi = i / D, d = i - qi * D, n = qi / group, h = g * group + qi % group;
-    qs[qi][d] = __ldcg(b.qkv + (size_t)(base + n) * p.qkv_dim + h * D + d);
-  }
-  for (int i = tid; i < nk * D; i += blockDim.x) {
-    const int j = i / D, d = i - j * D;
-    if (j < pos0) {
-      ks[j][d] = __ldcg(p.kcache + cache_off + (size_t)j * D + d);
-      vs[j][d] = __ldcg(p.vcache + cache_off + (size_t)j * D + d);
-    } else {
-      const size_t rb = (size_t)(base + j - pos0) * p.qkv_dim;
-      ks[j][d] = __ldcg(b.qkv + rb + p.NH * D + g * D + d);
-      vs[j][d] = __ldcg(b.qkv + rb + p.NH * D + p.NKV * D + g * D + d);
+  const int D4 = D >> 2;
+  // loads: queries, then keys and values (cached rows, then the new rows), as 16-byte chunks,
+  // a batch of up to 6 per thread in flight before the stores
+  {
+    const int n_q = nq * D4, n_kv = nk * D4, total = n_q + 2 * n_kv;
+    constexpr int kL = 6;
+    for (int b0 = 0; b0 < total; b0 += kL * 256) {
+      float4 v[kL];
+      float4* dst[kL];
+#pragma unroll
+      for (int u = 0; u < kL; ++u) {
+        const int i = b0 + tid + u * 256;
+        dst[u] = nullptr;
+        if (i < total) {
+          const float4* src;
+          if (i < n_q) {
+            const int qi = i / D4, d4 = i - qi * D4, n = qi / group, h = g * group + qi % group;
+            src = reinterpret_cast<const float4*>(b.qkv + (size_t)(base + n) * p.qkv_dim + h * D) + d4;
+            dst[u] = reinterpret_cast<float4*>(qs[qi]) + d4;
+          } else {
+            const int i2 = i - n_q, isv = i2 >= n_kv, i3 = isv ? i2 - n_kv : i2, j = i3 / D4, d4 = i3 - j * D4;
+            if (j < pos0)
+              src = reinterpret_cast<const float4*>((isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D) + d4;
+            else
+              src = reinterpret_cast<const float4*>(b.qkv + (size_t)(base + j - pos0) * p.qkv_dim + p.NH * D +
+                                                    (isv ? p.NKV * D : 0) + g * D) + d4;
+            dst[u] = reinterpret_cast<float4*>(isv ? vs[j] : ks[j]) + d4;
+          }
+          v[u] = __ldcg(src);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kL; ++u)
+        if (dst[u]) *dst[u] = v[u];
     }
   }
   __syncthreads();
@@ -813,14 +833,28 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
     }
   }
   __syncthreads();
-  // scores (one thread per (query, key)), softmax (one warp per query), P.V
+  // scores: four adjacent threads per (query, key), each over every fourth 16-byte chunk,
+  // summed by shuffles (every thread runs the same number of rounds); softmax (one warp per
+  // query); P.V
   const float scale = rsqrtf((float)D);
-  for (int t = tid; t < nq * nk; t += blockDim.x) {
-    const int qi = t / nk, j = t - qi * nk, n = qi / group;
+  const int n_dot = nq * nk;
+  for (int t0 = 0; t0 < 4 * n_dot; t0 += 256) {
+    const int t = t0 + tid, qd = t >> 2, part = t & 3;
+    const bool live = qd < n_dot;
+    const int qi = live ? qd / nk : 0, j = live ? qd - qi * nk : 0, n = qi / group;
+    const bool causal = live && j <= pos0 + n;
     float acc = 0.f;
-    if (j <= pos0 + n)
-      for (int d = 0; d < D; ++d) acc += qs[qi][d] * ks[j][d];
-    sc[qi][j] = j <= pos0 + n ? acc * scale : -INFINITY;
+    if (causal) {
+      const float4* q4 = reinterpret_cast<const float4*>(qs[qi]);
+      const float4* k4 = reinterpret_cast<const float4*>(ks[j]);
+      for (int d4 = part; d4 < D4; d4 += 4) {
+        const float4 a = q4[d4], k = k4[d4];
+        acc += a.x * k.x + a.y * k.y + a.z * k.z + a.w * k.w;
+      }
+    }
+    acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
+    acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 2);
+    if (live && part == 0) sc[qi][j] = causal ? acc * scale : -INFINITY;
   }
   __syncthreads();
   for (int qi = warp; qi < nq; qi += 8) {
@@ -835,16 +869,25 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
     if (lane < nk) sc[qi][lane] = e / l;
   }
   __syncthreads();
-  for (int t = tid; t < nq * D; t += blockDim.x) {
-    const int qi = t / D, d = t - qi * D, n = qi / group, h = g * group + qi % group;
-    float acc = 0.f;
-    for (int j = 0; j <= pos0 + n; ++j) acc += sc[qi][j] * vs[j][d];
-    const int f = h * D + d;
+  // one thread per (query, 4 dims)
+  for (int t = tid; t < nq * D4; t += blockDim.x) {
+    const int qi = t / D4, d4 = t - qi * D4, n = qi / group, h = g * group + qi % group;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = 0; j <= pos0 + n; ++j) {
+      const float pj = sc[qi][j];
+      const float4 v = reinterpret_cast<const float4*>(vs[j])[d4];
+      acc.x += pj * v.x;
+      acc.y += pj * v.y;
+      acc.z += pj * v.z;
+      acc.w += pj * v.w;
+    }
+    const int f = h * D + 4 * d4;
+    const uint2 packed = make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
     if (b.att_t)        // the Wo product's operand, SW128 tiles (tensor-core path)
-      *reinterpret_cast<uint16_t*>(b.att_t + tc::sw128_offset(b.Rtc, base + n, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
-          f32_to_bf16(acc);
+      *reinterpret_cast<uint2*>(b.att_t + tc::sw128_offset(b.Rtc, base + n, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
+          packed;
     else
-      b.att[(size_t)(base + n) * p.NH * D + f] = f32_to_bf16(acc);
+      *reinterpret_cast<uint2*>(b.att + (size_t)(base + n) * p.NH * D + f) = packed;
   }
 }
 
