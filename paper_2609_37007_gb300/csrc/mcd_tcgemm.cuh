@@ -10,7 +10,8 @@
 // (8-row groups 1024 bytes apart).  No tensor map is needed.
 //
 // One CTA computes a 128 x BN tile of D (UMMA M = 128, N = BN, K = 16 per instruction): a
-// producer thread streams the k-slices of A and B through a 4-stage ring (mbarrier
+// producer thread streams the k-slices of A and B through a ring of as many stages as fit in
+// 200 KB (4 to 6; mbarrier
 // complete_tx), one thread issues the MMAs and returns each stage with tcgen05.commit, and
 // after the last commit the four warps read the accumulator back from TMEM (warp w owns
 // lanes 32w..32w+31 = rows m of the tile) and hand every value to the epilogue functor.
@@ -24,7 +25,7 @@ namespace tc {
 
 constexpr int kBM = 128;         // rows of A per tile (UMMA M)
 constexpr int kBK = 64;          // k per stage: one 128-byte swizzled row
-constexpr int kStages = 4;
+constexpr int kStageBudget = 200 * 1024;   // shared memory for the ring (stages of one k-slice)
 constexpr int kThreads = 128;
 
 // Byte offset of (row, 16-byte chunk c) of k-slice kt in the SW128 tile layout of a matrix
@@ -43,6 +44,7 @@ struct Layout {
   static constexpr int kBBytes = BN * 128;
   static constexpr int kStageBytes = (kDualA ? 2 : 1) * kABytes + (kDualB ? 2 : 1) * kBBytes;
   static constexpr int kTmemCols = (kDualA ? 2 : 1) * BN;
+  static constexpr int kStages = kStageBudget / kStageBytes > 8 ? 8 : kStageBudget / kStageBytes;
   static constexpr int kBarOff = kStages * kStageBytes;                 // full[s], empty[s], accum
   static constexpr int kTmemSlotOff = kBarOff + (2 * kStages + 1) * 8;
   static constexpr int kFlagOff = kTmemSlotOff + 4;
@@ -143,14 +145,14 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
   if (nk <= 0) return;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
-  uint64_t* empty = full + kStages;
-  uint64_t* accum = empty + kStages;
+  uint64_t* empty = full + L::kStages;
+  uint64_t* accum = empty + L::kStages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kTmemSlotOff);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kFlagOff);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < L::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -174,8 +176,8 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
     const uint64_t pol_a = policy_evict_first(), pol_b = policy_evict_last();
     int issued = 0;
     for (int i = 0; i < nk; ++i) {
-      const int s = i % kStages, kt = kt0 + i;
-      if (i >= kStages && !tc_wait(&empty[s], ((i / kStages) - 1) & 1, g.err, g.wait_ns)) {
+      const int s = i % L::kStages, kt = kt0 + i;
+      if (i >= L::kStages && !tc_wait(&empty[s], ((i / L::kStages) - 1) & 1, g.err, g.wait_ns)) {
         *abort_flag = 1;
         break;
       }
@@ -191,14 +193,14 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
       ++issued;
     }
     // every issued copy lands before the CTA may exit
-    for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i)
-      tc_wait(&full[i % kStages], (i / kStages) & 1, g.err, g.wait_ns);
+    for (int i = (issued > L::kStages ? issued - L::kStages : 0); i < issued; ++i)
+      tc_wait(&full[i % L::kStages], (i / L::kStages) & 1, g.err, g.wait_ns);
   } else if (warp == 1 && lane == 0) {
     // MMA issuer
     constexpr uint32_t idesc = idesc_bf16<BN>();
     for (int i = 0; i < nk; ++i) {
-      const int s = i % kStages;
-      if (!tc_wait(&full[s], (i / kStages) & 1, g.err, g.wait_ns)) {
+      const int s = i % L::kStages;
+      if (!tc_wait(&full[s], (i / L::kStages) & 1, g.err, g.wait_ns)) {
         *abort_flag = 1;
         break;
       }
