@@ -25,6 +25,7 @@
 #include "mcd_internal.cuh"
 #include "mcd_sampler.cuh"
 #include "mcd_tcgemm.cuh"
+#include "mcd_tcops.cuh"
 
 namespace mcd {
 
@@ -104,7 +105,7 @@ struct BatchBufs {
 // Weights of the tensor-core GEMMs: per layer the row-major matrices as SW128 tiles.
 struct TcWeights {
   uint8_t* arena = nullptr;
-  size_t qkv = 0, g = 0, u = 0, o = 0, d = 0, layer = 0;     // offsets within a layer, layer stride
+  TcLayerOffsets off;                                         // within a layer, layer stride
   uint8_t* heads = nullptr;                                   // [n_pos][V x H] SW128 tiles
 };
 
@@ -493,148 +494,6 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
   }
 }
 
-// ---- tensor-core GEMM path (tcgen05, mcd_tcgemm.cuh) ---------------------------------------
-// With all of qkv_dim, F and H multiples of 128 the QKV, Wo, gate/up and down products run on
-// the tcgen05 GEMM.  Their operand rows are written as SW128 tiles by the kernel that produces
-// them: the normalised rows by the pass that also folds the k-split partial sums of the
-// previous residual product into the residual stream, the attention outputs by the attention
-// kernel, the SwiGLU outputs by the gate/up epilogue.
-
-// Normalised operand rows x * gain / rms(x) of the call's packed rows as SW128 tiles (hi; with
-// lo also the bf16 remainder), one 8-element chunk per thread.
-__global__ void __launch_bounds__(256) tc_norm_operand_kernel(const float* __restrict__ X, const float* __restrict__ gain,
-                                                              const float* __restrict__ ss, int H, float eps,
-                                                              const BatchInfo* info, int Rtc, uint8_t* hi, uint8_t* lo) {
-  const int M = info->M, cpr = H / 8;
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * cpr; i += gridDim.x * blockDim.x) {
-    const int r = i / cpr, ch = i - r * cpr, k = ch * 8;
-    const float s = rsqrtf(ss[r] / (float)H + eps);
-    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k));
-    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k + 4));
-    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + k));
-    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + k + 4));
-    const float v[8] = {x0.x * g0.x * s, x0.y * g0.y * s, x0.z * g0.z * s, x0.w * g0.w * s,
-                        x1.x * g1.x * s, x1.y * g1.y * s, x1.z * g1.z * s, x1.w * g1.w * s};
-    uint32_t h[4], l[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
-      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
-    }
-    const size_t off = tc::sw128_offset(Rtc, r, ch >> 3, ch & 7);
-    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
-    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
-  }
-}
-
-// Row-major bf16 [rows][K] -> rows row0.. of an SW128-tiled matrix of R rows (weight load).
-__global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0,
-                                      uint8_t* __restrict__ dst) {
-  const long long total = (long long)rows * (K / 8);
-  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
-    const int r = (int)(i / (K / 8)), ch = (int)(i % (K / 8));
-    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(R, row0 + r, ch >> 3, ch & 7)) =
-        *reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8);
-  }
-}
-
-constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
-constexpr int kTcBNGU = 128;      // gate/up (two accumulators)
-constexpr int kTcSplit = 4;       // k-splits of the residual products
-
-// q, k, v = W (x . g / rms) with the hi + lo operand.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
-                                                                  const BatchInfo* info) {
-  const int M = __ldg(&info->M);
-  tc::gemm_tile<kTcBN, false, true>(g, [&](int m, int n, float v, float) {
-    if (n < M) out[(size_t)n * ld + m] = v;
-  });
-}
-
-// gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
-// product (element (row n, feature m)).
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
-                                                                 const BatchInfo* info) {
-  const int M = __ldg(&info->M);
-  tc::gemm_tile<kTcBNGU, true, false>(g, [&](int m, int n, float gt, float up) {
-    if (n < M) {
-      const float v = gt / (1.0f + __expf(-gt)) * up;
-      *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
-          f32_to_bf16(v);
-    }
-  });
-}
-
-// Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
-// part[z][n][m] (plain stores); tc_resid_norm_kernel adds them into the residual stream.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
-                                                                    const BatchInfo* info) {
-  const int M = __ldg(&info->M);
-  float* pz = part + (size_t)blockIdx.z * Rtc * ld;
-  tc::gemm_tile<kTcBN, false, false>(g, [&](int m, int n, float v, float) {
-    if (n < M) pz[(size_t)n * ld + m] = v;
-  });
-}
-
-// Per packed row (one CTA, thread t owns elements 8t..8t+7): X += the nz partial sums, the
-// row's sum of squares (the next RMSNorm), and with a gain the next product's normalised
-// operand (hi; with lo also the remainder) as SW128 tiles.
-__global__ void __launch_bounds__(128) tc_resid_norm_kernel(float* X, const float* __restrict__ part, int nz, int Rtc,
-                                                            int H, const BatchInfo* info, float* ss_out,
-                                                            const float* __restrict__ gain, float eps, uint8_t* hi,
-                                                            uint8_t* lo) {
-  const int r = blockIdx.x;
-  if (r >= info->M) return;
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  const bool live = t < H / 8;
-  __shared__ float red[4];
-  float x[8];
-  float ss = 0.f;
-  if (live) {
-    float4* xr = reinterpret_cast<float4*>(X + (size_t)r * H + 8 * t);
-    float4 a = xr[0], b = xr[1];
-    for (int z = 0; z < nz; ++z) {
-      const float4* pr = reinterpret_cast<const float4*>(part + ((size_t)z * Rtc + r) * H + 8 * t);
-      const float4 u = __ldcg(pr), w = __ldcg(pr + 1);
-      a.x += u.x; a.y += u.y; a.z += u.z; a.w += u.w;
-      b.x += w.x; b.y += w.y; b.z += w.z; b.w += w.w;
-    }
-    xr[0] = a;
-    xr[1] = b;
-    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) ss += x[i] * x[i];
-  }
-#pragma unroll
-  for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
-  if (lane == 0) red[warp] = ss;
-  __syncthreads();
-  const float tot = red[0] + red[1] + red[2] + red[3];
-  if (t == 0) ss_out[r] = tot;
-  if (gain && live) {
-    const float s = rsqrtf(tot / (float)H + eps);
-    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t));
-    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t + 4));
-    const float v[8] = {x[0] * g0.x * s, x[1] * g0.y * s, x[2] * g0.z * s, x[3] * g0.w * s,
-                        x[4] * g1.x * s, x[5] * g1.y * s, x[6] * g1.z * s, x[7] * g1.w * s};
-    uint32_t h[4], l[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
-      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
-    }
-    const size_t off = tc::sw128_offset(Rtc, r, t >> 3, t & 7);
-    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
-    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
-  }
-}
-
-// Non-empty k-splits of a residual product over K (gemm_tile's split of the k-slices).
-static int tc_splits(int K) {
-  const int nk = K / tc::kBK, per = (nk + kTcSplit - 1) / kTcSplit;
-  return (nk + per - 1) / per;
-}
-
 // LM heads.  The (row, j) pairs of the call are grouped by head (head_list); group P starts at
 // operand row qoff(P) = the sum of the earlier groups rounded up to the tile width, so every
 // tile of the product belongs to one head.
@@ -712,11 +571,6 @@ __global__ void __launch_bounds__(tc::kThreads, 1) tc_heads_kernel(const tc::Gem
       logits[((size_t)r * kRecSlots + j) * V + m] = v + bias;
     }
   });
-}
-
-bool tc_supported(const FrameParams& p) {
-  return p.wdtype == MCD_WEIGHT_BF16 && p.qkv_dim % 128 == 0 && p.F % 128 == 0 && p.H % 128 == 0 &&
-         (p.NH * p.D) % 64 == 0 && p.H % 64 == 0 && p.F % 64 == 0;
 }
 
 // Per-row sums of squares of the residual stream after a residual GEMM (one warp per row):
@@ -1085,7 +939,7 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
   BATCH_ALLOC(b.act, sizeof(uint16_t) * R * p.F);
   BATCH_ALLOC(b.logits, sizeof(float) * R * kRecSlots * p.V);
   BATCH_ALLOC(b.recs, sizeof(TopkRec) * 2 * R * kRecSlots);
-  bs->use_tc = tc_supported(p);
+  bs->use_tc = tc_block_supported(p);
   if (bs->use_tc) {
     const int Rtc = (R + 127) / 128 * 128;
     b.Rtc = Rtc;
@@ -1101,14 +955,8 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
       BATCH_ALLOC(bs->tw.heads, (size_t)p.P * p.V * p.H * 2);
     }
     TcWeights& tw = bs->tw;
-    const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
-    tw.qkv = 0;
-    tw.g = tw.qkv + (size_t)p.qkv_dim * H * 2;
-    tw.u = tw.g + F * H * 2;
-    tw.o = tw.u + F * H * 2;
-    tw.d = tw.o + H * qd * 2;
-    tw.layer = tw.d + H * F * 2;
-    BATCH_ALLOC(tw.arena, tw.layer * p.L);
+    tw.off = tc_layer_offsets(p);
+    BATCH_ALLOC(tw.arena, tw.off.layer * p.L);
   }
 #undef BATCH_ALLOC
   if (cudaMemset(b.info, 0, sizeof(BatchInfo)) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -1119,12 +967,7 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmemHilo) != cudaSuccess)
       return fail(MCD_ERR_CUDA);
   if (bs->use_tc &&
-      (cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            tc::Layout<kTcBN, false, true>::kSmemBytes) != cudaSuccess ||
-       cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            tc::Layout<kTcBNGU, true, false>::kSmemBytes) != cudaSuccess ||
-       cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            tc::Layout<kTcBN, false, false>::kSmemBytes) != cudaSuccess ||
+      (tc_block_set_smem() != cudaSuccess ||
        cudaFuncSetAttribute(tc_heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                             tc::Layout<kTcBN, false, true>::kSmemBytes) != cudaSuccess))
     return fail(MCD_ERR_CUDA);
@@ -1135,19 +978,7 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
 // The tcgen05 GEMMs' copies of layer l's matrices (row-major bf16 sources, device).
 mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t st, const LayerSrc& src, int l) {
   if (!bs || !bs->use_tc) return MCD_OK;
-  const TcWeights& tw = bs->tw;
-  uint8_t* base = tw.arena + (size_t)l * tw.layer;
-  const int H = p.H, F = p.F, qd = p.NH * p.D, kd = p.NKV * p.D;
-  auto tile = [&](const uint8_t* s, int rows, int K, int R, int row0, size_t off) {
-    tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(s), rows, K, R, row0, base + off);
-  };
-  tile(src.wq, qd, H, p.qkv_dim, 0, tw.qkv);
-  tile(src.wk, kd, H, p.qkv_dim, qd, tw.qkv);
-  tile(src.wv, kd, H, p.qkv_dim, qd + kd, tw.qkv);
-  tile(src.wg, F, H, F, 0, tw.g);
-  tile(src.wu, F, H, F, 0, tw.u);
-  tile(src.wo, H, qd, H, 0, tw.o);
-  tile(src.wd, H, F, H, 0, tw.d);
+  tc_tile_layer(p, st, src.wq, src.wk, src.wv, src.wo, src.wg, src.wu, src.wd, bs->tw.arena + (size_t)l * bs->tw.off.layer);
   return cudaGetLastError() == cudaSuccess ? MCD_OK : MCD_ERR_CUDA;
 }
 
@@ -1188,41 +1019,41 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
     batch_pack_kernel<<<1, 256, 0, s>>>(p, b);
     batch_embed_kernel<<<R, 256, 0, s>>>(p, b);
     for (int l = 0; l < L && bs->use_tc; ++l) {
-      const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.layer;
+      const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.off.layer;
       const int Rtc = b.Rtc, qd = p.NH * p.D;
       const dim3 tblk(tc::kThreads);
       // RMSNorm -> QKV (hi + lo operand; after layer 0 written by the previous layer's last
       // residual pass)
       if (l == 0)
-        tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm, b.ss, H, p.eps, b.info, Rtc, b.xn_hi, b.xn_lo);
+        tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm, b.ss, H, p.eps, &b.info->M, Rtc, b.xn_hi, b.xn_lo);
       {
-        const tc::GemmArgs g{wl + bs->tw.qkv, nullptr, b.xn_hi, b.xn_lo, p.qkv_dim, Rtc, H, &b.info->M, p.err, p.wait_ns};
+        const tc::GemmArgs g{wl + bs->tw.off.qkv, nullptr, b.xn_hi, b.xn_lo, p.qkv_dim, Rtc, H, &b.info->M, p.err, p.wait_ns};
         tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
-            g, b.qkv, p.qkv_dim, b.info);
+            g, b.qkv, p.qkv_dim, &b.info->M);
       }
       batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);      // -> att_t
       // Wo (k-split partials) -> residual, ss, the gate/up operand
       {
-        const tc::GemmArgs g{wl + bs->tw.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
+        const tc::GemmArgs g{wl + bs->tw.off.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
         tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.part, H, Rtc, b.info);
+            g, b.part, H, Rtc, &b.info->M);
       }
-      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, b.info, b.ss + (size_t)(2 * l + 1) * R,
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 1) * R,
                                              p.ffn_norm + (size_t)l * H, p.eps, b.xn_hi, nullptr);
       // gate/up -> SwiGLU (into the down product's operand)
       {
-        const tc::GemmArgs g{wl + bs->tw.g, wl + bs->tw.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
+        const tc::GemmArgs g{wl + bs->tw.off.g, wl + bs->tw.off.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
         tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
-            g, b.act_t, Rtc, b.info);
+            g, b.act_t, Rtc, &b.info->M);
       }
       // down (k-split partials) -> residual, ss, the next layer's QKV operand
       {
-        const tc::GemmArgs g{wl + bs->tw.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
+        const tc::GemmArgs g{wl + bs->tw.off.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
         tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.part, H, Rtc, b.info);
+            g, b.part, H, Rtc, &b.info->M);
       }
       const bool last = l + 1 == L;
-      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(p.F), Rtc, H, b.info, b.ss + (size_t)(2 * l + 2) * R,
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(p.F), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 2) * R,
                                              last ? nullptr : p.attn_norm + (size_t)(l + 1) * H, p.eps, b.xn_hi, b.xn_lo);
     }
     for (int l = 0; l < L && !bs->use_tc; ++l) {

@@ -27,6 +27,7 @@
 #include "mcd_internal.cuh"
 #include "mcd_sampler.cuh"
 #include "mcd_stage.cuh"
+#include "mcd_tcops.cuh"
 
 namespace mcd {
 
@@ -600,8 +601,177 @@ using namespace mcd;
 // ------------------------------------------------------------------------------------
 // Host side
 // ------------------------------------------------------------------------------------
+// Prompt prefill on the tensor cores: rows 0..T-2 of a T-token prompt go through the 28
+// layers as one batch (tcgen05 products, causal attention, K / V written to the cache); the
+// last row then runs through outer_kernel, which reads that cache and samples c0.
+struct OuterTc {
+  bool on = false;
+  int Rtc = 0;                     // prompt rows, rounded up to the tile width
+  uint8_t* w = nullptr;            // per layer: SW128 copies of the weights
+  TcLayerOffsets off;
+  float* X = nullptr;              // [Rtc][H] residual stream
+  float* ss = nullptr;             // [Rtc] sums of squares (the next RMSNorm)
+  float* qkv = nullptr;            // [Rtc][qkv_dim]
+  float* q = nullptr;              // [Rtc][NH * D] normalised, rotated queries
+  float* part = nullptr;           // [kTcSplit][Rtc][H] partial sums of the residual products
+  uint8_t *xn_hi = nullptr, *xn_lo = nullptr, *att_t = nullptr, *act_t = nullptr;   // operands
+  int* rows = nullptr;             // device: live rows
+};
+
+__global__ void pf_set_rows_kernel(int* rows, int n) { *rows = n; }
+
+// Prompt rows: X = the rows' text embeddings (bf16 table), ss = their sums of squares.  One
+// CTA per row, thread t owns elements 8t..8t+7.
+__global__ void __launch_bounds__(128) pf_embed_kernel(const int* __restrict__ ids, const int* nrows,
+                                                       const uint8_t* __restrict__ table, int vocab, int H, float* X,
+                                                       float* ss, int* err) {
+  const int r = blockIdx.x;
+  if (r >= *nrows) return;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  int id = ids[r];
+  if (id < 0 || id >= vocab) {              // an id outside the text table fails the prefill
+    if (t == 0) atomicCAS(err, 0, (int)MCD_ERR_INVALID_ARG);
+    id = 0;
+  }
+  __shared__ float red[4];
+  float s2 = 0.f;
+  if (t < H / 8) {
+    const uint4 w = __ldg(reinterpret_cast<const uint4*>(table + ((size_t)id * H + 8 * t) * 2));
+    const float v[8] = {bf16_lo_f32(w.x), bf16_hi_f32(w.x), bf16_lo_f32(w.y), bf16_hi_f32(w.y),
+                        bf16_lo_f32(w.z), bf16_hi_f32(w.z), bf16_lo_f32(w.w), bf16_hi_f32(w.w)};
+    float4* xr = reinterpret_cast<float4*>(X + (size_t)r * H + 8 * t);
+    xr[0] = make_float4(v[0], v[1], v[2], v[3]);
+    xr[1] = make_float4(v[4], v[5], v[6], v[7]);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s2 += v[i] * v[i];
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) s2 += __shfl_xor_sync(0xFFFFFFFFu, s2, off);
+  if (lane == 0) red[warp] = s2;
+  __syncthreads();
+  if (t == 0) ss[r] = red[0] + red[1] + red[2] + red[3];
+}
+
+// QK-norm + RoPE (position = row index) of every prompt row's query and key heads; K and V
+// rounded to bf16 into layer l's cache ([NKV][cap][D]), the rotated queries (fp32) into q.
+// One warp per (row, vector), lane holding dims lane + 32 i.
+__global__ void __launch_bounds__(256) pf_rope_kv_kernel(const float* __restrict__ qkv, int qkv_dim, const int* nrows,
+                                                         int NH, int NKV, int D, int qk_norm, const float* qn,
+                                                         const float* kn, float eps, const float2* __restrict__ rope,
+                                                         uint16_t* kc, uint16_t* vc, int cap, float* q) {
+  const int vecs = NH + 2 * NKV, w = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  const int r = w / vecs, vi = w - r * vecs;
+  if (r >= *nrows) return;
+  const int kind = vi < NH ? 0 : (vi < NH + NKV ? 1 : 2), h = kind == 0 ? vi : (kind == 1 ? vi - NH : vi - NH - NKV);
+  const int nd = D >> 5, half = D >> 1;
+  const float* src = qkv + (size_t)r * qkv_dim + (kind == 0 ? h * D : NH * D + (kind == 2 ? NKV * D : 0) + h * D);
+  float x[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) x[i] = i < nd ? __ldcg(src + lane + 32 * i) : 0.f;
+  if (kind < 2) {
+    if (qk_norm) {
+      float ssq = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ssq += x[i] * x[i];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ssq += __shfl_xor_sync(0xFFFFFFFFu, ssq, off);
+      const float scl = rsqrtf(ssq / (float)D + eps);
+      const float* gg = kind == 0 ? qn : kn;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) x[i] = x[i] * scl * __ldg(gg + lane + 32 * i);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if (i < nd / 2) {
+        const float2 cs = __ldg(rope + (size_t)r * half + lane + 32 * i);
+        const float a = x[i], b = x[i + nd / 2];
+        x[i] = a * cs.x - b * cs.y;
+        x[i + nd / 2] = b * cs.x + a * cs.y;
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (i < nd) {
+      const int d = lane + 32 * i;
+      if (kind == 0)
+        q[(size_t)r * NH * D + h * D + d] = x[i];
+      else
+        (kind == 1 ? kc : vc)[((size_t)h * cap + r) * D + d] = (uint16_t)bf16_rn_bits(x[i]);
+    }
+  }
+}
+
+// Causal attention of the prompt rows over the bf16 cache: one warp per (row, query head),
+// keys in blocks of 32 (lane j scores key j0 + j over all dims against the query in shared
+// memory; running max and sum), P.V with lane owning dims lane + 32 i; the output row goes to
+// the Wo operand (SW128 tiles, bf16).
+__global__ void __launch_bounds__(256) pf_attn_kernel(const float* __restrict__ q, const int* nrows, int NH, int NKV,
+                                                      int D, const uint16_t* __restrict__ kc,
+                                                      const uint16_t* __restrict__ vc, int cap, int Rtc,
+                                                      uint8_t* att_t) {
+  __shared__ __align__(16) float qsh[8][128];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, w = blockIdx.x * 8 + warp;
+  const int r = w / NH, h = w - r * NH;
+  if (r >= *nrows) return;                  // whole warp
+  const int g = h / (NH / NKV), nd = D >> 5;
+  for (int d = lane; d < D; d += 32) qsh[warp][d] = __ldcg(q + (size_t)r * NH * D + h * D + d);
+  __syncwarp();
+  const float scale = rsqrtf((float)D);
+  const uint16_t* kb = kc + (size_t)g * cap * D;
+  const uint16_t* vb = vc + (size_t)g * cap * D;
+  float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j0 = 0; j0 <= r; j0 += 32) {
+    const int j = j0 + lane;
+    float sc = -INFINITY;
+    if (j <= r) {
+      const uint4* kr = reinterpret_cast<const uint4*>(kb + (size_t)j * D);
+      float a0 = 0.f, a1 = 0.f;
+      for (int c = 0; c < D / 8; ++c) {
+        const uint4 kk = __ldg(kr + c);
+        const float* qq = qsh[warp] + 8 * c;
+        a0 += qq[0] * bf16_lo_f32(kk.x) + qq[1] * bf16_hi_f32(kk.x) + qq[2] * bf16_lo_f32(kk.y) + qq[3] * bf16_hi_f32(kk.y);
+        a1 += qq[4] * bf16_lo_f32(kk.z) + qq[5] * bf16_hi_f32(kk.z) + qq[6] * bf16_lo_f32(kk.w) + qq[7] * bf16_hi_f32(kk.w);
+      }
+      sc = (a0 + a1) * scale;
+    }
+    float mb = sc;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) mb = fmaxf(mb, __shfl_xor_sync(0xFFFFFFFFu, mb, off));
+    const float mn = fmaxf(m, mb);                       // finite: key j0 <= r is live
+    const float corr = __expf(m - mn);
+    const float pj = j <= r ? __expf(sc - mn) : 0.f;
+    float ps = pj;
+#pragma unroll
+    for (int off = 16; off; off >>= 1) ps += __shfl_xor_sync(0xFFFFFFFFu, ps, off);
+    l = l * corr + ps;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[i] *= corr;
+    const int nk = min(32, r - j0 + 1);
+    for (int jj = 0; jj < nk; ++jj) {
+      const float pb = __shfl_sync(0xFFFFFFFFu, pj, jj);
+      const uint16_t* vr = vb + (size_t)(j0 + jj) * D;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) acc[i] += pb * bf16_lo_f32((uint32_t)__ldg(vr + lane + 32 * i));
+    }
+    m = mn;
+  }
+  const float inv = 1.0f / l;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (i < nd) {
+      const int f = h * D + lane + 32 * i;
+      *reinterpret_cast<uint16_t*>(att_t + tc::sw128_offset(Rtc, r, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
+          (uint16_t)bf16_rn_bits(acc[i] * inv);
+    }
+  }
+}
+
 struct mcd_outer {
   mcd_outer_config cfg;
+  OuterTc tc;
   mcd_ctx* inner = nullptr;
   cudaStream_t stream = nullptr;
   FrameParams fp;
@@ -794,6 +964,25 @@ mcd_status mcd_outer_create(const mcd_outer_config* cfg, mcd_ctx* inner, mcd_out
   OUTER_ALLOC(o->cond, sizeof(float) * p.H);
   OUTER_ALLOC(o->c0emb, sizeof(float) * p.H);
   OUTER_ALLOC(o->last_codes, sizeof(int) * (o->P + 1));
+  OuterTc& t = o->tc;
+  t.on = tc_block_supported(p) && s.cap >= 2;
+  if (t.on) {
+    const int Rtc = (s.cap + tc::kBM - 1) / tc::kBM * tc::kBM;
+    t.Rtc = Rtc;
+    t.off = tc_layer_offsets(p);
+    OUTER_ALLOC(t.w, t.off.layer * p.L);
+    OUTER_ALLOC(t.X, sizeof(float) * (size_t)Rtc * p.H);
+    OUTER_ALLOC(t.ss, sizeof(float) * (size_t)Rtc);
+    OUTER_ALLOC(t.qkv, sizeof(float) * (size_t)Rtc * p.qkv_dim);
+    OUTER_ALLOC(t.q, sizeof(float) * (size_t)Rtc * p.NH * p.D);
+    OUTER_ALLOC(t.part, sizeof(float) * (size_t)kTcSplit * Rtc * p.H);
+    OUTER_ALLOC(t.xn_hi, (size_t)Rtc * p.H * 2);
+    OUTER_ALLOC(t.xn_lo, (size_t)Rtc * p.H * 2);
+    OUTER_ALLOC(t.att_t, (size_t)Rtc * p.NH * p.D * 2);
+    OUTER_ALLOC(t.act_t, (size_t)Rtc * p.F * 2);
+    OUTER_ALLOC(t.rows, sizeof(int));
+    if (tc_block_set_smem() != cudaSuccess) return fail(MCD_ERR_CUDA);
+  }
 #undef OUTER_ALLOC
   s.c0_out = o->c0_buf;
   s.cond_out = o->cond;
@@ -879,6 +1068,9 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
                 at[pre + "wd"], at[pre + "attn_norm"], at[pre + "ffn_norm"],
                 p.qk_norm ? at[pre + "q_norm"] : nullptr, p.qk_norm ? at[pre + "k_norm"] : nullptr};
     load_layer(p, o->stream, ls, l);
+    if (o->tc.on)
+      tc_tile_layer(p, o->stream, ls.wq, ls.wk, ls.wv, ls.wo, ls.wg, ls.wu, ls.wd,
+                    o->tc.w + (size_t)l * o->tc.off.layer);
   }
   if (cudaStreamSynchronize(o->stream) != cudaSuccess) return cleanup(MCD_ERR_CUDA);
   off = 0;
@@ -906,6 +1098,57 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
   return s;
 }
 
+// Rows 0..n-1 of the prompt (positions 0..n-1) through every layer on the tensor cores,
+// leaving their K / V in the cache.
+static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n) {
+  const FrameParams& p = o->fp;
+  const OuterTc& t = o->tc;
+  const OuterStep& st = o->st;
+  cudaStream_t s = o->stream;
+  const int H = p.H, L = p.L, Rtc = t.Rtc, qd = p.NH * p.D, kvl = p.NKV * st.cap * p.D;
+  const dim3 tblk(tc::kThreads);
+  pf_set_rows_kernel<<<1, 1, 0, s>>>(t.rows, n);
+  pf_embed_kernel<<<n, 128, 0, s>>>(text_ids, t.rows, st.text_table, st.text_vocab, H, t.X, t.ss, p.err);
+  tc_norm_operand_kernel<<<256, 256, 0, s>>>(t.X, p.attn_norm, t.ss, H, p.eps, t.rows, Rtc, t.xn_hi, t.xn_lo);
+  for (int l = 0; l < L; ++l) {
+    const uint8_t* wl = t.w + (size_t)l * t.off.layer;
+    uint16_t* kc = reinterpret_cast<uint16_t*>(st.kcache) + (size_t)l * kvl;
+    uint16_t* vc = reinterpret_cast<uint16_t*>(st.vcache) + (size_t)l * kvl;
+    {
+      const tc::GemmArgs g{wl + t.off.qkv, nullptr, t.xn_hi, t.xn_lo, p.qkv_dim, Rtc, H, t.rows, p.err, p.wait_ns};
+      tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
+          g, t.qkv, p.qkv_dim, t.rows);
+    }
+    const int vecs = p.NH + 2 * p.NKV;
+    pf_rope_kv_kernel<<<(n * vecs + 7) / 8, 256, 0, s>>>(t.qkv, p.qkv_dim, t.rows, p.NH, p.NKV, p.D, p.qk_norm,
+                                                         p.q_norm + (size_t)l * p.D, p.k_norm + (size_t)l * p.D, p.eps,
+                                                         st.rope, kc, vc, st.cap, t.q);
+    pf_attn_kernel<<<(n * p.NH + 7) / 8, 256, 0, s>>>(t.q, t.rows, p.NH, p.NKV, p.D, kc, vc, st.cap, Rtc, t.att_t);
+    {
+      const tc::GemmArgs g{wl + t.off.o, nullptr, t.att_t, nullptr, H, Rtc, qd, t.rows, p.err, p.wait_ns};
+      tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+          g, t.part, H, Rtc, t.rows);
+    }
+    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(qd), Rtc, H, t.rows, t.ss, p.ffn_norm + (size_t)l * H,
+                                           p.eps, t.xn_hi, nullptr);
+    {
+      const tc::GemmArgs g{wl + t.off.g, wl + t.off.u, t.xn_hi, nullptr, p.F, Rtc, H, t.rows, p.err, p.wait_ns};
+      tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
+          g, t.act_t, Rtc, t.rows);
+    }
+    {
+      const tc::GemmArgs g{wl + t.off.d, nullptr, t.act_t, nullptr, H, Rtc, p.F, t.rows, p.err, p.wait_ns};
+      tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+          g, t.part, H, Rtc, t.rows);
+    }
+    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(p.F), Rtc, H, t.rows, t.ss,
+                                           l + 1 < L ? p.attn_norm + (size_t)(l + 1) * H : nullptr, p.eps, t.xn_hi,
+                                           t.xn_lo);
+  }
+  MCD_CHECK(cudaGetLastError());
+  return MCD_OK;
+}
+
 mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens, const int32_t* text_ids,
                              int32_t* c0_out) {
   if (!o || !text_ids || n_tokens < 1) return MCD_ERR_INVALID_ARG;
@@ -914,7 +1157,15 @@ mcd_status mcd_outer_prefill(mcd_outer* o, uint32_t stream_id, int32_t n_tokens,
   const int R = prefill_rows(o);
   o->stream_id = stream_id;
   o->st.stream_id = stream_id;
-  for (int s0 = 0; s0 < n_tokens; s0 += R) {
+  // all but the last row on the tensor cores (when the shapes allow), the last through
+  // outer_kernel (c0 head and sampling)
+  int first = 0;
+  if (o->tc.on && n_tokens >= 2) {
+    mcd_status r = outer_tc_prefill(o, text_ids, n_tokens - 1);
+    if (r != MCD_OK) return r;
+    first = n_tokens - 1;
+  }
+  for (int s0 = first; s0 < n_tokens; s0 += R) {
     OuterStep s = o->st;
     s.pos0 = s0;
     s.nr = std::min(R, n_tokens - s0);

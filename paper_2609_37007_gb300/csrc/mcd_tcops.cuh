@@ -1,0 +1,205 @@
+// The transformer-block products of many rows on the tcgen05 GEMM (mcd_tcgemm.cuh), shared by
+// the batched path (many streams per call) and the CodeDecoder prompt prefill: with bf16
+// weights and qkv_dim, F, H multiples of 128 the QKV, Wo, gate/up and down products run on
+// the tensor cores.  Their operand rows are written as SW128 tiles by the kernel that
+// produces them: the normalised rows by the pass that also folds the k-split partial sums of
+// the previous residual product into the residual stream (tc_resid_norm_kernel), the
+// attention outputs by the attention kernel, the SwiGLU outputs by the gate/up epilogue.
+// Every kernel reads its live row count from device memory (*nrows, rows beyond it are
+// neither computed nor written).  Internal linkage: each translation unit has its copy.
+#pragma once
+#include "mcd_internal.cuh"
+#include "mcd_tcgemm.cuh"
+
+namespace mcd {
+namespace {
+
+
+// Normalised operand rows x * gain / rms(x) of the call's packed rows as SW128 tiles (hi; with
+// lo also the bf16 remainder), one 8-element chunk per thread.
+__global__ void __launch_bounds__(256) tc_norm_operand_kernel(const float* __restrict__ X, const float* __restrict__ gain,
+                                                              const float* __restrict__ ss, int H, float eps,
+                                                              const int* nrows, int Rtc, uint8_t* hi, uint8_t* lo) {
+  const int M = *nrows, cpr = H / 8;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < M * cpr; i += gridDim.x * blockDim.x) {
+    const int r = i / cpr, ch = i - r * cpr, k = ch * 8;
+    const float s = rsqrtf(ss[r] / (float)H + eps);
+    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k));
+    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(X + (size_t)r * H + k + 4));
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + k));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + k + 4));
+    const float v[8] = {x0.x * g0.x * s, x0.y * g0.y * s, x0.z * g0.z * s, x0.w * g0.w * s,
+                        x1.x * g1.x * s, x1.y * g1.y * s, x1.z * g1.z * s, x1.w * g1.w * s};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
+    }
+    const size_t off = tc::sw128_offset(Rtc, r, ch >> 3, ch & 7);
+    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+// Row-major bf16 [rows][K] -> rows row0.. of an SW128-tiled matrix of R rows (weight load).
+__global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0,
+                                      uint8_t* __restrict__ dst) {
+  const long long total = (long long)rows * (K / 8);
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+    const int r = (int)(i / (K / 8)), ch = (int)(i % (K / 8));
+    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(R, row0 + r, ch >> 3, ch & 7)) =
+        *reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8);
+  }
+}
+
+constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
+constexpr int kTcBNGU = 128;      // gate/up (two accumulators)
+constexpr int kTcSplit = 4;       // k-splits of the residual products
+
+// q, k, v = W (x . g / rms) with the hi + lo operand.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
+                                                                  const int* nrows) {
+  const int M = *nrows;
+  tc::gemm_tile<kTcBN, false, true>(g, [&](int m, int n, float v, float) {
+    if (n < M) out[(size_t)n * ld + m] = v;
+  });
+}
+
+// gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
+// product (element (row n, feature m)).
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
+                                                                 const int* nrows) {
+  const int M = *nrows;
+  tc::gemm_tile<kTcBNGU, true, false>(g, [&](int m, int n, float gt, float up) {
+    if (n < M) {
+      const float v = gt / (1.0f + __expf(-gt)) * up;
+      *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
+          (uint16_t)bf16_rn_bits(v);
+    }
+  });
+}
+
+// Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
+// part[z][n][m] (plain stores); tc_resid_norm_kernel adds them into the residual stream.
+__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
+                                                                    const int* nrows) {
+  const int M = *nrows;
+  float* pz = part + (size_t)blockIdx.z * Rtc * ld;
+  tc::gemm_tile<kTcBN, false, false>(g, [&](int m, int n, float v, float) {
+    if (n < M) pz[(size_t)n * ld + m] = v;
+  });
+}
+
+// Per packed row (one CTA, thread t owns elements 8t..8t+7): X += the nz partial sums, the
+// row's sum of squares (the next RMSNorm), and with a gain the next product's normalised
+// operand (hi; with lo also the remainder) as SW128 tiles.
+__global__ void __launch_bounds__(128) tc_resid_norm_kernel(float* X, const float* __restrict__ part, int nz, int Rtc,
+                                                            int H, const int* nrows, float* ss_out,
+                                                            const float* __restrict__ gain, float eps, uint8_t* hi,
+                                                            uint8_t* lo) {
+  const int r = blockIdx.x;
+  if (r >= *nrows) return;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const bool live = t < H / 8;
+  __shared__ float red[4];
+  float x[8];
+  float ss = 0.f;
+  if (live) {
+    float4* xr = reinterpret_cast<float4*>(X + (size_t)r * H + 8 * t);
+    float4 a = xr[0], b = xr[1];
+    for (int z = 0; z < nz; ++z) {
+      const float4* pr = reinterpret_cast<const float4*>(part + ((size_t)z * Rtc + r) * H + 8 * t);
+      const float4 u = __ldcg(pr), w = __ldcg(pr + 1);
+      a.x += u.x; a.y += u.y; a.z += u.z; a.w += u.w;
+      b.x += w.x; b.y += w.y; b.z += w.z; b.w += w.w;
+    }
+    xr[0] = a;
+    xr[1] = b;
+    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss += x[i] * x[i];
+  }
+#pragma unroll
+  for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  const float tot = red[0] + red[1] + red[2] + red[3];
+  if (t == 0) ss_out[r] = tot;
+  if (gain && live) {
+    const float s = rsqrtf(tot / (float)H + eps);
+    const float4 g0 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t));
+    const float4 g1 = __ldg(reinterpret_cast<const float4*>(gain + 8 * t + 4));
+    const float v[8] = {x[0] * g0.x * s, x[1] * g0.y * s, x[2] * g0.z * s, x[3] * g0.w * s,
+                        x[4] * g1.x * s, x[5] * g1.y * s, x[6] * g1.z * s, x[7] * g1.w * s};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      h[q] = pack_bf16x2(v[2 * q], v[2 * q + 1]);
+      l[q] = pack_bf16x2(v[2 * q] - bf16_lo_f32(h[q]), v[2 * q + 1] - bf16_hi_f32(h[q]));
+    }
+    const size_t off = tc::sw128_offset(Rtc, r, t >> 3, t & 7);
+    *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+    if (lo) *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+  }
+}
+
+// Non-empty k-splits of a residual product over K (gemm_tile's split of the k-slices).
+static int tc_splits(int K) {
+  const int nk = K / tc::kBK, per = (nk + kTcSplit - 1) / kTcSplit;
+  return (nk + per - 1) / per;
+}
+
+
+// The transformer-block products can use the tensor-core GEMM (shape and dtype limits).
+bool tc_block_supported(const FrameParams& p) {
+  return p.wdtype == MCD_WEIGHT_BF16 && p.qkv_dim % 128 == 0 && p.F % 128 == 0 && p.H % 128 == 0 &&
+         (p.NH * p.D) % 64 == 0 && p.H % 64 == 0 && p.F % 64 == 0 && p.H <= 1024;
+}
+
+// SW128 copies of one layer's weights: [qkv | g | u | o | d], offsets within a layer.
+struct TcLayerOffsets {
+  size_t qkv = 0, g = 0, u = 0, o = 0, d = 0, layer = 0;
+};
+inline TcLayerOffsets tc_layer_offsets(const FrameParams& p) {
+  TcLayerOffsets t;
+  const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
+  t.qkv = 0;
+  t.g = t.qkv + (size_t)p.qkv_dim * H * 2;
+  t.u = t.g + F * H * 2;
+  t.o = t.u + F * H * 2;
+  t.d = t.o + H * qd * 2;
+  t.layer = t.d + H * F * 2;
+  return t;
+}
+// Tile layer l's row-major bf16 sources (device) into the SW128 copies at base.
+inline void tc_tile_layer(const FrameParams& p, cudaStream_t st, const uint8_t* wq, const uint8_t* wk, const uint8_t* wv,
+                          const uint8_t* wo, const uint8_t* wg, const uint8_t* wu, const uint8_t* wd, uint8_t* base) {
+  const TcLayerOffsets t = tc_layer_offsets(p);
+  const int H = p.H, F = p.F, qd = p.NH * p.D, kd = p.NKV * p.D;
+  auto tile = [&](const uint8_t* s, int rows, int K, int R, int row0, size_t off) {
+    tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(s), rows, K, R, row0, base + off);
+  };
+  tile(wq, qd, H, p.qkv_dim, 0, t.qkv);
+  tile(wk, kd, H, p.qkv_dim, qd, t.qkv);
+  tile(wv, kd, H, p.qkv_dim, qd + kd, t.qkv);
+  tile(wg, F, H, F, 0, t.g);
+  tile(wu, F, H, F, 0, t.u);
+  tile(wo, H, qd, H, 0, t.o);
+  tile(wd, H, F, H, 0, t.d);
+}
+// Dynamic shared memory of the block kernels (once per translation unit).
+inline cudaError_t tc_block_set_smem() {
+  cudaError_t e = cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       tc::Layout<kTcBN, false, true>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::Layout<kTcBNGU, true, false>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::Layout<kTcBN, false, false>::kSmemBytes);
+  return e;
+}
+
+}  // namespace
+}  // namespace mcd
