@@ -1021,21 +1021,21 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
     for (int l = 0; l < L && bs->use_tc; ++l) {
       const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.off.layer;
       const int Rtc = b.Rtc, qd = p.NH * p.D;
-      const dim3 tblk(tc::kThreads);
+      const dim3 tblk(tc::kThreads), pblk(tc::kPThreads);
       // RMSNorm -> QKV (hi + lo operand; after layer 0 written by the previous layer's last
       // residual pass)
       if (l == 0)
         tc_norm_operand_kernel<<<256, blk, 0, s>>>(b.X, p.attn_norm, b.ss, H, p.eps, &b.info->M, Rtc, b.xn_hi, b.xn_lo);
       {
         const tc::GemmArgs g{wl + bs->tw.off.qkv, nullptr, b.xn_hi, b.xn_lo, p.qkv_dim, Rtc, H, &b.info->M, p.err, p.wait_ns};
-        tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
+        tc_qkv_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, p.qkv_dim, 1), p.n_cta), pblk, tc::PLayout<kTcBN, false, true>::kSmemBytes, s>>>(
             g, b.qkv, p.qkv_dim, &b.info->M);
       }
       batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);      // -> att_t
       // Wo (k-split partials) -> residual, ss, the gate/up operand
       {
         const tc::GemmArgs g{wl + bs->tw.off.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
-        tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+        tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
             g, b.part, H, Rtc, &b.info->M);
       }
       tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 1) * R,
@@ -1043,13 +1043,13 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       // gate/up -> SwiGLU (into the down product's operand)
       {
         const tc::GemmArgs g{wl + bs->tw.off.g, wl + bs->tw.off.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
-        tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
+        tc_gu_kernel<<<tc_grid(tc_tiles(Rtc, kTcBNGU, p.F, 1), p.n_cta), pblk, tc::PLayout<kTcBNGU, true, false>::kSmemBytes, s>>>(
             g, b.act_t, Rtc, &b.info->M);
       }
       // down (k-split partials) -> residual, ss, the next layer's QKV operand
       {
         const tc::GemmArgs g{wl + bs->tw.off.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
-        tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+        tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
             g, b.part, H, Rtc, &b.info->M);
       }
       const bool last = l + 1 == L;

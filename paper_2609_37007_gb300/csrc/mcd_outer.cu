@@ -1106,7 +1106,7 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
   const OuterStep& st = o->st;
   cudaStream_t s = o->stream;
   const int H = p.H, L = p.L, Rtc = t.Rtc, qd = p.NH * p.D, kvl = p.NKV * st.cap * p.D;
-  const dim3 tblk(tc::kThreads);
+  const dim3 tblk(tc::kThreads), pblk(tc::kPThreads);
   pf_set_rows_kernel<<<1, 1, 0, s>>>(t.rows, n);
   pf_embed_kernel<<<n, 128, 0, s>>>(text_ids, t.rows, st.text_table, st.text_vocab, H, t.X, t.ss, p.err);
   tc_norm_operand_kernel<<<256, 256, 0, s>>>(t.X, p.attn_norm, t.ss, H, p.eps, t.rows, Rtc, t.xn_hi, t.xn_lo);
@@ -1116,7 +1116,7 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
     uint16_t* vc = reinterpret_cast<uint16_t*>(st.vcache) + (size_t)l * kvl;
     {
       const tc::GemmArgs g{wl + t.off.qkv, nullptr, t.xn_hi, t.xn_lo, p.qkv_dim, Rtc, H, t.rows, p.err, p.wait_ns};
-      tc_qkv_kernel<<<dim3(Rtc / kTcBN, p.qkv_dim / tc::kBM, 1), tblk, tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(
+      tc_qkv_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, p.qkv_dim, 1), p.n_cta), pblk, tc::PLayout<kTcBN, false, true>::kSmemBytes, s>>>(
           g, t.qkv, p.qkv_dim, t.rows);
     }
     const int vecs = p.NH + 2 * p.NKV;
@@ -1126,19 +1126,19 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
     pf_attn_kernel<<<(n * p.NH + 7) / 8, 256, 0, s>>>(t.q, t.rows, p.NH, p.NKV, p.D, kc, vc, st.cap, Rtc, t.att_t);
     {
       const tc::GemmArgs g{wl + t.off.o, nullptr, t.att_t, nullptr, H, Rtc, qd, t.rows, p.err, p.wait_ns};
-      tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+      tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
           g, t.part, H, Rtc, t.rows);
     }
     tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(qd), Rtc, H, t.rows, t.ss, p.ffn_norm + (size_t)l * H,
                                            p.eps, t.xn_hi, nullptr);
     {
       const tc::GemmArgs g{wl + t.off.g, wl + t.off.u, t.xn_hi, nullptr, p.F, Rtc, H, t.rows, p.err, p.wait_ns};
-      tc_gu_kernel<<<dim3(Rtc / kTcBNGU, p.F / tc::kBM, 1), tblk, tc::Layout<kTcBNGU, true, false>::kSmemBytes, s>>>(
+      tc_gu_kernel<<<tc_grid(tc_tiles(Rtc, kTcBNGU, p.F, 1), p.n_cta), pblk, tc::PLayout<kTcBNGU, true, false>::kSmemBytes, s>>>(
           g, t.act_t, Rtc, t.rows);
     }
     {
       const tc::GemmArgs g{wl + t.off.d, nullptr, t.act_t, nullptr, H, Rtc, p.F, t.rows, p.err, p.wait_ns};
-      tc_resid_kernel<<<dim3(Rtc / kTcBN, H / tc::kBM, kTcSplit), tblk, tc::Layout<kTcBN, false, false>::kSmemBytes, s>>>(
+      tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
           g, t.part, H, Rtc, t.rows);
     }
     tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(p.F), Rtc, H, t.rows, t.ss,

@@ -243,5 +243,191 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
                  : "memory");
 }
 
+// ---- persistent form ----------------------------------------------------------------------
+// Tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... over (n tile fastest, then m tile, then
+// k split) of an (N / BN) x (M / 128) x splits grid.  Six warps: warp 0 streams k-slices
+// through the shared-memory ring across tile boundaries, warp 1 issues the MMAs into one of
+// two TMEM accumulator buffers (tile i uses buffer i % 2), warps 2..5 read a finished buffer
+// back (warp w: TMEM lanes 32 (w % 4) ..) while the MMAs of the next tile already run, then
+// release it.  epi(m, n, split, v, v2).  Tiles whose first column is at or past *n_active are
+// skipped by every role alike.
+constexpr int kPThreads = 192;
+template <int BN, bool kDualA, bool kDualB>
+struct PLayout {
+  using L = Layout<BN, kDualA, kDualB>;
+  static constexpr int kAccCols = (kDualA ? 2 : 1) * BN;     // one accumulator buffer
+  static constexpr int kTmemCols = 2 * kAccCols;
+  static_assert(kTmemCols <= 512, "TMEM columns");
+  static constexpr int kBarOff = L::kStages * L::kStageBytes;  // full[S], empty[S], acc_full[2], acc_empty[2], drain
+  static constexpr int kTmemSlotOff = kBarOff + (2 * L::kStages + 5) * 8;
+  static constexpr int kFlagOff = kTmemSlotOff + 4;
+  static constexpr int kSmemBytes = kFlagOff + 4 + 1024;
+  static_assert(kSmemBytes <= 227 * 1024, "tensor-core GEMM stages exceed shared memory");
+};
+
+template <int BN, bool kDualA, bool kDualB, class Epi>
+__device__ __forceinline__ void gemm_persistent(const GemmArgs& g, int splits, Epi epi) {
+  using L = Layout<BN, kDualA, kDualB>;
+  using PL = PLayout<BN, kDualA, kDualB>;
+  constexpr int S = L::kStages;
+  extern __shared__ uint8_t tc_smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + PL::kBarOff);
+  uint64_t* empty = full + S;
+  uint64_t* acc_full = empty + S;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + PL::kTmemSlotOff);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + PL::kFlagOff);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_nt = g.N / BN, n_mt = g.M / kBM, n_tiles = n_nt * n_mt * splits;
+  const int nk_all = g.K / kBK, per = (nk_all + splits - 1) / splits;
+  const int n_live = g.n_active ? *g.n_active : g.N;
+  // tile t -> (n0, m0, split, k-slice range); false for a skipped tile
+  auto tile_of = [&](int t, int& n0, int& m0, int& z, int& kt0, int& nk) {
+    const int nt = t % n_nt, rest = t / n_nt;
+    n0 = nt * BN;
+    m0 = (rest % n_mt) * kBM;
+    z = rest / n_mt;
+    kt0 = z * per;
+    nk = min(nk_all, kt0 + per) - kt0;
+    return n0 < n_live && nk > 0;
+  };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);            // the four epilogue warps
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"((uint32_t)PL::kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {                          // producer
+      const uint64_t pol_a = policy_evict_first(), pol_b = policy_evict_last();
+      uint32_t c = 0;                         // k-slices issued
+      for (int t = blockIdx.x; t < n_tiles && !*abort_flag; t += gridDim.x) {
+        int n0, m0, z, kt0, nk;
+        if (!tile_of(t, n0, m0, z, kt0, nk)) continue;
+        for (int i = 0; i < nk; ++i, ++c) {
+          const int s = c % S;
+          if (c >= (uint32_t)S && !tc_wait(&empty[s], ((c / S) - 1) & 1, g.err, g.wait_ns)) {
+            *abort_flag = 1;
+            break;
+          }
+          if (*abort_flag) break;
+          const int kt = kt0 + i;
+          uint8_t* st = smem + s * L::kStageBytes;
+          const size_t ao = (size_t)kt * g.M * 128 + (size_t)m0 * 128, bo = (size_t)kt * g.N * 128 + (size_t)n0 * 128;
+          mbar_arrive_expect_tx(&full[s], L::kStageBytes);
+          bulk_g2s(st, g.a + ao, L::kABytes, &full[s], pol_a);
+          if (kDualA) bulk_g2s(st + L::kABytes, g.a2 + ao, L::kABytes, &full[s], pol_a);
+          uint8_t* sb = st + (kDualA ? 2 : 1) * L::kABytes;
+          bulk_g2s(sb, g.b + bo, L::kBBytes, &full[s], pol_b);
+          if (kDualB) bulk_g2s(sb + L::kBBytes, g.b2 + bo, L::kBBytes, &full[s], pol_b);
+        }
+      }
+      // every issued copy lands before the CTA may exit
+      for (uint32_t i = c > (uint32_t)S ? c - S : 0u; i < c; ++i) tc_wait(&full[i % S], (i / S) & 1, g.err, g.wait_ns);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {                          // MMA issuer
+      constexpr uint32_t idesc = idesc_bf16<BN>();
+      uint32_t c = 0;                         // k-slices consumed
+      int i_tile = 0;                         // tiles computed by this CTA
+      for (int t = blockIdx.x; t < n_tiles && !*abort_flag; t += gridDim.x) {
+        int n0, m0, z, kt0, nk;
+        if (!tile_of(t, n0, m0, z, kt0, nk)) continue;
+        const int b = i_tile & 1, v = i_tile >> 1;
+        if (v >= 1 && !tc_wait(&acc_empty[b], (v - 1) & 1, g.err, g.wait_ns)) {
+          *abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc = tmem + (uint32_t)(b * PL::kAccCols);
+        for (int i = 0; i < nk; ++i, ++c) {
+          const int s = c % S;
+          if (!tc_wait(&full[s], (c / S) & 1, g.err, g.wait_ns)) {
+            *abort_flag = 1;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * L::kStageBytes);
+          const uint32_t sb = sa + (kDualA ? 2 : 1) * L::kABytes;
+#pragma unroll
+          for (int j = 0; j < kBK / 16; ++j) {
+            const bool ac = (i | j) != 0;
+            umma_bf16(acc, sw128_desc(sa + 32 * j), sw128_desc(sb + 32 * j), idesc, ac);
+            if (kDualB) umma_bf16(acc, sw128_desc(sa + 32 * j), sw128_desc(sb + L::kBBytes + 32 * j), idesc, true);
+            if (kDualA)
+              umma_bf16(acc + BN, sw128_desc(sa + L::kABytes + 32 * j), sw128_desc(sb + 32 * j), idesc, ac);
+          }
+          umma_commit(&empty[s]);
+        }
+        umma_commit(&acc_full[b]);            // the tile's accumulator is complete
+        ++i_tile;
+      }
+    }
+  } else {
+    // epilogue warps 2..5: TMEM lane quarter (warp % 4)
+    const int q = warp & 3;
+    int i_tile = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+      int n0, m0, z, kt0, nk;
+      if (!tile_of(t, n0, m0, z, kt0, nk)) continue;
+      const int b = i_tile & 1, v = i_tile >> 1;
+      const bool ok = tc_wait(&acc_full[b], v & 1, g.err, g.wait_ns) && !*abort_flag;
+      __syncwarp();
+      tc_fence_after();
+      if (!ok) {
+        *abort_flag = 1;
+        break;
+      }
+      const int m = m0 + q * 32 + lane;
+      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(b * PL::kAccCols);
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 16) {
+        float vv[16], v2[16];
+        tmem_ld16(base + (uint32_t)c0, vv);
+        if (kDualA) tmem_ld16(base + (uint32_t)(BN + c0), v2);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) epi(m, n0 + c0 + j, z, vv[j], kDualA ? v2[j] : 0.f);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[b]);
+      ++i_tile;
+    }
+  }
+  // every MMA this CTA issued has completed before its TMEM is freed (also after an abort)
+  if (warp == 1 && lane == 0) {
+    umma_commit(drain);
+    tc_wait(drain, 0, g.err, g.wait_ns);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)PL::kTmemCols)
+                 : "memory");
+  }
+}
+
 }  // namespace tc
 }  // namespace mcd

@@ -58,20 +58,20 @@ constexpr int kTcBNGU = 128;      // gate/up (two accumulators)
 constexpr int kTcSplit = 4;       // k-splits of the residual products
 
 // q, k, v = W (x . g / rms) with the hi + lo operand.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
-                                                                  const int* nrows) {
+__global__ void __launch_bounds__(tc::kPThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
+                                                                   const int* nrows) {
   const int M = *nrows;
-  tc::gemm_tile<kTcBN, false, true>(g, [&](int m, int n, float v, float) {
+  tc::gemm_persistent<kTcBN, false, true>(g, 1, [&](int m, int n, int, float v, float) {
     if (n < M) out[(size_t)n * ld + m] = v;
   });
 }
 
 // gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
 // product (element (row n, feature m)).
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
-                                                                 const int* nrows) {
+__global__ void __launch_bounds__(tc::kPThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
+                                                                  const int* nrows) {
   const int M = *nrows;
-  tc::gemm_tile<kTcBNGU, true, false>(g, [&](int m, int n, float gt, float up) {
+  tc::gemm_persistent<kTcBNGU, true, false>(g, 1, [&](int m, int n, int, float gt, float up) {
     if (n < M) {
       const float v = gt / (1.0f + __expf(-gt)) * up;
       *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
@@ -82,12 +82,11 @@ __global__ void __launch_bounds__(tc::kThreads, 1) tc_gu_kernel(const tc::GemmAr
 
 // Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
 // part[z][n][m] (plain stores); tc_resid_norm_kernel adds them into the residual stream.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
-                                                                    const int* nrows) {
+__global__ void __launch_bounds__(tc::kPThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
+                                                                     const int* nrows) {
   const int M = *nrows;
-  float* pz = part + (size_t)blockIdx.z * Rtc * ld;
-  tc::gemm_tile<kTcBN, false, false>(g, [&](int m, int n, float v, float) {
-    if (n < M) pz[(size_t)n * ld + m] = v;
+  tc::gemm_persistent<kTcBN, false, false>(g, kTcSplit, [&](int m, int n, int z, float v, float) {
+    if (n < M) part[((size_t)z * Rtc + n) * ld + m] = v;
   });
 }
 
@@ -191,15 +190,19 @@ inline void tc_tile_layer(const FrameParams& p, cudaStream_t st, const uint8_t* 
 // Dynamic shared memory of the block kernels (once per translation unit).
 inline cudaError_t tc_block_set_smem() {
   cudaError_t e = cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       tc::Layout<kTcBN, false, true>::kSmemBytes);
+                                       tc::PLayout<kTcBN, false, true>::kSmemBytes);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::Layout<kTcBNGU, true, false>::kSmemBytes);
+                             tc::PLayout<kTcBNGU, true, false>::kSmemBytes);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::Layout<kTcBN, false, false>::kSmemBytes);
+                             tc::PLayout<kTcBN, false, false>::kSmemBytes);
   return e;
 }
+
+// Persistent launch shape: one CTA per SM at most, one per tile at least.
+inline dim3 tc_grid(int n_tiles, int n_sm) { return dim3(n_tiles < n_sm ? n_tiles : n_sm); }
+inline int tc_tiles(int N, int BN, int M, int splits) { return (N / BN) * (M / tc::kBM) * splits; }
 
 }  // namespace
 }  // namespace mcd
