@@ -1043,8 +1043,7 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       // gate/up -> SwiGLU (into the down product's operand)
       {
         const tc::GemmArgs g{wl + bs->tw.off.g, wl + bs->tw.off.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
-        tc_gu_kernel<<<tc_grid(tc_tiles(Rtc, kTcBNGU, p.F, 1), p.n_cta), pblk, tc::PLayout<kTcBNGU, true, false>::kSmemBytes, s>>>(
-            g, b.act_t, Rtc, &b.info->M);
+        tc_launch_gu(g, b.act_t, Rtc, &b.info->M, p.F, p.n_cta, s);
       }
       // down (k-split partials) -> residual, ss, the next layer's QKV operand
       {

@@ -1133,8 +1133,7 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
                                            p.eps, t.xn_hi, nullptr);
     {
       const tc::GemmArgs g{wl + t.off.g, wl + t.off.u, t.xn_hi, nullptr, p.F, Rtc, H, t.rows, p.err, p.wait_ns};
-      tc_gu_kernel<<<tc_grid(tc_tiles(Rtc, kTcBNGU, p.F, 1), p.n_cta), pblk, tc::PLayout<kTcBNGU, true, false>::kSmemBytes, s>>>(
-          g, t.act_t, Rtc, t.rows);
+      tc_launch_gu(g, t.act_t, Rtc, t.rows, p.F, p.n_cta, s);
     }
     {
       const tc::GemmArgs g{wl + t.off.d, nullptr, t.act_t, nullptr, H, Rtc, p.F, t.rows, p.err, p.wait_ns};

@@ -54,7 +54,8 @@ __global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows
 }
 
 constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
-constexpr int kTcBNGU = 128;      // gate/up (two accumulators)
+// gate/up (two accumulators): 128-row tiles from 512 packed rows on, else 64 (more tiles)
+inline int tc_bn_gu(int Rtc) { return Rtc >= 512 ? 128 : 64; }
 constexpr int kTcSplit = 4;       // k-splits of the residual products
 
 // q, k, v = W (x . g / rms) with the hi + lo operand.
@@ -68,10 +69,11 @@ __global__ void __launch_bounds__(tc::kPThreads, 1) tc_qkv_kernel(const tc::Gemm
 
 // gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
 // product (element (row n, feature m)).
+template <int BN>
 __global__ void __launch_bounds__(tc::kPThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
                                                                   const int* nrows) {
   const int M = *nrows;
-  tc::gemm_persistent<kTcBNGU, true, false>(g, 1, [&](int m, int n, int, float gt, float up) {
+  tc::gemm_persistent<BN, true, false>(g, 1, [&](int m, int n, int, float gt, float up) {
     if (n < M) {
       const float v = gt / (1.0f + __expf(-gt)) * up;
       *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
@@ -192,17 +194,34 @@ inline cudaError_t tc_block_set_smem() {
   cudaError_t e = cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        tc::PLayout<kTcBN, false, true>::kSmemBytes);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_gu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::PLayout<kTcBNGU, true, false>::kSmemBytes);
+    e = cudaFuncSetAttribute(tc_gu_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::PLayout<128, true, false>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_gu_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::PLayout<64, true, false>::kSmemBytes);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              tc::PLayout<kTcBN, false, false>::kSmemBytes);
   return e;
 }
 
+// gate/up -> SwiGLU into the down product's operand, at the tile width for Rtc rows.
+inline void tc_launch_gu(const tc::GemmArgs& g, uint8_t* act_t, int Rtc, const int* nrows, int F, int n_sm,
+                         cudaStream_t s);
+
 // Persistent launch shape: one CTA per SM at most, one per tile at least.
 inline dim3 tc_grid(int n_tiles, int n_sm) { return dim3(n_tiles < n_sm ? n_tiles : n_sm); }
 inline int tc_tiles(int N, int BN, int M, int splits) { return (N / BN) * (M / tc::kBM) * splits; }
+
+inline void tc_launch_gu(const tc::GemmArgs& g, uint8_t* act_t, int Rtc, const int* nrows, int F, int n_sm,
+                         cudaStream_t s) {
+  if (tc_bn_gu(Rtc) == 128)
+    tc_gu_kernel<128><<<tc_grid(tc_tiles(Rtc, 128, F, 1), n_sm), tc::kPThreads, tc::PLayout<128, true, false>::kSmemBytes, s>>>(
+        g, act_t, Rtc, nrows);
+  else
+    tc_gu_kernel<64><<<tc_grid(tc_tiles(Rtc, 64, F, 1), n_sm), tc::kPThreads, tc::PLayout<64, true, false>::kSmemBytes, s>>>(
+        g, act_t, Rtc, nrows);
+}
 
 }  // namespace
 }  // namespace mcd
