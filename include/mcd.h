@@ -91,7 +91,10 @@ typedef struct {
                          * Up to 8 streams and 32 packed rows (streams x max(K + 1, 2)) a
                          * frame is one persistent-kernel launch; beyond that calls run on
                          * the batched GEMM path (bf16 weights, <= 512 packed rows, one
-                         * CUDA graph launch per frame).  NOISY_TARGET and TREE need 1     */
+                         * CUDA graph launch per frame), which also takes launches of 5 or
+                         * more streams when the shapes allow its tensor-core products
+                         * (bf16; q / kv / ffn widths multiples of 128).  NOISY_TARGET and
+                         * TREE need 1                                                     */
 } mcd_config;
 
 /* Per-frame counters written by the device (device memory, caller-owned). */

@@ -544,7 +544,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   rope_kernel<<<8, 256, 0, c->stream>>>(rope, p.D, (double)k.rope_base, kMaxPos);
   if (cudaGetLastError() != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
-  if (k.max_streams > kMaxStreams || batch_rows(p, k.max_streams) > kMaxCols) {
+  if (k.max_streams > kMaxStreams || batch_rows(p, k.max_streams) > kMaxCols || batch_prefers(p, k.max_streams)) {
     mcd_status bs = batch_create(p, k.max_streams, &c->batch);
     if (bs != MCD_OK) return fail(bs);
   }
@@ -713,7 +713,8 @@ mcd_status mcd_decode_frames(mcd_ctx* c, int32_t n_streams, const uint32_t* stre
                              mcd_frame_stats* stats) {
   if (!c || !codes_out) return MCD_ERR_INVALID_ARG;
   if (!c->weights_loaded) return MCD_ERR_STATE;
-  if (n_streams > kMaxStreams || batch_rows(c->fp, n_streams) > kMaxCols) {
+  if (n_streams > kMaxStreams || batch_rows(c->fp, n_streams) > kMaxCols ||
+      (c->batch && batch_prefers(c->fp, n_streams))) {
     // many streams: the batched GEMM path (one CUDA graph launch per frame)
     const FrameParams& p = c->fp;
     if (!c->batch || n_streams > c->cfg.max_streams) return MCD_ERR_INVALID_ARG;

@@ -62,6 +62,9 @@ mcd_status cuda_status(cudaError_t e);
 // Batched decoding of many streams (GEMM path, mcd_batch.cu).
 struct BatchState;
 int batch_rows(const FrameParams& p, int max_streams);
+constexpr int kBatchMinStreams = 5;
+// Launches of this many streams go to the batched path even when the frame kernel fits them.
+bool batch_prefers(const FrameParams& p, int n_streams);
 mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out);
 // The batched path's copies of layer l's weights for its tensor-core GEMMs (no-op without).
 mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t st, const LayerSrc& src, int l);
