@@ -10,13 +10,15 @@
 //
 // captured once per context as a CUDA graph holding n_pos call bodies (a call never emits
 // fewer than one code, so n_pos calls always finish a frame; bodies after the last active
-// call find no rows and return at once).  RMSNorm never gets its own pass: the kernels that
-// write the residual stream also accumulate each row's sum of squares, and the next GEMM
-// scales its operand rows by gain / rms while staging them.  The GEMMs take the weights in
-// the same tiled unit layout as the frame kernel (each 16 x 16 tile in mma.m16n8k16
-// A-fragment order), stream them with cp.async through a 4-stage shared-memory pipeline and
-// multiply 128 weight rows x 64 packed rows per CTA with mma.sync (bf16 operands, fp32
-// accumulation).  Sampling and acceptance use the same integer sampler as the frame kernel.
+// call find no rows and return at once).  RMSNorm never gets its own pass.  With bf16
+// weights whose widths are multiples of 128 (the MultiCodeDecoder's) every product runs on
+// the tcgen05 GEMM (mcd_tcgemm.cuh, block kernels in mcd_tcops.cuh): weights and operand
+// rows as 128-byte swizzled tiles, TMEM accumulators, the residual products split over k
+// into partial sums that one per-row pass folds into the residual stream while it writes
+// the next product's normalised operand.  Other shapes use the mma.sync GEMM below (the
+// weights in the frame kernel's tiled unit layout, 128 weight rows x 64 packed rows per CTA
+// through a 4-stage cp.async pipeline, the norm folded into the operand staging).  Sampling
+// and acceptance use the same integer sampler as the frame kernel.
 #include <algorithm>
 #include <cstring>
 #include <vector>

@@ -9,14 +9,15 @@
 // is exactly the canonical K-major layout with 128-byte swizzle that tcgen05.mma reads
 // (8-row groups 1024 bytes apart).  No tensor map is needed.
 //
-// One CTA computes a 128 x BN tile of D (UMMA M = 128, N = BN, K = 16 per instruction): a
-// producer thread streams the k-slices of A and B through a ring of as many stages as fit in
-// 200 KB (4 to 6; mbarrier
-// complete_tx), one thread issues the MMAs and returns each stage with tcgen05.commit, and
-// after the last commit the four warps read the accumulator back from TMEM (warp w owns
-// lanes 32w..32w+31 = rows m of the tile) and hand every value to the epilogue functor.
-// Every wait is bounded (p.wait_ns); on a timeout the CTA records MCD_ERR_TIMEOUT, lets the
-// copies and MMAs it started finish, frees its TMEM and returns.
+// gemm_tile: one CTA computes a 128 x BN tile of D (UMMA M = 128, N = BN, K = 16 per
+// instruction): a producer thread streams the k-slices of A and B through a ring of as many
+// stages as fit in 200 KB (4 to 6; mbarrier complete_tx), one thread issues the MMAs and
+// returns each stage with tcgen05.commit, and after the last commit the four warps read the
+// accumulator back from TMEM (warp w owns lanes 32w..32w+31 = rows m of the tile) and hand
+// every value to the epilogue functor.  gemm_persistent (below) runs the same pipeline over
+// many tiles per CTA with two TMEM accumulators, so one tile's epilogue overlaps the next
+// tile's MMAs.  Every wait is bounded (wait_ns); on a timeout the CTA records
+// MCD_ERR_TIMEOUT, lets the copies and MMAs it started finish, frees its TMEM and returns.
 #pragma once
 #include "mcd_internal.cuh"
 
