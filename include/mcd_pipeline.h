@@ -75,8 +75,9 @@ mcd_status mcd_outer_load_weights(mcd_outer* o, int32_t n, const char* const* na
                                   const int64_t* nbytes);
 
 /* Start an utterance of stream `stream_id`: reset the KV cache and run the prompt rows
- * text_ids[0..n_tokens) (device int32) at positions 0..n_tokens-1, up to 16 rows per
- * launch; the last row gives frame 0's c0 and inner inputs (c0_out, device int32,
+ * text_ids[0..n_tokens) (device int32) at positions 0..n_tokens-1 (bf16 shapes that the
+ * tensor-core block products take: all rows but the last as one batch; otherwise up to 16
+ * rows per launch); the last row gives frame 0's c0 and inner inputs (c0_out, device int32,
  * optional, also receives c0).  Errors: MCD_ERR_INVALID_ARG, MCD_ERR_STATE (weights not
  * loaded), MCD_ERR_UNSUPPORTED (n_tokens > max_tokens); an id outside the text table is
  * reported by mcd_outer_sync as MCD_ERR_INVALID_ARG. */

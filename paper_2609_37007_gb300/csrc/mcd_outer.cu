@@ -5,7 +5,10 @@
 // / temperature sampling, Philox counter of position 0), and its post-norm hidden state plus
 // the c0 embedding start the MultiCodeDecoder's frame, which emits c1..c15.  The next
 // frame's CodeDecoder input is the sum of the text row (if any) and the embeddings of the 16
-// codes just emitted.  Before frame 0 the text prompt is prefilled, up to 16 rows per launch.
+// codes just emitted.  Before frame 0 the text prompt is prefilled: with the shapes the
+// tcgen05 block kernels take, all rows but the last as one batch on the tensor cores
+// (outer_tc_prefill), else up to 16 rows per outer_kernel launch; the last row always runs
+// through outer_kernel, which samples frame 0's c0.
 //
 // outer_kernel is one cooperative launch of one CTA per SM, built on the same weight ring
 // and unit GEMMs as the frame kernel (mcd_stage.cuh): per layer QKV -> attention -> Wo ->
