@@ -715,7 +715,8 @@ def main():
         t_e = time.perf_counter() - t0
         assert (st_p[:, 1] == cfg.n_pos).all() and (st_p[:, 4] == 0).all(), "device-side failure (e2e)"
         e2e = {"value": float(n_e * cfg.n_pos / t_e), "unit": UNIT,
-               "h2d_bytes_per_step": cfg.hidden * 4 + 4, "d2h_bytes_per_step": cfg.n_pos * 4 + 32,
+               # the library's two transfers: cond + c0 slot in; codes, stats, error word out
+               "h2d_bytes_per_step": cfg.hidden * 4 + 16, "d2h_bytes_per_step": 112,
                "frames": n_e, "api": "mcd_decode_frame_host (synchronous per frame, host clock)"}
 
     if rank != 0:

@@ -177,11 +177,14 @@ mcd_status mcd_decode_frames(mcd_ctx* ctx, int32_t n_streams, const uint32_t* st
                              const float* c0_emb, int32_t* codes_out, mcd_frame_stats* stats);
 
 /* mcd_decode_frame on host buffers: cond (host float [hidden]), c0 (host int32 [1]) or
- * c0_emb (host float [hidden]) are copied to the context's device staging area, the
- * frame is decoded, codes_out (host int32 [n_pos]) and stats (host, optional) are copied
- * back, and the call waits for the stream before returning (pinned host memory makes the
- * copies cheaper; pageable memory also works).  Returns the first device-side failure
- * like mcd_sync.  The per-frame entry point of a host-driven TTS loop. */
+ * c0_emb (host float [hidden]) are gathered into the context's pinned host mirror and
+ * copied to its device staging area in one transfer, the frame is decoded, and codes,
+ * stats and the device error word come back in one transfer; the call waits for the
+ * stream once, then fills codes_out (host int32 [n_pos]) and stats (host, optional).
+ * Bytes moved per frame: hidden*4 + 16 in (hidden*8 + 16 with c0_emb), 112 out.
+ * Any host memory works, pinned or pageable.  Returns the first device-side failure like
+ * mcd_sync (clearing it); codes_out and stats are then left unwritten.  The per-frame
+ * entry point of a host-driven TTS loop. */
 mcd_status mcd_decode_frame_host(mcd_ctx* ctx, uint32_t stream_id, uint32_t frame_idx,
                                  const float* cond, const int32_t* c0, const float* c0_emb,
                                  int32_t* codes_out, mcd_frame_stats* stats);

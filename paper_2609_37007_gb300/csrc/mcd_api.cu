@@ -237,7 +237,8 @@ struct mcd_ctx {
   size_t w_bytes = 0;
   size_t off_qkv = 0, off_wo = 0, off_gu = 0, off_wd = 0, off_head = 0, off_embed = 0;
   float* f32_arena = nullptr;   // norms + offsets
-  uint8_t* host_stage = nullptr;  // device staging for mcd_decode_frame_host
+  uint8_t* host_stage = nullptr;  // device staging for mcd_decode_frame_host (holds the err word)
+  uint8_t* host_pin = nullptr;    // pinned host mirror of host_stage
   bool weights_loaded = false;
   bool frame_begun = false;
   int h_err = 0;                 // host-side sticky CUDA error
@@ -396,13 +397,18 @@ const char* mcd_status_str(mcd_status s) {
   return "unknown status";
 }
 
-// Staging area of mcd_decode_frame_host: cond [H] | c0_emb [H] | c0 | codes [n_pos] | stats.
+// Staging area of mcd_decode_frame_host, mirrored in pinned host memory:
+//   cond [H] | c0 (16 B) | c0_emb [H] | codes [n_pos <= 15] (64 B) | stats (32 B) | err (16 B).
+// The inputs are one contiguous H2D range and the results plus the device error word one
+// contiguous D2H range, so a host-buffer frame costs two copies and one stream wait.
 static size_t stage_cond(const FrameParams&) { return 0; }
-static size_t stage_emb(const FrameParams& p) { return (size_t)p.H * 4; }
-static size_t stage_c0(const FrameParams& p) { return (size_t)p.H * 8; }
+static size_t stage_c0(const FrameParams& p) { return (size_t)p.H * 4; }
+static size_t stage_emb(const FrameParams& p) { return (size_t)p.H * 4 + 16; }
 static size_t stage_codes(const FrameParams& p) { return (size_t)p.H * 8 + 16; }
 static size_t stage_stats(const FrameParams& p) { return stage_codes(p) + 64; }
-static size_t host_stage_bytes(const FrameParams& p) { return stage_stats(p) + sizeof(mcd_frame_stats); }
+static size_t stage_err(const FrameParams& p) { return stage_stats(p) + 32; }
+static size_t host_stage_bytes(const FrameParams& p) { return stage_err(p) + 16; }
+static_assert(sizeof(mcd_frame_stats) <= 32, "stats slot of the staging area");
 
 mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if (!out) return MCD_ERR_INVALID_ARG;
@@ -523,7 +529,13 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.st, sizeof(DevState) * k.max_streams)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.ctr, sizeof(unsigned) * kMaxSlots * p.ctr_stride)) != cudaSuccess)
     return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.err, sizeof(int))) != cudaSuccess) return fail(cuda_status(e));
+  if ((e = ctx_alloc(c, &c->host_stage, host_stage_bytes(p))) != cudaSuccess) return fail(cuda_status(e));
+  p.err = reinterpret_cast<int*>(c->host_stage + stage_err(p));
+  if ((e = cudaHostAlloc(reinterpret_cast<void**>(&c->host_pin), host_stage_bytes(p), cudaHostAllocDefault)) !=
+      cudaSuccess) {
+    c->host_pin = nullptr;
+    return fail(cuda_status(e));
+  }
   if ((e = ctx_alloc(c, &p.tree_cand, sizeof(int) * kMaxDraft * kMaxTreeRank)) != cudaSuccess)
     return fail(cuda_status(e));
   if (k.draft_mode == MCD_DRAFT_TREE) {       // until mcd_set_tree: the chain of K rank-0 nodes
@@ -536,7 +548,6 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
       p.tree_m[i] = 1;
     }
   }
-  if ((e = ctx_alloc(c, &c->host_stage, host_stage_bytes(p))) != cudaSuccess) return fail(cuda_status(e));
   if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.kcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
   if (cudaMemsetAsync(p.vcache, 0, kvsz, c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -557,6 +568,7 @@ void mcd_destroy(mcd_ctx* c) {
   cudaStreamSynchronize(c->stream);
   batch_destroy(c->batch);
   for (void* q : c->allocs) cudaFree(q);
+  if (c->host_pin) cudaFreeHost(c->host_pin);
   delete c;
 }
 
@@ -751,22 +763,39 @@ mcd_status mcd_decode_frame_host(mcd_ctx* c, uint32_t stream_id, uint32_t frame_
   if (p.C0V > 0 && !c0) return MCD_ERR_INVALID_ARG;
   if (p.C0V == 0 && !c0_emb) return MCD_ERR_INVALID_ARG;
   uint8_t* st = c->host_stage;
+  uint8_t* hp = c->host_pin;
+  std::memcpy(hp + stage_cond(p), cond, (size_t)p.H * 4);
+  size_t in_bytes;
+  if (p.C0V > 0) {
+    std::memcpy(hp + stage_c0(p), c0, 4);
+    in_bytes = stage_emb(p);
+  } else {
+    std::memcpy(hp + stage_emb(p), c0_emb, (size_t)p.H * 4);
+    in_bytes = stage_codes(p);
+  }
+  MCD_CHECK(cudaMemcpyAsync(st, hp, in_bytes, cudaMemcpyHostToDevice, c->stream));
   float* d_cond = reinterpret_cast<float*>(st + stage_cond(p));
   float* d_emb = reinterpret_cast<float*>(st + stage_emb(p));
   int32_t* d_c0 = reinterpret_cast<int32_t*>(st + stage_c0(p));
   int32_t* d_codes = reinterpret_cast<int32_t*>(st + stage_codes(p));
   mcd_frame_stats* d_stats = reinterpret_cast<mcd_frame_stats*>(st + stage_stats(p));
-  MCD_CHECK(cudaMemcpyAsync(d_cond, cond, (size_t)p.H * 4, cudaMemcpyHostToDevice, c->stream));
-  if (p.C0V > 0)
-    MCD_CHECK(cudaMemcpyAsync(d_c0, c0, 4, cudaMemcpyHostToDevice, c->stream));
-  else
-    MCD_CHECK(cudaMemcpyAsync(d_emb, c0_emb, (size_t)p.H * 4, cudaMemcpyHostToDevice, c->stream));
   mcd_status s = mcd_decode_frame(c, stream_id, frame_idx, d_cond, p.C0V > 0 ? d_c0 : nullptr,
                                   p.C0V > 0 ? nullptr : d_emb, d_codes, d_stats);
   if (s != MCD_OK) return s;
-  MCD_CHECK(cudaMemcpyAsync(codes_out, d_codes, (size_t)p.P * 4, cudaMemcpyDeviceToHost, c->stream));
-  if (stats) MCD_CHECK(cudaMemcpyAsync(stats, d_stats, sizeof(mcd_frame_stats), cudaMemcpyDeviceToHost, c->stream));
-  return mcd_sync(c);
+  // codes | stats | err in one copy; the wait on the stream is the only synchronisation.
+  MCD_CHECK(cudaMemcpyAsync(hp + stage_codes(p), d_codes, host_stage_bytes(p) - stage_codes(p),
+                            cudaMemcpyDeviceToHost, c->stream));
+  MCD_CHECK(cudaStreamSynchronize(c->stream));
+  int err;
+  std::memcpy(&err, hp + stage_err(p), sizeof(int));
+  if (err != 0) {
+    MCD_CHECK(cudaMemsetAsync(c->fp.err, 0, sizeof(int), c->stream));
+    MCD_CHECK(cudaStreamSynchronize(c->stream));
+    return (mcd_status)err;
+  }
+  std::memcpy(codes_out, hp + stage_codes(p), (size_t)p.P * 4);
+  if (stats) std::memcpy(stats, hp + stage_stats(p), sizeof(mcd_frame_stats));
+  return MCD_OK;
 }
 
 mcd_status mcd_set_tree(mcd_ctx* c, int32_t n_nodes, const int32_t* parent, const int32_t* rank) {

@@ -595,6 +595,46 @@ def test_bad_c0_fails_the_frame_without_faulting(big):
     assert st[4] == 0 and st[1] == cfg.n_pos
 
 
+@pytest.mark.parametrize("env_name,pinned", [("tiny", False), ("tiny", True), ("big", True)])
+def test_host_buffer_api_matches_device_api(env_name, pinned, request):
+    """mcd_decode_frame_host (one gathered H2D copy, one D2H copy of codes, stats and the
+    error word) returns what mcd_decode_frame returns on device buffers; tiny feeds c0 as
+    an embedding, the full-size model as a token."""
+    env = request.getfixturevalue(env_name)
+    cfg = env.cfg
+    for f in range(4):
+        fr = make_frame(cfg, 300 + f)
+        ref_codes, ref_st, _ = env.decode(fr, 300 + f, stream_id=1)
+        cond = torch.from_numpy(np.ascontiguousarray(fr.cond, dtype=np.float32))
+        c0 = torch.tensor([fr.c0], dtype=torch.int32) if cfg.c0_vocab > 0 else None
+        emb = torch.from_numpy(np.ascontiguousarray(fr.c0_emb, dtype=np.float32)) if cfg.c0_vocab == 0 else None
+        codes = torch.full((cfg.n_pos,), -1, dtype=torch.int32)
+        st = torch.zeros(8, dtype=torch.int32)
+        if pinned:
+            cond, codes, st = cond.pin_memory(), codes.pin_memory(), st.pin_memory()
+            c0 = c0.pin_memory() if c0 is not None else None
+            emb = emb.pin_memory() if emb is not None else None
+        mcd.mcd_decode_frame_host(env.dec.ctx, 1, 300 + f, cond, c0, emb, codes, st)
+        assert codes.numpy().tolist() == ref_codes.tolist()
+        assert st.numpy().tolist() == ref_st.tolist()
+
+
+def test_host_buffer_api_reports_bad_c0_and_recovers(big):
+    cfg = big.cfg
+    fr = make_frame(cfg, 0)
+    cond = np.ascontiguousarray(fr.cond, dtype=np.float32)
+    codes = np.full(cfg.n_pos, -7, dtype=np.int32)
+    with pytest.raises(mcd.MCDError) as e:
+        mcd.mcd_decode_frame_host(big.dec.ctx, 0, 0, cond, np.array([cfg.c0_vocab + 5], dtype=np.int32), None, codes)
+    assert e.value.status == 1
+    assert (codes == -7).all()                     # results of a failed frame are not written
+    mcd.mcd_sync(big.dec.ctx)                      # the error was cleared by the failing call
+    st = np.zeros(8, dtype=np.int32)
+    mcd.mcd_decode_frame_host(big.dec.ctx, 0, 0, cond, np.array([fr.c0], dtype=np.int32), None, codes, st)
+    ref_codes, ref_st, _ = big.decode(fr, 0)
+    assert codes.tolist() == ref_codes.tolist() and st.tolist() == ref_st.tolist()
+
+
 # ---------------------------------------------------------------- distribution -----
 def test_chi_square_of_gpu_codes_against_exact_law(tiny):
     cfg = tiny.cfg
