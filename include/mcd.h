@@ -308,6 +308,18 @@ mcd_status mcd_set_timeline(mcd_ctx* ctx, uint64_t* timeline);
 /* Wait for the context's stream; returns the first device-side failure, if any. */
 mcd_status mcd_sync(mcd_ctx* ctx);
 
+/* Failure-detection hook: runs, in a one-CTA kernel on the context's stream, the bounded
+ * wait that every kernel of the library uses on something nothing will ever signal, and
+ * reports the outcome.  kind 0 waits on a device counter that is never incremented (the
+ * grid-level arrival counters' wait); kind 1 waits on a shared-memory mbarrier that never
+ * completes (the weight ring's wait).  The wait gives up after wait_ns (1 us .. 10 s),
+ * records MCD_ERR_TIMEOUT in the context like any device-side timeout, and the call waits
+ * for the stream and returns that status (clearing it, like mcd_sync), so MCD_ERR_TIMEOUT
+ * is the expected result; the context stays usable.  waited_ns (host, optional) receives
+ * the device-measured (%globaltimer) duration of the wait.  Errors: MCD_ERR_INVALID_ARG
+ * (kind or wait_ns out of range), MCD_ERR_STATE (a device-side failure was pending). */
+mcd_status mcd_test_bounded_wait(mcd_ctx* ctx, int32_t kind, uint64_t wait_ns, uint64_t* waited_ns);
+
 /* Bytes of weights one verify call streams for a call that reads `n_heads` LM heads
  * (backbone + heads), the algorithmic traffic used for roofline accounting. */
 int64_t mcd_call_weight_bytes(const mcd_ctx* ctx, int32_t n_heads);

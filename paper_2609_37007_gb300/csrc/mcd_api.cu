@@ -460,8 +460,10 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.trace_stride = (long long)sizeof(mcd_call_trace) * kMaxCalls + (long long)2 * kMaxCalls * kMaxRows * p.V * 4;
   if (k.draft_mode == MCD_DRAFT_TREE)   // + the tree records and every row's verify logits
     p.trace_stride += (long long)sizeof(mcd_tree_trace) * kMaxCalls + (long long)kMaxCalls * kMaxCols * p.V * 4;
+  // MCD_WAIT_NS overrides the bound, never below 100 ms: the same bound limits how long an
+  // aborting CTA waits for its copies and MMAs in flight, which must land before it exits.
   const char* wn = getenv("MCD_WAIT_NS");
-  if (wn) p.wait_ns = strtoull(wn, nullptr, 10);
+  if (wn) p.wait_ns = std::max(strtoull(wn, nullptr, 10), 100000000ull);
 
   const int es = k.weight_dtype == MCD_WEIGHT_F32 ? 4 : 2;     // embedding tables (bf16 for W8A16)
   const bool ok = backbone_geom(p, p.V);
@@ -907,6 +909,51 @@ mcd_status mcd_set_timeline(mcd_ctx* c, uint64_t* timeline) {
   if (!c) return MCD_ERR_INVALID_ARG;
   c->fp.timeline = reinterpret_cast<unsigned long long*>(timeline);
   return MCD_OK;
+}
+
+}  // extern "C"
+
+namespace {
+// One thread waits with the library's bounded waits on a counter nobody increments (kind 0)
+// or an mbarrier nobody arrives on (kind 1); the elapsed %globaltimer time goes to waited.
+__global__ void bounded_wait_test_kernel(const unsigned* never, int* err, unsigned long long wait_ns, int kind,
+                                         unsigned long long* waited) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  const uint64_t t0 = globaltimer();
+  bool ok;
+  if (kind == 0)
+    ok = wait_counter(never, 1u, err, wait_ns);
+  else
+    ok = wait_mbar(&bar, 0u, err, wait_ns, nullptr);
+  *waited = globaltimer() - t0;
+  if (ok) atomicCAS(err, 0, (int)MCD_ERR_STATE);     // cannot happen: nothing signals
+}
+}  // namespace
+
+extern "C" {
+
+mcd_status mcd_test_bounded_wait(mcd_ctx* c, int32_t kind, uint64_t wait_ns, uint64_t* waited_ns) {
+  if (!c || (kind != 0 && kind != 1) || wait_ns < 1000ull || wait_ns > 10000000000ull) return MCD_ERR_INVALID_ARG;
+  const FrameParams& p = c->fp;
+  int pending = 0;
+  MCD_CHECK(cudaStreamSynchronize(c->stream));
+  MCD_CHECK(cudaMemcpy(&pending, p.err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (pending != 0) return MCD_ERR_STATE;
+  // the 16-byte error slot of the staging area: err | never-set counter | waited (ns)
+  uint8_t* slot = c->host_stage + stage_err(p);
+  unsigned* never = reinterpret_cast<unsigned*>(slot + 4);
+  unsigned long long* waited = reinterpret_cast<unsigned long long*>(slot + 8);
+  MCD_CHECK(cudaMemsetAsync(slot + 4, 0, 12, c->stream));
+  bounded_wait_test_kernel<<<1, 32, 0, c->stream>>>(never, p.err, (unsigned long long)wait_ns, kind, waited);
+  MCD_CHECK(cudaGetLastError());
+  MCD_CHECK(cudaStreamSynchronize(c->stream));
+  unsigned long long w = 0;
+  MCD_CHECK(cudaMemcpy(&w, waited, sizeof(w), cudaMemcpyDeviceToHost));
+  if (waited_ns) *waited_ns = w;
+  return mcd_sync(c);
 }
 
 mcd_status mcd_sync(mcd_ctx* c) {

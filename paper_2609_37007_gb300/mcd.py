@@ -9,7 +9,7 @@ from __future__ import annotations
 
 import ctypes
 import os
-from typing import Dict, Optional
+from typing import Dict, Optional, Tuple
 
 import numpy as np
 
@@ -98,6 +98,7 @@ def load_library() -> ctypes.CDLL:
         "mcd_set_trace": (I32, [P, P]),
         "mcd_set_timeline": (I32, [P, P]),
         "mcd_sync": (I32, [P]),
+        "mcd_test_bounded_wait": (I32, [P, I32, ctypes.c_uint64, P]),
         "mcd_call_weight_bytes": (I64, [P, I32]),
         "mcd_num_ctas": (I32, [P]),
         "mcd_destroy": (None, [P]),
@@ -252,6 +253,14 @@ def mcd_set_timeline(ctx, timeline):
 
 def mcd_sync(ctx):
     _check("mcd_sync", load_library().mcd_sync(ctx))
+
+
+def mcd_test_bounded_wait(ctx, kind: int, wait_ns: int) -> Tuple[int, int]:
+    """(status, device-measured wait in ns) of one bounded wait on something nothing
+    signals; MCD_ERR_TIMEOUT is the expected status."""
+    waited = ctypes.c_uint64(0)
+    st = int(load_library().mcd_test_bounded_wait(ctx, kind, wait_ns, ctypes.addressof(waited)))
+    return st, int(waited.value)
 
 
 def mcd_call_weight_bytes(ctx, n_heads: int) -> int:

@@ -635,6 +635,25 @@ def test_host_buffer_api_reports_bad_c0_and_recovers(big):
     assert codes.tolist() == ref_codes.tolist() and st.tolist() == ref_st.tolist()
 
 
+@pytest.mark.parametrize("kind", [0, 1])
+def test_bounded_wait_times_out_and_the_context_stays_usable(big, kind):
+    """Failure detection without a fault: the library's bounded wait, run on a counter
+    (kind 0) or an mbarrier (kind 1) that nothing signals, gives up after its limit,
+    reports MCD_ERR_TIMEOUT through the status word, and the context decodes the next
+    frame exactly as before."""
+    cfg = big.cfg
+    fr = make_frame(cfg, 11)
+    ref_codes, ref_st, _ = big.decode(fr, 11)
+    status, waited = mcd.mcd_test_bounded_wait(big.dec.ctx, kind, 2_000_000)
+    assert status == 5, mcd.mcd_status_str(status)                 # MCD_ERR_TIMEOUT
+    assert 2_000_000 <= waited < 1_000_000_000, waited
+    mcd.mcd_sync(big.dec.ctx)                                       # cleared by the call
+    codes, st, _ = big.decode(fr, 11)
+    assert codes.tolist() == ref_codes.tolist() and st.tolist() == ref_st.tolist()
+    with pytest.raises(mcd.MCDError):
+        mcd._check("mcd_test_bounded_wait", mcd.load_library().mcd_test_bounded_wait(big.dec.ctx, 2, 2_000_000, None))
+
+
 # ---------------------------------------------------------------- distribution -----
 def test_chi_square_of_gpu_codes_against_exact_law(tiny):
     cfg = tiny.cfg
