@@ -60,7 +60,14 @@ def test_chain_tree_equals_greedy_chain(K):
 SMALL = Tree(parent=[-1, -1, 0, 1], rank=[0, 1, 0, 0])
 
 
-@pytest.mark.parametrize("tree", [SMALL, Tree(parent=[-1, -1, -1, 0], rank=[0, 1, 2, 0]), Tree.chain(2)])
+# the sizes of the paper's tree sweep (Fig. 4: N = 32 deployed, N = 64 the largest), grown
+# greedily for rank-decreasing statistics: 8 candidates at depth 1, the rest at depth 2
+_ACC = [[0.6 / (r + 1) ** 0.5 for r in range(8)] for _ in range(2)]
+
+
+@pytest.mark.parametrize("tree", [SMALL, Tree(parent=[-1, -1, -1, 0], rank=[0, 1, 2, 0]), Tree.chain(2),
+                                  grow_tree(_ACC, 32), grow_tree(_ACC, 64)],
+                         ids=["small", "wide3", "chain2", "grown32", "grown64"])
 def test_tree_law_equals_autoregressive_law(tree):
     cfg = TINY
     m = Model(cfg, weights_as_f32(cfg, make_weights(cfg)))
