@@ -7,7 +7,7 @@ input is the sum of the frame's text-token embedding and the embeddings of all 1
 of the frame before.  The CodeDecoder has 28 layers; its block is not described, so it
 is the MultiCodeDecoder's block (readings R-M1..R-M6 of oracle.model).
 
-Readings of what the paper leaves open (design notes R-C1..R-C7):
+Readings of what the paper leaves open (R-C1..R-C7):
   R-C1 positions are absolute over the utterance: the text prompt fills positions
        0..T-1 (one prefill), frame i >= 1 feeds one row at position T - 1 + i.
   R-C2 frame 0's c0 and MultiCodeDecoder input come from the last prompt row; after the

@@ -15,7 +15,7 @@ speculative procedure (Sec. 2.2, Fig. 3) runs one call per round:
   * the first call feeds the conditioning vector (position 0) and c0 (position 1) and
     emits c1 from LM head 1, which is exact autoregressive decoding (Fig. 3 caption).
 
-Readings (design notes R-F1..R-F4):
+Readings of what the paper leaves open (R-F1..R-F4):
   R-F1 rows per verify call = min(n_drafts + 1, P - a): no row is fed for a bonus past c_P.
   R-F2 round r uses counters (round r, position s, purpose); see oracle.philox.
   R-F3 NOISY_TARGET drafts (controlled-acceptance workload): q for position s is the

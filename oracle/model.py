@@ -4,7 +4,7 @@ What the paper fixes (Sec. 1, Fig. 1; Sec. 2.1): the MultiCodeDecoder is a 5-lay
 transformer run inside each 80 ms frame; code c_i is looked up in its own embedding
 table i and the hidden state read by LM head i emits c_i; it restarts every frame from
 the outer model's output.  The block internals are not in the paper; they follow the
-Qwen3 decoder layer that Qwen3-TTS uses (readings R-M1..R-M6 of the design notes):
+Qwen3 decoder layer that Qwen3-TTS uses (readings R-M1..R-M6, stated here):
 
   R-M1 pre-norm block without biases:
          x += Wo * Attn(RoPE(QKnorm(Wq n(x), Wk n(x))), Wv n(x))

@@ -1,7 +1,7 @@
 """W8A16 weights (Sec. 3.3: the deployed model streams 8-bit weights with 16-bit
 activations).  TEST INFRASTRUCTURE ONLY.
 
-The paper does not give its quantiser; the reading taken here (design note R-Q1):
+The paper does not give its quantiser; the reading taken here (R-Q1):
   R-Q1 every matrix the decoder streams (Wq, Wk, Wv, Wo, Wg, Wu, Wd of every layer and
        every LM head) is quantised per output row, symmetrically: with w the row's values
        as fp32 (the bf16 model's values, exact in fp32), m = max |w|,

@@ -5,7 +5,7 @@ sampling configuration") and verifies drafts with the standard speculative accep
 rule with residual resampling (Sec. 2.2 "Tree attention ..."; Sec. 3.2): a draft d drawn
 from q is kept with probability min(1, p(d)/q(d)); otherwise a replacement is drawn from
 max(0, p - q) renormalised.  The paper fixes no arithmetic for this, so this module fixes
-it (readings R-S1..R-S7 of the design notes).  Every distribution is a list of integer
+it (readings R-S1..R-S7, stated here).  Every distribution is a list of integer
 weights, so that each decision is an exact rational comparison:
 
   R-S1 top-k set: sort by (fp32 logit descending, id ascending), keep the first k;

@@ -11,7 +11,7 @@ a subset of the paths and is grown greedily from per-depth, per-rank acceptance
 statistics, each step adding the node with the largest expected contribution to the
 accepted length, until the node budget N is reached (depth at most K).
 
-Readings of what the paper leaves open (design notes R-T1..R-T6):
+Readings of what the paper leaves open (R-T1..R-T6):
   R-T1 a tree is a list of nodes in breadth-first order; node i has a parent (-1: a child
        of the call's first row) and a rank; depth = parent's depth + 1 <= K; siblings have
        distinct ranks.
