@@ -594,7 +594,7 @@ __global__ void __launch_bounds__(256) batch_rowss_kernel(const float* X, int H,
 // ------------------------------------------------------------------------------------
 // attention: one CTA per (stream, KV head)
 // ------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBufs b, int layer) {
+__global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, BatchBufs b, int layer) {
   const int s = blockIdx.x, g = blockIdx.y;
   if (s >= b.frame->S) return;
   const int base = b.sbase[s];
@@ -614,7 +614,7 @@ __global__ void __launch_bounds__(256) batch_attn_kernel(FrameParams p, BatchBuf
   // a batch of up to 6 per thread in flight before the stores
   {
     const int n_q = nq * D4, n_kv = nk * D4, total = n_q + 2 * n_kv;
-    constexpr int kL = 6;
+    constexpr int kL = 3;
     for (int b0 = 0; b0 < total; b0 += kL * 256) {
       float4 v[kL];
       float4* dst[kL];
