@@ -592,7 +592,8 @@ __global__ void __launch_bounds__(256) batch_rowss_kernel(const float* X, int H,
 }
 
 // ------------------------------------------------------------------------------------
-// attention: one CTA per (stream, KV head)
+// attention: one CTA per (stream, KV head).  At most 32 registers per thread, so that seven
+// CTAs share an SM and the 1024 CTAs of 128 streams run as one wave.
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, BatchBufs b, int layer) {
   const int s = blockIdx.x, g = blockIdx.y;
@@ -611,7 +612,7 @@ __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, Batch
   const int nk = pos0 + nr;
   const int D4 = D >> 2;
   // loads: queries, then keys and values (cached rows, then the new rows), as 16-byte chunks,
-  // a batch of up to 6 per thread in flight before the stores
+  // a batch of up to 3 per thread in flight before the stores
   {
     const int n_q = nq * D4, n_kv = nk * D4, total = n_q + 2 * n_kv;
     constexpr int kL = 3;
