@@ -41,6 +41,12 @@ def test_every_declared_symbol_is_exported(lib):
     assert not missing, missing
 
 
+def test_every_declared_symbol_has_a_binding_of_the_same_name():
+    from paper_2609_37007_gb300 import mcd
+    missing = [f for f in declared_functions() if not callable(getattr(mcd, f, None))]
+    assert not missing, missing
+
+
 def test_struct_layouts_match_the_binding(tmp_path):
     from paper_2609_37007_gb300 import mcd
     src = tmp_path / "sz.c"
