@@ -52,7 +52,7 @@ __device__ __forceinline__ unsigned call_heads_mask(const FrameParams& p) {
 // ------------------------------------------------------------------------------------
 // Producer: one thread streams this CTA's units into the ring.
 // ------------------------------------------------------------------------------------
-__device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
+__device__ __forceinline__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
   const int cta = blockIdx.x, n_cta = p.n_cta;
   const uint64_t pol = policy_evict_first();
   uint32_t issued = 0;
@@ -111,15 +111,16 @@ __device__ void producer_loop(const FrameParams& p, Smem& sm, int call0) {
 // writer, stores the new k / v rows to the cache; (C1) two threads per (row, key) score it
 // over interleaved 16-byte chunks (rows padded to D + 8 floats: conflict-free reads); (C2)
 // one warp per row takes the softmax; (C3) one thread per (row, dim pair) sums P.V.
-__device__ void attention_stream(Cons& c, int layer, int h, bool write_kv, int nr, int pos0, int base, int s) {
-  const FrameParams& p = c.p;
+__device__ __noinline__ void attention_stream(const FrameParams& p, int layer, int h, bool write_kv, int nr, int pos0, int base,
+                                             int s) {
+  Smem sm = smem_layout(mcd_dyn_smem);
   const int D = p.D, half = D >> 1, g = h / (p.NH / p.NKV);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cs_shift = D == 128 ? 5 : 4;           // 16-byte chunks per row = D / 4
   const int cpr = 1 << cs_shift;
   const int KS = D + 8;                            // padded row stride (floats) of q and k rows
   constexpr int kAttnPos = 16;                     // sequence positions 0..15 (c15 is never fed)
-  float* o = c.sm.act;                             // [kMaxCols][D]: every stream's packed rows
+  float* o = sm.act;                             // [kMaxCols][D]: every stream's packed rows
   float* qs = o + kMaxCols * 128;                  // [8][KS]
   float* ks = qs + kMaxRows * 136;                 // [kAttnPos][KS]
   float* vs = ks + kAttnPos * 136;                 // [kAttnPos][D]
@@ -290,13 +291,168 @@ __device__ void attention_stream(Cons& c, int layer, int h, bool write_kv, int n
 }
 
 
+// Attention of query head h for the nr rows of stream s (packed rows base..base+nr-1), the
+// single-stream form; same outputs and cache writes as attention_stream (o[base + n][D] in
+// act).  (A) all threads stage the stream's cached K / V rows, the new rows' raw q / k / v,
+// their RoPE rows and the QK-norm gains in shared memory (independent 16-byte loads, all in
+// flight together); (B) one warp per new q / k vector applies QK-norm and RoPE in registers
+// (lane l holds dims l + 32 i, so each rotate-half pair sits in one lane) and the KV writer
+// stores the new keys and values; (C) the warp of query row n scores its keys with two lanes
+// per key (interleaved 16-byte chunks, one shuffle), takes the softmax across its lanes and
+// sums P.V with four dims per lane.  Three barriers in all; keys: positions 0..15 (c15 is
+// never fed).
+constexpr int kAttnKeys = 16;
+__device__ __noinline__ void attention_rows(const FrameParams& p, int layer, int h, bool write_kv, int nr, int pos0, int base,
+                                           int s) {
+  Smem sm = smem_layout(mcd_dyn_smem);
+  const int D = p.D, half = D >> 1, g = h / (p.NH / p.NKV);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int cs_shift = D == 128 ? 5 : 4, cpr = 1 << cs_shift;   // 16-byte chunks per row
+  constexpr int KS = 136;                                       // padded q / k row stride
+  float* o = sm.act;                                          // [kMaxCols][D]
+  float* ks = o + kMaxCols * 128;                               // [kAttnKeys][KS]
+  float* vs = ks + kAttnKeys * KS;                              // [kAttnKeys][128]
+  float* qs = vs + kAttnKeys * 128;                             // [kMaxRows][KS]
+  float2* cs = reinterpret_cast<float2*>(qs + kMaxRows * KS);   // [kMaxRows][D/2]
+  float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);     // [D]
+  float* gk = gq + 128;                                         // [D]
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  const float* qkv = p.qkv;
+  const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
+  if (pos0 + nr > kAttnKeys) {                // positions beyond c14's row are never fed
+    if (tid == 0) atomicCAS(p.err, 0, (int)MCD_ERR_STATE);
+    nr = max(0, kAttnKeys - pos0);
+  }
+  // ---- (A) staging: rows [cached K | cached V | q | k | v | RoPE | gains], 16-byte chunks --
+  {
+    const int n_rows = 2 * pos0 + 4 * nr + (p.qk_norm ? 2 : 0);
+    for (int i = tid; i < (n_rows << cs_shift); i += kConsumerThreads) {
+      int r = i >> cs_shift;
+      const int ch = i & (cpr - 1);
+      const float* src;
+      float* dst;
+      if (r < 2 * pos0) {
+        const bool isv = r >= pos0;
+        const int j = isv ? r - pos0 : r;
+        src = (isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D;
+        dst = isv ? vs + j * 128 : ks + j * KS;
+      } else if ((r -= 2 * pos0) < 3 * nr) {
+        const int seg = r >= 2 * nr ? 2 : r >= nr ? 1 : 0, m = r - seg * nr;
+        src = qkv + (size_t)(base + m) * p.qkv_dim + (seg == 0 ? qoff : seg == 1 ? koff : voff);
+        dst = seg == 0 ? qs + m * KS : seg == 1 ? ks + (pos0 + m) * KS : vs + (pos0 + m) * 128;
+      } else if ((r -= 3 * nr) < nr) {
+        src = reinterpret_cast<const float*>(p.rope + (size_t)(pos0 + r) * half);
+        dst = reinterpret_cast<float*>(cs + r * 64);
+      } else {
+        r -= nr;
+        src = (r == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D;
+        dst = r == 0 ? gq : gk;
+      }
+      cpa16(dst + 4 * ch, src + 4 * ch);
+    }
+    cpa_wait_all();
+  }
+  consumer_sync();
+  // ---- (B) QK-norm + RoPE of the new q / k rows; the KV writer stores k / v -------------
+  const int nd = D >> 5;   // dims per lane: 4 (D = 128) or 2 (D = 64)
+  for (int vi = warp; vi < 2 * nr; vi += kConsumerWarps) {
+    const bool isq = vi < nr;
+    const int n = isq ? vi : vi - nr;
+    float* row = isq ? qs + n * KS : ks + (pos0 + n) * KS;
+    float x[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) x[i] = i < nd ? row[lane + 32 * i] : 0.f;
+    if (p.qk_norm) {
+      float ss = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ss += x[i] * x[i];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+      const float sc = rsqrtf(ss / (float)D + p.eps);
+      const float* gg = isq ? gq : gk;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) x[i] = x[i] * sc * gg[lane + 32 * i];
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if (i < nd / 2) {
+        const float2 r = cs[n * 64 + lane + 32 * i];
+        const float a = x[i], b = x[i + nd / 2];
+        x[i] = a * r.x - b * r.y;
+        x[i + nd / 2] = b * r.x + a * r.y;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (i < nd) row[lane + 32 * i] = x[i];
+    if (write_kv && !isq) {
+      float* kdst = p.kcache + cache_off + (size_t)(pos0 + n) * D;
+      float* vdst = p.vcache + cache_off + (size_t)(pos0 + n) * D;
+      const float* vrow = vs + (pos0 + n) * 128;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (i < nd) {
+          kdst[lane + 32 * i] = x[i];
+          vdst[lane + 32 * i] = vrow[lane + 32 * i];
+        }
+    }
+  }
+  consumer_sync();
+  // ---- (C) warp n: scores (lanes 2j, 2j+1 for key j), softmax, P.V -----------------------
+  if (warp < nr) {
+    const int n = warp, npos = pos0 + n + 1;
+    const int j = lane >> 1, hf = lane & 1;
+    const bool live = j < npos;                      // causal: keys 0..pos0+n
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    if (live) {
+      const float4* q4 = reinterpret_cast<const float4*>(qs + n * KS) + hf;
+      const float4* k4 = reinterpret_cast<const float4*>(ks + j * KS) + hf;
+#pragma unroll 4
+      for (int ch = 0; ch < (cpr >> 1); ++ch) {
+        const float4 q = q4[2 * ch], k = k4[2 * ch];
+        a0 += q.x * k.x;
+        a1 += q.y * k.y;
+        a2 += q.z * k.z;
+        a3 += q.w * k.w;
+      }
+    }
+    float sc = (a0 + a1) + (a2 + a3);
+    sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 1);
+    sc = live ? sc * rsqrtf((float)D) : -INFINITY;
+    float mx = sc;
+#pragma unroll
+    for (int off = 16; off > 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, off));
+    const float e = live ? __expf(sc - mx) : 0.f;
+    float sum = e;                                   // lanes of one parity hold every key once
+#pragma unroll
+    for (int off = 16; off > 1; off >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, off);
+    const float pj = e / sum;
+    const int d0 = 4 * lane;                         // four dims per lane
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int jj = 0; jj < npos; ++jj) {
+      const float w = __shfl_sync(0xFFFFFFFFu, pj, 2 * jj);
+      if (d0 < D) {
+        const float4 v = *reinterpret_cast<const float4*>(vs + jj * 128 + d0);
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
+    }
+    if (d0 < D) *reinterpret_cast<float4*>(o + (base + n) * D + d0) = acc;
+  }
+  consumer_sync();
+}
+
 // Attention of query head h for every stream with rows in the call (outputs at the
 // streams' packed rows).
 __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   const CallInfo* ci = c.sm.ci;
   for (int i = 0; i < ci->n_act; ++i) {
     const int s = ci->act[i];
-    attention_stream(c, layer, h, write_kv, ci->st[s].n_rows, ci->st[s].pos0, ci->base[s], s);
+    attention_rows(c.p, layer, h, write_kv, ci->st[s].n_rows, ci->st[s].pos0, ci->base[s], s);
   }
 }
 
@@ -308,16 +464,16 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
 // the acceptance step commits the kept ones.  Outputs go to p.attn.  Scratch (act + bfrag,
 // 62 KB): k [48][D + 8], v [48][D], q [8][D + 8], RoPE rows by depth [9][D/2], QK-norm
 // gains, scores [8][48].
-__device__ void attention_tree_task(Cons& c, int layer, int h, int lo, int hi, int pos0) {
-  const FrameParams& p = c.p;
-  const CallInfo* ci = c.sm.ci;
+__device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer, int h, int lo, int hi, int pos0) {
+  Smem sm = smem_layout(mcd_dyn_smem);
+  const CallInfo* ci = sm.ci;
   const int D = p.D, half = D >> 1, group = p.NH / p.NKV, g = h / group;
   const bool write_kv = (h % group) == 0;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cs_shift = D == 128 ? 5 : 4, cpr = 1 << cs_shift;   // 16-byte chunks per row
   const int KS = D + 8;
   constexpr int kKeys = 48, kDepths = 9;
-  float* ks = c.sm.act;
+  float* ks = sm.act;
   float* vs = ks + kKeys * 136;
   float* qs = vs + kKeys * 128;
   float2* cs = reinterpret_cast<float2*>(qs + 8 * 136);
@@ -484,7 +640,7 @@ __device__ void attention_tree_task(Cons& c, int layer, int h, int lo, int hi, i
 // One call
 // ------------------------------------------------------------------------------------
 template <int WT, bool WIDE>
-__device__ void run_call(Cons& c, int call) {
+__device__ __forceinline__ void run_call(Cons& c, int call) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
   const CallInfo* ci = sm.ci;
@@ -544,13 +700,13 @@ __device__ void run_call(Cons& c, int call) {
         // tree call (one stream): one task per (query head, group of 8 rows)
         const int nr = ci->M, n_rg = (nr + 7) >> 3;
         for (int t = blockIdx.x; t < p.NH * n_rg; t += p.n_cta)
-          attention_tree_task(c, l, t % p.NH, 8 * (t / p.NH), min(8 * (t / p.NH) + 8, nr), ci->st[0].pos0);
+          attention_tree_task(p, l, t % p.NH, 8 * (t / p.NH), min(8 * (t / p.NH) + 8, nr), ci->st[0].pos0);
       } else {
         const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
         for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
           const int i = t / p.NH, h = t - i * p.NH, s = ci->act[i];
           const int nr = ci->st[s].n_rows, base = ci->base[s];
-          attention_stream(c, l, h, (h % group) == 0, nr, ci->st[s].pos0, base, s);
+          attention_stream(p, l, h, (h % group) == 0, nr, ci->st[s].pos0, base, s);
           for (int q = threadIdx.x; q < nr * (D >> 2); q += kConsumerThreads) {
             const int n = q / (D >> 2), d4 = q - n * (D >> 2);
             reinterpret_cast<float4*>(p.attn + (size_t)(base + n) * p.NH * D + h * D)[d4] =
@@ -564,7 +720,7 @@ __device__ void run_call(Cons& c, int call) {
       const MatGeom& g = p.g[MAT_WO];
       if (threadIdx.x == 0) sm.flags[3] = -1;
       consumer_sync();
-      run_stage<WT, WIDE>(
+      run_stage<WT, WIDE, true>(
           c, call, sp_wo, D, wo_key,
           [&](int u, int, int) {
             const int h = u / g.n_mb;
@@ -575,15 +731,18 @@ __device__ void run_call(Cons& c, int call) {
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
-          [&](int u, int mi, int rr, int n, float v, float) {
-            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wo, (size_t)l * H + row));
+          [&](int u, int mi, int rr0, int n, float4 v) {
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr0;
+            const size_t si = (size_t)l * H + row;
+            red_add_f32x4(p.x + (size_t)n * H + row,
+                          make_float4(v.x * wscale<WT>(p.s_wo, si), v.y * wscale<WT>(p.s_wo, si + 1),
+                                      v.z * wscale<WT>(p.s_wo, si + 2), v.w * wscale<WT>(p.s_wo, si + 3)));
           });
       if (c.abort_) return;
     } else {
       const MatGeom& g = p.g[MAT_WO];
       const int group = p.NH / p.NKV;
-      run_stage<WT, WIDE>(
+      run_stage<WT, WIDE, true>(
           c, call, sp_wo, D, wo_key,
           [&](int u, int cnt, int step) {
             const int h = u / g.n_mb;
@@ -597,9 +756,12 @@ __device__ void run_call(Cons& c, int call) {
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
-          [&](int u, int mi, int rr, int n, float v, float) {
-            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wo, (size_t)l * H + row));
+          [&](int u, int mi, int rr0, int n, float4 v) {
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr0;
+            const size_t si = (size_t)l * H + row;
+            red_add_f32x4(p.x + (size_t)n * H + row,
+                          make_float4(v.x * wscale<WT>(p.s_wo, si), v.y * wscale<WT>(p.s_wo, si + 1),
+                                      v.z * wscale<WT>(p.s_wo, si + 2), v.w * wscale<WT>(p.s_wo, si + 3)));
           });
       if (c.abort_) return;
     }
@@ -636,7 +798,7 @@ __device__ void run_call(Cons& c, int call) {
     {
       const MatGeom& g = p.g[MAT_WD];
       const int Kc = g.Ku * 16;
-      run_stage<WT, WIDE>(
+      run_stage<WT, WIDE, true>(
           c, call, sp_wd, Kc, wd_key,
           [&](int u, int, int) {
             const int kc = u / g.n_mb;
@@ -647,9 +809,12 @@ __device__ void run_call(Cons& c, int call) {
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
           },
-          [&](int u, int mi, int rr, int n, float v, float) {
-            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr;
-            atomicAdd(p.x + (size_t)n * H + row, v * wscale<WT>(p.s_wd, (size_t)l * H + row));
+          [&](int u, int mi, int rr0, int n, float4 v) {
+            const int row = (u % g.n_mb) * g.Mu * 16 + mi * 16 + rr0;
+            const size_t si = (size_t)l * H + row;
+            red_add_f32x4(p.x + (size_t)n * H + row,
+                          make_float4(v.x * wscale<WT>(p.s_wd, si), v.y * wscale<WT>(p.s_wd, si + 1),
+                                      v.z * wscale<WT>(p.s_wd, si + 2), v.w * wscale<WT>(p.s_wd, si + 3)));
           });
       if (c.abort_) return;
     }
@@ -773,42 +938,29 @@ __device__ void run_call(Cons& c, int call) {
   if (*(volatile int*)&sm.flags[1]) c.abort_ = true;
 }
 
-// Copy distribution records into shared memory with independent word loads: the header,
-// ids[0..k) and W[0..k) of each (k = top_k; entries past a record's n are never read).
-// Threads t0 .. t0 + nt - 1 take part; each issues a batch of up to 8 loads before its
-// stores, so a copy costs about one memory round trip per batch.
+// Copy distribution records into shared memory: the header with ids[0..k) and W[0..k) of
+// each (k = top_k; entries past a record's n are never read) as 16-byte cp.async chunks, all
+// in flight together.  Threads t0 .. t0 + nt - 1 take part; a barrier must follow.
 template <class Src>
 __device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src, int t0 = 0,
                                               int nt = kConsumerThreads) {
-  constexpr int kIdsWord = offsetof(TopkRec, ids) / 4, kWWord = offsetof(TopkRec, W) / 4;
-  constexpr int kB = 8;
-  const int words = kIdsWord + 2 * k, total = nrec * words, me = (int)threadIdx.x - t0;
+  const int c_ids = (int)((offsetof(TopkRec, ids) + 4 * k + 15) / 16), c_w = (4 * k + 15) / 16;
+  const int per = c_ids + c_w, total = nrec * per, me = (int)threadIdx.x - t0;
   if (me < 0 || me >= nt) return;
-  for (int b = 0; b < total; b += kB * nt) {
-    int v[kB];
-    int* d[kB];
-#pragma unroll
-    for (int u = 0; u < kB; ++u) {
-      const int i = b + me + u * nt;
-      d[u] = nullptr;
-      if (i < total) {
-        const int r = i / words, w = i - r * words;
-        const int off = w < kIdsWord ? w : (w < kIdsWord + k ? w : kWWord + (w - kIdsWord - k));
-        v[u] = __ldcg(reinterpret_cast<const int*>(src(r)) + off);
-        d[u] = reinterpret_cast<int*>(dst + r) + off;
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kB; ++u)
-      if (d[u]) *d[u] = v[u];
+  for (int i = me; i < total; i += nt) {
+    const int r = i / per, ch = i - r * per;
+    const int off = ch < c_ids ? ch * 16 : (int)offsetof(TopkRec, W) + (ch - c_ids) * 16;
+    cpa16(reinterpret_cast<uint8_t*>(dst + r) + off, reinterpret_cast<const uint8_t*>(src(r)) + off);
   }
+  cpa_wait_all();
 }
+static_assert(sizeof(TopkRec) % 16 == 0 && offsetof(TopkRec, ids) % 16 == 0 && offsetof(TopkRec, W) % 16 == 0,
+              "records are copied in 16-byte chunks");
 
 // Acceptance step and next drafts (run by the CTA that finished top-k last).  Every record
 // it reads is first staged in shared memory (act + bfrag, 64 KB).
-__device__ void accept_step(Cons& c, int call, int s) {
-  const FrameParams& p = c.p;
-  Smem& sm = c.sm;
+__device__ __noinline__ void accept_step(const FrameParams& p, int call, int s) {
+  Smem sm = smem_layout(mcd_dyn_smem);
   const CallInfo* ci = sm.ci;
   const int a = ci->st[s].a, n_d = ci->st[s].n_d, pos0 = ci->st[s].pos0, n_rows = ci->st[s].n_rows;
   const int qrow = ci->st[s].q_row, round = ci->st[s].round, base = ci->base[s];
@@ -820,7 +972,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
   TopkRec* srec = reinterpret_cast<TopkRec*>(sm.act);            // staged records
   const int n_p = (a + 1 + n_d <= p.P) ? n_d + 1 : n_d;
   __shared__ int s_emit[kMaxRows], s_nemit, s_nacc, s_next[kMaxDraft], s_nnext;
-  if (s == 0) timeline(c, call, 4, true);
+  if (s == 0) timeline_p(p, sm.ci, 4, true);
   // p of positions a+1..: this call's verify records (packed rows base + ...); q of the
   // drafts: the previous call's records of its packed row qrow, or the noisy-target passes'
   const int n_pq = n_p + n_d;
@@ -834,7 +986,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
   const bool pre = !noisy && idle0 < kConsumerThreads &&
                    (size_t)(n_pq + n_rows * p.K) * sizeof(TopkRec) <= (size_t)(kActBytes + kBfragBytes);
   consumer_sync();
-  if (s == 0) timeline(c, call, 5, true);
+  if (s == 0) timeline_p(p, sm.ci, 5, true);
   // The acceptance rule of every draft in parallel, warp i for draft i (its accept test and
   // the residual draw it would take if it were the first rejection) and warp n_d for the
   // bonus draw; then the chain is read off in order: drafts kept up to the first rejection,
@@ -883,7 +1035,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
     s_nacc = na;
   }
   consumer_sync();
-  if (s == 0) timeline(c, call, 6, true);
+  if (s == 0) timeline_p(p, sm.ci, 6, true);
   const int a_new = a + s_nemit;
   const int m = a_new - pos0;
   const int n_next = min(p.K, p.P - a_new);
@@ -1000,7 +1152,7 @@ __device__ void accept_step(Cons& c, int call, int s) {
     }
   }
   consumer_sync();
-  if (s == 0) timeline(c, call, 7, true);
+  if (s == 0) timeline_p(p, sm.ci, 7, true);
   if (threadIdx.x == 0) {
     // the last acceptance of the call releases the next call
     __threadfence();
@@ -1020,9 +1172,8 @@ __device__ void accept_step(Cons& c, int call, int s) {
 // and the call ends.  Then: the next call's candidates (the top-m ids by logit of each
 // draft distribution of the last visited row), the kept nodes' K / V moved to their
 // positions, the state update, the trace and the release of the next call.
-__device__ void accept_tree(Cons& c, int call) {
-  const FrameParams& p = c.p;
-  Smem& sm = c.sm;
+__device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
+  Smem sm = smem_layout(mcd_dyn_smem);
   const CallInfo* ci = sm.ci;
   const DevState& st0 = ci->st[0];
   const int a = st0.a, pos0 = st0.pos0, n_rows = st0.n_rows, round = st0.round;
@@ -1246,9 +1397,8 @@ __device__ void accept_tree(Cons& c, int call) {
 // Draft step of noisy-target pass j (run by the CTA that finished top-k last): draw the
 // draft of position pos0 from the pass's noisy distribution with the draft-purpose uniform
 // of the verify round, then set up pass j+1 or, after the last pass, the verify call.
-__device__ void emu_step(Cons& c, int call) {
-  const FrameParams& p = c.p;
-  Smem& sm = c.sm;
+__device__ __noinline__ void emu_step(const FrameParams& p, int call) {
+  Smem sm = smem_layout(mcd_dyn_smem);
   const CallInfo* ci = sm.ci;
   const int j = ci->emu, n = ci->st[0].emu_n, round = ci->st[0].round, pos0 = ci->st[0].pos0, a = ci->st[0].a;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1289,7 +1439,7 @@ __device__ void emu_step(Cons& c, int call) {
 }
 
 template <bool WIDE>
-__device__ bool read_call_state(Cons& c, int call, bool first) {
+__device__ __forceinline__ bool read_call_state(Cons& c, int call, bool first) {
   const FrameParams& p = c.p;
   Smem& sm = c.sm;
   if (!first) {
@@ -1406,8 +1556,7 @@ __device__ bool read_call_state(Cons& c, int call, bool first) {
 
 template <int WT, bool WIDE>
 __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constant__ FrameParams p) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  Smem sm = smem_layout(smem_raw);
+  Smem sm = smem_layout(mcd_dyn_smem);
   const int tid = threadIdx.x, warp = tid >> 5;
   if (tid == 0) {
     for (int s = 0; s < kNumSlots; ++s) {
@@ -1435,11 +1584,11 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
       if (c.abort_) break;
       if (sm.flags[2]) {
         if (sm.ci->emu)
-          emu_step(c, call);
+          emu_step(p, call);
         else if (WIDE && p.draft_mode == MCD_DRAFT_TREE)
-          accept_tree(c, call);
+          accept_tree(p, call);
         else
-          accept_step(c, call, sm.flags[4]);
+          accept_step(p, call, sm.flags[4]);
       }
     }
     if (tid == 0) sm.flags[0] = 1;  // stop the producer

@@ -249,6 +249,18 @@ __device__ __forceinline__ uint32_t ld_acquire(const unsigned* p) {
 __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+// 16-byte global -> shared copy through L2 (cp.async.cg: other CTAs' writes are seen once
+// they are visible at GPU scope); cpa_wait_all waits for this thread's copies.
+__device__ __forceinline__ void cpa16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cpa_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+// fp32 add of four consecutive words (16-byte aligned) at GPU scope as one vector reduction:
+// a quarter of the L2 atomic operations of four scalar adds.
+__device__ __forceinline__ void red_add_f32x4(float* p, float4 v) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
 __device__ __forceinline__ uint64_t globaltimer() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -333,8 +345,9 @@ __host__ __device__ inline void philox_block(unsigned long long seed, uint32_t s
   out[3] = purpose;
   philox4x32_10(out, (uint32_t)(seed & 0xFFFFFFFFull), (uint32_t)(seed >> 32));
 }
-// The 53-bit integer uniform of a decision: u = U / 2^53 = res53(w0, w1).
-__host__ __device__ inline unsigned long long uniform_U(unsigned long long seed, uint32_t stream, uint32_t frame,
+// The 53-bit integer uniform of a decision: u = U / 2^53 = res53(w0, w1).  (Not inlined on
+// the device: the acceptance step draws several, and one copy of the rounds is enough.)
+__host__ __device__ inline __noinline__ unsigned long long uniform_U(unsigned long long seed, uint32_t stream, uint32_t frame,
                                                         int call, int pos, uint32_t purpose) {
   uint32_t w[4];
   philox_block(seed, stream, frame, call, pos, purpose, w);
@@ -347,7 +360,7 @@ constexpr uint32_t kPurposeSibling = 0x10000u;   // + i: test i >= 1 at a tree n
 // Two N(0,1) draws for vocabulary entries (2 pair, 2 pair + 1) of a noisy draft row: the
 // Box-Muller transform (Box and Muller, 1958) of the 53-bit uniforms of words (0,1) and
 // (2,3) of purpose 3 + pair, radius sqrt(-2 ln(1 - u1)), angle 2 pi u2, in fp64.
-__device__ inline double2 normal_pair(unsigned long long seed, uint32_t stream, uint32_t frame, int round,
+__device__ inline __noinline__ double2 normal_pair(unsigned long long seed, uint32_t stream, uint32_t frame, int round,
                                       int position, int pair) {
   uint32_t c[4] = {stream, frame, ((uint32_t)round << 8) | (uint32_t)position, (uint32_t)(PURPOSE_NOISE + pair)};
   philox4x32_10(c, (uint32_t)seed, (uint32_t)(seed >> 32));

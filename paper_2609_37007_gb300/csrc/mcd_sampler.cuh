@@ -26,6 +26,8 @@ struct TopkScratch {
   uint32_t part[2][kConsumerWarps][8];   // per-warp counts of the threshold search (double-buffered)
   uint32_t wred[2][kConsumerWarps];      // per-warp maxima / scan totals (double-buffered)
   unsigned long long wsum[kConsumerWarps];
+  uint32_t kept_key[kMaxTopK];           // the set in id order: keys and ids
+  int kept_id[kMaxTopK];
 };
 static_assert(sizeof(TopkScratch) <= kActBytes, "top-k scratch must fit the activation region");
 
@@ -112,16 +114,19 @@ __device__ __forceinline__ uint32_t block_exscan(uint32_t v, TopkScratch& s, int
 //       otherwise (or for a non-finite range) a counting search over key thresholds, 3 bits
 //       per step, finds Tk;
 //   (4) one prefix scan of the packed per-thread counts (keys > Tk, keys == Tk) places the
-//       set in id order (ties at the threshold keep the lowest ids) and gives every weight.
+//       set in id order (ties at the threshold keep the lowest ids) in shared memory; then
+//       thread i computes the weight of entry i (one exponential per thread, not one per key).
 // `greedy` replaces the distribution by the one-hot of the argmax (ties: lowest id).  `dbg`,
 // when not null, receives clock64() stamps at the phase boundaries (profiling only).
-static __device__ __noinline__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
-                                  TopkScratch& s, TopkRec* out, long long* dbg = nullptr) {
+// kJ = float4 chunks per thread the instantiation holds (ceil(V / 1024) <= kJ): block_topk
+// runs the smallest instantiation that fits V, so a call executes only the code it needs.
+template <int kJ>
+static __device__ __noinline__ void block_topk_j(const float* __restrict__ logits, int V, int k, float T, int greedy,
+                                                 TopkScratch& s, TopkRec* out, long long* dbg) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
 #define MCD_TOPK_STAMP(i) \
   if (dbg && tid == 0) dbg[i] = clock64();
   MCD_TOPK_STAMP(0)
-  constexpr int kJ = kMaxVocab / 1024;
   constexpr int kBins = TopkScratch::kBins;
   static_assert(kBins == kConsumerThreads, "one histogram bin per consumer thread");
   const int nj = (V + 1023) >> 10;                 // float4 chunks per thread
@@ -311,9 +316,6 @@ static __device__ __noinline__ void block_topk(const float* __restrict__ logits,
   const uint32_t krem = (uint32_t)k - (tot & 0xFFFFu);      // threshold keys to keep (>= 1)
   uint32_t tie = pre >> 16;
   uint32_t pos = (pre & 0xFFFFu) + min(tie, krem);
-  const float Td = T;
-  const float zmax = __fdiv_rn(key_f32(kmax), Td);
-  unsigned long long wsum = 0;
 #pragma unroll
   for (int e = 0; e < 4 * kJ; ++e) {
     if (e < n_valid) {
@@ -322,14 +324,22 @@ static __device__ __noinline__ void block_topk(const float* __restrict__ logits,
       const bool inc = kv > Tk || (eq && tie < krem);
       tie += eq ? 1u : 0u;
       if (inc) {
-        const float z = __fdiv_rn(key_f32(kv), Td);
-        const uint32_t w = weight24(exp32_cw(__fsub_rn(z, zmax)));
-        out->ids[pos] = E * tid + e;
-        out->W[pos] = w;
-        wsum += w;
+        s.kept_key[pos] = kv;
+        s.kept_id[pos] = E * tid + e;
         ++pos;
       }
     }
+  }
+  consumer_sync();
+  unsigned long long wsum = 0;
+  if (tid < k) {
+    const float Td = T;
+    const float zmax = __fdiv_rn(key_f32(kmax), Td);
+    const float z = __fdiv_rn(key_f32(s.kept_key[tid]), Td);
+    const uint32_t w = weight24(exp32_cw(__fsub_rn(z, zmax)));
+    out->ids[tid] = s.kept_id[tid];
+    out->W[tid] = w;
+    wsum = w;
   }
   MCD_TOPK_STAMP(4)
 #pragma unroll
@@ -346,12 +356,22 @@ static __device__ __noinline__ void block_topk(const float* __restrict__ logits,
   MCD_TOPK_STAMP(5)
 #undef MCD_TOPK_STAMP
 }
+static_assert(kMaxVocab <= 4 * 1024, "block_topk instantiates at most four float4 chunks per thread");
+static __device__ __forceinline__ void block_topk(const float* __restrict__ logits, int V, int k, float T, int greedy,
+                                                  TopkScratch& s, TopkRec* out, long long* dbg = nullptr) {
+  switch ((V + 1023) >> 10) {
+    case 1: block_topk_j<1>(logits, V, k, T, greedy, s, out, dbg); break;
+    case 2: block_topk_j<2>(logits, V, k, T, greedy, s, out, dbg); break;
+    case 3: block_topk_j<3>(logits, V, k, T, greedy, s, out, dbg); break;
+    default: block_topk_j<4>(logits, V, k, T, greedy, s, out, dbg); break;
+  }
+}
 
 // The record helpers read through generic pointers: the frame kernel stages records in
 // shared memory, the standalone sampler kernels read the copies their own CTA wrote.
 
 // W_x of a record (0 outside it), evaluated by a full warp (same value on every lane).
-__device__ __forceinline__ uint32_t warp_weight(const TopkRec* r, int x) {
+__device__ inline __noinline__ uint32_t warp_weight(const TopkRec* r, int x) {
   const int lane = threadIdx.x & 31;
   const int n = r->n;
   int found = -1;
@@ -367,7 +387,7 @@ __device__ __forceinline__ uint32_t warp_weight(const TopkRec* r, int x) {
 // 4L..4L+3 in v[0..3]); returns the first i with U * S < 2^53 * (v_0 + ... + v_i).  The
 // prefix sums are exact integers, so the result equals the sequential walk's.
 constexpr int kDrawPerLane = kMaxTopK / 32;
-__device__ __forceinline__ int warp_draw_lanes(const unsigned long long (&v)[kDrawPerLane], int n,
+__device__ inline __noinline__ int warp_draw_lanes(const unsigned long long (&v)[kDrawPerLane], int n,
                                                unsigned long long S, unsigned long long U) {
   const int lane = threadIdx.x & 31;
   unsigned long long tot = 0;
@@ -394,7 +414,7 @@ __device__ __forceinline__ int warp_draw_lanes(const unsigned long long (&v)[kDr
 }
 
 // Categorical draw from a record, evaluated by a full warp.
-__device__ __forceinline__ int warp_draw(const TopkRec* r, unsigned long long U) {
+__device__ inline __noinline__ int warp_draw(const TopkRec* r, unsigned long long U) {
   const int lane = threadIdx.x & 31, n = r->n;
   unsigned long long v[kDrawPerLane];
 #pragma unroll
@@ -426,7 +446,7 @@ __device__ __forceinline__ int warp_draw_excluding(const TopkRec* r, const int* 
 }
 
 // Residual draw from normalise(max(0, p - q)) over p's entries in p's order, by a full warp.
-static __device__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U) {
+static __device__ __noinline__ int warp_residual(const TopkRec* p, const TopkRec* q, unsigned long long U) {
   const int lane = threadIdx.x & 31;
   const int np = p->n, nq = q->n;
   const unsigned long long Sp = p->S, Sq = q->S;

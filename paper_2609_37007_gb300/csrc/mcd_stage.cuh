@@ -71,6 +71,12 @@ constexpr int kInfoOff = kRmsOff + kMaxCols * 4;
 constexpr int kSmemBytes = kInfoOff + (int)((sizeof(CallInfo) + 15) / 16 * 16);
 static_assert(kSmemBytes <= 227 * 1024, "frame kernel shared memory exceeds the per-CTA limit");
 
+// The dynamic shared memory of the persistent kernels: functions that are not inlined
+// (called once per call or per layer) rebuild the layout from it rather than taking the
+// consumer state by reference, so the inlined stage code keeps its parameters in the
+// constant bank.
+extern __shared__ __align__(1024) uint8_t mcd_dyn_smem[];
+
 __device__ __forceinline__ Smem smem_layout(uint8_t* base) {
   Smem s;
   s.ring = base + kRingOff;
@@ -183,11 +189,13 @@ constexpr int kWoOperandOff = 48 * 1024;
 // +2 last epilogue done and +3 signalled (latest CTA).
 constexpr int kTimelineSlots = 128;
 // (Indexed by verify round; noisy-target passes are not stamped.)
-__device__ __forceinline__ void timeline(const Cons& c, int, int idx, bool any_cta = false) {
-  const CallInfo* ci = c.sm.ci;
-  if (c.p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots && !ci->emu &&
+__device__ __forceinline__ void timeline_p(const FrameParams& p, const CallInfo* ci, int idx, bool any_cta = false) {
+  if (p.timeline && threadIdx.x == 0 && (any_cta || blockIdx.x == 0) && idx < kTimelineSlots && !ci->emu &&
       ci->round0 < kMaxCalls)
-    c.p.timeline[ci->round0 * kTimelineSlots + idx] = globaltimer();
+    p.timeline[ci->round0 * kTimelineSlots + idx] = globaltimer();
+}
+__device__ __forceinline__ void timeline(const Cons& c, int, int idx, bool any_cta = false) {
+  timeline_p(c.p, c.sm.ci, idx, any_cta);
 }
 __device__ __forceinline__ void timeline_max(const Cons& c, int, int idx) {
   const CallInfo* ci = c.sm.ci;
@@ -230,7 +238,7 @@ __device__ __forceinline__ bool hilo_operand(int ncols) { return ncols <= 16; }
 // kt*16 + 2(lane%4) + {0,1,8,9}; fp32 weights get fp32 rows [ncols][ldk] from column kt0*16.
 // Only the first ncp columns are written: an mma output column depends only on its own B
 // column and columns >= ncols are never read back.  Every load of a batch is issued before
-// any of its stores (one memory round trip per 2048 entries).
+// any of its stores (one memory round trip per 1024 entries).
 template <int WT, bool WIDE, class Ld>
 __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
                                              bool want_ss, Ld ld, float* store_raw = nullptr) {
@@ -240,7 +248,7 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
   const int n = (tid >> 2) & ((1 << lg) - 1), t = tid & 3;
   const bool live = n < ncols;
   const int items = (Kdim >> 4) << (2 + lg);       // (k-tile, column, t)
-  constexpr int kE = 8;
+  constexpr int kE = 4;
   float ss = 0.f;
   for (int base = 0; base < items; base += kE * kConsumerThreads) {
     float2 va[kE], vb[kE];
@@ -481,8 +489,9 @@ __device__ __forceinline__ StagePlan plan_stage(const Cons& c, int si, int n_uni
 // they multiply; prep(u0, cnt, step) builds it for the chunk), as many as the reduction
 // buffer holds.  Each chunk: wait for its units' weights, multiply them all, one barrier,
 // then one epilogue pass epi(u, mi, rr, n, v, v8) over the live outputs (columns n < ncols;
-// v8 = row rr + 8 for gate/up pairs).
-template <int WT, bool WIDE, class Key, class Prep, class Epi>
+// v8 = row rr + 8 for gate/up pairs).  QUAD: the epilogue takes rows rr0..rr0+3 of one
+// column at once, epi(u, mi, rr0, n, float4 v) (not with gate/up pairs).
+template <int WT, bool WIDE, bool QUAD = false, class Key, class Prep, class Epi>
 __device__ __forceinline__ void run_stage(Cons& c, int call, const StagePlan& sp, int Kdim, Key opkey, Prep prep,
                                           Epi epi) {
   const FrameParams& p = c.p;
@@ -518,14 +527,29 @@ __device__ __forceinline__ void run_stage(Cons& c, int call, const StagePlan& sp
       c.abort_ = true;
       return;
     }
-    for (int o = threadIdx.x; o < (cnt << lg_unit); o += kConsumerThreads) {
-      const int r = o >> lg_unit, q = o & ((1 << lg_unit) - 1);
-      const int row = q >> lgn, n = q & ((1 << lgn) - 1);
-      if (n < ncols) {
-        const int mi = row >> (pairs_rows ? 3 : 4), rr = row & (pairs_rows ? 7 : 15);
-        const float v = red_sum(c, g, sp.role, r, mi, rr, n);
-        const float v8 = pairs_rows ? red_sum(c, g, sp.role, r, mi, rr + 8, n) : 0.f;
-        epi(u0 + r * ur.step, mi, rr, n, v, v8);
+    if constexpr (QUAD) {
+      const int lg_q = lg_unit - 2;
+      for (int o = threadIdx.x; o < (cnt << lg_q); o += kConsumerThreads) {
+        const int r = o >> lg_q, q = o & ((1 << lg_q) - 1);
+        const int row4 = q >> lgn, n = q & ((1 << lgn) - 1);
+        if (n < ncols) {
+          const int mi = row4 >> 2, rr0 = (row4 & 3) << 2;
+          const float4 v = make_float4(red_sum(c, g, sp.role, r, mi, rr0, n), red_sum(c, g, sp.role, r, mi, rr0 + 1, n),
+                                       red_sum(c, g, sp.role, r, mi, rr0 + 2, n),
+                                       red_sum(c, g, sp.role, r, mi, rr0 + 3, n));
+          epi(u0 + r * ur.step, mi, rr0, n, v);
+        }
+      }
+    } else {
+      for (int o = threadIdx.x; o < (cnt << lg_unit); o += kConsumerThreads) {
+        const int r = o >> lg_unit, q = o & ((1 << lg_unit) - 1);
+        const int row = q >> lgn, n = q & ((1 << lgn) - 1);
+        if (n < ncols) {
+          const int mi = row >> (pairs_rows ? 3 : 4), rr = row & (pairs_rows ? 7 : 15);
+          const float v = red_sum(c, g, sp.role, r, mi, rr, n);
+          const float v8 = pairs_rows ? red_sum(c, g, sp.role, r, mi, rr + 8, n) : 0.f;
+          epi(u0 + r * ur.step, mi, rr, n, v, v8);
+        }
       }
     }
     u0 += cnt * ur.step;
