@@ -129,12 +129,17 @@ typedef struct {
   int32_t reserved[24];
 } mcd_call_trace;
 
-/* Create a context on the current CUDA device.  `cfg` (host) is copied.  `cuda_stream`
- * is a cudaStream_t (NULL = legacy default stream) used by every later call.
- * Allocates device buffers and sets kernel attributes.  On failure *out is NULL. */
+/* Create a context on the current CUDA device for one MultiCodeDecoder (the 5-layer
+ * inner model of Sec. 1 and Fig. 1 that emits c1..c15 after c0, with one embedding table
+ * and one LM head per residual position, Sec. 2.1) and its sampling configuration.
+ * `cfg` (host) is copied.  `cuda_stream` is a cudaStream_t (NULL = legacy default stream)
+ * used by every later call.  Allocates device buffers and sets kernel attributes.  On
+ * failure *out is NULL. */
 mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out);
 
-/* Load all weights.  `names`, `host_ptrs`, `nbytes`: n host arrays describing named
+/* Load all weights of the model of Sec. 1 / Fig. 1 (the backbone, the per-position tables
+ * and LM heads of Sec. 2.1, and the offsets b_1..b_K of Sec. 2.2 "RVQ position aware
+ * offsets", Fig. 3).  `names`, `host_ptrs`, `nbytes`: n host arrays describing named
  * tensors in the dtype of cfg.weight_dtype (bf16 as raw 16-bit patterns), row-major,
  * matrices [out, in].  Required names (l = layer, i = table, P = position, j = offset):
  *   layers.l.{attn_norm[H], wq[Hq*D,H], wk[Hkv*D,H], wv[Hkv*D,H], q_norm[D], k_norm[D]
@@ -146,7 +151,9 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out);
 mcd_status mcd_load_weights(mcd_ctx* ctx, int32_t n, const char* const* names,
                             const void* const* host_ptrs, const int64_t* nbytes);
 
-/* Decode one frame: emit c1..c_{n_pos} into codes_out (dev int32 [n_pos]).
+/* Decode one frame: emit c1..c_{n_pos} into codes_out (dev int32 [n_pos]) -- the per-frame
+ * inner loop of Sec. 1 / Fig. 1, run with the draft-and-verify calls of Sec. 2.2 / Fig. 3
+ * until every residual code of the frame is emitted.
  *   cond   dev float [hidden], 16-byte aligned: the outer model's hidden state
  *          (sequence position 0).
  *   c0     dev int32 [1]: the frame's c0 id (c0_vocab > 0), else NULL; an id outside
@@ -189,7 +196,10 @@ mcd_status mcd_decode_frame_host(mcd_ctx* ctx, uint32_t stream_id, uint32_t fram
                                  const float* cond, const int32_t* c0, const float* c0_emb,
                                  int32_t* codes_out, mcd_frame_stats* stats);
 
-/* Stepwise use of the same kernels.  mcd_begin_frame resets the per-frame state and
+/* Stepwise use of the same kernels: one verify call of Sec. 2.2 / Fig. 3 at a time
+ * (LMH_k reads h_k and emits the verified code, LMH_{k+j} reads h_k + b_j and drafts;
+ * acceptance min(1, p/q) with residual resampling, Sec. 3.2).  mcd_begin_frame resets the
+ * per-frame state (Sec. 1: every frame starts at c1 after c0) and
  * selects the (stream id, frame index) of the Philox counters; it needs no weights, so
  * the sampler hooks below can run on a context without them;
  * mcd_verify_accept runs exactly one verify call (the first call feeds cond and c0) and,
@@ -213,7 +223,9 @@ mcd_status mcd_verify_accept(mcd_ctx* ctx, int32_t* emitted, int32_t* n_emitted,
 mcd_status mcd_draft(mcd_ctx* ctx, int32_t pos_k, int32_t call_idx, const float* h_k,
                      int32_t* draft_ids, int32_t* q_ids, uint32_t* q_weights, float* z_out);
 
-/* Sampler on given fp32 logits (parity hook for the acceptance rule).  p_logits dev
+/* Sampler on given fp32 logits: the acceptance rule of Sec. 2.2 and Sec. 3.2 (accept d
+ * with probability min(1, p(d)/q(d)), else resample from normalised max(0, p - q); the
+ * bonus code from p when every draft is kept), as a parity hook.  p_logits dev
  * float [n_drafts+1, vocab] are the verify rows of positions a+1..a+1+n_drafts (the last
  * row is only read when a bonus position exists), q_logits dev float [n_drafts, vocab]
  * the draft rows, draft_ids dev int32 [n_drafts].  Uniforms use (call_idx, position)
@@ -246,11 +258,15 @@ mcd_status mcd_topk_softmax(mcd_ctx* ctx, int32_t n_rows, const float* logits,
  *            [n_rows, top_k]; sums dev uint64 [n_rows]; any output may be NULL
  *   top_k in 1..min(128, vocab); temperature > 0; cuda_stream a cudaStream_t (NULL = legacy
  *   default stream).  Results are the ones mcd_topk_softmax gives for the same rows.
- * Errors: MCD_ERR_INVALID_ARG for a bad pointer, alignment, vocab, top_k or temperature;
- * MCD_ERR_UNSUPPORTED for n_rows > MCD_STATIC_TOPK_MAX_ROWS (nothing is launched) or
- * vocab > 4096; MCD_ERR_CUDA if the set-up or the launch fails.
+ * Errors: MCD_ERR_INVALID_ARG for a bad pointer, alignment, vocab (< 16 or not a multiple
+ * of 16), top_k < 1 or top_k > vocab, or temperature; MCD_ERR_UNSUPPORTED for
+ * n_rows > MCD_STATIC_TOPK_MAX_ROWS (nothing is launched), top_k > 128 or vocab > 4096
+ * (the limits mcd_create reports the same way); MCD_ERR_CUDA if the set-up or the launch
+ * fails.
  * The first call on each device (made with that device current) does a one-time set-up
  * that looks up the scratch's device address; make it before any stream capture begins.
+ * Later calls take no lock.  After cudaDeviceReset the cached address is stale: do not
+ * call this entry point on that device again in the same process.
  * Nothing in the scratch needs to start at zero.  The scratch is shared by every call on
  * a device: calls whose work can overlap (other streams, other host threads) race on it,
  * so serialise them, e.g. on one stream. */

@@ -2,6 +2,7 @@
 // callers that must not allocate device memory.  Its per-row records live in one
 // file-scope __device__ array (kStaticTopkRows records) instead of context scratch, so
 // the call needs no mcd_ctx (whose creation allocates) and allocates nothing itself.
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -18,21 +19,31 @@ constexpr int kMaxDevices = 64;
 // writes every field a row's copy-out reads before it is read.
 __device__ __align__(256) TopkRec g_topk_scratch[kStaticTopkRows];
 
+// Per-device address of the scratch.  After the first call on a device every call reads it
+// with one acquire load and takes no lock (the point of this entry point is a caller that
+// must not block on locks other threads hold); only the one-time look-up is serialised.
+// A cudaDeviceReset invalidates the cached address: this entry point must not be used on
+// that device again in the process afterwards.
 std::mutex g_setup_mutex;
-TopkRec* g_scratch_ptr[kMaxDevices] = {};
+std::atomic<TopkRec*> g_scratch_ptr[kMaxDevices] = {};
 
 // Device address of the scratch on the current device, looked up once per device.
 mcd_status scratch_for_current_device(TopkRec** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return MCD_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return MCD_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_topk_scratch) != cudaSuccess || !p) return MCD_ERR_CUDA;
-    g_scratch_ptr[dev] = static_cast<TopkRec*>(p);
+  TopkRec* ptr = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (!ptr) {
+    std::lock_guard<std::mutex> lock(g_setup_mutex);
+    ptr = g_scratch_ptr[dev].load(std::memory_order_relaxed);
+    if (!ptr) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_topk_scratch) != cudaSuccess || !p) return MCD_ERR_CUDA;
+      ptr = static_cast<TopkRec*>(p);
+      g_scratch_ptr[dev].store(ptr, std::memory_order_release);
+    }
   }
-  *out = g_scratch_ptr[dev];
+  *out = ptr;
   return MCD_OK;
 }
 

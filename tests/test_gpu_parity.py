@@ -180,28 +180,66 @@ def test_tiny_frames_trace_parity(tiny):
     print("tiny max |dlogit|", worst)
 
 
+def _first_round_explained_by_a_near_tie(cfg, model, fr, frame_idx, trace, ref):
+    """The GPU's decisions are the oracle sampler's on the GPU's fp32 logits (the trace
+    check), so a frame whose codes differ from the oracle's own decode must first differ in
+    a round fed identical inputs where the two fp32 logit rows -- within the tolerance of
+    each other -- give different top-k / temperature distributions (a set or a weight on
+    the other side of a boundary).  Returns that round; fails if every distribution of the
+    first differing round is the same."""
+    recs, vlog, dlog = mcd.parse_trace(np.asarray(trace, dtype=np.uint8), cfg.vocab)
+    k, T = cfg.top_k, cfg.temperature
+    for c, rd in enumerate(ref.rounds):
+        r = recs[c]
+        g_emit = [int(v) for v in r["emitted"][: int(r["n_emit"])]]
+        g_next = [int(v) for v in r["next_drafts"][: int(r["n_next"])]]
+        if g_emit == rd.emitted and g_next == rd.next_drafts:
+            continue
+        first = 1 if c == 0 else 0
+        gp = [topk_dist(vlog[c, n], k, T) for n in range(first, int(r["n_rows"]))]
+        op = [topk_dist(rd.verify_logits[pos], k, T) for pos in sorted(rd.verify_logits)]
+        gq = [topk_dist(dlog[c, j], k, T) for j in range(len(g_next))]
+        oq = [topk_dist(z, k, T) for z in rd.draft_logits]
+        assert len(gp) == len(op) and len(gq) == len(oq), c
+        differ = [i for i, (a, b) in enumerate(zip(gp + gq, op + oq)) if a.ids != b.ids or a.W != b.W]
+        assert differ, f"frame {frame_idx} round {c}: same distributions, different decisions"
+        return c
+    raise AssertionError(f"frame {frame_idx}: codes differ but every round agrees")
+
+
 def test_tiny_codes_equal_oracle_end_to_end(tiny):
+    """The GPU's codes equal the oracle's own decode (its fp64 rows rounded to fp32); a frame
+    may differ only where a near-tie in some distribution explains it."""
     cfg = tiny.cfg
     same = 0
     n = 40
     for f in range(n):
         fr = make_frame(cfg, 100 + f)
         codes, st, _ = tiny.decode(fr, 100 + f)
-        ref = decode_frame(tiny.model, fr, frame_idx=100 + f)
-        same += list(codes) == ref.codes
+        ref = decode_frame(tiny.model, fr, frame_idx=100 + f, keep_logits=True)
         if list(codes) == ref.codes:
+            same += 1
             assert int(st[0]) == ref.calls
-    assert same >= n - 1, f"{n - same} of {n} frames differ from the oracle"
+            continue
+        codes2, st2, tr = tiny.decode(fr, 100 + f, trace=True)
+        assert list(codes2) == list(codes)                        # deterministic
+        check_trace_against_oracle(cfg, tiny.model, fr, 0, 100 + f, tr, codes2, int(st2[0]), logit_tol=1e-5)
+        _first_round_explained_by_a_near_tie(cfg, tiny.model, fr, 100 + f, tr, ref)
+    assert same >= n - 4, f"{n - same} of {n} frames differ from the oracle"
 
 
 def test_mcd_frame_trace_parity_full_size(big):
+    """Eight full-size frames at the bench's launch configuration: every call's verify and
+    draft logits within 2e-2 of the oracle's fp64 rows, every decision identical."""
     cfg = big.cfg
-    for f in (0, 1):
+    worst = 0.0
+    for f in range(8):
         fr = make_frame(cfg, f)
         codes, st, tr = big.decode(fr, f, trace=True)
         assert st[4] == 0 and st[1] == cfg.n_pos
-        err = check_trace_against_oracle(cfg, big.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=2e-2)
-        print("bf16 max |dlogit|", err)
+        worst = max(worst, check_trace_against_oracle(cfg, big.model, fr, 0, f, tr, codes, int(st[0]),
+                                                      logit_tol=2e-2))
+    print("bf16 max |dlogit|", worst)
 
 
 def test_mcd_frames_are_complete_and_bounded(big):
@@ -327,10 +365,11 @@ def test_gemm_path_trace_parity_tiny_bf16(cfg):
     env.dec.close()
 
 
-@pytest.mark.parametrize("n_streams,checked", [(32, (0, 13, 31)), (128, (0, 77, 127))])
+@pytest.mark.parametrize("n_streams,checked", [(32, (0, 13, 31)), (128, tuple(range(128)))])
 def test_gemm_path_full_size(n_streams, checked):
     """MultiCodeDecoder bf16 at B = 32 and 128 streams (128 and 512 packed rows): every
-    stream finishes its frame; sampled streams replay exactly against the oracle."""
+    stream finishes its frame; at B = 128 every stream (three sampled ones at B = 32)
+    replays exactly against the oracle."""
     cfg = MCD.replace(max_streams=n_streams)
     env = Env(cfg)
     fidx, sids = [7 + s for s in range(n_streams)], [1000 + s for s in range(n_streams)]
@@ -444,15 +483,26 @@ def test_noise_free_target_drafts_are_all_kept_on_gpu():
     env.dec.close()
 
 
-def test_mcd_noisy_target_trace_parity_full_size():
-    cfg = MCD.replace(draft_mode=DRAFT_NOISY_TARGET, noise_sigma=1.0)
+@pytest.mark.parametrize("sigma,frames", [(1.0, 1), (0.25, 6)])
+def test_mcd_noisy_target_trace_parity_full_size(sigma, frames):
+    """Full-size noisy-target frames; at sigma = 0.25 most drafts are kept, so calls that
+    accept two or three drafts (and the bonus draw after them) run at full size."""
+    cfg = MCD.replace(draft_mode=DRAFT_NOISY_TARGET, noise_sigma=sigma)
     env = Env(cfg)
-    fr = make_frame(cfg, 3)
-    codes, st, tr = env.decode(fr, 3, trace=True)
-    assert st[4] == 0 and st[1] == cfg.n_pos
-    err = check_trace_against_oracle(cfg, env.model, fr, 0, 3, tr, codes, int(st[0]), logit_tol=2e-2,
-                                     draft_mode=cfg.draft_mode)
-    print("mcd noisy max |dlogit|", err)
+    accepted = multi = 0
+    for f in range(3, 3 + frames):
+        fr = make_frame(cfg, f)
+        codes, st, tr = env.decode(fr, f, trace=True)
+        assert st[4] == 0 and st[1] == cfg.n_pos
+        err = check_trace_against_oracle(cfg, env.model, fr, 0, f, tr, codes, int(st[0]), logit_tol=2e-2,
+                                         draft_mode=cfg.draft_mode)
+        recs, _, _ = mcd.parse_trace(np.asarray(tr, dtype=np.uint8), cfg.vocab)
+        n_acc = [int(recs[c]["n_acc"]) for c in range(int(st[0]))]
+        accepted += sum(n_acc)
+        multi += sum(1 for v in n_acc if v >= 2)
+        print("mcd noisy sigma", sigma, "max |dlogit|", err)
+    if sigma <= 0.25:
+        assert multi >= frames, (accepted, multi)
     env.dec.close()
 
 
@@ -690,3 +740,79 @@ def test_chi_square_of_gpu_codes_against_exact_law(tiny):
     mean_calls = stats[:, 0].mean()
     exp_calls = float(exp_calls)
     assert abs(mean_calls - exp_calls) < 4 * stats[:, 0].std() / math.sqrt(n) + 1e-3, (mean_calls, exp_calls)
+
+
+def _decode_fixed_input(env, n, stream_id, frame0):
+    """n frames of one fixed frame input (frame 0's cond and c0), frame indices frame0 + i, so
+    only the Philox counters differ between frames."""
+    cfg = env.cfg
+    cond, c0, emb = env.frame_inputs(make_frame(cfg, 0))
+    codes = torch.zeros((n, cfg.n_pos), dtype=torch.int32, device=DEV)
+    stats = torch.zeros((n, 8), dtype=torch.int32, device=DEV)
+    for i in range(n):
+        mcd.mcd_decode_frame(env.dec.ctx, stream_id, frame0 + i, cond, c0, emb, codes[i], stats[i])
+    mcd.mcd_sync(env.dec.ctx)
+    codes, stats = codes.cpu().numpy(), stats.cpu().numpy()
+    assert (stats[:, 4] == 0).all() and (stats[:, 1] == cfg.n_pos).all()
+    return codes, stats
+
+
+def _chi2_goodness(obs: Counter, law: dict, n: int, min_expected=5.0):
+    from scipy import stats as ss
+    keys = sorted(law)
+    e = np.array([law[k] * n for k in keys])
+    o = np.array([obs.get(k, 0) for k in keys])
+    assert o.sum() == n, "codes outside the law's support"
+    big_ = e >= min_expected
+    o2, e2 = np.append(o[big_], o[~big_].sum()), np.append(e[big_], e[~big_].sum())
+    if e2[-1] == 0:
+        o2, e2 = o2[:-1], e2[:-1]
+    return ss.chisquare(o2, e2 * o2.sum() / e2.sum()).pvalue
+
+
+def test_chi_square_full_size_against_exact_law_and_ar(big):
+    """MCD bf16 workload (V = 2048, top-k 50, T 0.9, K = 3): 20,000 frames of one fixed
+    frame input.  (1) The c1 histogram and the (c1, c2) histogram against the exact law the
+    oracle gives for that input (c1 ~ p_1; c2 | c1 ~ p_2 of the row fed c1: one pass for c1
+    and one row per c1 in its top-50), i.e. speculative decoding emits the target's top-k
+    law (Sec. 3.2).  (2) A two-sample test of the speculative codes against 20,000 frames
+    of the non-speculative decoder (K = 0, same kernels) at every position c1..c15."""
+    from scipy import stats as ss
+    cfg = big.cfg
+    n = 20000
+    spec, _ = _decode_fixed_input(big, n, 2, 50_000)
+    # exact law of c1 and of (c1, c2) from the oracle's fp64 rows
+    m, fr = big.model, make_frame(cfg, 0)
+    kv = m.new_kv()
+    m.row(kv, np.asarray(fr.cond, dtype=np.float64), 0)
+    h1 = m.row(kv, m.c0_row(fr.c0, fr.c0_emb), 1)
+    p1 = topk_dist(m.verify_logits(1, h1).astype(np.float32), cfg.top_k, cfg.temperature)
+    law1 = {(x,): p1.prob(x) for x in p1.ids}
+    law12 = {}
+    for x in p1.ids:
+        h2 = m.row(kv, m.code_row(1, x), 2)
+        p2 = topk_dist(m.verify_logits(2, h2).astype(np.float32), cfg.top_k, cfg.temperature)
+        for y in p2.ids:
+            law12[(x, y)] = p1.prob(x) * p2.prob(y)
+    pv1 = _chi2_goodness(Counter((int(r[0]),) for r in spec), law1, n)
+    pv12 = _chi2_goodness(Counter((int(r[0]), int(r[1])) for r in spec), law12, n)
+    print("full-size chi-square p: c1", pv1, "(c1, c2)", pv12)
+    assert pv1 > 1e-4 and pv12 > 1e-4, (pv1, pv12)
+    # speculative vs autoregressive, position by position
+    ar_env = Env(cfg.replace(draft_len=0), big.w)
+    try:
+        ar, _ = _decode_fixed_input(ar_env, n, 3, 90_000)
+    finally:
+        ar_env.dec.close()
+    worst = 1.0
+    for t in range(cfg.n_pos):
+        cs, ca = Counter(spec[:, t].tolist()), Counter(ar[:, t].tolist())
+        keys = sorted(set(cs) | set(ca))
+        tab = np.array([[cs.get(k, 0) for k in keys], [ca.get(k, 0) for k in keys]], dtype=np.float64)
+        common = tab.sum(axis=0) >= 10
+        tab = np.concatenate([tab[:, common], tab[:, ~common].sum(axis=1, keepdims=True)], axis=1)
+        tab = tab[:, tab.sum(axis=0) > 0]
+        p = ss.chi2_contingency(tab)[1] if tab.shape[1] > 1 else 1.0
+        worst = min(worst, p)
+        assert p > 1e-5, (t, p)
+    print("spec vs AR two-sample chi-square: smallest p over c1..c15", worst)
