@@ -824,11 +824,28 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
   // ---- S5: final RMSNorm -> verify and draft heads ---------------------------------------
   // Operand column r is packed row r (h before its 1/rms).  LM head P's output for row r at
   // position pos is its verify logits (j = P - pos = 0) or the draft logits of offset j
-  // (1 <= j <= K), whose LMH_P b_j term comes from the precomputed bias table (staged per
-  // chunk in `vec`, which is free once the operand is built).  The call streams the union
-  // of the heads its streams need.
+  // (1 <= j <= K), whose LMH_P b_j term comes from the precomputed bias table.  The call
+  // streams the union of the heads its streams need.  The bias depends only on the call's
+  // heads and row positions: a single stream with at most kPreUnits head units in this CTA
+  // loads its tiles before waiting for the last layer (upper half of `vec`, the gain stays
+  // in the lower half); otherwise each chunk stages them once the operand is built.
   g2s_vec(sm.vec, p.final_norm, H);
   const StagePlan sp_head = plan_stage<WT, WIDE>(c, 4 * L, ci->n_heads * p.g[MAT_HEAD].n_units, n_rows, no_key);
+  constexpr int kPreUnits = kVecFloats / 2 / (16 * 8);
+  const int n_head_units = sp_head.ur.end - sp_head.ur.first;         // contiguous range, step 1
+  const bool pre_bias = !WIDE && n_rows <= 8 && H <= kVecFloats / 2 && n_head_units <= kPreUnits;
+  float* bias_pre = sm.vec + kVecFloats / 2;                          // [unit][16 rows][8 columns]
+  auto head_bias_at = [&](int u, int rr, int n) -> float {
+    const MatGeom& g = p.g[MAT_HEAD];
+    const int P = ci->heads[u / g.n_units];
+    if (n >= n_rows) return 0.f;
+    const int j = P - ci->r_pos[n];
+    if (j < 1 || j > p.K || ci->r_pos[n] < 1) return 0.f;
+    return __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + (u % g.n_units) * 16 + rr);
+  };
+  if (pre_bias)
+    for (int o = threadIdx.x; o < n_head_units * 128; o += kConsumerThreads)
+      bias_pre[o] = head_bias_at(sp_head.ur.first + (o >> 7), (o >> 3) & 15, o & 7);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
   prep_operand<WT, WIDE>(c, n_rows, H, 0, H, sm.vec, true, from_x);
   {
@@ -839,28 +856,20 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
         c, call, sp_head, H, no_key,
         [&](int u0, int cnt, int step) {
           chunk_u0 = u0;
+          if (pre_bias) return;
           for (int o = threadIdx.x; o < cnt * 16 * kMaxCols; o += kConsumerThreads) {
             const int r = o / (16 * kMaxCols), rr = (o / kMaxCols) & 15, n = o % kMaxCols;
-            const int u = u0 + r * step;
-            const int P = ci->heads[u / g.n_units];
-            float bv = 0.f;
-            if (n < n_rows) {
-              const int j = P - ci->r_pos[n];
-              if (j >= 1 && j <= p.K && ci->r_pos[n] >= 1) {
-                const int id = (u % g.n_units) * 16 + rr;
-                bv = __ldg(p.head_bias + ((size_t)(P - 1) * p.K + (j - 1)) * p.V + id);
-              }
-            }
-            bias_s[o] = bv;
+            bias_s[o] = head_bias_at(u0 + r * step, rr, n);
           }
         },
         [&](int u, int mi, int rr, int n, float v, float) {
           const int P = ci->heads[u / g.n_units], pos = ci->r_pos[n], j = P - pos;
           if (pos >= 1 && j >= 0 && j <= p.K) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
+            const float b = pre_bias ? bias_pre[((u - sp_head.ur.first) * 16 + rr) * 8 + n]
+                                     : bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
             p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
-                v * sm.inv_rms[n] * wscale<WT>(p.s_head, (size_t)(P - 1) * p.V + id) +
-                bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
+                v * sm.inv_rms[n] * wscale<WT>(p.s_head, (size_t)(P - 1) * p.V + id) + b;
           }
         });
     if (c.abort_) return;
