@@ -171,6 +171,21 @@ def cpu_oracle_baseline(cfg, weights, budget_s: float, first_frame: int):
                       f"fp64 numpy oracle in {dt:.1f} s"}
 
 
+def cpu_oracle_single_thread(budget_s: float, first_frame: int):
+    """cpu_oracle_baseline with one BLAS / OpenMP thread, in a child process (the thread count
+    of numpy's BLAS is fixed when it is loaded)."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json, sys; sys.path.insert(0, sys.argv[1]); import bench; "
+            "from paper_2609_37007_gb300.synth import MCD, make_weights; "
+            "print(json.dumps(bench.cpu_oracle_baseline(MCD, make_weights(MCD), float(sys.argv[2]), int(sys.argv[3]))))")
+    try:
+        r = subprocess.run([sys.executable, "-c", code, ROOT, str(budget_s), str(first_frame)], env=env,
+                           capture_output=True, text=True, timeout=600)
+        return json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception as e:                                  # reported, not fatal
+        return {"value": None, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": f"not measured: {e}"}
+
+
 def blas_threads() -> int:
     v = os.environ.get("OPENBLAS_NUM_THREADS") or os.environ.get("OMP_NUM_THREADS")
     return int(v) if v else (os.cpu_count() or 1)
@@ -252,9 +267,12 @@ def run_sweep(args, weights):
         assert (st[:, 4] == 0).all() and (st[:, 1] == MCD.n_pos).all()
         return e0.elapsed_time(e1) * 1e3, int(st[:, 0].sum()), int(st[:, 1].sum())
 
+    clocks = Clocks(0)
     for K in range(1, 8):
         dec = mcd.Decoder(MCD.replace(draft_len=K), weights, stream)
+        clocks.start()
         t_us, calls, toks = frames(dec)
+        clk = clocks.stop()
         dec.close()
         us_per_call = t_us / calls
         for sigma in args.sigmas:
@@ -266,7 +284,8 @@ def run_sweep(args, weights):
             print(json.dumps({"sweep": "noisy-target draft length x sigma", "K": K, "sigma": sigma,
                               "tokens_per_call": tpc, "us_per_verify_call": us_per_call,
                               "tokens_per_s": tpc / us_per_call * 1e6, "frames": n,
-                              "us_per_call_from": "position-aware drafter frames at the same K"}), flush=True)
+                              "us_per_call_from": "position-aware drafter frames at the same K",
+                              "clocks": clk}), flush=True)
 
 
 def run_tree_sweep(args, weights):
@@ -363,11 +382,14 @@ def run_streams(args, weights):
             launch(i)
         mcd.mcd_sync(dec.ctx)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        clocks = Clocks(0)
+        clocks.start()
         e0.record(stream)
         for i in range(3, n + 3):
             launch(i)
         e1.record(stream)
         torch.cuda.synchronize(dev)
+        clk = clocks.stop()
         mcd.mcd_sync(dec.ctx)
         st = stats.cpu().numpy()[3:]
         assert (st[:, :, 4] == 0).all() and (st[:, :, 1] == cfg.n_pos).all()
@@ -377,8 +399,58 @@ def run_streams(args, weights):
         print(json.dumps({"streams": B, "tokens_per_s": toks / t, "launches_per_s": n / t,
                           "us_per_call": 1e6 * t / calls, "calls_per_launch": calls / n,
                           "tokens_per_call_per_stream": float(st[:, :, 1].sum() / st[:, :, 0].sum()),
-                          "launches": n, "workload": WORKLOAD.replace("single stream", f"{B} streams")}), flush=True)
+                          "launches": n, "workload": WORKLOAD.replace("single stream", f"{B} streams"),
+                          "clocks": clk}), flush=True)
         dec.close()
+
+
+def run_timeline(args, weights):
+    """Per-stage timeline of the frame kernel (profiling only): %globaltimer stamps the kernel
+    writes while a timeline buffer is set (mcd_set_timeline), medians over the verify calls
+    after the first of frames 10.. of args.timeline frames.  Stage s (4 per layer, then the
+    LM heads): "ready" = CTA 0 passed its input wait, "data" = its first weight unit was in
+    shared memory, "lastdone" = the last CTA's last epilogue, "signalled" = the last CTA's
+    arrival; then top-k, acceptance and the hand-over to the next call.  Prints one JSON line."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    from paper_2609_37007_gb300.synth import MCD, make_frames
+    _build.build()
+    cfg = MCD
+    dev = torch.device("cuda", 0)
+    dec = mcd.Decoder(cfg, weights)
+    n = max(12, args.timeline)
+    cond_h, c0_h, _ = make_frames(cfg, n, first=4_000_000)
+    cond, c0 = torch.from_numpy(cond_h).to(dev), torch.from_numpy(c0_h).to(dev)
+    codes = torch.zeros((n, cfg.n_pos), dtype=torch.int32, device=dev)
+    stats = torch.zeros((n, 8), dtype=torch.int32, device=dev)
+    tl = torch.zeros((n, 16, 128), dtype=torch.int64, device=dev)
+    for i in range(n):
+        mcd.mcd_set_timeline(dec.ctx, tl[i])
+        mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
+    mcd.mcd_sync(dec.ctx)
+    dec.close()
+    tl, st = tl.cpu().numpy().astype(np.float64), stats.cpu().numpy()
+    rows = np.array([tl[i, c] - tl[i, c, 0] for i in range(10, n) for c in range(1, int(st[i, 0]))]) / 1e3
+    med = lambda col: float(np.median(rows[:, col]))
+    names = [f"L{l}.{k}" for l in range(cfg.n_layers) for k in ("qkv", "att+wo", "gate/up", "down")] + ["heads"]
+    stages, prev = [], 0.0
+    for si, nm in enumerate(names):
+        b = 8 + 4 * si
+        r0, r1, r2, r3 = med(b), med(b + 1), med(b + 2), med(b + 3)
+        stages.append({"stage": nm, "ready_us": r0, "gap_us": r0 - prev, "data_us": r1 - r0, "lastdone_us": r2 - r0,
+                       "signalled_us": r3 - r2})
+        prev = r3
+    gaps = [(tl[i, c + 1, 0] - tl[i, c, 7]) / 1e3 for i in range(10, n) for c in range(int(st[i, 0]) - 1)]
+    line = {"timeline": "frame_kernel<bf16>, MultiCodeDecoder bf16 workload, K = 3, one stream",
+            "frames": n - 10, "calls": len(rows), "us_per_call": med(7), "stages": stages,
+            "topk": {"ready_us": med(1), "cta0_done_us": med(2) - med(1), "last_done_us": med(3) - med(1)},
+            "accept": {"start_us": med(4), "staged_us": med(5) - med(4), "decided_us": med(6) - med(5),
+                       "end_us": med(7) - med(6)},
+            "handover_us": float(np.median(gaps)) if gaps else None,
+            "note": "stamps add a global store per stage and an atomic max per CTA and stage: a stamped call is "
+                    "a few microseconds slower than an unstamped one"}
+    print(json.dumps(line), flush=True)
 
 
 PIPE_METRIC = "sustained frames/s of the full frame pipeline"
@@ -571,14 +643,18 @@ def main():
     ap.add_argument("--pipeline", action="store_true",
                     help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
     ap.add_argument("--utterances", type=int, default=2)
+    ap.add_argument("--timeline", type=int, default=0,
+                    help="print the frame kernel's per-stage timeline over this many frames instead of the bench line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
-    from paper_2609_37007_gb300.synth import MCD, WEIGHT_INT8, make_frames, make_weights
+    from paper_2609_37007_gb300.synth import MCD, WEIGHT_BF16, WEIGHT_INT8, make_frames, make_weights
     cfg = MCD.replace(weight_dtype=WEIGHT_INT8) if args.w8a16 else MCD
     weights = make_weights(cfg)
     if args.impl == "reference":
         return run_reference(args, cfg, weights)
+    if args.timeline:
+        return run_timeline(args, weights)
     if args.streams:
         return run_streams(args, weights)
     if args.pipeline:
@@ -614,6 +690,8 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         cpu = cpu_oracle_baseline(cfg, weights, args.cpu_budget, first_frame=100_000)
+        if cfg.weight_dtype == WEIGHT_BF16:          # the same oracle on one host thread
+            cpu["single_thread"] = cpu_oracle_single_thread(args.cpu_budget / 2, first_frame=200_000)
 
     dec = mcd.Decoder(cfg, weights, stream)
     ctx = dec.ctx
