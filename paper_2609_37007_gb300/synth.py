@@ -60,6 +60,11 @@ class MCDConfig:
     sample_seed: int = 1
     frames: int = 1
     max_streams: int = 1  # streams one launch may decode together
+    # Synthetic structure for the offset-training harness: the table feeding sequence
+    # position s (table 0 -> position 1, table i -> position i + 1) gets s * d added to every
+    # row, d ~ N(0, position_drift^2 / hidden) per dim from its own seeded stream, so hidden
+    # states drift with the position the way a per-lookahead offset can undo.  0 = none.
+    position_drift: float = 0.0
 
     def replace(self, **kw) -> "MCDConfig":
         return dataclasses.replace(self, **kw)
@@ -79,7 +84,11 @@ MCD = MCDConfig(name="mcd_bf16", n_layers=5, hidden=1024, n_q_heads=16, n_kv_hea
                 rope_base=10000.0, qk_norm=1, weight_dtype=WEIGHT_BF16, draft_len=3,
                 top_k=50, temperature=0.9, weight_seed=0, sample_seed=1, frames=1000)
 
-CONFIGS = {c.name: c for c in (TINY, MCD)}
+# The same models with a position drift in their embedding tables (offset-training harness).
+TINY_DRIFT = TINY.replace(name="tiny_fp32_drift", position_drift=2.0)
+MCD_DRIFT = MCD.replace(name="mcd_bf16_drift", position_drift=2.0)
+
+CONFIGS = {c.name: c for c in (TINY, MCD, TINY_DRIFT, MCD_DRIFT)}
 
 
 def tensor_specs(cfg: MCDConfig) -> List[Tuple[str, Tuple[int, ...], str]]:
@@ -122,6 +131,11 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (b.astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
+def _drift(cfg: MCDConfig) -> np.ndarray:
+    rng = np.random.Generator(np.random.PCG64(np.random.SeedSequence([cfg.weight_seed, 13])))
+    return rng.standard_normal(cfg.hidden) * (cfg.position_drift / np.sqrt(cfg.hidden))
+
+
 def make_weights(cfg: MCDConfig) -> Dict[str, np.ndarray]:
     """All weights of `cfg`: float32 arrays for F32 configs, uint16 bf16 bits for BF16."""
     out: Dict[str, np.ndarray] = {}
@@ -132,6 +146,9 @@ def make_weights(cfg: MCDConfig) -> Dict[str, np.ndarray]:
             vals = (1.0 + 0.1 * draw.astype(np.float64)).astype(np.float32)
         else:
             vals = (0.02 * draw.astype(np.float64)).astype(np.float32)
+        if cfg.position_drift and name.startswith("embed."):
+            pos = int(name.split(".")[1]) + 1                       # the sequence position it feeds
+            vals = (vals.astype(np.float64) + pos * _drift(cfg)[None, :]).astype(np.float32)
         out[name] = round_to_bf16_bits(vals) if cfg.weight_dtype in (WEIGHT_BF16, WEIGHT_INT8) else vals
     return out
 
