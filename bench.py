@@ -290,9 +290,9 @@ def run_sweep(args, weights):
 
 def run_tree_sweep(args, weights):
     """Sparse tree verification (Sec. 2.2, Fig. 4): acceptance statistics per (depth, rank)
-    from traced frames of a probe tree, greedy trees of N = 1..31 nodes grown from them,
+    from traced frames of a probe tree, greedy trees of N = 1..64 nodes grown from them,
     then per N: accepted tokens per call, microseconds per verify call and tokens/s.  One
-    JSON line per N."""
+    JSON line per N; a call of more than 32 rows runs in ceil(rows / 32) weight passes."""
     import torch
     from paper_2609_37007_gb300 import build as _build
     from paper_2609_37007_gb300 import mcd
@@ -330,6 +330,7 @@ def run_tree_sweep(args, weights):
     acc = trees.measure_acceptance(records, frame_codes, depth, ranks, cfg.n_pos)
     print(json.dumps({"tree_stats": "P(rank-r candidate of depth d is the emitted code)", "acc": acc,
                       "frames": len(records)}), flush=True)
+    clocks = Clocks(0)
     for N in args.tree_sizes:
         parent, rank = trees.grow_tree(acc, N)
         mcd.mcd_set_tree(dec.ctx, parent, rank)
@@ -337,19 +338,23 @@ def run_tree_sweep(args, weights):
             mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
         mcd.mcd_sync(dec.ctx)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        clocks.start()
         e0.record(stream)
         for i in range(3, n + 3):
             mcd.mcd_decode_frame(dec.ctx, 0, i, cond[i], c0[i:i + 1], None, codes[i], stats[i])
         e1.record(stream)
         torch.cuda.synchronize(dev)
+        clk = clocks.stop()
         mcd.mcd_sync(dec.ctx)
         st = stats.cpu().numpy()[3:]
         assert (st[:, 4] == 0).all() and (st[:, 1] == cfg.n_pos).all()
         t_us = e0.elapsed_time(e1) * 1e3
         calls, toks = int(st[:, 0].sum()), int(st[:, 1].sum())
-        print(json.dumps({"tree_nodes": len(parent), "rows_per_call": 1 + len(parent), "tokens_per_call": toks / calls,
-                          "us_per_verify_call": t_us / calls, "tokens_per_s": toks / t_us * 1e6, "frames": n,
-                          "parent": parent, "rank": rank}), flush=True)
+        rows = 1 + len(parent)
+        print(json.dumps({"tree_nodes": len(parent), "rows_per_call": rows, "passes_per_full_call": -(-rows // 32),
+                          "tokens_per_call": toks / calls, "us_per_verify_call": t_us / calls,
+                          "tokens_per_s": toks / t_us * 1e6, "frames": n, "parent": parent, "rank": rank,
+                          "clocks": clk}), flush=True)
     dec.close()
 
 
@@ -639,7 +644,7 @@ def main():
                     help="the bench line with int8 weights quantised per row at load (W8A16)")
     ap.add_argument("--tree-sweep", action="store_true",
                     help="sparse tree sizes N (greedy trees from measured statistics) instead of the bench line")
-    ap.add_argument("--tree-sizes", type=int, nargs="+", default=[1, 2, 4, 8, 16, 31])
+    ap.add_argument("--tree-sizes", type=int, nargs="+", default=[1, 2, 4, 8, 16, 31, 32, 48, 64])
     ap.add_argument("--pipeline", action="store_true",
                     help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
     ap.add_argument("--utterances", type=int, default=2)

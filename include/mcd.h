@@ -279,24 +279,28 @@ mcd_status mcd_topk_softmax_static(int32_t n_rows, int32_t vocab, int32_t top_k,
  * decoding writes one mcd_call_trace per call followed, after 16 records, by float
  * logits [16 calls][8 rows][vocab] (verify rows) and [16 calls][8 drafts][vocab] (the
  * draft rows used).  In TREE mode the block continues with 16 mcd_tree_trace records and
- * the verify logits of every row, [16 calls][32 rows][vocab].  NULL turns tracing off. */
+ * the verify logits of every row, [16 calls][MCD_MAX_TREE_ROWS rows][vocab].  NULL turns tracing off. */
 int64_t mcd_trace_bytes(const mcd_ctx* ctx);
 mcd_status mcd_set_trace(mcd_ctx* ctx, void* trace);
 
 /* Per-call record of TREE mode (after the mcd_call_trace records; see mcd_set_trace). */
+#define MCD_MAX_TREE_NODES 64
+#define MCD_MAX_TREE_ROWS 65   /* rows of one tree call: the last emitted code + the nodes */
 typedef struct {
   int32_t n_rows;         /* rows fed: row 0 = the last emitted code, then tree nodes     */
-  int32_t row_node[32];   /* tree node of each row (-1: row 0)                            */
-  int32_t row_id[32];     /* code fed at each row                                         */
+  int32_t row_node[MCD_MAX_TREE_ROWS];  /* tree node of each row (-1: row 0)              */
+  int32_t row_id[MCD_MAX_TREE_ROWS];    /* code fed at each row                           */
   int32_t path_len;       /* nodes kept                                                   */
   int32_t path[8];        /* kept nodes, root first                                       */
   int32_t draft_row;      /* row whose draft logits gave the next call's candidates       */
   int32_t n_next;         /* candidate depths of the next call                            */
   int32_t next_cand[8][8];/* [depth - 1][rank] candidate ids of the next call             */
-  int32_t reserved[20];
+  int32_t n_passes;       /* weight passes of the call: ceil(n_rows / 32)                 */
+  int32_t reserved[17];
 } mcd_tree_trace;
 
-/* Sparse tree of TREE mode (Sec. 2.2 "Tree attention ...", Fig. 2): n_nodes <= 31 nodes
+/* Sparse tree of TREE mode (Sec. 2.2 "Tree attention ...", Fig. 2; sizes N = 16..64 as in
+ * the tree sweep of Sec. 3.4, Fig. 4): n_nodes <= 64 (MCD_MAX_TREE_NODES) nodes
  * in breadth-first order (host arrays); node i has parent[i] (-1: a child of the call's
  * first row, else an earlier node) and rank[i] < 8 (distinct among siblings), depth =
  * parent's depth + 1 <= draft_len.  A node of depth d proposes the id of rank rank[i] in
@@ -307,7 +311,10 @@ typedef struct {
  * probability p'(x), p' being the node's distribution without the candidates already
  * rejected there (uniform of counter (call, code position, purpose 1 for i = 0, else
  * 0x10000 + i)); when none is kept, or the node has no children, a code is drawn from p'
- * with purpose 0.  The kept nodes' keys and values become the committed cache.  Until
+ * with purpose 0.  The kept nodes' keys and values become the committed cache.  A call
+ * of more than 32 rows runs as passes of up to 32 rows through the whole model (rows
+ * 32 t .. 32 t + 31 in pass t; later rows attend to earlier ones through the cache); the
+ * acceptance step follows the last pass.  Until
  * set, the tree is the chain of draft_len rank-0 nodes.  Errors: MCD_ERR_INVALID_ARG
  * (malformed tree), MCD_ERR_STATE (context not in TREE mode). */
 mcd_status mcd_set_tree(mcd_ctx* ctx, int32_t n_nodes, const int32_t* parent, const int32_t* rank);

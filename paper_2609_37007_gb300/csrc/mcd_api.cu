@@ -459,7 +459,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   p.S = 1;
   p.trace_stride = (long long)sizeof(mcd_call_trace) * kMaxCalls + (long long)2 * kMaxCalls * kMaxRows * p.V * 4;
   if (k.draft_mode == MCD_DRAFT_TREE)   // + the tree records and every row's verify logits
-    p.trace_stride += (long long)sizeof(mcd_tree_trace) * kMaxCalls + (long long)kMaxCalls * kMaxCols * p.V * 4;
+    p.trace_stride += (long long)sizeof(mcd_tree_trace) * kMaxCalls + (long long)kMaxCalls * kMaxTreeRows * p.V * 4;
   // MCD_WAIT_NS overrides the bound, never below 100 ms: the same bound limits how long an
   // aborting CTA waits for its copies and MMAs in flight, which must land before it exits.
   const char* wn = getenv("MCD_WAIT_NS");
@@ -519,13 +519,17 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
   if ((e = ctx_alloc(c, &p.qkv, sizeof(float) * kMaxCols * p.qkv_dim)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.mbuf, sizeof(float) * kMaxCols * p.F)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.attn, sizeof(float) * kMaxCols * p.NH * p.D)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxCols * (kMaxDraft + 1) * p.V)) != cudaSuccess)
+  if ((e = ctx_alloc(c, &p.logits, sizeof(float) * kMaxTreeRows * (kMaxDraft + 1) * p.V)) != cudaSuccess)
     return fail(cuda_status(e));
-  p.kv_stride = (long long)p.L * p.NKV * kKVSlots * p.D;
+  // cache entries per (layer, KV head): the frame's positions, then in TREE mode the rows of
+  // the current call (slot kMaxPos + row) until its acceptance step commits the kept ones
+  p.kv_slots = kMaxPos + (k.draft_mode == MCD_DRAFT_TREE ? kMaxTreeRows : 0);
+  p.kv_stride = (long long)p.L * p.NKV * p.kv_slots * p.D;
   const size_t kvsz = sizeof(float) * (size_t)p.kv_stride * k.max_streams;
   if ((e = ctx_alloc(c, &p.kcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.vcache, kvsz)) != cudaSuccess) return fail(cuda_status(e));
-  if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * 2 * kMaxCols * (kMaxDraft + 1))) != cudaSuccess)
+  static_assert(kMaxTreeRows <= 2 * kMaxCols + 1, "record buffer rows");
+  if ((e = ctx_alloc(c, &p.topk, sizeof(TopkRec) * (2 * kMaxCols + 1) * (kMaxDraft + 1))) != cudaSuccess)
     return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.draftq, sizeof(TopkRec) * (kMaxDraft + 1))) != cudaSuccess) return fail(cuda_status(e));
   if ((e = ctx_alloc(c, &p.st, sizeof(DevState) * k.max_streams)) != cudaSuccess) return fail(cuda_status(e));
@@ -548,6 +552,7 @@ mcd_status mcd_create(const mcd_config* cfg, void* cuda_stream, mcd_ctx** out) {
       p.tree_rank[i] = 0;
       p.tree_depth[i] = (signed char)(i + 1);
       p.tree_m[i] = 1;
+      p.tree_anc[i] = (2ull << i) - 1ull;
     }
   }
   if (cudaMemsetAsync(p.err, 0, sizeof(int), c->stream) != cudaSuccess) return fail(MCD_ERR_CUDA);
@@ -822,6 +827,7 @@ mcd_status mcd_set_tree(mcd_ctx* c, int32_t n_nodes, const int32_t* parent, cons
     p.tree_parent[i] = (signed char)parent[i];
     p.tree_rank[i] = (signed char)rank[i];
     p.tree_depth[i] = (signed char)depth[i];
+    p.tree_anc[i] = (parent[i] < 0 ? 0ull : p.tree_anc[parent[i]]) | (1ull << i);
   }
   for (int d = 0; d < kMaxDraft; ++d) p.tree_m[d] = m[d];
   return MCD_OK;

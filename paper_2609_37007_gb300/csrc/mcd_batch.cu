@@ -608,7 +608,7 @@ __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, Batch
   __shared__ __align__(16) float ks[kBatchKeys][132];
   __shared__ __align__(16) float vs[kBatchKeys][128];
   __shared__ float sc[kBatchQVec][kBatchKeys];
-  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * p.kv_slots * D;
   const int nk = pos0 + nr;
   const int D4 = D >> 2;
   // loads: queries, then keys and values (cached rows, then the new rows), as 16-byte chunks,

@@ -127,7 +127,7 @@ __device__ __noinline__ void attention_stream(const FrameParams& p, int layer, i
   float2* cs = reinterpret_cast<float2*>(vs + kAttnPos * 128);  // [8][D/2] (cos, sin)
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);      // [D]
   float* gk = gq + 128;                                          // [D]
-  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * p.kv_slots * D;
   const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
   // ---- (A) loads ----------------------------------------------------------------------
@@ -316,7 +316,7 @@ __device__ __noinline__ void attention_rows(const FrameParams& p, int layer, int
   float2* cs = reinterpret_cast<float2*>(qs + kMaxRows * KS);   // [kMaxRows][D/2]
   float* gq = reinterpret_cast<float*>(cs + kMaxRows * 64);     // [D]
   float* gk = gq + 128;                                         // [D]
-  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * p.kv_slots * D;
   const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
   if (pos0 + nr > kAttnKeys) {                // positions beyond c14's row are never fed
@@ -456,23 +456,27 @@ __device__ void attention_head(Cons& c, int layer, int h, bool write_kv) {
   }
 }
 
-// Attention of query head h for rows lo..hi-1 of a tree call (one stream, packed rows from
-// 0).  Keys: the committed positions 0..pos0-1 (cache slots) and the call's rows 0..hi-1,
-// row n seeing row m iff bit m of r_anc[n]; each row is rotated at its own position r_pos
-// (row 0 at pos0, a node of depth d at pos0 + d).  The task of a KV head's first query head
-// stores K / V of rows lo..hi-1: row 0 at its position, node rows at slot kMaxPos + n until
-// the acceptance step commits the kept ones.  Outputs go to p.attn.  Scratch (act + bfrag,
-// 62 KB): k [48][D + 8], v [48][D], q [8][D + 8], RoPE rows by depth [9][D/2], QK-norm
-// gains, scores [8][48].
+// Attention of query head h for rows lo..hi-1 of the current pass of a tree call (one
+// stream; pass row n is tree row row0 + n).  Tree row m >= 1 is node m - 1 at position
+// pos0 + depth; row 0 feeds the last emitted code at pos0.  A query row sees the committed
+// positions 0..pos0-1, row 0, its ancestors and itself (the sparse tree mask of Fig. 2).
+// Keys, compacted: positions 0..pos0-1 (cache slots), then the tree rows visible to at
+// least one query of the group, in tree order.  Rows of earlier passes come from the cache
+// (row 0 at slot pos0, node rows at kMaxPos + m), already normalised and rotated; rows of
+// this pass come from the QKV output and are normalised and rotated here at their own
+// position.  The task of a KV head's first query head stores K / V of rows lo..hi-1.
+// Outputs go to p.attn (pass rows).  Scratch (act + bfrag, 62.6 KB): k [48][D + 8],
+// v [48][D], q [8][D + 8], RoPE rows by depth [8][D/2], QK-norm gains, scores [8][48],
+// the key rows and the queries' ancestor masks.
 __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer, int h, int lo, int hi, int pos0) {
   Smem sm = smem_layout(mcd_dyn_smem);
   const CallInfo* ci = sm.ci;
-  const int D = p.D, half = D >> 1, group = p.NH / p.NKV, g = h / group;
+  const int D = p.D, half = D >> 1, group = p.NH / p.NKV, g = h / group, row0 = ci->row0;
   const bool write_kv = (h % group) == 0;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int cs_shift = D == 128 ? 5 : 4, cpr = 1 << cs_shift;   // 16-byte chunks per row
   const int KS = D + 8;
-  constexpr int kKeys = 48, kDepths = 9;
+  constexpr int kKeys = kTreeKeys, kDepths = kMaxDraft + 1;
   float* ks = sm.act;
   float* vs = ks + kKeys * 136;
   float* qs = vs + kKeys * 128;
@@ -480,16 +484,52 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
   float* gq = reinterpret_cast<float*>(cs + kDepths * 64);
   float* gk = gq + 128;
   float* sc = gk + 128;
-  const size_t cache_off = ((size_t)layer * p.NKV + g) * kKVSlots * D;
+  unsigned long long* qanc = reinterpret_cast<unsigned long long*>(sc + 8 * kKeys);   // [8]
+  int* krow = reinterpret_cast<int*>(qanc + 8);                  // [kKeys - pos0] tree row of key pos0 + i
+  __shared__ int s_nk, s_jc;
+  const size_t cache_off = ((size_t)layer * p.NKV + g) * p.kv_slots * D;
   const float* qkv = p.qkv;
   const int qoff = h * D, koff = p.NH * D + g * D, voff = p.NH * D + p.NKV * D + g * D;
-  const int nq = hi - lo, nk = pos0 + hi;
-  const int dmax = ci->r_pos[hi - 1] - pos0;       // rows are in tree order: depth nondecreasing
+  const int nq = hi - lo, dm = min(p.tree_maxd, kMaxPos - 1 - pos0);   // RoPE rows pos0 .. pos0 + dm
+  // ---- key list: row 0 and the union of the queries' ancestor-or-self sets -----------------
+  if (tid == 0) {
+    unsigned long long U = 0ull;
+    for (int n = lo; n < hi; ++n) {
+      const int m = row0 + n;
+      const unsigned long long am = m > 0 ? p.tree_anc[m - 1] : 0ull;
+      qanc[n - lo] = am;
+      U |= am;
+    }
+    int nk = pos0, jc = -1;
+    krow[0] = 0;
+    ++nk;
+    if (row0 == 0) jc = pos0;
+    while (U) {
+      const int m = __ffsll((long long)U);                       // node m - 1 -> tree row m
+      U &= U - 1ull;
+      if (nk >= kKeys) {                                           // groups are sized to fit
+        atomicCAS(p.err, 0, (int)MCD_ERR_STATE);
+        break;
+      }
+      if (jc < 0 && m >= row0) jc = nk;
+      krow[nk - pos0] = m;
+      ++nk;
+    }
+    s_nk = nk;
+    s_jc = jc < 0 ? nk : jc;                                       // keys jc.. are rows of this pass
+  }
+  consumer_sync();
+  const int nk = s_nk, jc = s_jc;
+  auto key_slot = [&](int j) {                                    // cache slot of an earlier key
+    if (j < pos0) return j;
+    const int m = krow[j - pos0];
+    return m == 0 ? pos0 : kMaxPos + m;
+  };
+  auto row_depth = [&](int m) { return m == 0 ? 0 : (int)p.tree_depth[m - 1]; };
   // ---- (A) loads, 16-byte chunks, batches of 8 per thread in flight --------------------------
   {
-    const int e_q = nq << cs_shift, e_k = e_q + (hi << cs_shift), e_v = e_k + (hi << cs_shift);
-    const int e_kc = e_v + (pos0 << cs_shift), e_vc = e_kc + (pos0 << cs_shift);
-    const int e_cs = e_vc + ((dmax + 1) << cs_shift), e_g = e_cs + (p.qk_norm ? 2 * cpr : 0);
+    const int e_q = nq << cs_shift, e_k = e_q + (nk << cs_shift), e_v = e_k + (nk << cs_shift);
+    const int e_cs = e_v + ((dm + 1) << cs_shift), e_g = e_cs + (p.qk_norm ? 2 * cpr : 0);
     for (int base = 0; base < e_g; base += 8 * kConsumerThreads) {
       float4 v[8];
       float4* dst[8];
@@ -506,16 +546,16 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
           dst[u] = reinterpret_cast<float4*>(qs + (n - lo) * KS) + ch;
         } else if (i < e_v) {
           const bool isv = i >= e_k;
-          const int n = (i - (isv ? e_k : e_q)) >> cs_shift;
-          src = reinterpret_cast<const float4*>(qkv + (size_t)n * p.qkv_dim + (isv ? voff : koff));
-          dst[u] = reinterpret_cast<float4*>(isv ? vs + (pos0 + n) * D : ks + (pos0 + n) * KS) + ch;
-        } else if (i < e_vc) {
-          const bool isv = i >= e_kc;
-          const int j = (i - (isv ? e_kc : e_v)) >> cs_shift;
-          src = reinterpret_cast<const float4*>((isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D);
+          const int j = (i - (isv ? e_k : e_q)) >> cs_shift;
+          if (j >= jc)
+            src = reinterpret_cast<const float4*>(qkv + (size_t)(krow[j - pos0] - row0) * p.qkv_dim +
+                                                  (isv ? voff : koff));
+          else
+            src = reinterpret_cast<const float4*>((isv ? p.vcache : p.kcache) + cache_off +
+                                                  (size_t)key_slot(j) * D);
           dst[u] = reinterpret_cast<float4*>(isv ? vs + j * D : ks + j * KS) + ch;
         } else if (i < e_cs) {
-          const int d = (i - e_vc) >> cs_shift;
+          const int d = (i - e_v) >> cs_shift;
           src = reinterpret_cast<const float4*>(p.rope + (size_t)(pos0 + d) * half);
           dst[u] = reinterpret_cast<float4*>(cs + d * 64) + ch;
         } else {
@@ -531,13 +571,14 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
     }
   }
   consumer_sync();
-  // ---- (B) QK-norm + RoPE of the queries and the new keys; K / V of rows lo..hi-1 stored ------
+  // ---- (B) QK-norm + RoPE of the queries and this pass's keys; K / V of rows lo..hi-1 stored ---
   const int nd = D >> 5;
-  for (int vi = warp; vi < nq + hi; vi += kConsumerWarps) {
+  for (int vi = warp; vi < nq + nk - jc; vi += kConsumerWarps) {
     const bool isq = vi < nq;
-    const int n = isq ? lo + vi : vi - nq;
-    float* row = isq ? qs + (n - lo) * KS : ks + (pos0 + n) * KS;
-    const int depth = ci->r_pos[n] - pos0;
+    const int j = jc + vi - nq;                                   // key index (keys only)
+    const int m = isq ? row0 + lo + vi : krow[j - pos0];          // tree row
+    float* row = isq ? qs + vi * KS : ks + j * KS;
+    const int depth = row_depth(m);
     float x[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) x[i] = i < nd ? row[lane + 32 * i] : 0.f;
@@ -565,11 +606,12 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
 #pragma unroll
     for (int i = 0; i < 4; ++i)
       if (i < nd) row[lane + 32 * i] = x[i];
-    if (!isq && write_kv && n >= lo) {
-      const int slot = n == 0 ? pos0 : kMaxPos + n;
+    const int n = m - row0;                                       // pass row of a key
+    if (!isq && write_kv && n >= lo && n < hi) {
+      const int slot = m == 0 ? pos0 : kMaxPos + m;
       float* kd = p.kcache + cache_off + (size_t)slot * D;
       float* vd = p.vcache + cache_off + (size_t)slot * D;
-      const float* vrow = vs + (pos0 + n) * D;
+      const float* vrow = vs + j * D;
 #pragma unroll
       for (int i = 0; i < 4; ++i)
         if (i < nd) {
@@ -584,8 +626,8 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
     const float scale = rsqrtf((float)D);
     for (int t = tid; t < nq * kKeys * 2; t += kConsumerThreads) {
       const int qi = t / (2 * kKeys), j = (t >> 1) % kKeys, hf = t & 1;
-      const int n = lo + qi;
-      const bool live = j < nk && (j < pos0 || ((ci->r_anc[n] >> (j - pos0)) & 1u));
+      bool live = j < nk;
+      if (live && j > pos0) live = (qanc[qi] >> (krow[j - pos0] - 1)) & 1ull;   // j == pos0: row 0
       float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
       if (live) {
         const float4* q4 = reinterpret_cast<const float4*>(qs + qi * KS) + hf;
@@ -620,12 +662,12 @@ __device__ __noinline__ void attention_tree_task(const FrameParams& p, int layer
     if (lane + 32 < kKeys) sc[qi * kKeys + lane + 32] = e1 / l;
   }
   consumer_sync();
-  // ---- (C3) o = sum_j p_j v_j over keys up to the row itself (ancestors precede it) ------------
+  // ---- (C3) o = sum_j p_j v_j over the keys (masked keys have p_j = 0) ----------------------
   for (int t = tid; t < nq * half; t += kConsumerThreads) {
-    const int qi = t / half, d = 2 * (t - qi * half), n = lo + qi, npos = pos0 + n + 1;
+    const int qi = t / half, d = 2 * (t - qi * half), n = lo + qi;
     const float* pr = sc + qi * kKeys;
     float2 acc = make_float2(0.f, 0.f);
-    for (int j = 0; j < npos; ++j) {
+    for (int j = 0; j < nk; ++j) {
       const float w = pr[j];
       const float2 v = *reinterpret_cast<const float2*>(vs + j * D + d);
       acc.x += w * v.x;
@@ -697,10 +739,11 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
     if (!cons_wait(c, ctr + ctr_stage(l, 0), N)) return;
     if (WIDE) {
       if (p.draft_mode == MCD_DRAFT_TREE && ci->st[0].pos0 > 0) {
-        // tree call (one stream): one task per (query head, group of 8 rows)
-        const int nr = ci->M, n_rg = (nr + 7) >> 3;
-        for (int t = blockIdx.x; t < p.NH * n_rg; t += p.n_cta)
-          attention_tree_task(p, l, t % p.NH, 8 * (t / p.NH), min(8 * (t / p.NH) + 8, nr), ci->st[0].pos0);
+        // tree call (one stream): one task per (query head, row group of the pass)
+        for (int t = blockIdx.x; t < p.NH * ci->n_tg; t += p.n_cta) {
+          const int gi = t / p.NH;
+          attention_tree_task(p, l, t - gi * p.NH, ci->tg[gi], ci->tg[gi + 1], ci->st[0].pos0);
+        }
       } else {
         const int group = p.NH / p.NKV, n_tasks = ci->n_act * p.NH;
         for (int t = blockIdx.x; t < n_tasks; t += p.n_cta) {
@@ -868,7 +911,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
             const int id = (u % g.n_units) * g.Mu * 16 + mi * 16 + rr;
             const float b = pre_bias ? bias_pre[((u - sp_head.ur.first) * 16 + rr) * 8 + n]
                                      : bias_s[((u - chunk_u0) * 16 + rr) * kMaxCols + n];
-            p.logits[((size_t)n * (kMaxDraft + 1) + j) * p.V + id] =
+            p.logits[((size_t)(ci->row0 + n) * (kMaxDraft + 1) + j) * p.V + id] =
                 v * sm.inv_rms[n] * wscale<WT>(p.s_head, (size_t)(P - 1) * p.V + id) + b;
           }
         });
@@ -906,7 +949,11 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
         consumer_sync();
       }
     } else {
-      TopkRec* recs = p.topk + (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1);
+      // records of call row row0 + r; a tree call keeps every row's records in buffer 0
+      const bool tree = WIDE && p.draft_mode == MCD_DRAFT_TREE;
+      TopkRec* recs = p.topk + (tree ? 0 : (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1)) +
+                      (size_t)ci->row0 * (kMaxDraft + 1);
+      const float* lgt = p.logits + (size_t)ci->row0 * (kMaxDraft + 1) * p.V;
       const bool noisy = p.draft_mode == MCD_DRAFT_NOISY_TARGET;
       int pair = 0;
       for (int r = 0; r < n_rows; ++r) {
@@ -916,7 +963,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
         for (int j = 0; j <= kn; ++j, ++pair) {
           if (pair % p.n_cta != (int)blockIdx.x) continue;
           const int greedy = (j > 0 && p.draft_mode == MCD_DRAFT_GREEDY) ? 1 : 0;
-          block_topk(p.logits + ((size_t)r * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
+          block_topk(lgt + ((size_t)r * (kMaxDraft + 1) + j) * p.V, p.V, p.top_k, p.T, greedy, ts,
                      recs + r * (kMaxDraft + 1) + j);
           consumer_sync();
         }
@@ -1188,7 +1235,7 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
   const int a = st0.a, pos0 = st0.pos0, n_rows = st0.n_rows, round = st0.round;
   const unsigned sid = p.stream_ids[0], fid = p.frame_ids[0];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const TopkRec* cur = p.topk + (size_t)(call & 1) * kMaxCols * (kMaxDraft + 1);
+  const TopkRec* cur = p.topk;                       // every row's records, buffer 0
   __shared__ int t_emit[kMaxDraft + 1], t_path[kMaxDraft + 1], t_path_row[kMaxDraft + 1], t_res[4];
   __shared__ int t_next[kMaxDraft][kMaxTreeRank];
   if (warp == 0) {
@@ -1220,9 +1267,8 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
         }
       }
       if (kept >= 0) {
-        int kr = -1;
-        for (int r2 = 0; r2 < n_rows; ++r2)
-          if (ci->r_node[r2] == kept) kr = r2;
+        // rows are the first nodes in tree order: node i was fed at row i + 1 if it exists
+        const int kr = kept + 1 < n_rows ? kept + 1 : -1;
         if (lane == 0) {
           t_emit[n_emit] = kx;
           t_path[plen] = kept;
@@ -1291,7 +1337,7 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
       const bool isv = i >= per;
       const int k = isv ? i - per : i;
       const int d4 = k % D4, t = (k / D4) % n_mv, lg = k / (D4 * n_mv);   // lg = layer * NKV + kv head
-      float* base = (isv ? p.vcache : p.kcache) + (size_t)lg * kKVSlots * p.D;
+      float* base = (isv ? p.vcache : p.kcache) + (size_t)lg * p.kv_slots * p.D;
       const float4 v = __ldcg(reinterpret_cast<const float4*>(base + (size_t)(kMaxPos + t_path_row[t]) * p.D) + d4);
       reinterpret_cast<float4*>(base + (size_t)(a + 2 + t) * p.D)[d4] = v;
     }
@@ -1317,7 +1363,7 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
       if (codes_out) codes_out[a + t] = t_emit[t];
       st->emitted_last[t] = t_emit[t];
     }
-    const int calls = st0.calls + 1, heads = st0.heads_read + ci->phi[0] - ci->plo[0] + 1;
+    const int calls = st0.calls + 1, heads = st0.heads_read + ci->phi[0] - ci->plo[0] + 1;   // + the last pass
     const int kvr = st0.kv_rows + pos0 + n_rows, rf = st0.rows_fed + n_rows;
     const int drafted = st0.drafted + t_res[3], accepted = st0.accepted + plen;
     st->n_emit_last = n_emit;
@@ -1328,6 +1374,7 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
     st->n_rows = 1 + nv;
     st->top_pos = a_new + 1 + md;
     st->round = round + 1;
+    st->tpass = 0;
     st->first_head_row = 0;
     st->calls = calls;
     st->heads_read = heads;
@@ -1369,7 +1416,15 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
       tr->n_rows = n_rows;
       tr->pos0 = pos0;
       tr->n_drafts = t_res[3];
-      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = n < n_rows ? ci->r_id[n] : -1;
+      // code fed at call row n: the first call is one pass of plain rows; a tree call feeds
+      // c_a, then node n - 1's candidate
+      auto row_id = [&](int n) {
+        if (n >= n_rows) return -1;
+        if (pos0 == 0) return ci->r_id[n];
+        if (n == 0) return st0.codes[a];
+        return ci->tcand[p.tree_depth[n - 1] - 1][p.tree_rank[n - 1]];
+      };
+      for (int n = 0; n < kMaxRows; ++n) tr->input_ids[n] = row_id(n);
       for (int i = 0; i < kMaxRows; ++i) tr->drafts[i] = -1;
       tr->n_acc = plen;
       tr->n_emit = n_emit;
@@ -1378,10 +1433,11 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
       for (int j = 0; j < kMaxRows; ++j) tr->next_drafts[j] = j < n_next ? t_next[j][0] : -1;
       tr->draft_row = drow;
       tt->n_rows = n_rows;
-      for (int n = 0; n < kMaxCols; ++n) {
-        tt->row_node[n] = n < n_rows ? ci->r_node[n] : -1;
-        tt->row_id[n] = n < n_rows ? ci->r_id[n] : -1;
+      for (int n = 0; n < kMaxTreeRows; ++n) {
+        tt->row_node[n] = n >= n_rows ? -1 : pos0 == 0 ? ci->r_node[n] : n - 1;
+        tt->row_id[n] = row_id(n);
       }
+      tt->n_passes = (n_rows + kMaxCols - 1) / kMaxCols;
       tt->path_len = plen;
       for (int t = 0; t < kMaxDraft + 1; ++t) tt->path[t] = t < plen ? t_path[t] : -1;
       tt->draft_row = drow;
@@ -1390,10 +1446,11 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
         for (int r = 0; r < kMaxTreeRank; ++r)
           tt->next_cand[d][r] = (d < n_next && d < kMaxDraft && r < p.tree_m[d]) ? t_next[d][r] : -1;
     }
-    for (int idx = threadIdx.x; idx < kMaxCols * p.V; idx += kConsumerThreads) {
+    for (int idx = threadIdx.x; idx < kMaxTreeRows * p.V; idx += kConsumerThreads) {
       const int n = idx / p.V, v = idx - n * p.V;
-      if (n < n_rows && ci->r_pos[n] >= 1)
-        vall[((size_t)round * kMaxCols + n) * p.V + v] = __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
+      if (n < n_rows && (pos0 > 0 || n > 0))                  // the conditioning row reads no head
+        vall[((size_t)round * kMaxTreeRows + n) * p.V + v] =
+            __ldcg(p.logits + ((size_t)n * (kMaxDraft + 1)) * p.V + v);
       if (n < n_next)
         dlog[((size_t)round * kMaxRows + n) * p.V + v] =
             __ldcg(p.logits + ((size_t)drow * (kMaxDraft + 1) + n + 1) * p.V + v);
@@ -1401,6 +1458,21 @@ __device__ __noinline__ void accept_tree(const FrameParams& p, int call) {
   }
   consumer_sync();
   if (threadIdx.x == 0) red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+}
+
+// End of a tree call's pass that another pass follows (run by the CTA that finished top-k
+// last): its rows' records and K / V stay in place; the next slot runs the next pass.
+__device__ __noinline__ void tree_pass_step(const FrameParams& p, int call) {
+  Smem sm = smem_layout(mcd_dyn_smem);
+  const CallInfo* ci = sm.ci;
+  if (threadIdx.x == 0) {
+    DevState* st = p.st;
+    st->tpass = ci->st[0].tpass + 1;
+    st->heads_read = ci->st[0].heads_read + ci->phi[0] - ci->plo[0] + 1;
+    st->call = call + 1;
+    __threadfence();
+    red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+  }
 }
 
 // Draft step of noisy-target pass j (run by the CTA that finished top-k last): draw the
@@ -1496,26 +1568,50 @@ __device__ __forceinline__ bool read_call_state(Cons& c, int call, bool first) {
       mask &= mask - 1;
     }
     ci->n_heads = nh;
+    ci->row0 = 0;
+    ci->tree_more = 0;
+    ci->n_tg = 0;
     if (tree_rows) {
+      // the call's rows: c_a, then the nodes of depth <= min(n_d, P - 1 - a), a prefix of the
+      // breadth-first node list (node i at row i + 1); pass t feeds rows 32 t .. 32 t + 31
       const DevState& st = sts[0];
-      int row_of[kMaxTree];
-      int n = 1;
-      ci->r_pos[0] = st.pos0;
-      ci->r_id[0] = st.codes[st.a];
-      ci->r_node[0] = -1;
-      ci->r_anc[0] = 1u;
-      for (int i = 0; i < p.tree_n; ++i) {
-        const int d = p.tree_depth[i];
-        row_of[i] = -1;
-        if (d > st.n_d || st.a + d >= p.P) continue;
-        const int pa = p.tree_parent[i];
-        ci->r_pos[n] = st.pos0 + d;
-        ci->r_id[n] = ci->tcand[d - 1][p.tree_rank[i]];
-        ci->r_node[n] = (signed char)i;
-        ci->r_anc[n] = (pa < 0 ? 1u : ci->r_anc[row_of[pa]]) | (1u << n);
-        row_of[i] = n++;
+      int R = 1;
+      while (R <= p.tree_n && p.tree_depth[R - 1] <= st.n_d && st.a + p.tree_depth[R - 1] < p.P) ++R;
+      const int row0 = st.tpass * kMaxCols, Mp = max(0, min(R - row0, kMaxCols));
+      if (R != st.n_rows || Mp == 0) atomicCAS(p.err, 0, (int)MCD_ERR_STATE);   // the acceptance step counted otherwise
+      ci->row0 = row0;
+      ci->M = Mp;
+      ci->tree_more = row0 + Mp < R ? 1 : 0;
+      for (int n = 0; n < Mp; ++n) {
+        const int m = row0 + n;
+        if (m == 0) {
+          ci->r_pos[n] = st.pos0;
+          ci->r_id[n] = st.codes[st.a];
+          ci->r_node[n] = -1;
+        } else {
+          const int d = p.tree_depth[m - 1];
+          ci->r_pos[n] = st.pos0 + d;
+          ci->r_id[n] = ci->tcand[d - 1][p.tree_rank[m - 1]];
+          ci->r_node[n] = (signed char)(m - 1);
+        }
       }
-      if (n != ci->M) atomicCAS(p.err, 0, (int)MCD_ERR_STATE);   // the acceptance step counted otherwise
+      // attention groups: up to 8 consecutive rows whose keys (the committed prefix, row 0
+      // and the union of their ancestor-or-self sets) fit one task
+      int ng = 0, r = 0;
+      while (r < Mp) {
+        const int start = r;
+        unsigned long long U = 0ull;
+        while (r < Mp && r - start < 8) {
+          const int m = row0 + r;
+          const unsigned long long am = m > 0 ? p.tree_anc[m - 1] : 0ull;
+          if (r > start && st.pos0 + 1 + __popcll(U | am) > kTreeKeys) break;
+          U |= am;
+          ++r;
+        }
+        ci->tg[ng++] = (signed char)start;
+      }
+      ci->tg[ng] = (signed char)Mp;
+      ci->n_tg = ng;
     }
   }
   consumer_sync();
@@ -1594,6 +1690,8 @@ __global__ void __launch_bounds__(kThreads, 1) frame_kernel(const __grid_constan
       if (sm.flags[2]) {
         if (sm.ci->emu)
           emu_step(p, call);
+        else if (WIDE && p.draft_mode == MCD_DRAFT_TREE && sm.ci->tree_more)
+          tree_pass_step(p, call);
         else if (WIDE && p.draft_mode == MCD_DRAFT_TREE)
           accept_tree(p, call);
         else

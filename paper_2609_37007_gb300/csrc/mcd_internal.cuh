@@ -27,9 +27,9 @@ constexpr int kMaxBatchRows = 512;     // packed rows of one batched call
 constexpr int kMaxDraft = 7;         // K
 constexpr int kMaxTopK = 128;
 constexpr int kMaxPos = 32;          // KV positions kept per frame (cond, c0, c1..c14 used)
-constexpr int kKVSlots = 2 * kMaxPos; // cache entries per (layer, KV head): positions, then the
-                                      // current tree call's node rows (kMaxPos + row)
-constexpr int kMaxTree = 31;         // tree nodes (rows = 1 + nodes <= kMaxCols)
+constexpr int kMaxTree = 64;         // tree nodes (a tree call feeds 1 + nodes rows)
+constexpr int kMaxTreeRows = kMaxTree + 1;
+constexpr int kTreeKeys = 48;        // keys of one tree attention task (prefix + visible rows)
 constexpr int kMaxTreeRank = 8;      // candidates per drafted position
 constexpr int kMaxCalls = 16;        // verify calls per frame (15 positions, first call emits 1)
 constexpr int kMaxSlots = 128;       // passes per frame: verify calls + noisy-target drafting passes
@@ -78,6 +78,7 @@ struct DevState {
   int err;
   int round;           // verify round of the next pass (Philox round, trace index)
   int emu;             // 0: the next pass is a verify call; j >= 1: noisy-target pass j
+  int tpass;           // TREE mode: pass of the next call (rows 32 t .. 32 t + 31 of the call)
   int emu_n;           // drafts the noisy-target passes make for the next verify call
   int emu_in;          // code fed to the next noisy-target pass
   int top_pos;         // largest row position of the next pass
@@ -96,6 +97,7 @@ __device__ inline void init_stream_state(DevState* st, int c0) {
   st->q_row = 0;
   st->round = 0;
   st->emu = 0;
+  st->tpass = 0;
   st->emu_n = 0;
   st->emu_in = -1;
   st->top_pos = 1;
@@ -151,10 +153,10 @@ struct FrameParams {
   float* qkv;                  // [kMaxCols][qkv_dim]
   float* mbuf;                 // [kMaxCols][F]
   float* attn;                 // [kMaxCols][NH*D] attention outputs (batched calls)
-  float* logits;               // [kMaxCols][kMaxDraft+1][V]
-  float* kcache;               // [S][L][NKV][kKVSlots][D]
+  float* logits;               // [kMaxTreeRows][kMaxDraft+1][V] (rows of one call)
+  float* kcache;               // [S][L][NKV][kv_slots][D]
   float* vcache;
-  TopkRec* topk;               // [2][kMaxCols][kMaxDraft+1]
+  TopkRec* topk;               // [2][kMaxCols][kMaxDraft+1]; a tree call: [kMaxTreeRows][kMaxDraft+1]
   TopkRec* draftq;             // [kMaxDraft] pending drafts' q
   DevState* st;                // [S]
   unsigned* ctr;               // [kMaxCalls][ctr_stride]
@@ -170,6 +172,8 @@ struct FrameParams {
   int* codes_out;              // [S][n_pos]
   mcd_frame_stats* stats;      // [S]
   long long kv_stride;         // floats between streams' KV caches
+  int kv_slots;                // cache entries per (layer, KV head): positions 0..kMaxPos-1, then
+                               // (TREE mode) the current tree call's rows at kMaxPos + row
   long long trace_stride;      // bytes between streams' trace blocks
   float* logits_out;           // stepwise: verify logits of the single call
   int* emitted_out;
@@ -180,6 +184,7 @@ struct FrameParams {
   int tree_n, tree_maxd;
   signed char tree_parent[kMaxTree], tree_rank[kMaxTree], tree_depth[kMaxTree];
   int tree_m[kMaxDraft];       // candidates needed per depth
+  unsigned long long tree_anc[kMaxTree];   // node i: bit j set iff node j is i or an ancestor of i
   int* tree_cand;              // [kMaxDraft][kMaxTreeRank] candidates of the next call
   int n_cta;
   unsigned long long wait_ns;  // bound of every device-side wait

@@ -37,6 +37,10 @@ struct CallInfo {
   unsigned r_anc[kMaxCols];
   signed char r_node[kMaxCols];                  // tree node of the row (-1: none)
   int tcand[kMaxDraft][kMaxTreeRank];            // tree call: candidates of its nodes
+  // tree call: the pass feeds rows row0 .. row0 + M - 1 of the call (tree_more: a later pass
+  // follows); attention groups g = tg[g] .. tg[g + 1] - 1 (pass rows), n_tg of them
+  int row0, tree_more, n_tg;
+  signed char tg[kMaxCols + 1];
   // per stream (index = stream): its state and the derived packing
   DevState st[kMaxStreams];
   int act[kMaxStreams];        // active streams in packing order

@@ -56,10 +56,13 @@ CALL_TRACE_DTYPE = np.dtype([("a", "<i4"), ("n_rows", "<i4"), ("pos0", "<i4"), (
                              ("next_drafts", "<i4", 8), ("draft_row", "<i4"), ("reserved", "<i4", 24)])
 assert CALL_TRACE_DTYPE.itemsize == 256
 
-TREE_TRACE_DTYPE = np.dtype([("n_rows", "<i4"), ("row_node", "<i4", 32), ("row_id", "<i4", 32),
-                             ("path_len", "<i4"), ("path", "<i4", 8), ("draft_row", "<i4"), ("n_next", "<i4"),
-                             ("next_cand", "<i4", (8, 8)), ("reserved", "<i4", 20)])
-assert TREE_TRACE_DTYPE.itemsize == 640
+MAX_TREE_NODES = 64            # MCD_MAX_TREE_NODES
+MAX_TREE_ROWS = 65             # MCD_MAX_TREE_ROWS
+TREE_TRACE_DTYPE = np.dtype([("n_rows", "<i4"), ("row_node", "<i4", MAX_TREE_ROWS),
+                             ("row_id", "<i4", MAX_TREE_ROWS), ("path_len", "<i4"), ("path", "<i4", 8),
+                             ("draft_row", "<i4"), ("n_next", "<i4"), ("next_cand", "<i4", (8, 8)),
+                             ("n_passes", "<i4"), ("reserved", "<i4", 17)])
+assert TREE_TRACE_DTYPE.itemsize == 896
 
 
 class MCDError(RuntimeError):
@@ -305,11 +308,12 @@ def mcd_set_tree(ctx, parent, rank):
 
 
 def parse_tree_trace(buf: np.ndarray, vocab: int):
-    """TREE mode: (tree records [16], verify logits of every row [16 calls][32 rows][vocab])."""
+    """TREE mode: (tree records [16], verify logits of every row [16 calls][65 rows][vocab])."""
     start = CALL_TRACE_DTYPE.itemsize * MAX_CALLS + 2 * MAX_CALLS * MAX_ROWS * vocab * 4
     n = TREE_TRACE_DTYPE.itemsize * MAX_CALLS
     recs = buf[start:start + n].view(TREE_TRACE_DTYPE)
-    vall = buf[start + n:start + n + MAX_CALLS * 32 * vocab * 4].view(np.float32).reshape(MAX_CALLS, 32, vocab)
+    nv = MAX_CALLS * MAX_TREE_ROWS * vocab
+    vall = buf[start + n:start + n + nv * 4].view(np.float32).reshape(MAX_CALLS, MAX_TREE_ROWS, vocab)
     return recs, vall
 
 

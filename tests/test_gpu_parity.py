@@ -392,14 +392,25 @@ def _trees():
     from oracle.tree import Tree, grow_tree
     fig2 = Tree(parent=[-1, -1, 0, 0, 1, 2, 4, 4], rank=[0, 1, 0, 1, 0, 0, 0, 1])
     big = grow_tree([[0.5, 0.3, 0.2, 0.1, 0.05], [0.4, 0.25, 0.1], [0.3, 0.2]], 31)
+    # the sweep's larger sizes (Fig. 4: N = 32, 48, 64), grown for rank-decreasing statistics
+    # of 8 candidates at each of 3 depths
+    acc = [[0.6 / (r + 1) ** 0.5 for r in range(8)] for _ in range(3)]
     return {"chain3": Tree.chain(3), "fig2": fig2, "wide": Tree(parent=[-1, -1, -1, -1], rank=[0, 1, 2, 3]),
-            "big31": big}
+            "big31": big, "grown32": grow_tree(acc, 32), "grown48": grow_tree(acc, 48),
+            "grown64": grow_tree(acc, 64)}
 
 
-@pytest.mark.parametrize("name", ["chain3", "fig2", "wide", "big31"])
+def test_grown_trees_need_two_and_three_passes():
+    t = _trees()
+    assert [t[k].n for k in ("big31", "grown32", "grown48", "grown64")] == [31, 32, 48, 64]
+    assert max(t["grown64"].depth) == 3 and max(t["grown64"].rank) == 7
+
+
+@pytest.mark.parametrize("name", ["chain3", "fig2", "wide", "big31", "grown32", "grown48", "grown64"])
 def test_tree_mode_trace_parity_tiny(name):
     """TREE mode: every call's rows, logits (1e-5), walk, kept path, codes and next candidates
-    against the oracle; the 31-node tree packs 32 rows per call."""
+    against the oracle; the 31-node tree packs 32 rows per call, the 32-, 48- and 64-node
+    trees run 33, 49 and 65 rows in two and three passes."""
     tree = _trees()[name]
     cfg = TINY.replace(draft_mode=3, draft_len=3, n_pos=8)
     env = Env(cfg)
@@ -412,6 +423,11 @@ def test_tree_mode_trace_parity_tiny(name):
         worst = max(worst, check_tree_trace_against_oracle(cfg, env.model, fr, 1, f, tr, codes, int(st[0]), tree,
                                                            logit_tol=1e-5))
     print(name, "max |dlogit|", worst)
+    if tree.n > 31:
+        trecs = mcd.parse_tree_trace(np.asarray(tr, dtype=np.uint8), cfg.vocab)[0]
+        rows = [int(r["n_rows"]) for r in trecs[1:int(st[0])]]
+        assert max(rows) == 1 + tree.n, rows                  # the full tree was fed at least once
+        assert all(int(r["n_passes"]) == (n + 31) // 32 for r, n in zip(trecs[1:], rows))
     env.dec.close()
 
 
@@ -428,12 +444,15 @@ def test_chain_tree_equals_greedy_drafts_on_gpu():
     greedy_env.dec.close()
 
 
-def test_tree_mode_full_size():
-    tree = _trees()["fig2"]
+@pytest.mark.parametrize("name,frames", [("fig2", (0, 1)), ("grown64", (2,))])
+def test_tree_mode_full_size(name, frames):
+    """The full-size model (bf16 weights, logits within 2e-2): the Fig. 2 tree and the 64-node
+    tree (65 rows in three passes)."""
+    tree = _trees()[name]
     cfg = MCD.replace(draft_mode=3, draft_len=3)
     env = Env(cfg)
     mcd.mcd_set_tree(env.dec.ctx, tree.parent, tree.rank)
-    for f in (0, 1):
+    for f in frames:
         fr = make_frame(cfg, f)
         codes, st, tr = env.decode(fr, f, trace=True)
         assert st[4] == 0 and st[1] == cfg.n_pos
