@@ -691,7 +691,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
   const int n_rows = ci->M;                 // packed rows of every stream in the call
   const unsigned N = (unsigned)p.n_cta;
   const float* x = p.x;
-  auto from_x = [&](int n, int k) { return ld_global2(x + (size_t)n * H + k); };
+  auto from_x = [&](int n, int k, auto w) { return ld_global_v<decltype(w)::value>(x + (size_t)n * H + k); };
 
   auto no_key = [](int) { return 0; };
   auto no_prep = [](int, int, int) {};
@@ -705,11 +705,10 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
       consumer_sync();                     // the gain is in shared memory
       prep_operand<WT, WIDE>(
           c, n_rows, H, 0, H, sm.vec, true,
-          [&](int n, int k) {
+          [&](int n, int k, auto w) {
+            constexpr int W = decltype(w)::value;
             const uint8_t* src = ci->r_src[n];
-            if (ci->r_f32[n]) return __ldg(reinterpret_cast<const float2*>(src) + (k >> 1));
-            const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(src) + (k >> 1));
-            return make_float2(bf16_bits_to_f32(w & 0xFFFFu), bf16_bits_to_f32(w >> 16));
+            return ci->r_f32[n] ? ldg_f32_v<W>(src, k) : ldg_bf16_v<W>(src, k);
           },
           blockIdx.x == 0 ? p.x : nullptr);
     } else {
@@ -770,7 +769,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
             if (sm.flags[3] != h) {
               const float* src = p.attn + h * D;
               prep_operand<WT, WIDE>(c, n_rows, D, 0, D, nullptr, false,
-                                     [&](int n, int k) { return ld_global2(src + (size_t)n * p.NH * D + k); });
+                                     [&](int n, int k, auto w) { return ld_global_v<decltype(w)::value>(src + (size_t)n * p.NH * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
@@ -795,7 +794,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
               attention_head(c, l, h, writer);
               c.op = reinterpret_cast<uint8_t*>(sm.act) + kWoOperandOff;
               prep_operand<WT, WIDE>(c, n_rows, D, 0, D, nullptr, false,
-                               [&](int n, int k) { return ld_shared2(sm.act + n * D + k); });
+                               [&](int n, int k, auto w) { return ld_shared_v<decltype(w)::value>(sm.act + n * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
@@ -848,7 +847,7 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
             if (sm.flags[3] != kc) {
               const float* m = p.mbuf + (size_t)kc * Kc;
               prep_operand<WT, WIDE>(c, n_rows, Kc, 0, Kc, nullptr, false,
-                               [&](int n, int k) { return ld_global2(m + (size_t)n * F + k); });
+                               [&](int n, int k, auto w) { return ld_global_v<decltype(w)::value>(m + (size_t)n * F + k); });
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
           },

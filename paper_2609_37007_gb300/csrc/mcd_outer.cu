@@ -402,32 +402,22 @@ __device__ void run_outer(Cons& c, const OuterStep& o) {
     }
     ids[t] = id;
   }
-  auto row2 = [&](const uint8_t* row, int k) -> float2 {
-    if (WT == MCD_WEIGHT_BF16) {
-      const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 1));
-      return make_float2(bf16_bits_to_f32(w & 0xFFFFu), bf16_bits_to_f32(w >> 16));
-    }
-    return __ldg(reinterpret_cast<const float2*>(row) + (k >> 1));
-  };
   // layer-0 row n: a prompt row, or the frame input text + E_c0(c0) + sum_j E_j(c_j)
-  auto ld0 = [&](int n, int k) -> float2 {
-    if (o.text_ids) return row2(o.text_table + (size_t)ids[n] * rb, k);
-    float2 s = make_float2(0.f, 0.f);
-    if (ids[o.P + 1] >= 0) s = row2(o.text_table + (size_t)ids[o.P + 1] * rb, k);
-    float2 v = row2(o.c0_table + (size_t)ids[0] * rb, k);
-    s.x += v.x;
-    s.y += v.y;
-    for (int j = 1; j < o.P; ++j) {
-      v = row2(o.code_tables + (long long)j * o.code_stride + (size_t)ids[j] * rb, k);
-      s.x += v.x;
-      s.y += v.y;
-    }
-    v = row2(o.last_table + (size_t)ids[o.P] * rb, k);
-    s.x += v.x;
-    s.y += v.y;
+  auto ld0 = [&](int n, int k, auto w) {
+    constexpr int W = decltype(w)::value;
+    auto row_v = [&](const uint8_t* row) {
+      if constexpr (WT == MCD_WEIGHT_BF16) return ldg_bf16_v<W>(row, k);
+      else return ldg_f32_v<W>(row, k);
+    };
+    if (o.text_ids) return row_v(o.text_table + (size_t)ids[n] * rb);
+    vecf<W> s{};
+    if (ids[o.P + 1] >= 0) s = row_v(o.text_table + (size_t)ids[o.P + 1] * rb);
+    add_v<W>(s, row_v(o.c0_table + (size_t)ids[0] * rb));
+    for (int j = 1; j < o.P; ++j) add_v<W>(s, row_v(o.code_tables + (long long)j * o.code_stride + (size_t)ids[j] * rb));
+    add_v<W>(s, row_v(o.last_table + (size_t)ids[o.P] * rb));
     return s;
   };
-  auto from_x = [&](int n, int k) { return ld_global2(p.x + (size_t)n * H + k); };
+  auto from_x = [&](int n, int k, auto w) { return ld_global_v<decltype(w)::value>(p.x + (size_t)n * H + k); };
   auto no_key = [](int) { return 0; };
   auto no_prep = [](int, int, int) {};
   const int n_blocks = (o.pos0 + nr + kKeyBlock - 1) / kKeyBlock;
@@ -472,7 +462,7 @@ __device__ void run_outer(Cons& c, const OuterStep& o) {
             if (sm.flags[3] != h) {
               outer_merge(c, o, h, ao);
               prep_operand<WT, WIDE>(c, nr, D, 0, D, nullptr, false,
-                                     [&](int n, int k) { return ld_shared2(ao + n * D + k); });
+                                     [&](int n, int k, auto w) { return ld_shared_v<decltype(w)::value>(ao + n * D + k); });
               if (threadIdx.x == 0) sm.flags[3] = h;
             }
           },
@@ -517,7 +507,7 @@ __device__ void run_outer(Cons& c, const OuterStep& o) {
             if (sm.flags[3] != kc) {
               const float* m = p.mbuf + (size_t)kc * Kc;
               prep_operand<WT, WIDE>(c, nr, Kc, 0, Kc, nullptr, false,
-                                     [&](int n, int k) { return ld_global2(m + (size_t)n * F + k); });
+                                     [&](int n, int k, auto w) { return ld_global_v<decltype(w)::value>(m + (size_t)n * F + k); });
               if (threadIdx.x == 0) sm.flags[3] = kc;
             }
           },
@@ -535,7 +525,7 @@ __device__ void run_outer(Cons& c, const OuterStep& o) {
   g2s_vec(sm.vec, p.final_norm, H);
   if (!cons_wait(c, ctr + ctr_stage(L - 1, 3), N)) return;
   const float* xl = p.x + (size_t)(nr - 1) * H;
-  prep_operand<WT, WIDE>(c, 1, H, 0, H, sm.vec, true, [&](int, int k) { return ld_global2(xl + k); });
+  prep_operand<WT, WIDE>(c, 1, H, 0, H, sm.vec, true, [&](int, int k, auto w) { return ld_global_v<decltype(w)::value>(xl + k); });
   {
     const MatGeom& g = p.g[MAT_HEAD];
     run_stage<WT, WIDE>(c, 0, 4 * L, g.n_units, H, 1, no_key, no_prep,

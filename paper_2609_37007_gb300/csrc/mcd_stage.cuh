@@ -15,9 +15,15 @@
 // columns per n-tile as B).  RMSNorm is applied as a per-column scale in the epilogue:
 // W (x . g) / rms.  Every wait is bounded.
 #pragma once
+#include <type_traits>
 #include "mcd_internal.cuh"
 
 namespace mcd {
+
+// Vector width tags of the operand loaders: ld(n, k, Vec2{}) -> float2, Vec4{} -> float4.
+using Vec2 = std::integral_constant<int, 2>;
+using Vec4 = std::integral_constant<int, 4>;
+template <int W> using vecf = typename std::conditional<W == 4, float4, float2>::type;
 
 
 // Snapshot of one call: the packed rows and every stream's state.
@@ -224,8 +230,8 @@ __device__ __forceinline__ void cons_signal(Cons& c, unsigned* ctr, int call, in
   timeline_max(c, call, slot + 1);
 }
 
-// Operand geometry of a call with ncols packed columns: ncp = 2^ceil(log2 ncols) columns
-// are written (columns >= ncols as zeros); NT = ncp / 8 n-tiles (at least 1).  Up to 16
+// Operand geometry of a call with ncols packed columns: ncp = 2^ceil(log2 ncols) columns,
+// NT = ncp / 8 n-tiles (at least 1).  Up to 16
 // columns the activations are a bf16 hi + lo pair (16 B per fragment entry, about 16
 // mantissa bits); beyond that a single bf16 (8 B per entry).
 __device__ __forceinline__ int col_log2(int ncols) {
@@ -234,18 +240,21 @@ __device__ __forceinline__ int col_log2(int ncols) {
 __device__ __forceinline__ int n_tiles(int ncols) { return max(1, (1 << col_log2(ncols)) >> 3); }
 __device__ __forceinline__ bool hilo_operand(int ncols) { return ncols <= 16; }
 
-// Activation operand in one pass.  `ld(n, k)` returns elements (k, k+1) of column n from
-// global or shared memory; `gain` (shared, may be null) multiplies them per input index;
-// with want_ss the per-column 1/rms of the raw values lands in inv_rms; store_raw (may be
-// null) receives the raw values as fp32 rows [ncols][ldk].  bf16 weights get B fragments of
-// mma.m16n8k16: entry ((kt0 + kt) * NT + nt, lane) holds column nt*8 + lane/4, inputs
-// kt*16 + 2(lane%4) + {0,1,8,9}; fp32 weights get fp32 rows [ncols][ldk] from column kt0*16.
-// Only the first ncp columns are written: an mma output column depends only on its own B
-// column and columns >= ncols are never read back.  Every load of a batch is issued before
-// any of its stores (one memory round trip per 1024 entries).
+// Activation operand in one pass.  `ld(n, k, VecW{})` returns elements k .. k+W-1 of column
+// n (W = 2 or 4, k a multiple of W) from global or shared memory; `gain` (shared, may be
+// null) multiplies them per input index; with want_ss the per-column 1/rms of the raw values
+// lands in inv_rms; store_raw (may be null) receives the raw values as fp32 rows
+// [ncols][ldk].  bf16 weights get B fragments of mma.m16n8k16: entry ((kt0 + kt) * NT + nt,
+// lane) holds column nt*8 + lane/4, inputs kt*16 + 2(lane%4) + {0,1,8,9}; fp32 weights get
+// fp32 rows [ncols][ldk] from column kt0*16.
+//
+// Narrow form (up to 8 columns): thread (column, lane % 4) loads its two input pairs of a
+// k-tile as 8-byte pieces and writes the whole entry; ncp = 2^ceil(log2 ncols) columns are
+// written (columns >= ncols as zeros).  Every load of a batch is issued before any of its
+// stores (one memory round trip per 1024 entries).
 template <int WT, bool WIDE, class Ld>
-__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
-                                             bool want_ss, Ld ld, float* store_raw = nullptr) {
+__device__ __forceinline__ void prep_operand_pairs(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
+                                                   bool want_ss, Ld ld, float* store_raw) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int lg = col_log2(ncols), NT = WIDE ? n_tiles(ncols) : 1;
   const bool hilo = WIDE ? hilo_operand(ncols) : true;
@@ -263,8 +272,8 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
       vb[e] = make_float2(0.f, 0.f);
       if (i < items && live) {
         const int k0 = ((i >> (2 + lg)) << 4) + 2 * t;
-        va[e] = ld(n, k0);
-        vb[e] = ld(n, k0 + 8);
+        va[e] = ld(n, k0, Vec2{});
+        vb[e] = ld(n, k0 + 8, Vec2{});
       }
     }
 #pragma unroll
@@ -325,6 +334,118 @@ __device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int k
     // no barrier: inv_rms is read only by epilogues, which follow the chunk barrier of the
     // stage, and part / inv_rms are rewritten only after the stage's closing barrier
   }
+}
+
+// Wide form (up to 32 columns): only the ncols live columns are written (an mma output
+// column depends only on its own B column and columns >= ncols are never read back).
+// Threads work in quads: quad j serves column j % ncols and k-tiles j / ncols, + R, ...
+// (R = 64 / ncols quads per column), each thread one 16-byte piece (4 inputs) of a k-tile,
+// whose two input pairs it writes as half entries.  Every load of a batch of kE pieces is
+// issued before any of its stores.
+template <int WT, bool WIDE, class Ld>
+__device__ __forceinline__ void prep_operand_quads(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
+                                                   bool want_ss, Ld ld, float* store_raw) {
+  constexpr int kQuads = kConsumerThreads / 4;
+  const int tid = threadIdx.x, q = tid & 3, quad = tid >> 2;
+  const int NT = WIDE ? n_tiles(ncols) : 1;
+  const bool hilo = WIDE ? hilo_operand(ncols) : true;
+  const int R = kQuads / ncols, n = quad % ncols, r = quad / ncols;
+  const bool live = r < R;
+  const int nkt = Kdim >> 4;
+  constexpr int kE = 8;
+  float ss = 0.f;
+  if (live) {
+    for (int kb = r; kb < nkt; kb += kE * R) {
+      float4 v[kE];
+#pragma unroll
+      for (int e = 0; e < kE; ++e) {
+        const int kt = kb + e * R;
+        v[e] = kt < nkt ? ld(n, (kt << 4) + 4 * q, Vec4{}) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int e = 0; e < kE; ++e) {
+        const int kt = kb + e * R;
+        if (kt >= nkt) break;
+        const int k0 = (kt << 4) + 4 * q;
+        float4 x = v[e];
+        ss += (x.x * x.x + x.y * x.y) + (x.z * x.z + x.w * x.w);
+        if (store_raw) *reinterpret_cast<float4*>(store_raw + (size_t)n * ldk + k0) = x;
+        if (gain) {
+          const float4 g = *reinterpret_cast<const float4*>(gain + k0);
+          x.x *= g.x;
+          x.y *= g.y;
+          x.z *= g.z;
+          x.w *= g.w;
+        }
+        if (WT != MCD_WEIGHT_F32) {
+          // inputs 4q, 4q+1 -> lane t = 2(q&1), 4q+2, 4q+3 -> t + 1; half (q >> 1) of the entry
+          const int entry = ((kt0 + kt) * NT + (n >> 3)) * 32 + 4 * (n & 7) + 2 * (q & 1), half = q >> 1;
+          const uint32_t h0 = pack_bf16x2(x.x, x.y), h1 = pack_bf16x2(x.z, x.w);
+          if (hilo) {
+            uint32_t* e4 = reinterpret_cast<uint32_t*>(c.op) + 4 * entry + half;
+            e4[0] = h0;
+            e4[4] = h1;
+            e4[2] = pack_bf16x2(x.x - bf16_lo_f32(h0), x.y - bf16_hi_f32(h0));
+            e4[6] = pack_bf16x2(x.z - bf16_lo_f32(h1), x.w - bf16_hi_f32(h1));
+          } else {
+            uint32_t* e2 = reinterpret_cast<uint32_t*>(c.op) + 2 * entry + half;
+            e2[0] = h0;
+            e2[2] = h1;
+          }
+        } else {
+          *reinterpret_cast<float4*>(reinterpret_cast<float*>(c.op) + n * ldk + kt0 * 16 + k0) = x;
+        }
+      }
+    }
+  }
+  // column sums in a fixed order: the quad's four lanes, then (ncols dividing 8) the warp's
+  // quads of the column and the 8 warps, else every quad of the column
+  const bool per_warp = (8 % ncols) == 0;
+  if (want_ss) {
+    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 1);
+    ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 2);
+    if (per_warp) {
+#pragma unroll
+      for (int off = 16; off >= 4; off >>= 1)
+        if (off >= 4 * ncols) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+      if ((tid & 31) < 4 * ncols && q == 0) c.sm.part[(tid >> 5) * 8 + quad % 8] = ss;
+    } else if (q == 0) {
+      c.sm.part[quad] = ss;                    // quad sums (0 for idle quads)
+    }
+  }
+  consumer_sync();
+  if (want_ss && tid < ncols) {
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    if (per_warp) {
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; w += 4) {
+        s0 += c.sm.part[w * 8 + tid];
+        s1 += c.sm.part[(w + 1) * 8 + tid];
+        s2 += c.sm.part[(w + 2) * 8 + tid];
+        s3 += c.sm.part[(w + 3) * 8 + tid];
+      }
+    } else {
+      for (int j = 0; j < R; j += 4) {
+        s0 += c.sm.part[j * ncols + tid];
+        if (j + 1 < R) s1 += c.sm.part[(j + 1) * ncols + tid];
+        if (j + 2 < R) s2 += c.sm.part[(j + 2) * ncols + tid];
+        if (j + 3 < R) s3 += c.sm.part[(j + 3) * ncols + tid];
+      }
+    }
+    const float s = (s0 + s1) + (s2 + s3);
+    c.sm.inv_rms[tid] = rsqrtf(__fmul_rn(s, __frcp_rn((float)Kdim)) + c.p.eps);
+    // no barrier: inv_rms is read only by epilogues, which follow the chunk barrier of the
+    // stage, and part / inv_rms are rewritten only after the stage's closing barrier
+  }
+}
+
+template <int WT, bool WIDE, class Ld>
+__device__ __forceinline__ void prep_operand(Cons& c, int ncols, int Kdim, int kt0, int ldk, const float* gain,
+                                             bool want_ss, Ld ld, float* store_raw = nullptr) {
+  if constexpr (WIDE)
+    prep_operand_quads<WT, WIDE>(c, ncols, Kdim, kt0, ldk, gain, want_ss, ld, store_raw);
+  else
+    prep_operand_pairs<WT, WIDE>(c, ncols, Kdim, kt0, ldk, gain, want_ss, ld, store_raw);
 }
 
 // Warp roles in a unit: m-tile mi of Mu, n-tile group gn of Gn (ntpw n-tiles each) and
@@ -580,7 +701,33 @@ __device__ __forceinline__ void g2s_vec(float* dst, const float* src, int n) {
     reinterpret_cast<float4*>(dst)[i] = __ldg(reinterpret_cast<const float4*>(src) + i);
 }
 
-__device__ __forceinline__ float2 ld_global2(const float* q) { return __ldcg(reinterpret_cast<const float2*>(q)); }
-__device__ __forceinline__ float2 ld_shared2(const float* q) { return *reinterpret_cast<const float2*>(q); }
+template <int W> __device__ __forceinline__ vecf<W> ld_global_v(const float* q) {
+  return __ldcg(reinterpret_cast<const vecf<W>*>(q));
+}
+template <int W> __device__ __forceinline__ vecf<W> ld_shared_v(const float* q) {
+  return *reinterpret_cast<const vecf<W>*>(q);
+}
+// elements k .. k+W-1 of a read-only row of fp32 or bf16 values (k a multiple of W)
+template <int W> __device__ __forceinline__ vecf<W> ldg_f32_v(const uint8_t* row, int k) {
+  return __ldg(reinterpret_cast<const vecf<W>*>(row) + k / W);
+}
+template <int W> __device__ __forceinline__ vecf<W> ldg_bf16_v(const uint8_t* row, int k) {
+  if constexpr (W == 4) {
+    const uint2 w = __ldg(reinterpret_cast<const uint2*>(row) + (k >> 2));
+    return make_float4(bf16_bits_to_f32(w.x & 0xFFFFu), bf16_bits_to_f32(w.x >> 16), bf16_bits_to_f32(w.y & 0xFFFFu),
+                       bf16_bits_to_f32(w.y >> 16));
+  } else {
+    const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 1));
+    return make_float2(bf16_bits_to_f32(w & 0xFFFFu), bf16_bits_to_f32(w >> 16));
+  }
+}
+template <int W> __device__ __forceinline__ void add_v(vecf<W>& a, const vecf<W>& b) {
+  a.x += b.x;
+  a.y += b.y;
+  if constexpr (W == 4) {
+    a.z += b.z;
+    a.w += b.w;
+  }
+}
 
 }  // namespace mcd
