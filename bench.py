@@ -458,6 +458,77 @@ def run_timeline(args, weights):
     print(json.dumps(line), flush=True)
 
 
+def run_tc_gemm(args):
+    """The stand-alone tensor-core product of the batched path (tcgen05, bf16 operands, fp32
+    accumulation in tensor memory) at its gate/up shape: M = 6144 weight rows, N = 512 packed
+    rows (128 streams x 4), K = 1024.  Operands are tiled once (mcd_tc_tile); the product
+    alone (mcd_tc_gemm_tiled) is timed with CUDA events on its stream: back to back with the
+    13.6 MB of operands resident in L2, and one launch at a time after a 256 MB L2 flush.
+    One JSON line per tile width."""
+    import torch
+    from paper_2609_37007_gb300 import build as _build
+    from paper_2609_37007_gb300 import mcd
+    _build.build()
+    dev = torch.device("cuda", 0)
+    st = torch.cuda.current_stream(dev)
+    M, N, K = 6144, 512, 1024
+    g = torch.Generator(device=dev).manual_seed(11)
+    A = (0.02 * torch.randn(M, K, generator=g, device=dev)).to(torch.bfloat16)
+    B = torch.randn(N, K, generator=g, device=dev).to(torch.bfloat16)
+
+    def aligned(nbytes):
+        t = torch.empty(nbytes + 1024, dtype=torch.uint8, device=dev)
+        return t[(-t.data_ptr()) % 1024:][:nbytes]
+    ta, tb = aligned(M * K * 2), aligned(N * K * 2)
+    mcd.mcd_tc_tile(M, K, A.view(torch.int16), ta, st)
+    mcd.mcd_tc_tile(N, K, B.view(torch.int16), tb, st)
+    Y = torch.empty((N, M), dtype=torch.float32, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    ref = (B.double() @ A.double().T).float()
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peak, kind = float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        peak, kind = 1900.0, "fallback"
+    flops = 2.0 * M * N * K
+    clocks = Clocks(0)
+    for bn in (128, 256, 0):
+        for _ in range(20):
+            mcd.mcd_tc_gemm_tiled(M, N, K, bn, ta, tb, Y, err, st)
+        torch.cuda.synchronize(dev)
+        rel = float((Y - ref).abs().max() / ref.abs().max())
+        clocks.start()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n_warm = 200
+        e0.record(st)
+        for _ in range(n_warm):
+            mcd.mcd_tc_gemm_tiled(M, N, K, bn, ta, tb, Y, err, st)
+        e1.record(st)
+        torch.cuda.synchronize(dev)
+        us_warm = e0.elapsed_time(e1) * 1e3 / n_warm
+        cold = []
+        for _ in range(50):
+            flush.fill_(1)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(st)
+            mcd.mcd_tc_gemm_tiled(M, N, K, bn, ta, tb, Y, err, st)
+            b.record(st)
+            torch.cuda.synchronize(dev)
+            cold.append(a.elapsed_time(b) * 1e3)
+        clk = clocks.stop()
+        assert int(err.item()) == 0
+        us_cold = float(np.median(cold))
+        tile = ("one 128 x %d tile per CTA" % bn) if bn else "one tile per CTA over all SMs (128 x 176 / 160)"
+        print(json.dumps({"tc_gemm": "tcgen05 bf16 product, " + tile, "bn": bn, "M": M, "N": N, "K": K,
+                          "us_l2_resident": us_warm, "tflops_l2_resident": flops / us_warm / 1e6,
+                          "us_after_l2_flush": us_cold, "tflops_after_l2_flush": flops / us_cold / 1e6,
+                          "peak_tflops": peak, "peak_kind": kind,
+                          "frac_l2_resident": flops / us_warm / 1e6 / peak,
+                          "frac_after_l2_flush": flops / us_cold / 1e6 / peak,
+                          "max_rel_err_vs_fp64": rel, "clocks": clk}), flush=True)
+
+
 PIPE_METRIC = "sustained frames/s of the full frame pipeline"
 PIPE_UNIT = "frames/s"
 PIPE_WORKLOAD = ("CodeDecoder bf16, 28 layers, hidden 1024, 16q/8kv x 128, SwiGLU 3072, c0 vocab 3072, text vocab "
@@ -648,11 +719,15 @@ def main():
     ap.add_argument("--pipeline", action="store_true",
                     help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
     ap.add_argument("--utterances", type=int, default=2)
+    ap.add_argument("--tc-gemm", action="store_true",
+                    help="time the stand-alone tensor-core product (6144 x 512 x 1024) instead of the bench line")
     ap.add_argument("--timeline", type=int, default=0,
                     help="print the frame kernel's per-stage timeline over this many frames instead of the bench line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
+    if args.tc_gemm:
+        return run_tc_gemm(args)
     from paper_2609_37007_gb300.synth import MCD, WEIGHT_BF16, WEIGHT_INT8, make_frames, make_weights
     cfg = MCD.replace(weight_dtype=WEIGHT_INT8) if args.w8a16 else MCD
     weights = make_weights(cfg)

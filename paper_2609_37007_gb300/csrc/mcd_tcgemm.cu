@@ -2,6 +2,8 @@
 // matrices and the stand-alone product behind mcd_tc_gemm (include/mcd_tc.h).
 #include <cuda_runtime.h>
 
+#include <algorithm>
+
 #include "mcd_host.cuh"
 #include "mcd_tcgemm.cuh"
 #include "../../include/mcd_tc.h"
@@ -19,8 +21,10 @@ __global__ void sw128_tile_kernel(const uint16_t* __restrict__ src, int R, int K
   }
 }
 
+// Stand-alone product: eight warps (two per TMEM lane quarter share the epilogue's columns).
+constexpr int kStoreThreads = 256;
 template <int BN>
-__global__ void __launch_bounds__(kThreads, 1) gemm_store_kernel(const GemmArgs g, float* __restrict__ Y) {
+__global__ void __launch_bounds__(kStoreThreads, 1) gemm_store_kernel(const GemmArgs g, float* __restrict__ Y) {
   gemm_tile<BN, false, false>(g, [&](int m, int n, float v, float) { Y[(size_t)n * g.M + m] = v; });
 }
 
@@ -29,8 +33,21 @@ static cudaError_t launch_store(const GemmArgs& g, float* Y, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(gemm_store_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Layout<BN>::kSmemBytes);
   if (e != cudaSuccess) return e;
-  gemm_store_kernel<BN><<<dim3(g.N / BN, g.M / kBM), kThreads, Layout<BN>::kSmemBytes, st>>>(g, Y);
+  const int pitch = g.bn ? g.bn : BN;
+  gemm_store_kernel<BN><<<dim3((g.N + pitch - 1) / pitch, g.M / kBM), kStoreThreads, Layout<BN>::kSmemBytes, st>>>(g, Y);
   return cudaGetLastError();
+}
+
+// Tile pitch over N that fills the GPU with one tile per CTA: T = SMs / (M / 128) tiles across
+// N (at least ceil(N / 256)), each a multiple of 16 columns.
+static int auto_pitch(int M, int N) {
+  int dev = 0, n_sm = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+  const int n_mt = M / kBM, units = N / 16;
+  int T = std::max(1, n_sm / std::max(1, n_mt));
+  T = std::max(T, (N + 255) / 256);
+  T = std::min(T, units);
+  return (units + T - 1) / T * 16;
 }
 
 }  // namespace tc
@@ -41,7 +58,8 @@ using namespace mcd;
 extern "C" mcd_status mcd_tc_gemm(int32_t M, int32_t N, int32_t K, int32_t bn, const uint16_t* A, const uint16_t* B,
                                   float* Y, void* stream) {
   if (!A || !B || !Y || M <= 0 || N <= 0 || K <= 0) return MCD_ERR_INVALID_ARG;
-  if (M % tc::kBM || K % tc::kBK || (bn != 128 && bn != 256) || N % bn) return MCD_ERR_UNSUPPORTED;
+  if (M % tc::kBM || K % tc::kBK || (bn != 0 && bn != 128 && bn != 256) || N % (bn ? bn : 16))
+    return MCD_ERR_UNSUPPORTED;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t *ta = nullptr, *tb = nullptr;
   int* err = nullptr;
@@ -56,8 +74,8 @@ extern "C" mcd_status mcd_tc_gemm(int32_t M, int32_t N, int32_t K, int32_t bn, c
   }
   int herr = 0;
   if (e == cudaSuccess) {
-    tc::GemmArgs g{ta, nullptr, tb, nullptr, M, N, K, nullptr, err, 2000000000ull};
-    e = bn == 256 ? tc::launch_store<256>(g, Y, st) : tc::launch_store<128>(g, Y, st);
+    tc::GemmArgs g{ta, nullptr, tb, nullptr, M, N, K, nullptr, err, 2000000000ull, bn ? 0 : tc::auto_pitch(M, N)};
+    e = bn == 128 ? tc::launch_store<128>(g, Y, st) : tc::launch_store<256>(g, Y, st);
   }
   if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, sizeof(int), cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
@@ -66,4 +84,26 @@ extern "C" mcd_status mcd_tc_gemm(int32_t M, int32_t N, int32_t K, int32_t bn, c
   cudaFree(err);
   if (e != cudaSuccess) return cuda_status(e);
   return herr ? (mcd_status)herr : MCD_OK;
+}
+
+extern "C" mcd_status mcd_tc_tile(int32_t R, int32_t K, int32_t ld, const uint16_t* src, void* dst, void* stream) {
+  if (!src || !dst || R <= 0 || K <= 0 || ld < K) return MCD_ERR_INVALID_ARG;
+  if (R % 16 || K % tc::kBK || (reinterpret_cast<uintptr_t>(dst) & 1023u) || (reinterpret_cast<uintptr_t>(src) & 15u) ||
+      ld % 8)
+    return MCD_ERR_UNSUPPORTED;
+  tc::sw128_tile_kernel<<<1024, 256, 0, static_cast<cudaStream_t>(stream)>>>(src, R, K, ld,
+                                                                             static_cast<uint8_t*>(dst));
+  return cuda_status(cudaGetLastError());
+}
+
+extern "C" mcd_status mcd_tc_gemm_tiled(int32_t M, int32_t N, int32_t K, int32_t bn, const void* A_tiled,
+                                        const void* B_tiled, float* Y, int32_t* err, void* stream) {
+  if (!A_tiled || !B_tiled || !Y || !err || M <= 0 || N <= 0 || K <= 0) return MCD_ERR_INVALID_ARG;
+  if (M % tc::kBM || K % tc::kBK || (bn != 0 && bn != 128 && bn != 256) || N % (bn ? bn : 16))
+    return MCD_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(A_tiled) | reinterpret_cast<uintptr_t>(B_tiled)) & 1023u) return MCD_ERR_UNSUPPORTED;
+  tc::GemmArgs g{static_cast<const uint8_t*>(A_tiled), nullptr, static_cast<const uint8_t*>(B_tiled), nullptr,
+                 M, N, K, nullptr, err, 2000000000ull, bn ? 0 : tc::auto_pitch(M, N)};
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return cuda_status(bn == 128 ? tc::launch_store<128>(g, Y, st) : tc::launch_store<256>(g, Y, st));
 }

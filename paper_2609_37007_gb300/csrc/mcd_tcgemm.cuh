@@ -65,10 +65,13 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t smem_addr) {
   return d;
 }
 
-// Instruction descriptor of kind::f16: bf16 A and B (K-major), fp32 D, M = 128, N = BN.
+// Instruction descriptor of kind::f16: bf16 A and B (K-major), fp32 D, M = 128, N = n.
+__host__ __device__ constexpr uint32_t idesc_bf16_n(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
 template <int BN>
 __host__ __device__ constexpr uint32_t idesc_bf16() {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+  return idesc_bf16_n(BN);
 }
 
 __device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, bool accumulate) {
@@ -99,6 +102,23 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// The same load without its wait: r is defined only after tmem_wait16(r), which names the
+// registers so that no use of them can move above the wait.
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
+
 __device__ __forceinline__ uint64_t policy_evict_last() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
@@ -127,6 +147,8 @@ struct GemmArgs {
   const int* n_active;   // optional (device): columns n >= *n_active are not computed
   int* err;
   unsigned long long wait_ns;
+  int bn;                // gemm_tile: 0 = tiles of BN columns; else tile x covers columns
+                         // x * bn .. min(N, (x + 1) * bn) - 1 (bn a multiple of 16, <= BN)
 };
 
 // The GEMM body for the tile of rows m0 = blockIdx.y * 128 of A and n0 = blockIdx.x * BN of B
@@ -139,7 +161,8 @@ template <int BN, bool kDualA, bool kDualB, class Epi>
 __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
   using L = Layout<BN, kDualA, kDualB>;
   extern __shared__ uint8_t tc_smem_raw[];
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * kBM;
+  const int pitch = g.bn ? g.bn : BN, n0 = blockIdx.x * pitch, m0 = blockIdx.y * kBM;
+  const int nw = min(pitch, g.N - n0);                            // this tile's columns
   if (g.n_active && n0 >= __ldg(g.n_active)) return;          // uniform over the CTA
   const int nk_all = g.K / kBK, per = (nk_all + gridDim.z - 1) / gridDim.z;
   const int kt0 = blockIdx.z * per, kt1 = min(nk_all, kt0 + per), nk = kt1 - kt0;
@@ -185,12 +208,13 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
       if (*abort_flag) break;
       uint8_t* st = smem + s * L::kStageBytes;
       const size_t ao = (size_t)kt * g.M * 128 + (size_t)m0 * 128, bo = (size_t)kt * g.N * 128 + (size_t)n0 * 128;
-      mbar_arrive_expect_tx(&full[s], L::kStageBytes);
+      const uint32_t b_bytes = (uint32_t)nw * 128u;
+      mbar_arrive_expect_tx(&full[s], (kDualA ? 2 : 1) * L::kABytes + (kDualB ? 2 : 1) * b_bytes);
       bulk_g2s(st, g.a + ao, L::kABytes, &full[s], pol_a);
       if (kDualA) bulk_g2s(st + L::kABytes, g.a2 + ao, L::kABytes, &full[s], pol_a);
       uint8_t* sb = st + (kDualA ? 2 : 1) * L::kABytes;
-      bulk_g2s(sb, g.b + bo, L::kBBytes, &full[s], pol_b);
-      if (kDualB) bulk_g2s(sb + L::kBBytes, g.b2 + bo, L::kBBytes, &full[s], pol_b);
+      bulk_g2s(sb, g.b + bo, b_bytes, &full[s], pol_b);
+      if (kDualB) bulk_g2s(sb + L::kBBytes, g.b2 + bo, b_bytes, &full[s], pol_b);
       ++issued;
     }
     // every issued copy lands before the CTA may exit
@@ -198,7 +222,7 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
       tc_wait(&full[i % L::kStages], (i / L::kStages) & 1, g.err, g.wait_ns);
   } else if (warp == 1 && lane == 0) {
     // MMA issuer
-    constexpr uint32_t idesc = idesc_bf16<BN>();
+    const uint32_t idesc = idesc_bf16_n(nw);
     for (int i = 0; i < nk; ++i) {
       const int s = i % L::kStages;
       if (!tc_wait(&full[s], (i / L::kStages) & 1, g.err, g.wait_ns)) {
@@ -226,15 +250,46 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
   __syncwarp();                       // the .sync.aligned TMEM loads need whole warps
   tc_fence_after();
   if (ok) {
-    const int m = m0 + warp * 32 + lane;
-    const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+    // warp w reads TMEM lanes 32 (w % 4) ..; with more than four warps the 16-column chunks
+    // are shared out (chunk c to the warps w / 4 == c mod (warps / 4))
+    const int quarter = warp & 3, part = warp >> 2, n_parts = (int)(blockDim.x >> 7);
+    const int m = m0 + quarter * 32 + lane, n_ch = nw >> 4;
+    const uint32_t lane_base = tmem + ((uint32_t)(quarter * 32) << 16);
+    if (kDualA) {
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 16) {
-      float v[16], v2[16];
-      tmem_ld16(lane_base + (uint32_t)c0, v);
-      if (kDualA) tmem_ld16(lane_base + (uint32_t)(BN + c0), v2);
+      for (int ch = part; ch < n_ch; ch += n_parts) {
+        float v[16], v2[16];
+        tmem_ld16(lane_base + (uint32_t)(16 * ch), v);
+        tmem_ld16(lane_base + (uint32_t)(BN + 16 * ch), v2);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) epi(m, n0 + c0 + j, v[j], kDualA ? v2[j] : 0.f);
+        for (int j = 0; j < 16; ++j) epi(m, n0 + 16 * ch + j, v[j], v2[j]);
+      }
+    } else if (part < n_ch) {
+      // the next chunk's TMEM load is in flight while this chunk's values are stored (two
+      // register sets, alternating)
+      uint32_t ra[16], rb[16];
+      auto store = [&](const uint32_t (&r)[16], int ch) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) epi(m, n0 + 16 * ch + j, __uint_as_float(r[j]), 0.f);
+      };
+      int ch = part;
+      tmem_ld16_async(lane_base + (uint32_t)(16 * ch), ra);
+      tmem_wait16(ra);
+#pragma unroll 1
+      while (true) {
+        int nx = ch + n_parts;
+        if (nx < n_ch) tmem_ld16_async(lane_base + (uint32_t)(16 * nx), rb);
+        store(ra, ch);
+        if (nx >= n_ch) break;
+        tmem_wait16(rb);
+        ch = nx;
+        nx = ch + n_parts;
+        if (nx < n_ch) tmem_ld16_async(lane_base + (uint32_t)(16 * nx), ra);
+        store(rb, ch);
+        if (nx >= n_ch) break;
+        tmem_wait16(ra);
+        ch = nx;
+      }
     }
   }
   tc_fence_before();

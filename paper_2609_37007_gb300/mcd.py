@@ -121,6 +121,8 @@ def load_library() -> ctypes.CDLL:
         "mcd_outer_sync": (I32, [P]),
         "mcd_outer_step_weight_bytes": (I64, [P]),
         "mcd_tc_gemm": (I32, [I32, I32, I32, I32, P, P, P, P]),
+        "mcd_tc_tile": (I32, [I32, I32, I32, P, P, P]),
+        "mcd_tc_gemm_tiled": (I32, [I32, I32, I32, I32, P, P, P, P, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -283,6 +285,21 @@ def mcd_tc_gemm(M: int, N: int, K: int, bn: int, A, B, Y, stream=None):
     [N, K], Y fp32 [N, M], all device tensors (synchronises the stream)."""
     _check("mcd_tc_gemm", load_library().mcd_tc_gemm(M, N, K, bn, _ptr(A), _ptr(B), _ptr(Y),
                                                      ctypes.c_void_p(stream.cuda_stream if stream is not None else None)))
+
+
+def mcd_tc_tile(R: int, K: int, src, dst, stream=None, ld=None):
+    """Re-lay device bf16 src [R][K] (row stride ld, default K) into the swizzled tile layout
+    of mcd_tc_gemm_tiled in dst (device, R * K * 2 bytes); asynchronous on the stream."""
+    _check("mcd_tc_tile", load_library().mcd_tc_tile(R, K, K if ld is None else ld, _ptr(src), _ptr(dst),
+                                                     ctypes.c_void_p(stream.cuda_stream if stream is not None else None)))
+
+
+def mcd_tc_gemm_tiled(M: int, N: int, K: int, bn: int, A_tiled, B_tiled, Y, err, stream=None):
+    """Y[n][m] = sum_k A[m][k] B[n][k] from tiled operands (mcd_tc_tile); err: device int32,
+    zeroed by the caller.  Asynchronous: launches the product on the stream and returns."""
+    _check("mcd_tc_gemm_tiled", load_library().mcd_tc_gemm_tiled(
+        M, N, K, bn, _ptr(A_tiled), _ptr(B_tiled), _ptr(Y), _ptr(err),
+        ctypes.c_void_p(stream.cuda_stream if stream is not None else None)))
 
 
 def mcd_status_str(status: int) -> str:
