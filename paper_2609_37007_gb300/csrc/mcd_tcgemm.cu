@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "mcd_host.cuh"
 #include "mcd_tcgemm.cuh"
@@ -22,20 +23,51 @@ __global__ void sw128_tile_kernel(const uint16_t* __restrict__ src, int R, int K
 }
 
 // Stand-alone product: eight warps (two per TMEM lane quarter share the epilogue's columns).
+// Launched as a programmatic dependent of the previous kernel in the stream: the grid is set
+// up while that kernel runs, and every thread waits for its completion (and the visibility
+// of its writes) before the first global access.
 constexpr int kStoreThreads = 256;
 template <int BN>
 __global__ void __launch_bounds__(kStoreThreads, 1) gemm_store_kernel(const GemmArgs g, float* __restrict__ Y) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   gemm_tile<BN, false, false>(g, [&](int m, int n, float v, float) { Y[(size_t)n * g.M + m] = v; });
 }
 
 template <int BN>
 static cudaError_t launch_store(const GemmArgs& g, float* Y, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(gemm_store_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Layout<BN>::kSmemBytes);
+  // the shared-memory opt-in is a property of the function: set once per device
+  static std::atomic<unsigned> opted{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  const unsigned bit = 1u << (dev & 31);
+  if (!(opted.load(std::memory_order_acquire) & bit)) {
+    e = cudaFuncSetAttribute(gemm_store_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<BN>::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    opted.fetch_or(bit, std::memory_order_acq_rel);
+  }
   const int pitch = g.bn ? g.bn : BN;
-  gemm_store_kernel<BN><<<dim3((g.N + pitch - 1) / pitch, g.M / kBM), kStoreThreads, Layout<BN>::kSmemBytes, st>>>(g, Y);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((g.N + pitch - 1) / pitch, g.M / kBM);
+  cfg.blockDim = dim3(kStoreThreads);
+  cfg.dynamicSmemBytes = Layout<BN>::kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_store_kernel<BN>, g, Y);
+}
+
+// The narrowest instantiation that holds a tile of `pitch` columns (smaller stages: more of
+// them in flight).
+static cudaError_t launch_store_pitch(const GemmArgs& g, float* Y, cudaStream_t st) {
+  const int pitch = g.bn;
+  if (pitch <= 128) return launch_store<128>(g, Y, st);
+  if (pitch <= 176) return launch_store<176>(g, Y, st);
+  return launch_store<256>(g, Y, st);
 }
 
 // Tile pitch over N that fills the GPU with one tile per CTA: T = SMs / (M / 128) tiles across
@@ -75,7 +107,8 @@ extern "C" mcd_status mcd_tc_gemm(int32_t M, int32_t N, int32_t K, int32_t bn, c
   int herr = 0;
   if (e == cudaSuccess) {
     tc::GemmArgs g{ta, nullptr, tb, nullptr, M, N, K, nullptr, err, 2000000000ull, bn ? 0 : tc::auto_pitch(M, N)};
-    e = bn == 128 ? tc::launch_store<128>(g, Y, st) : tc::launch_store<256>(g, Y, st);
+    e = bn == 128 ? tc::launch_store<128>(g, Y, st) : bn == 256 ? tc::launch_store<256>(g, Y, st)
+                                                             : tc::launch_store_pitch(g, Y, st);
   }
   if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, err, sizeof(int), cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
@@ -105,5 +138,7 @@ extern "C" mcd_status mcd_tc_gemm_tiled(int32_t M, int32_t N, int32_t K, int32_t
   tc::GemmArgs g{static_cast<const uint8_t*>(A_tiled), nullptr, static_cast<const uint8_t*>(B_tiled), nullptr,
                  M, N, K, nullptr, err, 2000000000ull, bn ? 0 : tc::auto_pitch(M, N)};
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  return cuda_status(bn == 128 ? tc::launch_store<128>(g, Y, st) : tc::launch_store<256>(g, Y, st));
+  return cuda_status(bn == 128   ? tc::launch_store<128>(g, Y, st)
+                     : bn == 256 ? tc::launch_store<256>(g, Y, st)
+                                 : tc::launch_store_pitch(g, Y, st));
 }

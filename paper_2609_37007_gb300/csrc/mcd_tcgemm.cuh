@@ -38,13 +38,20 @@ __host__ __device__ __forceinline__ size_t sw128_offset(int R, int row, int kt, 
 // kDualA: a second A matrix (same shape) multiplies the same B into a second accumulator
 // (gate and up projections side by side); kDualB: a second B operand (the low bf16 half of
 // a hi + lo split) accumulates into the same accumulator.
+// TMEM allocations are powers of two of at least 32 columns.
+__host__ __device__ constexpr int tmem_cols_for(int cols) {
+  int c = 32;
+  while (c < cols) c <<= 1;
+  return c;
+}
+
 template <int BN, bool kDualA = false, bool kDualB = false>
 struct Layout {
-  static_assert(BN % 16 == 0 && BN >= 32 && BN <= 256 && (BN & (BN - 1)) == 0, "UMMA N / TMEM columns");
+  static_assert(BN % 16 == 0 && BN >= 32 && BN <= 256, "UMMA N");
   static constexpr int kABytes = kBM * 128;
   static constexpr int kBBytes = BN * 128;
   static constexpr int kStageBytes = (kDualA ? 2 : 1) * kABytes + (kDualB ? 2 : 1) * kBBytes;
-  static constexpr int kTmemCols = (kDualA ? 2 : 1) * BN;
+  static constexpr int kTmemCols = tmem_cols_for((kDualA ? 2 : 1) * BN);
   static constexpr int kStages = kStageBudget / kStageBytes > 8 ? 8 : kStageBudget / kStageBytes;
   static constexpr int kBarOff = kStages * kStageBytes;                 // full[s], empty[s], accum
   static constexpr int kTmemSlotOff = kBarOff + (2 * kStages + 1) * 8;
@@ -312,7 +319,7 @@ template <int BN, bool kDualA, bool kDualB>
 struct PLayout {
   using L = Layout<BN, kDualA, kDualB>;
   static constexpr int kAccCols = (kDualA ? 2 : 1) * BN;     // one accumulator buffer
-  static constexpr int kTmemCols = 2 * kAccCols;
+  static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
   static_assert(kTmemCols <= 512, "TMEM columns");
   static constexpr int kBarOff = L::kStages * L::kStageBytes;  // full[S], empty[S], acc_full[2], acc_empty[2], drain
   static constexpr int kTmemSlotOff = kBarOff + (2 * L::kStages + 5) * 8;
