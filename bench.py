@@ -419,11 +419,20 @@ def run_timeline(args, weights):
     import torch
     from paper_2609_37007_gb300 import build as _build
     from paper_2609_37007_gb300 import mcd
-    from paper_2609_37007_gb300.synth import MCD, make_frames
+    from paper_2609_37007_gb300 import tree as trees
+    from paper_2609_37007_gb300.synth import DRAFT_TREE, MCD, make_frames
     _build.build()
     cfg = MCD
     dev = torch.device("cuda", 0)
+    tree_n = args.timeline_tree
+    if tree_n:
+        # a tree call: the greedy tree of tree_n nodes for rank-decreasing statistics of 8
+        # candidates at each of 3 depths (single pass: at most 31 nodes)
+        cfg = MCD.replace(draft_mode=DRAFT_TREE, draft_len=3)
+        acc = [[0.6 / (r + 1) ** 0.5 for r in range(8)] for _ in range(3)]
     dec = mcd.Decoder(cfg, weights)
+    if tree_n:
+        mcd.mcd_set_tree(dec.ctx, *trees.grow_tree(acc, tree_n))
     n = max(12, args.timeline)
     cond_h, c0_h, _ = make_frames(cfg, n, first=4_000_000)
     cond, c0 = torch.from_numpy(cond_h).to(dev), torch.from_numpy(c0_h).to(dev)
@@ -447,12 +456,16 @@ def run_timeline(args, weights):
                        "signalled_us": r3 - r2})
         prev = r3
     gaps = [(tl[i, c + 1, 0] - tl[i, c, 7]) / 1e3 for i in range(10, n) for c in range(int(st[i, 0]) - 1)]
-    line = {"timeline": "frame_kernel<bf16>, MultiCodeDecoder bf16 workload, K = 3, one stream",
-            "frames": n - 10, "calls": len(rows), "us_per_call": med(7), "stages": stages,
+    what = ("frame_kernel<bf16>, MultiCodeDecoder bf16 workload, K = 3, one stream" if not tree_n else
+            "frame_kernel<bf16> wide, MultiCodeDecoder bf16 workload, TREE mode, %d-node tree (%d rows), one stream"
+            % (tree_n, tree_n + 1))
+    line = {"timeline": what,
+            "frames": n - 10, "calls": len(rows), "us_per_call": med(7) if not tree_n else None, "stages": stages,
             "topk": {"ready_us": med(1), "cta0_done_us": med(2) - med(1), "last_done_us": med(3) - med(1)},
-            "accept": {"start_us": med(4), "staged_us": med(5) - med(4), "decided_us": med(6) - med(5),
-                       "end_us": med(7) - med(6)},
-            "handover_us": float(np.median(gaps)) if gaps else None,
+            "accept": None if tree_n else {"start_us": med(4), "staged_us": med(5) - med(4),
+                                           "decided_us": med(6) - med(5), "end_us": med(7) - med(6)},
+            "handover_us": float(np.median(gaps)) if gaps and not tree_n else None,
+            "topk_done_us": med(3),
             "note": "stamps add a global store per stage and an atomic max per CTA and stage: a stamped call is "
                     "a few microseconds slower than an unstamped one"}
     print(json.dumps(line), flush=True)
@@ -719,6 +732,8 @@ def main():
     ap.add_argument("--pipeline", action="store_true",
                     help="full frame pipeline (CodeDecoder + MultiCodeDecoder) instead of the bench line")
     ap.add_argument("--utterances", type=int, default=2)
+    ap.add_argument("--timeline-tree", type=int, default=0,
+                    help="with --timeline: time TREE-mode calls of a grown tree of this many nodes (<= 31)")
     ap.add_argument("--tc-gemm", action="store_true",
                     help="time the stand-alone tensor-core product (6144 x 512 x 1024) instead of the bench line")
     ap.add_argument("--timeline", type=int, default=0,
