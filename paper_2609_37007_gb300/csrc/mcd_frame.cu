@@ -1594,13 +1594,16 @@ __device__ __forceinline__ bool read_call_state(Cons& c, int call, bool first) {
           ci->r_node[n] = (signed char)(m - 1);
         }
       }
-      // attention groups: up to 8 consecutive rows whose keys (the committed prefix, row 0
-      // and the union of their ancestor-or-self sets) fit one task
+      // attention groups: up to G consecutive rows whose keys (the committed prefix, row 0
+      // and the union of their ancestor-or-self sets) fit one task; G spreads the
+      // (query head, group) tasks over the CTAs (at most 8 rows, the task's query capacity)
+      const int want = max(1, p.n_cta / p.NH);                    // groups per query head
+      const int G = min(8, max(1, (Mp + want - 1) / want));
       int ng = 0, r = 0;
       while (r < Mp) {
         const int start = r;
         unsigned long long U = 0ull;
-        while (r < Mp && r - start < 8) {
+        while (r < Mp && r - start < G) {
           const int m = row0 + r;
           const unsigned long long am = m > 0 ? p.tree_anc[m - 1] : 0ull;
           if (r > start && st.pos0 + 1 + __popcll(U | am) > kTreeKeys) break;
