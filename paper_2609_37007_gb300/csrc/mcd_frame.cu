@@ -976,8 +976,9 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
   // the CTA that arrives last runs its acceptance.  Several: CTA b runs the acceptance of
   // the b-th stream in the call once every CTA has arrived.
   if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned old = atomicAdd(ctr + ctr_topk(L), 1u);
+    // release this CTA's records; the last arriver also acquires every earlier arrival's
+    // (several streams: the acceptance CTAs acquire through the counter's acquire loads)
+    const unsigned old = atom_add_acq_rel(ctr + ctr_topk(L), 1u);
     int mine = -1;
     if (p.S == 1) {
       if (old == N - 1u) mine = 0;
@@ -985,7 +986,6 @@ __device__ __forceinline__ void run_call(Cons& c, int call) {
       if (wait_counter(ctr + ctr_topk(L), N, p.err, p.wait_ns)) mine = ci->act[blockIdx.x];
       else sm.flags[1] = 1;
     }
-    if (mine >= 0) __threadfence();
     sm.flags[2] = mine >= 0 ? 1 : 0;
     sm.flags[4] = mine;
   }
@@ -1209,13 +1209,11 @@ __device__ __noinline__ void accept_step(const FrameParams& p, int call, int s) 
   consumer_sync();
   if (s == 0) timeline_p(p, sm.ci, 7, true);
   if (threadIdx.x == 0) {
-    // the last acceptance of the call releases the next call
-    __threadfence();
+    // the last acceptance of the call releases the next call (having acquired the others'
+    // state writes through the acceptance counter)
     unsigned* ctr = p.ctr + (size_t)call * p.ctr_stride;
-    if (ci->n_act == 1 || atomicAdd(ctr + ctr_accept(p.L), 1u) == (unsigned)ci->n_act - 1u) {
-      if (ci->n_act > 1) __threadfence();
-      atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
-    }
+    if (ci->n_act == 1 || atom_add_acq_rel(ctr + ctr_accept(p.L), 1u) == (unsigned)ci->n_act - 1u)
+      red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
   }
 }
 
@@ -1469,7 +1467,6 @@ __device__ __noinline__ void tree_pass_step(const FrameParams& p, int call) {
     st->tpass = ci->st[0].tpass + 1;
     st->heads_read = ci->st[0].heads_read + ci->phi[0] - ci->plo[0] + 1;
     st->call = call + 1;
-    __threadfence();
     red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
   }
 }
@@ -1513,8 +1510,7 @@ __device__ __noinline__ void emu_step(const FrameParams& p, int call) {
     }
     st->call = call + 1;
     if (p.trace && round < kMaxCalls) reinterpret_cast<mcd_call_trace*>(p.trace)[round].next_drafts[j - 1] = d;
-    __threadfence();
-    atomicAdd(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
+    red_release_add(p.ctr + (size_t)(call + 1) * p.ctr_stride + ctr_ready(p.L), 1u);
   }
 }
 

@@ -254,6 +254,14 @@ __device__ __forceinline__ uint32_t ld_acquire(const unsigned* p) {
 __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
   asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+// Acquire-release add at GPU scope returning the old value: releases like red_release_add
+// and, for the caller (and its CTA after a barrier), acquires every write released by the
+// earlier adds to the same counter.
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
 // 16-byte global -> shared copy through L2 (cp.async.cg: other CTAs' writes are seen once
 // they are visible at GPU scope); cpa_wait_all waits for this thread's copies.
 __device__ __forceinline__ void cpa16(void* dst, const void* src) {
