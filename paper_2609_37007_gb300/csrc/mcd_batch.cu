@@ -595,6 +595,16 @@ __global__ void __launch_bounds__(256) batch_rowss_kernel(const float* X, int H,
 // attention: one CTA per (stream, KV head).  At most 32 registers per thread, so that seven
 // CTAs share an SM and the 1024 CTAs of 128 streams run as one wave.
 // ------------------------------------------------------------------------------------
+// Attention of the call's rows of stream s = blockIdx.x for KV head g = blockIdx.y and its
+// `group` query heads (QK-norm, RoPE, causal softmax over the stream's cached positions and
+// its new rows); outputs to the Wo product's operand.  Phases, with block barriers between
+// them: (A) every input (the nr x group query vectors, cached and new K / V rows, RoPE rows
+// of the new positions, QK-norm gains) copied into shared memory as 16-byte cp.async chunks,
+// all in flight; (B) one warp per new q / k vector applies QK-norm and RoPE in registers and
+// stores the new rows' K / V to the cache; (C) one warp per query vector: lanes 2j, 2j + 1
+// score key j over interleaved chunks, softmax across the warp, then four output dims per
+// lane summed over the keys.  Row and head of a query vector come from a table, not a
+// division.
 __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, BatchBufs b, int layer) {
   const int s = blockIdx.x, g = blockIdx.y;
   if (s >= b.frame->S) return;
@@ -604,54 +614,59 @@ __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, Batch
   const int nr = st->n_rows, pos0 = st->pos0;
   const int D = p.D, half = D >> 1, group = p.NH / p.NKV, nq = nr * group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  __shared__ __align__(16) float qs[kBatchQVec][132];        // nr x group query vectors
+  const int lg4 = D == 128 ? 5 : 4, D4 = 1 << lg4;                // 16-byte chunks per row
+  __shared__ __align__(16) float qs[kBatchQVec][132];
   __shared__ __align__(16) float ks[kBatchKeys][132];
   __shared__ __align__(16) float vs[kBatchKeys][128];
-  __shared__ float sc[kBatchQVec][kBatchKeys];
+  __shared__ __align__(16) float2 cs[kMaxRows][64];               // RoPE (cos, sin) of the new rows
+  __shared__ __align__(16) float gq[128], gk[128];
+  __shared__ int q_row[kBatchQVec], q_head[kBatchQVec];
   const size_t cache_off = (size_t)s * p.kv_stride + ((size_t)layer * p.NKV + g) * p.kv_slots * D;
   const int nk = pos0 + nr;
-  const int D4 = D >> 2;
-  // loads: queries, then keys and values (cached rows, then the new rows), as 16-byte chunks,
-  // a batch of up to 3 per thread in flight before the stores
-  {
-    const int n_q = nq * D4, n_kv = nk * D4, total = n_q + 2 * n_kv;
-    constexpr int kL = 3;
-    for (int b0 = 0; b0 < total; b0 += kL * 256) {
-      float4 v[kL];
-      float4* dst[kL];
-#pragma unroll
-      for (int u = 0; u < kL; ++u) {
-        const int i = b0 + tid + u * 256;
-        dst[u] = nullptr;
-        if (i < total) {
-          const float4* src;
-          if (i < n_q) {
-            const int qi = i / D4, d4 = i - qi * D4, n = qi / group, h = g * group + qi % group;
-            src = reinterpret_cast<const float4*>(b.qkv + (size_t)(base + n) * p.qkv_dim + h * D) + d4;
-            dst[u] = reinterpret_cast<float4*>(qs[qi]) + d4;
-          } else {
-            const int i2 = i - n_q, isv = i2 >= n_kv, i3 = isv ? i2 - n_kv : i2, j = i3 / D4, d4 = i3 - j * D4;
-            if (j < pos0)
-              src = reinterpret_cast<const float4*>((isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D) + d4;
-            else
-              src = reinterpret_cast<const float4*>(b.qkv + (size_t)(base + j - pos0) * p.qkv_dim + p.NH * D +
-                                                    (isv ? p.NKV * D : 0) + g * D) + d4;
-            dst[u] = reinterpret_cast<float4*>(isv ? vs[j] : ks[j]) + d4;
-          }
-          v[u] = __ldcg(src);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kL; ++u)
-        if (dst[u]) *dst[u] = v[u];
-    }
+  if (tid < nq) {
+    q_row[tid] = tid / group;
+    q_head[tid] = g * group + tid % group;
   }
   __syncthreads();
-  // QK-norm + RoPE of the queries and the new keys (one warp per vector); new K / V cached
+  // ---- (A) loads ----------------------------------------------------------------------
+  {
+    const int e_q = nq << lg4, e_k = e_q + (nk << lg4), e_v = e_k + (nk << lg4);
+    const int e_cs = e_v + (nr << lg4), e_g = e_cs + (p.qk_norm ? 2 << lg4 : 0);
+    for (int i = tid; i < e_g; i += 256) {
+      const int ch = i & (D4 - 1);
+      const float* src;
+      float* dst;
+      if (i < e_q) {
+        const int qi = i >> lg4;
+        src = b.qkv + (size_t)(base + q_row[qi]) * p.qkv_dim + q_head[qi] * D;
+        dst = qs[qi];
+      } else if (i < e_v) {
+        const bool isv = i >= e_k;
+        const int j = (i - (isv ? e_k : e_q)) >> lg4;
+        if (j < pos0)
+          src = (isv ? p.vcache : p.kcache) + cache_off + (size_t)j * D;
+        else
+          src = b.qkv + (size_t)(base + j - pos0) * p.qkv_dim + p.NH * D + (isv ? p.NKV * D : 0) + g * D;
+        dst = isv ? vs[j] : ks[j];
+      } else if (i < e_cs) {
+        const int n = (i - e_v) >> lg4;
+        src = reinterpret_cast<const float*>(p.rope + (size_t)(pos0 + n) * half);
+        dst = reinterpret_cast<float*>(cs[n]);
+      } else {
+        const int w = (i - e_cs) >> lg4;
+        src = (w == 0 ? p.q_norm : p.k_norm) + (size_t)layer * D;
+        dst = w == 0 ? gq : gk;
+      }
+      cpa16(dst + 4 * ch, src + 4 * ch);
+    }
+    cpa_wait_all();
+  }
+  __syncthreads();
+  // ---- (B) QK-norm + RoPE of the queries and the new keys; new K / V cached --------------
   const int nd = D >> 5;
   for (int vi = warp; vi < nq + nr; vi += 8) {
     const bool isq = vi < nq;
-    const int n = isq ? vi / group : vi - nq;
+    const int n = isq ? q_row[vi] : vi - nq;
     float* row = isq ? qs[vi] : ks[pos0 + n];
     float x[4];
 #pragma unroll
@@ -663,15 +678,15 @@ __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, Batch
 #pragma unroll
       for (int off = 16; off; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
       const float scl = rsqrtf(ss / (float)D + p.eps);
-      const float* gg = (isq ? p.q_norm : p.k_norm) + (size_t)layer * D;
+      const float* gg = isq ? gq : gk;
 #pragma unroll
       for (int i = 0; i < 4; ++i)
-        if (i < nd) x[i] = x[i] * scl * __ldg(gg + lane + 32 * i);
+        if (i < nd) x[i] = x[i] * scl * gg[lane + 32 * i];
     }
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
       if (i < nd / 2) {
-        const float2 r = __ldg(p.rope + (size_t)(pos0 + n) * half + lane + 32 * i);
+        const float2 r = cs[n][lane + 32 * i];
         const float a0 = x[i], b0 = x[i + nd / 2];
         x[i] = a0 * r.x - b0 * r.y;
         x[i + nd / 2] = b0 * r.x + a0 * r.y;
@@ -690,61 +705,57 @@ __global__ void __launch_bounds__(256, 7) batch_attn_kernel(FrameParams p, Batch
     }
   }
   __syncthreads();
-  // scores: four adjacent threads per (query, key), each over every fourth 16-byte chunk,
-  // summed by shuffles (every thread runs the same number of rounds); softmax (one warp per
-  // query); P.V
+  // ---- (C) one warp per query vector: scores (lanes 2j, 2j+1), softmax, P.V ---------------
   const float scale = rsqrtf((float)D);
-  const int n_dot = nq * nk;
-  for (int t0 = 0; t0 < 4 * n_dot; t0 += 256) {
-    const int t = t0 + tid, qd = t >> 2, part = t & 3;
-    const bool live = qd < n_dot;
-    const int qi = live ? qd / nk : 0, j = live ? qd - qi * nk : 0, n = qi / group;
-    const bool causal = live && j <= pos0 + n;
-    float acc = 0.f;
-    if (causal) {
-      const float4* q4 = reinterpret_cast<const float4*>(qs[qi]);
-      const float4* k4 = reinterpret_cast<const float4*>(ks[j]);
-      for (int d4 = part; d4 < D4; d4 += 4) {
-        const float4 a = q4[d4], k = k4[d4];
-        acc += a.x * k.x + a.y * k.y + a.z * k.z + a.w * k.w;
+  for (int qi = warp; qi < nq; qi += 8) {
+    const int n = q_row[qi], h = q_head[qi], npos = pos0 + n + 1;
+    const int j = lane >> 1, hf = lane & 1;
+    const bool live = j < npos;                      // causal: keys 0..pos0+n
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    if (live) {
+      const float4* q4 = reinterpret_cast<const float4*>(qs[qi]) + hf;
+      const float4* k4 = reinterpret_cast<const float4*>(ks[j]) + hf;
+#pragma unroll 4
+      for (int c2 = 0; c2 < (D4 >> 1); ++c2) {
+        const float4 q = q4[2 * c2], k = k4[2 * c2];
+        a0 += q.x * k.x;
+        a1 += q.y * k.y;
+        a2 += q.z * k.z;
+        a3 += q.w * k.w;
       }
     }
-    acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
-    acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 2);
-    if (live && part == 0) sc[qi][j] = causal ? acc * scale : -INFINITY;
-  }
-  __syncthreads();
-  for (int qi = warp; qi < nq; qi += 8) {
-    const float v = lane < nk ? sc[qi][lane] : -INFINITY;
-    float m = v;
+    float sc = (a0 + a1) + (a2 + a3);
+    sc += __shfl_xor_sync(0xFFFFFFFFu, sc, 1);
+    sc = live ? sc * scale : -INFINITY;
+    float mx = sc;
 #pragma unroll
-    for (int off = 16; off; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, off));
-    const float e = v == -INFINITY ? 0.f : __expf(v - m);
-    float l = e;
+    for (int off = 16; off > 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, off));
+    const float e = live ? __expf(sc - mx) : 0.f;
+    float sum = e;                                   // lanes of one parity hold every key once
 #pragma unroll
-    for (int off = 16; off; off >>= 1) l += __shfl_xor_sync(0xFFFFFFFFu, l, off);
-    if (lane < nk) sc[qi][lane] = e / l;
-  }
-  __syncthreads();
-  // one thread per (query, 4 dims)
-  for (int t = tid; t < nq * D4; t += blockDim.x) {
-    const int qi = t / D4, d4 = t - qi * D4, n = qi / group, h = g * group + qi % group;
+    for (int off = 16; off > 1; off >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, off);
+    const float pj = e / sum;
+    const int d0 = 4 * lane;                         // four dims per lane
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int j = 0; j <= pos0 + n; ++j) {
-      const float pj = sc[qi][j];
-      const float4 v = reinterpret_cast<const float4*>(vs[j])[d4];
-      acc.x += pj * v.x;
-      acc.y += pj * v.y;
-      acc.z += pj * v.z;
-      acc.w += pj * v.w;
+    for (int jj = 0; jj < npos; ++jj) {
+      const float w = __shfl_sync(0xFFFFFFFFu, pj, 2 * jj);
+      if (d0 < D) {
+        const float4 v = *reinterpret_cast<const float4*>(&vs[jj][d0]);
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
     }
-    const int f = h * D + 4 * d4;
-    const uint2 packed = make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
-    if (b.att_t)        // the Wo product's operand, SW128 tiles (tensor-core path)
-      *reinterpret_cast<uint2*>(b.att_t + tc::sw128_offset(b.Rtc, base + n, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
-          packed;
-    else
-      *reinterpret_cast<uint2*>(b.att + (size_t)(base + n) * p.NH * D + f) = packed;
+    if (d0 < D) {
+      const int f = h * D + d0;
+      const uint2 packed = make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
+      if (b.att_t)        // the Wo product's operand, SW128 tiles (tensor-core path)
+        *reinterpret_cast<uint2*>(b.att_t + tc::sw128_offset(b.Rtc, base + n, f >> 6, (f & 63) >> 3) + (f & 7) * 2) =
+            packed;
+      else
+        *reinterpret_cast<uint2*>(b.att + (size_t)(base + n) * p.NH * D + f) = packed;
+    }
   }
 }
 
