@@ -790,19 +790,28 @@ __global__ void __launch_bounds__(kConsumerThreads) batch_accept_kernel(FramePar
   const TopkRec* cur = b.recs + (size_t)(call & 1) * b.R * kRecSlots;
   const TopkRec* prev = b.recs + (size_t)((call + 1) & 1) * b.R * kRecSlots;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // every record the acceptance reads, staged in shared memory first: p of positions
+  // a+1 .. (the bonus row only when its position exists), then q of the drafts
+  __shared__ __align__(16) TopkRec srec[2 * kMaxDraft + 1];
+  const int n_p = a + 1 + n_d <= p.P ? n_d + 1 : n_d;
+  stage_records(srec, n_p + n_d, p.top_k, [&](int r) {
+    return r < n_p ? cur + (size_t)(base + a + 1 + r - pos0) * kRecSlots : prev + (size_t)qrow * kRecSlots + 1 + (r - n_p);
+  });
+  __syncthreads();
   if (warp == 0) {
-    const AcceptResult r = warp_accept(
-        a, n_d, p.P, s_old, [&](int i) { return cur + (size_t)(base + a + 1 + i - pos0) * kRecSlots; },
-        [&](int i) { return prev + (size_t)qrow * kRecSlots + 1 + i; }, p.seed, sid, fid, call);
+    const AcceptResult r = warp_accept(a, n_d, p.P, s_old, [&](int i) { return srec + i; },
+                                       [&](int i) { return srec + n_p + i; }, p.seed, sid, fid, call);
     if (lane == 0) s_res = r;
   }
   __syncthreads();
   const int n_emit = s_res.n_emit, n_acc = s_res.n_acc;
   const int a_new = a + n_emit, m = a_new - pos0, n_next = min(p.K, p.P - a_new);
   // next drafts from the draft distributions of row m, whose head emitted the last code
+  stage_records(srec, n_next, p.top_k, [&](int r) { return cur + (size_t)(base + m) * kRecSlots + 1 + r; });
+  __syncthreads();
   for (int j = 1 + warp; j <= n_next; j += kConsumerWarps) {
     const unsigned long long U = uniform_U(p.seed, sid, fid, call, a_new + j, PURPOSE_DRAFT);
-    const int d = warp_draw(cur + (size_t)(base + m) * kRecSlots + j, U);
+    const int d = warp_draw(srec + (j - 1), U);
     if (lane == 0) s_next[j - 1] = d;
   }
   __syncthreads();

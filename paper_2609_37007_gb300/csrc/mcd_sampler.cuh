@@ -13,6 +13,8 @@
 // Every decision is an exact integer comparison, so a CPU implementation that computes the
 // same fp32 exp32 agrees bit for bit; sums are order-free and need no fp64 arithmetic.
 #pragma once
+#include <cstddef>
+
 #include "mcd_internal.cuh"
 
 namespace mcd {
@@ -498,6 +500,25 @@ struct AcceptResult {
   int n_emit;
   int emitted[kMaxRows];
 };
+
+// Copy distribution records into shared memory: the header with ids[0..k) and W[0..k) of
+// each (k = top_k; entries past a record's n are never read) as 16-byte cp.async chunks, all
+// in flight together.  Threads t0 .. t0 + nt - 1 take part; a barrier must follow.
+template <class Src>
+__device__ __forceinline__ void stage_records(TopkRec* dst, int nrec, int k, Src src, int t0 = 0,
+                                              int nt = kConsumerThreads) {
+  const int c_ids = (int)((offsetof(TopkRec, ids) + 4 * k + 15) / 16), c_w = (4 * k + 15) / 16;
+  const int per = c_ids + c_w, total = nrec * per, me = (int)threadIdx.x - t0;
+  if (me < 0 || me >= nt) return;
+  for (int i = me; i < total; i += nt) {
+    const int r = i / per, ch = i - r * per;
+    const int off = ch < c_ids ? ch * 16 : (int)offsetof(TopkRec, W) + (ch - c_ids) * 16;
+    cpa16(reinterpret_cast<uint8_t*>(dst + r) + off, reinterpret_cast<const uint8_t*>(src(r)) + off);
+  }
+  cpa_wait_all();
+}
+static_assert(sizeof(TopkRec) % 16 == 0 && offsetof(TopkRec, ids) % 16 == 0 && offsetof(TopkRec, W) % 16 == 0,
+              "records are copied in 16-byte chunks");
 
 // The acceptance step of one call, evaluated by one full warp.
 //   p_row(i): record of the verify distribution of position a+1+i (i = 0..n_d)
