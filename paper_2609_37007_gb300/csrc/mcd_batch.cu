@@ -159,17 +159,44 @@ __global__ void __launch_bounds__(256) batch_pack_kernel(FrameParams p, BatchBuf
       }
     }
   }
-  s_cnt[tid] = nr;
-  s_pc[tid] = np;
-  __syncthreads();
-  for (int off = 1; off < 256; off <<= 1) {      // inclusive scans (Hillis-Steele)
-    const int a = tid >= off ? s_cnt[tid - off] : 0, c = tid >= off ? s_pc[tid - off] : 0;
-    __syncthreads();
-    s_cnt[tid] += a;
-    s_pc[tid] += c;
-    __syncthreads();
+  // inclusive scans of (rows, pairs) over the streams: within each warp by shuffles, then
+  // over the 8 warp totals
+  const int lane = tid & 31, warp = tid >> 5;
+  int cr = nr, cp = np;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int a = __shfl_up_sync(0xFFFFFFFFu, cr, off), c = __shfl_up_sync(0xFFFFFFFFu, cp, off);
+    if (lane >= off) {
+      cr += a;
+      cp += c;
+    }
   }
-  const int base = s_cnt[tid] - nr, pbase = s_pc[tid] - np;
+  if (lane == 31) {
+    s_cnt[warp] = cr;
+    s_pc[warp] = cp;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    int wr = lane < 8 ? s_cnt[lane] : 0, wp = lane < 8 ? s_pc[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 8; off <<= 1) {
+      const int a = __shfl_up_sync(0xFFFFFFFFu, wr, off), c = __shfl_up_sync(0xFFFFFFFFu, wp, off);
+      if (lane >= off) {
+        wr += a;
+        wp += c;
+      }
+    }
+    if (lane < 8) {
+      s_cnt[8 + lane] = wr;             // inclusive totals through warp `lane`
+      s_pc[8 + lane] = wp;
+    }
+  }
+  __syncthreads();
+  if (warp > 0) {
+    cr += s_cnt[8 + warp - 1];
+    cp += s_pc[8 + warp - 1];
+  }
+  const int base = cr - nr, pbase = cp - np;
   if (tid < S && nr > 0) {
     for (int n = 0; n < nr; ++n) {
       const int pos = st.pos0 + n, r = base + n;
@@ -208,8 +235,8 @@ __global__ void __launch_bounds__(256) batch_pack_kernel(FrameParams p, BatchBuf
       s_hcur[P] = off;
       off += s_head[P];
     }
-    b.info->M = s_cnt[255];
-    b.info->n_pairs = s_pc[255];
+    b.info->M = s_cnt[8 + 7];
+    b.info->n_pairs = s_pc[8 + 7];
   }
   __syncthreads();
   if (tid < S && nr > 0) {
