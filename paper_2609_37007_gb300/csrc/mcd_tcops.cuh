@@ -109,11 +109,22 @@ __global__ void __launch_bounds__(128) tc_resid_norm_kernel(float* X, const floa
   if (live) {
     float4* xr = reinterpret_cast<float4*>(X + (size_t)r * H + 8 * t);
     float4 a = xr[0], b = xr[1];
-    for (int z = 0; z < nz; ++z) {
-      const float4* pr = reinterpret_cast<const float4*>(part + ((size_t)z * Rtc + r) * H + 8 * t);
-      const float4 u = __ldcg(pr), w = __ldcg(pr + 1);
-      a.x += u.x; a.y += u.y; a.z += u.z; a.w += u.w;
-      b.x += w.x; b.y += w.y; b.z += w.z; b.w += w.w;
+    // every partial's loads issued before the first add (nz <= kTcSplit), added in split order
+    float4 u[kTcSplit], w[kTcSplit];
+#pragma unroll
+    for (int z = 0; z < kTcSplit; ++z) {
+      if (z < nz) {
+        const float4* pr = reinterpret_cast<const float4*>(part + ((size_t)z * Rtc + r) * H + 8 * t);
+        u[z] = __ldcg(pr);
+        w[z] = __ldcg(pr + 1);
+      }
+    }
+#pragma unroll
+    for (int z = 0; z < kTcSplit; ++z) {
+      if (z < nz) {
+        a.x += u[z].x; a.y += u[z].y; a.z += u[z].z; a.w += u[z].w;
+        b.x += w[z].x; b.y += w[z].y; b.z += w[z].z; b.w += w[z].w;
+      }
     }
     xr[0] = a;
     xr[1] = b;
