@@ -573,7 +573,8 @@ __global__ void __launch_bounds__(256) tc_heads_operand_kernel(const float* __re
 
 // Logits of every pair: tile (blockIdx.x) of head P's group times head P's weights, plus the
 // draft-offset bias for j >= 1.
-__global__ void __launch_bounds__(tc::kThreads, 1) tc_heads_kernel(const tc::GemmArgs g, const uint8_t* w_heads,
+constexpr int kHeadsThreads = 256;     // eight warps: two per TMEM lane quarter in the epilogue
+__global__ void __launch_bounds__(kHeadsThreads, 1) tc_heads_kernel(const tc::GemmArgs g, const uint8_t* w_heads,
                                                                     size_t head_bytes, float* logits,
                                                                     const float* head_bias, const BatchInfo* info,
                                                                     const int* head_list, int n_pos, int K, int V) {
@@ -588,15 +589,27 @@ __global__ void __launch_bounds__(tc::kThreads, 1) tc_heads_kernel(const tc::Gem
     o += span;
   }
   if (P == 0) return;                                   // past the last group (uniform per CTA)
-  const int rows = info->head_rows[P], off = info->head_off[P];
+  const int rows = info->head_rows[P], off = info->head_off[P], i0 = q0 - qoff;
+  // the tile's (row, j) entries in shared memory and this thread's bias of every offset j
+  // (the epilogue's output row m is fixed per thread), loaded while the products run
+  __shared__ int s_entry[kTcBN];
+  for (int i = threadIdx.x; i < kTcBN; i += blockDim.x) s_entry[i] = i0 + i < rows ? head_list[off + i0 + i] : -1;
+  const int m_t = blockIdx.y * tc::kBM + ((threadIdx.x >> 5) & 3) * 32 + (threadIdx.x & 31);
+  float bias_j[kMaxDraft];
+#pragma unroll
+  for (int q = 0; q < kMaxDraft; ++q)
+    bias_j[q] = q < K ? __ldg(head_bias + ((size_t)(P - 1) * K + q) * V + m_t) : 0.f;
   tc::GemmArgs ga = g;
   ga.a = w_heads + (size_t)(P - 1) * head_bytes;
   ga.n_active = nullptr;
   tc::gemm_tile<kTcBN, false, true>(ga, [&](int m, int n, float v, float) {
-    const int i = n - qoff;
-    if (i < rows) {
-      const int e = head_list[off + i], r = e >> 3, j = e & 7;
-      const float bias = j >= 1 ? __ldg(head_bias + ((size_t)(P - 1) * K + (j - 1)) * V + m) : 0.f;
+    const int e = s_entry[n - q0];
+    if (e >= 0) {
+      const int r = e >> 3, j = e & 7;
+      float bias = 0.f;
+#pragma unroll
+      for (int q = 1; q <= kMaxDraft; ++q)
+        if (j == q) bias = bias_j[q - 1];
       logits[((size_t)r * kRecSlots + j) * V + m] = v + bias;
     }
   });
@@ -1170,7 +1183,7 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       tc_heads_operand_kernel<<<512, blk, 0, s>>>(b.X, p.final_norm, b.ss + (size_t)(2 * L) * R, H, p.eps, b.info,
                                                  b.head_list, p.P, b.Qcap, b.hq_hi, b.hq_lo);
       const tc::GemmArgs g{nullptr, nullptr, b.hq_hi, b.hq_lo, p.V, b.Qcap, H, nullptr, p.err, p.wait_ns};
-      tc_heads_kernel<<<dim3(b.Qcap / kTcBN, p.V / tc::kBM, 1), dim3(tc::kThreads),
+      tc_heads_kernel<<<dim3(b.Qcap / kTcBN, p.V / tc::kBM, 1), dim3(kHeadsThreads),
                         tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(g, bs->tw.heads, (size_t)p.V * H * 2, b.logits,
                                                                         p.head_bias, b.info, b.head_list, p.P, p.K, p.V);
     } else {   // final RMSNorm -> LM heads, one grid slice per head
