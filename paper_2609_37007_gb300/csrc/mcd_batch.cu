@@ -838,10 +838,46 @@ __global__ void __launch_bounds__(kConsumerThreads) batch_accept_kernel(FramePar
     return r < n_p ? cur + (size_t)(base + a + 1 + r - pos0) * kRecSlots : prev + (size_t)qrow * kRecSlots + 1 + (r - n_p);
   });
   __syncthreads();
-  if (warp == 0) {
-    const AcceptResult r = warp_accept(a, n_d, p.P, s_old, [&](int i) { return srec + i; },
-                                       [&](int i) { return srec + n_p + i; }, p.seed, sid, fid, call);
-    if (lane == 0) s_res = r;
+  // every draft's accept test and the residual draw it would take as the first rejection in
+  // parallel (warp i for draft i), warp n_d the bonus draw; then the chain is read off in
+  // order, taking the same decisions as testing the drafts one after another
+  __shared__ int s_ok[kMaxDraft + 1], s_alt[kMaxDraft + 1];
+  if (warp <= n_d) {
+    const int i = warp, pos = a + 1 + i;
+    if (i < n_d) {
+      const TopkRec* pr = srec + i;
+      const TopkRec* qr = srec + n_p + i;
+      const int d = s_old[i];
+      const unsigned long long wp = warp_weight(pr, d), wq = warp_weight(qr, d);
+      const unsigned long long U = uniform_U(p.seed, sid, fid, call, pos, PURPOSE_ACCEPT);
+      const bool ok = lt128(mul128x64(mul64(U, wq), pr->S), shl53(wp * qr->S));
+      const int alt = ok ? -1 : warp_residual(pr, qr, uniform_U(p.seed, sid, fid, call, pos, PURPOSE_TARGET));
+      if (lane == 0) {
+        s_ok[i] = ok ? 1 : 0;
+        s_alt[i] = alt;
+      }
+    } else if (pos <= p.P) {
+      const int bonus = warp_draw(srec + n_d, uniform_U(p.seed, sid, fid, call, pos, PURPOSE_TARGET));
+      if (lane == 0) s_alt[i] = bonus;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    AcceptResult r;
+    r.n_acc = 0;
+    r.n_emit = 0;
+    bool rejected = false;
+    for (int i = 0; i < n_d && !rejected; ++i) {
+      if (s_ok[i]) {
+        r.emitted[r.n_emit++] = s_old[i];
+        ++r.n_acc;
+      } else {
+        r.emitted[r.n_emit++] = s_alt[i];
+        rejected = true;
+      }
+    }
+    if (!rejected && a + 1 + n_d <= p.P) r.emitted[r.n_emit++] = s_alt[n_d];
+    s_res = r;
   }
   __syncthreads();
   const int n_emit = s_res.n_emit, n_acc = s_res.n_acc;
