@@ -1093,7 +1093,7 @@ mcd_status batch_load_layer(BatchState* bs, const FrameParams& p, cudaStream_t s
 // The tcgen05 GEMM's copy of LM head P (row-major bf16 [V][H] source, device).
 mcd_status batch_load_head(BatchState* bs, const FrameParams& p, cudaStream_t st, const uint8_t* src, int P) {
   if (!bs || !bs->tw.heads) return MCD_OK;
-  tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(src), p.V, p.H, p.V, 0,
+  tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(src), p.V, p.H, p.V, 0, p.V, 0,
                                              bs->tw.heads + (size_t)(P - 1) * p.V * p.H * 2);
   return cudaGetLastError() == cudaSuccess ? MCD_OK : MCD_ERR_CUDA;
 }
@@ -1149,10 +1149,7 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 1) * R,
                                              p.ffn_norm + (size_t)l * H, p.eps, b.xn_hi, nullptr);
       // gate/up -> SwiGLU (into the down product's operand)
-      {
-        const tc::GemmArgs g{wl + bs->tw.off.g, wl + bs->tw.off.u, b.xn_hi, nullptr, p.F, Rtc, H, &b.info->M, p.err, p.wait_ns};
-        tc_launch_gu(g, b.act_t, Rtc, &b.info->M, p.F, p.n_cta, s);
-      }
+      tc_launch_gu(wl + bs->tw.off.gu, b.xn_hi, b.act_t, Rtc, &b.info->M, p.F, H, p.err, p.wait_ns, p.n_cta, s);
       // down (k-split partials) -> residual, ss, the next layer's QKV operand
       {
         const tc::GemmArgs g{wl + bs->tw.off.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};

@@ -1124,10 +1124,7 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
     }
     tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(qd), Rtc, H, t.rows, t.ss, p.ffn_norm + (size_t)l * H,
                                            p.eps, t.xn_hi, nullptr);
-    {
-      const tc::GemmArgs g{wl + t.off.g, wl + t.off.u, t.xn_hi, nullptr, p.F, Rtc, H, t.rows, p.err, p.wait_ns};
-      tc_launch_gu(g, t.act_t, Rtc, t.rows, p.F, p.n_cta, s);
-    }
+    tc_launch_gu(wl + t.off.gu, t.xn_hi, t.act_t, Rtc, t.rows, p.F, H, p.err, p.wait_ns, p.n_cta, s);
     {
       const tc::GemmArgs g{wl + t.off.d, nullptr, t.act_t, nullptr, H, Rtc, p.F, t.rows, p.err, p.wait_ns};
       tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(

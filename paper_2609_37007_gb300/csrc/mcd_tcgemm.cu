@@ -70,16 +70,11 @@ static cudaError_t launch_store_pitch(const GemmArgs& g, float* Y, cudaStream_t 
   return launch_store<256>(g, Y, st);
 }
 
-// Tile pitch over N that fills the GPU with one tile per CTA: T = SMs / (M / 128) tiles across
-// N (at least ceil(N / 256)), each a multiple of 16 columns.
+// Tile pitch over N that fills this GPU with one tile per CTA.
 static int auto_pitch(int M, int N) {
   int dev = 0, n_sm = 148;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-  const int n_mt = M / kBM, units = N / 16;
-  int T = std::max(1, n_sm / std::max(1, n_mt));
-  T = std::max(T, (N + 255) / 256);
-  T = std::min(T, units);
-  return (units + T - 1) / T * 16;
+  return tile_pitch(M, N, n_sm);
 }
 
 }  // namespace tc

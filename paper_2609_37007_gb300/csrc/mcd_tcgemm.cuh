@@ -158,22 +158,39 @@ struct GemmArgs {
                          // x * bn .. min(N, (x + 1) * bn) - 1 (bn a multiple of 16, <= BN)
 };
 
-// The GEMM body for the tile of rows m0 = blockIdx.y * 128 of A and n0 = blockIdx.x * BN of B
-// over the k-slices of split blockIdx.z of gridDim.z (the CTAs that share an A tile are
-// adjacent in launch order, so the weights stream from HBM about once while the activation
-// tiles stay in L2); epi(m, n, v, v2) for every m and n of the tile (each thread: one m, BN
-// values of n in order; v2 = the second accumulator with kDualA, else 0).  A tile whose
-// first column is at or past *n_active returns at once.
-template <int BN, bool kDualA, bool kDualB, class Epi>
-__device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
+// Tile pitch over N that fills n_sm SMs with one tile per CTA: T = n_sm / (M / 128) tiles
+// across N (at least ceil(N / 256)), each a multiple of 16 columns.
+inline int tile_pitch(int M, int N, int n_sm) {
+  const int n_mt = M / kBM, units = N / 16;
+  int T = n_sm / (n_mt > 1 ? n_mt : 1);
+  if (T < 1) T = 1;
+  if (T < (N + 255) / 256) T = (N + 255) / 256;
+  if (T > units) T = units;
+  return (units + T - 1) / T * 16;
+}
+
+// The tile of a CTA once its k-loop has run (gemm_tile_run).
+struct TileRun {
+  uint8_t* smem;   // the operand ring: idle once every MMA has completed
+  uint32_t tmem;   // the accumulator(s)
+  int m0, n0, nw;  // first row of A, first column and columns of the tile
+  bool ok;         // every MMA completed (false after a timeout)
+};
+
+// Set-up, operand stream and MMAs of the tile of this CTA.  false: the tile is empty (its
+// first column at or past *n_active, or no k-slices in its split) and nothing is held; else
+// every thread returns after the accumulator is complete (t.ok) or the tile gave up, and the
+// CTA must call gemm_tile_free.
+template <int BN, bool kDualA, bool kDualB>
+__device__ __forceinline__ bool gemm_tile_run(const GemmArgs& g, TileRun& t) {
   using L = Layout<BN, kDualA, kDualB>;
   extern __shared__ uint8_t tc_smem_raw[];
   const int pitch = g.bn ? g.bn : BN, n0 = blockIdx.x * pitch, m0 = blockIdx.y * kBM;
   const int nw = min(pitch, g.N - n0);                            // this tile's columns
-  if (g.n_active && n0 >= __ldg(g.n_active)) return;          // uniform over the CTA
+  if (g.n_active && n0 >= __ldg(g.n_active)) return false;    // uniform over the CTA
   const int nk_all = g.K / kBK, per = (nk_all + gridDim.z - 1) / gridDim.z;
   const int kt0 = blockIdx.z * per, kt1 = min(nk_all, kt0 + per), nk = kt1 - kt0;
-  if (nk <= 0) return;
+  if (nk <= 0) return false;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
   uint64_t* empty = full + L::kStages;
@@ -252,11 +269,43 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
     }
     umma_commit(accum);               // every MMA issued so far has completed
   }
-  // epilogue: all four warps, after the accumulator is complete
-  const bool ok = tc_wait(accum, 0, g.err, g.wait_ns) && !*abort_flag;
+  t.ok = tc_wait(accum, 0, g.err, g.wait_ns) && !*abort_flag;
   __syncwarp();                       // the .sync.aligned TMEM loads need whole warps
   tc_fence_after();
-  if (ok) {
+  t.smem = smem;
+  t.tmem = tmem;
+  t.m0 = m0;
+  t.n0 = n0;
+  t.nw = nw;
+  return true;
+}
+
+// Every thread of the CTA, after the last TMEM load: the accumulator's columns are freed.
+template <int BN, bool kDualA, bool kDualB>
+__device__ __forceinline__ void gemm_tile_free(const TileRun& t) {
+  using L = Layout<BN, kDualA, kDualB>;
+  tc_fence_before();
+  __syncthreads();
+  if ((threadIdx.x >> 5) == 1)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(t.tmem), "r"((uint32_t)L::kTmemCols)
+                 : "memory");
+}
+
+// The GEMM body for the tile of rows m0 = blockIdx.y * 128 of A and n0 = blockIdx.x * BN of B
+// over the k-slices of split blockIdx.z of gridDim.z (the CTAs that share an A tile are
+// adjacent in launch order, so the weights stream from HBM about once while the activation
+// tiles stay in L2); epi(m, n, v, v2) for every m and n of the tile (each thread: one m, BN
+// values of n in order; v2 = the second accumulator with kDualA, else 0).  A tile whose
+// first column is at or past *n_active returns at once.
+template <int BN, bool kDualA, bool kDualB, class Epi>
+__device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
+  TileRun t;
+  if (!gemm_tile_run<BN, kDualA, kDualB>(g, t)) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = t.m0, n0 = t.n0, nw = t.nw;
+  const uint32_t tmem = t.tmem;
+  // epilogue: every warp, after the accumulator is complete
+  if (t.ok) {
     // warp w reads TMEM lanes 32 (w % 4) ..; with more than four warps the 16-column chunks
     // are shared out (chunk c to the warps w / 4 == c mod (warps / 4))
     const int quarter = warp & 3, part = warp >> 2, n_parts = (int)(blockDim.x >> 7);
@@ -299,11 +348,7 @@ __device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
       }
     }
   }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1)
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)L::kTmemCols)
-                 : "memory");
+  gemm_tile_free<BN, kDualA, kDualB>(t);
 }
 
 // ---- persistent form ----------------------------------------------------------------------

@@ -42,20 +42,20 @@ __global__ void __launch_bounds__(256) tc_norm_operand_kernel(const float* __res
   }
 }
 
-// Row-major bf16 [rows][K] -> rows row0.. of an SW128-tiled matrix of R rows (weight load).
-__global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0,
-                                      uint8_t* __restrict__ dst) {
+// Row-major bf16 [rows][K] -> an SW128-tiled matrix of R rows (weight load): source row r
+// goes to row row0 + (r / grp) * gstride + r % grp (grp = rows: row0 + r).
+__global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows, int K, int R, int row0, int grp,
+                                      int gstride, uint8_t* __restrict__ dst) {
   const long long total = (long long)rows * (K / 8);
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
     const int r = (int)(i / (K / 8)), ch = (int)(i % (K / 8));
-    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(R, row0 + r, ch >> 3, ch & 7)) =
+    const int dr = row0 + (r / grp) * gstride + r % grp;
+    *reinterpret_cast<uint4*>(dst + tc::sw128_offset(R, dr, ch >> 3, ch & 7)) =
         *reinterpret_cast<const uint4*>(src + (size_t)r * K + (size_t)ch * 8);
   }
 }
 
 constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
-// gate/up (two accumulators): 128-row tiles from 512 packed rows on, else 64 (more tiles)
-inline int tc_bn_gu(int Rtc) { return Rtc >= 512 ? 128 : 64; }
 constexpr int kTcSplit = 4;       // k-splits of the residual products
 
 // q, k, v = W (x . g / rms) with the hi + lo operand.
@@ -67,19 +67,57 @@ __global__ void __launch_bounds__(tc::kPThreads, 1) tc_qkv_kernel(const tc::Gemm
   });
 }
 
-// gate and up side by side; writes silu(gate) * up as bf16 into the SW128 operand of the down
-// product (element (row n, feature m)).
+// gate/up -> SwiGLU, one 128 x pitch tile per CTA (gemm_tile_run).  A is the interleaved
+// gate/up matrix of 2F rows written by tc_tile_layer: rows 0..63 of tile b are the gate rows
+// of features 64b..64b+63, rows 64..127 the up rows of the same features.  The accumulator is
+// staged in shared memory (the idle operand ring, [column][tile row]) so that a thread holds
+// the gate and up values of eight consecutive features of one packed row; it writes
+// silu(gate) * up as one 16-byte bf16 chunk of the down product's SW128 operand (k-slice b,
+// element (row n, feature m)).  Packed rows at or past *nrows are not written.
+constexpr int kGuThreads = 256;
 template <int BN>
-__global__ void __launch_bounds__(tc::kPThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
-                                                                  const int* nrows) {
-  const int M = *nrows;
-  tc::gemm_persistent<BN, true, false>(g, 1, [&](int m, int n, int, float gt, float up) {
-    if (n < M) {
-      const float v = gt / (1.0f + __expf(-gt)) * up;
-      *reinterpret_cast<uint16_t*>(act_t + tc::sw128_offset(Rtc, n, m >> 6, (m & 63) >> 3) + (m & 7) * 2) =
-          (uint16_t)bf16_rn_bits(v);
+__global__ void __launch_bounds__(kGuThreads, 1) tc_gu_kernel(const tc::GemmArgs g, uint8_t* act_t, int Rtc,
+                                                               const int* nrows) {
+  using L = tc::Layout<BN>;
+  constexpr int kSP = tc::kBM + 4;                  // staged column stride (floats)
+  static_assert((size_t)BN * kSP * 4 <= (size_t)L::kStages * L::kStageBytes, "gate/up staging exceeds the ring");
+  tc::TileRun t;
+  if (!tc::gemm_tile_run<BN, false, false>(g, t)) return;
+  float* S = reinterpret_cast<float*>(t.smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int quarter = warp & 3, part = warp >> 2, n_parts = (int)(blockDim.x >> 7);
+  if (t.ok) {
+    // warp w drains TMEM lanes 32 (w % 4) .. (tile rows) for the column chunks c = w / 4 mod
+    // (warps / 4); a warp's 32 lanes store 32 consecutive floats of one column
+    const uint32_t lane_base = t.tmem + ((uint32_t)(quarter * 32) << 16);
+    const int r = quarter * 32 + lane, n_ch = t.nw >> 4;
+    for (int ch = part; ch < n_ch; ch += n_parts) {
+      float v[16];
+      tc::tmem_ld16(lane_base + (uint32_t)(16 * ch), v);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) S[(16 * ch + j) * kSP + r] = v[j];
     }
-  });
+  }
+  __syncthreads();
+  if (t.ok) {
+    const int M = *nrows, kt = t.m0 / tc::kBM;
+    for (int it = threadIdx.x; it < t.nw * 8; it += blockDim.x) {
+      const int nl = it >> 3, c = it & 7, n = t.n0 + nl;
+      if (n >= M) continue;
+      const float4* gs = reinterpret_cast<const float4*>(S + nl * kSP + 8 * c);
+      const float4* us = reinterpret_cast<const float4*>(S + nl * kSP + 64 + 8 * c);
+      const float4 g0 = gs[0], g1 = gs[1], u0 = us[0], u1 = us[1];
+      const float gt[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+      const float up[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+      float v[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = gt[e] / (1.0f + __expf(-gt[e])) * up[e];
+      *reinterpret_cast<uint4*>(act_t + tc::sw128_offset(Rtc, n, kt, c)) =
+          make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                     pack_bf16x2(v[6], v[7]));
+    }
+  }
+  tc::gemm_tile_free<BN, false, false>(t);
 }
 
 // Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
@@ -169,17 +207,17 @@ bool tc_block_supported(const FrameParams& p) {
          (p.NH * p.D) % 64 == 0 && p.H % 64 == 0 && p.F % 64 == 0 && p.H <= 1024;
 }
 
-// SW128 copies of one layer's weights: [qkv | g | u | o | d], offsets within a layer.
+// SW128 copies of one layer's weights: [qkv | gate/up interleaved (2F rows) | o | d], offsets
+// within a layer.
 struct TcLayerOffsets {
-  size_t qkv = 0, g = 0, u = 0, o = 0, d = 0, layer = 0;
+  size_t qkv = 0, gu = 0, o = 0, d = 0, layer = 0;
 };
 inline TcLayerOffsets tc_layer_offsets(const FrameParams& p) {
   TcLayerOffsets t;
   const size_t H = p.H, F = p.F, qd = (size_t)p.NH * p.D;
   t.qkv = 0;
-  t.g = t.qkv + (size_t)p.qkv_dim * H * 2;
-  t.u = t.g + F * H * 2;
-  t.o = t.u + F * H * 2;
+  t.gu = t.qkv + (size_t)p.qkv_dim * H * 2;
+  t.o = t.gu + 2 * F * H * 2;
   t.d = t.o + H * qd * 2;
   t.layer = t.d + H * F * 2;
   return t;
@@ -189,49 +227,53 @@ inline void tc_tile_layer(const FrameParams& p, cudaStream_t st, const uint8_t* 
                           const uint8_t* wo, const uint8_t* wg, const uint8_t* wu, const uint8_t* wd, uint8_t* base) {
   const TcLayerOffsets t = tc_layer_offsets(p);
   const int H = p.H, F = p.F, qd = p.NH * p.D, kd = p.NKV * p.D;
-  auto tile = [&](const uint8_t* s, int rows, int K, int R, int row0, size_t off) {
-    tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(s), rows, K, R, row0, base + off);
+  auto tile = [&](const uint8_t* s, int rows, int K, int R, int row0, int grp, int gstride, size_t off) {
+    tc_weight_tile_kernel<<<512, 256, 0, st>>>(reinterpret_cast<const uint16_t*>(s), rows, K, R, row0, grp, gstride,
+                                               base + off);
   };
-  tile(wq, qd, H, p.qkv_dim, 0, t.qkv);
-  tile(wk, kd, H, p.qkv_dim, qd, t.qkv);
-  tile(wv, kd, H, p.qkv_dim, qd + kd, t.qkv);
-  tile(wg, F, H, F, 0, t.g);
-  tile(wu, F, H, F, 0, t.u);
-  tile(wo, H, qd, H, 0, t.o);
-  tile(wd, H, F, H, 0, t.d);
+  tile(wq, qd, H, p.qkv_dim, 0, qd, 0, t.qkv);
+  tile(wk, kd, H, p.qkv_dim, qd, kd, 0, t.qkv);
+  tile(wv, kd, H, p.qkv_dim, qd + kd, kd, 0, t.qkv);
+  // gate rows 64b.. of tile b at its rows 0..63, the up rows at 64..127 (tc_gu_kernel)
+  tile(wg, F, H, 2 * F, 0, 64, 128, t.gu);
+  tile(wu, F, H, 2 * F, 64, 64, 128, t.gu);
+  tile(wo, H, qd, H, 0, H, 0, t.o);
+  tile(wd, H, F, H, 0, F, 0, t.d);
 }
 // Dynamic shared memory of the block kernels (once per translation unit).
 inline cudaError_t tc_block_set_smem() {
   cudaError_t e = cudaFuncSetAttribute(tc_qkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        tc::PLayout<kTcBN, false, true>::kSmemBytes);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_gu_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::PLayout<128, true, false>::kSmemBytes);
+    e = cudaFuncSetAttribute(tc_gu_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::Layout<128>::kSmemBytes);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_gu_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::PLayout<64, true, false>::kSmemBytes);
+    e = cudaFuncSetAttribute(tc_gu_kernel<176>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::Layout<176>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_gu_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::Layout<256>::kSmemBytes);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              tc::PLayout<kTcBN, false, false>::kSmemBytes);
   return e;
 }
 
-// gate/up -> SwiGLU into the down product's operand, at the tile width for Rtc rows.
-inline void tc_launch_gu(const tc::GemmArgs& g, uint8_t* act_t, int Rtc, const int* nrows, int F, int n_sm,
-                         cudaStream_t s);
-
 // Persistent launch shape: one CTA per SM at most, one per tile at least.
 inline dim3 tc_grid(int n_tiles, int n_sm) { return dim3(n_tiles < n_sm ? n_tiles : n_sm); }
 inline int tc_tiles(int N, int BN, int M, int splits) { return (N / BN) * (M / tc::kBM) * splits; }
 
-inline void tc_launch_gu(const tc::GemmArgs& g, uint8_t* act_t, int Rtc, const int* nrows, int F, int n_sm,
-                         cudaStream_t s) {
-  if (tc_bn_gu(Rtc) == 128)
-    tc_gu_kernel<128><<<tc_grid(tc_tiles(Rtc, 128, F, 1), n_sm), tc::kPThreads, tc::PLayout<128, true, false>::kSmemBytes, s>>>(
-        g, act_t, Rtc, nrows);
+// gate/up -> SwiGLU into the down product's operand.  gu: the interleaved gate/up matrix
+// (2F rows); xn: the normalised operand of Rtc rows.  The tile pitch over the packed rows fills
+// the SMs with one tile per CTA (three tiles of 176 / 176 / 160 rows at 512 rows, F = 3072).
+inline void tc_launch_gu(const uint8_t* gu, const uint8_t* xn, uint8_t* act_t, int Rtc, const int* nrows, int F,
+                         int H, int* err, unsigned long long wait_ns, int n_sm, cudaStream_t s) {
+  const int pitch = tc::tile_pitch(2 * F, Rtc, n_sm);
+  const tc::GemmArgs g{gu, nullptr, xn, nullptr, 2 * F, Rtc, H, nrows, err, wait_ns, pitch};
+  const dim3 grid((Rtc + pitch - 1) / pitch, 2 * F / tc::kBM);
+  if (pitch <= 128)
+    tc_gu_kernel<128><<<grid, kGuThreads, tc::Layout<128>::kSmemBytes, s>>>(g, act_t, Rtc, nrows);
+  else if (pitch <= 176)
+    tc_gu_kernel<176><<<grid, kGuThreads, tc::Layout<176>::kSmemBytes, s>>>(g, act_t, Rtc, nrows);
   else
-    tc_gu_kernel<64><<<tc_grid(tc_tiles(Rtc, 64, F, 1), n_sm), tc::kPThreads, tc::PLayout<64, true, false>::kSmemBytes, s>>>(
-        g, act_t, Rtc, nrows);
+    tc_gu_kernel<256><<<grid, kGuThreads, tc::Layout<256>::kSmemBytes, s>>>(g, act_t, Rtc, nrows);
 }
 
 }  // namespace
