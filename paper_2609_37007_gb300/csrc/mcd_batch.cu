@@ -524,13 +524,22 @@ __global__ void __launch_bounds__(256) batch_gemm_kernel(const __grid_constant__
 }
 
 // LM heads.  The (row, j) pairs of the call are grouped by head (head_list); group P starts at
-// operand row qoff(P) = the sum of the earlier groups rounded up to the tile width, so every
-// tile of the product belongs to one head.
+// operand row qoff(P) = the sum of the earlier groups rounded up to 16 rows, and its columns
+// are split into n_t = ceil(rows / kHeadTileMax) tiles of equal width (a multiple of 16), so
+// every tile of the product belongs to one head and is no wider than the group needs.
+constexpr int kHeadTileMax = 176;      // three 60 KB ring stages with the hi + lo operand
 __device__ __forceinline__ int tc_head_qoff(const BatchInfo* info, int P) {
   int o = 0;
-  for (int i = 1; i < P; ++i) o += (info->head_rows[i] + kTcBN - 1) / kTcBN * kTcBN;
+  for (int i = 1; i < P; ++i) o += (info->head_rows[i] + 15) / 16 * 16;
   return o;
 }
+__host__ __device__ __forceinline__ int tc_head_tiles(int rows) { return (rows + kHeadTileMax - 1) / kHeadTileMax; }
+__host__ __device__ __forceinline__ int tc_head_width(int rows) {
+  const int nt = tc_head_tiles(rows);
+  return nt ? ((rows + nt - 1) / nt + 15) / 16 * 16 : 0;
+}
+// Grid bound over the tiles of every group: at most (K + 1) pairs per packed row.
+inline int tc_head_grid_x(int R, int K, int n_pos) { return (R * (K + 1) + kHeadTileMax - 1) / kHeadTileMax + n_pos; }
 
 // The pairs' normalised rows (final RMSNorm, hi + lo) as SW128 tiles of Qcap rows.
 __global__ void __launch_bounds__(256) tc_heads_operand_kernel(const float* __restrict__ X, const float* __restrict__ gain,
@@ -571,29 +580,33 @@ __global__ void __launch_bounds__(256) tc_heads_operand_kernel(const float* __re
   }
 }
 
-// Logits of every pair: tile (blockIdx.x) of head P's group times head P's weights, plus the
-// draft-offset bias for j >= 1.
+// Logits of every pair: tile blockIdx.x (counted over the groups in head order) of head P's
+// group times head P's weights (m-tile blockIdx.y), plus the draft-offset bias for j >= 1.
 constexpr int kHeadsThreads = 256;     // eight warps: two per TMEM lane quarter in the epilogue
 __global__ void __launch_bounds__(kHeadsThreads, 1) tc_heads_kernel(const tc::GemmArgs g, const uint8_t* w_heads,
                                                                     size_t head_bytes, float* logits,
                                                                     const float* head_bias, const BatchInfo* info,
                                                                     const int* head_list, int n_pos, int K, int V) {
-  const int q0 = blockIdx.x * kTcBN;
-  int P = 0, qoff = 0;
-  for (int i = 1, o = 0; i <= n_pos; ++i) {
-    const int span = (info->head_rows[i] + kTcBN - 1) / kTcBN * kTcBN;
-    if (q0 >= o && q0 < o + span) {
+  int P = 0, qoff = 0, c0 = 0, nw = 0, rows = 0;
+  for (int i = 1, o = 0, t = blockIdx.x; i <= n_pos; ++i) {
+    const int r = info->head_rows[i], nt = tc_head_tiles(r);
+    if (P == 0 && t < nt) {
+      const int w = tc_head_width(r);
       P = i;
       qoff = o;
+      rows = r;
+      c0 = t * w;
+      nw = min(w, (r + 15) / 16 * 16 - c0);
     }
-    o += span;
+    t -= nt;
+    o += (r + 15) / 16 * 16;
   }
-  if (P == 0) return;                                   // past the last group (uniform per CTA)
-  const int rows = info->head_rows[P], off = info->head_off[P], i0 = q0 - qoff;
+  if (P == 0) return;                                   // past the last tile (uniform per CTA)
+  const int off = info->head_off[P];
   // the tile's (row, j) entries in shared memory and this thread's bias of every offset j
   // (the epilogue's output row m is fixed per thread), loaded while the products run
-  __shared__ int s_entry[kTcBN];
-  for (int i = threadIdx.x; i < kTcBN; i += blockDim.x) s_entry[i] = i0 + i < rows ? head_list[off + i0 + i] : -1;
+  __shared__ int s_entry[kHeadTileMax];
+  for (int i = threadIdx.x; i < nw; i += blockDim.x) s_entry[i] = c0 + i < rows ? head_list[off + c0 + i] : -1;
   const int m_t = blockIdx.y * tc::kBM + ((threadIdx.x >> 5) & 3) * 32 + (threadIdx.x & 31);
   float bias_j[kMaxDraft];
 #pragma unroll
@@ -602,17 +615,21 @@ __global__ void __launch_bounds__(kHeadsThreads, 1) tc_heads_kernel(const tc::Ge
   tc::GemmArgs ga = g;
   ga.a = w_heads + (size_t)(P - 1) * head_bytes;
   ga.n_active = nullptr;
-  tc::gemm_tile<kTcBN, false, true>(ga, [&](int m, int n, float v, float) {
-    const int e = s_entry[n - q0];
-    if (e >= 0) {
-      const int r = e >> 3, j = e & 7;
-      float bias = 0.f;
+  const int q0 = qoff + c0;
+  tc::gemm_tile<kHeadTileMax, false, true>(
+      ga,
+      [&](int m, int n, float v, float) {
+        const int e = s_entry[n - q0];
+        if (e >= 0) {
+          const int r = e >> 3, j = e & 7;
+          float bias = 0.f;
 #pragma unroll
-      for (int q = 1; q <= kMaxDraft; ++q)
-        if (j == q) bias = bias_j[q - 1];
-      logits[((size_t)r * kRecSlots + j) * V + m] = v + bias;
-    }
-  });
+          for (int q = 1; q <= kMaxDraft; ++q)
+            if (j == q) bias = bias_j[q - 1];
+          logits[((size_t)r * kRecSlots + j) * V + m] = v + bias;
+        }
+      },
+      q0, nw);
 }
 
 // Per-row sums of squares of the residual stream after a residual GEMM (one warp per row):
@@ -1077,7 +1094,7 @@ mcd_status batch_create(const FrameParams& p, int max_streams, BatchState** out)
   if (bs->use_tc &&
       (tc_block_set_smem() != cudaSuccess ||
        cudaFuncSetAttribute(tc_heads_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                            tc::Layout<kTcBN, false, true>::kSmemBytes) != cudaSuccess))
+                            tc::Layout<kHeadTileMax, false, true>::kSmemBytes) != cudaSuccess))
     return fail(MCD_ERR_CUDA);
   *out = bs;
   return MCD_OK;
@@ -1216,8 +1233,8 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       tc_heads_operand_kernel<<<512, blk, 0, s>>>(b.X, p.final_norm, b.ss + (size_t)(2 * L) * R, H, p.eps, b.info,
                                                  b.head_list, p.P, b.Qcap, b.hq_hi, b.hq_lo);
       const tc::GemmArgs g{nullptr, nullptr, b.hq_hi, b.hq_lo, p.V, b.Qcap, H, nullptr, p.err, p.wait_ns};
-      tc_heads_kernel<<<dim3(b.Qcap / kTcBN, p.V / tc::kBM, 1), dim3(kHeadsThreads),
-                        tc::Layout<kTcBN, false, true>::kSmemBytes, s>>>(g, bs->tw.heads, (size_t)p.V * H * 2, b.logits,
+      tc_heads_kernel<<<dim3(tc_head_grid_x(R, p.K, p.P), p.V / tc::kBM, 1), dim3(kHeadsThreads),
+                        tc::Layout<kHeadTileMax, false, true>::kSmemBytes, s>>>(g, bs->tw.heads, (size_t)p.V * H * 2, b.logits,
                                                                         p.head_bias, b.info, b.head_list, p.P, p.K, p.V);
     } else {   // final RMSNorm -> LM heads, one grid slice per head
       GemmArgs a = gemm_args(p, b);

@@ -177,16 +177,21 @@ struct TileRun {
   bool ok;         // every MMA completed (false after a timeout)
 };
 
-// Set-up, operand stream and MMAs of the tile of this CTA.  false: the tile is empty (its
-// first column at or past *n_active, or no k-slices in its split) and nothing is held; else
-// every thread returns after the accumulator is complete (t.ok) or the tile gave up, and the
-// CTA must call gemm_tile_free.
+// Set-up, operand stream and MMAs of the tile of this CTA: columns n0 .. n0 + nw - 1 (by
+// default x * pitch .. for x = blockIdx.x; else as given, n0 and nw multiples of 16, nw <= BN).
+// false: the tile is empty (its first column at or past *n_active, or no k-slices in its
+// split) and nothing is held; else every thread returns after the accumulator is complete
+// (t.ok) or the tile gave up, and the CTA must call gemm_tile_free.
 template <int BN, bool kDualA, bool kDualB>
-__device__ __forceinline__ bool gemm_tile_run(const GemmArgs& g, TileRun& t) {
+__device__ __forceinline__ bool gemm_tile_run(const GemmArgs& g, TileRun& t, int n0 = -1, int nw = 0) {
   using L = Layout<BN, kDualA, kDualB>;
   extern __shared__ uint8_t tc_smem_raw[];
-  const int pitch = g.bn ? g.bn : BN, n0 = blockIdx.x * pitch, m0 = blockIdx.y * kBM;
-  const int nw = min(pitch, g.N - n0);                            // this tile's columns
+  const int m0 = blockIdx.y * kBM;
+  if (n0 < 0) {
+    const int pitch = g.bn ? g.bn : BN;
+    n0 = blockIdx.x * pitch;
+    nw = min(pitch, g.N - n0);                                    // this tile's columns
+  }
   if (g.n_active && n0 >= __ldg(g.n_active)) return false;    // uniform over the CTA
   const int nk_all = g.K / kBK, per = (nk_all + gridDim.z - 1) / gridDim.z;
   const int kt0 = blockIdx.z * per, kt1 = min(nk_all, kt0 + per), nk = kt1 - kt0;
@@ -296,13 +301,16 @@ __device__ __forceinline__ void gemm_tile_free(const TileRun& t) {
 // adjacent in launch order, so the weights stream from HBM about once while the activation
 // tiles stay in L2); epi(m, n, v, v2) for every m and n of the tile (each thread: one m, BN
 // values of n in order; v2 = the second accumulator with kDualA, else 0).  A tile whose
-// first column is at or past *n_active returns at once.
+// first column is at or past *n_active returns at once.  n0 >= 0: the tile's columns are
+// n0 .. n0 + nw - 1 instead (see gemm_tile_run).
 template <int BN, bool kDualA, bool kDualB, class Epi>
-__device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi) {
+__device__ __forceinline__ void gemm_tile(const GemmArgs& g, Epi epi, int n0 = -1, int nw = 0) {
   TileRun t;
-  if (!gemm_tile_run<BN, kDualA, kDualB>(g, t)) return;
+  if (!gemm_tile_run<BN, kDualA, kDualB>(g, t, n0, nw)) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = t.m0, n0 = t.n0, nw = t.nw;
+  const int m0 = t.m0;
+  n0 = t.n0;
+  nw = t.nw;
   const uint32_t tmem = t.tmem;
   // epilogue: every warp, after the accumulator is complete
   if (t.ok) {
