@@ -1158,23 +1158,15 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
       }
       batch_attn_kernel<<<dim3(bs->max_streams, p.NKV), blk, 0, s>>>(p, b, l);      // -> att_t
       // Wo (k-split partials) -> residual, ss, the gate/up operand
-      {
-        const tc::GemmArgs g{wl + bs->tw.off.o, nullptr, b.att_t, nullptr, H, Rtc, qd, &b.info->M, p.err, p.wait_ns};
-        tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.part, H, Rtc, &b.info->M);
-      }
-      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 1) * R,
+      tc_launch_resid(wl + bs->tw.off.o, b.att_t, b.part, H, Rtc, qd, &b.info->M, p.err, p.wait_ns, p.n_cta, s);
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(qd, tc_resid_split(Rtc)), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 1) * R,
                                              p.ffn_norm + (size_t)l * H, p.eps, b.xn_hi, nullptr);
       // gate/up -> SwiGLU (into the down product's operand)
       tc_launch_gu(wl + bs->tw.off.gu, b.xn_hi, b.act_t, Rtc, &b.info->M, p.F, H, p.err, p.wait_ns, p.n_cta, s);
       // down (k-split partials) -> residual, ss, the next layer's QKV operand
-      {
-        const tc::GemmArgs g{wl + bs->tw.off.d, nullptr, b.act_t, nullptr, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns};
-        tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
-            g, b.part, H, Rtc, &b.info->M);
-      }
+      tc_launch_resid(wl + bs->tw.off.d, b.act_t, b.part, H, Rtc, p.F, &b.info->M, p.err, p.wait_ns, p.n_cta, s);
       const bool last = l + 1 == L;
-      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(p.F), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 2) * R,
+      tc_resid_norm_kernel<<<R, 128, 0, s>>>(b.X, b.part, tc_splits(p.F, tc_resid_split(Rtc)), Rtc, H, &b.info->M, b.ss + (size_t)(2 * l + 2) * R,
                                              last ? nullptr : p.attn_norm + (size_t)(l + 1) * H, p.eps, b.xn_hi, b.xn_lo);
     }
     for (int l = 0; l < L && !bs->use_tc; ++l) {

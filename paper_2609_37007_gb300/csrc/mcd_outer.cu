@@ -1117,20 +1117,12 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
                                                          p.q_norm + (size_t)l * p.D, p.k_norm + (size_t)l * p.D, p.eps,
                                                          st.rope, kc, vc, st.cap, t.q);
     pf_attn_kernel<<<(n * p.NH + 7) / 8, 256, 0, s>>>(t.q, t.rows, p.NH, p.NKV, p.D, kc, vc, st.cap, Rtc, t.att_t);
-    {
-      const tc::GemmArgs g{wl + t.off.o, nullptr, t.att_t, nullptr, H, Rtc, qd, t.rows, p.err, p.wait_ns};
-      tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
-          g, t.part, H, Rtc, t.rows);
-    }
-    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(qd), Rtc, H, t.rows, t.ss, p.ffn_norm + (size_t)l * H,
+    tc_launch_resid(wl + t.off.o, t.att_t, t.part, H, Rtc, qd, t.rows, p.err, p.wait_ns, p.n_cta, s);
+    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(qd, tc_resid_split(Rtc)), Rtc, H, t.rows, t.ss, p.ffn_norm + (size_t)l * H,
                                            p.eps, t.xn_hi, nullptr);
     tc_launch_gu(wl + t.off.gu, t.xn_hi, t.act_t, Rtc, t.rows, p.F, H, p.err, p.wait_ns, p.n_cta, s);
-    {
-      const tc::GemmArgs g{wl + t.off.d, nullptr, t.act_t, nullptr, H, Rtc, p.F, t.rows, p.err, p.wait_ns};
-      tc_resid_kernel<<<tc_grid(tc_tiles(Rtc, kTcBN, H, kTcSplit), p.n_cta), pblk, tc::PLayout<kTcBN, false, false>::kSmemBytes, s>>>(
-          g, t.part, H, Rtc, t.rows);
-    }
-    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(p.F), Rtc, H, t.rows, t.ss,
+    tc_launch_resid(wl + t.off.d, t.act_t, t.part, H, Rtc, p.F, t.rows, p.err, p.wait_ns, p.n_cta, s);
+    tc_resid_norm_kernel<<<n, 128, 0, s>>>(t.X, t.part, tc_splits(p.F, tc_resid_split(Rtc)), Rtc, H, t.rows, t.ss,
                                            l + 1 < L ? p.attn_norm + (size_t)(l + 1) * H : nullptr, p.eps, t.xn_hi,
                                            t.xn_lo);
   }

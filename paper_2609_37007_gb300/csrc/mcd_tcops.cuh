@@ -56,7 +56,11 @@ __global__ void tc_weight_tile_kernel(const uint16_t* __restrict__ src, int rows
 }
 
 constexpr int kTcBN = 128;        // packed rows per tile: QKV (hi + lo operand), Wo, down
-constexpr int kTcSplit = 4;       // k-splits of the residual products
+constexpr int kTcSplit = 6;       // k-splits of the residual products (at most)
+// Splits of the residual products at Rtc packed rows: four (128-column tiles, 128 CTAs at 512
+// rows) from 512 rows on, where more splits' partial sums cost more than they save; six below
+// (3 x 8 x 6 = 144 CTAs at 128 rows, where 128-column tiles would leave 32 CTAs).
+inline int tc_resid_split(int Rtc) { return Rtc >= 512 ? 4 : kTcSplit; }
 
 // q, k, v = W (x . g / rms) with the hi + lo operand.
 __global__ void __launch_bounds__(tc::kPThreads, 1) tc_qkv_kernel(const tc::GemmArgs g, float* out, int ld,
@@ -120,13 +124,17 @@ __global__ void __launch_bounds__(kGuThreads, 1) tc_gu_kernel(const tc::GemmArgs
   tc::gemm_tile_free<BN, false, false>(t);
 }
 
-// Residual products (Wo, down), k split over gridDim.z: split z writes its partial sums
-// part[z][n][m] (plain stores); tc_resid_norm_kernel adds them into the residual stream.
-__global__ void __launch_bounds__(tc::kPThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
+// Residual products (Wo, down): one 128 x pitch tile per CTA over the k-slices of split
+// blockIdx.z of kTcSplit; split z writes its partial sums part[z][n][m] (plain stores);
+// tc_resid_norm_kernel adds them into the residual stream.
+constexpr int kResidThreads = 256;
+template <int BN>
+__global__ void __launch_bounds__(kResidThreads, 1) tc_resid_kernel(const tc::GemmArgs g, float* part, int ld, int Rtc,
                                                                      const int* nrows) {
   const int M = *nrows;
-  tc::gemm_persistent<kTcBN, false, false>(g, kTcSplit, [&](int m, int n, int z, float v, float) {
-    if (n < M) part[((size_t)z * Rtc + n) * ld + m] = v;
+  const size_t zoff = (size_t)blockIdx.z * Rtc;
+  tc::gemm_tile<BN, false, false>(g, [&](int m, int n, float v, float) {
+    if (n < M) part[(zoff + n) * ld + m] = v;
   });
 }
 
@@ -194,9 +202,10 @@ __global__ void __launch_bounds__(128) tc_resid_norm_kernel(float* X, const floa
   }
 }
 
-// Non-empty k-splits of a residual product over K (gemm_tile's split of the k-slices).
-static int tc_splits(int K) {
-  const int nk = K / tc::kBK, per = (nk + kTcSplit - 1) / kTcSplit;
+// Non-empty k-splits of a residual product over K in z splits (gemm_tile's split of the
+// k-slices).
+static int tc_splits(int K, int z) {
+  const int nk = K / tc::kBK, per = (nk + z - 1) / z;
   return (nk + per - 1) / per;
 }
 
@@ -251,8 +260,14 @@ inline cudaError_t tc_block_set_smem() {
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(tc_gu_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, tc::Layout<256>::kSmemBytes);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(tc_resid_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             tc::PLayout<kTcBN, false, false>::kSmemBytes);
+    e = cudaFuncSetAttribute(tc_resid_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::Layout<128>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_resid_kernel<176>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::Layout<176>::kSmemBytes);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_resid_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             tc::Layout<256>::kSmemBytes);
   return e;
 }
 
@@ -274,6 +289,28 @@ inline void tc_launch_gu(const uint8_t* gu, const uint8_t* xn, uint8_t* act_t, i
     tc_gu_kernel<176><<<grid, kGuThreads, tc::Layout<176>::kSmemBytes, s>>>(g, act_t, Rtc, nrows);
   else
     tc_gu_kernel<256><<<grid, kGuThreads, tc::Layout<256>::kSmemBytes, s>>>(g, act_t, Rtc, nrows);
+}
+
+// Wo or down (A = w: H rows of K, B = act: Rtc rows) -> tc_resid_split(Rtc) partial sums.
+// T column tiles x (H / 128) weight tiles x z splits fill the SMs with one tile per CTA
+// (H = 1024: T = 4 of 128 packed rows at 512 rows, 128 CTAs; T = 3 of 48 / 48 / 32 at 128
+// rows, 144 CTAs).
+inline void tc_launch_resid(const uint8_t* w, const uint8_t* act, float* part, int H, int Rtc, int K, const int* nrows,
+                            int* err, unsigned long long wait_ns, int n_sm, cudaStream_t s) {
+  const int n_mt = H / tc::kBM, units = Rtc / 16, z = tc_resid_split(Rtc);
+  int T = n_sm / (n_mt * z);
+  if (T < 1) T = 1;
+  if (T < (Rtc + 255) / 256) T = (Rtc + 255) / 256;
+  if (T > units) T = units;
+  const int pitch = (units + T - 1) / T * 16;
+  const tc::GemmArgs g{w, nullptr, act, nullptr, H, Rtc, K, nrows, err, wait_ns, pitch};
+  const dim3 grid((Rtc + pitch - 1) / pitch, n_mt, z);
+  if (pitch <= 128)
+    tc_resid_kernel<128><<<grid, kResidThreads, tc::Layout<128>::kSmemBytes, s>>>(g, part, H, Rtc, nrows);
+  else if (pitch <= 176)
+    tc_resid_kernel<176><<<grid, kResidThreads, tc::Layout<176>::kSmemBytes, s>>>(g, part, H, Rtc, nrows);
+  else
+    tc_resid_kernel<256><<<grid, kResidThreads, tc::Layout<256>::kSmemBytes, s>>>(g, part, H, Rtc, nrows);
 }
 
 }  // namespace
