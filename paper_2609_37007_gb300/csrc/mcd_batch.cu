@@ -1146,7 +1146,7 @@ static cudaError_t enqueue_frame(const FrameParams& p, const BatchState* bs, cud
     for (int l = 0; l < L && bs->use_tc; ++l) {
       const uint8_t* wl = bs->tw.arena + (size_t)l * bs->tw.off.layer;
       const int Rtc = b.Rtc, qd = p.NH * p.D;
-      const dim3 tblk(tc::kThreads), pblk(tc::kPThreads);
+      const dim3 pblk(tc::kPThreads);
       // RMSNorm -> QKV (hi + lo operand; after layer 0 written by the previous layer's last
       // residual pass)
       if (l == 0)

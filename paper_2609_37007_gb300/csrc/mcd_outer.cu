@@ -1099,7 +1099,7 @@ static mcd_status outer_tc_prefill(mcd_outer* o, const int32_t* text_ids, int n)
   const OuterStep& st = o->st;
   cudaStream_t s = o->stream;
   const int H = p.H, L = p.L, Rtc = t.Rtc, qd = p.NH * p.D, kvl = p.NKV * st.cap * p.D;
-  const dim3 tblk(tc::kThreads), pblk(tc::kPThreads);
+  const dim3 pblk(tc::kPThreads);
   pf_set_rows_kernel<<<1, 1, 0, s>>>(t.rows, n);
   pf_embed_kernel<<<n, 128, 0, s>>>(text_ids, t.rows, st.text_table, st.text_vocab, H, t.X, t.ss, p.err);
   tc_norm_operand_kernel<<<256, 256, 0, s>>>(t.X, p.attn_norm, t.ss, H, p.eps, t.rows, Rtc, t.xn_hi, t.xn_lo);
